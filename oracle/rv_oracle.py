@@ -1,0 +1,262 @@
+"""CPU oracle of the Reflective Verification verify step (arXiv 2505.18629).
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and
+``bench.py``'s CPU-baseline / reference legs may import or run this module.  It
+shares no code with the CUDA path (``paper_2505_18629_gb300``) and imports
+nothing from it; the product never calls it.
+
+Plain NumPy in float64: every bf16 (uint16 bit pattern) or fp32 input is first
+widened exactly to float64, then each step below is its textbook definition.
+No tiling, fusion or reordering beyond what the definitions state (the LM-head
+product is computed a block of vocab rows at a time only to bound memory; each
+logit is still one full dot product).
+
+Notation follows the paper:
+  * gamma  -- number of draft tokens x_1..x_gamma (Alg. 1)
+  * template -- Prompt_reflection || Prefix_position (Eq. 1); R = |template|
+  * reflective_draft = [x_1..x_gamma, template, x_1..x_gamma]  (Alg. 1, Eq. 1)
+  * m = gamma + |template| + 1 (Alg. 1); shift_len = m - 1 (Eq. 2)
+  * o_i (i = 1..gamma+1) original logits, o_{m+i-1} reflective logits
+  * p_i = softmax((1-alpha) o_i + alpha o_{m+i-1})   (Eq. 2, Alg. 1)
+  * exact-match verification with the greedy choice x^_i = argmax p_i
+    (Alg. 2, read as "stop at the first mismatch"; see ``exact_match_accept``)
+
+Hidden-state rows: row 0 is the target's last hidden state after the prefix
+(gives o_1, "M_p(prefix)" in Alg. 1); row r (1..Lb) follows block token r-1.
+So o_i is row i-1 and its reflective partner o_{m+i-1} is row i-1+shift_len.
+
+Every function below is pinned by tests in ``tests/test_oracle_pins.py``
+against closed forms, library routines, invariants the paper states, or brute
+force; none is "parity unpinned".
+"""
+from __future__ import annotations
+
+import numpy as np
+
+# --------------------------------------------------------------------------
+# Widening
+# --------------------------------------------------------------------------
+
+
+def as_f64(x: np.ndarray) -> np.ndarray:
+    """Exact float64 view of a bf16 bit pattern (uint16) or fp32/fp64 array."""
+    x = np.asarray(x)
+    if x.dtype == np.uint16:
+        return (x.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    if x.dtype in (np.float32, np.float64):
+        return x.astype(np.float64)
+    raise TypeError(f"unsupported dtype {x.dtype}")
+
+
+# --------------------------------------------------------------------------
+# Block construction: Eq. 1, Alg. 1 ("Prepare the reflective draft template")
+# --------------------------------------------------------------------------
+
+
+def template(prompt_ids: np.ndarray, prefix_ids: np.ndarray) -> np.ndarray:
+    """template = Prompt_reflection || Prefix_position (Eq. 1)."""
+    return np.concatenate([np.asarray(prompt_ids, np.int64), np.asarray(prefix_ids, np.int64)])
+
+
+def reflective_draft(drafts: np.ndarray, tmpl: np.ndarray) -> np.ndarray:
+    """[x_1..x_gamma, template, x_1..x_gamma] (Alg. 1; Eq. 1 Draft_final)."""
+    d = np.asarray(drafts, np.int64)
+    return np.concatenate([d, np.asarray(tmpl, np.int64), d])
+
+
+def m_index(gamma: int, R: int) -> int:
+    """m = gamma + |template| + 1 (Alg. 1)."""
+    return gamma + R + 1
+
+
+def shift_len(gamma: int, R: int) -> int:
+    """Positions between o_i and its reflective partner (Eq. 2): m - 1."""
+    return m_index(gamma, R) - 1
+
+
+def original_row(i: int) -> int:
+    """Hidden row that yields o_i, i = 1..gamma+1 (row 0 = after the prefix)."""
+    return i - 1
+
+
+def reflective_row(i: int, gamma: int, R: int) -> int:
+    """Hidden row that yields o_{m+i-1}, the reflective partner of o_i."""
+    return original_row(i) + shift_len(gamma, R)
+
+
+def pack_block(drafts, prompt_ids, prefix_ids, ctx_lens):
+    """Verify block ids and position ids for every sequence.
+
+    drafts [B, gamma], prompt_ids [n_prompt], prefix_ids [B, n_prefix],
+    ctx_lens [B] -> block_ids [B, Lb], pos_ids [B, Lb] with Lb = 2 gamma + R.
+    Position ids run on from the context (ctx, ctx+1, ...) for the whole block.
+    """
+    drafts = np.asarray(drafts, np.int64)
+    B = drafts.shape[0]
+    rows, pos = [], []
+    for b in range(B):
+        blk = reflective_draft(drafts[b], template(prompt_ids, prefix_ids[b]))
+        rows.append(blk)
+        pos.append(int(ctx_lens[b]) + np.arange(blk.shape[0], dtype=np.int64))
+    return np.stack(rows).astype(np.int32), np.stack(pos).astype(np.int32)
+
+
+# --------------------------------------------------------------------------
+# One forward pass over the block: causal attention (Sec. 3.1)
+# --------------------------------------------------------------------------
+
+
+def verify_attention(q, k_blk, v_blk, k_cache, v_cache, ctx_lens):
+    """Causal attention of the verify block against the KV cache (Sec. 3.1).
+
+    q [B, Lb, Hq, D]; k_blk, v_blk [B, Lb, Hkv, D]; caches [B, Hkv, Cmax, D];
+    ctx_lens [B].  Block query j of sequence b sits at position ctx_b + j and
+    sees the cached keys 0..ctx_b-1 and block keys 0..j (unidirectional mask:
+    the template and the copy cannot change what the first segment sees).
+    Query head h reads key/value head h // (Hq / Hkv).
+
+    Returns (out [B, Lb, Hq, D] float64, k_cache', v_cache') where the caches
+    have the block's keys/values written at [ctx_b, ctx_b + Lb).
+    """
+    q, kb, vb = as_f64(q), as_f64(k_blk), as_f64(v_blk)
+    kc, vc = as_f64(k_cache).copy(), as_f64(v_cache).copy()
+    B, Lb, Hq, D = q.shape
+    Hkv = kb.shape[2]
+    G = Hq // Hkv
+    out = np.zeros((B, Lb, Hq, D))
+    scale = 1.0 / np.sqrt(D)
+    for b in range(B):
+        c = int(ctx_lens[b])
+        for h in range(Hq):
+            g = h // G
+            keys = np.concatenate([kc[b, g, :c], kb[b, :, g]], axis=0)    # [c+Lb, D]
+            vals = np.concatenate([vc[b, g, :c], vb[b, :, g]], axis=0)
+            for j in range(Lb):
+                n = c + j + 1                      # keys visible to query j
+                s = keys[:n] @ q[b, j, h] * scale
+                w = np.exp(s - s.max())
+                w /= w.sum()
+                out[b, j, h] = w @ vals[:n]
+        kc[b, :, c:c + Lb] = kb[b].transpose(1, 0, 2)
+        vc[b, :, c:c + Lb] = vb[b].transpose(1, 0, 2)
+    return out, kc, vc
+
+
+# --------------------------------------------------------------------------
+# LM head, fusion (Eq. 2), log-softmax
+# --------------------------------------------------------------------------
+
+
+def head_logits(W, rows, block_rows: int = 8192) -> np.ndarray:
+    """Logits W @ h for every row h: rows [N, H] -> [N, V] (no bias)."""
+    rows = as_f64(rows)
+    V = W.shape[0]
+    out = np.empty((rows.shape[0], V))
+    for v0 in range(0, V, block_rows):
+        v1 = min(V, v0 + block_rows)
+        out[:, v0:v1] = rows @ as_f64(W[v0:v1]).T
+    return out
+
+
+def logsumexp(x: np.ndarray, axis: int = -1) -> np.ndarray:
+    """log(sum(exp(x))) along ``axis``, shifted by the max for range safety."""
+    m = np.max(x, axis=axis, keepdims=True)
+    return (m + np.log(np.sum(np.exp(x - m), axis=axis, keepdims=True))).squeeze(axis)
+
+
+def fuse(o: np.ndarray, o_refl: np.ndarray, alpha: float) -> np.ndarray:
+    """(1 - alpha) * o_i + alpha * o_{i + shift_len}  (Eq. 2, before softmax)."""
+    return (1.0 - alpha) * o + alpha * o_refl
+
+
+def greedy_choice(z: np.ndarray) -> np.ndarray:
+    """argmax over the vocab (last axis); ties go to the lowest token id."""
+    return np.argmax(z, axis=-1)
+
+
+def verify_head(W, hidden, drafts, gamma: int, R: int, alpha: float):
+    """LM head for the original and reflective rows, fused distribution p_i.
+
+    W [V, H]; hidden [B, Lb+1, H]; drafts [B, gamma].
+    For i = 1..gamma+1 (array index i-1):
+      o_i = W h_{row i-1},  o_{m+i-1} = W h_{row i-1+shift_len},
+      z_i = (1-alpha) o_i + alpha o_{m+i-1},  log p_i = z_i - logsumexp(z_i).
+    Returns a dict of float64 / int64 arrays:
+      lse_orig, lse_refl, lse_fused        [B, gamma+1]
+      logp_fused, logp_orig, logp_refl     [B, gamma]  (at the draft x_i)
+      argmax                               [B, gamma+1] (greedy x^_i)
+      margin                               [B, gamma]  |z_i[x_i] - max_{v != x_i} z_i[v]|
+      z                                    [B, gamma+1, V] fused logits
+    """
+    hidden = as_f64(hidden)
+    drafts = np.asarray(drafts, np.int64)
+    B = hidden.shape[0]
+    orig_idx = [original_row(i) for i in range(1, gamma + 2)]
+    refl_idx = [reflective_row(i, gamma, R) for i in range(1, gamma + 2)]
+    h_o = hidden[:, orig_idx, :].reshape(B * (gamma + 1), -1)
+    h_r = hidden[:, refl_idx, :].reshape(B * (gamma + 1), -1)
+    logits = head_logits(W, np.concatenate([h_o, h_r], axis=0))
+    V = logits.shape[1]
+    o = logits[:B * (gamma + 1)].reshape(B, gamma + 1, V)
+    o_refl = logits[B * (gamma + 1):].reshape(B, gamma + 1, V)
+    z = fuse(o, o_refl, alpha)
+    lse_o, lse_r, lse_z = logsumexp(o), logsumexp(o_refl), logsumexp(z)
+    bi = np.arange(B)[:, None]
+    ii = np.arange(gamma)[None, :]
+    zx = z[bi, ii, drafts]
+    z_others = z[:, :gamma, :].copy()
+    z_others[bi, ii, drafts] = -np.inf
+    margin = np.abs(zx - z_others.max(axis=-1))
+    return dict(
+        lse_orig=lse_o, lse_refl=lse_r, lse_fused=lse_z,
+        logp_fused=zx - lse_z[:, :gamma],
+        logp_orig=o[bi, ii, drafts] - lse_o[:, :gamma],
+        logp_refl=o_refl[bi, ii, drafts] - lse_r[:, :gamma],
+        argmax=greedy_choice(z), margin=margin, z=z,
+    )
+
+
+# --------------------------------------------------------------------------
+# Exact-match verification (Alg. 2) with greedy x^_i, prefix, next token
+# --------------------------------------------------------------------------
+
+
+def exact_match_accept(drafts, choice):
+    """Alg. 2 with x^_i = greedy choice of p_i.
+
+    drafts [B, gamma], choice [B, gamma+1] (x^_1..x^_{gamma+1}).
+    accept_i = (x_i == x^_i).  Alg. 2 prints the stopping set as the positions
+    where x_i equals x^_i; the standard rule the paper says it keeps (Sec. 3.3:
+    everything after the fusion is unchanged) stops at the first MISMATCH, so
+    n = min({i-1 : x_i != x^_i} U {gamma}) and t = x^_{n+1}.
+    Returns accept_mask [B, gamma] (uint8), n [B], next_token [B].
+    """
+    drafts = np.asarray(drafts, np.int64)
+    choice = np.asarray(choice, np.int64)
+    B, gamma = drafts.shape
+    acc = (drafts == choice[:, :gamma])
+    n = np.empty(B, np.int64)
+    t = np.empty(B, np.int64)
+    for b in range(B):
+        stop = [i - 1 for i in range(1, gamma + 1) if not acc[b, i - 1]]
+        n[b] = min(stop + [gamma])
+        t[b] = choice[b, n[b]]
+    return acc.astype(np.uint8), n, t
+
+
+def verify_step(inp_W, hidden, q, k_blk, v_blk, k_cache, v_cache, ctx_lens,
+                drafts, prompt_ids, prefix_ids, gamma: int, R: int, alpha: float):
+    """One whole verify step: pack, attention, head + fusion, accept, prefix.
+
+    Returns a dict with every intermediate the CUDA path exposes.  The new
+    context length is ctx + n: of the block's keys/values only the accepted
+    drafts of the first segment stay valid (the template and copy are pruned,
+    Sec. 3.1).
+    """
+    block_ids, pos_ids = pack_block(drafts, prompt_ids, prefix_ids, ctx_lens)
+    attn, kc, vc = verify_attention(q, k_blk, v_blk, k_cache, v_cache, ctx_lens)
+    head = verify_head(inp_W, hidden, drafts, gamma, R, alpha)
+    acc, n, t = exact_match_accept(drafts, head["argmax"])
+    return dict(block_ids=block_ids, pos_ids=pos_ids, attn=attn, k_cache=kc, v_cache=vc,
+                accept_mask=acc, accepted_len=n, next_token=t,
+                ctx_out=np.asarray(ctx_lens, np.int64) + n, **head)

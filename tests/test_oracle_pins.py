@@ -1,0 +1,385 @@
+"""Pins of the CPU oracle against facts fixed outside the oracle itself.
+
+Each test ties an oracle function to something it does not compute itself:
+values the paper prints (Table 3 / Table 4 fixtures under tests/golden/),
+closed forms, library routines (torch SDPA, scipy logsumexp / log_softmax),
+invariants the paper states (Sec. 3.1 causality, Eq. 2 at alpha = 0 / 1), and
+brute force on tiny inputs (lossless greedy exact-match verification).  The last
+block plants plausible mistakes in the oracle and checks that a pin catches each.
+"""
+import itertools
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import scipy.special
+import torch
+
+import oracle.rv_oracle as orc
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _golden(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return json.load(f)
+
+
+# --------------------------------------------------------------------------
+# Block layout: Table 3 {5+3+4+5} and Alg. 1's m
+# --------------------------------------------------------------------------
+
+def test_table3_block_layout():
+    g = _golden("table3_block_layout.json")
+    gamma, n_prompt, n_prefix = g["gamma"], g["n_prompt"], g["n_prefix"]
+    R = n_prompt + n_prefix
+    drafts = np.array([[101, 102, 103, 104, 105]])
+    prompt = np.array([201, 202, 203])
+    prefix = np.array([[301, 302, 303, 304]])
+    blk, pos = orc.pack_block(drafts, prompt, prefix, np.array([40]))
+    assert blk.shape == (1, g["budget"])               # 5 + 3 + 4 + 5 = 17 inputs
+    assert orc.m_index(gamma, R) == g["m"]
+    b = blk[0]
+    assert list(b[:gamma]) == list(drafts[0])
+    assert list(b[gamma:gamma + n_prompt]) == list(prompt)
+    assert list(b[gamma + n_prompt:gamma + R]) == list(prefix[0])
+    assert list(b[gamma + R:]) == list(drafts[0])
+    assert list(pos[0]) == list(range(40, 40 + g["budget"]))
+
+
+@pytest.mark.parametrize("gamma,R", [(5, 7), (1, 0), (4, 4), (8, 8), (3, 1)])
+def test_rows_score_their_draft(gamma, R):
+    """Hidden row r predicts block token r; o_i and o_{m+i-1} must both score x_i.
+
+    The original row of o_i predicts block position i-1 (first segment) and the
+    reflective row predicts the copy's i-th token, for i = 1..gamma.
+    """
+    drafts = np.arange(1, gamma + 1)[None, :] + 1000
+    prompt = np.arange(max(R - min(R, 4), 0)) + 2000
+    prefix = (np.arange(min(R, 4)) + 3000)[None, :]
+    blk, _ = orc.pack_block(drafts, prompt, prefix, np.array([0]))
+    b = blk[0]
+    Lb = b.shape[0]
+    assert Lb == 2 * gamma + R
+    for i in range(1, gamma + 1):
+        assert b[orc.original_row(i)] == drafts[0, i - 1]
+        assert b[orc.reflective_row(i, gamma, R)] == drafts[0, i - 1]
+    # o_{gamma+1} / o_{m+gamma}: the rows after the last draft of each segment.
+    assert orc.original_row(gamma + 1) == gamma
+    assert orc.reflective_row(gamma + 1, gamma, R) == Lb
+
+
+def test_table4_hyperparameters_are_the_defaults():
+    from paper_2505_18629_gb300 import synth
+    g = _golden("table4_hyperparameters.json")
+    assert synth.DEFAULT_ALPHA == g["alpha"]
+    assert synth.DEFAULT_PREFIX_LEN == g["prefix_len"]
+
+
+# --------------------------------------------------------------------------
+# Attention: torch SDPA (library), causality invariant, cache append
+# --------------------------------------------------------------------------
+
+def _rand_attn(rng, B, Lb, Hq, Hkv, D, ctx, cmax):
+    q = rng.standard_normal((B, Lb, Hq, D))
+    kb = rng.standard_normal((B, Lb, Hkv, D))
+    vb = rng.standard_normal((B, Lb, Hkv, D))
+    kc = rng.standard_normal((B, Hkv, cmax, D))
+    vc = rng.standard_normal((B, Hkv, cmax, D))
+    return q, kb, vb, kc, vc, np.asarray(ctx)
+
+
+def _sdpa_reference(q, kb, vb, kc, vc, ctx):
+    """torch.nn.functional.scaled_dot_product_attention, one sequence at a time."""
+    B, Lb, Hq, D = q.shape
+    Hkv = kb.shape[2]
+    out = np.zeros_like(q)
+    for b in range(B):
+        c = int(ctx[b])
+        K = np.concatenate([kc[b, :, :c], kb[b].transpose(1, 0, 2)], axis=1)   # [Hkv, c+Lb, D]
+        Vv = np.concatenate([vc[b, :, :c], vb[b].transpose(1, 0, 2)], axis=1)
+        Kt = torch.from_numpy(K).repeat_interleave(Hq // Hkv, dim=0)
+        Vt = torch.from_numpy(Vv).repeat_interleave(Hq // Hkv, dim=0)
+        Qt = torch.from_numpy(q[b].transpose(1, 0, 2).copy())                  # [Hq, Lb, D]
+        mask = torch.ones(Lb, c + Lb, dtype=torch.bool)
+        mask[:, c:] = torch.tril(torch.ones(Lb, Lb, dtype=torch.bool))
+        o = torch.nn.functional.scaled_dot_product_attention(Qt, Kt, Vt, attn_mask=mask)
+        out[b] = o.numpy().transpose(1, 0, 2)
+    return out
+
+
+@pytest.mark.parametrize("B,Lb,Hq,Hkv,D,ctx", [
+    (1, 12, 4, 4, 16, [64]),          # tiny-config shape, MHA
+    (2, 7, 8, 2, 16, [0, 5]),         # GQA, empty cache for one sequence
+    (1, 1, 4, 1, 8, [9]),             # Lb = 1: plain decode attention
+    (3, 5, 6, 3, 8, [3, 0, 11]),      # ragged contexts
+])
+def test_attention_matches_torch_sdpa(B, Lb, Hq, Hkv, D, ctx):
+    rng = np.random.default_rng(7)
+    args = _rand_attn(rng, B, Lb, Hq, Hkv, D, ctx, max(ctx) + Lb + 2)
+    out, _, _ = orc.verify_attention(*args)
+    ref = _sdpa_reference(*args)
+    np.testing.assert_allclose(out, ref, rtol=1e-12, atol=1e-12)
+
+
+def test_attention_first_segment_unaffected_by_template_and_copy():
+    """Sec. 3.1: the appended template and copy leave the first segment unchanged."""
+    rng = np.random.default_rng(3)
+    gamma, R = 4, 5
+    Lb = 2 * gamma + R
+    q, kb, vb, kc, vc, ctx = _rand_attn(rng, 2, Lb, 4, 2, 8, [6, 0], 30)
+    full, _, _ = orc.verify_attention(q, kb, vb, kc, vc, ctx)
+    first, _, _ = orc.verify_attention(q[:, :gamma], kb[:, :gamma], vb[:, :gamma], kc, vc, ctx)
+    np.testing.assert_array_equal(full[:, :gamma], first)
+
+
+def test_attention_appends_block_kv():
+    rng = np.random.default_rng(4)
+    q, kb, vb, kc, vc, ctx = _rand_attn(rng, 2, 3, 2, 2, 4, [2, 5], 10)
+    _, kc2, vc2 = orc.verify_attention(q, kb, vb, kc, vc, ctx)
+    for b, c in enumerate(ctx):
+        np.testing.assert_array_equal(kc2[b, :, c:c + 3], kb[b].transpose(1, 0, 2))
+        np.testing.assert_array_equal(vc2[b, :, c:c + 3], vb[b].transpose(1, 0, 2))
+        np.testing.assert_array_equal(kc2[b, :, :c], kc[b, :, :c])
+        np.testing.assert_array_equal(kc2[b, :, c + 3:], kc[b, :, c + 3:])
+
+
+def test_widening_is_exact():
+    x = np.array([1.0, -2.5, 3.140625, 65280.0, 1e-3], dtype=np.float32)
+    bits = torch.from_numpy(x).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    ref = torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16).to(torch.float64).numpy()
+    np.testing.assert_array_equal(orc.as_f64(bits), ref)
+
+
+# --------------------------------------------------------------------------
+# Head, log-softmax, fusion (Eq. 2)
+# --------------------------------------------------------------------------
+
+def test_logsumexp_closed_forms_and_library():
+    rng = np.random.default_rng(0)
+    x = rng.standard_normal((5, 1000)) * 30
+    np.testing.assert_allclose(orc.logsumexp(x), scipy.special.logsumexp(x, axis=-1), rtol=1e-13)
+    c = 7.25
+    assert orc.logsumexp(np.full((1, 4096), c))[0] == pytest.approx(c + math.log(4096), abs=1e-12)
+    lp = x - orc.logsumexp(x)[:, None]
+    np.testing.assert_allclose(np.exp(lp).sum(-1), 1.0, atol=1e-12)
+    np.testing.assert_allclose(lp, scipy.special.log_softmax(x, axis=-1), atol=1e-12)
+
+
+def _hand_example(alpha):
+    """H=2, V=3: o = log[1,2,3] from hidden (1,0), o' = log[3,2,1] from (0,1)."""
+    W = np.array([[0.0, math.log(3)], [math.log(2), math.log(2)], [math.log(3), 0.0]])
+    gamma, R = 1, 1
+    hidden = np.zeros((1, 2 * gamma + R + 1, 2))
+    hidden[0, 0] = (1, 0)          # row of o_1
+    hidden[0, 1] = (1, 0)          # row of o_2
+    hidden[0, 2] = (0, 1)          # row of o_m     (reflective partner of o_1)
+    hidden[0, 3] = (0, 1)          # row of o_{m+1}
+    return orc.verify_head(W, hidden, np.array([[0]]), gamma, R, alpha)
+
+
+def test_fusion_closed_form_alpha_03():
+    """alpha = 0.3: p_1 is proportional to [3^0.3, 2, 3^0.7] (Eq. 2 by hand)."""
+    r = _hand_example(0.3)
+    w = np.array([3 ** 0.3, 2.0, 3 ** 0.7])
+    assert r["lse_fused"][0, 0] == pytest.approx(math.log(w.sum()), abs=1e-14)
+    assert r["logp_fused"][0, 0] == pytest.approx(math.log(w[0] / w.sum()), abs=1e-14)
+    assert r["lse_orig"][0, 0] == pytest.approx(math.log(6), abs=1e-14)
+    assert r["lse_refl"][0, 0] == pytest.approx(math.log(6), abs=1e-14)
+    assert r["argmax"][0, 0] == 2
+    assert r["margin"][0, 0] == pytest.approx(0.4 * math.log(3), abs=1e-14)   # z_2 - z_0
+
+
+def test_fusion_closed_form_alpha_05_tie_breaks_low():
+    """alpha = 0.5: p proportional to [sqrt3, 2, sqrt3]; argmax 1."""
+    r = _hand_example(0.5)
+    w = np.array([math.sqrt(3), 2.0, math.sqrt(3)])
+    assert r["logp_fused"][0, 0] == pytest.approx(math.log(w[0] / w.sum()), abs=1e-14)
+    assert r["argmax"][0, 0] == 1
+    # alpha = 1 gives o' = log[3,2,1]: the argmax is token 0.
+    assert _hand_example(1.0)["argmax"][0, 0] == 0
+
+
+def _rand_head(rng, B, gamma, R, V, H):
+    W = (rng.standard_normal((V, H)) * 0.5).astype(np.float32)
+    hidden = rng.standard_normal((B, 2 * gamma + R + 1, H)).astype(np.float32)
+    drafts = rng.integers(0, V, size=(B, gamma))
+    return W, hidden, drafts
+
+
+def _copy_rows(hidden, gamma, R):
+    """Rows predicting the copy's tokens: block position Lb - gamma + i - 1 (i = 1..gamma+1)."""
+    Lb = 2 * gamma + R
+    return hidden[:, [Lb - gamma + i - 1 for i in range(1, gamma + 2)]]
+
+
+@pytest.mark.parametrize("alpha", [0.0, 0.3, 1.0])
+def test_fused_lse_is_lse_of_blended_hidden(alpha):
+    """The head is linear (no bias): W((1-a)h_i + a h'_i) = (1-a) o_i + a o'_i."""
+    rng = np.random.default_rng(11)
+    gamma, R = 3, 5
+    W, hidden, drafts = _rand_head(rng, 2, gamma, R, 300, 16)
+    r = orc.verify_head(W, hidden, drafts, gamma, R, alpha)
+    h_o = hidden[:, :gamma + 1].astype(np.float64)
+    h_r = _copy_rows(hidden, gamma, R).astype(np.float64)
+    blend = (1 - alpha) * h_o + alpha * h_r
+    z = blend @ W.astype(np.float64).T
+    np.testing.assert_allclose(r["lse_fused"], scipy.special.logsumexp(z, axis=-1), atol=1e-10)
+    np.testing.assert_allclose(r["lse_orig"],
+                               scipy.special.logsumexp(h_o @ W.astype(np.float64).T, axis=-1),
+                               atol=1e-10)
+    np.testing.assert_allclose(r["lse_refl"],
+                               scipy.special.logsumexp(h_r @ W.astype(np.float64).T, axis=-1),
+                               atol=1e-10)
+    lsm = scipy.special.log_softmax(z, axis=-1)
+    bi, ii = np.arange(2)[:, None], np.arange(gamma)[None, :]
+    np.testing.assert_allclose(r["logp_fused"], lsm[bi, ii, drafts], atol=1e-10)
+
+
+def test_alpha_zero_is_standard_verification():
+    """Eq. 2 at alpha = 0: p_i = softmax(o_i), the standard target distribution."""
+    rng = np.random.default_rng(12)
+    gamma, R = 4, 4
+    W, hidden, drafts = _rand_head(rng, 3, gamma, R, 200, 8)
+    r = orc.verify_head(W, hidden, drafts, gamma, R, 0.0)
+    np.testing.assert_array_equal(r["lse_fused"], r["lse_orig"])
+    np.testing.assert_array_equal(r["logp_fused"], r["logp_orig"])
+    o = hidden[:, :gamma + 1].astype(np.float64) @ W.astype(np.float64).T
+    np.testing.assert_array_equal(r["argmax"], np.argmax(o, axis=-1))
+
+
+def test_margin_from_sorted_logits():
+    rng = np.random.default_rng(13)
+    gamma, R = 3, 2
+    W, hidden, drafts = _rand_head(rng, 4, gamma, R, 50, 6)
+    drafts[0, 0] = 0
+    r = orc.verify_head(W, hidden, drafts, gamma, R, 0.3)
+    z = r["z"]
+    for b in range(4):
+        for i in range(gamma):
+            s = np.sort(z[b, i])
+            zx = z[b, i, drafts[b, i]]
+            want = s[-1] - s[-2] if zx == s[-1] else s[-1] - zx
+            assert r["margin"][b, i] == pytest.approx(want, abs=1e-12)
+
+
+# --------------------------------------------------------------------------
+# Acceptance (Alg. 2, greedy): lossless w.r.t. greedy decoding, brute force
+# --------------------------------------------------------------------------
+
+def _greedy_tables(rng, gamma, V):
+    """Random distinct-valued per-position greedy choices x^_1..x^_{gamma+1}."""
+    z = rng.standard_normal((1, gamma + 1, V))
+    return orc.greedy_choice(z)[0]
+
+
+@pytest.mark.parametrize("V,gamma", [(3, 1), (4, 2), (5, 3), (6, 3)])
+def test_accept_is_lossless_greedy_decoding_brute_force(V, gamma):
+    """Every draft tuple in V^gamma: the output [x_1..x_n, t] is exactly the
+    first n+1 tokens of greedy decoding, and n is maximal (x_{n+1} differs)."""
+    rng = np.random.default_rng(V * 10 + gamma)
+    for _ in range(3):
+        g = _greedy_tables(rng, gamma, V)
+        for d in itertools.product(range(V), repeat=gamma):
+            d = np.array(d)[None, :]
+            acc, n, t = orc.exact_match_accept(d, g[None, :])
+            n, t = int(n[0]), int(t[0])
+            out = list(d[0, :n]) + [t]
+            assert out == list(g[:n + 1])
+            assert 0 <= n <= gamma
+            assert (n == gamma) == bool(acc.all())
+            if n < gamma:
+                assert d[0, n] != g[n]
+            assert acc[0, :n].all()
+
+
+def test_literal_alg2_set_is_not_lossless():
+    """The stopping set as printed (first MATCH) breaks losslessness; the
+    first-mismatch reading used by the oracle keeps it."""
+    g = np.array([[1, 2, 0]])
+    d = np.array([[0, 2]])          # x_1 rejected, x_2 happens to match
+    literal_n = min([i - 1 for i in range(1, 3) if d[0, i - 1] == g[0, i - 1]] + [2])
+    literal_out = list(d[0, :literal_n]) + [g[0, literal_n]]
+    assert literal_out == [0, 2] and literal_out != list(g[0, :literal_n + 1])
+    _, n, t = orc.exact_match_accept(d, g)
+    assert int(n[0]) == 0 and int(t[0]) == 1
+
+
+def test_verify_step_end_to_end_small():
+    rng = np.random.default_rng(21)
+    B, gamma, R, V, H = 2, 3, 4, 64, 8
+    Lb = 2 * gamma + R
+    W = rng.standard_normal((V, H)).astype(np.float32)
+    hidden = rng.standard_normal((B, Lb + 1, H)).astype(np.float32)
+    q, kb, vb, kc, vc, ctx = _rand_attn(rng, B, Lb, 2, 1, 4, [3, 9], 30)
+    first = orc.verify_head(W, hidden, np.zeros((B, gamma), np.int64), gamma, R, 0.3)["argmax"]
+    drafts = first[:, :gamma].copy()
+    drafts[1, 1] = (drafts[1, 1] + 1) % V              # sequence 1 rejects x_2
+    r = orc.verify_step(W, hidden, q, kb, vb, kc, vc, ctx, drafts, np.array([5, 6]),
+                        np.array([[1, 2], [3, 4]]), gamma, R, 0.3)
+    assert list(r["accepted_len"]) == [3, 1]
+    assert list(r["ctx_out"]) == [6, 10]
+    assert r["next_token"][0] == r["argmax"][0, 3]
+    assert r["next_token"][1] == r["argmax"][1, 1]
+
+
+# --------------------------------------------------------------------------
+# Planted mistakes: each plausible slip in the oracle must fail a pin above
+# --------------------------------------------------------------------------
+
+def _fails(fn):
+    try:
+        fn()
+    except AssertionError:
+        return True
+    return False
+
+
+def test_pins_catch_off_by_one_shift(monkeypatch):
+    monkeypatch.setattr(orc, "shift_len", lambda gamma, R: gamma + R - 1)
+    assert _fails(lambda: test_rows_score_their_draft(5, 7))
+    assert _fails(lambda: test_fused_lse_is_lse_of_blended_hidden(0.3))
+
+
+def test_pins_catch_swapped_alpha(monkeypatch):
+    monkeypatch.setattr(orc, "fuse", lambda o, r, a: a * o + (1 - a) * r)
+    assert _fails(test_fusion_closed_form_alpha_03)
+    assert _fails(lambda: test_fused_lse_is_lse_of_blended_hidden(0.3))
+
+
+def test_pins_catch_literal_stopping_rule(monkeypatch):
+    def literal(drafts, choice):
+        drafts, choice = np.asarray(drafts), np.asarray(choice)
+        B, gamma = drafts.shape
+        acc = drafts == choice[:, :gamma]
+        n = np.array([min([i - 1 for i in range(1, gamma + 1) if acc[b, i - 1]] + [gamma])
+                      for b in range(B)])
+        return acc.astype(np.uint8), n, choice[np.arange(B), n]
+    monkeypatch.setattr(orc, "exact_match_accept", literal)
+    assert _fails(lambda: test_accept_is_lossless_greedy_decoding_brute_force(4, 2))
+
+
+def test_pins_catch_dropped_causal_mask(monkeypatch):
+    real = orc.verify_attention
+
+    def no_mask(q, k_blk, v_blk, k_cache, v_cache, ctx_lens):
+        # planted slip: every block query sees the whole block
+        out, kc, vc = real(q, k_blk, v_blk, k_cache, v_cache, ctx_lens)
+        qf, kb, vb = orc.as_f64(q), orc.as_f64(k_blk), orc.as_f64(v_blk)
+        B, Lb, Hq, D = qf.shape
+        G = Hq // kb.shape[2]
+        for b in range(B):
+            c = int(ctx_lens[b])
+            for h in range(Hq):
+                keys = np.concatenate([orc.as_f64(k_cache)[b, h // G, :c], kb[b, :, h // G]])
+                vals = np.concatenate([orc.as_f64(v_cache)[b, h // G, :c], vb[b, :, h // G]])
+                for j in range(Lb):
+                    s = keys @ qf[b, j, h] / np.sqrt(D)
+                    w = np.exp(s - s.max())
+                    out[b, j, h] = (w / w.sum()) @ vals
+        return out, kc, vc
+    monkeypatch.setattr(orc, "verify_attention", no_mask)
+    assert _fails(lambda: test_attention_matches_torch_sdpa(2, 7, 8, 2, 16, [0, 5]))
+    assert _fails(test_attention_first_segment_unaffected_by_template_and_copy)

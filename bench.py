@@ -1,0 +1,440 @@
+#!/usr/bin/env python3
+"""Verify-step benchmark of Reflective Verification on GB300.
+
+One step = the whole hot path on one batch: pack the block (Eq. 1), causal
+attention of the block against the KV cache (Sec. 3.1), LM head + fused online
+log-softmax for the original and reflective rows (Alg. 1, Eq. 2), exact-match
+acceptance + longest accepted prefix (Alg. 2).  Default workload: the
+Llama-3-8B-shaped step at batch 1 (hidden 4096, vocab 128256, 32/8 heads of
+128, ctx 2048, gamma 5, template 8), bf16, synthetic seeded inputs.
+
+Prints ONE JSON line: value = verified block positions per second (B*Lb per
+step, all ranks), device-timed with CUDA events; `e2e` = the same metric
+through rv_verify_step_host from pinned host buffers; `roofline` = the LM-head
+kernel's achieved HBM bandwidth against the measured peak; `cpu_baseline` = the
+fp64 CPU oracle on a bounded sample of the same step (rank 0).
+
+`--impl reference` times the CPU oracle alone (the paper ships no code; the
+oracle written from the paper stands in for it) on the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "verify-step µs & positions/s at 1 GB300; % of roofline (HBM-bound head/attn)"
+UNIT = "positions/s"
+ALPHA = 0.3
+FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0
+
+# DRAM traffic of one LM-head kernel launch, from `ncu --metrics dram__bytes_read.sum,
+# dram__bytes_write.sum` on the workload named (see profiles/), valid only while
+# the kernel sources hash to `src_sha`.
+NCU_TRAFFIC = {}
+
+
+def _kernel_src_hash() -> str:
+    h = hashlib.sha256()
+    for f in ("k_head_tc.cu", "head_epilogue.cuh", "rv_device.cuh"):
+        with open(os.path.join(ROOT, "paper_2505_18629_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d.get("hbm_gbs", FALLBACK_HBM_GBS), d.get("bf16_tflops", FALLBACK_BF16_TFLOPS), \
+            d.get("bf16_tflops_sustained", None), "measured"
+    return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, 1700.0, "fallback"
+
+
+# ---------------------------------------------------------------------------- distributed
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def aggregate(ms_local: float, units_local: float, world: int):
+    """Max step time and total units over ranks (barrier-bracketed timing)."""
+    if world == 1:
+        return ms_local, units_local
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([ms_local], dtype=torch.float64, device=dev)
+    u = torch.tensor([units_local], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    return float(t.item()), float(u.item())
+
+
+# ---------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi sampling during the timed region (clock, power, throttle reasons)."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.dev = device_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.dev), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100", "-f", self.path],
+                stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.15)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 7:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm = [float(r[0]) for r in rows if r[0].replace(".", "").isdigit()]
+        mx = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[3 + i].lower() == "active"})
+        pw = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows), "power_w_max": max(pw) if pw else None}
+
+
+# ---------------------------------------------------------------------------- CPU oracle legs
+
+def oracle_sample_step(inp, drafts, heads, vocab_rows):
+    """One oracle verify step on a bounded sample: attention for `heads` query
+    heads (all sequences, all block rows), the LM head + fusion + log-softmax
+    over the first `vocab_rows` vocab rows, acceptance.  Returns (t_attn, t_head)."""
+    import oracle.rv_oracle as orc
+    wl = inp.wl
+    G = wl.Hq // wl.Hkv
+    kv_heads = max(1, (heads + G - 1) // G)
+    t0 = time.perf_counter()
+    orc.verify_attention(inp.q[:, :, :kv_heads * G][:, :, :heads], inp.k_blk[:, :, :kv_heads],
+                         inp.v_blk[:, :, :kv_heads], inp.k_cache[:, :kv_heads],
+                         inp.v_cache[:, :kv_heads], inp.ctx_lens)
+    t1 = time.perf_counter()
+    head = orc.verify_head(inp.W[:vocab_rows], inp.hidden, np.minimum(drafts, vocab_rows - 1),
+                           wl.gamma, wl.R, ALPHA)
+    orc.exact_match_accept(drafts, head["argmax"])
+    t2 = time.perf_counter()
+    return t1 - t0, t2 - t1
+
+
+def cpu_step_estimate(inp, drafts, budget_s: float):
+    """Time oracle samples for about `budget_s`; extrapolate one full step (s)."""
+    wl = inp.wl
+    heads = min(wl.Hq, 2)
+    rows = min(wl.V, 4096)
+    ta, th = oracle_sample_step(inp, drafts, heads, rows)       # calibration
+    per = ta + th
+    reps = max(1, int(budget_s / max(per, 1e-3)))
+    sa, sh = [], []
+    for _ in range(reps):
+        a, h = oracle_sample_step(inp, drafts, heads, rows)
+        sa.append(a)
+        sh.append(h)
+    t_full = statistics.median(sa) * wl.Hq / heads + statistics.median(sh) * wl.V / rows
+    sample = (f"attention over {heads}/{wl.Hq} query heads and LM head over {rows}/{wl.V} vocab "
+              f"rows (all {wl.B} sequences), x{reps} reps, extrapolated linearly to the full step")
+    return t_full, sample, reps * (sa[0] + sh[0])
+
+
+def cores_used() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+# ---------------------------------------------------------------------------- reference arm
+
+def run_reference(args, wl):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    from paper_2505_18629_gb300 import synth
+    inp = synth.generate(wl)
+    drafts = inp.draft_alt.copy()
+    per_step_budget = min(0.5, 120.0 / max(1, args.steps + args.warmup))
+    heads = 1
+    rows = min(wl.V, 4096)
+    ta, th = oracle_sample_step(inp, drafts, heads, rows)
+    scale_rows = max(64, min(wl.V, int(rows * max(0.05, (per_step_budget - ta) / max(th, 1e-4)))))
+    rows = scale_rows
+    for _ in range(args.warmup):
+        oracle_sample_step(inp, drafts, heads, rows)
+    est = []
+    for _ in range(args.steps):
+        a, h = oracle_sample_step(inp, drafts, heads, rows)
+        est.append(a * wl.Hq / heads + h * wl.V / rows)
+    t_step = statistics.median(est)
+    value = wl.B * wl.Lb / t_step
+    sample = (f"each step: attention over {heads}/{wl.Hq} query heads, LM head over {rows}/{wl.V} "
+              f"vocab rows, extrapolated linearly to the full step")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_step * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": _config(wl),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores_used(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def _config(wl, world=1):
+    return {"workload": wl.name, "B": wl.B, "gamma": wl.gamma, "template": wl.R, "Lb": wl.Lb,
+            "ctx": list(wl.ctx), "hidden": wl.H, "vocab": wl.V, "q_heads": wl.Hq,
+            "kv_heads": wl.Hkv, "head_dim": wl.D, "alpha": ALPHA,
+            "parallelism": f"replicas x{world} (independent batches per GPU)",
+            "l2": "inputs larger than L2: the LM-head weight (V*H*2 bytes) streams every step"}
+
+
+# ---------------------------------------------------------------------------- main arm
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="rv", choices=["rv", "reference"])
+    ap.add_argument("--workload", default="llama3-8b-b1")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=200)
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    from paper_2505_18629_gb300 import synth
+    wl = synth.workload(args.workload)
+    if args.impl == "reference":
+        run_reference(args, wl)
+        return
+
+    import torch
+    import torch.distributed as dist
+    world, rank, local = dist_env()
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(dev)
+    from paper_2505_18629_gb300 import rv
+
+    inp = synth.generate(wl.replace(seed=wl.seed + 1000 * rank) if rank else wl)
+    B, g, R, Lb = wl.B, wl.gamma, wl.R, wl.Lb
+
+    def dev_t(x):
+        if x.dtype == np.uint16:
+            return torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).to(dev)
+        return torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+
+    W = dev_t(inp.W)
+    hidden, q, kb, vb = dev_t(inp.hidden), dev_t(inp.q), dev_t(inp.k_blk), dev_t(inp.v_blk)
+    kc, vc = dev_t(inp.k_cache), dev_t(inp.v_cache)
+    ctx = dev_t(inp.ctx_lens.astype(np.int32))
+    prompt = dev_t(inp.prompt_ids.astype(np.int32)) if inp.prompt_ids.size else None
+    prefix = dev_t(inp.prefix_ids.astype(np.int32))
+    h = rv.rv_create(wl.H, wl.V, wl.Hq, wl.Hkv, wl.D, B, g, R, wl.capacity,
+                     rv.RV_DTYPE_BF16 if wl.dtype == "bf16" else rv.RV_DTYPE_F32)
+    block = torch.empty((B, Lb), dtype=torch.int32, device=dev)
+    pos = torch.empty_like(block)
+    attn = torch.empty_like(q)
+    scores = torch.empty((B, g + 1, rv.RV_NSCORES), device=dev)
+    argmax = torch.empty((B, g + 1), dtype=torch.int32, device=dev)
+    margin = torch.empty((B, g), device=dev)
+    acc = torch.empty((B, g), dtype=torch.uint8, device=dev)
+    alen = torch.empty((B,), dtype=torch.int32, device=dev)
+    nxt = torch.empty_like(alen)
+    ctx_out = torch.empty_like(alen)
+
+    # Drafts: the target's greedy choice (from one call of our own head) with
+    # probability p_argmax, else the workload's random alternative.
+    d0 = torch.zeros((B, g), dtype=torch.int32, device=dev)
+    rv.rv_verify_head(h, hidden, W, d0, g, R, ALPHA, scores, argmax, margin)
+    choice = argmax[:, :g].cpu().numpy()
+    drafts_np = synth.make_drafts(inp, choice)
+    drafts = dev_t(drafts_np)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        rv.rv_pack_block(h, drafts, prompt, prefix, ctx, block, pos, stream)
+        rv.rv_verify_step(h, q, kb, vb, kc, vc, hidden, W, drafts, ctx, g, R, ALPHA, attn, scores,
+                          argmax, margin, acc, alen, nxt, ctx_out, stream)
+
+    for _ in range(args.warmup):
+        step()
+    st = rv.rv_read_status(h, stream)
+    if st:
+        raise RuntimeError(f"device status 0x{st:x} during warm-up")
+    mean_accepted = float(alen.float().mean().item())
+
+    clocks = ClockSampler(dev.index if dev.index is not None else 0)
+    clocks.start()
+    rv.rv_profile_enable(h, True)
+    launches0 = rv.rv_launch_count(h)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    launches = rv.rv_launch_count(h) - launches0
+    clk = clocks.stop()
+    ms_total = e0.elapsed_time(e1)
+    gemm_ms, gemm_n = rv.rv_profile_read(h, rv.RV_PROF_HEAD_GEMM)
+    attn_ms, attn_n = rv.rv_profile_read(h, rv.RV_PROF_ATTENTION)
+    headall_ms, headall_n = rv.rv_profile_read(h, rv.RV_PROF_HEAD)
+    rv.rv_profile_enable(h, False)
+    st = rv.rv_read_status(h, stream)
+    if st:
+        raise RuntimeError(f"device status 0x{st:x} in the timed region")
+
+    ms_step_local = ms_total / args.steps
+    ms_step, units = aggregate(ms_step_local, float(B * Lb), world)
+    value = units / (ms_step * 1e-3)
+
+    # ---- end to end through the host-buffer entry point (pinned memory)
+    def pin(x):
+        t = torch.from_numpy(x.view(np.int16) if x.dtype == np.uint16 else np.ascontiguousarray(x))
+        t = t.view(torch.bfloat16) if x.dtype == np.uint16 else t
+        return t.pin_memory()
+    hq, hkb, hvb, hhid = pin(inp.q), pin(inp.k_blk), pin(inp.v_blk), pin(inp.hidden)
+    hdr = pin(drafts_np.astype(np.int32))
+    hctx = pin(inp.ctx_lens.astype(np.int32))
+    o_sc = torch.empty((B, g + 1, rv.RV_NSCORES)).pin_memory()
+    o_am = torch.empty((B, g + 1), dtype=torch.int32).pin_memory()
+    o_mg = torch.empty((B, g)).pin_memory()
+    o_acc = torch.empty((B, g), dtype=torch.uint8).pin_memory()
+    o_al = torch.empty((B,), dtype=torch.int32).pin_memory()
+    o_nt = torch.empty_like(o_al).pin_memory()
+    o_co = torch.empty_like(o_al).pin_memory()
+
+    def step_host():
+        return rv.rv_verify_step_host(h, hq, hkb, hvb, kc, vc, hhid, W, hdr, hctx, g, R, ALPHA,
+                                      None, o_sc, o_am, o_mg, o_acc, o_al, o_nt, o_co, stream)
+    for _ in range(3):
+        step_host()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    t0 = time.perf_counter()
+    for _ in range(args.e2e_steps):
+        h2d, d2h = step_host()
+    e2e_ms_local = (time.perf_counter() - t0) * 1e3 / args.e2e_steps
+    e2e_ms, e2e_units = aggregate(e2e_ms_local, float(B * Lb), world)
+
+    # ---- roofline of the LM-head kernel
+    hbm, tf_burst, tf_sus, peak_src = _peaks()
+    n_rows = 2 * (g + 1) * B
+    head_bytes = wl.V * wl.H * 2 + n_rows * wl.H * 2
+    head_flops = 2.0 * n_rows * wl.H * wl.V
+    gemm_avg_s = gemm_ms * 1e-3 / max(gemm_n, 1)
+    achieved_gbs = head_bytes / gemm_avg_s / 1e9
+    achieved_tf = head_flops / gemm_avg_s / 1e12
+    t_hbm = head_bytes / (hbm * 1e9)
+    t_tc = head_flops / (tf_burst * 1e12)
+    bound = "hbm" if t_hbm >= t_tc else "tensor"
+    traffic = None
+    rec = NCU_TRAFFIC.get(wl.name)
+    if rec and rec.get("src_sha") == _kernel_src_hash():
+        traffic = rec["bytes"]
+    if bound == "hbm":
+        roof = {"bound": "hbm", "achieved": achieved_gbs, "peak": hbm, "unit": "GB/s",
+                "frac": achieved_gbs / hbm, "traffic": traffic}
+    else:
+        roof = {"bound": "tensor", "achieved": achieved_tf, "peak": tf_burst, "unit": "TFLOP/s",
+                "frac": achieved_tf / tf_burst, "traffic": traffic}
+    roof.update({"kernel": "head_tc_kernel (LM head GEMM + online log-softmax)",
+                 "peak_source": f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured"
+                 else "fallback", "algorithmic_bytes": head_bytes,
+                 "algorithmic_flops": head_flops, "avg_us": gemm_avg_s * 1e6, "launches": gemm_n})
+    # attention kernels (one layer): KV read + block Q/K/V/O
+    ctx_mean = float(np.mean(inp.ctx_lens))
+    attn_bytes = (B * (ctx_mean + Lb) * wl.Hkv * wl.D * 2 * 2 + B * Lb * wl.Hq * wl.D * 2 * 2
+                  + B * Lb * wl.Hkv * wl.D * 2 * 2)
+    attn_avg_s = attn_ms * 1e-3 / max(attn_n, 1)
+    step_roof_s = max(head_flops / (tf_burst * 1e12),
+                      (wl.V * wl.H * 2 + B * ctx_mean * wl.Hkv * wl.D * 4) / (hbm * 1e9))
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32",
+        "data": "synthetic (seeded Gaussian weights/activations shaped like Llama-3-8B)",
+        "config": _config(wl, world),
+        "step_us": ms_step * 1e3,
+        "drafts_per_s": units / B / Lb * B * g / (ms_step * 1e-3),
+        "step_roofline_frac": step_roof_s / (ms_step * 1e-3),
+        "roofline": roof,
+        "attention": {"avg_us": attn_avg_s * 1e6, "algorithmic_bytes": attn_bytes,
+                      "achieved_gbs": attn_bytes / attn_avg_s / 1e9 if attn_n else None,
+                      "frac_hbm": attn_bytes / attn_avg_s / 1e9 / hbm if attn_n else None},
+        "head_call_us": headall_ms * 1e3 / max(headall_n, 1),
+        "mean_accepted": mean_accepted,
+        "e2e": {"value": e2e_units / (e2e_ms * 1e-3), "unit": UNIT, "ms_per_step": e2e_ms,
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "api": "rv_verify_step_host (pinned host buffers, synchronous)"},
+        "gpu_launches": launches,
+        "clocks": clk,
+    }
+    if rank == 0 and not args.no_cpu_baseline and world == 1:
+        t_full, sample, spent = cpu_step_estimate(inp, drafts_np, args.cpu_seconds)
+        line["cpu_baseline"] = {"value": B * Lb / t_full, "unit": UNIT, "cores": cores_used(),
+                                "kind": "oracle", "sample": sample, "seconds": spent}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    h.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,228 @@
+/*
+ * rv.h -- C ABI of the GB300 (sm_103a) verify step of Reflective Verification
+ * (arXiv 2505.18629, "Think Before You Accept").
+ *
+ * The target model verifies gamma draft tokens x_1..x_gamma in ONE forward pass
+ * over the packed block (Eq. 1, Alg. 1)
+ *
+ *     [x_1..x_gamma | template | x_1..x_gamma],   template = prompt || prefix,
+ *
+ * of length Lb = 2*gamma + R (R = |template|).  The first segment yields the
+ * original logits o_1..o_{gamma+1}, the copy after the template yields the
+ * reflective logits o_m..o_{m+gamma}, m = gamma + R + 1 (Alg. 1).  They are
+ * fused as p_i = softmax((1-alpha) o_i + alpha o_{m+i-1}) (Eq. 2) and the
+ * drafts are checked by exact match against the greedy choice of p_i (Alg. 2),
+ * keeping the longest accepted prefix.
+ *
+ * Conventions for every entry point
+ *   - Tensor arguments are DEVICE pointers to caller-owned, contiguous,
+ *     row-major memory on the handle's device, unless the name ends in _host.
+ *     bf16 tensors hold IEEE bfloat16 bit patterns; with RV_DTYPE_F32 the same
+ *     arguments hold float32.  Ids and lengths are int32.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *     Calls only enqueue work on it: they never synchronize (except the
+ *     functions documented as synchronous) and are safe to capture in a CUDA
+ *     graph.
+ *   - The handle owns only its scratch workspace (allocated once in rv_create).
+ *     Calls that share a handle must be ordered on one stream.
+ *   - Return 0 (RV_OK) on success or a negative RV_ERR_* code; the message is
+ *     available from rv_last_error().  Arguments are validated on the host
+ *     before anything is launched.  Values that live in device memory
+ *     (ctx_lens, draft ids) are checked by the kernels: an out-of-range value
+ *     is skipped (never dereferenced) and raises a bit in the device status
+ *     word read by rv_read_status().  No kernel traps or asserts.
+ */
+#ifndef RV_H_
+#define RV_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#define RV_API __attribute__((visibility("default")))
+#else
+#define RV_API
+#endif
+
+/* ---- status codes ------------------------------------------------------- */
+#define RV_OK 0
+#define RV_ERR_INVALID_ARG (-1)     /* NULL pointer, bad enum, alpha not finite */
+#define RV_ERR_SHAPE (-2)           /* sizes inconsistent with the config */
+#define RV_ERR_CAPACITY (-3)        /* batch / gamma / template above the config maxima */
+#define RV_ERR_CUDA (-4)            /* a CUDA runtime call or launch failed */
+#define RV_ERR_NOT_IMPLEMENTED (-5) /* combination not built (e.g. head_dim) */
+#define RV_ERR_UNSUPPORTED (-6)     /* device is not sm_103 / lacks resources */
+#define RV_ERR_DEVICE (-7)          /* rv_read_status found a device-side error bit */
+
+/* ---- device status bits (rv_read_status) -------------------------------- */
+#define RV_DEV_CTX_RANGE 1u     /* ctx_len < 0 or ctx_len + Lb > max_ctx: sequence skipped */
+#define RV_DEV_DRAFT_RANGE 2u   /* draft id outside [0, vocab): treated as rejected */
+#define RV_DEV_TIMEOUT 4u       /* a pipeline wait in a kernel gave up (no hang) */
+
+/* ---- data types ---------------------------------------------------------- */
+#define RV_DTYPE_BF16 0         /* bf16 storage, fp32 accumulation (tensor cores) */
+#define RV_DTYPE_F32 1          /* fp32 storage and accumulation (CUDA cores) */
+
+/* ---- per-position scores written by rv_verify_head ---------------------- */
+#define RV_NSCORES 6
+#define RV_SCORE_LSE_ORIG 0     /* logsumexp_v o_i[v]                         */
+#define RV_SCORE_LSE_REFL 1     /* logsumexp_v o_{m+i-1}[v]                   */
+#define RV_SCORE_LSE_FUSED 2    /* logsumexp_v z_i[v], z_i = (1-a)o_i + a o'_i */
+#define RV_SCORE_LOGP_FUSED 3   /* log p_i(x_i) = z_i[x_i] - lse_fused (NaN at i = gamma+1) */
+#define RV_SCORE_LOGP_ORIG 4    /* o_i[x_i] - lse_orig                        */
+#define RV_SCORE_LOGP_REFL 5    /* o'_i[x_i] - lse_refl                       */
+
+/* Model / capacity description fixed at creation. */
+typedef struct rv_config {
+    int32_t hidden;       /* H: hidden size (multiple of 8)                     */
+    int32_t vocab;        /* V: LM-head rows                                    */
+    int32_t n_q_heads;    /* Hq                                                 */
+    int32_t n_kv_heads;   /* Hkv (Hq % Hkv == 0; query head h uses h / (Hq/Hkv)) */
+    int32_t head_dim;     /* D: 64 or 128 for bf16; multiple of 32, <= 256 for f32 */
+    int32_t max_batch;    /* largest B of any call                               */
+    int32_t max_gamma;    /* largest gamma                                        */
+    int32_t max_template; /* largest R = |template|                               */
+    int32_t max_ctx;      /* KV-cache capacity Cmax (positions per sequence)      */
+    int32_t dtype;        /* RV_DTYPE_BF16 or RV_DTYPE_F32                        */
+} rv_config;
+
+typedef struct rv_handle rv_handle;
+
+/* Create a handle on the current CUDA device.  Validates the config, checks
+ * that the device is sm_103, and allocates the scratch workspace (attention
+ * split partials, head partial statistics, gathered hidden rows, status word,
+ * staging for rv_verify_step_host).  The library owns that memory until
+ * rv_destroy.  *out is set only on success. */
+RV_API int rv_create(const rv_config* cfg, rv_handle** out);
+
+/* Free the handle and its workspace.  Synchronizes the device first.  NULL is a no-op. */
+RV_API int rv_destroy(rv_handle* h);
+
+/* Message of the last failed call on this handle ("" if none).  Valid until the
+ * next call on the handle.  h == NULL returns the last rv_create failure. */
+RV_API const char* rv_last_error(const rv_handle* h);
+
+/* Workspace bytes the handle holds (for capacity planning). */
+RV_API int rv_workspace_bytes(const rv_handle* h, uint64_t* bytes);
+
+/* Build the verify block of Eq. 1 / Alg. 1 ("reflective_draft") for each sequence:
+ *   block_ids[b] = [x_1..x_gamma, prompt_1..prompt_P, prefix_1..prefix_L, x_1..x_gamma]
+ *   pos_ids[b][j] = ctx_lens[b] + j            (positions run on from the context)
+ * draft_ids [B, gamma]; prompt_ids [n_prompt] (shared by all sequences, may be
+ * NULL if n_prompt == 0); prefix_ids [B, n_prefix] (the last n_prefix context
+ * tokens of each sequence: Prefix_position of Eq. 1); ctx_lens [B].
+ * Outputs block_ids, pos_ids [B, Lb], Lb = 2*gamma + n_prompt + n_prefix. */
+RV_API int rv_pack_block(rv_handle* h, const int32_t* draft_ids, const int32_t* prompt_ids,
+                         const int32_t* prefix_ids, const int32_t* ctx_lens, int32_t B,
+                         int32_t gamma, int32_t n_prompt, int32_t n_prefix, int32_t* block_ids,
+                         int32_t* pos_ids, void* stream);
+
+/* One attention layer of the verify forward pass (Sec. 3.1): causal attention
+ * of the block's queries against the KV cache plus the block itself.  Query j
+ * of sequence b (position ctx_b + j) attends to cached keys [0, ctx_b) and
+ * block keys [0, j]; query head h reads KV head h / (Hq / Hkv).
+ *   q      [B, Lb, Hq, D]   post-RoPE queries
+ *   k_blk  [B, Lb, Hkv, D]  post-RoPE keys of the block; v_blk likewise
+ *   k_cache, v_cache [B, Hkv, max_ctx, D]: read at [0, ctx_b); the block's
+ *          keys/values are written at [ctx_b, ctx_b + Lb) (the append; the
+ *          caller prunes by advancing ctx_lens, see rv_accept)
+ *   ctx_lens [B]  (device)
+ *   out    [B, Lb, Hq, D]   softmax(q K^T / sqrt(D)) V
+ * A sequence with ctx_b < 0 or ctx_b + Lb > max_ctx is skipped (its output
+ * rows are left untouched) and RV_DEV_CTX_RANGE is raised. */
+RV_API int rv_verify_attention(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
+                               void* k_cache, void* v_cache, const int32_t* ctx_lens, int32_t B,
+                               int32_t Lb, void* out, void* stream);
+
+/* LM head + fusion for the original and reflective rows (Alg. 1, Eq. 2),
+ * without ever writing logits to memory.
+ *   hidden [B, Lb+1, H]: row 0 = last context position (gives o_1), row r =
+ *          after block token r-1.  Original rows 0..gamma, reflective rows
+ *          gamma+R .. 2*gamma+R (shift_len = gamma + R = m - 1).
+ *   w_head [V, H] LM-head weight (no bias)
+ *   draft_ids [B, gamma] (device)
+ *   alpha  weight of the reflective logits (Eq. 2; the paper uses 0.3)
+ * Outputs, per sequence b and position i = 1..gamma+1 (index i-1):
+ *   scores [B, gamma+1, RV_NSCORES] float (see RV_SCORE_*)
+ *   argmax [B, gamma+1] int32: greedy choice x^_i = argmax_v z_i[v]; ties go to
+ *          the lowest token id
+ *   margin [B, gamma] float: |z_i[x_i] - max_{v != x_i} z_i[v]|, the distance of
+ *          the accept decision from its boundary (fused-logit units)
+ * A draft id outside [0, V) raises RV_DEV_DRAFT_RANGE; its position gets NaN
+ * log-probabilities and margin and an argmax that can never equal it. */
+RV_API int rv_verify_head(rv_handle* h, const void* hidden, const void* w_head,
+                          const int32_t* draft_ids, int32_t B, int32_t gamma, int32_t R,
+                          float alpha, float* scores, int32_t* argmax, float* margin,
+                          void* stream);
+
+/* Exact-match verification (Alg. 2) with the greedy choice, prefix and next token:
+ *   accept_mask[b][i-1] = (x_i == x^_i)                         uint8 [B, gamma]
+ *   accepted_len[b] = n = min({i-1 : x_i != x^_i} U {gamma})    int32 [B]
+ *   next_token[b]   = t = x^_{n+1}                              int32 [B]
+ *   ctx_out[b]      = ctx_in[b] + n   (prunes template, copy and rejected
+ *                     drafts from the cache by length; may alias ctx_in)
+ * argmax [B, gamma+1] as written by rv_verify_head. */
+RV_API int rv_accept(rv_handle* h, const int32_t* draft_ids, const int32_t* argmax, int32_t B,
+                     int32_t gamma, uint8_t* accept_mask, int32_t* accepted_len,
+                     int32_t* next_token, const int32_t* ctx_in, int32_t* ctx_out, void* stream);
+
+/* The whole verify step on device buffers: rv_verify_attention, rv_verify_head
+ * and rv_accept in order on one stream (the block ids, if wanted, come from
+ * rv_pack_block).  Arguments as in those calls; R is the template length. */
+RV_API int rv_verify_step(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
+                          void* k_cache, void* v_cache, const void* hidden, const void* w_head,
+                          const int32_t* draft_ids, const int32_t* ctx_in, int32_t B,
+                          int32_t gamma, int32_t R, float alpha, void* attn_out, float* scores,
+                          int32_t* argmax, float* margin, uint8_t* accept_mask,
+                          int32_t* accepted_len, int32_t* next_token, int32_t* ctx_out,
+                          void* stream);
+
+/* The whole verify step from HOST buffers (synchronous).  The per-step inputs
+ * (q, k_blk, v_blk, hidden, draft ids, ctx lens) are copied from host memory
+ * (pinned memory gives asynchronous copies) into the handle's device staging,
+ * the step runs, and the per-step results are copied back into host memory
+ * before the call returns.  The model state stays on the device: w_head,
+ * k_cache and v_cache are device pointers.  Host buffers have the layouts of
+ * rv_verify_step; attn_out_host may be NULL to skip reading the attention
+ * output back.  *h2d_bytes / *d2h_bytes (optional) receive the bytes copied. */
+RV_API int rv_verify_step_host(rv_handle* h, const void* q_host, const void* k_blk_host,
+                               const void* v_blk_host, void* k_cache, void* v_cache,
+                               const void* hidden_host, const void* w_head,
+                               const int32_t* draft_ids_host, const int32_t* ctx_in_host,
+                               int32_t B, int32_t gamma, int32_t R, float alpha,
+                               void* attn_out_host, float* scores_host, int32_t* argmax_host,
+                               float* margin_host, uint8_t* accept_mask_host,
+                               int32_t* accepted_len_host, int32_t* next_token_host,
+                               int32_t* ctx_out_host, uint64_t* h2d_bytes, uint64_t* d2h_bytes,
+                               void* stream);
+
+/* Synchronize `stream`, read the device status word (RV_DEV_* bits) into
+ * *status and clear it.  Returns RV_ERR_DEVICE if any bit was set. */
+RV_API int rv_read_status(rv_handle* h, void* stream, uint32_t* status);
+
+/* ---- kernel timing (CUDA events recorded by the library itself) ---------- */
+#define RV_PROF_ATTENTION 0   /* attention kernels of rv_verify_attention */
+#define RV_PROF_HEAD_GEMM 1   /* the LM-head GEMM + online log-softmax kernel */
+#define RV_PROF_HEAD 2        /* everything rv_verify_head launches */
+#define RV_PROF_ACCEPT 3      /* rv_accept */
+#define RV_PROF_COUNT 4
+
+/* enable != 0: from now on, record a CUDA event pair on the launching stream
+ * around each profiled region (up to 4096 per region, then recording stops).
+ * Not for use inside graph capture. */
+RV_API int rv_profile_enable(rv_handle* h, int32_t enable);
+/* Synchronize the recorded events and return the summed duration (ms) and
+ * number of recorded launches of `region`; then forget them. */
+RV_API int rv_profile_read(rv_handle* h, int32_t region, double* total_ms, int32_t* count);
+
+/* Number of kernel launches the library has issued on this handle (all
+ * entry points), for launch accounting. */
+RV_API int rv_launch_count(const rv_handle* h, uint64_t* count);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* RV_H_ */

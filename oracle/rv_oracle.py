@@ -186,6 +186,8 @@ def verify_head(W, hidden, drafts, gamma: int, R: int, alpha: float):
       logp_fused, logp_orig, logp_refl     [B, gamma]  (at the draft x_i)
       argmax                               [B, gamma+1] (greedy x^_i)
       margin                               [B, gamma]  |z_i[x_i] - max_{v != x_i} z_i[v]|
+      choice_gap                           [B, gamma+1] z_i[x^_i] - max_{v != x^_i} z_i[v]
+                                           (how far the greedy choice is from a tie)
       z                                    [B, gamma+1, V] fused logits
     """
     hidden = as_f64(hidden)
@@ -207,12 +209,16 @@ def verify_head(W, hidden, drafts, gamma: int, R: int, alpha: float):
     z_others = z[:, :gamma, :].copy()
     z_others[bi, ii, drafts] = -np.inf
     margin = np.abs(zx - z_others.max(axis=-1))
+    choice = greedy_choice(z)
+    z_rest = z.copy()
+    np.put_along_axis(z_rest, choice[..., None], -np.inf, axis=-1)
+    choice_gap = np.take_along_axis(z, choice[..., None], axis=-1)[..., 0] - z_rest.max(axis=-1)
     return dict(
         lse_orig=lse_o, lse_refl=lse_r, lse_fused=lse_z,
         logp_fused=zx - lse_z[:, :gamma],
         logp_orig=o[bi, ii, drafts] - lse_o[:, :gamma],
         logp_refl=o_refl[bi, ii, drafts] - lse_r[:, :gamma],
-        argmax=greedy_choice(z), margin=margin, z=z,
+        argmax=choice, margin=margin, choice_gap=choice_gap, z=z,
     )
 
 

@@ -1,0 +1,650 @@
+// Host side of the C ABI declared in include/rv.h: argument validation,
+// workspace ownership, launch planning, TMA descriptor encoding, device
+// status, kernel timing.  Every compute step runs in the CUDA kernels.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "rv.h"
+#include "rv_kernels.h"
+
+using namespace rv;
+
+namespace {
+
+thread_local std::string g_create_error;
+
+struct ProfRegion {
+  std::vector<cudaEvent_t> ev;  // pairs: [2i] start, [2i+1] stop
+  int used = 0;
+};
+constexpr int PROF_PAIRS = 1024;
+
+struct Workspace {
+  void* base = nullptr;
+  size_t bytes = 0;
+  unsigned* status = nullptr;
+  float* head_partials = nullptr;
+  float* gathered = nullptr;
+  void* hsel = nullptr;
+  float* attn_part = nullptr;  // part_o followed by part_ml
+  size_t attn_part_floats = 0;
+  // staging for rv_verify_step_host
+  void* st_q = nullptr;
+  void* st_kb = nullptr;
+  void* st_vb = nullptr;
+  void* st_hidden = nullptr;
+  void* st_attn = nullptr;
+  int32_t* st_drafts = nullptr;
+  int32_t* st_ctx_in = nullptr;
+  int32_t* st_ctx_out = nullptr;
+  float* st_scores = nullptr;
+  int32_t* st_argmax = nullptr;
+  float* st_margin = nullptr;
+  uint8_t* st_accept = nullptr;
+  int32_t* st_acc_len = nullptr;
+  int32_t* st_next = nullptr;
+};
+
+}  // namespace
+
+struct rv_handle {
+  rv_config cfg;
+  int device = 0;
+  int num_sms = 0;
+  size_t smem_optin = 0;
+  Workspace ws;
+  std::string err;
+  PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+  // cached tensor maps
+  const void* tm_w_ptr = nullptr;
+  CUtensorMap tm_w;
+  int tm_h_N = -1;
+  int tm_h_rows = -1;
+  CUtensorMap tm_h;
+  bool profiling = false;
+  ProfRegion prof[RV_PROF_COUNT];
+  unsigned long long launches = 0;
+  int head_tc_stages_cached_N = -1;
+  int head_tc_stages = 0;
+};
+
+namespace {
+
+int fail(rv_handle* h, int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  if (h)
+    h->err = buf;
+  else
+    g_create_error = buf;
+  return code;
+}
+
+int cuda_fail(rv_handle* h, cudaError_t e, const char* what) {
+  return fail(h, RV_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+size_t esize(const rv_config& c) { return c.dtype == RV_DTYPE_BF16 ? 2 : 4; }
+int lb_max(const rv_config& c) { return 2 * c.max_gamma + c.max_template; }
+
+HeadPlan head_plan(int B, int gamma, int V, int num_sms, bool tc) {
+  HeadPlan p;
+  p.P = B * (gamma + 1);
+  p.n_chunks = (p.P + MAX_PAIRS_PER_CHUNK - 1) / MAX_PAIRS_PER_CHUNK;
+  p.pairs_per_chunk = (p.P + p.n_chunks - 1) / p.n_chunks;
+  p.pad_pairs = (p.pairs_per_chunk + 7) / 8 * 8;
+  p.N = 2 * p.pad_pairs;
+  p.n_vtiles = (V + 127) / 128;
+  const int per_chunk = std::max(1, (tc ? num_sms : 4 * num_sms) / p.n_chunks);
+  p.slots = std::max(1, std::min(per_chunk, p.n_vtiles));
+  return p;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+struct ProfScope {
+  rv_handle* h;
+  int region;
+  cudaStream_t s;
+  int idx = -1;
+  ProfScope(rv_handle* h_, int r, cudaStream_t s_) : h(h_), region(r), s(s_) {
+    if (h->profiling && h->prof[r].used < PROF_PAIRS) {
+      idx = h->prof[r].used++;
+      cudaEventRecord(h->prof[r].ev[2 * idx], s);
+    }
+  }
+  ~ProfScope() {
+    if (idx >= 0) cudaEventRecord(h->prof[region].ev[2 * idx + 1], s);
+  }
+};
+
+int validate_config(const rv_config* c) {
+  if (!c) return fail(nullptr, RV_ERR_INVALID_ARG, "cfg is NULL");
+  if (c->dtype != RV_DTYPE_BF16 && c->dtype != RV_DTYPE_F32)
+    return fail(nullptr, RV_ERR_INVALID_ARG, "dtype %d is neither RV_DTYPE_BF16 nor RV_DTYPE_F32",
+                c->dtype);
+  if (c->hidden <= 0 || c->vocab <= 0 || c->n_q_heads <= 0 || c->n_kv_heads <= 0 ||
+      c->head_dim <= 0 || c->max_batch <= 0 || c->max_gamma <= 0 || c->max_template < 0 ||
+      c->max_ctx <= 0)
+    return fail(nullptr, RV_ERR_INVALID_ARG, "config sizes must be positive (max_template >= 0)");
+  if (c->hidden % 8 != 0)
+    return fail(nullptr, RV_ERR_SHAPE, "hidden %d is not a multiple of 8", c->hidden);
+  if (c->n_q_heads % c->n_kv_heads != 0)
+    return fail(nullptr, RV_ERR_SHAPE, "n_q_heads %d is not a multiple of n_kv_heads %d",
+                c->n_q_heads, c->n_kv_heads);
+  if (c->dtype == RV_DTYPE_BF16 && c->head_dim != 64 && c->head_dim != 128)
+    return fail(nullptr, RV_ERR_NOT_IMPLEMENTED, "bf16 attention is built for head_dim 64/128, not %d",
+                c->head_dim);
+  if (c->dtype == RV_DTYPE_F32 && (c->head_dim % 32 != 0 || c->head_dim > 256))
+    return fail(nullptr, RV_ERR_NOT_IMPLEMENTED,
+                "fp32 attention needs head_dim a multiple of 32 and <= 256, not %d", c->head_dim);
+  if (c->max_gamma > 64 || c->max_template > 256)
+    return fail(nullptr, RV_ERR_CAPACITY, "max_gamma <= 64 and max_template <= 256 are supported");
+  if (static_cast<long long>(c->max_batch) * (c->max_gamma + 1) > (1 << 20))
+    return fail(nullptr, RV_ERR_CAPACITY, "max_batch * (max_gamma + 1) too large");
+  return RV_OK;
+}
+
+}  // namespace
+
+// ============================================================================ create / destroy
+
+extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
+  g_create_error.clear();
+  if (!out) return fail(nullptr, RV_ERR_INVALID_ARG, "out is NULL");
+  int rc = validate_config(cfg);
+  if (rc != RV_OK) return rc;
+
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail(nullptr, RV_ERR_CUDA, "no CUDA device: %s", cudaGetErrorString(e));
+  cudaDeviceProp prop;
+  e = cudaGetDeviceProperties(&prop, dev);
+  if (e != cudaSuccess) return fail(nullptr, RV_ERR_CUDA, "cudaGetDeviceProperties: %s", cudaGetErrorString(e));
+  if (!(prop.major == 10 && prop.minor == 3))
+    return fail(nullptr, RV_ERR_UNSUPPORTED, "librv is built for sm_103a; device is sm_%d%d (%s)",
+                prop.major, prop.minor, prop.name);
+
+  rv_handle* h = new (std::nothrow) rv_handle();
+  if (!h) return fail(nullptr, RV_ERR_CUDA, "out of host memory");
+  h->cfg = *cfg;
+  h->device = dev;
+  h->num_sms = prop.multiProcessorCount;
+  h->smem_optin = prop.sharedMemPerBlockOptin;
+  const bool bf16 = cfg->dtype == RV_DTYPE_BF16;
+  const rv_config& c = *cfg;
+  const int Lbm = lb_max(c);
+
+  // ---- workspace layout (every piece 256-byte aligned)
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off += (bytes + 255) / 256 * 256;
+    return o;
+  };
+  const size_t o_status = take(256);
+  const int Pmax = c.max_batch * (c.max_gamma + 1);
+  const int slots_max = 4 * h->num_sms;
+  const size_t o_part = take(static_cast<size_t>(slots_max) * Pmax * HEAD_STAT_FIELDS * 4);
+  const size_t o_gath = take(static_cast<size_t>(Pmax) * GATHER_FIELDS * 4);
+  size_t hsel_rows = 0;
+  if (bf16) {
+    for (int P = 1; P <= Pmax; ++P) {
+      const int nch = (P + MAX_PAIRS_PER_CHUNK - 1) / MAX_PAIRS_PER_CHUNK;
+      const int pc = (P + nch - 1) / nch;
+      hsel_rows = std::max(hsel_rows, static_cast<size_t>(nch) * 2 * ((pc + 7) / 8 * 8));
+    }
+  }
+  const size_t o_hsel = take(hsel_rows * c.hidden * 2);
+  size_t attn_floats = 0;
+  if (bf16) {
+    for (int B = 1; B <= c.max_batch; ++B)
+      for (int Lb = 1; Lb <= Lbm; ++Lb)
+        attn_floats = std::max(attn_floats,
+                               attn_partial_floats(attn_plan(B, Lb, c.n_q_heads, c.n_kv_heads,
+                                                             c.max_ctx, h->num_sms, true),
+                                                   B, Lb, c.n_q_heads, c.head_dim));
+  }
+  const size_t o_attn = take(attn_floats * 4);
+  const size_t es = esize(c);
+  const size_t n_q = static_cast<size_t>(c.max_batch) * Lbm * c.n_q_heads * c.head_dim;
+  const size_t n_kv = static_cast<size_t>(c.max_batch) * Lbm * c.n_kv_heads * c.head_dim;
+  const size_t n_hid = static_cast<size_t>(c.max_batch) * (Lbm + 1) * c.hidden;
+  const size_t o_q = take(n_q * es), o_kb = take(n_kv * es), o_vb = take(n_kv * es);
+  const size_t o_hid = take(n_hid * es), o_ao = take(n_q * es);
+  const size_t o_dr = take(static_cast<size_t>(c.max_batch) * c.max_gamma * 4);
+  const size_t o_ci = take(c.max_batch * 4), o_co = take(c.max_batch * 4);
+  const size_t o_sc = take(static_cast<size_t>(Pmax) * RV_NSCORES * 4);
+  const size_t o_am = take(static_cast<size_t>(Pmax) * 4);
+  const size_t o_mg = take(static_cast<size_t>(c.max_batch) * c.max_gamma * 4);
+  const size_t o_acc = take(static_cast<size_t>(c.max_batch) * c.max_gamma);
+  const size_t o_al = take(c.max_batch * 4), o_nt = take(c.max_batch * 4);
+
+  e = cudaMalloc(&h->ws.base, off);
+  if (e != cudaSuccess) {
+    delete h;
+    return fail(nullptr, RV_ERR_CUDA, "workspace cudaMalloc(%zu): %s", off, cudaGetErrorString(e));
+  }
+  h->ws.bytes = off;
+  char* b = static_cast<char*>(h->ws.base);
+  h->ws.status = reinterpret_cast<unsigned*>(b + o_status);
+  h->ws.head_partials = reinterpret_cast<float*>(b + o_part);
+  h->ws.gathered = reinterpret_cast<float*>(b + o_gath);
+  h->ws.hsel = b + o_hsel;
+  h->ws.attn_part = reinterpret_cast<float*>(b + o_attn);
+  h->ws.attn_part_floats = attn_floats;
+  h->ws.st_q = b + o_q;
+  h->ws.st_kb = b + o_kb;
+  h->ws.st_vb = b + o_vb;
+  h->ws.st_hidden = b + o_hid;
+  h->ws.st_attn = b + o_ao;
+  h->ws.st_drafts = reinterpret_cast<int32_t*>(b + o_dr);
+  h->ws.st_ctx_in = reinterpret_cast<int32_t*>(b + o_ci);
+  h->ws.st_ctx_out = reinterpret_cast<int32_t*>(b + o_co);
+  h->ws.st_scores = reinterpret_cast<float*>(b + o_sc);
+  h->ws.st_argmax = reinterpret_cast<int32_t*>(b + o_am);
+  h->ws.st_margin = reinterpret_cast<float*>(b + o_mg);
+  h->ws.st_accept = reinterpret_cast<uint8_t*>(b + o_acc);
+  h->ws.st_acc_len = reinterpret_cast<int32_t*>(b + o_al);
+  h->ws.st_next = reinterpret_cast<int32_t*>(b + o_nt);
+  e = cudaMemset(h->ws.base, 0, off);
+  if (e == cudaSuccess && bf16) e = attn_configure();
+  if (e == cudaSuccess && bf16) e = head_tc_configure(h->smem_optin);
+  if (e == cudaSuccess && bf16) {
+    cudaDriverEntryPointQueryResult q;
+    void* fn = nullptr;
+    e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (e == cudaSuccess && (q != cudaDriverEntryPointSuccess || !fn)) e = cudaErrorNotSupported;
+    h->encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  }
+  if (e != cudaSuccess) {
+    cudaFree(h->ws.base);
+    delete h;
+    return fail(nullptr, RV_ERR_CUDA, "rv_create setup: %s", cudaGetErrorString(e));
+  }
+  *out = h;
+  return RV_OK;
+}
+
+extern "C" RV_API int rv_destroy(rv_handle* h) {
+  if (!h) return RV_OK;
+  cudaDeviceSynchronize();
+  for (auto& r : h->prof)
+    for (auto ev : r.ev) cudaEventDestroy(ev);
+  cudaFree(h->ws.base);
+  delete h;
+  return RV_OK;
+}
+
+extern "C" RV_API const char* rv_last_error(const rv_handle* h) {
+  return h ? h->err.c_str() : g_create_error.c_str();
+}
+
+extern "C" RV_API int rv_workspace_bytes(const rv_handle* h, uint64_t* bytes) {
+  if (!h || !bytes) return RV_ERR_INVALID_ARG;
+  *bytes = h->ws.bytes;
+  return RV_OK;
+}
+
+// ============================================================================ pack
+
+extern "C" RV_API int rv_pack_block(rv_handle* h, const int32_t* draft_ids, const int32_t* prompt_ids,
+                                    const int32_t* prefix_ids, const int32_t* ctx_lens, int32_t B,
+                                    int32_t gamma, int32_t n_prompt, int32_t n_prefix,
+                                    int32_t* block_ids, int32_t* pos_ids, void* stream) {
+  if (!h) return RV_ERR_INVALID_ARG;
+  h->err.clear();
+  if (B < 0 || gamma < 0 || n_prompt < 0 || n_prefix < 0)
+    return fail(h, RV_ERR_SHAPE, "negative size");
+  if (B > h->cfg.max_batch || gamma > h->cfg.max_gamma || n_prompt + n_prefix > h->cfg.max_template)
+    return fail(h, RV_ERR_CAPACITY, "B/gamma/template above the handle's maxima");
+  if (B == 0) return RV_OK;
+  if (!draft_ids || !ctx_lens || !block_ids || !pos_ids || (n_prompt > 0 && !prompt_ids) ||
+      (n_prefix > 0 && !prefix_ids))
+    return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument");
+  cudaError_t e = launch_pack_block(draft_ids, prompt_ids, prefix_ids, ctx_lens, B, gamma, n_prompt,
+                                    n_prefix, block_ids, pos_ids, static_cast<cudaStream_t>(stream));
+  h->launches += 1;
+  return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "pack_block launch");
+}
+
+// ============================================================================ attention
+
+extern "C" RV_API int rv_verify_attention(rv_handle* h, const void* q, const void* k_blk,
+                                          const void* v_blk, void* k_cache, void* v_cache,
+                                          const int32_t* ctx_lens, int32_t B, int32_t Lb, void* out,
+                                          void* stream) {
+  if (!h) return RV_ERR_INVALID_ARG;
+  h->err.clear();
+  const rv_config& c = h->cfg;
+  if (B < 0 || Lb < 0) return fail(h, RV_ERR_SHAPE, "negative B or Lb");
+  if (B > c.max_batch || Lb > lb_max(c))
+    return fail(h, RV_ERR_CAPACITY, "B %d / Lb %d above max_batch %d / 2*max_gamma+max_template %d",
+                B, Lb, c.max_batch, lb_max(c));
+  if (B == 0 || Lb == 0) return RV_OK;
+  if (!q || !k_blk || !v_blk || !k_cache || !v_cache || !ctx_lens || !out)
+    return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument");
+  const bool bf16 = c.dtype == RV_DTYPE_BF16;
+  if (!aligned16(q) || !aligned16(k_blk) || !aligned16(v_blk) || !aligned16(k_cache) ||
+      !aligned16(v_cache) || !aligned16(out))
+    return fail(h, RV_ERR_INVALID_ARG, "attention tensors must be 16-byte aligned");
+  AttnArgs a{q, k_blk, v_blk, k_cache, v_cache, ctx_lens, out, B, Lb, c.n_q_heads, c.n_kv_heads,
+             c.head_dim, c.max_ctx, h->ws.status};
+  const AttnPlan p = attn_plan(B, Lb, c.n_q_heads, c.n_kv_heads, c.max_ctx, h->num_sms, bf16);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  ProfScope prof(h, RV_PROF_ATTENTION, s);
+  cudaError_t e;
+  if (bf16) {
+    const size_t nf = attn_partial_floats(p, B, Lb, c.n_q_heads, c.head_dim);
+    if (nf > h->ws.attn_part_floats) return fail(h, RV_ERR_CAPACITY, "attention workspace too small");
+    float* part_o = h->ws.attn_part;
+    float* part_ml = part_o + static_cast<size_t>(p.splits) * B * Lb * c.n_q_heads * c.head_dim;
+    e = launch_attention_bf16(a, p, part_o, part_ml, s);
+    h->launches += 1;
+    if (e == cudaSuccess && p.splits > 1) {
+      e = launch_attention_combine(a, p, part_o, part_ml, true, s);
+      h->launches += 1;
+    }
+  } else {
+    e = launch_attention_f32(a, p, nullptr, nullptr, s);
+    h->launches += 1;
+  }
+  return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "attention launch");
+}
+
+// ============================================================================ head
+
+namespace {
+
+int encode_maps(rv_handle* h, const void* w, const HeadPlan& pl, HeadTcLaunch& l) {
+  const rv_config& c = h->cfg;
+  if (h->tm_w_ptr != w) {
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(c.hidden), static_cast<cuuint64_t>(c.vocab)};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(c.hidden) * 2};
+    const cuuint32_t box[2] = {64, 128};
+    const cuuint32_t es[2] = {1, 1};
+    CUresult r = h->encode(&h->tm_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(w), dims,
+                           strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                           CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+      h->tm_w_ptr = nullptr;
+      return fail(h, RV_ERR_CUDA, "cuTensorMapEncodeTiled(W) failed: %d", static_cast<int>(r));
+    }
+    h->tm_w_ptr = w;
+  }
+  const int rows = pl.n_chunks * pl.N;
+  if (h->tm_h_N != pl.N || h->tm_h_rows != rows) {
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(c.hidden), static_cast<cuuint64_t>(rows)};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(c.hidden) * 2};
+    const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(pl.N)};
+    const cuuint32_t es[2] = {1, 1};
+    CUresult r = h->encode(&h->tm_h, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, h->ws.hsel, dims, strides,
+                           box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+      h->tm_h_N = -1;
+      return fail(h, RV_ERR_CUDA, "cuTensorMapEncodeTiled(hidden rows) failed: %d", static_cast<int>(r));
+    }
+    h->tm_h_N = pl.N;
+    h->tm_h_rows = rows;
+  }
+  l.tm_w = h->tm_w;
+  l.tm_h = h->tm_h;
+  if (h->head_tc_stages_cached_N != pl.N) {
+    h->head_tc_stages = head_tc_max_stages(pl.N, h->smem_optin);
+    h->head_tc_stages_cached_N = pl.N;
+  }
+  l.stages = h->head_tc_stages;
+  if (l.stages < 2) return fail(h, RV_ERR_UNSUPPORTED, "not enough shared memory for the head pipeline");
+  l.smem_bytes = head_tc_smem_bytes(pl.N, l.stages);
+  return RV_OK;
+}
+
+int check_head_args(rv_handle* h, const void* hidden, const void* w_head, const int32_t* draft_ids,
+                    int B, int gamma, int R, float alpha, const void* o1, const void* o2,
+                    const void* o3) {
+  const rv_config& c = h->cfg;
+  if (B < 0 || gamma < 1 || R < 0) return fail(h, RV_ERR_SHAPE, "need B >= 0, gamma >= 1, R >= 0");
+  if (B > c.max_batch || gamma > c.max_gamma || R > c.max_template)
+    return fail(h, RV_ERR_CAPACITY, "B %d / gamma %d / R %d above the handle's maxima (%d/%d/%d)", B,
+                gamma, R, c.max_batch, c.max_gamma, c.max_template);
+  if (!std::isfinite(alpha)) return fail(h, RV_ERR_INVALID_ARG, "alpha is not finite");
+  if (B == 0) return RV_OK;
+  if (!hidden || !w_head || !draft_ids || !o1 || !o2 || !o3)
+    return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument");
+  if (!aligned16(hidden) || !aligned16(w_head))
+    return fail(h, RV_ERR_INVALID_ARG, "hidden and w_head must be 16-byte aligned");
+  return RV_OK;
+}
+
+int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_t* draft_ids, int B,
+              int gamma, int R, float alpha, float* scores, int32_t* argmax, float* margin,
+              cudaStream_t s) {
+  const rv_config& c = h->cfg;
+  const bool bf16 = c.dtype == RV_DTYPE_BF16;
+  HeadArgs a{hidden, w_head, draft_ids, B, gamma, R, c.vocab, c.hidden, alpha,
+             h->ws.head_partials, h->ws.gathered, h->ws.status};
+  const HeadPlan pl = head_plan(B, gamma, c.vocab, h->num_sms, bf16);
+  ProfScope prof_all(h, RV_PROF_HEAD, s);
+  cudaError_t e;
+  if (bf16) {
+    HeadTcLaunch l;
+    int rc = encode_maps(h, w_head, pl, l);
+    if (rc != RV_OK) return rc;
+    e = launch_gather_rows(a, pl, h->ws.hsel, s);
+    h->launches += 1;
+    if (e != cudaSuccess) return cuda_fail(h, e, "gather_rows launch");
+    {
+      ProfScope prof(h, RV_PROF_HEAD_GEMM, s);
+      e = launch_head_tc(a, pl, l, s);
+      h->launches += 1;
+    }
+    if (e != cudaSuccess) return cuda_fail(h, e, "head_tc launch");
+  } else {
+    {
+      ProfScope prof(h, RV_PROF_HEAD_GEMM, s);
+      e = launch_head_simt(a, pl, s);
+      h->launches += 1;
+    }
+    if (e != cudaSuccess) return cuda_fail(h, e, "head_simt launch");
+  }
+  e = launch_head_merge(a, pl, scores, argmax, margin, s);
+  h->launches += 1;
+  return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "head_merge launch");
+}
+
+int accept_impl(rv_handle* h, const int32_t* draft_ids, const int32_t* argmax, int B, int gamma,
+                uint8_t* accept_mask, int32_t* accepted_len, int32_t* next_token,
+                const int32_t* ctx_in, int32_t* ctx_out, cudaStream_t s) {
+  ProfScope prof(h, RV_PROF_ACCEPT, s);
+  cudaError_t e = launch_accept(draft_ids, argmax, B, gamma, accept_mask, accepted_len, next_token,
+                                ctx_in, ctx_out, s);
+  h->launches += 1;
+  return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "accept launch");
+}
+
+}  // namespace
+
+extern "C" RV_API int rv_verify_head(rv_handle* h, const void* hidden, const void* w_head,
+                                     const int32_t* draft_ids, int32_t B, int32_t gamma, int32_t R,
+                                     float alpha, float* scores, int32_t* argmax, float* margin,
+                                     void* stream) {
+  if (!h) return RV_ERR_INVALID_ARG;
+  h->err.clear();
+  int rc = check_head_args(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin);
+  if (rc != RV_OK || B == 0) return rc;
+  return head_impl(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin,
+                   static_cast<cudaStream_t>(stream));
+}
+
+extern "C" RV_API int rv_accept(rv_handle* h, const int32_t* draft_ids, const int32_t* argmax,
+                                int32_t B, int32_t gamma, uint8_t* accept_mask,
+                                int32_t* accepted_len, int32_t* next_token, const int32_t* ctx_in,
+                                int32_t* ctx_out, void* stream) {
+  if (!h) return RV_ERR_INVALID_ARG;
+  h->err.clear();
+  if (B < 0 || gamma < 1) return fail(h, RV_ERR_SHAPE, "need B >= 0 and gamma >= 1");
+  if (B > h->cfg.max_batch || gamma > h->cfg.max_gamma)
+    return fail(h, RV_ERR_CAPACITY, "B / gamma above the handle's maxima");
+  if (B == 0) return RV_OK;
+  if (!draft_ids || !argmax || !accept_mask || !accepted_len || !next_token || !ctx_in || !ctx_out)
+    return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument");
+  return accept_impl(h, draft_ids, argmax, B, gamma, accept_mask, accepted_len, next_token, ctx_in,
+                     ctx_out, static_cast<cudaStream_t>(stream));
+}
+
+// ============================================================================ whole step
+
+extern "C" RV_API int rv_verify_step(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
+                                     void* k_cache, void* v_cache, const void* hidden,
+                                     const void* w_head, const int32_t* draft_ids,
+                                     const int32_t* ctx_in, int32_t B, int32_t gamma, int32_t R,
+                                     float alpha, void* attn_out, float* scores, int32_t* argmax,
+                                     float* margin, uint8_t* accept_mask, int32_t* accepted_len,
+                                     int32_t* next_token, int32_t* ctx_out, void* stream) {
+  if (!h) return RV_ERR_INVALID_ARG;
+  int rc = rv_verify_attention(h, q, k_blk, v_blk, k_cache, v_cache, ctx_in, B, 2 * gamma + R,
+                               attn_out, stream);
+  if (rc != RV_OK) return rc;
+  rc = rv_verify_head(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin,
+                      stream);
+  if (rc != RV_OK) return rc;
+  return rv_accept(h, draft_ids, argmax, B, gamma, accept_mask, accepted_len, next_token, ctx_in,
+                   ctx_out, stream);
+}
+
+extern "C" RV_API int rv_verify_step_host(
+    rv_handle* h, const void* q_host, const void* k_blk_host, const void* v_blk_host, void* k_cache,
+    void* v_cache, const void* hidden_host, const void* w_head, const int32_t* draft_ids_host,
+    const int32_t* ctx_in_host, int32_t B, int32_t gamma, int32_t R, float alpha,
+    void* attn_out_host, float* scores_host, int32_t* argmax_host, float* margin_host,
+    uint8_t* accept_mask_host, int32_t* accepted_len_host, int32_t* next_token_host,
+    int32_t* ctx_out_host, uint64_t* h2d_bytes, uint64_t* d2h_bytes, void* stream) {
+  if (!h) return RV_ERR_INVALID_ARG;
+  h->err.clear();
+  const rv_config& c = h->cfg;
+  if (B < 1 || gamma < 1 || R < 0) return fail(h, RV_ERR_SHAPE, "need B >= 1, gamma >= 1, R >= 0");
+  if (B > c.max_batch || gamma > c.max_gamma || R > c.max_template)
+    return fail(h, RV_ERR_CAPACITY, "B / gamma / R above the handle's maxima");
+  if (!q_host || !k_blk_host || !v_blk_host || !k_cache || !v_cache || !hidden_host || !w_head ||
+      !draft_ids_host || !ctx_in_host || !scores_host || !argmax_host || !margin_host ||
+      !accept_mask_host || !accepted_len_host || !next_token_host || !ctx_out_host)
+    return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t es = esize(c);
+  const int Lb = 2 * gamma + R;
+  const size_t nq = static_cast<size_t>(B) * Lb * c.n_q_heads * c.head_dim * es;
+  const size_t nkv = static_cast<size_t>(B) * Lb * c.n_kv_heads * c.head_dim * es;
+  const size_t nh = static_cast<size_t>(B) * (Lb + 1) * c.hidden * es;
+  const size_t nd = static_cast<size_t>(B) * gamma * 4, nc = static_cast<size_t>(B) * 4;
+  const size_t P = static_cast<size_t>(B) * (gamma + 1);
+  Workspace& w = h->ws;
+  cudaError_t e = cudaSuccess;
+  auto h2d = [&](void* dst, const void* src, size_t n) {
+    if (e == cudaSuccess) e = cudaMemcpyAsync(dst, src, n, cudaMemcpyHostToDevice, s);
+  };
+  auto d2h = [&](void* dst, const void* src, size_t n) {
+    if (e == cudaSuccess) e = cudaMemcpyAsync(dst, src, n, cudaMemcpyDeviceToHost, s);
+  };
+  h2d(w.st_q, q_host, nq);
+  h2d(w.st_kb, k_blk_host, nkv);
+  h2d(w.st_vb, v_blk_host, nkv);
+  h2d(w.st_hidden, hidden_host, nh);
+  h2d(w.st_drafts, draft_ids_host, nd);
+  h2d(w.st_ctx_in, ctx_in_host, nc);
+  if (e != cudaSuccess) return cuda_fail(h, e, "host->device copy");
+  int rc = rv_verify_step(h, w.st_q, w.st_kb, w.st_vb, k_cache, v_cache, w.st_hidden, w_head,
+                          w.st_drafts, w.st_ctx_in, B, gamma, R, alpha, w.st_attn, w.st_scores,
+                          w.st_argmax, w.st_margin, w.st_accept, w.st_acc_len, w.st_next,
+                          w.st_ctx_out, stream);
+  if (rc != RV_OK) return rc;
+  size_t out_bytes = 0;
+  if (attn_out_host) {
+    d2h(attn_out_host, w.st_attn, nq);
+    out_bytes += nq;
+  }
+  d2h(scores_host, w.st_scores, P * RV_NSCORES * 4);
+  d2h(argmax_host, w.st_argmax, P * 4);
+  d2h(margin_host, w.st_margin, nd);
+  d2h(accept_mask_host, w.st_accept, static_cast<size_t>(B) * gamma);
+  d2h(accepted_len_host, w.st_acc_len, nc);
+  d2h(next_token_host, w.st_next, nc);
+  d2h(ctx_out_host, w.st_ctx_out, nc);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(h, e, "device->host copy");
+  out_bytes += P * RV_NSCORES * 4 + P * 4 + nd + static_cast<size_t>(B) * gamma + 3 * nc;
+  if (h2d_bytes) *h2d_bytes = nq + 2 * nkv + nh + nd + nc;
+  if (d2h_bytes) *d2h_bytes = out_bytes;
+  return RV_OK;
+}
+
+// ============================================================================ status / timing
+
+extern "C" RV_API int rv_read_status(rv_handle* h, void* stream, uint32_t* status) {
+  if (!h || !status) return RV_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  unsigned v = 0;
+  cudaError_t e = cudaStreamSynchronize(s);
+  if (e == cudaSuccess) e = cudaMemcpy(&v, h->ws.status, sizeof(v), cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess) e = cudaMemset(h->ws.status, 0, sizeof(unsigned));
+  if (e != cudaSuccess) return cuda_fail(h, e, "rv_read_status");
+  *status = v;
+  if (v != 0) return fail(h, RV_ERR_DEVICE, "device status 0x%x", v);
+  return RV_OK;
+}
+
+extern "C" RV_API int rv_profile_enable(rv_handle* h, int32_t enable) {
+  if (!h) return RV_ERR_INVALID_ARG;
+  if (enable) {
+    for (auto& r : h->prof) {
+      if (r.ev.empty()) {
+        r.ev.resize(2 * PROF_PAIRS);
+        for (auto& ev : r.ev) {
+          cudaError_t e = cudaEventCreate(&ev);
+          if (e != cudaSuccess) return cuda_fail(h, e, "cudaEventCreate");
+        }
+      }
+      r.used = 0;
+    }
+  }
+  h->profiling = enable != 0;
+  return RV_OK;
+}
+
+extern "C" RV_API int rv_profile_read(rv_handle* h, int32_t region, double* total_ms,
+                                      int32_t* count) {
+  if (!h || !total_ms || !count || region < 0 || region >= RV_PROF_COUNT) return RV_ERR_INVALID_ARG;
+  ProfRegion& r = h->prof[region];
+  double sum = 0;
+  for (int i = 0; i < r.used; ++i) {
+    cudaError_t e = cudaEventSynchronize(r.ev[2 * i + 1]);
+    float ms = 0.f;
+    if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, r.ev[2 * i], r.ev[2 * i + 1]);
+    if (e != cudaSuccess) return cuda_fail(h, e, "rv_profile_read");
+    sum += ms;
+  }
+  *total_ms = sum;
+  *count = r.used;
+  r.used = 0;
+  return RV_OK;
+}
+
+extern "C" RV_API int rv_launch_count(const rv_handle* h, uint64_t* count) {
+  if (!h || !count) return RV_ERR_INVALID_ARG;
+  *count = h->launches;
+  return RV_OK;
+}

@@ -1,0 +1,110 @@
+// Launch interface between the C-ABI host code (rv_host.cpp) and the CUDA
+// translation units.  Plain structs of sizes and device pointers; every
+// launcher enqueues on `stream` and returns the cudaGetLastError() of the launch.
+#pragma once
+
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+namespace rv {
+
+// Per-pair partial statistics written by each head CTA, merged by head_merge.
+// Layout [slot][pair][HEAD_STAT_FIELDS].
+enum HeadStat : int {
+  ST_M_O = 0,  // running max of o_i over the CTA's vocab rows
+  ST_S_O,      // sum exp(o_i - m)
+  ST_M_R,      // same for the reflective logits o'_i
+  ST_S_R,
+  ST_M_Z,      // same for the fused logits z_i
+  ST_S_Z,
+  ST_BEST_V,   // max of z_i over rows v != x_i
+  ST_BEST_I,   // its row (int bits; smallest on ties)
+  HEAD_STAT_FIELDS
+};
+constexpr int GATHER_FIELDS = 4;  // o_i[x_i], o'_i[x_i], z_i[x_i], unused
+
+// Pair p = b * (gamma + 1) + i scores x_{i+1} (none for i = gamma).  Pairs are
+// split into chunks of at most MAX_PAIRS_PER_CHUNK; chunk c holds pairs
+// [c*pairs_per_chunk, ...).  Its gathered hidden rows form a block of
+// 2*pad_pairs rows: original rows first, reflective rows after pad_pairs.
+constexpr int MAX_PAIRS_PER_CHUNK = 128;
+
+struct HeadPlan {
+  int P;               // total pairs B*(gamma+1)
+  int n_chunks;
+  int pairs_per_chunk; // Pc
+  int pad_pairs;       // Pcp = round_up(Pc, 8)
+  int N;               // 2*Pcp: MMA N (columns of the TMEM accumulator)
+  int n_vtiles;        // ceil(V / 128)
+  int slots;           // CTAs per chunk (= partial slots)
+};
+
+struct HeadArgs {
+  const void* hidden;      // [B, Lb+1, H]
+  const void* w;           // [V, H]
+  const int32_t* drafts;   // [B, gamma]
+  int B, gamma, R, V, H;
+  float alpha;
+  float* partials;         // [slots][P][HEAD_STAT_FIELDS]
+  float* gathered;         // [P][GATHER_FIELDS]
+  unsigned* status;
+};
+
+// ---- small kernels (k_small.cu)
+cudaError_t launch_pack_block(const int32_t* drafts, const int32_t* prompt, const int32_t* prefix,
+                              const int32_t* ctx, int B, int gamma, int n_prompt, int n_prefix,
+                              int32_t* block_ids, int32_t* pos_ids, cudaStream_t s);
+// hidden rows of every chunk into hsel [n_chunks * N, H] (bf16), pads zeroed
+cudaError_t launch_gather_rows(const HeadArgs& a, const HeadPlan& p, void* hsel, cudaStream_t s);
+cudaError_t launch_head_merge(const HeadArgs& a, const HeadPlan& p, float* scores,
+                              int32_t* argmax, float* margin, cudaStream_t s);
+cudaError_t launch_accept(const int32_t* drafts, const int32_t* argmax, int B, int gamma,
+                          uint8_t* accept_mask, int32_t* accepted_len, int32_t* next_token,
+                          const int32_t* ctx_in, int32_t* ctx_out, cudaStream_t s);
+
+// ---- LM head (k_head_tc.cu: bf16 tcgen05; k_head_simt.cu: fp32)
+struct HeadTcLaunch {
+  CUtensorMap tm_w;    // W [V, H] bf16, box {64, 128}, 128B swizzle
+  CUtensorMap tm_h;    // hsel [n_chunks*N, H] bf16, box {64, N}, 128B swizzle
+  int stages;
+  size_t smem_bytes;
+};
+size_t head_tc_smem_bytes(int N, int stages);
+int head_tc_max_stages(int N, size_t smem_limit);
+cudaError_t head_tc_configure(size_t smem_bytes);  // cudaFuncSetAttribute
+cudaError_t launch_head_tc(const HeadArgs& a, const HeadPlan& p, const HeadTcLaunch& l,
+                           cudaStream_t s);
+cudaError_t launch_head_simt(const HeadArgs& a, const HeadPlan& p, cudaStream_t s);
+
+// ---- attention (k_attention.cu)
+struct AttnArgs {
+  const void* q;      // [B, Lb, Hq, D]
+  const void* k_blk;  // [B, Lb, Hkv, D]
+  const void* v_blk;
+  void* k_cache;      // [B, Hkv, Cmax, D]
+  void* v_cache;
+  const int32_t* ctx;
+  void* out;          // [B, Lb, Hq, D]
+  int B, Lb, Hq, Hkv, D, Cmax;
+  unsigned* status;
+};
+struct AttnPlan {
+  int rows;        // query rows per KV head: Lb * G
+  int row_groups;  // CTAs along the rows (<= 128 rows each)
+  int splits;      // key splits
+  int warps;       // warps per CTA
+};
+AttnPlan attn_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms, bool bf16);
+size_t attn_partial_floats(const AttnPlan& p, int B, int Lb, int Hq, int D);
+size_t attn_bf16_smem_bytes(int D, int warps);
+cudaError_t attn_configure();
+// part_o [splits][B*Lb*Hq][D] fp32, part_ml [splits][B*Lb*Hq][2]
+cudaError_t launch_attention_bf16(const AttnArgs& a, const AttnPlan& p, float* part_o,
+                                  float* part_ml, cudaStream_t s);
+cudaError_t launch_attention_f32(const AttnArgs& a, const AttnPlan& p, float* part_o,
+                                 float* part_ml, cudaStream_t s);
+cudaError_t launch_attention_combine(const AttnArgs& a, const AttnPlan& p, const float* part_o,
+                                     const float* part_ml, bool bf16, cudaStream_t s);
+
+}  // namespace rv

@@ -1,0 +1,245 @@
+"""Thin ctypes binding of ``librv.so`` (declared in ``include/rv.h``).
+
+Argument marshalling only: every function passes tensor data pointers, sizes
+and the CUDA stream to the C entry point of the same name and raises
+``RVError`` on a negative status.  All compute happens in the library's CUDA
+kernels.  Importing this module fails loudly (``RVLibraryMissing``) when the
+library has not been built; there is no other code path.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_lib", "librv.so")
+
+RV_OK = 0
+RV_ERR_INVALID_ARG = -1
+RV_ERR_SHAPE = -2
+RV_ERR_CAPACITY = -3
+RV_ERR_CUDA = -4
+RV_ERR_NOT_IMPLEMENTED = -5
+RV_ERR_UNSUPPORTED = -6
+RV_ERR_DEVICE = -7
+
+RV_DEV_CTX_RANGE = 1
+RV_DEV_DRAFT_RANGE = 2
+RV_DEV_TIMEOUT = 4
+
+RV_DTYPE_BF16 = 0
+RV_DTYPE_F32 = 1
+
+RV_NSCORES = 6
+RV_SCORE_LSE_ORIG, RV_SCORE_LSE_REFL, RV_SCORE_LSE_FUSED = 0, 1, 2
+RV_SCORE_LOGP_FUSED, RV_SCORE_LOGP_ORIG, RV_SCORE_LOGP_REFL = 3, 4, 5
+
+RV_PROF_ATTENTION, RV_PROF_HEAD_GEMM, RV_PROF_HEAD, RV_PROF_ACCEPT = 0, 1, 2, 3
+
+
+class RVLibraryMissing(ImportError):
+    pass
+
+
+class RVError(RuntimeError):
+    def __init__(self, code, msg):
+        super().__init__(f"rv error {code}: {msg}")
+        self.code = code
+
+
+class rv_config(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in (
+        "hidden", "vocab", "n_q_heads", "n_kv_heads", "head_dim", "max_batch", "max_gamma",
+        "max_template", "max_ctx", "dtype")]
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise RVLibraryMissing(
+            f"{LIB_PATH} is missing: build it with `python -m paper_2505_18629_gb300.build`")
+    lib = ctypes.CDLL(LIB_PATH)
+    P, I, F, U64P = ctypes.c_void_p, ctypes.c_int32, ctypes.c_float, ctypes.POINTER(ctypes.c_uint64)
+    sig = {
+        "rv_create": (I, [ctypes.POINTER(rv_config), ctypes.POINTER(P)]),
+        "rv_destroy": (I, [P]),
+        "rv_last_error": (ctypes.c_char_p, [P]),
+        "rv_workspace_bytes": (I, [P, U64P]),
+        "rv_pack_block": (I, [P, P, P, P, P, I, I, I, I, P, P, P]),
+        "rv_verify_attention": (I, [P, P, P, P, P, P, P, I, I, P, P]),
+        "rv_verify_head": (I, [P, P, P, P, I, I, I, F, P, P, P, P]),
+        "rv_accept": (I, [P, P, P, I, I, P, P, P, P, P, P]),
+        "rv_verify_step": (I, [P, P, P, P, P, P, P, P, P, P, I, I, I, F, P, P, P, P, P, P, P, P, P]),
+        "rv_verify_step_host": (I, [P, P, P, P, P, P, P, P, P, P, I, I, I, F, P, P, P, P, P, P, P,
+                                    P, U64P, U64P, P]),
+        "rv_read_status": (I, [P, P, ctypes.POINTER(ctypes.c_uint32)]),
+        "rv_profile_enable": (I, [P, I]),
+        "rv_profile_read": (I, [P, I, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(I)]),
+        "rv_launch_count": (I, [P, U64P]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    return lib
+
+
+_lib = _load()
+
+
+def lib():
+    return _lib
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if isinstance(t, torch.Tensor):
+        if not t.is_contiguous():
+            raise ValueError("tensor arguments must be contiguous")
+        return ctypes.c_void_p(t.data_ptr())
+    return t
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    if isinstance(stream, torch.cuda.Stream):
+        return ctypes.c_void_p(stream.cuda_stream)
+    return ctypes.c_void_p(int(stream))
+
+
+class Handle:
+    """Owns an ``rv_handle*``; ``close()`` (or garbage collection) destroys it."""
+
+    def __init__(self, ptr, cfg):
+        self._p = ptr
+        self.cfg = cfg
+
+    @property
+    def ptr(self):
+        if not self._p:
+            raise ValueError("handle is closed")
+        return self._p
+
+    def close(self):
+        if self._p:
+            _lib.rv_destroy(self._p)
+            self._p = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def last_error(self) -> str:
+        return _lib.rv_last_error(self._p).decode()
+
+
+def _check(h, rc):
+    if rc != RV_OK:
+        msg = _lib.rv_last_error(h.ptr if isinstance(h, Handle) else h)
+        raise RVError(rc, msg.decode() if msg else "")
+    return rc
+
+
+def rv_create(hidden, vocab, n_q_heads, n_kv_heads, head_dim, max_batch, max_gamma,
+              max_template, max_ctx, dtype=RV_DTYPE_BF16) -> Handle:
+    cfg = rv_config(hidden, vocab, n_q_heads, n_kv_heads, head_dim, max_batch, max_gamma,
+                    max_template, max_ctx, dtype)
+    out = ctypes.c_void_p()
+    rc = _lib.rv_create(ctypes.byref(cfg), ctypes.byref(out))
+    if rc != RV_OK:
+        raise RVError(rc, _lib.rv_last_error(None).decode())
+    return Handle(out, cfg)
+
+
+def rv_workspace_bytes(h: Handle) -> int:
+    v = ctypes.c_uint64()
+    _check(h, _lib.rv_workspace_bytes(h.ptr, ctypes.byref(v)))
+    return v.value
+
+
+def rv_pack_block(h, draft_ids, prompt_ids, prefix_ids, ctx_lens, block_ids, pos_ids,
+                  stream=None):
+    B, gamma = draft_ids.shape
+    n_prompt = 0 if prompt_ids is None else prompt_ids.numel()
+    n_prefix = prefix_ids.shape[1]
+    _check(h, _lib.rv_pack_block(h.ptr, _ptr(draft_ids), _ptr(prompt_ids), _ptr(prefix_ids),
+                                 _ptr(ctx_lens), B, gamma, n_prompt, n_prefix, _ptr(block_ids),
+                                 _ptr(pos_ids), _stream(stream)))
+
+
+def rv_verify_attention(h, q, k_blk, v_blk, k_cache, v_cache, ctx_lens, out, stream=None):
+    B, Lb = q.shape[0], q.shape[1]
+    _check(h, _lib.rv_verify_attention(h.ptr, _ptr(q), _ptr(k_blk), _ptr(v_blk), _ptr(k_cache),
+                                       _ptr(v_cache), _ptr(ctx_lens), B, Lb, _ptr(out),
+                                       _stream(stream)))
+
+
+def rv_verify_head(h, hidden, w_head, draft_ids, gamma, R, alpha, scores, argmax, margin,
+                   stream=None):
+    B = hidden.shape[0]
+    _check(h, _lib.rv_verify_head(h.ptr, _ptr(hidden), _ptr(w_head), _ptr(draft_ids), B, gamma,
+                                  R, float(alpha), _ptr(scores), _ptr(argmax), _ptr(margin),
+                                  _stream(stream)))
+
+
+def rv_accept(h, draft_ids, argmax, accept_mask, accepted_len, next_token, ctx_in, ctx_out,
+              stream=None):
+    B, gamma = draft_ids.shape
+    _check(h, _lib.rv_accept(h.ptr, _ptr(draft_ids), _ptr(argmax), B, gamma, _ptr(accept_mask),
+                             _ptr(accepted_len), _ptr(next_token), _ptr(ctx_in), _ptr(ctx_out),
+                             _stream(stream)))
+
+
+def rv_verify_step(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, ctx_in,
+                   gamma, R, alpha, attn_out, scores, argmax, margin, accept_mask, accepted_len,
+                   next_token, ctx_out, stream=None):
+    B = hidden.shape[0]
+    _check(h, _lib.rv_verify_step(
+        h.ptr, _ptr(q), _ptr(k_blk), _ptr(v_blk), _ptr(k_cache), _ptr(v_cache), _ptr(hidden),
+        _ptr(w_head), _ptr(draft_ids), _ptr(ctx_in), B, gamma, R, float(alpha), _ptr(attn_out),
+        _ptr(scores), _ptr(argmax), _ptr(margin), _ptr(accept_mask), _ptr(accepted_len),
+        _ptr(next_token), _ptr(ctx_out), _stream(stream)))
+
+
+def rv_verify_step_host(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, ctx_in,
+                        gamma, R, alpha, attn_out, scores, argmax, margin, accept_mask,
+                        accepted_len, next_token, ctx_out, stream=None):
+    """Host tensors in/out (pin them for asynchronous copies); returns (h2d, d2h) bytes."""
+    B = hidden.shape[0]
+    hb, db = ctypes.c_uint64(), ctypes.c_uint64()
+    _check(h, _lib.rv_verify_step_host(
+        h.ptr, _ptr(q), _ptr(k_blk), _ptr(v_blk), _ptr(k_cache), _ptr(v_cache), _ptr(hidden),
+        _ptr(w_head), _ptr(draft_ids), _ptr(ctx_in), B, gamma, R, float(alpha), _ptr(attn_out),
+        _ptr(scores), _ptr(argmax), _ptr(margin), _ptr(accept_mask), _ptr(accepted_len),
+        _ptr(next_token), _ptr(ctx_out), ctypes.byref(hb), ctypes.byref(db), _stream(stream)))
+    return hb.value, db.value
+
+
+def rv_read_status(h, stream=None) -> int:
+    """Synchronizes; returns the device status bits (and clears them)."""
+    st = ctypes.c_uint32()
+    rc = _lib.rv_read_status(h.ptr, _stream(stream), ctypes.byref(st))
+    if rc not in (RV_OK, RV_ERR_DEVICE):
+        _check(h, rc)
+    return st.value
+
+
+def rv_profile_enable(h, enable=True):
+    _check(h, _lib.rv_profile_enable(h.ptr, 1 if enable else 0))
+
+
+def rv_profile_read(h, region):
+    ms, n = ctypes.c_double(), ctypes.c_int32()
+    _check(h, _lib.rv_profile_read(h.ptr, region, ctypes.byref(ms), ctypes.byref(n)))
+    return ms.value, n.value
+
+
+def rv_launch_count(h) -> int:
+    v = ctypes.c_uint64()
+    _check(h, _lib.rv_launch_count(h.ptr, ctypes.byref(v)))
+    return v.value

@@ -1,0 +1,176 @@
+"""GPU parity: the CUDA path (through the C ABI) against the fp64 oracle.
+
+Small cases span several vocab tiles, KV tiles and a ragged tail; the named
+workloads run at their full sizes in the same launch configuration as the
+bench (sampled sequences where the oracle would take minutes).
+"""
+import numpy as np
+import pytest
+
+pytestmark = pytest.mark.gpu
+
+ALPHA = 0.3
+
+
+@pytest.fixture(scope="module")
+def gu():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2505_18629_gb300 import build
+    build.build()
+    import tests.gpu_util as gu
+    return gu
+
+
+def _wl(**kw):
+    from paper_2505_18629_gb300 import synth
+    base = synth.Workload("case", B=3, gamma=4, R=5, ctx=(0, 300), H=320, Hq=8, Hkv=2, D=128,
+                          V=1000, dtype="bf16", p_argmax=0.7, seed=42)
+    return base.replace(**kw)
+
+
+def _check(gu, wl, alpha=ALPHA, ctx=None, seqs=None, check_attn=True, drafts=None):
+    from paper_2505_18629_gb300 import synth
+    if ctx is not None:
+        wl = wl.replace(ctx=(min(ctx), max(ctx)))
+    inp = synth.generate(wl)
+    if ctx is not None:
+        inp.ctx_lens[:] = np.asarray(ctx, np.int32)
+    if drafts is None:
+        drafts = gu.oracle_drafts(inp, alpha, seqs=seqs)
+    gpu = gu.run_gpu(inp, drafts, alpha)
+    ref = gu.oracle_step(inp, drafts, alpha, seqs=seqs, with_attn=check_attn)
+    rep = gu.compare(inp, drafts, alpha, ref, gpu, check_attn=check_attn, seqs=seqs)
+    print(f"\n{wl.name}: {rep}")
+    return inp, drafts, gpu, ref, rep
+
+
+# ------------------------------------------------------------------ small cases
+
+def test_tiny_fp32_workload(gu):
+    from paper_2505_18629_gb300 import synth
+    _check(gu, synth.WORKLOADS["tiny"])
+
+
+def test_bf16_several_tiles_ragged(gu):
+    # V=1000: 8 vocab tiles, last one 104 rows; H=320: 5 k-blocks; ctx 0 / 77 / 300
+    _check(gu, _wl(), ctx=[0, 77, 300])
+
+
+def test_bf16_head_dim_64(gu):
+    _check(gu, _wl(D=64, Hq=4, Hkv=4, seed=43), ctx=[5, 129, 64])
+
+
+def test_bf16_gqa8_two_row_groups(gu):
+    # G=8, Lb=20 -> 160 query rows per KV head: two row groups
+    _check(gu, _wl(Hq=16, Hkv=2, gamma=6, R=8, B=2, seed=44), ctx=[1000, 3])
+
+
+def test_bf16_max_pairs_single_chunk(gu):
+    # B*(gamma+1) = 126 pairs -> N = 256 columns, the widest MMA
+    _check(gu, _wl(B=14, gamma=8, R=8, V=777, H=256, ctx=(10, 60), seed=45), check_attn=False)
+
+
+def test_bf16_multi_chunk(gu):
+    # 180 pairs -> two chunks of 90 (N = 192 each)
+    _check(gu, _wl(B=20, gamma=8, R=2, V=1500, H=128, ctx=(1, 40), seed=46), check_attn=False)
+
+
+def test_bf16_no_template_gamma1(gu):
+    _check(gu, _wl(gamma=1, R=0, B=2, seed=47), ctx=[3, 0])
+
+
+def test_alpha_zero_fused_equals_original(gu):
+    _, _, gpu, _, _ = _check(gu, _wl(seed=48), alpha=0.0, ctx=[2, 3, 4])
+    np.testing.assert_array_equal(gpu.scores[..., 2], gpu.scores[..., 0])
+    np.testing.assert_array_equal(gpu.scores[:, :-1, 3], gpu.scores[:, :-1, 4])
+
+
+def test_alpha_one_fused_equals_reflective(gu):
+    _, _, gpu, _, _ = _check(gu, _wl(seed=49), alpha=1.0, ctx=[2, 3, 4])
+    np.testing.assert_array_equal(gpu.scores[..., 2], gpu.scores[..., 1])
+
+
+def test_all_accepted_and_none_accepted(gu):
+    from paper_2505_18629_gb300 import synth
+    wl = _wl(seed=50, B=2)
+    inp = synth.generate(wl)
+    inp.ctx_lens[:] = [10, 20]
+    choice = gu.oracle_choice(inp, ALPHA).astype(np.int32)
+    drafts = choice.copy()
+    drafts[1] = (choice[1] + 1) % wl.V                      # every draft of seq 1 is wrong
+    gpu = gu.run_gpu(inp, drafts, ALPHA)
+    ref = gu.oracle_step(inp, drafts, ALPHA)
+    gu.compare(inp, drafts, ALPHA, ref, gpu)
+    assert int(ref["accepted_len"][0]) == wl.gamma and int(ref["accepted_len"][1]) == 0
+
+
+# ------------------------------------------------------------------ device-side checks
+
+def test_out_of_range_draft_sets_status(gu):
+    from paper_2505_18629_gb300 import rv, synth
+    wl = _wl(seed=51, B=2)
+    inp = synth.generate(wl)
+    inp.ctx_lens[:] = [4, 4]
+    drafts = gu.oracle_drafts(inp, ALPHA)
+    drafts[0, 1] = wl.V + 5
+    gpu = gu.run_gpu(inp, drafts, ALPHA)
+    assert gpu.status & rv.RV_DEV_DRAFT_RANGE
+    assert gpu.accept_mask[0, 1] == 0 and gpu.accepted_len[0] <= 1
+    assert np.isnan(gpu.scores[0, 1, 3]) and np.isnan(gpu.margin[0, 1])
+
+
+def test_context_overflow_sets_status_and_skips(gu):
+    from paper_2505_18629_gb300 import rv, synth
+    wl = _wl(seed=52, B=2)
+    inp = synth.generate(wl)
+    inp.ctx_lens[:] = [wl.capacity - wl.Lb + 1, 5]          # seq 0 does not fit
+    drafts = gu.oracle_drafts(inp, ALPHA)
+    gpu = gu.run_gpu(inp, drafts, ALPHA)
+    assert gpu.status & rv.RV_DEV_CTX_RANGE
+    assert (gpu.attn[0] == 0).all()                         # left untouched (zeros)
+    np.testing.assert_array_equal(gpu.k_cache[0], inp.k_cache[0])
+
+
+def test_host_validation_errors(gu):
+    import torch
+    from paper_2505_18629_gb300 import rv
+    h = gu.make_handle(_wl())
+    z = torch.zeros(8, device="cuda")
+    with pytest.raises(rv.RVError) as e:
+        rv.rv_verify_head(h, torch.zeros((4, 14, 320), dtype=torch.bfloat16, device="cuda"), z,
+                          torch.zeros((4, 4), dtype=torch.int32, device="cuda"), 4, 5, 0.3, z, z, z)
+    assert e.value.code == rv.RV_ERR_CAPACITY                # B=4 > max_batch=3
+    with pytest.raises(rv.RVError) as e:
+        rv.rv_verify_head(h, torch.zeros((1, 14, 320), dtype=torch.bfloat16, device="cuda"), z,
+                          torch.zeros((1, 4), dtype=torch.int32, device="cuda"), 4, 5,
+                          float("nan"), z, z, z)
+    assert e.value.code == rv.RV_ERR_INVALID_ARG
+    h.close()
+
+
+# ------------------------------------------------------------------ full-size workloads
+
+def test_llama3_8b_b1_full(gu):
+    from paper_2505_18629_gb300 import synth
+    _, _, gpu, ref, rep = _check(gu, synth.WORKLOADS["llama3-8b-b1"])
+    assert rep.max_lse_err < 1e-3
+
+
+def test_llama3_8b_b16_full(gu):
+    from paper_2505_18629_gb300 import synth
+    _check(gu, synth.WORKLOADS["llama3-8b-b16"])
+
+
+def test_llama3_70b_b32_sampled(gu):
+    from paper_2505_18629_gb300 import synth
+    _check(gu, synth.WORKLOADS["llama3-70b-b32"], seqs=[0, 17, 31])
+
+
+@pytest.mark.parametrize("name", ["sweep-b1-g2-c1024", "sweep-b64-g8-c8192", "sweep-b4-g4-c8192"])
+def test_sweep_points(gu, name):
+    from paper_2505_18629_gb300 import synth
+    wl = synth.workload(name)
+    seqs = None if wl.B <= 4 else [0, 33, 63]
+    _check(gu, wl, seqs=seqs)

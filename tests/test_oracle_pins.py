@@ -263,6 +263,10 @@ def test_margin_from_sorted_logits():
             zx = z[b, i, drafts[b, i]]
             want = s[-1] - s[-2] if zx == s[-1] else s[-1] - zx
             assert r["margin"][b, i] == pytest.approx(want, abs=1e-12)
+        for i in range(gamma + 1):
+            s = np.sort(z[b, i])
+            assert r["choice_gap"][b, i] == pytest.approx(s[-1] - s[-2], abs=1e-12)
+            assert z[b, i, r["argmax"][b, i]] == s[-1]
 
 
 # --------------------------------------------------------------------------

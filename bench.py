@@ -300,9 +300,8 @@ def main():
     stream = torch.cuda.current_stream(dev)
 
     def step():
-        rv.rv_pack_block(h, drafts, prompt, prefix, ctx, block, pos, stream)
-        rv.rv_verify_step(h, q, kb, vb, kc, vc, hidden, W, drafts, ctx, g, R, ALPHA, attn, scores,
-                          argmax, margin, acc, alen, nxt, ctx_out, stream)
+        rv.rv_verify_step(h, q, kb, vb, kc, vc, hidden, W, drafts, prompt, prefix, ctx, ALPHA,
+                          block, pos, attn, scores, argmax, margin, acc, alen, nxt, ctx_out, stream)
 
     for _ in range(args.warmup):
         step()
@@ -349,6 +348,10 @@ def main():
     hq, hkb, hvb, hhid = pin(inp.q), pin(inp.k_blk), pin(inp.v_blk), pin(inp.hidden)
     hdr = pin(drafts_np.astype(np.int32))
     hctx = pin(inp.ctx_lens.astype(np.int32))
+    hprompt = pin(inp.prompt_ids.astype(np.int32)) if inp.prompt_ids.size else None
+    hprefix = pin(inp.prefix_ids.astype(np.int32))
+    o_blk = torch.empty((B, Lb), dtype=torch.int32).pin_memory()
+    o_pos = torch.empty_like(o_blk).pin_memory()
     o_sc = torch.empty((B, g + 1, rv.RV_NSCORES)).pin_memory()
     o_am = torch.empty((B, g + 1), dtype=torch.int32).pin_memory()
     o_mg = torch.empty((B, g)).pin_memory()
@@ -358,8 +361,9 @@ def main():
     o_co = torch.empty_like(o_al).pin_memory()
 
     def step_host():
-        return rv.rv_verify_step_host(h, hq, hkb, hvb, kc, vc, hhid, W, hdr, hctx, g, R, ALPHA,
-                                      None, o_sc, o_am, o_mg, o_acc, o_al, o_nt, o_co, stream)
+        return rv.rv_verify_step_host(h, hq, hkb, hvb, kc, vc, hhid, W, hdr, hprompt, hprefix,
+                                      hctx, ALPHA, o_blk, o_pos, None, o_sc, o_am, o_mg, o_acc,
+                                      o_al, o_nt, o_co, stream)
     for _ in range(3):
         step_host()
     if world > 1:

@@ -92,8 +92,8 @@ typedef struct rv_config {
 typedef struct rv_handle rv_handle;
 
 /* Create a handle on the current CUDA device.  Validates the config, checks
- * that the device is sm_103, and allocates the scratch workspace (attention
- * split partials, head partial statistics, gathered hidden rows, status word,
+ * that the device is sm_103, and allocates the scratch workspace (per-CTA
+ * partial statistics of the LM head, gathered hidden rows, status word,
  * staging for rv_verify_step_host).  The library owns that memory until
  * rv_destroy.  *out is set only on success. */
 RV_API int rv_create(const rv_config* cfg, rv_handle** out);
@@ -169,30 +169,39 @@ RV_API int rv_accept(rv_handle* h, const int32_t* draft_ids, const int32_t* argm
                      int32_t gamma, uint8_t* accept_mask, int32_t* accepted_len,
                      int32_t* next_token, const int32_t* ctx_in, int32_t* ctx_out, void* stream);
 
-/* The whole verify step on device buffers: rv_verify_attention, rv_verify_head
- * and rv_accept in order on one stream (the block ids, if wanted, come from
- * rv_pack_block).  Arguments as in those calls; R is the template length. */
+/* The whole verify step on device buffers, in one call and four kernel
+ * launches on `stream`: attention (rv_verify_attention), then one launch that
+ * gathers the LM-head rows and packs the block (rv_pack_block; skipped when
+ * block_ids is NULL), the LM head, and one launch that merges the head's
+ * statistics and runs the acceptance (rv_accept).  Arguments as in those
+ * calls; the template is n_prompt prompt ids + n_prefix prefix ids, so
+ * R = n_prompt + n_prefix and Lb = 2*gamma + R.  ctx_out may alias ctx_in. */
 RV_API int rv_verify_step(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
                           void* k_cache, void* v_cache, const void* hidden, const void* w_head,
-                          const int32_t* draft_ids, const int32_t* ctx_in, int32_t B,
-                          int32_t gamma, int32_t R, float alpha, void* attn_out, float* scores,
+                          const int32_t* draft_ids, const int32_t* prompt_ids,
+                          const int32_t* prefix_ids, const int32_t* ctx_in, int32_t B,
+                          int32_t gamma, int32_t n_prompt, int32_t n_prefix, float alpha,
+                          int32_t* block_ids, int32_t* pos_ids, void* attn_out, float* scores,
                           int32_t* argmax, float* margin, uint8_t* accept_mask,
                           int32_t* accepted_len, int32_t* next_token, int32_t* ctx_out,
                           void* stream);
 
 /* The whole verify step from HOST buffers (synchronous).  The per-step inputs
- * (q, k_blk, v_blk, hidden, draft ids, ctx lens) are copied from host memory
- * (pinned memory gives asynchronous copies) into the handle's device staging,
- * the step runs, and the per-step results are copied back into host memory
- * before the call returns.  The model state stays on the device: w_head,
- * k_cache and v_cache are device pointers.  Host buffers have the layouts of
- * rv_verify_step; attn_out_host may be NULL to skip reading the attention
- * output back.  *h2d_bytes / *d2h_bytes (optional) receive the bytes copied. */
+ * (q, k_blk, v_blk, hidden, draft / prompt / prefix ids, ctx lens) are copied
+ * from host memory (pinned memory gives asynchronous copies) into the handle's
+ * device staging, rv_verify_step runs, and the per-step results are copied
+ * back into host memory before the call returns.  The model state stays on
+ * the device: w_head, k_cache and v_cache are device pointers.  Host buffers
+ * have the layouts of rv_verify_step; attn_out_host may be NULL to skip
+ * reading the attention output back, block_ids_host NULL to skip the packing.
+ * *h2d_bytes / *d2h_bytes (optional) receive the bytes copied each way. */
 RV_API int rv_verify_step_host(rv_handle* h, const void* q_host, const void* k_blk_host,
                                const void* v_blk_host, void* k_cache, void* v_cache,
                                const void* hidden_host, const void* w_head,
-                               const int32_t* draft_ids_host, const int32_t* ctx_in_host,
-                               int32_t B, int32_t gamma, int32_t R, float alpha,
+                               const int32_t* draft_ids_host, const int32_t* prompt_ids_host,
+                               const int32_t* prefix_ids_host, const int32_t* ctx_in_host,
+                               int32_t B, int32_t gamma, int32_t n_prompt, int32_t n_prefix,
+                               float alpha, int32_t* block_ids_host, int32_t* pos_ids_host,
                                void* attn_out_host, float* scores_host, int32_t* argmax_host,
                                float* margin_host, uint8_t* accept_mask_host,
                                int32_t* accepted_len_host, int32_t* next_token_host,
@@ -207,7 +216,7 @@ RV_API int rv_read_status(rv_handle* h, void* stream, uint32_t* status);
 #define RV_PROF_ATTENTION 0   /* attention kernels of rv_verify_attention */
 #define RV_PROF_HEAD_GEMM 1   /* the LM-head GEMM + online log-softmax kernel */
 #define RV_PROF_HEAD 2        /* everything rv_verify_head launches */
-#define RV_PROF_ACCEPT 3      /* rv_accept */
+#define RV_PROF_ACCEPT 3      /* rv_accept (inside rv_verify_step it is part of RV_PROF_HEAD) */
 #define RV_PROF_COUNT 4
 
 /* enable != 0: from now on, record a CUDA event pair on the launching stream

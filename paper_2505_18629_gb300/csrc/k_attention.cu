@@ -8,8 +8,12 @@
 // of 64 with 16-byte cp.async loads (double buffered, XOR-swizzled rows) and
 // runs QK^T and PV on the tensor cores (mma.sync m16n8k16 bf16, fp32
 // accumulate).  All G*Lb query rows that share a KV head live in one CTA
-// (16 rows per warp), so each key/value byte is read once per head.  Partial
-// (O/l, m, l) per split are merged by attention_combine.  The block's own
+// (16 rows per warp), so each key/value byte is read once per head.  The
+// splits of one (sequence, KV head, row group) form a thread-block cluster:
+// each CTA leaves its partial (O/l, m, l) in its own shared memory and, after
+// a cluster barrier, every CTA merges a slice of the rows by reading all the
+// partials through distributed shared memory.  No partials touch global
+// memory and no second kernel is launched.  The block's own
 // keys/values are read from k_blk/v_blk and appended to the cache at
 // [ctx_b, ctx_b + Lb) by one CTA per (sequence, KV head); no CTA reads those
 // cache positions, so the append does not race.
@@ -17,13 +21,18 @@
 // fp32 path: one warp per query row on the CUDA cores (tiny fp32 models).
 #include <cfloat>
 
+#include <cooperative_groups.h>
+
 #include "rv_device.cuh"
 #include "rv_kernels.h"
 
 namespace rv {
 
+namespace cg = cooperative_groups;
+
 constexpr int AT_KT = 64;         // keys per shared-memory tile
 constexpr int AT_MAX_WARPS = 8;   // 16 query rows per warp -> 128 rows per CTA
+constexpr int AT_MAX_SPLITS = 16; // cluster size limit (non-portable above 8)
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool pred) {
   const int n = pred ? 16 : 0;  // zero-fill when the source is out of range
@@ -81,23 +90,24 @@ struct AttnKernelArgs {
   __nv_bfloat16* v_cache;
   const int32_t* ctx;
   __nv_bfloat16* out;
-  float* part_o;
-  float* part_ml;
   int B, Lb, Hq, Hkv, Cmax, G, rows, splits;
   float scale_log2;  // log2(e) / sqrt(D)
   unsigned* status;
 };
 
+// 168 registers let two CTAs of up to 6 warps share an SM.
 template <int D>
-__global__ void __launch_bounds__(AT_MAX_WARPS * 32)
-    attention_bf16_kernel(const AttnKernelArgs a) {
+__global__ void __maxnreg__(168) attention_bf16_kernel(const AttnKernelArgs a) {
   constexpr int CH = D / 8;            // 16-byte chunks per row
   constexpr int TILE_BYTES = AT_KT * D * 2;
+  constexpr int Q_BYTES = AT_MAX_WARPS * 16 * D * 2;
   extern __shared__ __align__(128) uint8_t smem[];
-  // [Q: 128 rows][K buf 0][V buf 0][K buf 1][V buf 1]
+  // [Q: 128 rows][K buf 0][V buf 0][K buf 1][V buf 1][merge weights]
+  // After the key loop the Q region holds (m, l) per row and the K/V region
+  // the fp32 partial O/l of every row (read by the other CTAs of the cluster).
   const uint32_t s_base = smem_u32(smem);
   const uint32_t s_q = s_base;
-  const uint32_t s_kv = s_base + AT_MAX_WARPS * 16 * D * 2;
+  const uint32_t s_kv = s_base + Q_BYTES;
 
   const int split = blockIdx.x, kvh = blockIdx.y;
   const int n_rg = (a.rows + AT_MAX_WARPS * 16 - 1) / (AT_MAX_WARPS * 16);
@@ -112,29 +122,19 @@ __global__ void __launch_bounds__(AT_MAX_WARPS * 32)
     return;
   }
   const int T = ctx + a.Lb;
-  // Append the block's keys/values (positions ctx..ctx+Lb-1) once per (b, kvh).
-  if (split == 0 && rg == 0) {
-    for (int e = tid; e < a.Lb * CH; e += nthr) {
-      const int j = e / CH, c = e % CH;
-      const long long src = ((static_cast<long long>(b) * a.Lb + j) * a.Hkv + kvh) * D + c * 8;
-      const long long dst = ((static_cast<long long>(b) * a.Hkv + kvh) * a.Cmax + ctx + j) * D + c * 8;
-      *reinterpret_cast<uint4*>(a.k_cache + dst) = *reinterpret_cast<const uint4*>(a.k_blk + src);
-      *reinterpret_cast<uint4*>(a.v_cache + dst) = *reinterpret_cast<const uint4*>(a.v_blk + src);
-    }
-  }
-  // Key range of this split (multiples of the tile).
-  const int per = (((T + a.splits - 1) / a.splits) + AT_KT - 1) / AT_KT * AT_KT;
-  const int k_lo = split * per;
+  // Key range of this split: near-equal shares in multiples of 16 keys.
+  const int per = ((T + a.splits - 1) / a.splits + 15) / 16 * 16;
+  const int k_lo = min(T, split * per);
   const int k_hi = min(T, k_lo + per);
 
   const int row0 = rg * AT_MAX_WARPS * 16;  // first query row of this CTA (within the KV head)
-  // Rows of this thread: r0 = row0 + warp*16 + g, r1 = r0 + 8.  Row r <-> (j = r / G, h = kvh*G + r % G).
+  // Rows of this thread: r_a = row0 + warp*16 + g, r_b = r_a + 8.  Row r <-> (j = r / G, h = kvh*G + r % G).
   const int r_a = row0 + warp * 16 + g, r_b = r_a + 8;
   const bool va = r_a < a.rows, vb = r_b < a.rows;
   const int lim_a = va ? ctx + r_a / a.G : -1;  // last visible key
   const int lim_b = vb ? ctx + r_b / a.G : -1;
 
-  // ---- load Q rows into shared memory, then into A fragments
+  // ---- Q rows -> shared memory (group 0)
   for (int e = tid; e < AT_MAX_WARPS * 16 * CH; e += nthr) {
     const int r = e / CH, c = e % CH;
     const int rr = row0 + r;
@@ -165,20 +165,24 @@ __global__ void __launch_bounds__(AT_MAX_WARPS * 32)
       cp_async16(sk + swz<D>(r, c), ks, ok);
       cp_async16(sv + swz<D>(r, c), vs, ok);
     }
-    cp_async_commit();
   };
 
-  const int n_tiles = k_hi > k_lo ? (k_hi - k_lo + AT_KT - 1) / AT_KT : 0;
+  // Two tiles in flight from the start (groups 1 and 2; empty groups are fine).
+  const int n_tiles = (k_hi - k_lo + AT_KT - 1) / AT_KT;
   if (n_tiles > 0) load_kv(k_lo, 0);
-  cp_async_wait_all();  // Q (and the first tile) have landed
-  __syncthreads();
+  cp_async_commit();
+  if (n_tiles > 1) load_kv(k_lo + AT_KT, 1);
+  cp_async_commit();
 
-  uint32_t qf[D / 16][4];
-#pragma unroll
-  for (int ks = 0; ks < D / 16; ++ks) {
-    const int mi = lane >> 3;
-    const int r = warp * 16 + (mi & 1) * 8 + (lane & 7);
-    ldsm_x4(s_q + swz<D>(r, 2 * ks + (mi >> 1)), qf[ks][0], qf[ks][1], qf[ks][2], qf[ks][3]);
+  // Append the block's keys/values (positions ctx..ctx+Lb-1) once per (b, kvh).
+  if (split == 0 && rg == 0) {
+    for (int e = tid; e < a.Lb * CH; e += nthr) {
+      const int j = e / CH, c = e % CH;
+      const long long src = ((static_cast<long long>(b) * a.Lb + j) * a.Hkv + kvh) * D + c * 8;
+      const long long dst = ((static_cast<long long>(b) * a.Hkv + kvh) * a.Cmax + ctx + j) * D + c * 8;
+      *reinterpret_cast<uint4*>(a.k_cache + dst) = *reinterpret_cast<const uint4*>(a.k_blk + src);
+      *reinterpret_cast<uint4*>(a.v_cache + dst) = *reinterpret_cast<const uint4*>(a.v_blk + src);
+    }
   }
 
   float o[D / 8][4];
@@ -188,30 +192,28 @@ __global__ void __launch_bounds__(AT_MAX_WARPS * 32)
 
   for (int it = 0; it < n_tiles; ++it) {
     const int buf = it & 1;
-    if (it + 1 < n_tiles) {
-      load_kv(k_lo + (it + 1) * AT_KT, buf ^ 1);
-      cp_async_wait_1();
-    } else {
-      cp_async_wait_all();
-    }
+    cp_async_wait_1();  // all but the newest group: Q and tile `it` have landed
     __syncthreads();
     const uint32_t sk = s_kv + buf * 2 * TILE_BYTES, sv = sk + TILE_BYTES;
     const int kbase = k_lo + it * AT_KT;
 
-    // S = Q K^T for 16 rows x 64 keys
+    // S = Q K^T for 16 rows x 64 keys (Q fragments re-read from shared memory)
     float s[AT_KT / 8][4];
 #pragma unroll
     for (int nt = 0; nt < AT_KT / 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
 #pragma unroll
     for (int ks = 0; ks < D / 16; ++ks) {
+      const int mi = lane >> 3;
+      uint32_t qf[4];
+      ldsm_x4(s_q + swz<D>(warp * 16 + (mi & 1) * 8 + (lane & 7), 2 * ks + (mi >> 1)), qf[0], qf[1],
+              qf[2], qf[3]);
 #pragma unroll
       for (int nt = 0; nt < AT_KT / 8; nt += 2) {
-        const int mi = lane >> 3;
         const int key = 8 * (nt + (mi >> 1)) + (lane & 7);
         uint32_t b0, b1, b2, b3;
         ldsm_x4(sk + swz<D>(key, 2 * ks + (mi & 1)), b0, b1, b2, b3);
-        mma_bf16_16816(s[nt], qf[ks], b0, b1);
-        mma_bf16_16816(s[nt + 1], qf[ks], b2, b3);
+        mma_bf16_16816(s[nt], qf, b0, b1);
+        mma_bf16_16816(s[nt + 1], qf, b2, b3);
       }
     }
     // mask + online softmax (rows r_a: s[.][0..1], r_b: s[.][2..3])
@@ -273,8 +275,11 @@ __global__ void __launch_bounds__(AT_MAX_WARPS * 32)
         mma_bf16_16816(o[dt + 1], pa, b2, b3);
       }
     }
-    __syncthreads();  // buffer `buf` is refilled two iterations later
+    __syncthreads();  // every warp is done with buffer `buf`
+    if (it + 2 < n_tiles) load_kv(k_lo + (it + 2) * AT_KT, buf);
+    cp_async_commit();
   }
+  cp_async_wait_all();
 
   l_a += __shfl_xor_sync(0xffffffffu, l_a, 1);
   l_a += __shfl_xor_sync(0xffffffffu, l_a, 2);
@@ -297,65 +302,72 @@ __global__ void __launch_bounds__(AT_MAX_WARPS * 32)
         *reinterpret_cast<uint32_t*>(a.out + row_index(r_b) * D + d) =
             pack_bf16(o[dt][2] * ib, o[dt][3] * ib);
     }
-  } else {
-    const long long nrows = static_cast<long long>(a.B) * a.Lb * a.Hq;
-#pragma unroll
-    for (int dt = 0; dt < D / 8; ++dt) {
-      const int d = dt * 8 + 2 * t4;
-      if (va)
-        *reinterpret_cast<float2*>(a.part_o + (split * nrows + row_index(r_a)) * D + d) =
-            make_float2(o[dt][0] * ia, o[dt][1] * ia);
-      if (vb)
-        *reinterpret_cast<float2*>(a.part_o + (split * nrows + row_index(r_b)) * D + d) =
-            make_float2(o[dt][2] * ib, o[dt][3] * ib);
-    }
-    if (t4 == 0) {
-      if (va)
-        *reinterpret_cast<float2*>(a.part_ml + (split * nrows + row_index(r_a)) * 2) =
-            make_float2(m_a * a.scale_log2, l_a);
-      if (vb)
-        *reinterpret_cast<float2*>(a.part_ml + (split * nrows + row_index(r_b)) * 2) =
-            make_float2(m_b * a.scale_log2, l_b);
-    }
+    return;
   }
-}
 
-// Merge split partials: O = sum_s w_s O_s / sum_s w_s, w_s = l_s 2^(m_s - M).
-// One warp per output row (b, j, h).
-template <typename OutT>
-__global__ void attention_combine_kernel(const float* __restrict__ part_o,
-                                         const float* __restrict__ part_ml,
-                                         const int32_t* __restrict__ ctx, OutT* __restrict__ out,
-                                         int B, int Lb, int Hq, int D, int Cmax, int splits) {
-  const long long nrows = static_cast<long long>(B) * Lb * Hq;
-  const long long row = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (row >= nrows) return;
-  const int b = static_cast<int>(row / (static_cast<long long>(Lb) * Hq));
-  const int c = ctx[b];
-  if (c < 0 || c + Lb > Cmax) return;
-  float M = NEG_INF;
-  for (int s = 0; s < splits; ++s) {
-    const float l = part_ml[(s * nrows + row) * 2 + 1];
-    if (l > 0.f) M = fmaxf(M, part_ml[(s * nrows + row) * 2]);
+  // ---- split-KV merge through distributed shared memory
+  __syncthreads();  // all warps done with Q and the K/V buffers
+  float* const part = reinterpret_cast<float*>(smem + Q_BYTES);    // [128][D]
+  float* const ml = reinterpret_cast<float*>(smem);                // [128][2]
+  float* const wsm = reinterpret_cast<float*>(smem + Q_BYTES + 4 * TILE_BYTES);  // [128][16]
+  const int la = warp * 16 + g, lbr = la + 8;  // rows within the CTA window
+#pragma unroll
+  for (int dt = 0; dt < D / 8; ++dt) {
+    const int d = dt * 8 + 2 * t4;
+    *reinterpret_cast<float2*>(part + la * D + d) = make_float2(o[dt][0] * ia, o[dt][1] * ia);
+    *reinterpret_cast<float2*>(part + lbr * D + d) = make_float2(o[dt][2] * ib, o[dt][3] * ib);
   }
-  for (int d = lane; d < D; d += 32) {
-    float num = 0.f, den = 0.f;
-    for (int s = 0; s < splits; ++s) {
-      const float m = part_ml[(s * nrows + row) * 2];
-      const float l = part_ml[(s * nrows + row) * 2 + 1];
-      if (l > 0.f) {
-        const float w = l * exp2f(m - M);
-        num += w * part_o[(s * nrows + row) * D + d];
-        den += w;
-      }
+  if (t4 == 0) {
+    ml[2 * la] = m_a * a.scale_log2;
+    ml[2 * la + 1] = l_a;
+    ml[2 * lbr] = m_b * a.scale_log2;
+    ml[2 * lbr + 1] = l_b;
+  }
+  cg::cluster_group cluster = cg::this_cluster();
+  cluster.sync();
+  const int S = a.splits;
+  const int rank = static_cast<int>(cluster.block_rank());
+  const int nrow = min(AT_MAX_WARPS * 16, a.rows - row0);
+  const int per_rank = (nrow + S - 1) / S;
+  const int r_lo = min(nrow, rank * per_rank), r_hi = min(nrow, r_lo + per_rank);
+  // weights w_s = l_s 2^(m_s - M) / sum_s(...): one thread per (row, split)
+  for (int it = tid; it < (r_hi - r_lo) * S; it += nthr) {
+    const int rl = r_lo + it / S, sp = it % S;
+    float M = NEG_INF;
+    for (int q = 0; q < S; ++q) {
+      const float* rml = cluster.map_shared_rank(ml, q);
+      if (rml[2 * rl + 1] > 0.f) M = fmaxf(M, rml[2 * rl]);
     }
-    const float v = den > 0.f ? num / den : 0.f;
-    if constexpr (sizeof(OutT) == 2)
-      out[row * D + d] = __float2bfloat16_rn(v);
-    else
-      out[row * D + d] = v;
+    float den = 0.f, mine = 0.f;
+    for (int q = 0; q < S; ++q) {
+      const float* rml = cluster.map_shared_rank(ml, q);
+      const float l = rml[2 * rl + 1];
+      const float w = l > 0.f ? l * exp2f(rml[2 * rl] - M) : 0.f;
+      den += w;
+      if (q == sp) mine = w;
+    }
+    wsm[rl * AT_MAX_SPLITS + sp] = den > 0.f ? mine / den : 0.f;
   }
+  __syncthreads();
+  constexpr int D4 = D / 4;
+  for (int it = tid; it < (r_hi - r_lo) * D4; it += nthr) {
+    const int rl = r_lo + it / D4, d = (it % D4) * 4;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+    for (int sp = 0; sp < S; ++sp) {
+      const float w = wsm[rl * AT_MAX_SPLITS + sp];
+      const float4 v = *reinterpret_cast<const float4*>(cluster.map_shared_rank(part, sp) + rl * D + d);
+      acc.x = fmaf(w, v.x, acc.x);
+      acc.y = fmaf(w, v.y, acc.y);
+      acc.z = fmaf(w, v.z, acc.z);
+      acc.w = fmaf(w, v.w, acc.w);
+    }
+    uint2 pk;
+    pk.x = pack_bf16(acc.x, acc.y);
+    pk.y = pack_bf16(acc.z, acc.w);
+    *reinterpret_cast<uint2*>(a.out + row_index(row0 + rl) * D + d) = pk;
+  }
+  cluster.sync();  // partials stay alive until every CTA of the cluster has read them
 }
 
 // ---------------------------------------------------------------- fp32 path
@@ -430,7 +442,8 @@ __global__ void attention_f32_kernel(const float* __restrict__ q, const float* _
 
 // ---------------------------------------------------------------- planning / launch
 
-AttnPlan attn_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms, bool bf16) {
+AttnPlan attn_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms, bool bf16,
+                   int max_cluster) {
   AttnPlan p;
   const int G = Hq / Hkv;
   p.rows = Lb * G;
@@ -444,34 +457,59 @@ AttnPlan attn_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms, bool b
   p.warps = std::min(AT_MAX_WARPS, (p.rows + 15) / 16);
   if (p.row_groups > 1) p.warps = AT_MAX_WARPS;
   const int base = B * Hkv * p.row_groups;
-  int s = (num_sms + base - 1) / base;              // about one wave of CTAs
+  int s = (2 * num_sms + base - 1) / base;          // about two CTAs per SM
   const int max_useful = (Cmax + 2 * AT_KT - 1) / (2 * AT_KT);  // >= 128 keys per split
-  s = std::max(1, std::min(s, std::min(max_useful, 32)));
+  s = std::max(1, std::min(s, std::min(max_useful, std::min(max_cluster, AT_MAX_SPLITS))));
   p.splits = s;
   return p;
 }
 
-size_t attn_partial_floats(const AttnPlan& p, int B, int Lb, int Hq, int D) {
-  if (p.splits <= 1) return 0;
-  return static_cast<size_t>(p.splits) * B * Lb * Hq * (D + 2);
+size_t attn_bf16_smem_bytes(int D) {
+  return static_cast<size_t>(AT_MAX_WARPS) * 16 * D * 2 + 4 * static_cast<size_t>(AT_KT) * D * 2 +
+         static_cast<size_t>(AT_MAX_WARPS) * 16 * AT_MAX_SPLITS * 4;
 }
 
-size_t attn_bf16_smem_bytes(int D, int /*warps*/) {
-  return static_cast<size_t>(AT_MAX_WARPS) * 16 * D * 2 + 4 * static_cast<size_t>(AT_KT) * D * 2;
-}
-
-cudaError_t attn_configure() {
-  cudaError_t e = cudaFuncSetAttribute(attention_bf16_kernel<128>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(attn_bf16_smem_bytes(128, 8)));
+template <int D>
+static cudaError_t attn_configure_d() {
+  auto k = attention_bf16_kernel<D>;
+  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(attn_bf16_smem_bytes(D)));
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(attention_bf16_kernel<64>,
-                              cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(attn_bf16_smem_bytes(64, 8)));
+  return cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
 }
 
-cudaError_t launch_attention_bf16(const AttnArgs& x, const AttnPlan& p, float* part_o,
-                                  float* part_ml, cudaStream_t s) {
+// Largest cluster size (<= 16) for which clusters of the D=128 kernel can be resident.
+static int max_cluster_for(int D) {
+  for (int cs = AT_MAX_SPLITS; cs > 1; cs >>= 1) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(cs, 1, 1);
+    cfg.blockDim = dim3(AT_MAX_WARPS * 32, 1, 1);
+    cfg.dynamicSmemBytes = attn_bf16_smem_bytes(D);
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = cs;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    cudaError_t e = D == 128 ? cudaOccupancyMaxActiveClusters(&n, attention_bf16_kernel<128>, &cfg)
+                             : cudaOccupancyMaxActiveClusters(&n, attention_bf16_kernel<64>, &cfg);
+    if (e == cudaSuccess && n > 0) return cs;
+    cudaGetLastError();
+  }
+  return 1;
+}
+
+cudaError_t attn_configure(int* max_cluster) {
+  cudaError_t e = attn_configure_d<128>();
+  if (e == cudaSuccess) e = attn_configure_d<64>();
+  if (e != cudaSuccess) return e;
+  *max_cluster = std::min(max_cluster_for(128), max_cluster_for(64));
+  return cudaSuccess;
+}
+
+cudaError_t launch_attention_bf16(const AttnArgs& x, const AttnPlan& p, cudaStream_t s) {
   AttnKernelArgs a;
   a.q = static_cast<const __nv_bfloat16*>(x.q);
   a.k_blk = static_cast<const __nv_bfloat16*>(x.k_blk);
@@ -480,8 +518,6 @@ cudaError_t launch_attention_bf16(const AttnArgs& x, const AttnPlan& p, float* p
   a.v_cache = static_cast<__nv_bfloat16*>(x.v_cache);
   a.ctx = x.ctx;
   a.out = static_cast<__nv_bfloat16*>(x.out);
-  a.part_o = part_o;
-  a.part_ml = part_ml;
   a.B = x.B;
   a.Lb = x.Lb;
   a.Hq = x.Hq;
@@ -492,35 +528,24 @@ cudaError_t launch_attention_bf16(const AttnArgs& x, const AttnPlan& p, float* p
   a.splits = p.splits;
   a.scale_log2 = LOG2E / sqrtf(static_cast<float>(x.D));
   a.status = x.status;
-  dim3 grid(p.splits, x.Hkv, x.B * p.row_groups);
-  const size_t smem = attn_bf16_smem_bytes(x.D, p.warps);
-  if (x.D == 128)
-    attention_bf16_kernel<128><<<grid, p.warps * 32, smem, s>>>(a);
-  else if (x.D == 64)
-    attention_bf16_kernel<64><<<grid, p.warps * 32, smem, s>>>(a);
-  else
-    return cudaErrorInvalidValue;
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.splits, x.Hkv, x.B * p.row_groups);
+  cfg.blockDim = dim3(p.warps * 32, 1, 1);
+  cfg.dynamicSmemBytes = attn_bf16_smem_bytes(x.D);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = p.splits;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = p.splits > 1 ? 1 : 0;
+  if (x.D == 128) return cudaLaunchKernelEx(&cfg, attention_bf16_kernel<128>, a);
+  if (x.D == 64) return cudaLaunchKernelEx(&cfg, attention_bf16_kernel<64>, a);
+  return cudaErrorInvalidValue;
 }
 
-cudaError_t launch_attention_combine(const AttnArgs& x, const AttnPlan& p, const float* part_o,
-                                     const float* part_ml, bool bf16, cudaStream_t s) {
-  const long long nrows = static_cast<long long>(x.B) * x.Lb * x.Hq;
-  const int threads = 128;
-  const int blocks = static_cast<int>((nrows * 32 + threads - 1) / threads);
-  if (bf16)
-    attention_combine_kernel<__nv_bfloat16><<<blocks, threads, 0, s>>>(
-        part_o, part_ml, x.ctx, static_cast<__nv_bfloat16*>(x.out), x.B, x.Lb, x.Hq, x.D, x.Cmax,
-        p.splits);
-  else
-    attention_combine_kernel<float><<<blocks, threads, 0, s>>>(
-        part_o, part_ml, x.ctx, static_cast<float*>(x.out), x.B, x.Lb, x.Hq, x.D, x.Cmax,
-        p.splits);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_attention_f32(const AttnArgs& x, const AttnPlan& /*p*/, float* /*part_o*/,
-                                 float* /*part_ml*/, cudaStream_t s) {
+cudaError_t launch_attention_f32(const AttnArgs& x, cudaStream_t s) {
   const long long nrows = static_cast<long long>(x.B) * x.Lb * x.Hq;
   const int threads = 128;
   const int blocks = static_cast<int>((nrows * 32 + threads - 1) / threads);

@@ -8,6 +8,11 @@
 // logit is ever written to memory.  Swap-AB orientation: the vocab is the MMA
 // M dimension (128 TMEM lanes), the few hidden rows are N (16..256 columns).
 //
+// The vocab is split across the CTAs of a chunk in units of 16 rows, so every
+// CTA streams the same number of weight bytes to within one unit.  Full tiles
+// arrive as one 128-row TMA box; a CTA's last, partial tile as 16-row boxes
+// (its missing rows are never loaded and their accumulator lanes are masked).
+//
 // Persistent CTA per SM, warp-specialised:
 //   warp 0      TMA producer: W tile [128 x 64] + hsel tile [N x 64] per stage
 //               into a ring of `stages` 128B-swizzled shared-memory buffers
@@ -25,14 +30,16 @@
 
 namespace rv {
 
-constexpr int HT_BM = 128;
+constexpr int HT_BM = HEAD_TILE_ROWS;
 constexpr int HT_BK = 64;
 constexpr int HT_THREADS = 192;
 constexpr int HT_EPI_WARPS = 4;
+constexpr int HT_WBOX = HEAD_W_BOX_ROWS;             // vocab rows per TMA box of W
 constexpr uint32_t HT_A_BYTES = HT_BM * HT_BK * 2;  // 16 KB
+constexpr uint32_t HT_BOX_BYTES = HT_WBOX * HT_BK * 2;  // 2 KB
 
 struct HeadTcParams {
-  int V, n_kb, N, Pcp, Pc, P, n_vtiles, slots, stages, gamma;
+  int V, n_kb, N, Pcp, Pc, P, units, slots, stages, gamma;  // units = ceil(V / 16)
   uint32_t tmem_cols;
   float alpha;
   const int32_t* drafts;
@@ -68,6 +75,7 @@ __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
 
 __global__ void __launch_bounds__(HT_THREADS, 1)
     head_tc_kernel(const __grid_constant__ CUtensorMap tm_w,
+                   const __grid_constant__ CUtensorMap tm_w16,
                    const __grid_constant__ CUtensorMap tm_h, const HeadTcParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
@@ -96,8 +104,12 @@ __global__ void __launch_bounds__(HT_THREADS, 1)
 
   const int pair0 = chunk * p.Pc;
   const int npairs = min(p.Pc, p.P - pair0);
-  const int t0 = static_cast<int>(static_cast<long long>(slot_id) * p.n_vtiles / p.slots);
-  const int t1 = static_cast<int>(static_cast<long long>(slot_id + 1) * p.n_vtiles / p.slots);
+  // vocab rows [v_lo, v_hi) of this CTA, in tiles of 128 rows
+  const int v_lo = HT_WBOX * static_cast<int>(static_cast<long long>(slot_id) * p.units / p.slots);
+  const int v_hi = min(p.V, HT_WBOX * static_cast<int>(static_cast<long long>(slot_id + 1) *
+                                                        p.units / p.slots));
+  const int t0 = 0;
+  const int t1 = v_hi > v_lo ? (v_hi - v_lo + HT_BM - 1) / HT_BM : 0;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -114,6 +126,7 @@ __global__ void __launch_bounds__(HT_THREADS, 1)
   }
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tm_w);
+    tma_prefetch_desc(&tm_w16);
     tma_prefetch_desc(&tm_h);
   }
   if (warp == 1) tmem_alloc(smem_u32(tmem_slot), p.tmem_cols);
@@ -137,13 +150,21 @@ __global__ void __launch_bounds__(HT_THREADS, 1)
       uint32_t ph = 0;
       bool ok = true;
       for (int t = t0; t < t1 && ok; ++t) {
+        const int v0 = v_lo + t * HT_BM;
+        const int rows = min(HT_BM, v_hi - v0);
+        const int nbox = rows == HT_BM ? 0 : (rows + HT_WBOX - 1) / HT_WBOX;  // 0: one full box
+        const uint32_t a_bytes = nbox == 0 ? HT_A_BYTES : nbox * HT_BOX_BYTES;
         for (int kb = 0; kb < p.n_kb; ++kb) {
           if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag, p.status)) {
             ok = false;
             break;
           }
-          mbar_arrive_expect_tx(full_bar(s), HT_A_BYTES + b_bytes);
-          tma_load_2d(a_tiles + s * HT_A_BYTES, &tm_w, kb * HT_BK, t * HT_BM, full_bar(s), pol_w);
+          mbar_arrive_expect_tx(full_bar(s), a_bytes + b_bytes);
+          if (nbox == 0)
+            tma_load_2d(a_tiles + s * HT_A_BYTES, &tm_w, kb * HT_BK, v0, full_bar(s), pol_w);
+          for (int j = 0; j < nbox; ++j)
+            tma_load_2d(a_tiles + s * HT_A_BYTES + j * HT_BOX_BYTES, &tm_w16, kb * HT_BK,
+                        v0 + j * HT_WBOX, full_bar(s), pol_w);
           tma_load_2d(b_tiles + s * b_bytes, &tm_h, kb * HT_BK, chunk * p.N, full_bar(s), pol_h);
           ++issued;
           if (++s == S) {
@@ -210,8 +231,8 @@ __global__ void __launch_bounds__(HT_THREADS, 1)
       bool ok = mbar_wait(accf0 + 8u * slot, aph, abort_flag, p.status);
       if (!__all_sync(0xffffffffu, ok)) break;
       tc_fence_after();
-      const int v = t * HT_BM + q * 32 + lane;
-      const bool valid = v < p.V;
+      const int v = v_lo + t * HT_BM + q * 32 + lane;
+      const bool valid = v < v_hi;
       const uint32_t trow =
           tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(slot * p.N);
       for (int g8 = 0; g8 < npairs; g8 += 8) {
@@ -259,7 +280,7 @@ cudaError_t launch_head_tc(const HeadArgs& a, const HeadPlan& pl, const HeadTcLa
   p.Pcp = pl.pad_pairs;
   p.Pc = pl.pairs_per_chunk;
   p.P = pl.P;
-  p.n_vtiles = pl.n_vtiles;
+  p.units = (a.V + HT_WBOX - 1) / HT_WBOX;
   p.slots = pl.slots;
   p.stages = l.stages;
   p.gamma = a.gamma;
@@ -270,7 +291,7 @@ cudaError_t launch_head_tc(const HeadArgs& a, const HeadPlan& pl, const HeadTcLa
   p.gathered = a.gathered;
   p.status = a.status;
   dim3 grid(pl.slots, pl.n_chunks);
-  head_tc_kernel<<<grid, HT_THREADS, l.smem_bytes, s>>>(l.tm_w, l.tm_h, p);
+  head_tc_kernel<<<grid, HT_THREADS, l.smem_bytes, s>>>(l.tm_w, l.tm_w16, l.tm_h, p);
   return cudaGetLastError();
 }
 

@@ -1,7 +1,9 @@
-// Small kernels of the verify step: block packing (Eq. 1), gathering of the
-// original / reflective hidden rows for the LM head, the merge of the head's
-// per-CTA statistics into per-position scores (Eq. 2), and exact-match
-// acceptance with the longest accepted prefix (Alg. 2).
+// Small kernels of the verify step: block packing (Eq. 1); the prep kernel
+// that gathers the original / reflective hidden rows for the LM head (and
+// packs the block in the same launch); the finalize kernel that merges the
+// head's per-CTA statistics into per-position scores (Eq. 2) and, inside
+// rv_verify_step, runs the exact-match acceptance with the longest accepted
+// prefix (Alg. 2); the stand-alone acceptance kernel of rv_accept.
 #include <cfloat>
 #include <climits>
 
@@ -46,16 +48,36 @@ cudaError_t launch_pack_block(const int32_t* drafts, const int32_t* prompt, cons
   return cudaGetLastError();
 }
 
-// ---------------------------------------------------------------- gather rows
+// ---------------------------------------------------------------- prep: gather rows (+ pack)
 // hsel row (c*N + j)        = hidden[b][i]            (original row of pair c*Pc+j)
 // hsel row (c*N + Pcp + j)  = hidden[b][gamma+R+i]    (reflective row, shift_len = gamma+R)
-// padding rows are zero.  One 16-byte vector per thread.
-__global__ void gather_rows_kernel(const uint4* __restrict__ hidden, uint4* __restrict__ hsel,
-                                   int P, int gamma, int R, int Lh, int Hv, int Pc, int Pcp,
-                                   int N, int n_chunks) {
+// padding rows are zero.  One 16-byte vector per thread and step.  When the
+// block is to be packed too, the first B*Lb threads of the grid also do that.
+__global__ void prep_kernel(const uint4* __restrict__ hidden, uint4* __restrict__ hsel, int P,
+                            int gamma, int R, int Lh, int Hv, int Pc, int Pcp, int N, int n_chunks,
+                            const PackArgs pk) {
+  const long long tid0 = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x;
+  if (pk.block != nullptr) {
+    const int Lb = 2 * pk.gamma + pk.n_prompt + pk.n_prefix;
+    for (long long idx = tid0; idx < static_cast<long long>(pk.B) * Lb;
+         idx += static_cast<long long>(gridDim.x) * blockDim.x) {
+      const int b = static_cast<int>(idx / Lb), j = static_cast<int>(idx % Lb);
+      int tok;
+      if (j < pk.gamma)
+        tok = pk.drafts[b * pk.gamma + j];
+      else if (j < pk.gamma + pk.n_prompt)
+        tok = pk.prompt[j - pk.gamma];
+      else if (j < pk.gamma + pk.n_prompt + pk.n_prefix)
+        tok = pk.prefix[b * pk.n_prefix + (j - pk.gamma - pk.n_prompt)];
+      else
+        tok = pk.drafts[b * pk.gamma + (j - pk.gamma - pk.n_prompt - pk.n_prefix)];
+      pk.block[idx] = tok;
+      pk.pos[idx] = pk.ctx[b] + j;
+    }
+  }
+  if (hsel == nullptr) return;
   const long long total = static_cast<long long>(n_chunks) * N * Hv;
-  for (long long idx = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; idx < total;
-       idx += static_cast<long long>(gridDim.x) * blockDim.x) {
+  for (long long idx = tid0; idx < total; idx += static_cast<long long>(gridDim.x) * blockDim.x) {
     const int col = static_cast<int>(idx % Hv);
     const int row = static_cast<int>(idx / Hv);
     const int c = row / N, r = row % N;
@@ -72,96 +94,154 @@ __global__ void gather_rows_kernel(const uint4* __restrict__ hidden, uint4* __re
   }
 }
 
-cudaError_t launch_gather_rows(const HeadArgs& a, const HeadPlan& p, void* hsel, cudaStream_t s) {
+cudaError_t launch_prep(const HeadArgs& a, const HeadPlan& p, void* hsel, const PackArgs* pack,
+                        cudaStream_t s) {
+  PackArgs pk = {};
+  long long work = 0;
+  if (pack) {
+    pk = *pack;
+    work = static_cast<long long>(pk.B) * (2 * pk.gamma + pk.n_prompt + pk.n_prefix);
+  }
   const int Hv = a.H / 8;  // 8 bf16 per 16-byte vector
   const int Lh = 2 * a.gamma + a.R + 1;
-  const long long total = static_cast<long long>(p.n_chunks) * p.N * Hv;
+  if (hsel) work = std::max(work, static_cast<long long>(p.n_chunks) * p.N * Hv);
+  if (work == 0) return cudaSuccess;
   const int threads = 256;
-  const int blocks = static_cast<int>(std::min<long long>((total + threads - 1) / threads, 4096));
-  gather_rows_kernel<<<blocks, threads, 0, s>>>(static_cast<const uint4*>(a.hidden),
-                                                static_cast<uint4*>(hsel), p.P, a.gamma, a.R, Lh,
-                                                Hv, p.pairs_per_chunk, p.pad_pairs, p.N,
-                                                p.n_chunks);
+  const int blocks = static_cast<int>(std::min<long long>((work + threads - 1) / threads, 4096));
+  prep_kernel<<<blocks, threads, 0, s>>>(static_cast<const uint4*>(a.hidden),
+                                         static_cast<uint4*>(hsel), p.P, a.gamma, a.R, Lh, Hv,
+                                         p.pairs_per_chunk, p.pad_pairs, p.N, p.n_chunks, pk);
   return cudaGetLastError();
 }
 
-// ---------------------------------------------------------------- head merge
-// One warp per pair: merge the slots' (max, sum) triples and argmax, then
-// finish the per-position scores.
-__global__ void head_merge_kernel(const float* __restrict__ partials,
-                                  const float* __restrict__ gathered,
-                                  const int32_t* __restrict__ drafts, int P, int gamma, int V,
-                                  int slots, float* __restrict__ scores,
-                                  int32_t* __restrict__ argmax_out, float* __restrict__ margin,
-                                  unsigned* status) {
-  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (warp >= P) return;
-  const int p = warp;
-  float mo = NEG_INF, so = 0.f, mr = NEG_INF, sr = 0.f, mz = NEG_INF, sz = 0.f;
-  float bv = NEG_INF;
-  int bi = INT_MAX;
-  for (int g = lane; g < slots; g += 32) {
-    const float* st = partials + (static_cast<long long>(g) * P + p) * HEAD_STAT_FIELDS;
-    lse_merge(mo, so, st[ST_M_O], st[ST_S_O]);
-    lse_merge(mr, sr, st[ST_M_R], st[ST_S_R]);
-    lse_merge(mz, sz, st[ST_M_Z], st[ST_S_Z]);
-    const float v = st[ST_BEST_V];
-    const int i = __float_as_int(st[ST_BEST_I]);
-    if (v > bv || (v == bv && i < bi)) {
-      bv = v;
-      bi = i;
-    }
+// ---------------------------------------------------------------- head finalize
+// One CTA per sequence; `wpp` warps per position i (pair p = b*(gamma+1)+i)
+// merge the slots' (max, sum) triples and argmax (each lane about one slot),
+// then one thread finishes the position's scores.  Inside rv_verify_step the
+// CTA then runs the exact-match acceptance of its sequence (Alg. 2).
+constexpr int FIN_MAX_WARPS = 32;
+
+struct MergeStat {
+  float mo, so, mr, sr, mz, sz, bv;
+  int bi;
+};
+
+__device__ __forceinline__ void merge_into(MergeStat& a, const MergeStat& b) {
+  lse_merge(a.mo, a.so, b.mo, b.so);
+  lse_merge(a.mr, a.sr, b.mr, b.sr);
+  lse_merge(a.mz, a.sz, b.mz, b.sz);
+  if (b.bv > a.bv || (b.bv == a.bv && b.bi < a.bi)) {
+    a.bv = b.bv;
+    a.bi = b.bi;
   }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    lse_merge(mo, so, __shfl_xor_sync(0xffffffffu, mo, o), __shfl_xor_sync(0xffffffffu, so, o));
-    lse_merge(mr, sr, __shfl_xor_sync(0xffffffffu, mr, o), __shfl_xor_sync(0xffffffffu, sr, o));
-    lse_merge(mz, sz, __shfl_xor_sync(0xffffffffu, mz, o), __shfl_xor_sync(0xffffffffu, sz, o));
-  }
-  warp_argmax(bv, bi);
-  if (lane != 0) return;
-  const int b = p / (gamma + 1), i = p % (gamma + 1);
-  const float lse_o = mo + logf(so);
-  const float lse_r = mr + logf(sr);
-  const float lse_z = mz + logf(sz);
-  float* sc = scores + static_cast<long long>(p) * RV_NSCORES;
-  sc[RV_SCORE_LSE_ORIG] = lse_o;
-  sc[RV_SCORE_LSE_REFL] = lse_r;
-  sc[RV_SCORE_LSE_FUSED] = lse_z;
-  const float nan = __int_as_float(0x7fc00000);
-  int choice = bi;
-  if (i < gamma) {
-    const int x = drafts[b * gamma + i];
-    if (x >= 0 && x < V) {
-      const float* gx = gathered + static_cast<long long>(p) * GATHER_FIELDS;
-      const float zx = gx[2];
-      sc[RV_SCORE_LOGP_FUSED] = zx - lse_z;
-      sc[RV_SCORE_LOGP_ORIG] = gx[0] - lse_o;
-      sc[RV_SCORE_LOGP_REFL] = gx[1] - lse_r;
-      if (zx > bv || (zx == bv && x < bi)) choice = x;
-      margin[b * gamma + i] = fabsf(zx - bv);
-    } else {
-      raise_status(status, RV_DEV_DRAFT_RANGE);
-      sc[RV_SCORE_LOGP_FUSED] = nan;
-      sc[RV_SCORE_LOGP_ORIG] = nan;
-      sc[RV_SCORE_LOGP_REFL] = nan;
-      margin[b * gamma + i] = nan;
-    }
-  } else {
-    sc[RV_SCORE_LOGP_FUSED] = nan;
-    sc[RV_SCORE_LOGP_ORIG] = nan;
-    sc[RV_SCORE_LOGP_REFL] = nan;
-  }
-  argmax_out[p] = choice;
 }
 
-cudaError_t launch_head_merge(const HeadArgs& a, const HeadPlan& p, float* scores,
-                              int32_t* argmax, float* margin, cudaStream_t s) {
-  const int threads = 128;
-  const int blocks = (p.P * 32 + threads - 1) / threads;
-  head_merge_kernel<<<blocks, threads, 0, s>>>(a.partials, a.gathered, a.drafts, p.P, a.gamma,
-                                               a.V, p.slots, scores, argmax, margin, a.status);
+__device__ __forceinline__ MergeStat shfl_stat(const MergeStat& s, int o) {
+  MergeStat r;
+  r.mo = __shfl_xor_sync(0xffffffffu, s.mo, o);
+  r.so = __shfl_xor_sync(0xffffffffu, s.so, o);
+  r.mr = __shfl_xor_sync(0xffffffffu, s.mr, o);
+  r.sr = __shfl_xor_sync(0xffffffffu, s.sr, o);
+  r.mz = __shfl_xor_sync(0xffffffffu, s.mz, o);
+  r.sz = __shfl_xor_sync(0xffffffffu, s.sz, o);
+  r.bv = __shfl_xor_sync(0xffffffffu, s.bv, o);
+  r.bi = __shfl_xor_sync(0xffffffffu, s.bi, o);
+  return r;
+}
+
+__global__ void head_finalize_kernel(const float* __restrict__ partials,
+                                     const float* __restrict__ gathered,
+                                     const int32_t* __restrict__ drafts, int P, int gamma, int V,
+                                     int slots, int wpp, float* __restrict__ scores,
+                                     int32_t* __restrict__ argmax_out, float* __restrict__ margin,
+                                     unsigned* status, AcceptArgs acc) {
+  __shared__ MergeStat red[FIN_MAX_WARPS];
+  __shared__ int s_choice[65];
+  const int b = blockIdx.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  const int npos = gamma + 1, per_pass = nw / wpp;
+  const int sub = warp % wpp;
+  const float nan = __int_as_float(0x7fc00000);
+  for (int base = 0; base < npos; base += per_pass) {
+    const int i = base + warp / wpp;
+    const bool active = i < npos;
+    MergeStat st{NEG_INF, 0.f, NEG_INF, 0.f, NEG_INF, 0.f, NEG_INF, INT_MAX};
+    if (active) {
+      const int p = b * npos + i;
+      for (int g = sub * 32 + lane; g < slots; g += wpp * 32) {
+        const float* q = partials + (static_cast<long long>(g) * P + p) * HEAD_STAT_FIELDS;
+        const MergeStat o{q[ST_M_O], q[ST_S_O], q[ST_M_R], q[ST_S_R],
+                          q[ST_M_Z], q[ST_S_Z], q[ST_BEST_V], __float_as_int(q[ST_BEST_I])};
+        merge_into(st, o);
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) merge_into(st, shfl_stat(st, o));
+    if (lane == 0) red[warp] = st;
+    __syncthreads();
+    if (active && sub == 0 && lane == 0) {
+      for (int w = 1; w < wpp; ++w) merge_into(st, red[warp + w]);
+      const int p = b * npos + i;
+      const float lse_o = st.mo + logf(st.so);
+      const float lse_r = st.mr + logf(st.sr);
+      const float lse_z = st.mz + logf(st.sz);
+      float* sc = scores + static_cast<long long>(p) * RV_NSCORES;
+      sc[RV_SCORE_LSE_ORIG] = lse_o;
+      sc[RV_SCORE_LSE_REFL] = lse_r;
+      sc[RV_SCORE_LSE_FUSED] = lse_z;
+      int choice = st.bi;
+      float lp_z = nan, lp_o = nan, lp_r = nan;
+      if (i < gamma) {
+        const int x = drafts[b * gamma + i];
+        if (x >= 0 && x < V) {
+          const float* gx = gathered + static_cast<long long>(p) * GATHER_FIELDS;
+          const float zx = gx[2];
+          lp_z = zx - lse_z;
+          lp_o = gx[0] - lse_o;
+          lp_r = gx[1] - lse_r;
+          if (zx > st.bv || (zx == st.bv && x < st.bi)) choice = x;
+          margin[b * gamma + i] = fabsf(zx - st.bv);
+        } else {
+          raise_status(status, RV_DEV_DRAFT_RANGE);
+          margin[b * gamma + i] = nan;
+        }
+      }
+      sc[RV_SCORE_LOGP_FUSED] = lp_z;
+      sc[RV_SCORE_LOGP_ORIG] = lp_o;
+      sc[RV_SCORE_LOGP_REFL] = lp_r;
+      argmax_out[p] = choice;
+      s_choice[i] = choice;
+    }
+    __syncthreads();
+  }
+  if (acc.accepted_len == nullptr) return;
+  if (threadIdx.x == 0) {
+    int n = gamma;
+    for (int i = 0; i < gamma; ++i) {
+      const bool ok = drafts[b * gamma + i] == s_choice[i];
+      acc.accept_mask[b * gamma + i] = ok ? 1 : 0;
+      if (!ok && n == gamma) n = i;
+    }
+    acc.accepted_len[b] = n;
+    acc.next_token[b] = s_choice[n];
+    acc.ctx_out[b] = acc.ctx_in[b] + n;
+  }
+}
+
+cudaError_t launch_head_finalize(const HeadArgs& a, const HeadPlan& p, float* scores,
+                                 int32_t* argmax, float* margin, const AcceptArgs* acc,
+                                 cudaStream_t s) {
+  AcceptArgs ac = {};
+  if (acc) ac = *acc;
+  const int npos = a.gamma + 1;
+  int wpp = 1, warps = FIN_MAX_WARPS;
+  if (npos <= FIN_MAX_WARPS) {
+    wpp = std::max(1, std::min((p.slots + 31) / 32, FIN_MAX_WARPS / npos));
+    warps = npos * wpp;
+  }
+  head_finalize_kernel<<<a.B, warps * 32, 0, s>>>(a.partials, a.gathered, a.drafts, p.P, a.gamma,
+                                                  a.V, p.slots, wpp, scores, argmax, margin,
+                                                  a.status, ac);
   return cudaGetLastError();
 }
 

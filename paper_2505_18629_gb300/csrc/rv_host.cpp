@@ -36,8 +36,6 @@ struct Workspace {
   float* head_partials = nullptr;
   float* gathered = nullptr;
   void* hsel = nullptr;
-  float* attn_part = nullptr;  // part_o followed by part_ml
-  size_t attn_part_floats = 0;
   // staging for rv_verify_step_host
   void* st_q = nullptr;
   void* st_kb = nullptr;
@@ -45,6 +43,10 @@ struct Workspace {
   void* st_hidden = nullptr;
   void* st_attn = nullptr;
   int32_t* st_drafts = nullptr;
+  int32_t* st_prompt = nullptr;
+  int32_t* st_prefix = nullptr;
+  int32_t* st_block = nullptr;
+  int32_t* st_pos = nullptr;
   int32_t* st_ctx_in = nullptr;
   int32_t* st_ctx_out = nullptr;
   float* st_scores = nullptr;
@@ -62,12 +64,14 @@ struct rv_handle {
   int device = 0;
   int num_sms = 0;
   size_t smem_optin = 0;
+  int attn_max_cluster = 1;
   Workspace ws;
   std::string err;
   PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
   // cached tensor maps
   const void* tm_w_ptr = nullptr;
   CUtensorMap tm_w;
+  CUtensorMap tm_w16;
   int tm_h_N = -1;
   int tm_h_rows = -1;
   CUtensorMap tm_h;
@@ -108,8 +112,12 @@ HeadPlan head_plan(int B, int gamma, int V, int num_sms, bool tc) {
   p.pad_pairs = (p.pairs_per_chunk + 7) / 8 * 8;
   p.N = 2 * p.pad_pairs;
   p.n_vtiles = (V + 127) / 128;
-  const int per_chunk = std::max(1, (tc ? num_sms : 4 * num_sms) / p.n_chunks);
-  p.slots = std::max(1, std::min(per_chunk, p.n_vtiles));
+  if (tc) {  // one persistent CTA per SM; the vocab is split in 16-row units
+    const int units = (V + 15) / 16;
+    p.slots = std::max(1, std::min(num_sms / p.n_chunks, units));
+  } else {
+    p.slots = std::max(1, std::min(4 * num_sms / p.n_chunks, p.n_vtiles));
+  }
   return p;
 }
 
@@ -209,16 +217,6 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
     }
   }
   const size_t o_hsel = take(hsel_rows * c.hidden * 2);
-  size_t attn_floats = 0;
-  if (bf16) {
-    for (int B = 1; B <= c.max_batch; ++B)
-      for (int Lb = 1; Lb <= Lbm; ++Lb)
-        attn_floats = std::max(attn_floats,
-                               attn_partial_floats(attn_plan(B, Lb, c.n_q_heads, c.n_kv_heads,
-                                                             c.max_ctx, h->num_sms, true),
-                                                   B, Lb, c.n_q_heads, c.head_dim));
-  }
-  const size_t o_attn = take(attn_floats * 4);
   const size_t es = esize(c);
   const size_t n_q = static_cast<size_t>(c.max_batch) * Lbm * c.n_q_heads * c.head_dim;
   const size_t n_kv = static_cast<size_t>(c.max_batch) * Lbm * c.n_kv_heads * c.head_dim;
@@ -226,6 +224,10 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
   const size_t o_q = take(n_q * es), o_kb = take(n_kv * es), o_vb = take(n_kv * es);
   const size_t o_hid = take(n_hid * es), o_ao = take(n_q * es);
   const size_t o_dr = take(static_cast<size_t>(c.max_batch) * c.max_gamma * 4);
+  const size_t o_pr = take(static_cast<size_t>(c.max_template) * 4 + 4);
+  const size_t o_px = take(static_cast<size_t>(c.max_batch) * c.max_template * 4 + 4);
+  const size_t o_bl = take(static_cast<size_t>(c.max_batch) * Lbm * 4);
+  const size_t o_ps = take(static_cast<size_t>(c.max_batch) * Lbm * 4);
   const size_t o_ci = take(c.max_batch * 4), o_co = take(c.max_batch * 4);
   const size_t o_sc = take(static_cast<size_t>(Pmax) * RV_NSCORES * 4);
   const size_t o_am = take(static_cast<size_t>(Pmax) * 4);
@@ -244,14 +246,16 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
   h->ws.head_partials = reinterpret_cast<float*>(b + o_part);
   h->ws.gathered = reinterpret_cast<float*>(b + o_gath);
   h->ws.hsel = b + o_hsel;
-  h->ws.attn_part = reinterpret_cast<float*>(b + o_attn);
-  h->ws.attn_part_floats = attn_floats;
   h->ws.st_q = b + o_q;
   h->ws.st_kb = b + o_kb;
   h->ws.st_vb = b + o_vb;
   h->ws.st_hidden = b + o_hid;
   h->ws.st_attn = b + o_ao;
   h->ws.st_drafts = reinterpret_cast<int32_t*>(b + o_dr);
+  h->ws.st_prompt = reinterpret_cast<int32_t*>(b + o_pr);
+  h->ws.st_prefix = reinterpret_cast<int32_t*>(b + o_px);
+  h->ws.st_block = reinterpret_cast<int32_t*>(b + o_bl);
+  h->ws.st_pos = reinterpret_cast<int32_t*>(b + o_ps);
   h->ws.st_ctx_in = reinterpret_cast<int32_t*>(b + o_ci);
   h->ws.st_ctx_out = reinterpret_cast<int32_t*>(b + o_co);
   h->ws.st_scores = reinterpret_cast<float*>(b + o_sc);
@@ -261,7 +265,7 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
   h->ws.st_acc_len = reinterpret_cast<int32_t*>(b + o_al);
   h->ws.st_next = reinterpret_cast<int32_t*>(b + o_nt);
   e = cudaMemset(h->ws.base, 0, off);
-  if (e == cudaSuccess && bf16) e = attn_configure();
+  if (e == cudaSuccess && bf16) e = attn_configure(&h->attn_max_cluster);
   if (e == cudaSuccess && bf16) e = head_tc_configure(h->smem_optin);
   if (e == cudaSuccess && bf16) {
     cudaDriverEntryPointQueryResult q;
@@ -343,25 +347,17 @@ extern "C" RV_API int rv_verify_attention(rv_handle* h, const void* q, const voi
     return fail(h, RV_ERR_INVALID_ARG, "attention tensors must be 16-byte aligned");
   AttnArgs a{q, k_blk, v_blk, k_cache, v_cache, ctx_lens, out, B, Lb, c.n_q_heads, c.n_kv_heads,
              c.head_dim, c.max_ctx, h->ws.status};
-  const AttnPlan p = attn_plan(B, Lb, c.n_q_heads, c.n_kv_heads, c.max_ctx, h->num_sms, bf16);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   ProfScope prof(h, RV_PROF_ATTENTION, s);
   cudaError_t e;
   if (bf16) {
-    const size_t nf = attn_partial_floats(p, B, Lb, c.n_q_heads, c.head_dim);
-    if (nf > h->ws.attn_part_floats) return fail(h, RV_ERR_CAPACITY, "attention workspace too small");
-    float* part_o = h->ws.attn_part;
-    float* part_ml = part_o + static_cast<size_t>(p.splits) * B * Lb * c.n_q_heads * c.head_dim;
-    e = launch_attention_bf16(a, p, part_o, part_ml, s);
-    h->launches += 1;
-    if (e == cudaSuccess && p.splits > 1) {
-      e = launch_attention_combine(a, p, part_o, part_ml, true, s);
-      h->launches += 1;
-    }
+    const AttnPlan p = attn_plan(B, Lb, c.n_q_heads, c.n_kv_heads, c.max_ctx, h->num_sms, true,
+                                 h->attn_max_cluster);
+    e = launch_attention_bf16(a, p, s);
   } else {
-    e = launch_attention_f32(a, p, nullptr, nullptr, s);
-    h->launches += 1;
+    e = launch_attention_f32(a, s);
   }
+  h->launches += 1;
   return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "attention launch");
 }
 
@@ -374,12 +370,17 @@ int encode_maps(rv_handle* h, const void* w, const HeadPlan& pl, HeadTcLaunch& l
   if (h->tm_w_ptr != w) {
     const cuuint64_t dims[2] = {static_cast<cuuint64_t>(c.hidden), static_cast<cuuint64_t>(c.vocab)};
     const cuuint64_t strides[1] = {static_cast<cuuint64_t>(c.hidden) * 2};
-    const cuuint32_t box[2] = {64, 128};
     const cuuint32_t es[2] = {1, 1};
+    const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(HEAD_TILE_ROWS)};
+    const cuuint32_t box16[2] = {64, static_cast<cuuint32_t>(HEAD_W_BOX_ROWS)};
     CUresult r = h->encode(&h->tm_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(w), dims,
                            strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
                            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r == CUDA_SUCCESS)
+      r = h->encode(&h->tm_w16, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(w), dims,
+                    strides, box16, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) {
       h->tm_w_ptr = nullptr;
       return fail(h, RV_ERR_CUDA, "cuTensorMapEncodeTiled(W) failed: %d", static_cast<int>(r));
@@ -403,6 +404,7 @@ int encode_maps(rv_handle* h, const void* w, const HeadPlan& pl, HeadTcLaunch& l
     h->tm_h_rows = rows;
   }
   l.tm_w = h->tm_w;
+  l.tm_w16 = h->tm_w16;
   l.tm_h = h->tm_h;
   if (h->head_tc_stages_cached_N != pl.N) {
     h->head_tc_stages = head_tc_max_stages(pl.N, h->smem_optin);
@@ -433,38 +435,33 @@ int check_head_args(rv_handle* h, const void* hidden, const void* w_head, const 
 
 int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_t* draft_ids, int B,
               int gamma, int R, float alpha, float* scores, int32_t* argmax, float* margin,
-              cudaStream_t s) {
+              const PackArgs* pack, const AcceptArgs* acc, cudaStream_t s) {
   const rv_config& c = h->cfg;
   const bool bf16 = c.dtype == RV_DTYPE_BF16;
   HeadArgs a{hidden, w_head, draft_ids, B, gamma, R, c.vocab, c.hidden, alpha,
              h->ws.head_partials, h->ws.gathered, h->ws.status};
   const HeadPlan pl = head_plan(B, gamma, c.vocab, h->num_sms, bf16);
   ProfScope prof_all(h, RV_PROF_HEAD, s);
-  cudaError_t e;
+  cudaError_t e = cudaSuccess;
+  HeadTcLaunch l;
   if (bf16) {
-    HeadTcLaunch l;
     int rc = encode_maps(h, w_head, pl, l);
     if (rc != RV_OK) return rc;
-    e = launch_gather_rows(a, pl, h->ws.hsel, s);
-    h->launches += 1;
-    if (e != cudaSuccess) return cuda_fail(h, e, "gather_rows launch");
-    {
-      ProfScope prof(h, RV_PROF_HEAD_GEMM, s);
-      e = launch_head_tc(a, pl, l, s);
-      h->launches += 1;
-    }
-    if (e != cudaSuccess) return cuda_fail(h, e, "head_tc launch");
-  } else {
-    {
-      ProfScope prof(h, RV_PROF_HEAD_GEMM, s);
-      e = launch_head_simt(a, pl, s);
-      h->launches += 1;
-    }
-    if (e != cudaSuccess) return cuda_fail(h, e, "head_simt launch");
   }
-  e = launch_head_merge(a, pl, scores, argmax, margin, s);
+  if (bf16 || pack) {
+    e = launch_prep(a, pl, bf16 ? h->ws.hsel : nullptr, pack, s);
+    h->launches += 1;
+    if (e != cudaSuccess) return cuda_fail(h, e, "prep launch");
+  }
+  {
+    ProfScope prof(h, RV_PROF_HEAD_GEMM, s);
+    e = bf16 ? launch_head_tc(a, pl, l, s) : launch_head_simt(a, pl, s);
+    h->launches += 1;
+  }
+  if (e != cudaSuccess) return cuda_fail(h, e, "LM head launch");
+  e = launch_head_finalize(a, pl, scores, argmax, margin, acc, s);
   h->launches += 1;
-  return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "head_merge launch");
+  return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "head finalize launch");
 }
 
 int accept_impl(rv_handle* h, const int32_t* draft_ids, const int32_t* argmax, int B, int gamma,
@@ -488,7 +485,7 @@ extern "C" RV_API int rv_verify_head(rv_handle* h, const void* hidden, const voi
   int rc = check_head_args(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin);
   if (rc != RV_OK || B == 0) return rc;
   return head_impl(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin,
-                   static_cast<cudaStream_t>(stream));
+                   nullptr, nullptr, static_cast<cudaStream_t>(stream));
 }
 
 extern "C" RV_API int rv_accept(rv_handle* h, const int32_t* draft_ids, const int32_t* argmax,
@@ -509,41 +506,60 @@ extern "C" RV_API int rv_accept(rv_handle* h, const int32_t* draft_ids, const in
 
 // ============================================================================ whole step
 
-extern "C" RV_API int rv_verify_step(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
-                                     void* k_cache, void* v_cache, const void* hidden,
-                                     const void* w_head, const int32_t* draft_ids,
-                                     const int32_t* ctx_in, int32_t B, int32_t gamma, int32_t R,
-                                     float alpha, void* attn_out, float* scores, int32_t* argmax,
-                                     float* margin, uint8_t* accept_mask, int32_t* accepted_len,
-                                     int32_t* next_token, int32_t* ctx_out, void* stream) {
+extern "C" RV_API int rv_verify_step(
+    rv_handle* h, const void* q, const void* k_blk, const void* v_blk, void* k_cache, void* v_cache,
+    const void* hidden, const void* w_head, const int32_t* draft_ids, const int32_t* prompt_ids,
+    const int32_t* prefix_ids, const int32_t* ctx_in, int32_t B, int32_t gamma, int32_t n_prompt,
+    int32_t n_prefix, float alpha, int32_t* block_ids, int32_t* pos_ids, void* attn_out,
+    float* scores, int32_t* argmax, float* margin, uint8_t* accept_mask, int32_t* accepted_len,
+    int32_t* next_token, int32_t* ctx_out, void* stream) {
   if (!h) return RV_ERR_INVALID_ARG;
-  int rc = rv_verify_attention(h, q, k_blk, v_blk, k_cache, v_cache, ctx_in, B, 2 * gamma + R,
-                               attn_out, stream);
+  h->err.clear();
+  if (n_prompt < 0 || n_prefix < 0) return fail(h, RV_ERR_SHAPE, "negative template part");
+  const int R = n_prompt + n_prefix;
+  int rc = check_head_args(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin);
+  if (rc != RV_OK || B == 0) return rc;
+  if (!ctx_in || !accept_mask || !accepted_len || !next_token || !ctx_out)
+    return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument");
+  const bool do_pack = block_ids != nullptr;
+  if (do_pack && (!pos_ids || (n_prompt > 0 && !prompt_ids) || (n_prefix > 0 && !prefix_ids)))
+    return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument for the block packing");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  rc = rv_verify_attention(h, q, k_blk, v_blk, k_cache, v_cache, ctx_in, B, 2 * gamma + R,
+                           attn_out, stream);
   if (rc != RV_OK) return rc;
-  rc = rv_verify_head(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin,
-                      stream);
-  if (rc != RV_OK) return rc;
-  return rv_accept(h, draft_ids, argmax, B, gamma, accept_mask, accepted_len, next_token, ctx_in,
-                   ctx_out, stream);
+  PackArgs pk{draft_ids, prompt_ids, prefix_ids, ctx_in, B, gamma, n_prompt, n_prefix, block_ids,
+              pos_ids};
+  AcceptArgs ac{accept_mask, accepted_len, next_token, ctx_in, ctx_out};
+  return head_impl(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin,
+                   do_pack ? &pk : nullptr, &ac, s);
 }
 
 extern "C" RV_API int rv_verify_step_host(
     rv_handle* h, const void* q_host, const void* k_blk_host, const void* v_blk_host, void* k_cache,
     void* v_cache, const void* hidden_host, const void* w_head, const int32_t* draft_ids_host,
-    const int32_t* ctx_in_host, int32_t B, int32_t gamma, int32_t R, float alpha,
-    void* attn_out_host, float* scores_host, int32_t* argmax_host, float* margin_host,
-    uint8_t* accept_mask_host, int32_t* accepted_len_host, int32_t* next_token_host,
-    int32_t* ctx_out_host, uint64_t* h2d_bytes, uint64_t* d2h_bytes, void* stream) {
+    const int32_t* prompt_ids_host, const int32_t* prefix_ids_host, const int32_t* ctx_in_host,
+    int32_t B, int32_t gamma, int32_t n_prompt, int32_t n_prefix, float alpha,
+    int32_t* block_ids_host, int32_t* pos_ids_host, void* attn_out_host, float* scores_host,
+    int32_t* argmax_host, float* margin_host, uint8_t* accept_mask_host, int32_t* accepted_len_host,
+    int32_t* next_token_host, int32_t* ctx_out_host, uint64_t* h2d_bytes, uint64_t* d2h_bytes,
+    void* stream) {
   if (!h) return RV_ERR_INVALID_ARG;
   h->err.clear();
   const rv_config& c = h->cfg;
-  if (B < 1 || gamma < 1 || R < 0) return fail(h, RV_ERR_SHAPE, "need B >= 1, gamma >= 1, R >= 0");
+  if (B < 1 || gamma < 1 || n_prompt < 0 || n_prefix < 0)
+    return fail(h, RV_ERR_SHAPE, "need B >= 1, gamma >= 1, template parts >= 0");
+  const int R = n_prompt + n_prefix;
   if (B > c.max_batch || gamma > c.max_gamma || R > c.max_template)
     return fail(h, RV_ERR_CAPACITY, "B / gamma / R above the handle's maxima");
   if (!q_host || !k_blk_host || !v_blk_host || !k_cache || !v_cache || !hidden_host || !w_head ||
       !draft_ids_host || !ctx_in_host || !scores_host || !argmax_host || !margin_host ||
       !accept_mask_host || !accepted_len_host || !next_token_host || !ctx_out_host)
     return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument");
+  const bool do_pack = block_ids_host != nullptr;
+  if (do_pack && (!pos_ids_host || (n_prompt > 0 && !prompt_ids_host) ||
+                  (n_prefix > 0 && !prefix_ids_host)))
+    return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument for the block packing");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const size_t es = esize(c);
   const int Lb = 2 * gamma + R;
@@ -551,14 +567,19 @@ extern "C" RV_API int rv_verify_step_host(
   const size_t nkv = static_cast<size_t>(B) * Lb * c.n_kv_heads * c.head_dim * es;
   const size_t nh = static_cast<size_t>(B) * (Lb + 1) * c.hidden * es;
   const size_t nd = static_cast<size_t>(B) * gamma * 4, nc = static_cast<size_t>(B) * 4;
+  const size_t npr = static_cast<size_t>(n_prompt) * 4, npx = static_cast<size_t>(B) * n_prefix * 4;
+  const size_t nbl = static_cast<size_t>(B) * Lb * 4;
   const size_t P = static_cast<size_t>(B) * (gamma + 1);
   Workspace& w = h->ws;
   cudaError_t e = cudaSuccess;
+  size_t in_bytes = 0, out_bytes = 0;
   auto h2d = [&](void* dst, const void* src, size_t n) {
-    if (e == cudaSuccess) e = cudaMemcpyAsync(dst, src, n, cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess && n) e = cudaMemcpyAsync(dst, src, n, cudaMemcpyHostToDevice, s);
+    in_bytes += n;
   };
   auto d2h = [&](void* dst, const void* src, size_t n) {
-    if (e == cudaSuccess) e = cudaMemcpyAsync(dst, src, n, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess && n) e = cudaMemcpyAsync(dst, src, n, cudaMemcpyDeviceToHost, s);
+    out_bytes += n;
   };
   h2d(w.st_q, q_host, nq);
   h2d(w.st_kb, k_blk_host, nkv);
@@ -566,16 +587,21 @@ extern "C" RV_API int rv_verify_step_host(
   h2d(w.st_hidden, hidden_host, nh);
   h2d(w.st_drafts, draft_ids_host, nd);
   h2d(w.st_ctx_in, ctx_in_host, nc);
+  if (do_pack) {
+    h2d(w.st_prompt, prompt_ids_host, npr);
+    h2d(w.st_prefix, prefix_ids_host, npx);
+  }
   if (e != cudaSuccess) return cuda_fail(h, e, "host->device copy");
   int rc = rv_verify_step(h, w.st_q, w.st_kb, w.st_vb, k_cache, v_cache, w.st_hidden, w_head,
-                          w.st_drafts, w.st_ctx_in, B, gamma, R, alpha, w.st_attn, w.st_scores,
-                          w.st_argmax, w.st_margin, w.st_accept, w.st_acc_len, w.st_next,
-                          w.st_ctx_out, stream);
+                          w.st_drafts, w.st_prompt, w.st_prefix, w.st_ctx_in, B, gamma, n_prompt,
+                          n_prefix, alpha, do_pack ? w.st_block : nullptr, w.st_pos, w.st_attn,
+                          w.st_scores, w.st_argmax, w.st_margin, w.st_accept, w.st_acc_len,
+                          w.st_next, w.st_ctx_out, stream);
   if (rc != RV_OK) return rc;
-  size_t out_bytes = 0;
-  if (attn_out_host) {
-    d2h(attn_out_host, w.st_attn, nq);
-    out_bytes += nq;
+  if (attn_out_host) d2h(attn_out_host, w.st_attn, nq);
+  if (do_pack) {
+    d2h(block_ids_host, w.st_block, nbl);
+    d2h(pos_ids_host, w.st_pos, nbl);
   }
   d2h(scores_host, w.st_scores, P * RV_NSCORES * 4);
   d2h(argmax_host, w.st_argmax, P * 4);
@@ -586,8 +612,7 @@ extern "C" RV_API int rv_verify_step_host(
   d2h(ctx_out_host, w.st_ctx_out, nc);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return cuda_fail(h, e, "device->host copy");
-  out_bytes += P * RV_NSCORES * 4 + P * 4 + nd + static_cast<size_t>(B) * gamma + 3 * nc;
-  if (h2d_bytes) *h2d_bytes = nq + 2 * nkv + nh + nd + nc;
+  if (h2d_bytes) *h2d_bytes = in_bytes;
   if (d2h_bytes) *d2h_bytes = out_bytes;
   return RV_OK;
 }

@@ -55,17 +55,46 @@ struct HeadArgs {
 cudaError_t launch_pack_block(const int32_t* drafts, const int32_t* prompt, const int32_t* prefix,
                               const int32_t* ctx, int B, int gamma, int n_prompt, int n_prefix,
                               int32_t* block_ids, int32_t* pos_ids, cudaStream_t s);
-// hidden rows of every chunk into hsel [n_chunks * N, H] (bf16), pads zeroed
-cudaError_t launch_gather_rows(const HeadArgs& a, const HeadPlan& p, void* hsel, cudaStream_t s);
-cudaError_t launch_head_merge(const HeadArgs& a, const HeadPlan& p, float* scores,
-                              int32_t* argmax, float* margin, cudaStream_t s);
+// Optional block packing (Eq. 1) for rv_verify_step: pack.block == nullptr skips it.
+struct PackArgs {
+  const int32_t* drafts;
+  const int32_t* prompt;
+  const int32_t* prefix;
+  const int32_t* ctx;
+  int B, gamma, n_prompt, n_prefix;
+  int32_t* block;
+  int32_t* pos;
+};
+// hidden rows of every chunk into hsel [n_chunks * N, H] (bf16), pads zeroed;
+// also packs the block when `pack` is given (one launch for both).
+cudaError_t launch_prep(const HeadArgs& a, const HeadPlan& p, void* hsel, const PackArgs* pack,
+                        cudaStream_t s);
+// Optional acceptance fused into the head merge (rv_verify_step).
+struct AcceptArgs {
+  uint8_t* accept_mask;
+  int32_t* accepted_len;
+  int32_t* next_token;
+  const int32_t* ctx_in;
+  int32_t* ctx_out;
+};
+// Merge the head's per-CTA statistics into scores / argmax / margin, and run
+// the acceptance of each sequence when `acc` is given.
+cudaError_t launch_head_finalize(const HeadArgs& a, const HeadPlan& p, float* scores,
+                                 int32_t* argmax, float* margin, const AcceptArgs* acc,
+                                 cudaStream_t s);
 cudaError_t launch_accept(const int32_t* drafts, const int32_t* argmax, int B, int gamma,
                           uint8_t* accept_mask, int32_t* accepted_len, int32_t* next_token,
                           const int32_t* ctx_in, int32_t* ctx_out, cudaStream_t s);
 
 // ---- LM head (k_head_tc.cu: bf16 tcgen05; k_head_simt.cu: fp32)
+// Vocab rows per TMA box of the weight: full tiles use HEAD_TILE_ROWS, the
+// partial last tile of a CTA HEAD_W_BOX_ROWS; the tensor maps (host) and the
+// kernel's transaction byte counts (device) both use them.
+constexpr int HEAD_TILE_ROWS = 128;
+constexpr int HEAD_W_BOX_ROWS = 16;
 struct HeadTcLaunch {
   CUtensorMap tm_w;    // W [V, H] bf16, box {64, 128}, 128B swizzle
+  CUtensorMap tm_w16;  // W [V, H] bf16, box {64, 16}, 128B swizzle
   CUtensorMap tm_h;    // hsel [n_chunks*N, H] bf16, box {64, N}, 128B swizzle
   int stages;
   size_t smem_bytes;
@@ -95,16 +124,12 @@ struct AttnPlan {
   int splits;      // key splits
   int warps;       // warps per CTA
 };
-AttnPlan attn_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms, bool bf16);
-size_t attn_partial_floats(const AttnPlan& p, int B, int Lb, int Hq, int D);
-size_t attn_bf16_smem_bytes(int D, int warps);
-cudaError_t attn_configure();
-// part_o [splits][B*Lb*Hq][D] fp32, part_ml [splits][B*Lb*Hq][2]
-cudaError_t launch_attention_bf16(const AttnArgs& a, const AttnPlan& p, float* part_o,
-                                  float* part_ml, cudaStream_t s);
-cudaError_t launch_attention_f32(const AttnArgs& a, const AttnPlan& p, float* part_o,
-                                 float* part_ml, cudaStream_t s);
-cudaError_t launch_attention_combine(const AttnArgs& a, const AttnPlan& p, const float* part_o,
-                                     const float* part_ml, bool bf16, cudaStream_t s);
+// max_cluster: largest thread-block cluster the attention kernel can use (<= 16)
+AttnPlan attn_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms, bool bf16,
+                   int max_cluster);
+size_t attn_bf16_smem_bytes(int D);
+cudaError_t attn_configure(int* max_cluster);
+cudaError_t launch_attention_bf16(const AttnArgs& a, const AttnPlan& p, cudaStream_t s);
+cudaError_t launch_attention_f32(const AttnArgs& a, cudaStream_t s);
 
 }  // namespace rv

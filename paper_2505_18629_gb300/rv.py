@@ -70,9 +70,10 @@ def _load():
         "rv_verify_attention": (I, [P, P, P, P, P, P, P, I, I, P, P]),
         "rv_verify_head": (I, [P, P, P, P, I, I, I, F, P, P, P, P]),
         "rv_accept": (I, [P, P, P, I, I, P, P, P, P, P, P]),
-        "rv_verify_step": (I, [P, P, P, P, P, P, P, P, P, P, I, I, I, F, P, P, P, P, P, P, P, P, P]),
-        "rv_verify_step_host": (I, [P, P, P, P, P, P, P, P, P, P, I, I, I, F, P, P, P, P, P, P, P,
-                                    P, U64P, U64P, P]),
+        "rv_verify_step": (I, [P, P, P, P, P, P, P, P, P, P, P, P, I, I, I, I, F, P, P, P, P, P, P,
+                               P, P, P, P, P]),
+        "rv_verify_step_host": (I, [P, P, P, P, P, P, P, P, P, P, P, P, I, I, I, I, F, P, P, P, P,
+                                    P, P, P, P, P, P, U64P, U64P, P]),
         "rv_read_status": (I, [P, P, ctypes.POINTER(ctypes.c_uint32)]),
         "rv_profile_enable": (I, [P, I]),
         "rv_profile_read": (I, [P, I, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(I)]),
@@ -195,26 +196,34 @@ def rv_accept(h, draft_ids, argmax, accept_mask, accepted_len, next_token, ctx_i
                              _stream(stream)))
 
 
-def rv_verify_step(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, ctx_in,
-                   gamma, R, alpha, attn_out, scores, argmax, margin, accept_mask, accepted_len,
-                   next_token, ctx_out, stream=None):
-    B = hidden.shape[0]
+def rv_verify_step(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, prompt_ids,
+                   prefix_ids, ctx_in, alpha, block_ids, pos_ids, attn_out, scores, argmax, margin,
+                   accept_mask, accepted_len, next_token, ctx_out, stream=None):
+    """Whole step; prompt_ids may be None (empty prompt), block_ids None skips packing."""
+    B, gamma = draft_ids.shape
+    n_prompt = 0 if prompt_ids is None else prompt_ids.numel()
+    n_prefix = prefix_ids.shape[1]
     _check(h, _lib.rv_verify_step(
         h.ptr, _ptr(q), _ptr(k_blk), _ptr(v_blk), _ptr(k_cache), _ptr(v_cache), _ptr(hidden),
-        _ptr(w_head), _ptr(draft_ids), _ptr(ctx_in), B, gamma, R, float(alpha), _ptr(attn_out),
+        _ptr(w_head), _ptr(draft_ids), _ptr(prompt_ids), _ptr(prefix_ids), _ptr(ctx_in), B, gamma,
+        n_prompt, n_prefix, float(alpha), _ptr(block_ids), _ptr(pos_ids), _ptr(attn_out),
         _ptr(scores), _ptr(argmax), _ptr(margin), _ptr(accept_mask), _ptr(accepted_len),
         _ptr(next_token), _ptr(ctx_out), _stream(stream)))
 
 
-def rv_verify_step_host(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, ctx_in,
-                        gamma, R, alpha, attn_out, scores, argmax, margin, accept_mask,
-                        accepted_len, next_token, ctx_out, stream=None):
+def rv_verify_step_host(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids,
+                        prompt_ids, prefix_ids, ctx_in, alpha, block_ids, pos_ids, attn_out,
+                        scores, argmax, margin, accept_mask, accepted_len, next_token, ctx_out,
+                        stream=None):
     """Host tensors in/out (pin them for asynchronous copies); returns (h2d, d2h) bytes."""
-    B = hidden.shape[0]
+    B, gamma = draft_ids.shape
+    n_prompt = 0 if prompt_ids is None else prompt_ids.numel()
+    n_prefix = prefix_ids.shape[1]
     hb, db = ctypes.c_uint64(), ctypes.c_uint64()
     _check(h, _lib.rv_verify_step_host(
         h.ptr, _ptr(q), _ptr(k_blk), _ptr(v_blk), _ptr(k_cache), _ptr(v_cache), _ptr(hidden),
-        _ptr(w_head), _ptr(draft_ids), _ptr(ctx_in), B, gamma, R, float(alpha), _ptr(attn_out),
+        _ptr(w_head), _ptr(draft_ids), _ptr(prompt_ids), _ptr(prefix_ids), _ptr(ctx_in), B, gamma,
+        n_prompt, n_prefix, float(alpha), _ptr(block_ids), _ptr(pos_ids), _ptr(attn_out),
         _ptr(scores), _ptr(argmax), _ptr(margin), _ptr(accept_mask), _ptr(accepted_len),
         _ptr(next_token), _ptr(ctx_out), ctypes.byref(hb), ctypes.byref(db), _stream(stream)))
     return hb.value, db.value

@@ -106,9 +106,8 @@ def run_gpu(inp: synth.VerifyInputs, drafts: np.ndarray, alpha: float, h=None) -
     alen = torch.full((B,), -7, dtype=torch.int32, device="cuda")
     nxt = torch.full((B,), -7, dtype=torch.int32, device="cuda")
     ctx_out = torch.full((B,), -7, dtype=torch.int32, device="cuda")
-    rv.rv_pack_block(h, d, prompt, prefix, ctx, block, pos)
-    rv.rv_verify_step(h, q, kb, vb, kc, vc, hidden, W, d, ctx, g, R, alpha, attn, scores, argmax,
-                      margin, acc, alen, nxt, ctx_out)
+    rv.rv_verify_step(h, q, kb, vb, kc, vc, hidden, W, d, prompt, prefix, ctx, alpha, block, pos,
+                      attn, scores, argmax, margin, acc, alen, nxt, ctx_out)
     status = rv.rv_read_status(h)
     out = GpuRun(to_np(attn), to_np(kc), to_np(vc), to_np(scores), to_np(argmax), to_np(margin),
                  to_np(acc), to_np(alen), to_np(nxt), to_np(ctx_out), to_np(block), to_np(pos),

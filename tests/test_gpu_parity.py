@@ -106,6 +106,93 @@ def test_all_accepted_and_none_accepted(gu):
     assert int(ref["accepted_len"][0]) == wl.gamma and int(ref["accepted_len"][1]) == 0
 
 
+def test_pack_block_entry_point(gu):
+    import torch
+    import oracle.rv_oracle as orc
+    from paper_2505_18629_gb300 import rv, synth
+    wl = _wl(seed=53, B=3, gamma=5, R=7)
+    inp = synth.generate(wl)
+    h = gu.make_handle(wl)
+    d = gu.to_dev(inp.draft_alt)
+    blk = torch.full((3, wl.Lb), -1, dtype=torch.int32, device="cuda")
+    pos = torch.full_like(blk, -1)
+    rv.rv_pack_block(h, d, gu.to_dev(inp.prompt_ids), gu.to_dev(inp.prefix_ids),
+                     gu.to_dev(inp.ctx_lens), blk, pos)
+    ref_b, ref_p = orc.pack_block(inp.draft_alt, inp.prompt_ids, inp.prefix_ids, inp.ctx_lens)
+    np.testing.assert_array_equal(gu.to_np(blk), ref_b)
+    np.testing.assert_array_equal(gu.to_np(pos), ref_p)
+    h.close()
+
+
+def test_separate_entry_points_match_step(gu):
+    """rv_verify_attention + rv_verify_head + rv_accept == rv_verify_step."""
+    import torch
+    from paper_2505_18629_gb300 import rv, synth
+    wl = _wl(seed=54, B=3)
+    inp = synth.generate(wl)
+    drafts = gu.oracle_drafts(inp, ALPHA)
+    step = gu.run_gpu(inp, drafts, ALPHA)
+    h = gu.make_handle(wl)
+    g = wl.gamma
+    q, kb, vb = gu.to_dev(inp.q), gu.to_dev(inp.k_blk), gu.to_dev(inp.v_blk)
+    kc, vc = gu.to_dev(inp.k_cache), gu.to_dev(inp.v_cache)
+    ctx, d = gu.to_dev(inp.ctx_lens), gu.to_dev(drafts.astype(np.int32))
+    attn = torch.zeros_like(q)
+    rv.rv_verify_attention(h, q, kb, vb, kc, vc, ctx, attn)
+    sc = torch.empty((wl.B, g + 1, rv.RV_NSCORES), device="cuda")
+    am = torch.empty((wl.B, g + 1), dtype=torch.int32, device="cuda")
+    mg = torch.empty((wl.B, g), device="cuda")
+    rv.rv_verify_head(h, gu.to_dev(inp.hidden), gu.to_dev(inp.W), d, g, wl.R, ALPHA, sc, am, mg)
+    acc = torch.empty((wl.B, g), dtype=torch.uint8, device="cuda")
+    al = torch.empty((wl.B,), dtype=torch.int32, device="cuda")
+    nt, co = torch.empty_like(al), torch.empty_like(al)
+    rv.rv_accept(h, d, am, acc, al, nt, ctx, co)
+    assert rv.rv_read_status(h) == 0
+    np.testing.assert_array_equal(gu.to_np(attn), step.attn)
+    np.testing.assert_array_equal(gu.to_np(sc), step.scores)
+    np.testing.assert_array_equal(gu.to_np(am), step.argmax)
+    np.testing.assert_array_equal(gu.to_np(acc), step.accept_mask)
+    np.testing.assert_array_equal(gu.to_np(al), step.accepted_len)
+    np.testing.assert_array_equal(gu.to_np(nt), step.next_token)
+    np.testing.assert_array_equal(gu.to_np(co), step.ctx_out)
+    h.close()
+
+
+def test_host_buffer_step_matches_device_step(gu):
+    import torch
+    from paper_2505_18629_gb300 import rv, synth
+    wl = _wl(seed=55, B=2)
+    inp = synth.generate(wl)
+    drafts = gu.oracle_drafts(inp, ALPHA)
+    step = gu.run_gpu(inp, drafts, ALPHA)
+    h = gu.make_handle(wl)
+    g, B, Lb = wl.gamma, wl.B, wl.Lb
+
+    def host(x):
+        t = torch.from_numpy(x.view(np.int16) if x.dtype == np.uint16 else np.ascontiguousarray(x))
+        return (t.view(torch.bfloat16) if x.dtype == np.uint16 else t).pin_memory()
+    kc, vc = gu.to_dev(inp.k_cache), gu.to_dev(inp.v_cache)
+    outs = dict(blk=torch.empty((B, Lb), dtype=torch.int32), pos=torch.empty((B, Lb), dtype=torch.int32),
+                attn=torch.empty(inp.q.shape, dtype=torch.bfloat16),
+                sc=torch.empty((B, g + 1, rv.RV_NSCORES)), am=torch.empty((B, g + 1), dtype=torch.int32),
+                mg=torch.empty((B, g)), acc=torch.empty((B, g), dtype=torch.uint8),
+                al=torch.empty((B,), dtype=torch.int32), nt=torch.empty((B,), dtype=torch.int32),
+                co=torch.empty((B,), dtype=torch.int32))
+    outs = {k: v.pin_memory() for k, v in outs.items()}
+    h2d, d2h = rv.rv_verify_step_host(
+        h, host(inp.q), host(inp.k_blk), host(inp.v_blk), kc, vc, host(inp.hidden),
+        gu.to_dev(inp.W), host(drafts.astype(np.int32)), host(inp.prompt_ids), host(inp.prefix_ids),
+        host(inp.ctx_lens), ALPHA, outs["blk"], outs["pos"], outs["attn"], outs["sc"], outs["am"],
+        outs["mg"], outs["acc"], outs["al"], outs["nt"], outs["co"])
+    assert h2d > 0 and d2h > 0
+    np.testing.assert_array_equal(outs["blk"].numpy(), step.block_ids)
+    np.testing.assert_array_equal(outs["attn"].view(torch.int16).numpy().view(np.uint16), step.attn)
+    np.testing.assert_array_equal(outs["sc"].numpy(), step.scores)
+    np.testing.assert_array_equal(outs["al"].numpy(), step.accepted_len)
+    np.testing.assert_array_equal(outs["nt"].numpy(), step.next_token)
+    h.close()
+
+
 # ------------------------------------------------------------------ device-side checks
 
 def test_out_of_range_draft_sets_status(gu):

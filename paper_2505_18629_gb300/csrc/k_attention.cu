@@ -330,37 +330,42 @@ __global__ void __maxnreg__(168) attention_bf16_kernel(const AttnKernelArgs a) {
   const int nrow = min(AT_MAX_WARPS * 16, a.rows - row0);
   const int per_rank = (nrow + S - 1) / S;
   const int r_lo = min(nrow, rank * per_rank), r_hi = min(nrow, r_lo + per_rank);
-  // weights w_s = l_s 2^(m_s - M) / sum_s(...): one thread per (row, split)
-  for (int it = tid; it < (r_hi - r_lo) * S; it += nthr) {
-    const int rl = r_lo + it / S, sp = it % S;
-    float M = NEG_INF;
-    for (int q = 0; q < S; ++q) {
-      const float* rml = cluster.map_shared_rank(ml, q);
-      if (rml[2 * rl + 1] > 0.f) M = fmaxf(M, rml[2 * rl]);
+  // weights w_s = l_s 2^(m_s - M) / sum_s(...): one thread per (row, split);
+  // S is a power of two <= 16, so a row's S threads are adjacent lanes of one warp.
+  const int n_items = (r_hi - r_lo) * S;
+  for (int base = 0; base < n_items; base += nthr) {
+    const int it = base + tid;
+    const bool act = it < n_items;
+    const int rl = r_lo + (act ? it / S : 0), sp = it % S;
+    float m = NEG_INF, l = 0.f;
+    if (act) {
+      const float* rml = cluster.map_shared_rank(ml, sp);
+      m = rml[2 * rl];
+      l = rml[2 * rl + 1];
     }
-    float den = 0.f, mine = 0.f;
-    for (int q = 0; q < S; ++q) {
-      const float* rml = cluster.map_shared_rank(ml, q);
-      const float l = rml[2 * rl + 1];
-      const float w = l > 0.f ? l * exp2f(rml[2 * rl] - M) : 0.f;
-      den += w;
-      if (q == sp) mine = w;
-    }
-    wsm[rl * AT_MAX_SPLITS + sp] = den > 0.f ? mine / den : 0.f;
+    float M = l > 0.f ? m : NEG_INF;
+    for (int o = 1; o < S; o <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    const float w = l > 0.f ? l * exp2f(m - M) : 0.f;
+    float den = w;
+    for (int o = 1; o < S; o <<= 1) den += __shfl_xor_sync(0xffffffffu, den, o);
+    if (act) wsm[rl * AT_MAX_SPLITS + sp] = den > 0.f ? w / den : 0.f;
   }
   __syncthreads();
   constexpr int D4 = D / 4;
   for (int it = tid; it < (r_hi - r_lo) * D4; it += nthr) {
     const int rl = r_lo + it / D4, d = (it % D4) * 4;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 4
-    for (int sp = 0; sp < S; ++sp) {
-      const float w = wsm[rl * AT_MAX_SPLITS + sp];
-      const float4 v = *reinterpret_cast<const float4*>(cluster.map_shared_rank(part, sp) + rl * D + d);
-      acc.x = fmaf(w, v.x, acc.x);
-      acc.y = fmaf(w, v.y, acc.y);
-      acc.z = fmaf(w, v.z, acc.z);
-      acc.w = fmaf(w, v.w, acc.w);
+#pragma unroll
+    for (int sp = 0; sp < AT_MAX_SPLITS; ++sp) {
+      if (sp < S) {
+        const float w = wsm[rl * AT_MAX_SPLITS + sp];
+        const float4 v =
+            *reinterpret_cast<const float4*>(cluster.map_shared_rank(part, sp) + rl * D + d);
+        acc.x = fmaf(w, v.x, acc.x);
+        acc.y = fmaf(w, v.y, acc.y);
+        acc.z = fmaf(w, v.z, acc.z);
+        acc.w = fmaf(w, v.w, acc.w);
+      }
     }
     uint2 pk;
     pk.x = pack_bf16(acc.x, acc.y);
@@ -460,7 +465,9 @@ AttnPlan attn_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms, bool b
   int s = (2 * num_sms + base - 1) / base;          // about two CTAs per SM
   const int max_useful = (Cmax + 2 * AT_KT - 1) / (2 * AT_KT);  // >= 128 keys per split
   s = std::max(1, std::min(s, std::min(max_useful, std::min(max_cluster, AT_MAX_SPLITS))));
-  p.splits = s;
+  int pow2 = 1;  // the merge groups a row's splits inside one warp: power of two
+  while (pow2 * 2 <= s) pow2 *= 2;
+  p.splits = pow2;
   return p;
 }
 

@@ -8,10 +8,10 @@
 // logit is ever written to memory.  Swap-AB orientation: the vocab is the MMA
 // M dimension (128 TMEM lanes), the few hidden rows are N (16..256 columns).
 //
-// The vocab is split across the CTAs of a chunk in units of 16 rows, so every
-// CTA streams the same number of weight bytes to within one unit.  Full tiles
-// arrive as one 128-row TMA box; a CTA's last, partial tile as 16-row boxes
-// (its missing rows are never loaded and their accumulator lanes are masked).
+// The vocab is split across the CTAs of a chunk in units of `unit_rows` rows
+// (a multiple of 16, at most 128).  Full tiles arrive as one 128-row TMA box;
+// a partial tile as 16-row boxes (its missing rows are never loaded and their
+// accumulator lanes are masked).
 //
 // Persistent CTA per SM, warp-specialised:
 //   warp 0      TMA producer: W tile [128 x 64] + hsel tile [N x 64] per stage
@@ -39,7 +39,9 @@ constexpr uint32_t HT_A_BYTES = HT_BM * HT_BK * 2;  // 16 KB
 constexpr uint32_t HT_BOX_BYTES = HT_WBOX * HT_BK * 2;  // 2 KB
 
 struct HeadTcParams {
-  int V, n_kb, N, Pcp, Pc, P, units, slots, stages, gamma;  // units = ceil(V / 16)
+  int V, n_kb, N, Pcp, Pc, P, slots, stages, gamma;
+  int unit_rows;  // the vocab is split across CTAs in multiples of this (16..128)
+  int units;      // ceil(V / unit_rows)
   uint32_t tmem_cols;
   float alpha;
   const int32_t* drafts;
@@ -63,6 +65,14 @@ int head_tc_max_stages(int N, size_t smem_limit) {
   if (smem_limit <= ht_fixed_bytes()) return 0;
   const int s = static_cast<int>((smem_limit - ht_fixed_bytes()) / per);
   return s > 12 ? 12 : s;
+}
+
+// Pipeline depth: about 144 KB of tiles in flight per SM streams the weight at
+// full HBM bandwidth (measured on GB300: 8 stages of 18 KB beat both 6 and 11).
+int head_tc_stages(int N, size_t smem_limit) {
+  const int per = static_cast<int>(HT_A_BYTES) + N * 128;
+  const int want = (144 * 1024 + per - 1) / per;
+  return std::max(2, std::min(head_tc_max_stages(N, smem_limit), std::max(4, want)));
 }
 
 // Wait used while draining after an abort: ignores the abort flag.
@@ -105,9 +115,9 @@ __global__ void __launch_bounds__(HT_THREADS, 1)
   const int pair0 = chunk * p.Pc;
   const int npairs = min(p.Pc, p.P - pair0);
   // vocab rows [v_lo, v_hi) of this CTA, in tiles of 128 rows
-  const int v_lo = HT_WBOX * static_cast<int>(static_cast<long long>(slot_id) * p.units / p.slots);
-  const int v_hi = min(p.V, HT_WBOX * static_cast<int>(static_cast<long long>(slot_id + 1) *
-                                                        p.units / p.slots));
+  const int v_lo = p.unit_rows * static_cast<int>(static_cast<long long>(slot_id) * p.units / p.slots);
+  const int v_hi = min(p.V, p.unit_rows * static_cast<int>(static_cast<long long>(slot_id + 1) *
+                                                            p.units / p.slots));
   const int t0 = 0;
   const int t1 = v_hi > v_lo ? (v_hi - v_lo + HT_BM - 1) / HT_BM : 0;
 
@@ -280,7 +290,8 @@ cudaError_t launch_head_tc(const HeadArgs& a, const HeadPlan& pl, const HeadTcLa
   p.Pcp = pl.pad_pairs;
   p.Pc = pl.pairs_per_chunk;
   p.P = pl.P;
-  p.units = (a.V + HT_WBOX - 1) / HT_WBOX;
+  p.unit_rows = l.unit_rows;
+  p.units = (a.V + l.unit_rows - 1) / l.unit_rows;
   p.slots = pl.slots;
   p.stages = l.stages;
   p.gamma = a.gamma;

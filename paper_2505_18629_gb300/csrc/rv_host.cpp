@@ -112,9 +112,8 @@ HeadPlan head_plan(int B, int gamma, int V, int num_sms, bool tc) {
   p.pad_pairs = (p.pairs_per_chunk + 7) / 8 * 8;
   p.N = 2 * p.pad_pairs;
   p.n_vtiles = (V + 127) / 128;
-  if (tc) {  // one persistent CTA per SM; the vocab is split in 16-row units
-    const int units = (V + 15) / 16;
-    p.slots = std::max(1, std::min(num_sms / p.n_chunks, units));
+  if (tc) {  // one persistent CTA per SM; the vocab is split in whole tiles
+    p.slots = std::max(1, std::min(num_sms / p.n_chunks, p.n_vtiles));
   } else {
     p.slots = std::max(1, std::min(4 * num_sms / p.n_chunks, p.n_vtiles));
   }
@@ -407,10 +406,11 @@ int encode_maps(rv_handle* h, const void* w, const HeadPlan& pl, HeadTcLaunch& l
   l.tm_w16 = h->tm_w16;
   l.tm_h = h->tm_h;
   if (h->head_tc_stages_cached_N != pl.N) {
-    h->head_tc_stages = head_tc_max_stages(pl.N, h->smem_optin);
+    h->head_tc_stages = head_tc_stages(pl.N, h->smem_optin);
     h->head_tc_stages_cached_N = pl.N;
   }
   l.stages = h->head_tc_stages;
+  l.unit_rows = HEAD_TILE_ROWS;  // whole tiles: one TMA box per stage
   if (l.stages < 2) return fail(h, RV_ERR_UNSUPPORTED, "not enough shared memory for the head pipeline");
   l.smem_bytes = head_tc_smem_bytes(pl.N, l.stages);
   return RV_OK;

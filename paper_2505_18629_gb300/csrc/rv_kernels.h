@@ -97,10 +97,12 @@ struct HeadTcLaunch {
   CUtensorMap tm_w16;  // W [V, H] bf16, box {64, 16}, 128B swizzle
   CUtensorMap tm_h;    // hsel [n_chunks*N, H] bf16, box {64, N}, 128B swizzle
   int stages;
+  int unit_rows;       // vocab split granularity across CTAs (multiple of 16, <= 128)
   size_t smem_bytes;
 };
 size_t head_tc_smem_bytes(int N, int stages);
 int head_tc_max_stages(int N, size_t smem_limit);
+int head_tc_stages(int N, size_t smem_limit);  // the depth the launcher uses
 cudaError_t head_tc_configure(size_t smem_bytes);  // cudaFuncSetAttribute
 cudaError_t launch_head_tc(const HeadArgs& a, const HeadPlan& p, const HeadTcLaunch& l,
                            cudaStream_t s);

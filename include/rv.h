@@ -208,6 +208,32 @@ RV_API int rv_verify_step_host(rv_handle* h, const void* q_host, const void* k_b
                                int32_t* ctx_out_host, uint64_t* h2d_bytes, uint64_t* d2h_bytes,
                                void* stream);
 
+/* ---- allocation-free LM head ------------------------------------------------
+ * The paper has no counterpart: this entry point exists for callers that may
+ * not allocate device memory (code running where cudaMalloc is unavailable or
+ * forbidden, e.g. inside host callbacks, under an allocator that owns the whole
+ * device, or in plug-ins whose host forbids extra allocations).  It computes
+ * exactly what rv_verify_head computes, without a handle and without
+ * allocating: its scratch is one fixed file-scope device array of about
+ * 2.6 MB that every GPU loading this library keeps until the process exits.
+ *   hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin:
+ *           as in rv_verify_head (bf16 only); vocab / hidden_size give V, H.
+ *   dev_status: optional device word; the RV_DEV_* bits of this call are
+ *           OR-ed into it (NULL: they go to the shared array and are lost).
+ * Limits: B * (gamma + 1) <= RV_STATIC_MAX_PAIRS and hidden_size <=
+ * RV_STATIC_MAX_HIDDEN, else RV_ERR_CAPACITY before anything is launched.
+ * The first call on a device (make it before any stream capture) looks up the
+ * array's device address and configures the kernel; later calls only launch.
+ * All calls share the array: calls that may run at the same time on the GPU
+ * (unordered streams) race; order them on one stream. */
+#define RV_STATIC_MAX_PAIRS 64
+#define RV_STATIC_MAX_HIDDEN 8192
+RV_API int rv_verify_head_static(const void* hidden, const void* w_head,
+                                 const int32_t* draft_ids, int32_t B, int32_t gamma, int32_t R,
+                                 int32_t vocab, int32_t hidden_size, float alpha, float* scores,
+                                 int32_t* argmax, float* margin, uint32_t* dev_status,
+                                 void* stream);
+
 /* Synchronize `stream`, read the device status word (RV_DEV_* bits) into
  * *status and clear it.  Returns RV_ERR_DEVICE if any bit was set. */
 RV_API int rv_read_status(rv_handle* h, void* stream, uint32_t* status);

@@ -74,6 +74,7 @@ def _load():
                                P, P, P, P, P]),
         "rv_verify_step_host": (I, [P, P, P, P, P, P, P, P, P, P, P, P, I, I, I, I, F, P, P, P, P,
                                     P, P, P, P, P, P, U64P, U64P, P]),
+        "rv_verify_head_static": (I, [P, P, P, I, I, I, I, I, F, P, P, P, P, P]),
         "rv_read_status": (I, [P, P, ctypes.POINTER(ctypes.c_uint32)]),
         "rv_profile_enable": (I, [P, I]),
         "rv_profile_read": (I, [P, I, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(I)]),
@@ -227,6 +228,23 @@ def rv_verify_step_host(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, dr
         _ptr(scores), _ptr(argmax), _ptr(margin), _ptr(accept_mask), _ptr(accepted_len),
         _ptr(next_token), _ptr(ctx_out), ctypes.byref(hb), ctypes.byref(db), _stream(stream)))
     return hb.value, db.value
+
+
+RV_STATIC_MAX_PAIRS = 64
+RV_STATIC_MAX_HIDDEN = 8192
+
+
+def rv_verify_head_static(hidden, w_head, draft_ids, gamma, R, alpha, scores, argmax, margin,
+                          dev_status=None, stream=None):
+    """rv_verify_head without a handle or any device allocation (fixed internal
+    scratch; limits RV_STATIC_MAX_PAIRS / RV_STATIC_MAX_HIDDEN)."""
+    B = hidden.shape[0]
+    V, H = w_head.shape
+    rc = _lib.rv_verify_head_static(_ptr(hidden), _ptr(w_head), _ptr(draft_ids), B, gamma, R, V,
+                                    H, float(alpha), _ptr(scores), _ptr(argmax), _ptr(margin),
+                                    _ptr(dev_status), _stream(stream))
+    if rc != RV_OK:
+        raise RVError(rc, "rv_verify_head_static")
 
 
 def rv_read_status(h, stream=None) -> int:

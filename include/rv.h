@@ -170,10 +170,13 @@ RV_API int rv_accept(rv_handle* h, const int32_t* draft_ids, const int32_t* argm
                      int32_t* next_token, const int32_t* ctx_in, int32_t* ctx_out, void* stream);
 
 /* The whole verify step on device buffers, in one call and four kernel
- * launches on `stream`: attention (rv_verify_attention), then one launch that
- * gathers the LM-head rows and packs the block (rv_pack_block; skipped when
- * block_ids is NULL), the LM head, and one launch that merges the head's
- * statistics and runs the acceptance (rv_accept).  Arguments as in those
+ * launches: the attention (rv_verify_attention) on an internal stream forked
+ * from `stream`, concurrently with -- on `stream` -- one launch that gathers
+ * the LM-head rows and packs the block (rv_pack_block; skipped when block_ids
+ * is NULL), the LM head, and one launch that merges the head's statistics and
+ * runs the acceptance (rv_accept).  The internal stream is joined back into
+ * `stream` before the call returns, so later work on `stream` sees every
+ * output; the pattern is also valid inside stream capture.  Arguments as in those
  * calls; the template is n_prompt prompt ids + n_prefix prefix ids, so
  * R = n_prompt + n_prefix and Lb = 2*gamma + R.  ctx_out may alias ctx_in. */
 RV_API int rv_verify_step(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,

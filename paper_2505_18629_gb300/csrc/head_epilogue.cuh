@@ -5,8 +5,9 @@
 // lane.  For each pair (original row, reflective row) the lane has o = o_i[v]
 // and r = o'_i[v]; it forms the fused logit z = (1-alpha) o + alpha r (Eq. 2)
 // and the warp reduces, across its 32 rows, the max and sum-exp of o, r and z
-// and the argmax of z over v != x_i.  The lane that owns the pair (pair % 32)
-// folds the tile's result into the warp's running statistics in shared memory.
+// and the argmax of z over v != x_i.  Lane j of the warp folds the tile result
+// of the j-th pair of a group of eight into the warp's running statistics in
+// shared memory.
 // The lane whose row equals the draft x_i stores o, r, z at x_i (unique writer).
 #pragma once
 
@@ -17,10 +18,14 @@
 
 namespace rv {
 
+// Shared-memory statistics tables use a stride of 9 floats per pair: eight
+// lanes updating consecutive pairs then hit different banks.
+constexpr int HEAD_STAT_STRIDE = HEAD_STAT_FIELDS + 1;
+
 __device__ __forceinline__ void head_stats_init(float* stats, int n_entries, int tid,
                                                 int nthreads) {
   for (int e = tid; e < n_entries; e += nthreads) {
-    float* s = stats + e * HEAD_STAT_FIELDS;
+    float* s = stats + e * HEAD_STAT_STRIDE;
     s[ST_M_O] = NEG_INF;
     s[ST_S_O] = 0.f;
     s[ST_M_R] = NEG_INF;
@@ -33,60 +38,108 @@ __device__ __forceinline__ void head_stats_init(float* stats, int n_entries, int
 }
 
 // Eight pairs g8..g8+7 of one tile.  o[j], r[j]: this lane's logits of pair
-// g8+j at vocab row v.  `warp_stats` points at this warp's [128][FIELDS] table;
-// `gathered` at the chunk's first pair.
+// g8+j at vocab row v (pairs at or beyond `npairs` are padding: computed, never
+// stored).  The eight pairs' warp reductions run interleaved so that their
+// shuffle chains overlap.  `warp_stats` points at this warp's [pairs][FIELDS]
+// table; `gathered` at the chunk's first pair.
 __device__ __forceinline__ void head_tile_pairs8(const float (&o)[8], const float (&r)[8], int g8,
                                                  int npairs, int v, bool valid, float alpha,
                                                  const int* s_drafts, float* warp_stats,
                                                  float* gathered, int lane) {
   const float beta = 1.f - alpha;
+  float ov[8], rv[8], zv[8], Mo[8], Mr[8], Mz[8], bv[8];
+  int bi[8];
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
     const int pj = g8 + j;
-    if (pj >= npairs) break;  // uniform across the warp
     const int x = s_drafts[pj];
-    const float ov = valid ? o[j] : NEG_INF;
-    const float rv = valid ? r[j] : NEG_INF;
-    const float zv = valid ? fmaf(alpha, r[j], beta * o[j]) : NEG_INF;
-    if (valid && v == x) {
+    ov[j] = valid ? o[j] : NEG_INF;
+    rv[j] = valid ? r[j] : NEG_INF;
+    zv[j] = valid ? fmaf(alpha, r[j], beta * o[j]) : NEG_INF;
+    if (valid && v == x && pj < npairs) {
       float* gx = gathered + pj * GATHER_FIELDS;
-      gx[0] = ov;
-      gx[1] = rv;
-      gx[2] = zv;
+      gx[0] = ov[j];
+      gx[1] = rv[j];
+      gx[2] = zv[j];
     }
-    float bv = (v == x) ? NEG_INF : zv;
-    int bi = (bv == NEG_INF) ? INT_MAX : v;
-    const float Mo = warp_max(ov);
-    const float Mr = warp_max(rv);
-    const float Mz = warp_max(zv);
-    const float So = warp_sum(exp_shifted(ov, Mo));
-    const float Sr = warp_sum(exp_shifted(rv, Mr));
-    const float Sz = warp_sum(exp_shifted(zv, Mz));
-    warp_argmax(bv, bi);
-    if (lane == (pj & 31)) {
-      float* s = warp_stats + pj * HEAD_STAT_FIELDS;
-      lse_merge(s[ST_M_O], s[ST_S_O], Mo, So);
-      lse_merge(s[ST_M_R], s[ST_S_R], Mr, Sr);
-      lse_merge(s[ST_M_Z], s[ST_S_Z], Mz, Sz);
-      const int si = __float_as_int(s[ST_BEST_I]);
-      if (bv > s[ST_BEST_V] || (bv == s[ST_BEST_V] && bi < si)) {
-        s[ST_BEST_V] = bv;
-        s[ST_BEST_I] = __int_as_float(bi);
+    bv[j] = (v == x) ? NEG_INF : zv[j];
+    bi[j] = (bv[j] == NEG_INF) ? INT_MAX : v;
+    Mo[j] = ov[j];
+    Mr[j] = rv[j];
+    Mz[j] = zv[j];
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      Mo[j] = fmaxf(Mo[j], __shfl_xor_sync(0xffffffffu, Mo[j], off));
+      Mr[j] = fmaxf(Mr[j], __shfl_xor_sync(0xffffffffu, Mr[j], off));
+      Mz[j] = fmaxf(Mz[j], __shfl_xor_sync(0xffffffffu, Mz[j], off));
+    }
+  }
+  float So[8], Sr[8], Sz[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    So[j] = exp_shifted(ov[j], Mo[j]);
+    Sr[j] = exp_shifted(rv[j], Mr[j]);
+    Sz[j] = exp_shifted(zv[j], Mz[j]);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      So[j] += __shfl_xor_sync(0xffffffffu, So[j], off);
+      Sr[j] += __shfl_xor_sync(0xffffffffu, Sr[j], off);
+      Sz[j] += __shfl_xor_sync(0xffffffffu, Sz[j], off);
+      const float ov2 = __shfl_xor_sync(0xffffffffu, bv[j], off);
+      const int oi2 = __shfl_xor_sync(0xffffffffu, bi[j], off);
+      if (ov2 > bv[j] || (ov2 == bv[j] && oi2 < bi[j])) {
+        bv[j] = ov2;
+        bi[j] = oi2;
       }
+    }
+  }
+  // Every lane now holds the tile results of all eight pairs; lane j < 8
+  // folds pair g8+j into the running statistics (one SIMT pass, no divergence
+  // between the pairs).
+  float cMo = Mo[0], cSo = So[0], cMr = Mr[0], cSr = Sr[0], cMz = Mz[0], cSz = Sz[0], cbv = bv[0];
+  int cbi = bi[0];
+#pragma unroll
+  for (int j = 1; j < 8; ++j) {
+    const bool me = lane == j;
+    cMo = me ? Mo[j] : cMo;
+    cSo = me ? So[j] : cSo;
+    cMr = me ? Mr[j] : cMr;
+    cSr = me ? Sr[j] : cSr;
+    cMz = me ? Mz[j] : cMz;
+    cSz = me ? Sz[j] : cSz;
+    cbv = me ? bv[j] : cbv;
+    cbi = me ? bi[j] : cbi;
+  }
+  const int pj = g8 + lane;
+  if (lane < 8 && pj < npairs) {
+    float* s = warp_stats + pj * HEAD_STAT_STRIDE;
+    lse_merge(s[ST_M_O], s[ST_S_O], cMo, cSo);
+    lse_merge(s[ST_M_R], s[ST_S_R], cMr, cSr);
+    lse_merge(s[ST_M_Z], s[ST_S_Z], cMz, cSz);
+    const int si = __float_as_int(s[ST_BEST_I]);
+    if (cbv > s[ST_BEST_V] || (cbv == s[ST_BEST_V] && cbi < si)) {
+      s[ST_BEST_V] = cbv;
+      s[ST_BEST_I] = __int_as_float(cbi);
     }
   }
 }
 
-// Combine the warps' tables into one partial per pair and store it.
-// `out` points at partials[slot][chunk's first pair].
-__device__ __forceinline__ void head_stats_finish(const float* stats, int nwarps, int npairs,
-                                                  float* out, int tid, int nthreads) {
+// Combine the warps' tables (each `tab` pairs long) into one partial per pair
+// and store it.  `out` points at partials[slot][chunk's first pair].
+__device__ __forceinline__ void head_stats_finish(const float* stats, int nwarps, int tab,
+                                                  int npairs, float* out, int tid, int nthreads) {
   for (int pj = tid; pj < npairs; pj += nthreads) {
     float mo = NEG_INF, so = 0.f, mr = NEG_INF, sr = 0.f, mz = NEG_INF, sz = 0.f;
     float bv = NEG_INF;
     int bi = INT_MAX;
     for (int w = 0; w < nwarps; ++w) {
-      const float* s = stats + (w * MAX_PAIRS_PER_CHUNK + pj) * HEAD_STAT_FIELDS;
+      const float* s = stats + (w * tab + pj) * HEAD_STAT_STRIDE;
       lse_merge(mo, so, s[ST_M_O], s[ST_S_O]);
       lse_merge(mr, sr, s[ST_M_R], s[ST_S_R]);
       lse_merge(mz, sz, s[ST_M_Z], s[ST_S_Z]);

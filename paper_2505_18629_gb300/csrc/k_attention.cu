@@ -5,7 +5,7 @@
 //
 // bf16 path: split-KV flash-decoding.  One CTA per (key split, KV head,
 // sequence, row group) stages its keys/values through shared memory in tiles
-// of 64 with 16-byte cp.async loads (double buffered, XOR-swizzled rows) and
+// of 32 with 16-byte cp.async loads (a ring of three, XOR-swizzled rows) and
 // runs QK^T and PV on the tensor cores (mma.sync m16n8k16 bf16, fp32
 // accumulate).  All G*Lb query rows that share a KV head live in one CTA
 // (16 rows per warp), so each key/value byte is read once per head.  The
@@ -30,7 +30,8 @@ namespace rv {
 
 namespace cg = cooperative_groups;
 
-constexpr int AT_KT = 64;         // keys per shared-memory tile
+constexpr int AT_KT = 32;         // keys per shared-memory tile
+constexpr int AT_STAGES = 3;      // K/V tiles in flight (cp.async ring)
 constexpr int AT_MAX_WARPS = 8;   // 16 query rows per warp -> 128 rows per CTA
 constexpr int AT_MAX_SPLITS = 16; // cluster size limit (non-portable above 8)
 
@@ -45,8 +46,9 @@ __device__ __forceinline__ void cp_async_commit() {
 __device__ __forceinline__ void cp_async_wait_all() {
   asm volatile("cp.async.wait_group 0;" ::: "memory");
 }
-__device__ __forceinline__ void cp_async_wait_1() {
-  asm volatile("cp.async.wait_group 1;" ::: "memory");
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
@@ -100,9 +102,10 @@ template <int D>
 __global__ void __maxnreg__(168) attention_bf16_kernel(const AttnKernelArgs a) {
   constexpr int CH = D / 8;            // 16-byte chunks per row
   constexpr int TILE_BYTES = AT_KT * D * 2;
-  constexpr int Q_BYTES = AT_MAX_WARPS * 16 * D * 2;
+  const int WROWS = static_cast<int>(blockDim.x / 32) * 16;  // query rows of this CTA
+  const int Q_BYTES = WROWS * D * 2;
   extern __shared__ __align__(128) uint8_t smem[];
-  // [Q: 128 rows][K buf 0][V buf 0][K buf 1][V buf 1][merge weights]
+  // [Q: WROWS rows][K/V ring: AT_STAGES x (K tile, V tile)][merge weights]
   // After the key loop the Q region holds (m, l) per row and the K/V region
   // the fp32 partial O/l of every row (read by the other CTAs of the cluster).
   const uint32_t s_base = smem_u32(smem);
@@ -128,6 +131,8 @@ __global__ void __maxnreg__(168) attention_bf16_kernel(const AttnKernelArgs a) {
   const int k_hi = min(T, k_lo + per);
 
   const int row0 = rg * AT_MAX_WARPS * 16;  // first query row of this CTA (within the KV head)
+  // (a row group spans up to 128 rows; a CTA with fewer warps only exists when
+  // there is a single row group, whose rows then all fit its warps)
   // Rows of this thread: r_a = row0 + warp*16 + g, r_b = r_a + 8.  Row r <-> (j = r / G, h = kvh*G + r % G).
   const int r_a = row0 + warp * 16 + g, r_b = r_a + 8;
   const bool va = r_a < a.rows, vb = r_b < a.rows;
@@ -135,7 +140,7 @@ __global__ void __maxnreg__(168) attention_bf16_kernel(const AttnKernelArgs a) {
   const int lim_b = vb ? ctx + r_b / a.G : -1;
 
   // ---- Q rows -> shared memory (group 0)
-  for (int e = tid; e < AT_MAX_WARPS * 16 * CH; e += nthr) {
+  for (int e = tid; e < WROWS * CH; e += nthr) {
     const int r = e / CH, c = e % CH;
     const int rr = row0 + r;
     const bool ok = rr < a.rows;
@@ -167,12 +172,14 @@ __global__ void __maxnreg__(168) attention_bf16_kernel(const AttnKernelArgs a) {
     }
   };
 
-  // Two tiles in flight from the start (groups 1 and 2; empty groups are fine).
+  // AT_STAGES tiles in flight from the start (one commit group each; empty
+  // groups are fine).
   const int n_tiles = (k_hi - k_lo + AT_KT - 1) / AT_KT;
-  if (n_tiles > 0) load_kv(k_lo, 0);
-  cp_async_commit();
-  if (n_tiles > 1) load_kv(k_lo + AT_KT, 1);
-  cp_async_commit();
+#pragma unroll
+  for (int t = 0; t < AT_STAGES; ++t) {
+    if (t < n_tiles) load_kv(k_lo + t * AT_KT, t);
+    cp_async_commit();
+  }
 
   // Append the block's keys/values (positions ctx..ctx+Lb-1) once per (b, kvh).
   if (split == 0 && rg == 0) {
@@ -191,8 +198,8 @@ __global__ void __maxnreg__(168) attention_bf16_kernel(const AttnKernelArgs a) {
   float m_a = NEG_INF, m_b = NEG_INF, l_a = 0.f, l_b = 0.f;
 
   for (int it = 0; it < n_tiles; ++it) {
-    const int buf = it & 1;
-    cp_async_wait_1();  // all but the newest group: Q and tile `it` have landed
+    const int buf = it % AT_STAGES;
+    cp_async_wait<AT_STAGES - 1>();  // Q and tile `it` have landed
     __syncthreads();
     const uint32_t sk = s_kv + buf * 2 * TILE_BYTES, sv = sk + TILE_BYTES;
     const int kbase = k_lo + it * AT_KT;
@@ -276,7 +283,7 @@ __global__ void __maxnreg__(168) attention_bf16_kernel(const AttnKernelArgs a) {
       }
     }
     __syncthreads();  // every warp is done with buffer `buf`
-    if (it + 2 < n_tiles) load_kv(k_lo + (it + 2) * AT_KT, buf);
+    if (it + AT_STAGES < n_tiles) load_kv(k_lo + (it + AT_STAGES) * AT_KT, buf);
     cp_async_commit();
   }
   cp_async_wait_all();
@@ -307,9 +314,13 @@ __global__ void __maxnreg__(168) attention_bf16_kernel(const AttnKernelArgs a) {
 
   // ---- split-KV merge through distributed shared memory
   __syncthreads();  // all warps done with Q and the K/V buffers
-  float* const part = reinterpret_cast<float*>(smem + Q_BYTES);    // [128][D]
-  float* const ml = reinterpret_cast<float*>(smem);                // [128][2]
-  float* const wsm = reinterpret_cast<float*>(smem + Q_BYTES + 4 * TILE_BYTES);  // [128][16]
+  // After the key loop: the fp32 partial O/l [WROWS][D] overwrites Q and the
+  // K/V ring (WROWS*D*4 <= WROWS*D*2 + ring bytes for WROWS <= 128), the merge
+  // weights [WROWS][16] and (m, l) [WROWS][2] follow the ring.
+  static_assert(AT_MAX_WARPS * 16 <= 2 * AT_STAGES * AT_KT, "merge buffer exceeds Q + ring");
+  float* const part = reinterpret_cast<float*>(smem);
+  float* const wsm = reinterpret_cast<float*>(smem + Q_BYTES + 2 * AT_STAGES * TILE_BYTES);
+  float* const ml = wsm + WROWS * AT_MAX_SPLITS;
   const int la = warp * 16 + g, lbr = la + 8;  // rows within the CTA window
 #pragma unroll
   for (int dt = 0; dt < D / 8; ++dt) {
@@ -327,7 +338,7 @@ __global__ void __maxnreg__(168) attention_bf16_kernel(const AttnKernelArgs a) {
   cluster.sync();
   const int S = a.splits;
   const int rank = static_cast<int>(cluster.block_rank());
-  const int nrow = min(AT_MAX_WARPS * 16, a.rows - row0);
+  const int nrow = min(WROWS, a.rows - row0);
   const int per_rank = (nrow + S - 1) / S;
   const int r_lo = min(nrow, rank * per_rank), r_hi = min(nrow, r_lo + per_rank);
   // weights w_s = l_s 2^(m_s - M) / sum_s(...): one thread per (row, split);
@@ -471,16 +482,21 @@ AttnPlan attn_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms, bool b
   return p;
 }
 
-size_t attn_bf16_smem_bytes(int D) {
-  return static_cast<size_t>(AT_MAX_WARPS) * 16 * D * 2 + 4 * static_cast<size_t>(AT_KT) * D * 2 +
-         static_cast<size_t>(AT_MAX_WARPS) * 16 * AT_MAX_SPLITS * 4;
+// Q rows + the K/V ring + merge weights + (m, l).  The fp32 partial [rows][D]
+// of the merge reuses the Q and K/V space (rows*D*4 <= Q + ring).
+size_t attn_bf16_smem_bytes(int D, int warps) {
+  return static_cast<size_t>(warps) * 16 * D * 2 + 2 * AT_STAGES * static_cast<size_t>(AT_KT) * D * 2 +
+         static_cast<size_t>(warps) * 16 * (AT_MAX_SPLITS + 2) * 4;
 }
 
 template <int D>
 static cudaError_t attn_configure_d() {
   auto k = attention_bf16_kernel<D>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(attn_bf16_smem_bytes(D)));
+                                       static_cast<int>(attn_bf16_smem_bytes(D, AT_MAX_WARPS)));
+  if (e == cudaSuccess)  // share SMs with the concurrently running LM head
+    e = cudaFuncSetAttribute(k, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             cudaSharedmemCarveoutMaxShared);
   if (e != cudaSuccess) return e;
   return cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
 }
@@ -491,7 +507,7 @@ static int max_cluster_for(int D) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(cs, 1, 1);
     cfg.blockDim = dim3(AT_MAX_WARPS * 32, 1, 1);
-    cfg.dynamicSmemBytes = attn_bf16_smem_bytes(D);
+    cfg.dynamicSmemBytes = attn_bf16_smem_bytes(D, AT_MAX_WARPS);
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = cs;
@@ -538,7 +554,7 @@ cudaError_t launch_attention_bf16(const AttnArgs& x, const AttnPlan& p, cudaStre
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.splits, x.Hkv, x.B * p.row_groups);
   cfg.blockDim = dim3(p.warps * 32, 1, 1);
-  cfg.dynamicSmemBytes = attn_bf16_smem_bytes(x.D);
+  cfg.dynamicSmemBytes = attn_bf16_smem_bytes(x.D, p.warps);
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;

@@ -29,7 +29,7 @@ __global__ void __launch_bounds__(HS_BM) head_simt_kernel(const HeadSimtParams p
   __shared__ float ws[HS_BM][HS_BK + 1];
   __shared__ float hs[16][HS_BK];
   __shared__ int s_drafts[MAX_PAIRS_PER_CHUNK];
-  __shared__ float stats[4 * MAX_PAIRS_PER_CHUNK * HEAD_STAT_FIELDS];
+  __shared__ float stats[4 * MAX_PAIRS_PER_CHUNK * HEAD_STAT_STRIDE];
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int slot_id = blockIdx.x, chunk = blockIdx.y;
@@ -43,7 +43,7 @@ __global__ void __launch_bounds__(HS_BM) head_simt_kernel(const HeadSimtParams p
   head_stats_init(stats, 4 * MAX_PAIRS_PER_CHUNK, tid, HS_BM);
   __syncthreads();
 
-  float* const wstats = stats + warp * MAX_PAIRS_PER_CHUNK * HEAD_STAT_FIELDS;
+  float* const wstats = stats + warp * MAX_PAIRS_PER_CHUNK * HEAD_STAT_STRIDE;
   float* const gathered = p.gathered + static_cast<long long>(pair0) * GATHER_FIELDS;
 
   for (int t = t0; t < t1; ++t) {
@@ -86,7 +86,7 @@ __global__ void __launch_bounds__(HS_BM) head_simt_kernel(const HeadSimtParams p
     }
   }
   __syncthreads();
-  head_stats_finish(stats, 4, npairs,
+  head_stats_finish(stats, 4, MAX_PAIRS_PER_CHUNK, npairs,
                     p.partials + (static_cast<long long>(slot_id) * p.P + pair0) * HEAD_STAT_FIELDS,
                     tid, HS_BM);
 }

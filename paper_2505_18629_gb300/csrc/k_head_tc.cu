@@ -8,18 +8,26 @@
 // logit is ever written to memory.  Swap-AB orientation: the vocab is the MMA
 // M dimension (128 TMEM lanes), the few hidden rows are N (16..256 columns).
 //
-// The vocab is split across the CTAs of a chunk in units of `unit_rows` rows
-// (a multiple of 16, at most 128).  Full tiles arrive as one 128-row TMA box;
-// a partial tile as 16-row boxes (its missing rows are never loaded and their
-// accumulator lanes are masked).
+// Vocab tiles of 128 rows: with one pair chunk the producer warp claims them
+// from a shared counter (dynamic: a CTA slowed by other work on its SM takes
+// fewer), and passes each tile to the MMA and epilogue warps through a small
+// mbarrier-guarded ring.  With several chunks each CTA takes a static range
+// (units of `unit_rows` rows) so the chunk CTAs of a cluster stay in step.
+// Full tiles arrive as one 128-row TMA box; a partial tile as 16-row boxes
+// (its missing rows are never loaded and their accumulator lanes are masked).
 //
 // Persistent CTA per SM, warp-specialised:
 //   warp 0      TMA producer: W tile [128 x 64] + hsel tile [N x 64] per stage
 //               into a ring of `stages` 128B-swizzled shared-memory buffers
 //   warp 1      allocates TMEM (2 accumulator slots of N columns) and issues
 //               tcgen05.mma (M=128, N, K=16) from one thread
-//   warps 2..5  epilogue: tcgen05.ld of the finished accumulator slot, fusion,
-//               warp-shuffle max/sum/argmax, running statistics in shared memory
+//   warps 2..    epilogue (4 warps, or 8 above 32 pairs per chunk): tcgen05.ld of
+//               the finished accumulator slot, fusion, warp-shuffle
+//               max/sum/argmax, running statistics in shared memory; with 8,
+//               the two warps of a lane quadrant take alternate groups of 8 pairs
+// When the pairs need several chunks, the chunk CTAs of one vocab range form a
+// cluster: they stream the same weight tiles together, so the second read of
+// each tile is served by L2.
 // The weight streams from HBM exactly once per step (evict-first); the small
 // hidden operand is re-read from L2 per tile (evict-last).
 #include <cfloat>
@@ -32,14 +40,20 @@ namespace rv {
 
 constexpr int HT_BM = HEAD_TILE_ROWS;
 constexpr int HT_BK = 64;
-constexpr int HT_THREADS = 192;
-constexpr int HT_EPI_WARPS = 4;
+// Epilogue warps: 4 (one per TMEM lane quadrant) for up to 32 pairs per chunk,
+// else 8 (two per quadrant, taking alternate groups of 8 pairs).
+constexpr int HT_SMALL_PAIRS = 32;
+__host__ __device__ constexpr int ht_threads(int epi_warps) { return 64 + epi_warps * 32; }
 constexpr int HT_WBOX = HEAD_W_BOX_ROWS;             // vocab rows per TMA box of W
 constexpr uint32_t HT_A_BYTES = HT_BM * HT_BK * 2;  // 16 KB
 constexpr uint32_t HT_BOX_BYTES = HT_WBOX * HT_BK * 2;  // 2 KB
 
+constexpr int HT_TRING = 4;  // tile-index ring between the producer and the consumers
+
 struct HeadTcParams {
   int V, n_kb, N, Pcp, Pc, P, slots, stages, gamma;
+  int n_vtiles;              // ceil(V / 128): tiles handed out by the counter
+  unsigned* tile_counter;    // one chunk: shared tile counter (zeroed before launch); else null
   int unit_rows;  // the vocab is split across CTAs in multiples of this (16..128)
   int units;      // ceil(V / unit_rows)
   uint32_t tmem_cols;
@@ -50,28 +64,31 @@ struct HeadTcParams {
   unsigned* status;
 };
 
-static size_t ht_fixed_bytes() {
-  // alignment slack + barriers/misc + drafts + per-warp statistics
+static int ht_epi_warps(int N) { return N / 2 <= HT_SMALL_PAIRS ? 4 : 8; }
+
+static size_t ht_fixed_bytes(int N) {
+  // alignment slack + barriers/tile ring/misc + drafts + per-warp statistics (Pcp = N/2 pairs)
   return 1024 + 512 + MAX_PAIRS_PER_CHUNK * 4 +
-         HT_EPI_WARPS * MAX_PAIRS_PER_CHUNK * HEAD_STAT_FIELDS * 4;
+         static_cast<size_t>(ht_epi_warps(N)) * (N / 2) * HEAD_STAT_STRIDE * 4;
 }
 
 size_t head_tc_smem_bytes(int N, int stages) {
-  return ht_fixed_bytes() + static_cast<size_t>(stages) * (HT_A_BYTES + N * 128);
+  return ht_fixed_bytes(N) + static_cast<size_t>(stages) * (HT_A_BYTES + N * 128);
 }
 
 int head_tc_max_stages(int N, size_t smem_limit) {
   const size_t per = HT_A_BYTES + N * 128;
-  if (smem_limit <= ht_fixed_bytes()) return 0;
-  const int s = static_cast<int>((smem_limit - ht_fixed_bytes()) / per);
+  if (smem_limit <= ht_fixed_bytes(N)) return 0;
+  const int s = static_cast<int>((smem_limit - ht_fixed_bytes(N)) / per);
   return s > 12 ? 12 : s;
 }
 
-// Pipeline depth: about 144 KB of tiles in flight per SM streams the weight at
-// full HBM bandwidth (measured on GB300: 8 stages of 18 KB beat both 6 and 11).
+// Pipeline depth: about 128 KB of tiles in flight per SM streams the weight at
+// full HBM bandwidth (measured on GB300: 7-8 stages of 18 KB beat both 4-6 and
+// 11) and leaves room on the SM for the concurrent attention kernel.
 int head_tc_stages(int N, size_t smem_limit) {
   const int per = static_cast<int>(HT_A_BYTES) + N * 128;
-  const int want = (144 * 1024 + per - 1) / per;
+  const int want = (128 * 1024 + per - 1) / per;
   return std::max(2, std::min(head_tc_max_stages(N, smem_limit), std::max(4, want)));
 }
 
@@ -83,7 +100,8 @@ __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
   }
 }
 
-__global__ void __launch_bounds__(HT_THREADS, 1)
+template <int EPI>
+__global__ void __launch_bounds__(ht_threads(EPI), 1)
     head_tc_kernel(const __grid_constant__ CUtensorMap tm_w,
                    const __grid_constant__ CUtensorMap tm_w16,
                    const __grid_constant__ CUtensorMap tm_h, const HeadTcParams p) {
@@ -106,20 +124,23 @@ __global__ void __launch_bounds__(HT_THREADS, 1)
   const uint32_t accf0 = bars + 8u * (2 * S);
   const uint32_t acce0 = accf0 + 16u;
   const uint32_t drain_bar = acce0 + 16u;
-  const uint32_t misc = (drain_bar + 8u + 15u) & ~15u;
+  const uint32_t tfull0 = drain_bar + 8u;            // tile ring: HT_TRING full barriers
+  const uint32_t tempty0 = tfull0 + 8u * HT_TRING;   //            and HT_TRING empty barriers
+  const uint32_t misc = (tempty0 + 8u * HT_TRING + 15u) & ~15u;
   uint32_t* const tmem_slot = reinterpret_cast<uint32_t*>(gbase + (misc - base));
   volatile int* const abort_flag = reinterpret_cast<volatile int*>(gbase + (misc - base) + 4);
-  int* const s_drafts = reinterpret_cast<int*>(gbase + (misc - base) + 16);
-  float* const stats = reinterpret_cast<float*>(gbase + (misc - base) + 16 + MAX_PAIRS_PER_CHUNK * 4);
+  int2* const tring = reinterpret_cast<int2*>(gbase + (misc - base) + 16);  // (v0, v_end) or v0 < 0
+  int* const s_drafts = reinterpret_cast<int*>(gbase + (misc - base) + 16 + 8 * HT_TRING);
+  float* const stats =
+      reinterpret_cast<float*>(gbase + (misc - base) + 16 + 8 * HT_TRING + MAX_PAIRS_PER_CHUNK * 4);
+  const int tab = p.Pcp;  // pairs per statistics table
 
   const int pair0 = chunk * p.Pc;
   const int npairs = min(p.Pc, p.P - pair0);
-  // vocab rows [v_lo, v_hi) of this CTA, in tiles of 128 rows
+  // Static split (several chunks): vocab rows [v_lo, v_hi) of this CTA.
   const int v_lo = p.unit_rows * static_cast<int>(static_cast<long long>(slot_id) * p.units / p.slots);
   const int v_hi = min(p.V, p.unit_rows * static_cast<int>(static_cast<long long>(slot_id + 1) *
                                                             p.units / p.slots));
-  const int t0 = 0;
-  const int t1 = v_hi > v_lo ? (v_hi - v_lo + HT_BM - 1) / HT_BM : 0;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -128,9 +149,13 @@ __global__ void __launch_bounds__(HT_THREADS, 1)
     }
     mbar_init(accf0, 1);
     mbar_init(accf0 + 8, 1);
-    mbar_init(acce0, HT_EPI_WARPS);
-    mbar_init(acce0 + 8, HT_EPI_WARPS);
+    mbar_init(acce0, EPI);
+    mbar_init(acce0 + 8, EPI);
     mbar_init(drain_bar, 1);
+    for (int k = 0; k < HT_TRING; ++k) {
+      mbar_init(tfull0 + 8u * k, 1);
+      mbar_init(tempty0 + 8u * k, 1 + EPI);  // the MMA thread + one lane per epilogue warp
+    }
     *abort_flag = 0;
     fence_barrier_init();
   }
@@ -142,9 +167,9 @@ __global__ void __launch_bounds__(HT_THREADS, 1)
   if (warp == 1) tmem_alloc(smem_u32(tmem_slot), p.tmem_cols);
   if (warp >= 2) {
     const int e = threadIdx.x - 64;
-    for (int j = e; j < MAX_PAIRS_PER_CHUNK; j += 128)
+    for (int j = e; j < MAX_PAIRS_PER_CHUNK; j += EPI * 32)
       s_drafts[j] = (j < npairs) ? pair_draft(p.drafts, pair0 + j, p.gamma) : -1;
-    head_stats_init(stats, HT_EPI_WARPS * MAX_PAIRS_PER_CHUNK, e, 128);
+    head_stats_init(stats, EPI * tab, e, EPI * 32);
   }
   tc_fence_before();
   __syncthreads();
@@ -159,9 +184,29 @@ __global__ void __launch_bounds__(HT_THREADS, 1)
       int s = 0, issued = 0;
       uint32_t ph = 0;
       bool ok = true;
-      for (int t = t0; t < t1 && ok; ++t) {
-        const int v0 = v_lo + t * HT_BM;
-        const int rows = min(HT_BM, v_hi - v0);
+      // Tile source: the shared counter (one chunk: CTAs slowed by other work
+      // on their SM simply take fewer tiles) or this CTA's static range.
+      int t_next = p.tile_counter ? static_cast<int>(atomicAdd(p.tile_counter, 1u)) : 0;
+      for (int lt = 0; ok; ++lt) {
+        int v0, v_end;
+        if (p.tile_counter) {
+          const int t = t_next;
+          v0 = t < p.n_vtiles ? t * HT_BM : -1;
+          v_end = v0 >= 0 ? min(p.V, v0 + HT_BM) : 0;
+          if (v0 >= 0) t_next = static_cast<int>(atomicAdd(p.tile_counter, 1u));
+        } else {
+          v0 = v_lo + lt * HT_BM < v_hi ? v_lo + lt * HT_BM : -1;
+          v_end = v0 >= 0 ? min(v_hi, v0 + HT_BM) : 0;
+        }
+        const int k = lt % HT_TRING;
+        if (!mbar_wait(tempty0 + 8u * k, ((lt / HT_TRING) & 1) ^ 1u, abort_flag, p.status)) {
+          ok = false;
+          break;
+        }
+        tring[k] = make_int2(v0, v_end);
+        mbar_arrive(tfull0 + 8u * k);
+        if (v0 < 0) break;
+        const int rows = v_end - v0;
         const int nbox = rows == HT_BM ? 0 : (rows + HT_WBOX - 1) / HT_WBOX;  // 0: one full box
         const uint32_t a_bytes = nbox == 0 ? HT_A_BYTES : nbox * HT_BOX_BYTES;
         for (int kb = 0; kb < p.n_kb; ++kb) {
@@ -196,7 +241,12 @@ __global__ void __launch_bounds__(HT_THREADS, 1)
       int s = 0;
       uint32_t ph = 0;
       bool ok = true;
-      for (int t = t0, lt = 0; t < t1 && ok; ++t, ++lt) {
+      for (int lt = 0; ok; ++lt) {
+        const int k = lt % HT_TRING;
+        if (!mbar_wait(tfull0 + 8u * k, (lt / HT_TRING) & 1, abort_flag, p.status)) break;
+        const int v0 = tring[k].x;
+        mbar_arrive(tempty0 + 8u * k);
+        if (v0 < 0) break;
         const int slot = lt & 1;
         const uint32_t aph = (lt >> 1) & 1;
         if (!mbar_wait(acce0 + 8u * slot, aph ^ 1u, abort_flag, p.status)) {
@@ -214,8 +264,8 @@ __global__ void __launch_bounds__(HT_THREADS, 1)
           const uint64_t ad = sw128_kmajor_desc(a_tiles + s * HT_A_BYTES);
           const uint64_t bd = sw128_kmajor_desc(b_tiles + s * b_bytes);
 #pragma unroll
-          for (int k = 0; k < HT_BK / 16; ++k)
-            tc_mma_bf16(d_tmem, ad + 2u * k, bd + 2u * k, idesc, (kb | k) != 0 ? 1u : 0u);
+          for (int kk = 0; kk < HT_BK / 16; ++kk)
+            tc_mma_bf16(d_tmem, ad + 2u * kk, bd + 2u * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
           tc_commit(empty_bar(s));
           if (++s == S) {
             s = 0;
@@ -233,19 +283,27 @@ __global__ void __launch_bounds__(HT_THREADS, 1)
     // ------------------------------------------------------------ epilogue
     const int q = warp & 3;       // TMEM lane quadrant this warp may access
     const int ew = warp - 2;      // statistics table of this warp
-    float* const wstats = stats + ew * MAX_PAIRS_PER_CHUNK * HEAD_STAT_FIELDS;
+    const int half = ew >> 2;     // which alternate groups of 8 pairs it takes
+    float* const wstats = stats + ew * tab * HEAD_STAT_STRIDE;
     float* const gathered = p.gathered + static_cast<long long>(pair0) * GATHER_FIELDS;
-    for (int t = t0, lt = 0; t < t1; ++t, ++lt) {
+    for (int lt = 0;; ++lt) {
+      const int k = lt % HT_TRING;
+      bool ok = mbar_wait(tfull0 + 8u * k, (lt / HT_TRING) & 1, abort_flag, p.status);
+      if (!__all_sync(0xffffffffu, ok)) break;
+      const int2 tile = tring[k];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(tempty0 + 8u * k);
+      if (tile.x < 0) break;
       const int slot = lt & 1;
       const uint32_t aph = (lt >> 1) & 1;
-      bool ok = mbar_wait(accf0 + 8u * slot, aph, abort_flag, p.status);
+      ok = mbar_wait(accf0 + 8u * slot, aph, abort_flag, p.status);
       if (!__all_sync(0xffffffffu, ok)) break;
       tc_fence_after();
-      const int v = v_lo + t * HT_BM + q * 32 + lane;
-      const bool valid = v < v_hi;
+      const int v = tile.x + q * 32 + lane;
+      const bool valid = v < tile.y;
       const uint32_t trow =
           tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(slot * p.N);
-      for (int g8 = 0; g8 < npairs; g8 += 8) {
+      for (int g8 = 8 * half; g8 < npairs; g8 += 8 * (EPI / 4)) {
         float o[8], r[8];
         tmem_ld8(trow + g8, o);
         tmem_ld8(trow + p.Pcp + g8, r);
@@ -256,10 +314,10 @@ __global__ void __launch_bounds__(HT_THREADS, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(acce0 + 8u * slot);
     }
-    named_bar_sync(1, 128);
-    head_stats_finish(stats, HT_EPI_WARPS, npairs,
+    named_bar_sync(1, EPI * 32);
+    head_stats_finish(stats, EPI, tab, npairs,
                       p.partials + (static_cast<long long>(slot_id) * p.P + pair0) * HEAD_STAT_FIELDS,
-                      threadIdx.x - 64, 128);
+                      threadIdx.x - 64, EPI * 32);
   }
 
   tc_fence_before();
@@ -270,9 +328,22 @@ __global__ void __launch_bounds__(HT_THREADS, 1)
   }
 }
 
+// The maximum shared-memory carveout lets the attention kernel's CTAs share an
+// SM with this kernel's (the SM is otherwise configured just large enough for
+// whichever kernel arrives first).
+template <int EPI>
+static cudaError_t head_tc_configure_one(size_t smem_bytes) {
+  cudaError_t e = cudaFuncSetAttribute(head_tc_kernel<EPI>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem_bytes));
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(head_tc_kernel<EPI>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                              cudaSharedmemCarveoutMaxShared);
+}
+
 cudaError_t head_tc_configure(size_t smem_bytes) {
-  return cudaFuncSetAttribute(head_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(smem_bytes));
+  cudaError_t e = head_tc_configure_one<4>(smem_bytes);
+  return e != cudaSuccess ? e : head_tc_configure_one<8>(smem_bytes);
 }
 
 static uint32_t tmem_cols_for(int N) {
@@ -292,6 +363,8 @@ cudaError_t launch_head_tc(const HeadArgs& a, const HeadPlan& pl, const HeadTcLa
   p.P = pl.P;
   p.unit_rows = l.unit_rows;
   p.units = (a.V + l.unit_rows - 1) / l.unit_rows;
+  p.n_vtiles = (a.V + HT_BM - 1) / HT_BM;
+  p.tile_counter = pl.n_chunks == 1 ? a.tile_counter : nullptr;
   p.slots = pl.slots;
   p.stages = l.stages;
   p.gamma = a.gamma;
@@ -301,9 +374,21 @@ cudaError_t launch_head_tc(const HeadArgs& a, const HeadPlan& pl, const HeadTcLa
   p.partials = a.partials;
   p.gathered = a.gathered;
   p.status = a.status;
-  dim3 grid(pl.slots, pl.n_chunks);
-  head_tc_kernel<<<grid, HT_THREADS, l.smem_bytes, s>>>(l.tm_w, l.tm_w16, l.tm_h, p);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(pl.slots, pl.n_chunks, 1);
+  const int epi = ht_epi_warps(pl.N);
+  cfg.blockDim = dim3(ht_threads(epi), 1, 1);
+  cfg.dynamicSmemBytes = l.smem_bytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 1;
+  attr[0].val.clusterDim.y = pl.n_chunks;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = (pl.n_chunks >= 2 && pl.n_chunks <= 8) ? 1 : 0;
+  if (epi == 4) return cudaLaunchKernelEx(&cfg, head_tc_kernel<4>, l.tm_w, l.tm_w16, l.tm_h, p);
+  return cudaLaunchKernelEx(&cfg, head_tc_kernel<8>, l.tm_w, l.tm_w16, l.tm_h, p);
 }
 
 }  // namespace rv

@@ -55,8 +55,9 @@ cudaError_t launch_pack_block(const int32_t* drafts, const int32_t* prompt, cons
 // block is to be packed too, the first B*Lb threads of the grid also do that.
 __global__ void prep_kernel(const uint4* __restrict__ hidden, uint4* __restrict__ hsel, int P,
                             int gamma, int R, int Lh, int Hv, int Pc, int Pcp, int N, int n_chunks,
-                            const PackArgs pk) {
+                            const PackArgs pk, unsigned* tile_counter) {
   const long long tid0 = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x;
+  if (tid0 == 0 && tile_counter) *tile_counter = 0u;  // the LM head that follows claims tiles from 0
   if (pk.block != nullptr) {
     const int Lb = 2 * pk.gamma + pk.n_prompt + pk.n_prefix;
     for (long long idx = tid0; idx < static_cast<long long>(pk.B) * Lb;
@@ -105,12 +106,14 @@ cudaError_t launch_prep(const HeadArgs& a, const HeadPlan& p, void* hsel, const 
   const int Hv = a.H / 8;  // 8 bf16 per 16-byte vector
   const int Lh = 2 * a.gamma + a.R + 1;
   if (hsel) work = std::max(work, static_cast<long long>(p.n_chunks) * p.N * Hv);
+  if (a.tile_counter) work = std::max(work, 1LL);
   if (work == 0) return cudaSuccess;
   const int threads = 256;
   const int blocks = static_cast<int>(std::min<long long>((work + threads - 1) / threads, 4096));
   prep_kernel<<<blocks, threads, 0, s>>>(static_cast<const uint4*>(a.hidden),
                                          static_cast<uint4*>(hsel), p.P, a.gamma, a.R, Lh, Hv,
-                                         p.pairs_per_chunk, p.pad_pairs, p.N, p.n_chunks, pk);
+                                         p.pairs_per_chunk, p.pad_pairs, p.N, p.n_chunks, pk,
+                                         a.tile_counter);
   return cudaGetLastError();
 }
 

@@ -75,6 +75,10 @@ struct rv_handle {
   int tm_h_N = -1;
   int tm_h_rows = -1;
   CUtensorMap tm_h;
+  // rv_verify_step runs the attention on this stream, concurrently with the
+  // LM head on the caller's stream (fork / join through the two events).
+  cudaStream_t side = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   bool profiling = false;
   ProfRegion prof[RV_PROF_COUNT];
   unsigned long long launches = 0;
@@ -264,6 +268,9 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
   h->ws.st_acc_len = reinterpret_cast<int32_t*>(b + o_al);
   h->ws.st_next = reinterpret_cast<int32_t*>(b + o_nt);
   e = cudaMemset(h->ws.base, 0, off);
+  if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming);
   if (e == cudaSuccess && bf16) e = attn_configure(&h->attn_max_cluster);
   if (e == cudaSuccess && bf16) e = head_tc_configure(h->smem_optin);
   if (e == cudaSuccess && bf16) {
@@ -274,6 +281,9 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
     h->encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
   }
   if (e != cudaSuccess) {
+    if (h->ev_join) cudaEventDestroy(h->ev_join);
+    if (h->ev_fork) cudaEventDestroy(h->ev_fork);
+    if (h->side) cudaStreamDestroy(h->side);
     cudaFree(h->ws.base);
     delete h;
     return fail(nullptr, RV_ERR_CUDA, "rv_create setup: %s", cudaGetErrorString(e));
@@ -287,6 +297,9 @@ extern "C" RV_API int rv_destroy(rv_handle* h) {
   cudaDeviceSynchronize();
   for (auto& r : h->prof)
     for (auto ev : r.ev) cudaEventDestroy(ev);
+  cudaEventDestroy(h->ev_join);
+  cudaEventDestroy(h->ev_fork);
+  cudaStreamDestroy(h->side);
   cudaFree(h->ws.base);
   delete h;
   return RV_OK;
@@ -439,7 +452,8 @@ int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_
   const rv_config& c = h->cfg;
   const bool bf16 = c.dtype == RV_DTYPE_BF16;
   HeadArgs a{hidden, w_head, draft_ids, B, gamma, R, c.vocab, c.hidden, alpha,
-             h->ws.head_partials, h->ws.gathered, h->ws.status};
+             h->ws.head_partials, h->ws.gathered, h->ws.status,
+             bf16 ? h->ws.status + 16 : nullptr};  // tile counter: its own 64-byte line
   const HeadPlan pl = head_plan(B, gamma, c.vocab, h->num_sms, bf16);
   ProfScope prof_all(h, RV_PROF_HEAD, s);
   cudaError_t e = cudaSuccess;
@@ -525,14 +539,24 @@ extern "C" RV_API int rv_verify_step(
   if (do_pack && (!pos_ids || (n_prompt > 0 && !prompt_ids) || (n_prefix > 0 && !prefix_ids)))
     return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument for the block packing");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // Fork: the attention (independent of the LM head) runs on the side stream
+  // and shares the SMs with the HBM-bound head; join before returning.
+  cudaError_t e = cudaEventRecord(h->ev_fork, s);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(h->side, h->ev_fork, 0);
+  if (e != cudaSuccess) return cuda_fail(h, e, "stream fork");
   rc = rv_verify_attention(h, q, k_blk, v_blk, k_cache, v_cache, ctx_in, B, 2 * gamma + R,
-                           attn_out, stream);
-  if (rc != RV_OK) return rc;
-  PackArgs pk{draft_ids, prompt_ids, prefix_ids, ctx_in, B, gamma, n_prompt, n_prefix, block_ids,
-              pos_ids};
-  AcceptArgs ac{accept_mask, accepted_len, next_token, ctx_in, ctx_out};
-  return head_impl(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin,
+                           attn_out, h->side);
+  if (rc == RV_OK) {
+    PackArgs pk{draft_ids, prompt_ids, prefix_ids, ctx_in, B, gamma, n_prompt, n_prefix, block_ids,
+                pos_ids};
+    AcceptArgs ac{accept_mask, accepted_len, next_token, ctx_in, ctx_out};
+    rc = head_impl(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin,
                    do_pack ? &pk : nullptr, &ac, s);
+  }
+  e = cudaEventRecord(h->ev_join, h->side);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(s, h->ev_join, 0);
+  if (e != cudaSuccess && rc == RV_OK) return cuda_fail(h, e, "stream join");
+  return rc;
 }
 
 extern "C" RV_API int rv_verify_step_host(

@@ -49,6 +49,7 @@ struct HeadArgs {
   float* partials;         // [slots][P][HEAD_STAT_FIELDS]
   float* gathered;         // [P][GATHER_FIELDS]
   unsigned* status;
+  unsigned* tile_counter;  // LM-head tile counter, zeroed by the prep kernel
 };
 
 // ---- small kernels (k_small.cu)
@@ -129,7 +130,7 @@ struct AttnPlan {
 // max_cluster: largest thread-block cluster the attention kernel can use (<= 16)
 AttnPlan attn_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms, bool bf16,
                    int max_cluster);
-size_t attn_bf16_smem_bytes(int D);
+size_t attn_bf16_smem_bytes(int D, int warps);
 cudaError_t attn_configure(int* max_cluster);
 cudaError_t launch_attention_bf16(const AttnArgs& a, const AttnPlan& p, cudaStream_t s);
 cudaError_t launch_attention_f32(const AttnArgs& a, cudaStream_t s);

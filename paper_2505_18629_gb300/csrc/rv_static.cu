@@ -138,12 +138,13 @@ extern "C" RV_API int rv_verify_head_static(const void* hidden, const void* w_he
                                 : reinterpret_cast<unsigned*>(s + ST_OFF_STATUS);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   // The shared array keeps the previous call's contents: the status word must
-  // start at zero.  Partials and gathered rows are fully rewritten each call.
+  // start at zero (the LM head's tile counter is zeroed by the prep launch).
+  // Partials and gathered rows are fully rewritten each call.
   if (!dev_status && cudaMemsetAsync(s + ST_OFF_STATUS, 0, sizeof(unsigned), st) != cudaSuccess)
     return RV_ERR_CUDA;
   HeadArgs a{hidden, w_head, draft_ids, B, gamma, R, vocab, hidden_size, alpha,
              reinterpret_cast<float*>(s + ST_OFF_PART), reinterpret_cast<float*>(s + ST_OFF_GATHER),
-             status};
+             status, reinterpret_cast<unsigned*>(s + ST_OFF_STATUS + 64)};
   HeadTcLaunch l;
   l.stages = head_tc_stages(pl.N, d->smem_optin);
   l.unit_rows = HEAD_TILE_ROWS;

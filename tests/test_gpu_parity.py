@@ -149,13 +149,21 @@ def test_separate_entry_points_match_step(gu):
     rv.rv_accept(h, d, am, acc, al, nt, ctx, co)
     assert rv.rv_read_status(h) == 0
     np.testing.assert_array_equal(gu.to_np(attn), step.attn)
-    np.testing.assert_array_equal(gu.to_np(sc), step.scores)
-    np.testing.assert_array_equal(gu.to_np(am), step.argmax)
+    # The LM head claims vocab tiles dynamically, so the order in which the
+    # per-CTA statistics merge (and their fp32 rounding) varies run to run.
+    _same_decisions(gu, gu.to_np(sc), gu.to_np(am), gu.to_np(mg), step)
     np.testing.assert_array_equal(gu.to_np(acc), step.accept_mask)
     np.testing.assert_array_equal(gu.to_np(al), step.accepted_len)
     np.testing.assert_array_equal(gu.to_np(nt), step.next_token)
     np.testing.assert_array_equal(gu.to_np(co), step.ctx_out)
     h.close()
+
+
+def _same_decisions(gu, scores, argmax, margin, step, atol=1e-4):
+    np.testing.assert_allclose(scores, step.scores, atol=atol, rtol=0)
+    np.testing.assert_allclose(margin, step.margin, atol=atol, rtol=0)
+    clear = np.concatenate([step.margin, np.full((step.margin.shape[0], 1), np.inf)], 1) > atol
+    assert ((argmax == step.argmax) | ~clear).all()
 
 
 def test_host_buffer_step_matches_device_step(gu):
@@ -187,7 +195,7 @@ def test_host_buffer_step_matches_device_step(gu):
     assert h2d > 0 and d2h > 0
     np.testing.assert_array_equal(outs["blk"].numpy(), step.block_ids)
     np.testing.assert_array_equal(outs["attn"].view(torch.int16).numpy().view(np.uint16), step.attn)
-    np.testing.assert_array_equal(outs["sc"].numpy(), step.scores)
+    _same_decisions(gu, outs["sc"].numpy(), outs["am"].numpy(), outs["mg"].numpy(), step)
     np.testing.assert_array_equal(outs["al"].numpy(), step.accepted_len)
     np.testing.assert_array_equal(outs["nt"].numpy(), step.next_token)
     h.close()

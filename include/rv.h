@@ -242,16 +242,19 @@ RV_API int rv_verify_head_static(const void* hidden, const void* w_head,
 RV_API int rv_read_status(rv_handle* h, void* stream, uint32_t* status);
 
 /* ---- kernel timing (CUDA events recorded by the library itself) ---------- */
-#define RV_PROF_ATTENTION 0   /* attention kernels of rv_verify_attention */
-#define RV_PROF_HEAD_GEMM 1   /* the LM-head GEMM + online log-softmax kernel */
-#define RV_PROF_HEAD 2        /* everything rv_verify_head launches */
+#define RV_PROF_ATTENTION 0   /* attention kernel of rv_verify_attention */
+#define RV_PROF_HEAD_GEMM 1   /* the LM-head GEMM + online log-softmax kernel alone */
+#define RV_PROF_HEAD 2        /* everything rv_verify_head launches (gather + LM head [+ merge]) */
 #define RV_PROF_ACCEPT 3      /* rv_accept (inside rv_verify_step it is part of RV_PROF_HEAD) */
 #define RV_PROF_COUNT 4
 
-/* enable != 0: from now on, record a CUDA event pair on the launching stream
- * around each profiled region (up to 4096 per region, then recording stops).
- * Not for use inside graph capture. */
-RV_API int rv_profile_enable(rv_handle* h, int32_t enable);
+/* mask: bit (1 << region) set = from now on, record a CUDA event pair on the
+ * launching stream around each such region (up to 1024 per region, then
+ * recording stops); 0 stops recording.  An event pair around RV_PROF_HEAD_GEMM
+ * sits between the row-gather launch and the LM-head launch and so disables
+ * their overlap (programmatic dependent launch); RV_PROF_HEAD brackets both
+ * without that cost.  Not for use inside graph capture. */
+RV_API int rv_profile_enable(rv_handle* h, int32_t mask);
 /* Synchronize the recorded events and return the summed duration (ms) and
  * number of recorded launches of `region`; then forget them. */
 RV_API int rv_profile_read(rv_handle* h, int32_t region, double* total_ms, int32_t* count);

@@ -162,6 +162,105 @@ __device__ __forceinline__ void head_stats_finish(const float* stats, int nwarps
   }
 }
 
+// Merge the slots' partial statistics of every pair and finish the
+// per-position outputs (one warp per pair), then, if asked, the exact-match
+// acceptance of every sequence (Alg. 2).  Run by every thread of one CTA, the
+// last LM-head CTA to finish; partials are read past L1 (other CTAs wrote
+// them).  Each lane issues the loads of all its slots before merging them, and
+// the choices go through shared memory (`s_choice`, P ints), so the tail costs
+// about one L2 round trip.
+constexpr int MERGE_SLOTS_PER_LANE = 8;
+
+// s_draft[p]: the draft scored by pair p (-1 for none), in shared memory.
+__device__ __forceinline__ void head_merge_all(const float* partials, const float* gathered,
+                                               const int* s_draft, int B, int gamma, int V,
+                                               int P, int slots, const HeadFinal& f,
+                                               unsigned* status, int* s_choice, int tid,
+                                               int nthreads) {
+  const int lane = tid & 31, warp = tid >> 5, nw = nthreads >> 5;
+  const float nan = __int_as_float(0x7fc00000);
+  for (int p = warp; p < P; p += nw) {
+    float mo = NEG_INF, so = 0.f, mr = NEG_INF, sr = 0.f, mz = NEG_INF, sz = 0.f;
+    float bv = NEG_INF;
+    int bi = INT_MAX;
+    for (int g0 = lane; g0 < slots; g0 += 32 * MERGE_SLOTS_PER_LANE) {
+      float4 lo[MERGE_SLOTS_PER_LANE], hi[MERGE_SLOTS_PER_LANE];
+#pragma unroll
+      for (int k = 0; k < MERGE_SLOTS_PER_LANE; ++k) {
+        const int g = g0 + 32 * k;
+        if (g < slots) {
+          const float4* q =
+              reinterpret_cast<const float4*>(partials + (static_cast<long long>(g) * P + p) * HEAD_STAT_FIELDS);
+          lo[k] = __ldcg(q);
+          hi[k] = __ldcg(q + 1);
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < MERGE_SLOTS_PER_LANE; ++k) {
+        if (g0 + 32 * k < slots) {
+          lse_merge(mo, so, lo[k].x, lo[k].y);
+          lse_merge(mr, sr, lo[k].z, lo[k].w);
+          lse_merge(mz, sz, hi[k].x, hi[k].y);
+          const int i = __float_as_int(hi[k].w);
+          if (hi[k].z > bv || (hi[k].z == bv && i < bi)) {
+            bv = hi[k].z;
+            bi = i;
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      lse_merge(mo, so, __shfl_xor_sync(0xffffffffu, mo, o), __shfl_xor_sync(0xffffffffu, so, o));
+      lse_merge(mr, sr, __shfl_xor_sync(0xffffffffu, mr, o), __shfl_xor_sync(0xffffffffu, sr, o));
+      lse_merge(mz, sz, __shfl_xor_sync(0xffffffffu, mz, o), __shfl_xor_sync(0xffffffffu, sz, o));
+    }
+    warp_argmax(bv, bi);
+    if (lane == 0) {
+      const int b = p / (gamma + 1), i = p % (gamma + 1);
+      const float lse_o = mo + logf(so), lse_r = mr + logf(sr), lse_z = mz + logf(sz);
+      float* sc = f.scores + static_cast<long long>(p) * RV_NSCORES;
+      sc[RV_SCORE_LSE_ORIG] = lse_o;
+      sc[RV_SCORE_LSE_REFL] = lse_r;
+      sc[RV_SCORE_LSE_FUSED] = lse_z;
+      int choice = bi;
+      float lp_z = nan, lp_o = nan, lp_r = nan;
+      if (i < gamma) {
+        const int x = s_draft[p];
+        if (x >= 0 && x < V) {
+          const float4 gx = __ldcg(reinterpret_cast<const float4*>(gathered) + p);
+          lp_z = gx.z - lse_z;
+          lp_o = gx.x - lse_o;
+          lp_r = gx.y - lse_r;
+          if (gx.z > bv || (gx.z == bv && x < bi)) choice = x;
+          f.margin[b * gamma + i] = fabsf(gx.z - bv);
+        } else {
+          raise_status(status, RV_DEV_DRAFT_RANGE);
+          f.margin[b * gamma + i] = nan;
+        }
+      }
+      sc[RV_SCORE_LOGP_FUSED] = lp_z;
+      sc[RV_SCORE_LOGP_ORIG] = lp_o;
+      sc[RV_SCORE_LOGP_REFL] = lp_r;
+      f.argmax[p] = choice;
+      s_choice[p] = choice;
+    }
+  }
+  if (f.acc.accepted_len == nullptr) return;
+  __syncthreads();  // every choice of this CTA is in s_choice
+  for (int b = tid; b < B; b += nthreads) {
+    int n = gamma;
+    for (int i = 0; i < gamma; ++i) {
+      const bool ok = s_draft[b * (gamma + 1) + i] == s_choice[b * (gamma + 1) + i];
+      f.acc.accept_mask[b * gamma + i] = ok ? 1 : 0;
+      if (!ok && n == gamma) n = i;
+    }
+    f.acc.accepted_len[b] = n;
+    f.acc.next_token[b] = s_choice[b * (gamma + 1) + n];
+    f.acc.ctx_out[b] = f.acc.ctx_in[b] + n;
+  }
+}
+
 // Draft id scored by pair `pair` (-1 for the last position of a sequence).
 __device__ __forceinline__ int pair_draft(const int32_t* drafts, int pair, int gamma) {
   const int b = pair / (gamma + 1), i = pair % (gamma + 1);

@@ -35,22 +35,6 @@ constexpr int AT_STAGES = 3;      // K/V tiles in flight (cp.async ring)
 constexpr int AT_MAX_WARPS = 8;   // 16 query rows per warp -> 128 rows per CTA
 constexpr int AT_MAX_SPLITS = 16; // cluster size limit (non-portable above 8)
 
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool pred) {
-  const int n = pred ? 16 : 0;  // zero-fill when the source is out of range
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(n)
-               : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() {
-  asm volatile("cp.async.commit_group;" ::: "memory");
-}
-__device__ __forceinline__ void cp_async_wait_all() {
-  asm volatile("cp.async.wait_group 0;" ::: "memory");
-}
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
                                         uint32_t& r3) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
@@ -73,10 +57,6 @@ __device__ __forceinline__ void mma_bf16_16816(float (&c)[4], const uint32_t (&a
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
-  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-  return *reinterpret_cast<uint32_t*>(&v);
-}
 
 // Byte offset of 16-byte chunk `c` of row `r` in a swizzled tile of rows of D bf16.
 template <int D>
@@ -459,14 +439,31 @@ __global__ void attention_f32_kernel(const float* __restrict__ q, const float* _
 // ---------------------------------------------------------------- planning / launch
 
 AttnPlan attn_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms, bool bf16,
-                   int max_cluster) {
+                   int max_cluster, int D) {
   AttnPlan p;
   const int G = Hq / Hkv;
   p.rows = Lb * G;
+  p.tc = false;
   if (!bf16) {
     p.row_groups = 1;
     p.splits = 1;
     p.warps = 0;
+    return p;
+  }
+  // tcgen05 kernel once there are enough (sequence, KV head) pairs to fill a
+  // quarter of the SMs; below that the step is latency-bound and the small
+  // mma.sync kernel shares the SMs with the LM head instead.
+  if (D == 128 && B * Hkv >= num_sms / 4) {
+    p.tc = true;
+    p.warps = 4;
+    p.row_groups = (p.rows + 127) / 128;
+    const int base = B * Hkv * p.row_groups;
+    int s = (num_sms + base - 1) / base;  // about one CTA per SM
+    const int max_useful = (Cmax + 255) / 256;  // >= 256 keys per split
+    s = std::max(1, std::min(s, std::min(max_useful, std::min(max_cluster, AT_MAX_SPLITS))));
+    int pow2 = 1;
+    while (pow2 * 2 <= s) pow2 *= 2;
+    p.splits = pow2;
     return p;
   }
   p.row_groups = (p.rows + AT_MAX_WARPS * 16 - 1) / (AT_MAX_WARPS * 16);

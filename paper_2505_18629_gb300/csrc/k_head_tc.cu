@@ -54,6 +54,9 @@ struct HeadTcParams {
   int V, n_kb, N, Pcp, Pc, P, slots, stages, gamma;
   int n_vtiles;              // ceil(V / 128): tiles handed out by the counter
   unsigned* tile_counter;    // one chunk: shared tile counter (zeroed before launch); else null
+  unsigned* done_counter;    // finished CTAs, for the fused merge (zeroed before launch)
+  int B, fused;              // fused != 0: the last CTA merges and writes `fin`
+  HeadFinal fin;
   int unit_rows;  // the vocab is split across CTAs in multiples of this (16..128)
   int units;      // ceil(V / unit_rows)
   uint32_t tmem_cols;
@@ -181,6 +184,9 @@ __global__ void __launch_bounds__(ht_threads(EPI), 1)
     if (lane == 0) {
       const uint64_t pol_w = policy_evict_first();
       const uint64_t pol_h = policy_evict_last();
+      // The prep launch before this kernel (programmatic dependent launch)
+      // gathers the hidden rows and zeroes the counters: wait for it here.
+      asm volatile("griddepcontrol.wait;" ::: "memory");
       int s = 0, issued = 0;
       uint32_t ph = 0;
       bool ok = true;
@@ -326,6 +332,22 @@ __global__ void __launch_bounds__(ht_threads(EPI), 1)
     tc_fence_after();
     tmem_dealloc(tmem_base, p.tmem_cols);
   }
+  if (!p.fused) return;
+  // Fused merge: the last CTA to finish (a ticket, no waiting) reads every
+  // CTA's partial statistics and writes the per-position outputs.
+  volatile int* const last = abort_flag + 1;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0)
+    *last = atomicAdd(p.done_counter, 1u) == gridDim.x * gridDim.y - 1 ? 1 : 0;
+  __syncthreads();
+  if (*last) {
+    __threadfence();
+    // the statistics tables are free now: reuse them for the choices
+    head_merge_all(p.partials, p.gathered, s_drafts, p.B, p.gamma, p.V, p.P, p.slots, p.fin,
+                   p.status, reinterpret_cast<int*>(stats), threadIdx.x, blockDim.x);
+    if (threadIdx.x == 0) *p.done_counter = 0u;
+  }
 }
 
 // The maximum shared-memory carveout lets the attention kernel's CTAs share an
@@ -353,7 +375,7 @@ static uint32_t tmem_cols_for(int N) {
 }
 
 cudaError_t launch_head_tc(const HeadArgs& a, const HeadPlan& pl, const HeadTcLaunch& l,
-                           cudaStream_t s) {
+                           const HeadFinal* fin, cudaStream_t s) {
   HeadTcParams p;
   p.V = a.V;
   p.n_kb = (a.H + HT_BK - 1) / HT_BK;
@@ -365,6 +387,10 @@ cudaError_t launch_head_tc(const HeadArgs& a, const HeadPlan& pl, const HeadTcLa
   p.units = (a.V + l.unit_rows - 1) / l.unit_rows;
   p.n_vtiles = (a.V + HT_BM - 1) / HT_BM;
   p.tile_counter = pl.n_chunks == 1 ? a.tile_counter : nullptr;
+  p.done_counter = a.done_counter;
+  p.B = a.B;
+  p.fused = fin != nullptr ? 1 : 0;
+  if (fin) p.fin = *fin;
   p.slots = pl.slots;
   p.stages = l.stages;
   p.gamma = a.gamma;
@@ -380,13 +406,20 @@ cudaError_t launch_head_tc(const HeadArgs& a, const HeadPlan& pl, const HeadTcLa
   cfg.blockDim = dim3(ht_threads(epi), 1, 1);
   cfg.dynamicSmemBytes = l.smem_bytes;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 1;
-  attr[0].val.clusterDim.y = pl.n_chunks;
-  attr[0].val.clusterDim.z = 1;
+  cudaLaunchAttribute attr[2];
+  int na = 0;
+  attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[na].val.programmaticStreamSerializationAllowed = 1;
+  ++na;
+  if (pl.n_chunks >= 2 && pl.n_chunks <= 8) {
+    attr[na].id = cudaLaunchAttributeClusterDimension;
+    attr[na].val.clusterDim.x = 1;
+    attr[na].val.clusterDim.y = pl.n_chunks;
+    attr[na].val.clusterDim.z = 1;
+    ++na;
+  }
   cfg.attrs = attr;
-  cfg.numAttrs = (pl.n_chunks >= 2 && pl.n_chunks <= 8) ? 1 : 0;
+  cfg.numAttrs = na;
   if (epi == 4) return cudaLaunchKernelEx(&cfg, head_tc_kernel<4>, l.tm_w, l.tm_w16, l.tm_h, p);
   return cudaLaunchKernelEx(&cfg, head_tc_kernel<8>, l.tm_w, l.tm_w16, l.tm_h, p);
 }

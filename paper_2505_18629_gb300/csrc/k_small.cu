@@ -55,9 +55,13 @@ cudaError_t launch_pack_block(const int32_t* drafts, const int32_t* prompt, cons
 // block is to be packed too, the first B*Lb threads of the grid also do that.
 __global__ void prep_kernel(const uint4* __restrict__ hidden, uint4* __restrict__ hsel, int P,
                             int gamma, int R, int Lh, int Hv, int Pc, int Pcp, int N, int n_chunks,
-                            const PackArgs pk, unsigned* tile_counter) {
+                            const PackArgs pk, unsigned* tile_counter, unsigned* done_counter) {
+  // The LM-head kernel that follows may start now (programmatic dependent
+  // launch); it waits for this grid before it reads anything written here.
+  asm volatile("griddepcontrol.launch_dependents;");
   const long long tid0 = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x;
   if (tid0 == 0 && tile_counter) *tile_counter = 0u;  // the LM head that follows claims tiles from 0
+  if (tid0 == 0 && done_counter) *done_counter = 0u;
   if (pk.block != nullptr) {
     const int Lb = 2 * pk.gamma + pk.n_prompt + pk.n_prefix;
     for (long long idx = tid0; idx < static_cast<long long>(pk.B) * Lb;
@@ -113,7 +117,7 @@ cudaError_t launch_prep(const HeadArgs& a, const HeadPlan& p, void* hsel, const 
   prep_kernel<<<blocks, threads, 0, s>>>(static_cast<const uint4*>(a.hidden),
                                          static_cast<uint4*>(hsel), p.P, a.gamma, a.R, Lh, Hv,
                                          p.pairs_per_chunk, p.pad_pairs, p.N, p.n_chunks, pk,
-                                         a.tile_counter);
+                                         a.tile_counter, a.done_counter);
   return cudaGetLastError();
 }
 

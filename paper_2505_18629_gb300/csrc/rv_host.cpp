@@ -79,7 +79,7 @@ struct rv_handle {
   // LM head on the caller's stream (fork / join through the two events).
   cudaStream_t side = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
-  bool profiling = false;
+  unsigned profiling = 0;  // bit mask of the regions being recorded
   ProfRegion prof[RV_PROF_COUNT];
   unsigned long long launches = 0;
   int head_tc_stages_cached_N = -1;
@@ -132,7 +132,7 @@ struct ProfScope {
   cudaStream_t s;
   int idx = -1;
   ProfScope(rv_handle* h_, int r, cudaStream_t s_) : h(h_), region(r), s(s_) {
-    if (h->profiling && h->prof[r].used < PROF_PAIRS) {
+    if ((h->profiling & (1u << r)) && h->prof[r].used < PROF_PAIRS) {
       idx = h->prof[r].used++;
       cudaEventRecord(h->prof[r].ev[2 * idx], s);
     }
@@ -272,6 +272,7 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming);
   if (e == cudaSuccess && bf16) e = attn_configure(&h->attn_max_cluster);
+  if (e == cudaSuccess && bf16) e = attn_tc_configure();
   if (e == cudaSuccess && bf16) e = head_tc_configure(h->smem_optin);
   if (e == cudaSuccess && bf16) {
     cudaDriverEntryPointQueryResult q;
@@ -364,8 +365,8 @@ extern "C" RV_API int rv_verify_attention(rv_handle* h, const void* q, const voi
   cudaError_t e;
   if (bf16) {
     const AttnPlan p = attn_plan(B, Lb, c.n_q_heads, c.n_kv_heads, c.max_ctx, h->num_sms, true,
-                                 h->attn_max_cluster);
-    e = launch_attention_bf16(a, p, s);
+                                 h->attn_max_cluster, c.head_dim);
+    e = p.tc ? launch_attention_tc(a, p, s) : launch_attention_bf16(a, p, s);
   } else {
     e = launch_attention_f32(a, s);
   }
@@ -453,7 +454,8 @@ int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_
   const bool bf16 = c.dtype == RV_DTYPE_BF16;
   HeadArgs a{hidden, w_head, draft_ids, B, gamma, R, c.vocab, c.hidden, alpha,
              h->ws.head_partials, h->ws.gathered, h->ws.status,
-             bf16 ? h->ws.status + 16 : nullptr};  // tile counter: its own 64-byte line
+             bf16 ? h->ws.status + 16 : nullptr,    // tile counter: its own 64-byte line
+             bf16 ? h->ws.status + 32 : nullptr};   // finished-CTA counter
   const HeadPlan pl = head_plan(B, gamma, c.vocab, h->num_sms, bf16);
   ProfScope prof_all(h, RV_PROF_HEAD, s);
   cudaError_t e = cudaSuccess;
@@ -467,12 +469,16 @@ int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_
     h->launches += 1;
     if (e != cudaSuccess) return cuda_fail(h, e, "prep launch");
   }
+  // Small pair counts: the head kernel's last CTA finishes the merge itself.
+  const bool fused = bf16 && pl.P <= HEAD_FUSED_FINAL_MAX_PAIRS;
+  HeadFinal fin{scores, argmax, margin, acc ? *acc : AcceptArgs{}};
   {
     ProfScope prof(h, RV_PROF_HEAD_GEMM, s);
-    e = bf16 ? launch_head_tc(a, pl, l, s) : launch_head_simt(a, pl, s);
+    e = bf16 ? launch_head_tc(a, pl, l, fused ? &fin : nullptr, s) : launch_head_simt(a, pl, s);
     h->launches += 1;
   }
   if (e != cudaSuccess) return cuda_fail(h, e, "LM head launch");
+  if (fused) return RV_OK;
   e = launch_head_finalize(a, pl, scores, argmax, margin, acc, s);
   h->launches += 1;
   return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "head finalize launch");
@@ -656,9 +662,9 @@ extern "C" RV_API int rv_read_status(rv_handle* h, void* stream, uint32_t* statu
   return RV_OK;
 }
 
-extern "C" RV_API int rv_profile_enable(rv_handle* h, int32_t enable) {
+extern "C" RV_API int rv_profile_enable(rv_handle* h, int32_t mask) {
   if (!h) return RV_ERR_INVALID_ARG;
-  if (enable) {
+  if (mask) {
     for (auto& r : h->prof) {
       if (r.ev.empty()) {
         r.ev.resize(2 * PROF_PAIRS);
@@ -670,7 +676,7 @@ extern "C" RV_API int rv_profile_enable(rv_handle* h, int32_t enable) {
       r.used = 0;
     }
   }
-  h->profiling = enable != 0;
+  h->profiling = static_cast<unsigned>(mask) & ((1u << RV_PROF_COUNT) - 1u);
   return RV_OK;
 }
 

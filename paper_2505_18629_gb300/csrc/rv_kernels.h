@@ -40,6 +40,26 @@ struct HeadPlan {
   int slots;           // CTAs per chunk (= partial slots)
 };
 
+// Optional acceptance fused into the head merge (rv_verify_step).
+struct AcceptArgs {
+  uint8_t* accept_mask;
+  int32_t* accepted_len;
+  int32_t* next_token;
+  const int32_t* ctx_in;
+  int32_t* ctx_out;
+};
+
+// Outputs of the merge when the LM-head kernel finishes it itself (its last
+// CTA), instead of the separate finalize launch.
+struct HeadFinal {
+  float* scores;
+  int32_t* argmax;
+  float* margin;
+  AcceptArgs acc;  // acc.accepted_len == nullptr: no acceptance
+};
+// Largest pair count whose merge the head kernel's last CTA finishes itself.
+constexpr int HEAD_FUSED_FINAL_MAX_PAIRS = 64;
+
 struct HeadArgs {
   const void* hidden;      // [B, Lb+1, H]
   const void* w;           // [V, H]
@@ -50,6 +70,7 @@ struct HeadArgs {
   float* gathered;         // [P][GATHER_FIELDS]
   unsigned* status;
   unsigned* tile_counter;  // LM-head tile counter, zeroed by the prep kernel
+  unsigned* done_counter;  // finished LM-head CTAs (fused merge), zeroed by the prep kernel
 };
 
 // ---- small kernels (k_small.cu)
@@ -70,14 +91,6 @@ struct PackArgs {
 // also packs the block when `pack` is given (one launch for both).
 cudaError_t launch_prep(const HeadArgs& a, const HeadPlan& p, void* hsel, const PackArgs* pack,
                         cudaStream_t s);
-// Optional acceptance fused into the head merge (rv_verify_step).
-struct AcceptArgs {
-  uint8_t* accept_mask;
-  int32_t* accepted_len;
-  int32_t* next_token;
-  const int32_t* ctx_in;
-  int32_t* ctx_out;
-};
 // Merge the head's per-CTA statistics into scores / argmax / margin, and run
 // the acceptance of each sequence when `acc` is given.
 cudaError_t launch_head_finalize(const HeadArgs& a, const HeadPlan& p, float* scores,
@@ -105,8 +118,11 @@ size_t head_tc_smem_bytes(int N, int stages);
 int head_tc_max_stages(int N, size_t smem_limit);
 int head_tc_stages(int N, size_t smem_limit);  // the depth the launcher uses
 cudaError_t head_tc_configure(size_t smem_bytes);  // cudaFuncSetAttribute
+// fin != nullptr: the kernel's last CTA merges the statistics and writes the
+// outputs (P <= HEAD_FUSED_FINAL_MAX_PAIRS).  The launch uses programmatic
+// dependent launch: it must directly follow the prep launch on `s`.
 cudaError_t launch_head_tc(const HeadArgs& a, const HeadPlan& p, const HeadTcLaunch& l,
-                           cudaStream_t s);
+                           const HeadFinal* fin, cudaStream_t s);
 cudaError_t launch_head_simt(const HeadArgs& a, const HeadPlan& p, cudaStream_t s);
 
 // ---- attention (k_attention.cu)
@@ -125,14 +141,19 @@ struct AttnPlan {
   int rows;        // query rows per KV head: Lb * G
   int row_groups;  // CTAs along the rows (<= 128 rows each)
   int splits;      // key splits
-  int warps;       // warps per CTA
+  int warps;       // warps per CTA (mma.sync kernel)
+  bool tc;         // tcgen05 kernel (head_dim 128, larger batches)
 };
 // max_cluster: largest thread-block cluster the attention kernel can use (<= 16)
 AttnPlan attn_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms, bool bf16,
-                   int max_cluster);
+                   int max_cluster, int D);
 size_t attn_bf16_smem_bytes(int D, int warps);
 cudaError_t attn_configure(int* max_cluster);
 cudaError_t launch_attention_bf16(const AttnArgs& a, const AttnPlan& p, cudaStream_t s);
 cudaError_t launch_attention_f32(const AttnArgs& a, cudaStream_t s);
+// tcgen05 attention (k_attention_tc.cu), head_dim 128
+size_t attn_tc_smem_bytes();
+cudaError_t attn_tc_configure();
+cudaError_t launch_attention_tc(const AttnArgs& a, const AttnPlan& p, cudaStream_t s);
 
 }  // namespace rv

@@ -144,7 +144,8 @@ extern "C" RV_API int rv_verify_head_static(const void* hidden, const void* w_he
     return RV_ERR_CUDA;
   HeadArgs a{hidden, w_head, draft_ids, B, gamma, R, vocab, hidden_size, alpha,
              reinterpret_cast<float*>(s + ST_OFF_PART), reinterpret_cast<float*>(s + ST_OFF_GATHER),
-             status, reinterpret_cast<unsigned*>(s + ST_OFF_STATUS + 64)};
+             status, reinterpret_cast<unsigned*>(s + ST_OFF_STATUS + 64),
+             reinterpret_cast<unsigned*>(s + ST_OFF_STATUS + 128)};
   HeadTcLaunch l;
   l.stages = head_tc_stages(pl.N, d->smem_optin);
   l.unit_rows = HEAD_TILE_ROWS;
@@ -155,7 +156,7 @@ extern "C" RV_API int rv_verify_head_static(const void* hidden, const void* w_he
       !encode_2d(d->encode, &l.tm_h, s + ST_OFF_HSEL, hidden_size, pl.N, 64, pl.N))
     return RV_ERR_CUDA;
   if (launch_prep(a, pl, s + ST_OFF_HSEL, nullptr, st) != cudaSuccess) return RV_ERR_CUDA;
-  if (launch_head_tc(a, pl, l, st) != cudaSuccess) return RV_ERR_CUDA;
+  if (launch_head_tc(a, pl, l, nullptr, st) != cudaSuccess) return RV_ERR_CUDA;
   if (launch_head_finalize(a, pl, scores, argmax, margin, nullptr, st) != cudaSuccess)
     return RV_ERR_CUDA;
   return RV_OK;

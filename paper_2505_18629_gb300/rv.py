@@ -256,8 +256,9 @@ def rv_read_status(h, stream=None) -> int:
     return st.value
 
 
-def rv_profile_enable(h, enable=True):
-    _check(h, _lib.rv_profile_enable(h.ptr, 1 if enable else 0))
+def rv_profile_enable(h, mask):
+    """mask: bit (1 << RV_PROF_*) per region to record; 0 stops."""
+    _check(h, _lib.rv_profile_enable(h.ptr, int(mask)))
 
 
 def rv_profile_read(h, region):

@@ -67,6 +67,17 @@ def test_bf16_gqa8_two_row_groups(gu):
     _check(gu, _wl(Hq=16, Hkv=2, gamma=6, R=8, B=2, seed=44), ctx=[1000, 3])
 
 
+def test_bf16_tcgen05_attention_ragged(gu):
+    # B*Hkv = 40 (sequence, KV head) pairs selects the tcgen05 attention kernel;
+    # ragged contexts, an empty cache, and a context spanning several key tiles
+    _check(gu, _wl(B=20, Hq=8, Hkv=2, gamma=3, R=4, V=600, H=256, ctx=(0, 700), seed=60))
+
+
+def test_bf16_tcgen05_attention_gqa8_two_row_groups(gu):
+    # G=8, Lb=20: 160 query rows per KV head -> two 128-row MMA groups
+    _check(gu, _wl(B=20, Hq=16, Hkv=2, gamma=6, R=8, V=500, H=128, ctx=(1, 300), seed=61))
+
+
 def test_bf16_max_pairs_single_chunk(gu):
     # B*(gamma+1) = 126 pairs -> N = 256 columns, the widest MMA
     _check(gu, _wl(B=14, gamma=8, R=8, V=777, H=256, ctx=(10, 60), seed=45), check_attn=False)

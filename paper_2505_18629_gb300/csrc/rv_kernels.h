@@ -58,7 +58,10 @@ struct HeadFinal {
   AcceptArgs acc;  // acc.accepted_len == nullptr: no acceptance
 };
 // Largest pair count whose merge the head kernel's last CTA finishes itself.
-constexpr int HEAD_FUSED_FINAL_MAX_PAIRS = 64;
+#ifndef RV_HEAD_FUSED_FINAL_MAX_PAIRS
+#define RV_HEAD_FUSED_FINAL_MAX_PAIRS 64
+#endif
+constexpr int HEAD_FUSED_FINAL_MAX_PAIRS = RV_HEAD_FUSED_FINAL_MAX_PAIRS;
 
 struct HeadArgs {
   const void* hidden;      // [B, Lb+1, H]

@@ -438,8 +438,11 @@ __global__ void attention_f32_kernel(const float* __restrict__ q, const float* _
 
 // ---------------------------------------------------------------- planning / launch
 
+#ifndef RV_ATTN_TC_MIN_UNITS
+#define RV_ATTN_TC_MIN_UNITS 0  // (sequence, KV head) pairs that select tcgen05; 0: SMs / 4
+#endif
 AttnPlan attn_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms, bool bf16,
-                   int max_cluster, int D) {
+                   int max_cluster, int D, bool allow_tc) {
   AttnPlan p;
   const int G = Hq / Hkv;
   p.rows = Lb * G;
@@ -450,20 +453,15 @@ AttnPlan attn_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms, bool b
     p.warps = 0;
     return p;
   }
-  // tcgen05 kernel once there are enough (sequence, KV head) pairs to fill a
-  // quarter of the SMs; below that the step is latency-bound and the small
-  // mma.sync kernel shares the SMs with the LM head instead.
-  if (D == 128 && B * Hkv >= num_sms / 4) {
+  // tcgen05 kernel (k_attention_tc.cu) once there are enough (sequence, KV
+  // head) pairs to fill a quarter of the SMs; below that the step is
+  // latency-bound and the small mma.sync kernel shares the SMs with the LM head.
+  if (allow_tc && attn_tc_supported(Hq, Hkv, D) &&
+      B * Hkv >= (RV_ATTN_TC_MIN_UNITS > 0 ? RV_ATTN_TC_MIN_UNITS : num_sms / 4)) {
     p.tc = true;
-    p.warps = 4;
-    p.row_groups = (p.rows + 127) / 128;
-    const int base = B * Hkv * p.row_groups;
-    int s = (num_sms + base - 1) / base;  // about one CTA per SM
-    const int max_useful = (Cmax + 255) / 256;  // >= 256 keys per split
-    s = std::max(1, std::min(s, std::min(max_useful, std::min(max_cluster, AT_MAX_SPLITS))));
-    int pow2 = 1;
-    while (pow2 * 2 <= s) pow2 *= 2;
-    p.splits = pow2;
+    p.row_groups = 0;
+    p.splits = 0;
+    p.warps = 0;
     return p;
   }
   p.row_groups = (p.rows + AT_MAX_WARPS * 16 - 1) / (AT_MAX_WARPS * 16);

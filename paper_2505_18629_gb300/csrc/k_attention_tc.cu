@@ -1,456 +1,739 @@
 // Verify-block attention (Sec. 3.1) on the 5th-generation tensor cores, for
-// head_dim 128 (bf16).  Same decomposition and split-KV cluster merge as the
-// mma.sync kernel in k_attention.cu; the two products run as tcgen05.mma with
-// the accumulators in TMEM:
+// head_dim 128 (bf16): every query row of the packed block attends causally to
+// the cached context and to the block positions up to its own.
 //
-//   S  = Q K^T   M = 128 query rows (the Lb*G rows that share a KV head, zero
-//                padded), N = KT keys, K = 128 (head dim); Q and the K tile are
-//                K-major, 128-byte swizzled (two 64-column halves each)
-//   O += P V     M = 128, N = 128 (head dim), K = KT keys; P (bf16, written by
-//                the softmax) is K-major, V is used as stored ([key][dim]) as an
-//                MN-major operand
+// Work items.  The Lb*G query rows that share a KV head (G = Hq / Hkv) form one
+// MMA tile of M = 128 rows (row groups of 128 when there are more).  The keys
+// of a sequence are cut into chunks of `chunk` cached keys; the block's own
+// keys belong to the last chunk.  An item is (sequence, KV head, row group,
+// chunk); persistent CTAs (at most one per SM) claim items from a counter, so
+// sequences of different lengths balance across the SMs.  An item that covers
+// the whole sequence writes its rows directly; otherwise it writes its
+// normalised partial O with (max, sum), and a second small kernel merges the
+// chunks (one warp per row).
 //
-// Thread t of the 4 warps owns query row t (TMEM lane t): it reads its S row
-// with tcgen05.ld, keeps the row max / sum, writes its P row to shared memory
-// and, when its max rises by more than 2^8, rescales its O row in TMEM.  K/V
-// tiles stream through a cp.async ring (XOR-swizzled into the 128-byte
-// pattern the MMA expects); the block's own keys/values are read from
-// k_blk/v_blk and appended to the cache by split 0.  Every mbarrier wait is
-// bounded.
+// Per CTA, warp-specialised:
+//   warp 0     claims items and loads with TMA: Q of the item (3-D box over
+//              [B*Lb][Hq][D] that selects the G heads of the KV head) into one
+//              of two Q buffers, then per tile of 128 keys the K and V tiles,
+//              from the cache ([B*Hkv*Cmax][D]) or, for the block's keys, from
+//              k_blk / v_blk (3-D box over [B*Lb][Hkv][D]), into a ring of stages
+//   warp 1     allocates TMEM and issues the MMAs from one thread:
+//                S_t  = Q K_t^T   (M 128, N 128, K 128) into S[t % 2]
+//                O   += P_t V_t   (M 128, N 128, K 128); P_t (bf16) is read from
+//                                 TMEM, where the softmax wrote it over the
+//                                 first half of S[t % 2]; V is used as stored,
+//                                 an MN-major operand
+//              QK of tile t+1 is issued before PV of tile t, so the tensor core
+//              computes the next scores while the softmax runs; the MMAs of a
+//              CTA execute in issue order, so QK of tile t+2 overwrites S[t % 2]
+//              only after PV of tile t has read P_t
+//   warps 2-5  one thread per query row (its TMEM lane): online softmax of
+//              S_t (base-2, the 1/sqrt(D) scale folded into the exponent),
+//              lazy rescale of its O row (only when its max rises by more than
+//              2^8), and at the end of the item the O row: output or partial
+// Every wait is bounded (a timeout is reported in the status word).  The CTA
+// that handles the last chunk of (sequence, KV head) in row group 0 appends
+// the block's keys and values to the cache.
 #include <cfloat>
-
-#include <cooperative_groups.h>
 
 #include "rv_device.cuh"
 #include "rv_kernels.h"
 
 namespace rv {
 
-namespace cg = cooperative_groups;
-
 namespace {
 
 constexpr int TC_D = 128;
-constexpr int TC_ROWS = 128;           // MMA M: query rows per CTA
-constexpr int TC_THREADS = 128;        // one thread per row
-constexpr int TC_MAX_SPLITS = 16;
-constexpr int TC_Q_BYTES = TC_ROWS * TC_D * 2;  // 32 KB, two 16 KB halves
-constexpr float TC_RESCALE_LOG2 = 8.f;  // rescale O only when the max rises by > 2^8
+constexpr int TC_M = 128;        // query rows per MMA tile
+constexpr int TC_KT = 128;       // keys per tile
+constexpr int TC_STAGES = 2;     // K/V ring depth
+constexpr int TC_THREADS = 192;  // producer, MMA, 4 softmax warps
+constexpr int TC_IRING = 4;      // item ring between the producer and the consumers
+constexpr float TC_RESCALE_LOG2 = 8.f;
+
+constexpr uint32_t TC_Q_BYTES = TC_M * TC_D * 2;    // 32 KB: two 64-dim halves
+constexpr uint32_t TC_KV_BYTES = TC_KT * TC_D * 2;  // 32 KB: two halves of [128 keys][128 B]
+constexpr uint32_t TC_Q_OFF = 0;
+constexpr uint32_t TC_K_OFF = TC_Q_OFF + 2 * TC_Q_BYTES;
+constexpr uint32_t TC_V_OFF = TC_K_OFF + TC_STAGES * TC_KV_BYTES;
+constexpr uint32_t TC_BAR_OFF = TC_V_OFF + TC_STAGES * TC_KV_BYTES;
+constexpr uint32_t TC_MISC_OFF = TC_BAR_OFF + 256;
+constexpr uint32_t TC_RING_OFF = TC_MISC_OFF + 16;  // TC_IRING items of 8 ints
+constexpr uint32_t TC_SCAN_OFF = TC_RING_OFF + TC_IRING * 32;
+// TMEM columns: S[0] [0, 128), S[1] [128, 256) (P_t over the first 64 columns
+// of S[t % 2], two bf16 per column), O [256, 384)
+constexpr uint32_t TC_TMEM_COLS = 512;
+constexpr uint32_t TC_O_COL = 256;
 
 struct TcArgs {
-  const __nv_bfloat16* q;
-  const __nv_bfloat16* k_blk;
-  const __nv_bfloat16* v_blk;
+  const int32_t* ctx;
   __nv_bfloat16* k_cache;
   __nv_bfloat16* v_cache;
-  const int32_t* ctx;
+  const __nv_bfloat16* k_blk;
+  const __nv_bfloat16* v_blk;
   __nv_bfloat16* out;
-  int B, Lb, Hq, Hkv, Cmax, G, rows, splits;
-  float scale_log2;
+  float* part_o;       // [slot][128][128] normalised partial O
+  float* part_ml;      // [slot][128][2]   (max in log2 units, sum)
+  unsigned* counters;  // [0] item counter, [1] CTAs finished
   unsigned* status;
+  int B, Lb, Hq, Hkv, G, Cmax, rows, n_rg, chunk, max_chunks;
+  float scale_log2;
+  int kv_evict_first;
 };
 
-template <int KT, int STAGES>
-struct TcLayout {
-  static constexpr int KV_TILE = KT * TC_D * 2;              // one K (or V) tile
-  static constexpr int P_ROW = KT < 64 ? 128 : KT * 2;       // bytes per P row (>= one 128 B atom row)
-  static constexpr int P_BYTES = TC_ROWS * P_ROW;
-  static constexpr int Q_OFF = 0;
-  static constexpr int K_OFF = TC_Q_BYTES;
-  static constexpr int V_OFF = K_OFF + STAGES * KV_TILE;
-  static constexpr int P_OFF = V_OFF + STAGES * KV_TILE;
-  static constexpr int BAR_OFF = P_OFF + P_BYTES;             // mbar_s, mbar_o, tmem slot, abort
-  static constexpr int W_OFF = BAR_OFF + 64;                  // merge weights [128][16]
-  static constexpr int ML_OFF = W_OFF + TC_ROWS * TC_MAX_SPLITS * 4;  // (m, l) [128][2]
-  static constexpr int BYTES = ML_OFF + TC_ROWS * 2 * 4;
-  // the fp32 partial [128][128] of the merge (64 KB) overlays Q and the K/V rings
-  static_assert(TC_ROWS * TC_D * 4 <= P_OFF, "merge buffer must fit in Q + K/V");
+struct Item {
+  int b, kvh, rg, c;  // b < 0: no more items
+  int ctx;            // -1: context length out of range (no tiles)
+  int kc_lo, kc_hi;   // cached keys of this chunk
+  int nch;            // chunks of the sequence
 };
 
-// byte offset of 16-byte chunk c (of 16) of row r in a [rows][128 dims] tile
-// stored as two 128B-swizzled halves of 64 dims
-__device__ __forceinline__ uint32_t tc_swz(int r, int c, int half_bytes) {
-  return static_cast<uint32_t>((c >> 3) * half_bytes + r * 128 + (((c & 7) ^ (r & 7)) << 4));
+__device__ __forceinline__ int item_cache_tiles(const Item& it) {
+  return it.kc_hi > it.kc_lo ? (it.kc_hi - it.kc_lo + TC_KT - 1) / TC_KT : 0;
+}
+__device__ __forceinline__ int item_tiles(const Item& it, int Lb) {
+  if (it.b < 0 || it.ctx < 0) return 0;
+  return item_cache_tiles(it) + (it.c == it.nch - 1 ? (Lb + TC_KT - 1) / TC_KT : 0);
+}
+
+// Chunks of a sequence (an invalid context length still gets one, empty, item).
+__device__ __forceinline__ int seq_chunks(int ctx, int Lb, int Cmax, int chunk) {
+  if (ctx < 0 || ctx + Lb > Cmax) return 1;
+  return ctx > 0 ? (ctx + chunk - 1) / chunk : 1;
 }
 
 }  // namespace
 
-template <int KT, int STAGES>
-__global__ void __launch_bounds__(TC_THREADS, 1) attention_tc_kernel(const TcArgs a) {
-  using L = TcLayout<KT, STAGES>;
+__global__ void __launch_bounds__(TC_THREADS, 1)
+    attention_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
+                        const __grid_constant__ CUtensorMap tm_kc,
+                        const __grid_constant__ CUtensorMap tm_vc,
+                        const __grid_constant__ CUtensorMap tm_kb,
+                        const __grid_constant__ CUtensorMap tm_vb, const TcArgs a) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* const smem = smem_raw + (base - raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  const int split = blockIdx.x, kvh = blockIdx.y;
-  const int n_rg = (a.rows + TC_ROWS - 1) / TC_ROWS;
-  const int b = blockIdx.z / n_rg, rg = blockIdx.z % n_rg;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t bars = base + TC_BAR_OFF;
+  auto q_full = [&](int i) { return bars + 8u * i; };  // 2 each
+  auto q_empty = [&](int i) { return bars + 16u + 8u * i; };
+  auto kv_full = [&](int i) { return bars + 32u + 8u * i; };  // TC_STAGES each
+  auto kv_empty = [&](int i) { return bars + 32u + 8u * (TC_STAGES + i); };
+  const uint32_t b2 = bars + 32u + 16u * TC_STAGES;
+  auto s_full = [&](int i) { return b2 + 8u * i; };  // 2 each
+  auto p_full = [&](int i) { return b2 + 16u + 8u * i; };
+  auto o_done = [&](int i) { return b2 + 32u + 8u * i; };
+  const uint32_t o_free = b2 + 48u;
+  const uint32_t drain_bar = b2 + 56u;
+  auto r_full = [&](int i) { return b2 + 64u + 8u * i; };  // TC_IRING each
+  auto r_empty = [&](int i) { return b2 + 64u + 8u * (TC_IRING + i); };
+  uint32_t* const tmem_slot = reinterpret_cast<uint32_t*>(smem + TC_MISC_OFF);
+  volatile int* const abort_flag = reinterpret_cast<volatile int*>(smem + TC_MISC_OFF + 4);
+  Item* const ring = reinterpret_cast<Item*>(smem + TC_RING_OFF);
+  int* const scan = reinterpret_cast<int*>(smem + TC_SCAN_OFF);  // [B + 1] first item of b
 
-  const int ctx = a.ctx[b];
-  if (ctx < 0 || ctx + a.Lb > a.Cmax) {
-    if (split == 0 && kvh == 0 && rg == 0 && tid == 0) raise_status(a.status, RV_DEV_CTX_RANGE);
-    return;
-  }
-  const int T = ctx + a.Lb;
-  const int per = ((T + a.splits - 1) / a.splits + 15) / 16 * 16;
-  const int k_lo = min(T, split * per);
-  const int k_hi = min(T, k_lo + per);
-  const int n_tiles = (k_hi - k_lo + KT - 1) / KT;
-
-  const int row0 = rg * TC_ROWS;
-  const int r = row0 + tid;  // this thread's query row
-  const bool rvalid = r < a.rows;
-  const int lim = rvalid ? ctx + r / a.G : -1;  // last key this row may see
-
-  const uint32_t bar_s = base + L::BAR_OFF, bar_o = bar_s + 8, bar_d = bar_s + 16;
-  uint32_t* const tmem_slot = reinterpret_cast<uint32_t*>(smem + L::BAR_OFF + 24);
-  volatile int* const abort_flag = reinterpret_cast<volatile int*>(smem + L::BAR_OFF + 28);
-  if (tid == 0) {
-    mbar_init(bar_s, 1);
-    mbar_init(bar_o, 1);
-    mbar_init(bar_d, 1);
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(q_full(i), 1);
+      mbar_init(q_empty(i), 1);
+      mbar_init(s_full(i), 1);
+      mbar_init(p_full(i), 4);
+      mbar_init(o_done(i), 1);
+    }
+    for (int i = 0; i < TC_STAGES; ++i) {
+      mbar_init(kv_full(i), 1);
+      mbar_init(kv_empty(i), 1);
+    }
+    mbar_init(o_free, 4);
+    mbar_init(drain_bar, 1);
+    for (int i = 0; i < TC_IRING; ++i) {
+      mbar_init(r_full(i), 1);
+      mbar_init(r_empty(i), 5);  // the MMA thread + one lane per softmax warp
+    }
     *abort_flag = 0;
     fence_barrier_init();
   }
-  if (warp == 0) tmem_alloc(smem_u32(tmem_slot), 256);  // S: cols [0, KT); O: [128, 256)
-
-  // ---- Q rows and the first K/V tiles (cp.async, swizzled)
-  for (int e = tid; e < TC_ROWS * 16; e += TC_THREADS) {
-    const int rr = e >> 4, c = e & 15;
-    const int qr = row0 + rr;
-    const bool ok = qr < a.rows;
-    const int j = ok ? qr / a.G : 0, hh = ok ? kvh * a.G + qr % a.G : 0;
-    const __nv_bfloat16* src = a.q + ((static_cast<long long>(b) * a.Lb + j) * a.Hq + hh) * TC_D + c * 8;
-    cp_async16(base + L::Q_OFF + tc_swz(rr, c, TC_ROWS * 128), src, ok);
-  }
-  auto load_kv = [&](int tile, int buf) {
-    const int k0 = k_lo + tile * KT;
-    const uint32_t kd = base + L::K_OFF + buf * L::KV_TILE;
-    const uint32_t vd = base + L::V_OFF + buf * L::KV_TILE;
-    for (int e = tid; e < KT * 16; e += TC_THREADS) {
-      const int rr = e >> 4, c = e & 15;
-      const int kk = k0 + rr;
-      const bool ok = kk < k_hi;
-      const __nv_bfloat16 *ks, *vs;
-      if (kk < ctx) {
-        const long long off = ((static_cast<long long>(b) * a.Hkv + kvh) * a.Cmax + kk) * TC_D + c * 8;
-        ks = a.k_cache + off;
-        vs = a.v_cache + off;
-      } else {
-        const int j = ok ? kk - ctx : 0;
-        const long long off = ((static_cast<long long>(b) * a.Lb + j) * a.Hkv + kvh) * TC_D + c * 8;
-        ks = a.k_blk + off;
-        vs = a.v_blk + off;
-      }
-      cp_async16(kd + tc_swz(rr, c, KT * 128), ks, ok);
-      cp_async16(vd + tc_swz(rr, c, KT * 128), vs, ok);
-    }
-  };
-  if (n_tiles > 0) load_kv(0, 0);
-  cp_async_commit();  // group: Q + tile 0
+  if (warp == 0) {
+    // items of sequence b: Hkv * n_rg * chunks(b), numbered sequence by sequence
+    const int per_seq = a.Hkv * a.n_rg;
+    int carry = 0;
+    for (int b0 = 0; b0 < a.B; b0 += 32) {
+      const int b = b0 + lane;
+      const int n = b < a.B ? per_seq * seq_chunks(a.ctx[b], a.Lb, a.Cmax, a.chunk) : 0;
+      int incl = n;
 #pragma unroll
-  for (int t = 1; t < STAGES - 1; ++t) {
-    if (t < n_tiles) load_kv(t, t);
-    cp_async_commit();
-  }
-
-  // Append the block's keys/values (positions ctx..ctx+Lb-1) once per (b, kvh).
-  if (split == 0 && rg == 0) {
-    for (int e = tid; e < a.Lb * 16; e += TC_THREADS) {
-      const int j = e >> 4, c = e & 15;
-      const long long src = ((static_cast<long long>(b) * a.Lb + j) * a.Hkv + kvh) * TC_D + c * 8;
-      const long long dst =
-          ((static_cast<long long>(b) * a.Hkv + kvh) * a.Cmax + ctx + j) * TC_D + c * 8;
-      *reinterpret_cast<uint4*>(a.k_cache + dst) = *reinterpret_cast<const uint4*>(a.k_blk + src);
-      *reinterpret_cast<uint4*>(a.v_cache + dst) = *reinterpret_cast<const uint4*>(a.v_blk + src);
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      if (b < a.B) scan[b] = carry + incl - n;
+      carry += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    if (lane == 0) {
+      scan[a.B] = carry;
+      tma_prefetch_desc(&tm_q);
+      tma_prefetch_desc(&tm_kc);
+      tma_prefetch_desc(&tm_vc);
+      tma_prefetch_desc(&tm_kb);
+      tma_prefetch_desc(&tm_vb);
     }
   }
-
+  if (warp == 1) tmem_alloc(smem_u32(tmem_slot), TC_TMEM_COLS);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t t_row = tmem + (static_cast<uint32_t>(warp * 32) << 16);  // this warp's lanes
-  const uint32_t s_cols = t_row, o_cols = t_row + 128u;
+  // the merge launch that follows may start (it waits for this grid's results)
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
-  const uint32_t idesc_s = idesc_bf16_f32(TC_ROWS, KT);
-  const uint32_t idesc_o = idesc_bf16_f32_bmn(TC_ROWS, TC_D);
-  float m_used = NEG_INF, l = 0.f;
-  bool ok_all = true;
-
-  for (int t = 0; t < n_tiles && ok_all; ++t) {
-    const int buf = t % STAGES;
-    cp_async_wait<STAGES - 2>();  // Q and tile t have landed
-    fence_proxy_async_smem();
-    __syncthreads();
-    if (tid == 0) {
-      tc_fence_after();
-      const uint32_t kb = base + L::K_OFF + buf * L::KV_TILE;
-#pragma unroll
-      for (int kk = 0; kk < TC_D / 16; ++kk) {
-        const uint32_t half = static_cast<uint32_t>(kk >> 2), off = static_cast<uint32_t>((kk & 3) * 32);
-        tc_mma_bf16(tmem, sw128_kmajor_desc(base + L::Q_OFF + half * (TC_ROWS * 128) + off),
-                    sw128_kmajor_desc(kb + half * (KT * 128) + off), idesc_s, kk > 0 ? 1u : 0u);
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      const uint64_t pol_q = policy_evict_last();
+      const uint64_t pol_kv = a.kv_evict_first ? policy_evict_first() : policy_evict_normal();
+      const int total = scan[a.B];
+      const int rows_j = TC_M / a.G;  // block positions per row group
+      int u = 0, it = 0, issued_q = 0;
+      bool ok = true;
+      for (int lt = 0; ok; ++lt) {
+        const int i = static_cast<int>(atomicAdd(&a.counters[0], 1u));
+        Item item;
+        item.b = -1;
+        item.kvh = item.rg = item.c = item.ctx = item.kc_lo = item.kc_hi = 0;
+        item.nch = 1;
+        if (i < total) {
+          int lo = 0, hi = a.B - 1;  // the last b with scan[b] <= i
+          while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (scan[mid] <= i)
+              lo = mid;
+            else
+              hi = mid - 1;
+          }
+          const int b = lo;
+          const int ctx = a.ctx[b];
+          const int nch = seq_chunks(ctx, a.Lb, a.Cmax, a.chunk);
+          int rem = i - scan[b];
+          item.b = b;
+          item.rg = rem % a.n_rg;
+          rem /= a.n_rg;
+          item.c = rem % nch;
+          item.kvh = rem / nch;
+          item.nch = nch;
+          const bool valid = ctx >= 0 && ctx + a.Lb <= a.Cmax;
+          item.ctx = valid ? ctx : -1;
+          if (!valid && item.kvh == 0 && item.rg == 0) raise_status(a.status, RV_DEV_CTX_RANGE);
+          item.kc_lo = valid ? min(ctx, item.c * a.chunk) : 0;
+          item.kc_hi = valid ? min(ctx, item.kc_lo + a.chunk) : 0;
+        }
+        const int k = lt % TC_IRING;
+        if (!mbar_wait(r_empty(k), ((lt / TC_IRING) & 1) ^ 1u, abort_flag, a.status)) {
+          ok = false;
+          break;
+        }
+        ring[k] = item;
+        mbar_arrive(r_full(k));
+        if (item.b < 0) break;
+        const int n = item_tiles(item, a.Lb);
+        if (n == 0) continue;
+        const int qb = it & 1;
+        if (!mbar_wait(q_empty(qb), ((it >> 1) & 1) ^ 1u, abort_flag, a.status)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(q_full(qb), TC_Q_BYTES);
+        const int qz = item.b * a.Lb + item.rg * rows_j;
+        const uint32_t qd = base + TC_Q_OFF + qb * TC_Q_BYTES;
+        tma_load_3d(qd, &tm_q, 0, item.kvh * a.G, qz, q_full(qb), pol_q);
+        tma_load_3d(qd + TC_Q_BYTES / 2, &tm_q, 64, item.kvh * a.G, qz, q_full(qb), pol_q);
+        ++issued_q;
+        const int n_cache = item_cache_tiles(item);
+        const int row_c = (item.b * a.Hkv + item.kvh) * a.Cmax;
+        for (int j = 0; j < n; ++j) {
+          const int st = u % TC_STAGES;
+          if (!mbar_wait(kv_empty(st), ((u / TC_STAGES) & 1) ^ 1u, abort_flag, a.status)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(kv_full(st), 2 * TC_KV_BYTES);
+          const uint32_t kd = base + TC_K_OFF + st * TC_KV_BYTES;
+          const uint32_t vd = base + TC_V_OFF + st * TC_KV_BYTES;
+          if (j < n_cache) {
+            const int y = row_c + item.kc_lo + j * TC_KT;
+            tma_load_2d(kd, &tm_kc, 0, y, kv_full(st), pol_kv);
+            tma_load_2d(kd + TC_KV_BYTES / 2, &tm_kc, 64, y, kv_full(st), pol_kv);
+            tma_load_2d(vd, &tm_vc, 0, y, kv_full(st), pol_kv);
+            tma_load_2d(vd + TC_KV_BYTES / 2, &tm_vc, 64, y, kv_full(st), pol_kv);
+          } else {
+            const int z = item.b * a.Lb + (j - n_cache) * TC_KT;
+            tma_load_3d(kd, &tm_kb, 0, item.kvh, z, kv_full(st), pol_q);
+            tma_load_3d(kd + TC_KV_BYTES / 2, &tm_kb, 64, item.kvh, z, kv_full(st), pol_q);
+            tma_load_3d(vd, &tm_vb, 0, item.kvh, z, kv_full(st), pol_q);
+            tma_load_3d(vd + TC_KV_BYTES / 2, &tm_vb, 64, item.kvh, z, kv_full(st), pol_q);
+          }
+          ++u;
+        }
+        ++it;
       }
-      tc_commit(bar_s);
+      if (!ok) {  // let the copies still in flight land before the CTA exits
+        for (int v = max(0, u - TC_STAGES); v < u; ++v)
+          drain_wait(kv_full(v % TC_STAGES), static_cast<uint32_t>((v / TC_STAGES) & 1));
+        for (int qq = max(0, issued_q - 2); qq < issued_q; ++qq)
+          drain_wait(q_full(qq & 1), static_cast<uint32_t>((qq >> 1) & 1));
+      }
     }
-    bool ok = mbar_wait(bar_s, t & 1, abort_flag, a.status);
-    if (ok && t > 0) ok = mbar_wait(bar_o, (t - 1) & 1, abort_flag, a.status);  // PV(t-1) done
-    if (!__syncthreads_and(ok)) {
-      ok_all = false;
-      break;
+    __syncwarp();
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      const uint32_t idesc_s = idesc_bf16_f32(TC_M, TC_KT);
+      const uint32_t idesc_o = idesc_bf16_f32_bmn(TC_M, TC_D);
+      int u = 0, it = 0;
+      bool ok = true;
+      // O += P_v V_v for tile v; the first tile of an item overwrites O, once
+      // the softmax warps have read the previous item's O
+      auto issue_pv = [&](int v, bool first) -> bool {
+        const int pb = v & 1;
+        if (!mbar_wait(p_full(pb), (v >> 1) & 1, abort_flag, a.status)) return false;
+        if (first && it > 0 && !mbar_wait(o_free, (it - 1) & 1, abort_flag, a.status)) return false;
+        tc_fence_after();
+        const uint32_t pcol = tmem + static_cast<uint32_t>(pb * TC_KT);
+        const uint32_t vb = base + TC_V_OFF + (v % TC_STAGES) * TC_KV_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < TC_KT / 16; ++kk)
+          tc_mma_bf16_tmem_a(tmem + TC_O_COL, pcol + kk * 8,
+                             sw128_mnmajor_desc(vb + kk * 16 * 128, TC_KV_BYTES / 2, 1024),
+                             idesc_o, (!first || kk > 0) ? 1u : 0u);
+        tc_commit(o_done(pb));
+        tc_commit(kv_empty(v % TC_STAGES));
+        return true;
+      };
+      for (int lt = 0; ok; ++lt) {
+        const int k = lt % TC_IRING;
+        if (!mbar_wait(r_full(k), (lt / TC_IRING) & 1, abort_flag, a.status)) break;
+        const Item item = ring[k];
+        mbar_arrive(r_empty(k));
+        if (item.b < 0) break;
+        const int n = item_tiles(item, a.Lb);
+        if (n == 0) continue;
+        const int qb = it & 1;
+        if (!mbar_wait(q_full(qb), (it >> 1) & 1, abort_flag, a.status)) break;
+        const uint32_t qbase = base + TC_Q_OFF + qb * TC_Q_BYTES;
+        for (int j = 0; j < n && ok; ++j) {
+          const int v = u + j;
+          const int st = v % TC_STAGES;
+          if (!mbar_wait(kv_full(st), (v / TC_STAGES) & 1, abort_flag, a.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t kb = base + TC_K_OFF + st * TC_KV_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < TC_D / 16; ++kk) {
+            const uint32_t half = static_cast<uint32_t>(kk >> 2);
+            const uint32_t off = static_cast<uint32_t>((kk & 3) * 32);
+            tc_mma_bf16(tmem + static_cast<uint32_t>((v & 1) * TC_KT),
+                        sw128_kmajor_desc(qbase + half * (TC_Q_BYTES / 2) + off),
+                        sw128_kmajor_desc(kb + half * (TC_KV_BYTES / 2) + off), idesc_s,
+                        kk > 0 ? 1u : 0u);
+          }
+          tc_commit(s_full(v & 1));
+          if (j == n - 1) tc_commit(q_empty(qb));
+          if (j > 0 && !issue_pv(v - 1, j == 1)) ok = false;
+        }
+        if (ok && !issue_pv(u + n - 1, n == 1)) ok = false;
+        u += n;
+        ++it;
+      }
+      // every MMA issued must be complete before TMEM is released
+      tc_commit(drain_bar);
+      drain_wait(drain_bar, 0);
     }
-    tc_fence_after();
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ softmax warps
+    const int q = warp & 3;       // TMEM lane quadrant
+    const int r = q * 32 + lane;  // query row within the row group (TMEM lane)
+    const int st_tid = threadIdx.x - 64;
+    const uint32_t t_row = tmem + (static_cast<uint32_t>(q * 32) << 16);
+    int u = 0;
+    for (int lt = 0;; ++lt) {
+      const int k = lt % TC_IRING;
+      bool ok = mbar_wait(r_full(k), (lt / TC_IRING) & 1, abort_flag, a.status);
+      if (!__all_sync(0xffffffffu, ok)) break;
+      const Item item = ring[k];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(r_empty(k));
+      if (item.b < 0) break;
+      const int n = item_tiles(item, a.Lb);
+      if (n == 0) continue;
+      const int n_cache = item_cache_tiles(item);
+      const int ctx = item.ctx;
+      const int gr = item.rg * TC_M + r;  // row among the Lb*G rows of (sequence, KV head)
+      const bool rvalid = gr < a.rows;
+      const int lim = rvalid ? ctx + gr / a.G : -1;  // last key this row may see
 
-    // ---- online softmax of this row over the tile's KT keys
-    float sv[KT];
+      // append the block's keys/values to the cache, once per (sequence, KV head)
+      if (item.c == item.nch - 1 && item.rg == 0) {
+        for (int e = st_tid; e < a.Lb * 16; e += 128) {
+          const int j = e >> 4, c16 = e & 15;
+          const long long src =
+              ((static_cast<long long>(item.b) * a.Lb + j) * a.Hkv + item.kvh) * TC_D + c16 * 8;
+          const long long dst =
+              ((static_cast<long long>(item.b) * a.Hkv + item.kvh) * a.Cmax + ctx + j) * TC_D +
+              c16 * 8;
+          *reinterpret_cast<uint4*>(a.k_cache + dst) = *reinterpret_cast<const uint4*>(a.k_blk + src);
+          *reinterpret_cast<uint4*>(a.v_cache + dst) = *reinterpret_cast<const uint4*>(a.v_blk + src);
+        }
+      }
+
+      float m_used = NEG_INF, l = 0.f;  // running max (log2 units) and sum of this row
+      bool good = true;
+      for (int j = 0; j < n; ++j) {
+        const int v = u + j;
+        const int sb = v & 1;
+        const uint32_t s_col = t_row + static_cast<uint32_t>(sb * TC_KT);
+        ok = mbar_wait(s_full(sb), (v >> 1) & 1, abort_flag, a.status);
+        if (!__all_sync(0xffffffffu, ok)) {
+          good = false;
+          break;
+        }
+        tc_fence_after();
+        float sv[4][32];
 #pragma unroll
-    for (int c = 0; c < KT; c += 32) {
-      float tmp[32];
-      tmem_ld32(s_cols + c, tmp);
+        for (int c = 0; c < 4; ++c) tmem_ld32(s_col + 32 * c, sv[c]);
+        tmem_ld_wait();
+        int kb, kend;
+        if (j < n_cache) {
+          kb = item.kc_lo + j * TC_KT;
+          kend = item.kc_hi;
+        } else {
+          kb = ctx + (j - n_cache) * TC_KT;
+          kend = ctx + a.Lb;
+        }
+        const int kmax = min(kend - 1, lim);  // last key of the tile this row sees
+        if (kb + TC_KT - 1 > kmax) {          // a partial tile for this row: mask
 #pragma unroll
-      for (int i = 0; i < 32; ++i) sv[c + i] = tmp[i];
-    }
-    tmem_ld_wait();
-    const int kbase = k_lo + t * KT;
-    float mt = NEG_INF;
+          for (int c = 0; c < 4; ++c)
 #pragma unroll
-    for (int j = 0; j < KT; ++j) {
-      const int key = kbase + j;
-      sv[j] = (key < k_hi && key <= lim) ? sv[j] * a.scale_log2 : NEG_INF;
-      mt = fmaxf(mt, sv[j]);
-    }
-    float fac = 1.f;
-    const bool rise = mt > m_used + TC_RESCALE_LOG2 || (m_used == NEG_INF && mt != NEG_INF);
-    if (rise) {
-      fac = (m_used == NEG_INF) ? 0.f : exp2f(m_used - mt);
-      m_used = mt;
-    }
-    // O already holds earlier tiles (t > 0): rescale this warp's rows if any rose
-    if (t > 0 && __any_sync(0xffffffffu, rise && fac != 1.f)) {
+            for (int i = 0; i < 32; ++i)
+              if (kb + 32 * c + i > kmax) sv[c][i] = NEG_INF;
+        }
+        float mx[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          mx[c] = sv[c][0];
+#pragma unroll
+          for (int i = 1; i < 32; ++i) mx[c] = fmaxf(mx[c], sv[c][i]);
+        }
+        const float mt = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * a.scale_log2;
+        float fac = 1.f;
+        const bool rise = mt > m_used + TC_RESCALE_LOG2 || (m_used == NEG_INF && mt != NEG_INF);
+        if (rise) {
+          fac = (m_used == NEG_INF) ? 0.f : exp2f(m_used - mt);
+          m_used = mt;
+        }
+        // O holds this item's earlier tiles: rescale this warp's rows if any rose
+        if (j > 0 && __any_sync(0xffffffffu, rise && fac != 1.f)) {
+          ok = mbar_wait(o_done((v - 1) & 1), ((v - 1) >> 1) & 1, abort_flag, a.status);
+          if (!__all_sync(0xffffffffu, ok)) {
+            good = false;
+            break;
+          }
+          tc_fence_after();
+#pragma unroll
+          for (int c = 0; c < TC_D; c += 32) {
+            float ov[32];
+            tmem_ld32(t_row + TC_O_COL + c, ov);
+            tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) ov[i] *= fac;
+            tmem_st32(t_row + TC_O_COL + c, ov);
+          }
+          tmem_st_wait();
+        }
+        // P = 2^(s * scale - m), bf16, over the first half of S[sb]
+        const float neg_m = (m_used == NEG_INF) ? 0.f : -m_used;
+        float ls[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int i = 0; i < 32; i += 2) {
+            const float p0 = ex2_approx(fmaf(sv[c][i], a.scale_log2, neg_m));
+            const float p1 = ex2_approx(fmaf(sv[c][i + 1], a.scale_log2, neg_m));
+            ls[c] += p0 + p1;
+            pk[i >> 1] = pack_bf16(p0, p1);
+          }
+          tmem_st16(s_col + 16 * c, pk);
+        }
+        l = l * fac + ((ls[0] + ls[1]) + (ls[2] + ls[3]));
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(p_full(sb));
+      }
+      if (!good) break;
+      // ---- item end: this row's O
+      const int vl = u + n - 1;
+      ok = mbar_wait(o_done(vl & 1), (vl >> 1) & 1, abort_flag, a.status);
+      if (!__all_sync(0xffffffffu, ok)) break;
+      tc_fence_after();
+      u += n;
+      const float inv = (l > 0.f) ? 1.f / l : 0.f;
+      const int group = (item.b * a.Hkv + item.kvh) * a.n_rg + item.rg;
+      const int slot = group * a.max_chunks + item.c;
+      const long long orow = (static_cast<long long>(item.b) * a.Lb + gr / a.G) * a.Hq +
+                             item.kvh * a.G + gr % a.G;
+      float* const po = a.part_o + (static_cast<long long>(slot) * TC_M + r) * TC_D;
 #pragma unroll
       for (int c = 0; c < TC_D; c += 32) {
         float ov[32];
-        tmem_ld32(o_cols + c, ov);
+        tmem_ld32(t_row + TC_O_COL + c, ov);
         tmem_ld_wait();
+        if (rvalid) {
+          if (item.nch == 1) {
+            __nv_bfloat16* dst = a.out + orow * TC_D + c;
 #pragma unroll
-        for (int i = 0; i < 32; ++i) ov[i] *= fac;
-        tmem_st32(o_cols + c, ov);
-      }
-      tmem_st_wait();
-    }
-    l *= fac;
-    // P row (bf16) into the K-major swizzled P tile
-    uint8_t* const prow = smem + L::P_OFF + tid * 128;
+            for (int i = 0; i < 32; i += 8) {
+              uint4 pk;
+              pk.x = pack_bf16(ov[i] * inv, ov[i + 1] * inv);
+              pk.y = pack_bf16(ov[i + 2] * inv, ov[i + 3] * inv);
+              pk.z = pack_bf16(ov[i + 4] * inv, ov[i + 5] * inv);
+              pk.w = pack_bf16(ov[i + 6] * inv, ov[i + 7] * inv);
+              *reinterpret_cast<uint4*>(dst + i) = pk;
+            }
+          } else {
 #pragma unroll
-    for (int c = 0; c < KT / 8; ++c) {
-      float p[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        p[i] = (m_used == NEG_INF) ? 0.f : exp2f(sv[c * 8 + i] - m_used);
-        l += p[i];
-      }
-      uint4 pk;
-      pk.x = pack_bf16(p[0], p[1]);
-      pk.y = pack_bf16(p[2], p[3]);
-      pk.z = pack_bf16(p[4], p[5]);
-      pk.w = pack_bf16(p[6], p[7]);
-      const int half = c >> 3, cc = c & 7;
-      *reinterpret_cast<uint4*>(prow + half * (TC_ROWS * 128) + ((cc ^ (tid & 7)) << 4)) = pk;
-    }
-    fence_proxy_async_smem();
-    tc_fence_before();
-    __syncthreads();
-    if (tid == 0) {
-      tc_fence_after();
-      const uint32_t vb = base + L::V_OFF + buf * L::KV_TILE;
-#pragma unroll
-      for (int kk = 0; kk < KT / 16; ++kk) {
-        const uint32_t half = static_cast<uint32_t>(kk >> 2), off = static_cast<uint32_t>((kk & 3) * 32);
-        tc_mma_bf16(tmem + 128u,
-                    sw128_kmajor_desc(base + L::P_OFF + half * (TC_ROWS * 128) + off),
-                    sw128_mnmajor_desc(vb + kk * 16 * 128, KT * 128, 1024), idesc_o,
-                    (t > 0 || kk > 0) ? 1u : 0u);
-      }
-      tc_commit(bar_o);
-    }
-    // refill: tile t+STAGES-1 into the buffer of tile t-1 (its PV is complete)
-    if (t + STAGES - 1 < n_tiles) load_kv(t + STAGES - 1, (t + STAGES - 1) % STAGES);
-    cp_async_commit();
-  }
-  cp_async_wait_all();
-  if (ok_all && n_tiles > 0) {
-    const bool ok = mbar_wait(bar_o, (n_tiles - 1) & 1, abort_flag, a.status);
-    ok_all = __syncthreads_and(ok);
-  } else {
-    ok_all = __syncthreads_and(ok_all) && ok_all;
-  }
-  tc_fence_after();
-
-  // ---- this row's O/l (zeros when the row saw no key)
-  const float inv = (l > 0.f) ? 1.f / l : 0.f;
-  auto row_index = [&](int rr) {
-    const int j = rr / a.G, hh = kvh * a.G + rr % a.G;
-    return (static_cast<long long>(b) * a.Lb + j) * a.Hq + hh;
-  };
-  float* const part = reinterpret_cast<float*>(smem);  // [128][128], overlays Q and K/V
-  __syncthreads();  // every thread is done with Q / K / V before the overlay is written
-#pragma unroll
-  for (int c = 0; c < TC_D; c += 32) {
-    float ov[32];
-    tmem_ld32(o_cols + c, ov);
-    tmem_ld_wait();
-#pragma unroll
-    for (int i = 0; i < 32; ++i) ov[i] = (n_tiles > 0 && l > 0.f) ? ov[i] * inv : 0.f;
-    if (a.splits == 1) {
-      if (rvalid) {
-        __nv_bfloat16* dst = a.out + row_index(r) * TC_D + c;
-#pragma unroll
-        for (int i = 0; i < 32; i += 8) {
-          uint4 pk;
-          pk.x = pack_bf16(ov[i], ov[i + 1]);
-          pk.y = pack_bf16(ov[i + 2], ov[i + 3]);
-          pk.z = pack_bf16(ov[i + 4], ov[i + 5]);
-          pk.w = pack_bf16(ov[i + 6], ov[i + 7]);
-          *reinterpret_cast<uint4*>(dst + i) = pk;
+            for (int i = 0; i < 32; i += 4)
+              __stcg(reinterpret_cast<float4*>(po + c + i),
+                     make_float4(ov[i] * inv, ov[i + 1] * inv, ov[i + 2] * inv, ov[i + 3] * inv));
+          }
         }
       }
-    } else {
-#pragma unroll
-      for (int i = 0; i < 32; i += 4) {
-        const int i2 = (i + 4 * (tid & 7)) & 31;  // rotate to spread banks
-        *reinterpret_cast<float4*>(part + tid * TC_D + c + i2) =
-            make_float4(ov[i2], ov[i2 + 1], ov[i2 + 2], ov[i2 + 3]);
-      }
+      if (rvalid && item.nch > 1)
+        __stcg(reinterpret_cast<float2*>(a.part_ml) + static_cast<long long>(slot) * TC_M + r,
+               make_float2(m_used, l));
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(o_free);
     }
   }
-  float* const wsm = reinterpret_cast<float*>(smem + L::W_OFF);
-  float* const ml = reinterpret_cast<float*>(smem + L::ML_OFF);
-  if (a.splits > 1) {
-    ml[2 * tid] = m_used;
-    ml[2 * tid + 1] = l;
-  }
-  // every MMA issued must be complete before TMEM is released (a no-op wait
-  // unless a pipeline wait above gave up)
-  if (tid == 0) {
-    tc_commit(bar_d);
-    const unsigned long long t0 = globaltimer_ns();
-    while (!mbar_try_wait(bar_d, 0) && globaltimer_ns() - t0 < RV_WAIT_TIMEOUT_NS / 4) {
-    }
-  }
+
   tc_fence_before();
   __syncthreads();
-  if (warp == 0) {
+  if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, 256);
+    tmem_dealloc(tmem, TC_TMEM_COLS);
   }
-  if (a.splits == 1) return;
-
-  // ---- split-KV merge through distributed shared memory (as in k_attention.cu)
-  cg::cluster_group cluster = cg::this_cluster();
-  cluster.sync();
-  const int S = a.splits;
-  const int rank = static_cast<int>(cluster.block_rank());
-  const int nrow = min(TC_ROWS, a.rows - row0);
-  const int per_rank = (nrow + S - 1) / S;
-  const int r_lo = min(nrow, rank * per_rank), r_hi = min(nrow, r_lo + per_rank);
-  const int n_items = (r_hi - r_lo) * S;
-  for (int b0 = 0; b0 < n_items; b0 += TC_THREADS) {
-    const int it = b0 + tid;
-    const bool act = it < n_items;
-    const int rl = r_lo + (act ? it / S : 0), sp = it % S;
-    float m = NEG_INF, lv = 0.f;
-    if (act) {
-      const float* rml = cluster.map_shared_rank(ml, sp);
-      m = rml[2 * rl];
-      lv = rml[2 * rl + 1];
+  // the last CTA to finish re-arms the item counter for the next launch
+  if (threadIdx.x == 0) {
+    __threadfence();
+    if (atomicAdd(&a.counters[1], 1u) == gridDim.x - 1) {
+      a.counters[0] = 0u;
+      a.counters[1] = 0u;
+      __threadfence();
     }
-    float M = lv > 0.f ? m : NEG_INF;
-    for (int o = 1; o < S; o <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    const float w = lv > 0.f ? lv * exp2f(m - M) : 0.f;
-    float den = w;
-    for (int o = 1; o < S; o <<= 1) den += __shfl_xor_sync(0xffffffffu, den, o);
-    if (act) wsm[rl * TC_MAX_SPLITS + sp] = den > 0.f ? w / den : 0.f;
   }
-  __syncthreads();
-  constexpr int D4 = TC_D / 4;
-  for (int it = tid; it < (r_hi - r_lo) * D4; it += TC_THREADS) {
-    const int rl = r_lo + it / D4, d = (it % D4) * 4;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-    for (int sp = 0; sp < TC_MAX_SPLITS; ++sp) {
-      if (sp < S) {
-        const float w = wsm[rl * TC_MAX_SPLITS + sp];
-        const float4 v =
-            *reinterpret_cast<const float4*>(cluster.map_shared_rank(part, sp) + rl * TC_D + d);
-        acc.x = fmaf(w, v.x, acc.x);
-        acc.y = fmaf(w, v.y, acc.y);
-        acc.z = fmaf(w, v.z, acc.z);
-        acc.w = fmaf(w, v.w, acc.w);
-      }
-    }
-    uint2 pk;
-    pk.x = pack_bf16(acc.x, acc.y);
-    pk.y = pack_bf16(acc.z, acc.w);
-    *reinterpret_cast<uint2*>(a.out + row_index(row0 + rl) * TC_D + d) = pk;
-  }
-  cluster.sync();
 }
 
-// ---------------------------------------------------------------- launch
+// Merge of the chunks of each (sequence, KV head, row group) whose sequence
+// needed several: one warp per query row, lane i holding dims 4i..4i+3.
+// out = sum_c w_c O_c / sum_c w_c with w_c = l_c 2^(m_c - max_c m_c).
+struct MergeArgs {
+  const int32_t* ctx;
+  const float* part_o;
+  const float* part_ml;
+  __nv_bfloat16* out;
+  int Lb, Hq, Hkv, G, Cmax, rows, n_rg, chunk, max_chunks;
+};
 
-namespace {
-constexpr int TC_KT = 64;
-constexpr int TC_STAGES = 3;
-}  // namespace
+__global__ void __launch_bounds__(256) attention_merge_kernel(const MergeArgs a) {
+  asm volatile("griddepcontrol.wait;" ::: "memory");  // the attention grid's results
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int group = blockIdx.x;
+  const int rg = group % a.n_rg, t = group / a.n_rg;
+  const int kvh = t % a.Hkv, b = t / a.Hkv;
+  const int rr = blockIdx.y * 8 + warp;  // row within the row group
+  const int gr = rg * TC_M + rr;
+  if (rr >= TC_M || gr >= a.rows) return;
+  const int ctx = a.ctx[b];
+  if (ctx < 0 || ctx + a.Lb > a.Cmax) return;
+  const int nch = seq_chunks(ctx, a.Lb, a.Cmax, a.chunk);
+  if (nch == 1) return;
+  const long long slot0 = static_cast<long long>(group) * a.max_chunks;
+  const float2* ml = reinterpret_cast<const float2*>(a.part_ml);
+  float M = NEG_INF;
+  for (int c = lane; c < nch; c += 32) {
+    const float2 v = __ldcg(ml + (slot0 + c) * TC_M + rr);
+    if (v.y > 0.f) M = fmaxf(M, v.x);
+  }
+  M = warp_max(M);
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  float den = 0.f;
+#pragma unroll 4
+  for (int c = 0; c < nch; ++c) {
+    const float2 v = __ldcg(ml + (slot0 + c) * TC_M + rr);
+    const float4 o =
+        __ldcg(reinterpret_cast<const float4*>(a.part_o + ((slot0 + c) * TC_M + rr) * TC_D) + lane);
+    const float w = v.y > 0.f ? v.y * exp2f(v.x - M) : 0.f;
+    acc.x = fmaf(w, o.x, acc.x);
+    acc.y = fmaf(w, o.y, acc.y);
+    acc.z = fmaf(w, o.z, acc.z);
+    acc.w = fmaf(w, o.w, acc.w);
+    den += w;
+  }
+  const float id = den > 0.f ? 1.f / den : 0.f;
+  const long long orow =
+      (static_cast<long long>(b) * a.Lb + gr / a.G) * a.Hq + kvh * a.G + gr % a.G;
+  uint2 pk;
+  pk.x = pack_bf16(acc.x * id, acc.y * id);
+  pk.y = pack_bf16(acc.z * id, acc.w * id);
+  *reinterpret_cast<uint2*>(a.out + orow * TC_D + lane * 4) = pk;
+}
 
-size_t attn_tc_smem_bytes() { return TcLayout<TC_KT, TC_STAGES>::BYTES + 1024; }
+// ---------------------------------------------------------------- planning / launch
 
-cudaError_t attn_tc_configure() {
-  auto k = attention_tc_kernel<TC_KT, TC_STAGES>;
-  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(attn_tc_smem_bytes()));
+AttnTcPlan attn_tc_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms) {
+  AttnTcPlan p;
+  const int G = Hq / Hkv;
+  p.rows = Lb * G;
+  p.n_rg = (p.rows + TC_M - 1) / TC_M;
+  const long long groups = static_cast<long long>(B) * Hkv * p.n_rg;
+  // chunks sized for about four items per SM when every sequence is full
+  long long ch = (groups * Cmax + 4LL * num_sms - 1) / (4LL * num_sms);
+  ch = std::max<long long>(256, (ch + TC_KT - 1) / TC_KT * TC_KT);
+  ch = std::min<long long>(ch, (Cmax + TC_KT - 1) / TC_KT * TC_KT + TC_KT);
+  p.chunk = static_cast<int>(ch);
+  p.max_chunks = std::max(1, (Cmax + p.chunk - 1) / p.chunk);
+  p.slots = static_cast<int>(groups) * p.max_chunks;
+  p.grid = static_cast<int>(std::min<long long>(num_sms, p.slots));
+  p.smem_bytes = TC_SCAN_OFF + static_cast<size_t>(B + 1) * 4 + 1024;
+  return p;
+}
+
+bool attn_tc_supported(int Hq, int Hkv, int D) {
+  return D == TC_D && Hkv > 0 && Hq % Hkv == 0 && TC_M % (Hq / Hkv) == 0;
+}
+
+size_t attn_tc_smem_max(int max_batch) {
+  return TC_SCAN_OFF + static_cast<size_t>(max_batch + 1) * 4 + 1024;
+}
+
+int attn_tc_max_slots(int max_batch, int Lb_max, int Hq, int Hkv, int num_sms) {
+  // chunk >= groups * Cmax / (4 * SMs), or one chunk per group: slots <= 4 * SMs + groups
+  const int n_rg = (Lb_max * (Hq / Hkv) + TC_M - 1) / TC_M;
+  return 4 * num_sms + max_batch * Hkv * n_rg;
+}
+
+cudaError_t attn_tc_configure(size_t smem_bytes) {
+  cudaError_t e = cudaFuncSetAttribute(attention_tc_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem_bytes));
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(k, cudaFuncAttributePreferredSharedMemoryCarveout,
+    e = cudaFuncSetAttribute(attention_tc_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
                              cudaSharedmemCarveoutMaxShared);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   return e;
 }
 
-cudaError_t launch_attention_tc(const AttnArgs& x, const AttnPlan& p, cudaStream_t s) {
+namespace {
+bool encode(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap* m, const void* ptr,
+            cuuint32_t rank, const cuuint64_t* dims, const cuuint64_t* strides,
+            const cuuint32_t* box) {
+  const cuuint32_t es[3] = {1, 1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(ptr), dims, strides, box,
+             es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+}  // namespace
+
+// Q and the block K/V as 3-D [B*Lb][heads][D], the caches as 2-D
+// [B*Hkv*Cmax][D]; boxes of 64 dims, 128-byte swizzled.
+bool attn_tc_encode(PFN_cuTensorMapEncodeTiled_v12000 enc, const AttnArgs& x, AttnTcMaps* m) {
+  const int G = x.Hq / x.Hkv;
+  const cuuint64_t rs = static_cast<cuuint64_t>(TC_D) * 2;
+  {
+    const cuuint64_t dims[3] = {TC_D, static_cast<cuuint64_t>(x.Hq),
+                                static_cast<cuuint64_t>(x.B) * x.Lb};
+    const cuuint64_t str[2] = {rs, rs * x.Hq};
+    const cuuint32_t box[3] = {64, static_cast<cuuint32_t>(G), static_cast<cuuint32_t>(TC_M / G)};
+    if (!encode(enc, &m->q, x.q, 3, dims, str, box)) return false;
+  }
+  {
+    const cuuint64_t dims[3] = {TC_D, static_cast<cuuint64_t>(x.Hkv),
+                                static_cast<cuuint64_t>(x.B) * x.Lb};
+    const cuuint64_t str[2] = {rs, rs * x.Hkv};
+    const cuuint32_t box[3] = {64, 1, TC_KT};
+    if (!encode(enc, &m->kb, x.k_blk, 3, dims, str, box)) return false;
+    if (!encode(enc, &m->vb, x.v_blk, 3, dims, str, box)) return false;
+  }
+  {
+    const cuuint64_t dims[2] = {TC_D, static_cast<cuuint64_t>(x.B) * x.Hkv * x.Cmax};
+    const cuuint64_t str[1] = {rs};
+    const cuuint32_t box[2] = {64, TC_KT};
+    if (!encode(enc, &m->kc, x.k_cache, 2, dims, str, box)) return false;
+    if (!encode(enc, &m->vc, x.v_cache, 2, dims, str, box)) return false;
+  }
+  return true;
+}
+
+cudaError_t launch_attention_tc(const AttnArgs& x, const AttnTcPlan& p, const AttnTcMaps& m,
+                                const AttnTcScratch& sc, cudaStream_t s) {
   TcArgs a;
-  a.q = static_cast<const __nv_bfloat16*>(x.q);
-  a.k_blk = static_cast<const __nv_bfloat16*>(x.k_blk);
-  a.v_blk = static_cast<const __nv_bfloat16*>(x.v_blk);
+  a.ctx = x.ctx;
   a.k_cache = static_cast<__nv_bfloat16*>(x.k_cache);
   a.v_cache = static_cast<__nv_bfloat16*>(x.v_cache);
-  a.ctx = x.ctx;
+  a.k_blk = static_cast<const __nv_bfloat16*>(x.k_blk);
+  a.v_blk = static_cast<const __nv_bfloat16*>(x.v_blk);
   a.out = static_cast<__nv_bfloat16*>(x.out);
+  a.part_o = sc.part_o;
+  a.part_ml = sc.part_ml;
+  a.counters = sc.counters;
+  a.status = x.status;
   a.B = x.B;
   a.Lb = x.Lb;
   a.Hq = x.Hq;
   a.Hkv = x.Hkv;
-  a.Cmax = x.Cmax;
   a.G = x.Hq / x.Hkv;
+  a.Cmax = x.Cmax;
   a.rows = p.rows;
-  a.splits = p.splits;
+  a.n_rg = p.n_rg;
+  a.chunk = p.chunk;
+  a.max_chunks = p.max_chunks;
   a.scale_log2 = LOG2E / sqrtf(static_cast<float>(x.D));
-  a.status = x.status;
+  a.kv_evict_first = p.n_rg == 1;  // with several row groups each K/V tile is read again
+  attention_tc_kernel<<<p.grid, TC_THREADS, p.smem_bytes, s>>>(m.q, m.kc, m.vc, m.kb, m.vb, a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess || p.max_chunks == 1) return e;
+
+  MergeArgs g;
+  g.ctx = x.ctx;
+  g.part_o = sc.part_o;
+  g.part_ml = sc.part_ml;
+  g.out = a.out;
+  g.Lb = x.Lb;
+  g.Hq = x.Hq;
+  g.Hkv = x.Hkv;
+  g.G = a.G;
+  g.Cmax = x.Cmax;
+  g.rows = p.rows;
+  g.n_rg = p.n_rg;
+  g.chunk = p.chunk;
+  g.max_chunks = p.max_chunks;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(p.splits, x.Hkv, x.B * ((p.rows + TC_ROWS - 1) / TC_ROWS));
-  cfg.blockDim = dim3(TC_THREADS, 1, 1);
-  cfg.dynamicSmemBytes = attn_tc_smem_bytes();
+  cfg.gridDim = dim3(x.B * x.Hkv * p.n_rg, (std::min(p.rows, TC_M) + 7) / 8, 1);
+  cfg.blockDim = dim3(256, 1, 1);
+  cfg.dynamicSmemBytes = 0;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = p.splits;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = p.splits > 1 ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, attention_tc_kernel<TC_KT, TC_STAGES>, a);
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, attention_merge_kernel, g);
 }
 
 }  // namespace rv

@@ -89,18 +89,13 @@ int head_tc_max_stages(int N, size_t smem_limit) {
 // Pipeline depth: about 128 KB of tiles in flight per SM streams the weight at
 // full HBM bandwidth (measured on GB300: 7-8 stages of 18 KB beat both 4-6 and
 // 11) and leaves room on the SM for the concurrent attention kernel.
+#ifndef RV_HEAD_STAGE_TARGET_KB
+#define RV_HEAD_STAGE_TARGET_KB 128
+#endif
 int head_tc_stages(int N, size_t smem_limit) {
   const int per = static_cast<int>(HT_A_BYTES) + N * 128;
-  const int want = (128 * 1024 + per - 1) / per;
+  const int want = (RV_HEAD_STAGE_TARGET_KB * 1024 + per - 1) / per;
   return std::max(2, std::min(head_tc_max_stages(N, smem_limit), std::max(4, want)));
-}
-
-// Wait used while draining after an abort: ignores the abort flag.
-__device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
-  const unsigned long long t0 = globaltimer_ns();
-  while (!mbar_try_wait(bar, parity)) {
-    if (globaltimer_ns() - t0 > RV_WAIT_TIMEOUT_NS / 4) return;
-  }
 }
 
 template <int EPI>

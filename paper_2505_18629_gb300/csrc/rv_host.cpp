@@ -36,6 +36,7 @@ struct Workspace {
   float* head_partials = nullptr;
   float* gathered = nullptr;
   void* hsel = nullptr;
+  AttnTcScratch attn{};  // tcgen05 attention: partial results, tickets, counters
   // staging for rv_verify_step_host
   void* st_q = nullptr;
   void* st_kb = nullptr;
@@ -84,6 +85,11 @@ struct rv_handle {
   unsigned long long launches = 0;
   int head_tc_stages_cached_N = -1;
   int head_tc_stages = 0;
+  bool attn_tc_ok = false;  // tcgen05 attention usable for this configuration
+  // tensor maps of the last tcgen05 attention call and what they were made for
+  AttnTcMaps attn_maps;
+  const void* attn_map_ptrs[5] = {nullptr, nullptr, nullptr, nullptr, nullptr};
+  int attn_map_B = -1, attn_map_Lb = -1;
 };
 
 namespace {
@@ -237,6 +243,13 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
   const size_t o_mg = take(static_cast<size_t>(c.max_batch) * c.max_gamma * 4);
   const size_t o_acc = take(static_cast<size_t>(c.max_batch) * c.max_gamma);
   const size_t o_al = take(c.max_batch * 4), o_nt = take(c.max_batch * 4);
+  h->attn_tc_ok = bf16 && attn_tc_supported(c.n_q_heads, c.n_kv_heads, c.head_dim) &&
+                  attn_tc_smem_max(c.max_batch) <= h->smem_optin;
+  const int a_slots =
+      h->attn_tc_ok ? attn_tc_max_slots(c.max_batch, Lbm, c.n_q_heads, c.n_kv_heads, h->num_sms) : 0;
+  const size_t o_apo = take(static_cast<size_t>(a_slots) * 128 * 128 * 4);
+  const size_t o_aml = take(static_cast<size_t>(a_slots) * 128 * 2 * 4);
+  const size_t o_act = take(64);
 
   e = cudaMalloc(&h->ws.base, off);
   if (e != cudaSuccess) {
@@ -249,6 +262,9 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
   h->ws.head_partials = reinterpret_cast<float*>(b + o_part);
   h->ws.gathered = reinterpret_cast<float*>(b + o_gath);
   h->ws.hsel = b + o_hsel;
+  h->ws.attn.part_o = reinterpret_cast<float*>(b + o_apo);
+  h->ws.attn.part_ml = reinterpret_cast<float*>(b + o_aml);
+  h->ws.attn.counters = reinterpret_cast<unsigned*>(b + o_act);
   h->ws.st_q = b + o_q;
   h->ws.st_kb = b + o_kb;
   h->ws.st_vb = b + o_vb;
@@ -272,7 +288,7 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming);
   if (e == cudaSuccess && bf16) e = attn_configure(&h->attn_max_cluster);
-  if (e == cudaSuccess && bf16) e = attn_tc_configure();
+  if (e == cudaSuccess && h->attn_tc_ok) e = attn_tc_configure(attn_tc_smem_max(c.max_batch));
   if (e == cudaSuccess && bf16) e = head_tc_configure(h->smem_optin);
   if (e == cudaSuccess && bf16) {
     cudaDriverEntryPointQueryResult q;
@@ -365,8 +381,24 @@ extern "C" RV_API int rv_verify_attention(rv_handle* h, const void* q, const voi
   cudaError_t e;
   if (bf16) {
     const AttnPlan p = attn_plan(B, Lb, c.n_q_heads, c.n_kv_heads, c.max_ctx, h->num_sms, true,
-                                 h->attn_max_cluster, c.head_dim);
-    e = p.tc ? launch_attention_tc(a, p, s) : launch_attention_bf16(a, p, s);
+                                 h->attn_max_cluster, c.head_dim, h->attn_tc_ok);
+    if (p.tc) {
+      const void* ptrs[5] = {q, k_blk, v_blk, k_cache, v_cache};
+      if (h->attn_map_B != B || h->attn_map_Lb != Lb ||
+          !std::equal(ptrs, ptrs + 5, h->attn_map_ptrs)) {
+        if (!attn_tc_encode(h->encode, a, &h->attn_maps)) {
+          h->attn_map_B = -1;
+          return fail(h, RV_ERR_CUDA, "cuTensorMapEncodeTiled(attention) failed");
+        }
+        std::copy(ptrs, ptrs + 5, h->attn_map_ptrs);
+        h->attn_map_B = B;
+        h->attn_map_Lb = Lb;
+      }
+      const AttnTcPlan tp = attn_tc_plan(B, Lb, c.n_q_heads, c.n_kv_heads, c.max_ctx, h->num_sms);
+      e = launch_attention_tc(a, tp, h->attn_maps, h->ws.attn, s);
+    } else {
+      e = launch_attention_bf16(a, p, s);
+    }
   } else {
     e = launch_attention_f32(a, s);
   }
@@ -545,13 +577,24 @@ extern "C" RV_API int rv_verify_step(
   if (do_pack && (!pos_ids || (n_prompt > 0 && !prompt_ids) || (n_prefix > 0 && !prefix_ids)))
     return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument for the block packing");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  // Fork: the attention (independent of the LM head) runs on the side stream
-  // and shares the SMs with the HBM-bound head; join before returning.
-  cudaError_t e = cudaEventRecord(h->ev_fork, s);
-  if (e == cudaSuccess) e = cudaStreamWaitEvent(h->side, h->ev_fork, 0);
-  if (e != cudaSuccess) return cuda_fail(h, e, "stream fork");
-  rc = rv_verify_attention(h, q, k_blk, v_blk, k_cache, v_cache, ctx_in, B, 2 * gamma + R,
-                           attn_out, h->side);
+  const rv_config& c = h->cfg;
+  const int Lb = 2 * gamma + R;
+  // Small batches: the attention (independent of the LM head) runs on the side
+  // stream and shares the SMs with the HBM-bound head; join before returning.
+  // Larger batches use the persistent tcgen05 attention, which fills every SM
+  // as the head does: there the two run one after the other on `stream`.
+  const bool fork = c.dtype != RV_DTYPE_BF16 ||
+                    !attn_plan(B, Lb, c.n_q_heads, c.n_kv_heads, c.max_ctx, h->num_sms, true,
+                               h->attn_max_cluster, c.head_dim, h->attn_tc_ok)
+                         .tc;
+  cudaError_t e = cudaSuccess;
+  if (fork) {
+    e = cudaEventRecord(h->ev_fork, s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(h->side, h->ev_fork, 0);
+    if (e != cudaSuccess) return cuda_fail(h, e, "stream fork");
+  }
+  rc = rv_verify_attention(h, q, k_blk, v_blk, k_cache, v_cache, ctx_in, B, Lb, attn_out,
+                           fork ? h->side : s);
   if (rc == RV_OK) {
     PackArgs pk{draft_ids, prompt_ids, prefix_ids, ctx_in, B, gamma, n_prompt, n_prefix, block_ids,
                 pos_ids};
@@ -559,9 +602,11 @@ extern "C" RV_API int rv_verify_step(
     rc = head_impl(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin,
                    do_pack ? &pk : nullptr, &ac, s);
   }
-  e = cudaEventRecord(h->ev_join, h->side);
-  if (e == cudaSuccess) e = cudaStreamWaitEvent(s, h->ev_join, 0);
-  if (e != cudaSuccess && rc == RV_OK) return cuda_fail(h, e, "stream join");
+  if (fork) {
+    e = cudaEventRecord(h->ev_join, h->side);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s, h->ev_join, 0);
+    if (e != cudaSuccess && rc == RV_OK) return cuda_fail(h, e, "stream join");
+  }
   return rc;
 }
 

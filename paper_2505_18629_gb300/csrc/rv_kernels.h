@@ -6,6 +6,7 @@
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_runtime.h>
+#include <cudaTypedefs.h>
 
 namespace rv {
 
@@ -148,15 +149,43 @@ struct AttnPlan {
   bool tc;         // tcgen05 kernel (head_dim 128, larger batches)
 };
 // max_cluster: largest thread-block cluster the attention kernel can use (<= 16)
+// allow_tc: the tcgen05 kernel may be chosen (its shapes and shared memory fit)
 AttnPlan attn_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms, bool bf16,
-                   int max_cluster, int D);
+                   int max_cluster, int D, bool allow_tc);
 size_t attn_bf16_smem_bytes(int D, int warps);
 cudaError_t attn_configure(int* max_cluster);
 cudaError_t launch_attention_bf16(const AttnArgs& a, const AttnPlan& p, cudaStream_t s);
 cudaError_t launch_attention_f32(const AttnArgs& a, cudaStream_t s);
-// tcgen05 attention (k_attention_tc.cu), head_dim 128
-size_t attn_tc_smem_bytes();
-cudaError_t attn_tc_configure();
-cudaError_t launch_attention_tc(const AttnArgs& a, const AttnPlan& p, cudaStream_t s);
+// tcgen05 attention (k_attention_tc.cu), head_dim 128: persistent CTAs that
+// claim (sequence, KV head, row group, key chunk) items, then (when a
+// sequence spans several chunks) a merge launch.
+struct AttnTcPlan {
+  int rows;        // query rows per KV head: Lb * G
+  int n_rg;        // row groups of 128
+  int chunk;       // cached keys per item
+  int max_chunks;  // chunks of a sequence at capacity
+  int slots;       // partial-result slots used: groups * max_chunks
+  int grid;        // CTAs
+  size_t smem_bytes;
+};
+struct AttnTcMaps {
+  CUtensorMap q;       // [B*Lb][Hq][D], box {64, G, 128/G}
+  CUtensorMap kc, vc;  // [B*Hkv*Cmax][D], box {64, 64}
+  CUtensorMap kb, vb;  // [B*Lb][Hkv][D], box {64, 1, 64}
+};
+struct AttnTcScratch {
+  float* part_o;       // [slots][128][128]
+  float* part_ml;      // [slots][128][2]
+  unsigned* counters;  // [2], zero between launches
+};
+AttnTcPlan attn_tc_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms);
+bool attn_tc_supported(int Hq, int Hkv, int D);
+size_t attn_tc_smem_max(int max_batch);
+// partial-result slots any launch within these maxima may use
+int attn_tc_max_slots(int max_batch, int Lb_max, int Hq, int Hkv, int num_sms);
+cudaError_t attn_tc_configure(size_t smem_bytes);
+bool attn_tc_encode(PFN_cuTensorMapEncodeTiled_v12000 enc, const AttnArgs& x, AttnTcMaps* m);
+cudaError_t launch_attention_tc(const AttnArgs& x, const AttnTcPlan& p, const AttnTcMaps& m,
+                                const AttnTcScratch& sc, cudaStream_t s);
 
 }  // namespace rv

@@ -13,13 +13,13 @@
 // chunks (one warp per row).
 //
 // Per CTA, warp-specialised:
-//   warp 0     claims items and loads with TMA: Q of the item (3-D box over
-//              [B*Lb][Hq][D] that selects the G heads of the KV head) into one
-//              of two Q buffers, then per tile of 128 keys the K and V tiles,
-//              from the cache ([B*Hkv*Cmax][D]) or, for the block's keys, from
-//              k_blk / v_blk (3-D box over [B*Lb][Hkv][D]), into a ring of stages
+//   warp 0     claims items and loads with TMA, per tile of 128 keys, the K
+//              and V tiles from the cache ([B*Hkv*Cmax][D]) or, for the
+//              block's keys, from k_blk / v_blk (3-D box over [B*Lb][Hkv][D])
+//              into a ring of stages
 //   warp 1     allocates TMEM and issues the MMAs from one thread:
-//                S_t  = Q K_t^T   (M 128, N 128, K 128) into S[t % 2]
+//                S_t  = Q K_t^T   (M 128, N 128, K 128) into S[t % 2]; Q is
+//                                 read from TMEM
 //                O   += P_t V_t   (M 128, N 128, K 128); P_t (bf16) is read from
 //                                 TMEM, where the softmax wrote it over the
 //                                 first half of S[t % 2]; V is used as stored,
@@ -28,10 +28,13 @@
 //              computes the next scores while the softmax runs; the MMAs of a
 //              CTA execute in issue order, so QK of tile t+2 overwrites S[t % 2]
 //              only after PV of tile t has read P_t
-//   warps 2-5  one thread per query row (its TMEM lane): online softmax of
-//              S_t (base-2, the 1/sqrt(D) scale folded into the exponent),
-//              lazy rescale of its O row (only when its max rises by more than
-//              2^8), and at the end of the item the O row: output or partial
+//   warps 2-5  one thread per query row (its TMEM lane): writes its Q row into
+//              TMEM, runs the online softmax of S_t (base-2, the 1/sqrt(D)
+//              scale folded into the exponent), rescales its O row lazily
+//              (only when its max rises by more than 2^8), and at the end of
+//              the item stores the O row (output or partial).  The next item's
+//              Q is written before this item's O is read out, so the tensor
+//              core starts the next item meanwhile.
 // Every wait is bounded (a timeout is reported in the status word).  The CTA
 // that handles the last chunk of (sequence, KV head) in row group 0 appends
 // the block's keys and values to the cache.
@@ -47,26 +50,26 @@ namespace {
 constexpr int TC_D = 128;
 constexpr int TC_M = 128;        // query rows per MMA tile
 constexpr int TC_KT = 128;       // keys per tile
-constexpr int TC_STAGES = 2;     // K/V ring depth
+constexpr int TC_STAGES = 3;     // K/V ring depth
 constexpr int TC_THREADS = 192;  // producer, MMA, 4 softmax warps
 constexpr int TC_IRING = 4;      // item ring between the producer and the consumers
 constexpr float TC_RESCALE_LOG2 = 8.f;
 
-constexpr uint32_t TC_Q_BYTES = TC_M * TC_D * 2;    // 32 KB: two 64-dim halves
 constexpr uint32_t TC_KV_BYTES = TC_KT * TC_D * 2;  // 32 KB: two halves of [128 keys][128 B]
-constexpr uint32_t TC_Q_OFF = 0;
-constexpr uint32_t TC_K_OFF = TC_Q_OFF + 2 * TC_Q_BYTES;
+constexpr uint32_t TC_K_OFF = 0;
 constexpr uint32_t TC_V_OFF = TC_K_OFF + TC_STAGES * TC_KV_BYTES;
 constexpr uint32_t TC_BAR_OFF = TC_V_OFF + TC_STAGES * TC_KV_BYTES;
 constexpr uint32_t TC_MISC_OFF = TC_BAR_OFF + 256;
 constexpr uint32_t TC_RING_OFF = TC_MISC_OFF + 16;  // TC_IRING items of 8 ints
 constexpr uint32_t TC_SCAN_OFF = TC_RING_OFF + TC_IRING * 32;
 // TMEM columns: S[0] [0, 128), S[1] [128, 256) (P_t over the first 64 columns
-// of S[t % 2], two bf16 per column), O [256, 384)
+// of S[t % 2], two bf16 per column), O [256, 384), Q [384, 448) (bf16 pairs)
 constexpr uint32_t TC_TMEM_COLS = 512;
 constexpr uint32_t TC_O_COL = 256;
+constexpr uint32_t TC_Q_COL = 384;
 
 struct TcArgs {
+  const __nv_bfloat16* q;
   const int32_t* ctx;
   __nv_bfloat16* k_cache;
   __nv_bfloat16* v_cache;
@@ -106,8 +109,7 @@ __device__ __forceinline__ int seq_chunks(int ctx, int Lb, int Cmax, int chunk) 
 }  // namespace
 
 __global__ void __launch_bounds__(TC_THREADS, 1)
-    attention_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
-                        const __grid_constant__ CUtensorMap tm_kc,
+    attention_tc_kernel(const __grid_constant__ CUtensorMap tm_kc,
                         const __grid_constant__ CUtensorMap tm_vc,
                         const __grid_constant__ CUtensorMap tm_kb,
                         const __grid_constant__ CUtensorMap tm_vb, const TcArgs a) {
@@ -118,8 +120,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   const uint32_t bars = base + TC_BAR_OFF;
-  auto q_full = [&](int i) { return bars + 8u * i; };  // 2 each
-  auto q_empty = [&](int i) { return bars + 16u + 8u * i; };
+  const uint32_t q_full = bars;  // Q of the next item is in TMEM (4 softmax warps)
   auto kv_full = [&](int i) { return bars + 32u + 8u * i; };  // TC_STAGES each
   auto kv_empty = [&](int i) { return bars + 32u + 8u * (TC_STAGES + i); };
   const uint32_t b2 = bars + 32u + 16u * TC_STAGES;
@@ -136,9 +137,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   int* const scan = reinterpret_cast<int*>(smem + TC_SCAN_OFF);  // [B + 1] first item of b
 
   if (threadIdx.x == 0) {
+    mbar_init(q_full, 4);
     for (int i = 0; i < 2; ++i) {
-      mbar_init(q_full(i), 1);
-      mbar_init(q_empty(i), 1);
       mbar_init(s_full(i), 1);
       mbar_init(p_full(i), 4);
       mbar_init(o_done(i), 1);
@@ -174,7 +174,6 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     }
     if (lane == 0) {
       scan[a.B] = carry;
-      tma_prefetch_desc(&tm_q);
       tma_prefetch_desc(&tm_kc);
       tma_prefetch_desc(&tm_vc);
       tma_prefetch_desc(&tm_kb);
@@ -192,11 +191,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
-      const uint64_t pol_q = policy_evict_last();
+      const uint64_t pol_blk = policy_evict_last();
       const uint64_t pol_kv = a.kv_evict_first ? policy_evict_first() : policy_evict_normal();
       const int total = scan[a.B];
-      const int rows_j = TC_M / a.G;  // block positions per row group
-      int u = 0, it = 0, issued_q = 0;
+      int u = 0;
       bool ok = true;
       for (int lt = 0; ok; ++lt) {
         const int i = static_cast<int>(atomicAdd(&a.counters[0], 1u));
@@ -239,17 +237,6 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         if (item.b < 0) break;
         const int n = item_tiles(item, a.Lb);
         if (n == 0) continue;
-        const int qb = it & 1;
-        if (!mbar_wait(q_empty(qb), ((it >> 1) & 1) ^ 1u, abort_flag, a.status)) {
-          ok = false;
-          break;
-        }
-        mbar_arrive_expect_tx(q_full(qb), TC_Q_BYTES);
-        const int qz = item.b * a.Lb + item.rg * rows_j;
-        const uint32_t qd = base + TC_Q_OFF + qb * TC_Q_BYTES;
-        tma_load_3d(qd, &tm_q, 0, item.kvh * a.G, qz, q_full(qb), pol_q);
-        tma_load_3d(qd + TC_Q_BYTES / 2, &tm_q, 64, item.kvh * a.G, qz, q_full(qb), pol_q);
-        ++issued_q;
         const int n_cache = item_cache_tiles(item);
         const int row_c = (item.b * a.Hkv + item.kvh) * a.Cmax;
         for (int j = 0; j < n; ++j) {
@@ -269,20 +256,17 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             tma_load_2d(vd + TC_KV_BYTES / 2, &tm_vc, 64, y, kv_full(st), pol_kv);
           } else {
             const int z = item.b * a.Lb + (j - n_cache) * TC_KT;
-            tma_load_3d(kd, &tm_kb, 0, item.kvh, z, kv_full(st), pol_q);
-            tma_load_3d(kd + TC_KV_BYTES / 2, &tm_kb, 64, item.kvh, z, kv_full(st), pol_q);
-            tma_load_3d(vd, &tm_vb, 0, item.kvh, z, kv_full(st), pol_q);
-            tma_load_3d(vd + TC_KV_BYTES / 2, &tm_vb, 64, item.kvh, z, kv_full(st), pol_q);
+            tma_load_3d(kd, &tm_kb, 0, item.kvh, z, kv_full(st), pol_blk);
+            tma_load_3d(kd + TC_KV_BYTES / 2, &tm_kb, 64, item.kvh, z, kv_full(st), pol_blk);
+            tma_load_3d(vd, &tm_vb, 0, item.kvh, z, kv_full(st), pol_blk);
+            tma_load_3d(vd + TC_KV_BYTES / 2, &tm_vb, 64, item.kvh, z, kv_full(st), pol_blk);
           }
           ++u;
         }
-        ++it;
       }
       if (!ok) {  // let the copies still in flight land before the CTA exits
         for (int v = max(0, u - TC_STAGES); v < u; ++v)
           drain_wait(kv_full(v % TC_STAGES), static_cast<uint32_t>((v / TC_STAGES) & 1));
-        for (int qq = max(0, issued_q - 2); qq < issued_q; ++qq)
-          drain_wait(q_full(qq & 1), static_cast<uint32_t>((qq >> 1) & 1));
       }
     }
     __syncwarp();
@@ -319,9 +303,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         if (item.b < 0) break;
         const int n = item_tiles(item, a.Lb);
         if (n == 0) continue;
-        const int qb = it & 1;
-        if (!mbar_wait(q_full(qb), (it >> 1) & 1, abort_flag, a.status)) break;
-        const uint32_t qbase = base + TC_Q_OFF + qb * TC_Q_BYTES;
+        if (!mbar_wait(q_full, it & 1, abort_flag, a.status)) break;
+        tc_fence_after();
         for (int j = 0; j < n && ok; ++j) {
           const int v = u + j;
           const int st = v % TC_STAGES;
@@ -335,13 +318,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           for (int kk = 0; kk < TC_D / 16; ++kk) {
             const uint32_t half = static_cast<uint32_t>(kk >> 2);
             const uint32_t off = static_cast<uint32_t>((kk & 3) * 32);
-            tc_mma_bf16(tmem + static_cast<uint32_t>((v & 1) * TC_KT),
-                        sw128_kmajor_desc(qbase + half * (TC_Q_BYTES / 2) + off),
-                        sw128_kmajor_desc(kb + half * (TC_KV_BYTES / 2) + off), idesc_s,
-                        kk > 0 ? 1u : 0u);
+            tc_mma_bf16_tmem_a(tmem + static_cast<uint32_t>((v & 1) * TC_KT), tmem + TC_Q_COL + kk * 8,
+                               sw128_kmajor_desc(kb + half * (TC_KV_BYTES / 2) + off), idesc_s,
+                               kk > 0 ? 1u : 0u);
           }
           tc_commit(s_full(v & 1));
-          if (j == n - 1) tc_commit(q_empty(qb));
           if (j > 0 && !issue_pv(v - 1, j == 1)) ok = false;
         }
         if (ok && !issue_pv(u + n - 1, n == 1)) ok = false;
@@ -359,17 +340,63 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     const int r = q * 32 + lane;  // query row within the row group (TMEM lane)
     const int st_tid = threadIdx.x - 64;
     const uint32_t t_row = tmem + (static_cast<uint32_t>(q * 32) << 16);
-    int u = 0;
-    for (int lt = 0;; ++lt) {
-      const int k = lt % TC_IRING;
-      bool ok = mbar_wait(r_full(k), (lt / TC_IRING) & 1, abort_flag, a.status);
-      if (!__all_sync(0xffffffffu, ok)) break;
-      const Item item = ring[k];
+    int lt = 0;
+    bool live = true;
+    // next ring entry with tiles (or the end); every entry is acknowledged
+    auto next_item = [&](Item& it) -> bool {
+      for (;;) {
+        const int k = lt % TC_IRING;
+        const bool ok = mbar_wait(r_full(k), (lt / TC_IRING) & 1, abort_flag, a.status);
+        if (!__all_sync(0xffffffffu, ok)) return false;
+        it = ring[k];
+        __syncwarp();
+        if (lane == 0) mbar_arrive(r_empty(k));
+        ++lt;
+        if (it.b < 0 || item_tiles(it, a.Lb) > 0) return true;
+      }
+    };
+    // this row of the item's Q: global -> registers (issued early) -> TMEM
+    uint4 qv[16];
+    auto q_fetch = [&](const Item& it) {
+      const int gr = it.rg * TC_M + r;
+      if (gr < a.rows) {
+        const uint4* src = reinterpret_cast<const uint4*>(
+            a.q + ((static_cast<long long>(it.b) * a.Lb + gr / a.G) * a.Hq + it.kvh * a.G + gr % a.G) * TC_D);
+#pragma unroll
+        for (int c = 0; c < 16; ++c) qv[c] = __ldg(src + c);
+      } else {
+#pragma unroll
+        for (int c = 0; c < 16; ++c) qv[c] = make_uint4(0u, 0u, 0u, 0u);
+      }
+    };
+    auto q_store = [&]() {
+#pragma unroll
+      for (int h = 0; h < 4; ++h) {
+        uint32_t w[16];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          w[4 * c] = qv[4 * h + c].x;
+          w[4 * c + 1] = qv[4 * h + c].y;
+          w[4 * c + 2] = qv[4 * h + c].z;
+          w[4 * c + 3] = qv[4 * h + c].w;
+        }
+        tmem_st16(t_row + TC_Q_COL + 16 * h, w);
+      }
+      tmem_st_wait();
+      tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(r_empty(k));
-      if (item.b < 0) break;
+      if (lane == 0) mbar_arrive(q_full);
+    };
+
+    Item item;
+    live = next_item(item);
+    if (live && item.b >= 0) {
+      q_fetch(item);
+      q_store();
+    }
+    int u = 0;
+    while (live && item.b >= 0) {
       const int n = item_tiles(item, a.Lb);
-      if (n == 0) continue;
       const int n_cache = item_cache_tiles(item);
       const int ctx = item.ctx;
       const int gr = item.rg * TC_M + r;  // row among the Lb*G rows of (sequence, KV head)
@@ -391,14 +418,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       }
 
       float m_used = NEG_INF, l = 0.f;  // running max (log2 units) and sum of this row
-      bool good = true;
-      for (int j = 0; j < n; ++j) {
+      for (int j = 0; j < n && live; ++j) {
         const int v = u + j;
         const int sb = v & 1;
         const uint32_t s_col = t_row + static_cast<uint32_t>(sb * TC_KT);
-        ok = mbar_wait(s_full(sb), (v >> 1) & 1, abort_flag, a.status);
+        bool ok = mbar_wait(s_full(sb), (v >> 1) & 1, abort_flag, a.status);
         if (!__all_sync(0xffffffffu, ok)) {
-          good = false;
+          live = false;
           break;
         }
         tc_fence_after();
@@ -440,7 +466,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         if (j > 0 && __any_sync(0xffffffffu, rise && fac != 1.f)) {
           ok = mbar_wait(o_done((v - 1) & 1), ((v - 1) >> 1) & 1, abort_flag, a.status);
           if (!__all_sync(0xffffffffu, ok)) {
-            good = false;
+            live = false;
             break;
           }
           tc_fence_after();
@@ -476,50 +502,64 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(p_full(sb));
       }
-      if (!good) break;
+      if (!live) break;
+
+      // ---- the next item's Q goes to TMEM first (every QK of this item is
+      // complete), so its first scores are computed during this item's end
+      Item nxt;
+      live = next_item(nxt);
+      if (!live) break;
+      if (nxt.b >= 0) {
+        q_fetch(nxt);
+        q_store();
+      }
+
       // ---- item end: this row's O
       const int vl = u + n - 1;
-      ok = mbar_wait(o_done(vl & 1), (vl >> 1) & 1, abort_flag, a.status);
+      bool ok = mbar_wait(o_done(vl & 1), (vl >> 1) & 1, abort_flag, a.status);
       if (!__all_sync(0xffffffffu, ok)) break;
       tc_fence_after();
       u += n;
-      const float inv = (l > 0.f) ? 1.f / l : 0.f;
-      const int group = (item.b * a.Hkv + item.kvh) * a.n_rg + item.rg;
-      const int slot = group * a.max_chunks + item.c;
-      const long long orow = (static_cast<long long>(item.b) * a.Lb + gr / a.G) * a.Hq +
-                             item.kvh * a.G + gr % a.G;
-      float* const po = a.part_o + (static_cast<long long>(slot) * TC_M + r) * TC_D;
+      float ov[4][32];
 #pragma unroll
-      for (int c = 0; c < TC_D; c += 32) {
-        float ov[32];
-        tmem_ld32(t_row + TC_O_COL + c, ov);
-        tmem_ld_wait();
-        if (rvalid) {
-          if (item.nch == 1) {
-            __nv_bfloat16* dst = a.out + orow * TC_D + c;
-#pragma unroll
-            for (int i = 0; i < 32; i += 8) {
-              uint4 pk;
-              pk.x = pack_bf16(ov[i] * inv, ov[i + 1] * inv);
-              pk.y = pack_bf16(ov[i + 2] * inv, ov[i + 3] * inv);
-              pk.z = pack_bf16(ov[i + 4] * inv, ov[i + 5] * inv);
-              pk.w = pack_bf16(ov[i + 6] * inv, ov[i + 7] * inv);
-              *reinterpret_cast<uint4*>(dst + i) = pk;
-            }
-          } else {
-#pragma unroll
-            for (int i = 0; i < 32; i += 4)
-              __stcg(reinterpret_cast<float4*>(po + c + i),
-                     make_float4(ov[i] * inv, ov[i + 1] * inv, ov[i + 2] * inv, ov[i + 3] * inv));
-          }
-        }
-      }
-      if (rvalid && item.nch > 1)
-        __stcg(reinterpret_cast<float2*>(a.part_ml) + static_cast<long long>(slot) * TC_M + r,
-               make_float2(m_used, l));
+      for (int c = 0; c < 4; ++c) tmem_ld32(t_row + TC_O_COL + 32 * c, ov[c]);
+      tmem_ld_wait();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(o_free);
+      const float inv = (l > 0.f) ? 1.f / l : 0.f;
+      const int group = (item.b * a.Hkv + item.kvh) * a.n_rg + item.rg;
+      const int slot = group * a.max_chunks + item.c;
+      if (rvalid) {
+        if (item.nch == 1) {
+          const long long orow = (static_cast<long long>(item.b) * a.Lb + gr / a.G) * a.Hq +
+                                 item.kvh * a.G + gr % a.G;
+          __nv_bfloat16* dst = a.out + orow * TC_D;
+#pragma unroll
+          for (int c = 0; c < 4; ++c)
+#pragma unroll
+            for (int i = 0; i < 32; i += 8) {
+              uint4 pk;
+              pk.x = pack_bf16(ov[c][i] * inv, ov[c][i + 1] * inv);
+              pk.y = pack_bf16(ov[c][i + 2] * inv, ov[c][i + 3] * inv);
+              pk.z = pack_bf16(ov[c][i + 4] * inv, ov[c][i + 5] * inv);
+              pk.w = pack_bf16(ov[c][i + 6] * inv, ov[c][i + 7] * inv);
+              *reinterpret_cast<uint4*>(dst + 32 * c + i) = pk;
+            }
+        } else {
+          float* const po = a.part_o + (static_cast<long long>(slot) * TC_M + r) * TC_D;
+#pragma unroll
+          for (int c = 0; c < 4; ++c)
+#pragma unroll
+            for (int i = 0; i < 32; i += 4)
+              __stcg(reinterpret_cast<float4*>(po + 32 * c + i),
+                     make_float4(ov[c][i] * inv, ov[c][i + 1] * inv, ov[c][i + 2] * inv,
+                                 ov[c][i + 3] * inv));
+          __stcg(reinterpret_cast<float2*>(a.part_ml) + static_cast<long long>(slot) * TC_M + r,
+                 make_float2(m_used, l));
+        }
+      }
+      item = nxt;
     }
   }
 
@@ -650,18 +690,10 @@ bool encode(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap* m, const void* p
 }
 }  // namespace
 
-// Q and the block K/V as 3-D [B*Lb][heads][D], the caches as 2-D
-// [B*Hkv*Cmax][D]; boxes of 64 dims, 128-byte swizzled.
+// The block K/V as 3-D [B*Lb][Hkv][D], the caches as 2-D [B*Hkv*Cmax][D];
+// boxes of 64 dims x 128 keys, 128-byte swizzled.
 bool attn_tc_encode(PFN_cuTensorMapEncodeTiled_v12000 enc, const AttnArgs& x, AttnTcMaps* m) {
-  const int G = x.Hq / x.Hkv;
   const cuuint64_t rs = static_cast<cuuint64_t>(TC_D) * 2;
-  {
-    const cuuint64_t dims[3] = {TC_D, static_cast<cuuint64_t>(x.Hq),
-                                static_cast<cuuint64_t>(x.B) * x.Lb};
-    const cuuint64_t str[2] = {rs, rs * x.Hq};
-    const cuuint32_t box[3] = {64, static_cast<cuuint32_t>(G), static_cast<cuuint32_t>(TC_M / G)};
-    if (!encode(enc, &m->q, x.q, 3, dims, str, box)) return false;
-  }
   {
     const cuuint64_t dims[3] = {TC_D, static_cast<cuuint64_t>(x.Hkv),
                                 static_cast<cuuint64_t>(x.B) * x.Lb};
@@ -683,6 +715,7 @@ bool attn_tc_encode(PFN_cuTensorMapEncodeTiled_v12000 enc, const AttnArgs& x, At
 cudaError_t launch_attention_tc(const AttnArgs& x, const AttnTcPlan& p, const AttnTcMaps& m,
                                 const AttnTcScratch& sc, cudaStream_t s) {
   TcArgs a;
+  a.q = static_cast<const __nv_bfloat16*>(x.q);
   a.ctx = x.ctx;
   a.k_cache = static_cast<__nv_bfloat16*>(x.k_cache);
   a.v_cache = static_cast<__nv_bfloat16*>(x.v_cache);
@@ -705,7 +738,7 @@ cudaError_t launch_attention_tc(const AttnArgs& x, const AttnTcPlan& p, const At
   a.max_chunks = p.max_chunks;
   a.scale_log2 = LOG2E / sqrtf(static_cast<float>(x.D));
   a.kv_evict_first = p.n_rg == 1;  // with several row groups each K/V tile is read again
-  attention_tc_kernel<<<p.grid, TC_THREADS, p.smem_bytes, s>>>(m.q, m.kc, m.vc, m.kb, m.vb, a);
+  attention_tc_kernel<<<p.grid, TC_THREADS, p.smem_bytes, s>>>(m.kc, m.vc, m.kb, m.vb, a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || p.max_chunks == 1) return e;
 

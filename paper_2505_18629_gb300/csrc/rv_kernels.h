@@ -169,9 +169,8 @@ struct AttnTcPlan {
   size_t smem_bytes;
 };
 struct AttnTcMaps {
-  CUtensorMap q;       // [B*Lb][Hq][D], box {64, G, 128/G}
-  CUtensorMap kc, vc;  // [B*Hkv*Cmax][D], box {64, 64}
-  CUtensorMap kb, vb;  // [B*Lb][Hkv][D], box {64, 1, 64}
+  CUtensorMap kc, vc;  // [B*Hkv*Cmax][D], box {64, 128}
+  CUtensorMap kb, vb;  // [B*Lb][Hkv][D], box {64, 1, 128}
 };
 struct AttnTcScratch {
   float* part_o;       // [slots][128][128]

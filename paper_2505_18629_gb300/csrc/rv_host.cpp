@@ -85,6 +85,10 @@ struct rv_handle {
   unsigned long long launches = 0;
   int head_tc_stages_cached_N = -1;
   int head_tc_stages = 0;
+  int head_pair_cached_N = -1;   // pair kernel: stages and co-resident pairs for this N
+  int head_pair_stages = 0;
+  int head_pair_max = 0;
+  int tm_h_box = -1;
   bool attn_tc_ok = false;  // tcgen05 attention usable for this configuration
   // tensor maps of the last tcgen05 attention call and what they were made for
   AttnTcMaps attn_maps;
@@ -122,6 +126,7 @@ HeadPlan head_plan(int B, int gamma, int V, int num_sms, bool tc) {
   p.pad_pairs = (p.pairs_per_chunk + 7) / 8 * 8;
   p.N = 2 * p.pad_pairs;
   p.n_vtiles = (V + 127) / 128;
+  p.pair = false;
   if (tc) {  // one persistent CTA per SM; the vocab is split in whole tiles
     p.slots = std::max(1, std::min(num_sms / p.n_chunks, p.n_vtiles));
   } else {
@@ -290,6 +295,7 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
   if (e == cudaSuccess && bf16) e = attn_configure(&h->attn_max_cluster);
   if (e == cudaSuccess && h->attn_tc_ok) e = attn_tc_configure(attn_tc_smem_max(c.max_batch));
   if (e == cudaSuccess && bf16) e = head_tc_configure(h->smem_optin);
+  if (e == cudaSuccess && bf16) e = head_tc2_configure(h->smem_optin);
   if (e == cudaSuccess && bf16) {
     cudaDriverEntryPointQueryResult q;
     void* fn = nullptr;
@@ -433,10 +439,11 @@ int encode_maps(rv_handle* h, const void* w, const HeadPlan& pl, HeadTcLaunch& l
     h->tm_w_ptr = w;
   }
   const int rows = pl.n_chunks * pl.N;
-  if (h->tm_h_N != pl.N || h->tm_h_rows != rows) {
+  const int box_rows = pl.pair ? pl.N / 2 : pl.N;
+  if (h->tm_h_N != pl.N || h->tm_h_rows != rows || h->tm_h_box != box_rows) {
     const cuuint64_t dims[2] = {static_cast<cuuint64_t>(c.hidden), static_cast<cuuint64_t>(rows)};
     const cuuint64_t strides[1] = {static_cast<cuuint64_t>(c.hidden) * 2};
-    const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(pl.N)};
+    const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(box_rows)};
     const cuuint32_t es[2] = {1, 1};
     CUresult r = h->encode(&h->tm_h, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, h->ws.hsel, dims, strides,
                            box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -447,10 +454,17 @@ int encode_maps(rv_handle* h, const void* w, const HeadPlan& pl, HeadTcLaunch& l
     }
     h->tm_h_N = pl.N;
     h->tm_h_rows = rows;
+    h->tm_h_box = box_rows;
   }
   l.tm_w = h->tm_w;
   l.tm_w16 = h->tm_w16;
   l.tm_h = h->tm_h;
+  if (pl.pair) {
+    l.stages = h->head_pair_stages;
+    l.unit_rows = HEAD_TILE_ROWS;
+    l.smem_bytes = head_tc2_smem_bytes(pl.N, l.stages);
+    return RV_OK;
+  }
   if (h->head_tc_stages_cached_N != pl.N) {
     h->head_tc_stages = head_tc_stages(pl.N, h->smem_optin);
     h->head_tc_stages_cached_N = pl.N;
@@ -488,7 +502,22 @@ int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_
              h->ws.head_partials, h->ws.gathered, h->ws.status,
              bf16 ? h->ws.status + 16 : nullptr,    // tile counter: its own 64-byte line
              bf16 ? h->ws.status + 32 : nullptr};   // finished-CTA counter
-  const HeadPlan pl = head_plan(B, gamma, c.vocab, h->num_sms, bf16);
+  HeadPlan pl = head_plan(B, gamma, c.vocab, h->num_sms, bf16);
+  if (bf16 && pl.N >= HEAD_PAIR_MIN_N) {
+    // CTA pairs: as many as fit at once (two CTAs of a pair share a GPC)
+    if (h->head_pair_cached_N != pl.N) {
+      h->head_pair_stages = head_tc2_stages(pl.N, h->smem_optin);
+      h->head_pair_max =
+          h->head_pair_stages >= 2 ? head_tc2_max_pairs(pl.N, h->head_pair_stages) : 0;
+      h->head_pair_cached_N = pl.N;
+    }
+    const int n_pt = (c.vocab + 255) / 256;
+    const int pairs = std::min({h->num_sms / 2 / pl.n_chunks, h->head_pair_max / pl.n_chunks, n_pt});
+    if (pairs >= 1) {
+      pl.pair = true;
+      pl.slots = 2 * pairs;
+    }
+  }
   ProfScope prof_all(h, RV_PROF_HEAD, s);
   cudaError_t e = cudaSuccess;
   HeadTcLaunch l;
@@ -506,7 +535,9 @@ int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_
   HeadFinal fin{scores, argmax, margin, acc ? *acc : AcceptArgs{}};
   {
     ProfScope prof(h, RV_PROF_HEAD_GEMM, s);
-    e = bf16 ? launch_head_tc(a, pl, l, fused ? &fin : nullptr, s) : launch_head_simt(a, pl, s);
+    e = !bf16    ? launch_head_simt(a, pl, s)
+        : pl.pair ? launch_head_tc2(a, pl, l, fused ? &fin : nullptr, s)
+                  : launch_head_tc(a, pl, l, fused ? &fin : nullptr, s);
     h->launches += 1;
   }
   if (e != cudaSuccess) return cuda_fail(h, e, "LM head launch");

@@ -39,6 +39,7 @@ struct HeadPlan {
   int N;               // 2*Pcp: MMA N (columns of the TMEM accumulator)
   int n_vtiles;        // ceil(V / 128)
   int slots;           // CTAs per chunk (= partial slots)
+  bool pair;           // CTA-pair kernel (k_head_tc2.cu): slots = 2 * pairs
 };
 
 // Optional acceptance fused into the head merge (rv_verify_step).
@@ -128,6 +129,20 @@ cudaError_t head_tc_configure(size_t smem_bytes);  // cudaFuncSetAttribute
 cudaError_t launch_head_tc(const HeadArgs& a, const HeadPlan& p, const HeadTcLaunch& l,
                            const HeadFinal* fin, cudaStream_t s);
 cudaError_t launch_head_simt(const HeadArgs& a, const HeadPlan& p, cudaStream_t s);
+// CTA-pair LM head (k_head_tc2.cu, tcgen05 cta_group::2): 256-row vocab tiles,
+// each CTA of a pair stages its 128 weight rows and half of the N hidden rows
+// (tm_h box {64, N/2}); the grid is p.slots (= 2 * pairs) x n_chunks in
+// clusters of 2.
+#ifndef RV_HEAD_PAIR_MIN_N
+#define RV_HEAD_PAIR_MIN_N 96
+#endif
+constexpr int HEAD_PAIR_MIN_N = RV_HEAD_PAIR_MIN_N;  // N from which pairs are used
+size_t head_tc2_smem_bytes(int N, int stages);
+int head_tc2_stages(int N, size_t smem_limit);
+cudaError_t head_tc2_configure(size_t smem_bytes);
+int head_tc2_max_pairs(int N, int stages);  // co-resident CTA pairs (occupancy query)
+cudaError_t launch_head_tc2(const HeadArgs& a, const HeadPlan& p, const HeadTcLaunch& l,
+                            const HeadFinal* fin, cudaStream_t s);
 
 // ---- attention (k_attention.cu)
 struct AttnArgs {

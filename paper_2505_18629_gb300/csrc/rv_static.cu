@@ -125,6 +125,7 @@ extern "C" RV_API int rv_verify_head_static(const void* hidden, const void* w_he
 
   // One chunk of P <= RV_STATIC_MAX_PAIRS pairs; vocab split in whole tiles.
   HeadPlan pl;
+  pl.pair = false;
   pl.P = B * (gamma + 1);
   pl.n_chunks = 1;
   pl.pairs_per_chunk = pl.P;

@@ -130,6 +130,88 @@ __device__ __forceinline__ void head_tile_pairs8(const float (&o)[8], const floa
   }
 }
 
+// Transposed variant of head_tile_pairs8 for the tensor-core kernels: the
+// warp stages its 32 rows x (o, r, z) of the eight pairs in shared memory
+// (`scr`: HEAD_SCR_FLOATS per warp), and lane c < 24 reduces column c (pair
+// c % 8; o, r or z for c / 8) over the 32 rows with plain loads - no shuffle
+// trees - then folds the result into the warp's running statistics.  Same
+// results as the shuffle version up to the order of the sums.
+constexpr int HEAD_SCR_STRIDE = 28;  // floats per staged row: 24 used, 16-byte aligned rows
+constexpr int HEAD_SCR_FLOATS = 32 * HEAD_SCR_STRIDE;
+
+__device__ __forceinline__ void head_tile_pairs8_t(const float (&o)[8], const float (&r)[8], int g8,
+                                                   int npairs, int v, bool valid, float alpha,
+                                                   const int* s_drafts, float* warp_stats,
+                                                   float* gathered, float* scr, int lane) {
+  const float beta = 1.f - alpha;
+  float zr[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const int pj = g8 + j;
+    zr[j] = fmaf(alpha, r[j], beta * o[j]);
+    if (valid && v == s_drafts[pj] && pj < npairs) {
+      float* gx = gathered + pj * GATHER_FIELDS;
+      gx[0] = o[j];
+      gx[1] = r[j];
+      gx[2] = zr[j];
+    }
+  }
+  float4* const row = reinterpret_cast<float4*>(scr + lane * HEAD_SCR_STRIDE);
+  const float ninf = NEG_INF;
+  row[0] = valid ? make_float4(o[0], o[1], o[2], o[3]) : make_float4(ninf, ninf, ninf, ninf);
+  row[1] = valid ? make_float4(o[4], o[5], o[6], o[7]) : make_float4(ninf, ninf, ninf, ninf);
+  row[2] = valid ? make_float4(r[0], r[1], r[2], r[3]) : make_float4(ninf, ninf, ninf, ninf);
+  row[3] = valid ? make_float4(r[4], r[5], r[6], r[7]) : make_float4(ninf, ninf, ninf, ninf);
+  row[4] = valid ? make_float4(zr[0], zr[1], zr[2], zr[3]) : make_float4(ninf, ninf, ninf, ninf);
+  row[5] = valid ? make_float4(zr[4], zr[5], zr[6], zr[7]) : make_float4(ninf, ninf, ninf, ninf);
+  __syncwarp();
+  if (lane < 24) {
+    const int j = lane & 7, kind = lane >> 3;  // 0: o, 1: r, 2: z
+    const int pj = g8 + j;
+    float val[32];
+    float m = NEG_INF;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      val[i] = scr[i * HEAD_SCR_STRIDE + lane];
+      m = fmaxf(m, val[i]);
+    }
+    float sum = 0.f;
+    if (m != NEG_INF) {
+      float s2[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int i = 0; i < 32; ++i) s2[i & 3] += __expf(val[i] - m);
+      sum = (s2[0] + s2[1]) + (s2[2] + s2[3]);
+    }
+    if (pj < npairs) {
+      float* st = warp_stats + pj * HEAD_STAT_STRIDE;
+      if (kind == 0) {
+        lse_merge(st[ST_M_O], st[ST_S_O], m, sum);
+      } else if (kind == 1) {
+        lse_merge(st[ST_M_R], st[ST_S_R], m, sum);
+      } else {
+        lse_merge(st[ST_M_Z], st[ST_S_Z], m, sum);
+        // best z over the rows v != x_i (lowest row on ties)
+        const int x = s_drafts[pj];
+        const int v0 = v - lane;  // vocab row of staged row 0
+        float bv = NEG_INF;
+        int bi = INT_MAX;
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          if (val[i] > bv && v0 + i != x) {
+            bv = val[i];
+            bi = v0 + i;
+          }
+        const int si = __float_as_int(st[ST_BEST_I]);
+        if (bv > st[ST_BEST_V] || (bv == st[ST_BEST_V] && bi < si)) {
+          st[ST_BEST_V] = bv;
+          st[ST_BEST_I] = __int_as_float(bi);
+        }
+      }
+    }
+  }
+  __syncwarp();  // the staging rows are reused by the next group
+}
+
 // Combine the warps' tables (each `tab` pairs long) into one partial per pair
 // and store it.  `out` points at partials[slot][chunk's first pair].
 __device__ __forceinline__ void head_stats_finish(const float* stats, int nwarps, int tab,

@@ -71,8 +71,10 @@ static int ht_epi_warps(int N) { return N / 2 <= HT_SMALL_PAIRS ? 4 : 8; }
 
 static size_t ht_fixed_bytes(int N) {
   // alignment slack + barriers/tile ring/misc + drafts + per-warp statistics (Pcp = N/2 pairs)
+  // + per-warp staging rows of the tile reduction
   return 1024 + 512 + MAX_PAIRS_PER_CHUNK * 4 +
-         static_cast<size_t>(ht_epi_warps(N)) * (N / 2) * HEAD_STAT_STRIDE * 4;
+         static_cast<size_t>(4) * (N / 2) * HEAD_STAT_STRIDE * 4 + 16 +
+         static_cast<size_t>(ht_epi_warps(N)) * HEAD_SCR_FLOATS * 4;
 }
 
 size_t head_tc_smem_bytes(int N, int stages) {
@@ -132,6 +134,9 @@ __global__ void __launch_bounds__(ht_threads(EPI), 1)
   float* const stats =
       reinterpret_cast<float*>(gbase + (misc - base) + 16 + 8 * HT_TRING + MAX_PAIRS_PER_CHUNK * 4);
   const int tab = p.Pcp;  // pairs per statistics table
+  // per-warp staging rows of the transposed tile reduction (16-byte aligned)
+  float* const scr_base = reinterpret_cast<float*>(
+      (reinterpret_cast<uintptr_t>(stats + 4 * tab * HEAD_STAT_STRIDE) + 15) & ~uintptr_t(15));
 
   const int pair0 = chunk * p.Pc;
   const int npairs = min(p.Pc, p.P - pair0);
@@ -167,7 +172,7 @@ __global__ void __launch_bounds__(ht_threads(EPI), 1)
     const int e = threadIdx.x - 64;
     for (int j = e; j < MAX_PAIRS_PER_CHUNK; j += EPI * 32)
       s_drafts[j] = (j < npairs) ? pair_draft(p.drafts, pair0 + j, p.gamma) : -1;
-    head_stats_init(stats, EPI * tab, e, EPI * 32);
+    head_stats_init(stats, 4 * tab, e, EPI * 32);
   }
   tc_fence_before();
   __syncthreads();
@@ -285,7 +290,8 @@ __global__ void __launch_bounds__(ht_threads(EPI), 1)
     const int q = warp & 3;       // TMEM lane quadrant this warp may access
     const int ew = warp - 2;      // statistics table of this warp
     const int half = ew >> 2;     // which alternate groups of 8 pairs it takes
-    float* const wstats = stats + ew * tab * HEAD_STAT_STRIDE;
+    // the two warps of a quadrant take disjoint pairs: they share one table
+    float* const wstats = stats + q * tab * HEAD_STAT_STRIDE;
     float* const gathered = p.gathered + static_cast<long long>(pair0) * GATHER_FIELDS;
     for (int lt = 0;; ++lt) {
       const int k = lt % HT_TRING;
@@ -309,14 +315,15 @@ __global__ void __launch_bounds__(ht_threads(EPI), 1)
         tmem_ld8(trow + g8, o);
         tmem_ld8(trow + p.Pcp + g8, r);
         tmem_ld_wait();
-        head_tile_pairs8(o, r, g8, npairs, v, valid, p.alpha, s_drafts, wstats, gathered, lane);
+        head_tile_pairs8_t(o, r, g8, npairs, v, valid, p.alpha, s_drafts, wstats, gathered,
+                           scr_base + ew * HEAD_SCR_FLOATS, lane);
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(acce0 + 8u * slot);
     }
     named_bar_sync(1, EPI * 32);
-    head_stats_finish(stats, EPI, tab, npairs,
+    head_stats_finish(stats, 4, tab, npairs,
                       p.partials + (static_cast<long long>(slot_id) * p.P + pair0) * HEAD_STAT_FIELDS,
                       threadIdx.x - 64, EPI * 32);
   }

@@ -148,6 +148,9 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
   float* const stats =
       reinterpret_cast<float*>(gbase + (misc - base) + 16 + MAX_PAIRS_PER_CHUNK * 4);
   const int tab = p.Pcp;
+  // per-warp staging rows of the transposed tile reduction (16-byte aligned)
+  float* const scr_base = reinterpret_cast<float*>(
+      (reinterpret_cast<uintptr_t>(stats + 4 * tab * HEAD_STAT_STRIDE) + 15) & ~uintptr_t(15));
 
   const int pair0 = chunk * p.Pc;
   const int npairs = min(p.Pc, p.P - pair0);
@@ -182,7 +185,7 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
     const int e = threadIdx.x - 64;
     for (int j = e; j < MAX_PAIRS_PER_CHUNK; j += EPI * 32)
       s_drafts[j] = (j < npairs) ? pair_draft(p.drafts, pair0 + j, p.gamma) : -1;
-    head_stats_init(stats, EPI * tab, e, EPI * 32);
+    head_stats_init(stats, 4 * tab, e, EPI * 32);
   }
   // both CTAs: barriers initialised and TMEM allocated before any cross-CTA use
   tc_fence_before();
@@ -283,7 +286,8 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
     const int q = warp & 3;    // TMEM lane quadrant this warp may access
     const int ew = warp - 2;   // statistics table of this warp
     const int half = ew >> 2;  // which alternate groups of 8 pairs it takes
-    float* const wstats = stats + ew * tab * HEAD_STAT_STRIDE;
+    // the two warps of a quadrant take disjoint pairs: they share one table
+    float* const wstats = stats + q * tab * HEAD_STAT_STRIDE;
     float* const gathered = p.gathered + static_cast<long long>(pair0) * GATHER_FIELDS;
     for (int pt = pt0, lt = 0; pt < pt1; ++pt, ++lt) {
       const int slot = lt & 1;
@@ -299,14 +303,15 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
         tmem_ld8(trow + g8, o);
         tmem_ld8(trow + p.Pcp + g8, r);
         tmem_ld_wait();
-        head_tile_pairs8(o, r, g8, npairs, v, valid, p.alpha, s_drafts, wstats, gathered, lane);
+        head_tile_pairs8_t(o, r, g8, npairs, v, valid, p.alpha, s_drafts, wstats, gathered,
+                           scr_base + ew * HEAD_SCR_FLOATS, lane);
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(mapa_shared(acce0 + 8u * slot, leader_rank));
     }
     named_bar_sync(1, EPI * 32);
-    head_stats_finish(stats, EPI, tab, npairs,
+    head_stats_finish(stats, 4, tab, npairs,
                       p.partials + (static_cast<long long>(slot_id) * p.P + pair0) * HEAD_STAT_FIELDS,
                       threadIdx.x - 64, EPI * 32);
   }
@@ -345,7 +350,8 @@ namespace {
 int h2_epi_warps(int N) { return N / 2 <= 32 ? 4 : 8; }
 size_t h2_fixed_bytes(int N) {
   return 1024 + 256 + 16 + MAX_PAIRS_PER_CHUNK * 4 +
-         static_cast<size_t>(h2_epi_warps(N)) * (N / 2) * HEAD_STAT_STRIDE * 4 + 64;
+         static_cast<size_t>(4) * (N / 2) * HEAD_STAT_STRIDE * 4 + 64 + 16 +
+         static_cast<size_t>(h2_epi_warps(N)) * HEAD_SCR_FLOATS * 4;
 }
 uint32_t h2_tmem_cols(int N) {
   uint32_t need = static_cast<uint32_t>(2 * N), c = 32;

@@ -90,13 +90,15 @@ int head_tc_max_stages(int N, size_t smem_limit) {
 
 // Pipeline depth: about 128 KB of tiles in flight per SM streams the weight at
 // full HBM bandwidth (measured on GB300: 7-8 stages of 18 KB beat both 4-6 and
-// 11) and leaves room on the SM for the concurrent attention kernel.
-#ifndef RV_HEAD_STAGE_TARGET_KB
-#define RV_HEAD_STAGE_TARGET_KB 128
+// 11), and a CTA of at most ~150 KB leaves room on the SM for the concurrent
+// small-batch attention kernel (75 KB).
+#ifndef RV_HEAD_SMEM_TARGET_KB
+#define RV_HEAD_SMEM_TARGET_KB 151
 #endif
 int head_tc_stages(int N, size_t smem_limit) {
   const int per = static_cast<int>(HT_A_BYTES) + N * 128;
-  const int want = (RV_HEAD_STAGE_TARGET_KB * 1024 + per - 1) / per;
+  const int room = RV_HEAD_SMEM_TARGET_KB * 1024 - static_cast<int>(ht_fixed_bytes(N));
+  const int want = room > 0 ? room / per : 0;
   return std::max(2, std::min(head_tc_max_stages(N, smem_limit), std::max(4, want)));
 }
 

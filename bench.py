@@ -44,16 +44,16 @@ FALLBACK_BF16_TFLOPS = 1900.0
 # dram__bytes_write.sum` on the workload named (see profiles/), valid only while
 # the kernel sources hash to `src_sha`.
 NCU_TRAFFIC = {
-    "llama3-8b-b1": {"bytes": 1050935000 + 2904576, "src_sha": "2ac78fa439b08095",
+    "llama3-8b-b1": {"bytes": 1051005000 + 3365120, "src_sha": "b979c3f2122d8134",
                      "summary": "profiles/head_tc_llama3-8b-b1.md"},
-    "llama3-8b-b16": {"bytes": 1053146000 + 2951936, "src_sha": "2ac78fa439b08095",
-                      "summary": "profiles/head_tc_llama3-8b-b16.md"},
+    "llama3-8b-b16": {"bytes": 1053148000 + 2957824, "src_sha": "b979c3f2122d8134",
+                      "summary": "profiles/head_tc2_llama3-8b-b16.md"},
 }
 
 
 def _kernel_src_hash() -> str:
     h = hashlib.sha256()
-    for f in ("k_head_tc.cu", "head_epilogue.cuh", "rv_device.cuh"):
+    for f in ("k_head_tc.cu", "k_head_tc2.cu", "head_epilogue.cuh", "rv_device.cuh"):
         with open(os.path.join(ROOT, "paper_2505_18629_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
@@ -419,8 +419,9 @@ def main():
     else:
         roof = {"bound": "tensor", "achieved": achieved_tf, "peak": tf_burst, "unit": "TFLOP/s",
                 "frac": achieved_tf / tf_burst, "traffic": traffic}
-    roof.update({"kernel": "head_tc_kernel (LM head GEMM + online log-softmax + merge), timed "
-                           "with the row-gather launch before it by an event pair on every 8th timed step",
+    roof.update({"kernel": "LM head (head_tc_kernel; head_tc2_kernel on CTA pairs from N >= 96 "
+                           "hidden rows per chunk): GEMM + online log-softmax (+ merge), timed with the "
+                           "row-gather launch before it by an event pair on every 8th timed step",
                  "peak_source": f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured"
                  else "fallback", "algorithmic_bytes": head_bytes,
                  "algorithmic_flops": head_flops, "avg_us": head_avg_s * 1e6, "launches": head_n,

@@ -78,6 +78,65 @@ def test_bf16_tcgen05_attention_gqa8_two_row_groups(gu):
     _check(gu, _wl(B=20, Hq=16, Hkv=2, gamma=6, R=8, V=500, H=128, ctx=(1, 300), seed=61))
 
 
+def _attention_only(gu, inp, ctx, h):
+    """rv_verify_attention alone on fresh cache copies; returns (out bits, status)."""
+    import torch
+    from paper_2505_18629_gb300 import rv
+    q, kb, vb = gu.to_dev(inp.q), gu.to_dev(inp.k_blk), gu.to_dev(inp.v_blk)
+    kc, vc = gu.to_dev(inp.k_cache), gu.to_dev(inp.v_cache)
+    out = torch.zeros_like(q)
+    rv.rv_verify_attention(h, q, kb, vb, kc, vc, gu.to_dev(np.asarray(ctx, np.int32)), out)
+    return gu.to_np(out), rv.rv_read_status(h), gu.to_np(kc)
+
+
+def test_tcgen05_attention_chunk_boundaries_and_repeated_launches(gu):
+    # B*Hkv = 40 selects the persistent tcgen05 kernel; its key chunks are 256
+    # keys here, so contexts at and around 128 / 256 / 512 / 768 hit tile and
+    # chunk edges, and three launches on one handle check that the item
+    # counter is re-armed between launches.
+    import oracle.rv_oracle as orc
+    from paper_2505_18629_gb300 import synth
+    wl = _wl(B=20, Hq=8, Hkv=2, gamma=3, R=4, V=600, H=256, ctx=(0, 1200), seed=62)
+    inp = synth.generate(wl)
+    h = gu.make_handle(wl)
+    edges = [0, 1, 127, 128, 255, 256, 257, 511, 512, 513, 767, 768, 769, 1023, 1024, 1100, 2, 64,
+             384, wl.capacity - wl.Lb]
+    rng = np.random.default_rng(7)
+    for rep in range(3):
+        ctx = np.asarray(edges if rep == 0 else rng.permutation(edges), np.int32)
+        out, status, kc = _attention_only(gu, inp, ctx, h)
+        assert status == 0
+        ref, rkc, _ = orc.verify_attention(inp.q, inp.k_blk, inp.v_blk, inp.k_cache, inp.v_cache, ctx)
+        ok, amax, nbad = gu.attn_close(out, ref)
+        assert ok, f"launch {rep}: {nbad} elements beyond tolerance (max {amax:.3g})"
+        for b in range(wl.B):
+            c = int(ctx[b])
+            np.testing.assert_array_equal(kc[b, :, :c + wl.Lb],
+                                          gu._bits_like(rkc[b, :, :c + wl.Lb], kc))
+    h.close()
+
+
+def test_tcgen05_attention_context_overflow(gu):
+    import oracle.rv_oracle as orc
+    from paper_2505_18629_gb300 import rv, synth
+    wl = _wl(B=20, Hq=8, Hkv=2, gamma=3, R=4, V=600, H=256, ctx=(0, 600), seed=63)
+    inp = synth.generate(wl)
+    ctx = inp.ctx_lens.astype(np.int32).copy()
+    ctx[3] = wl.capacity - wl.Lb + 1                        # does not fit
+    ctx[11] = -1                                            # negative
+    h = gu.make_handle(wl)
+    out, status, kc = _attention_only(gu, inp, ctx, h)
+    assert status & rv.RV_DEV_CTX_RANGE
+    assert (out[3] == 0).all() and (out[11] == 0).all()     # left untouched
+    np.testing.assert_array_equal(kc[3], inp.k_cache[3])
+    ok_seqs = [b for b in range(wl.B) if b not in (3, 11)]
+    ref, _, _ = orc.verify_attention(inp.q[ok_seqs], inp.k_blk[ok_seqs], inp.v_blk[ok_seqs],
+                                     inp.k_cache[ok_seqs], inp.v_cache[ok_seqs], ctx[ok_seqs])
+    ok, amax, nbad = gu.attn_close(out[ok_seqs], ref)
+    assert ok, f"{nbad} elements beyond tolerance (max {amax:.3g})"
+    h.close()
+
+
 def test_bf16_max_pairs_single_chunk(gu):
     # B*(gamma+1) = 126 pairs -> N = 256 columns, the widest MMA
     _check(gu, _wl(B=14, gamma=8, R=8, V=777, H=256, ctx=(10, 60), seed=45), check_attn=False)

@@ -164,6 +164,16 @@ def logsumexp(x: np.ndarray, axis: int = -1) -> np.ndarray:
     return (m + np.log(np.sum(np.exp(x - m), axis=axis, keepdims=True))).squeeze(axis)
 
 
+def entropy(logits: np.ndarray, axis: int = -1) -> np.ndarray:
+    """Shannon entropy (nats) of softmax(logits): H = -sum_v p_v log p_v with
+    log p_v = logits_v - logsumexp(logits).  Used by the entropy-based
+    threshold of typical acceptance (Alg. 3)."""
+    logits = np.asarray(logits, np.float64)
+    logp = logits - np.expand_dims(logsumexp(logits, axis=axis), axis)
+    p = np.exp(logp)
+    return -np.sum(np.where(p > 0, p * logp, 0.0), axis=axis)
+
+
 def fuse(o: np.ndarray, o_refl: np.ndarray, alpha: float) -> np.ndarray:
     """(1 - alpha) * o_i + alpha * o_{i + shift_len}  (Eq. 2, before softmax)."""
     return (1.0 - alpha) * o + alpha * o_refl
@@ -188,6 +198,8 @@ def verify_head(W, hidden, drafts, gamma: int, R: int, alpha: float):
       margin                               [B, gamma]  |z_i[x_i] - max_{v != x_i} z_i[v]|
       choice_gap                           [B, gamma+1] z_i[x^_i] - max_{v != x^_i} z_i[v]
                                            (how far the greedy choice is from a tie)
+      ent_orig                             [B, gamma+1] entropy of softmax(o_i), the
+                                           unfused original distribution (Alg. 3)
       z                                    [B, gamma+1, V] fused logits
     """
     hidden = as_f64(hidden)
@@ -218,7 +230,7 @@ def verify_head(W, hidden, drafts, gamma: int, R: int, alpha: float):
         logp_fused=zx - lse_z[:, :gamma],
         logp_orig=o[bi, ii, drafts] - lse_o[:, :gamma],
         logp_refl=o_refl[bi, ii, drafts] - lse_r[:, :gamma],
-        argmax=choice, margin=margin, choice_gap=choice_gap, z=z,
+        argmax=choice, margin=margin, choice_gap=choice_gap, ent_orig=entropy(o), z=z,
     )
 
 
@@ -248,6 +260,36 @@ def exact_match_accept(drafts, choice):
         n[b] = min(stop + [gamma])
         t[b] = choice[b, n[b]]
     return acc.astype(np.uint8), n, t
+
+
+def typical_accept(drafts, logp_fused, ent_orig, choice, eps: float, delta: float):
+    """Typical acceptance with Reflective Verification (Alg. 3).
+
+    Position i keeps its draft when p_i(x_i) exceeds the entropy-based
+    threshold min(eps, delta * exp(-H(p_original,i))), where p_i is the fused
+    distribution of Eq. 2 and p_original,i = softmax(o_i) the unfused original
+    one at the same position.  n is the number of leading kept drafts (the
+    printed stopping set is read as "stop at the first draft that fails the
+    threshold"), and the next token t is the greedy choice argmax p_{n+1}
+    (the sampling temperature of Alg. 3 taken to 0, as for Alg. 2).
+
+    Returns (accept_mask [B, gamma] bool, n [B], t [B], gap [B, gamma]) where
+    gap = log p_i(x_i) - log threshold_i (the decision's distance in nats).
+    """
+    logp = np.asarray(logp_fused, np.float64)
+    H = np.asarray(ent_orig, np.float64)[:, :logp.shape[1]]
+    log_thr = np.minimum(np.log(eps), np.log(delta) - H)
+    gap = logp - log_thr
+    acc = gap > 0
+    B, gamma = acc.shape
+    n = np.full(B, gamma, np.int64)
+    for b in range(B):
+        for i in range(gamma):
+            if not acc[b, i]:
+                n[b] = i
+                break
+    t = np.asarray(choice, np.int64)[np.arange(B), n]
+    return acc, n, t, gap
 
 
 def verify_step(inp_W, hidden, q, k_blk, v_blk, k_cache, v_cache, ctx_lens,

@@ -387,3 +387,102 @@ def test_pins_catch_dropped_causal_mask(monkeypatch):
     monkeypatch.setattr(orc, "verify_attention", no_mask)
     assert _fails(lambda: test_attention_matches_torch_sdpa(2, 7, 8, 2, 16, [0, 5]))
     assert _fails(test_attention_first_segment_unaffected_by_template_and_copy)
+
+
+# ------------------------------------------------------------------ Alg. 3: typical acceptance
+
+def test_entropy_closed_forms_and_library():
+    import scipy.stats
+    rng = np.random.default_rng(11)
+    # constant logits: the uniform distribution, H = ln V
+    for V in (2, 3, 1000):
+        assert abs(orc.entropy(np.full(V, 3.7)) - math.log(V)) < 1e-12
+    # two outcomes with logits (0, a): the binary entropy of sigma(a)
+    for a in (-3.0, 0.0, 0.5, 7.0):
+        p = 1.0 / (1.0 + math.exp(-a))
+        h = -(p * math.log(p) + (1 - p) * math.log(1 - p))
+        assert abs(orc.entropy(np.array([0.0, a])) - h) < 1e-12
+    # a library routine on random logits, batched along an axis
+    x = rng.normal(0, 3, (4, 5, 257))
+    ref = scipy.stats.entropy(scipy.special.softmax(x, axis=-1), axis=-1)
+    np.testing.assert_allclose(orc.entropy(x), ref, rtol=1e-12, atol=1e-12)
+    # a nearly one-hot distribution has (almost) no entropy; bounds 0 <= H <= ln V
+    assert 0.0 <= orc.entropy(np.array([200.0, 0.0, 0.0])) < 1e-80
+    h = orc.entropy(x)
+    assert (h >= 0).all() and (h <= math.log(257) + 1e-12).all()
+
+
+def test_entropy_in_head_is_of_the_unfused_original_logits():
+    # H(p_original) does not depend on alpha; at alpha = 0 the fused
+    # distribution is the original one, so it equals the fused entropy there
+    rng = np.random.default_rng(12)
+    V, H, gamma, R = 50, 8, 3, 2
+    W = rng.normal(0, 1, (V, H))
+    hidden = rng.normal(0, 1, (2, 2 * gamma + R + 1, H))
+    drafts = rng.integers(0, V, (2, gamma))
+    a0 = orc.verify_head(W, hidden, drafts, gamma, R, 0.0)
+    a1 = orc.verify_head(W, hidden, drafts, gamma, R, 0.7)
+    np.testing.assert_array_equal(a0["ent_orig"], a1["ent_orig"])
+    np.testing.assert_allclose(a0["ent_orig"], orc.entropy(a0["z"]), atol=1e-12)
+    assert not np.allclose(a1["ent_orig"], orc.entropy(a1["z"]))
+
+
+def test_typical_threshold_worked_example():
+    # uniform original distribution over V = 3: H = ln 3, so with delta = 0.3
+    # the entropy term is 0.3 / 3 = 0.1 and eps = 0.09 is the binding side
+    H = np.full((1, 3), math.log(3))
+    logp = np.log(np.array([[0.5, 0.2, 0.05]]))  # kept, kept, rejected
+    choice = np.array([[4, 5, 6]])
+    acc, n, t, gap = orc.typical_accept(np.zeros((1, 2)), logp[:, :2], H, choice, 0.09, 0.3)
+    assert acc.tolist() == [[True, True]] and n[0] == 2 and t[0] == 6
+    acc, n, t, gap = orc.typical_accept(np.zeros((1, 3)), logp, H, np.array([[4, 5, 6, 7]]), 0.09, 0.3)
+    assert acc.tolist() == [[True, True, False]] and n[0] == 2 and t[0] == 6
+    np.testing.assert_allclose(gap[0], np.log([0.5, 0.2, 0.05]) - math.log(0.09), atol=1e-12)
+    # a low-entropy original distribution lowers the threshold to delta * e^-H
+    acc, n, t, gap = orc.typical_accept(np.zeros((1, 1)), np.log([[0.05]]), np.array([[3.0]]),
+                                        np.array([[1, 2]]), 0.09, 0.3)
+    assert acc[0, 0] and abs(gap[0, 0] - (math.log(0.05) - (math.log(0.3) - 3.0))) < 1e-12
+
+
+def test_typical_accept_limits_and_monotonicity():
+    rng = np.random.default_rng(13)
+    B, gamma = 64, 6
+    logp = np.log(rng.uniform(1e-4, 1.0, (B, gamma)))
+    H = rng.uniform(0.0, 6.0, (B, gamma + 1))
+    choice = rng.integers(0, 1000, (B, gamma + 1))
+    # threshold above every probability: nothing is kept, t = the first choice
+    acc, n, t, _ = orc.typical_accept(np.zeros((B, gamma)), logp, H, choice, 2.0, 1e9)
+    assert not acc.any() and (n == 0).all() and (t == choice[:, 0]).all()
+    # a vanishing threshold keeps every draft, t = the bonus position's choice
+    acc, n, t, _ = orc.typical_accept(np.zeros((B, gamma)), logp, H, choice, 1e-300, 1e-300)
+    assert acc.all() and (n == gamma).all() and (t == choice[:, gamma]).all()
+    # n is the number of leading kept drafts, and falls as eps or delta grow
+    prev = None
+    for eps in (1e-3, 1e-2, 0.05, 0.1, 0.3):
+        acc, n, t, _ = orc.typical_accept(np.zeros((B, gamma)), logp, H, choice, eps, 0.3)
+        for b in range(B):
+            assert acc[b, :n[b]].all() and (n[b] == gamma or not acc[b, n[b]])
+            assert t[b] == choice[b, n[b]]
+        if prev is not None:
+            assert (n <= prev).all()
+        prev = n
+
+
+def test_pins_catch_fused_entropy(monkeypatch):
+    real = orc.verify_head
+
+    def fused_entropy(W, hidden, drafts, gamma, R, alpha):
+        out = real(W, hidden, drafts, gamma, R, alpha)
+        out["ent_orig"] = orc.entropy(out["z"])  # planted slip: entropy of p_i, not p_original
+        return out
+    monkeypatch.setattr(orc, "verify_head", fused_entropy)
+    assert _fails(test_entropy_in_head_is_of_the_unfused_original_logits)
+
+
+def test_pins_catch_swapped_threshold_parameters(monkeypatch):
+    def swapped(drafts, logp_fused, ent_orig, choice, eps, delta):
+        # planted slip: eps and delta exchanged in the threshold
+        return real(drafts, logp_fused, ent_orig, choice, delta, eps)
+    real = orc.typical_accept
+    monkeypatch.setattr(orc, "typical_accept", swapped)
+    assert _fails(test_typical_threshold_worked_example)

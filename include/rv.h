@@ -67,13 +67,19 @@ extern "C" {
 #define RV_DTYPE_F32 1          /* fp32 storage and accumulation (CUDA cores) */
 
 /* ---- per-position scores written by rv_verify_head ---------------------- */
-#define RV_NSCORES 6
+#define RV_NSCORES 7
 #define RV_SCORE_LSE_ORIG 0     /* logsumexp_v o_i[v]                         */
 #define RV_SCORE_LSE_REFL 1     /* logsumexp_v o_{m+i-1}[v]                   */
 #define RV_SCORE_LSE_FUSED 2    /* logsumexp_v z_i[v], z_i = (1-a)o_i + a o'_i */
 #define RV_SCORE_LOGP_FUSED 3   /* log p_i(x_i) = z_i[x_i] - lse_fused (NaN at i = gamma+1) */
 #define RV_SCORE_LOGP_ORIG 4    /* o_i[x_i] - lse_orig                        */
 #define RV_SCORE_LOGP_REFL 5    /* o'_i[x_i] - lse_refl                       */
+#define RV_SCORE_ENT_ORIG 6     /* H(softmax(o_i)): entropy (nats) of the unfused original
+                                   distribution, for the typical acceptance of Alg. 3 */
+
+/* Acceptance rules (rv_set_acceptance). */
+#define RV_ACCEPT_EXACT 0       /* exact match with the greedy choice (Alg. 2)               */
+#define RV_ACCEPT_TYPICAL 1     /* entropy-based threshold of typical acceptance (Alg. 3)     */
 
 /* Model / capacity description fixed at creation. */
 typedef struct rv_config {
@@ -169,12 +175,39 @@ RV_API int rv_accept(rv_handle* h, const int32_t* draft_ids, const int32_t* argm
                      int32_t gamma, uint8_t* accept_mask, int32_t* accepted_len,
                      int32_t* next_token, const int32_t* ctx_in, int32_t* ctx_out, void* stream);
 
+/* Typical acceptance with Reflective Verification (Alg. 3): position i keeps
+ * its draft when the fused probability exceeds an entropy-based threshold,
+ *   p_i(x_i) > min(eps, delta * exp(-H(softmax(o_i)))),
+ * with p_i the fused distribution (Eq. 2) and H the entropy of the unfused
+ * original distribution at the same position (scores[..., RV_SCORE_ENT_ORIG]);
+ * the test is taken in the log domain on scores[..., RV_SCORE_LOGP_FUSED]:
+ *   accept_mask[b][i-1] = logp > min(log eps, log delta - H)     uint8 [B, gamma]
+ *   accepted_len[b] = n = number of leading kept drafts             int32 [B]
+ *   next_token[b]   = argmax[b][n] (the greedy choice at n+1: the sampling
+ *                     temperature of Alg. 3 taken to 0)             int32 [B]
+ *   ctx_out[b]      = ctx_in[b] + n (may alias ctx_in)
+ * scores [B, gamma+1, RV_NSCORES] and argmax [B, gamma+1] as written by
+ * rv_verify_head.  eps > 0 and delta > 0, else RV_ERR_INVALID_ARG.  A draft
+ * whose log-probability is NaN (out-of-range id) is rejected. */
+RV_API int rv_accept_typical(rv_handle* h, const int32_t* draft_ids, const float* scores,
+                             const int32_t* argmax, int32_t B, int32_t gamma, float eps,
+                             float delta, uint8_t* accept_mask, int32_t* accepted_len,
+                             int32_t* next_token, const int32_t* ctx_in, int32_t* ctx_out,
+                             void* stream);
+
+/* Acceptance rule used by rv_verify_step (and rv_verify_step_host) on this
+ * handle: RV_ACCEPT_EXACT (the default; eps and delta ignored) or
+ * RV_ACCEPT_TYPICAL with its eps > 0 and delta > 0 (see rv_accept_typical).
+ * Host-side setting, takes effect for the following calls. */
+RV_API int rv_set_acceptance(rv_handle* h, int32_t mode, float eps, float delta);
+
 /* The whole verify step on device buffers, in one call and four kernel
  * launches: the attention (rv_verify_attention) on an internal stream forked
  * from `stream`, concurrently with -- on `stream` -- one launch that gathers
  * the LM-head rows and packs the block (rv_pack_block; skipped when block_ids
  * is NULL), the LM head, and one launch that merges the head's statistics and
- * runs the acceptance (rv_accept).  The internal stream is joined back into
+ * runs the acceptance (rv_accept, or rv_accept_typical when the handle's rule
+ * is RV_ACCEPT_TYPICAL; see rv_set_acceptance).  The internal stream is joined back into
  * `stream` before the call returns, so later work on `stream` sees every
  * output; the pattern is also valid inside stream capture.  Arguments as in those
  * calls; the template is n_prompt prompt ids + n_prefix prefix ids, so

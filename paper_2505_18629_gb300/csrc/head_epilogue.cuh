@@ -18,9 +18,24 @@
 
 namespace rv {
 
-// Shared-memory statistics tables use a stride of 9 floats per pair: eight
-// lanes updating consecutive pairs then hit different banks.
-constexpr int HEAD_STAT_STRIDE = HEAD_STAT_FIELDS + 1;
+// Shared-memory statistics tables use a stride of 10 floats per pair (the 9
+// fields used + 1): eight lanes updating consecutive pairs then hit different
+// banks.
+constexpr int HEAD_STAT_STRIDE = HEAD_STAT_USED + 1;
+
+// Merge running (m, s, t) with another (M, S, T), where s = sum exp(x - m) and
+// t = sum exp(x - m) (x - m): both are re-based to the larger maximum.  The
+// entropy of softmax(x) is then log(s) - t / s.
+__device__ __forceinline__ void lse_merge3(float& m, float& s, float& t, float M, float S,
+                                           float T) {
+  const float mn = fmaxf(m, M);
+  if (mn == NEG_INF) return;
+  const float a = (m == NEG_INF) ? 0.f : exp2f((m - mn) * LOG2E);
+  const float c = (M == NEG_INF) ? 0.f : exp2f((M - mn) * LOG2E);
+  t = (a == 0.f ? 0.f : a * (t + (m - mn) * s)) + (c == 0.f ? 0.f : c * (T + (M - mn) * S));
+  s = s * a + S * c;
+  m = mn;
+}
 
 __device__ __forceinline__ void head_stats_init(float* stats, int n_entries, int tid,
                                                 int nthreads) {
@@ -34,6 +49,7 @@ __device__ __forceinline__ void head_stats_init(float* stats, int n_entries, int
     s[ST_S_Z] = 0.f;
     s[ST_BEST_V] = NEG_INF;
     s[ST_BEST_I] = __int_as_float(INT_MAX);
+    s[ST_T_O] = 0.f;
   }
 }
 
@@ -77,10 +93,11 @@ __device__ __forceinline__ void head_tile_pairs8(const float (&o)[8], const floa
       Mz[j] = fmaxf(Mz[j], __shfl_xor_sync(0xffffffffu, Mz[j], off));
     }
   }
-  float So[8], Sr[8], Sz[8];
+  float So[8], Sr[8], Sz[8], To[8];
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
     So[j] = exp_shifted(ov[j], Mo[j]);
+    To[j] = So[j] == 0.f ? 0.f : So[j] * (ov[j] - Mo[j]);
     Sr[j] = exp_shifted(rv[j], Mr[j]);
     Sz[j] = exp_shifted(zv[j], Mz[j]);
   }
@@ -89,6 +106,7 @@ __device__ __forceinline__ void head_tile_pairs8(const float (&o)[8], const floa
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       So[j] += __shfl_xor_sync(0xffffffffu, So[j], off);
+      To[j] += __shfl_xor_sync(0xffffffffu, To[j], off);
       Sr[j] += __shfl_xor_sync(0xffffffffu, Sr[j], off);
       Sz[j] += __shfl_xor_sync(0xffffffffu, Sz[j], off);
       const float ov2 = __shfl_xor_sync(0xffffffffu, bv[j], off);
@@ -102,13 +120,15 @@ __device__ __forceinline__ void head_tile_pairs8(const float (&o)[8], const floa
   // Every lane now holds the tile results of all eight pairs; lane j < 8
   // folds pair g8+j into the running statistics (one SIMT pass, no divergence
   // between the pairs).
-  float cMo = Mo[0], cSo = So[0], cMr = Mr[0], cSr = Sr[0], cMz = Mz[0], cSz = Sz[0], cbv = bv[0];
+  float cMo = Mo[0], cSo = So[0], cTo = To[0], cMr = Mr[0], cSr = Sr[0], cMz = Mz[0], cSz = Sz[0],
+        cbv = bv[0];
   int cbi = bi[0];
 #pragma unroll
   for (int j = 1; j < 8; ++j) {
     const bool me = lane == j;
     cMo = me ? Mo[j] : cMo;
     cSo = me ? So[j] : cSo;
+    cTo = me ? To[j] : cTo;
     cMr = me ? Mr[j] : cMr;
     cSr = me ? Sr[j] : cSr;
     cMz = me ? Mz[j] : cMz;
@@ -119,7 +139,7 @@ __device__ __forceinline__ void head_tile_pairs8(const float (&o)[8], const floa
   const int pj = g8 + lane;
   if (lane < 8 && pj < npairs) {
     float* s = warp_stats + pj * HEAD_STAT_STRIDE;
-    lse_merge(s[ST_M_O], s[ST_S_O], cMo, cSo);
+    lse_merge3(s[ST_M_O], s[ST_S_O], s[ST_T_O], cMo, cSo, cTo);
     lse_merge(s[ST_M_R], s[ST_S_R], cMr, cSr);
     lse_merge(s[ST_M_Z], s[ST_S_Z], cMz, cSz);
     const int si = __float_as_int(s[ST_BEST_I]);
@@ -136,7 +156,7 @@ __device__ __forceinline__ void head_tile_pairs8(const float (&o)[8], const floa
 // c % 8; o, r or z for c / 8) over the 32 rows with plain loads - no shuffle
 // trees - then folds the result into the warp's running statistics.  Same
 // results as the shuffle version up to the order of the sums.
-constexpr int HEAD_SCR_STRIDE = 28;  // floats per staged row: 24 used, 16-byte aligned rows
+constexpr int HEAD_SCR_STRIDE = 24;  // floats per staged row (16-byte aligned rows)
 constexpr int HEAD_SCR_FLOATS = 32 * HEAD_SCR_STRIDE;
 
 __device__ __forceinline__ void head_tile_pairs8_t(const float (&o)[8], const float (&r)[8], int g8,
@@ -175,17 +195,23 @@ __device__ __forceinline__ void head_tile_pairs8_t(const float (&o)[8], const fl
       val[i] = scr[i * HEAD_SCR_STRIDE + lane];
       m = fmaxf(m, val[i]);
     }
-    float sum = 0.f;
+    float sum = 0.f, tsum = 0.f;  // tsum: sum exp(x - m) (x - m), for the entropy of o
     if (m != NEG_INF) {
-      float s2[4] = {0.f, 0.f, 0.f, 0.f};
+      float s2[4] = {0.f, 0.f, 0.f, 0.f}, t2[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int i = 0; i < 32; ++i) s2[i & 3] += __expf(val[i] - m);
+      for (int i = 0; i < 32; ++i) {
+        const float d = val[i] - m;
+        const float e = __expf(d);
+        s2[i & 3] += e;
+        t2[i & 3] += e == 0.f ? 0.f : e * d;
+      }
       sum = (s2[0] + s2[1]) + (s2[2] + s2[3]);
+      tsum = (t2[0] + t2[1]) + (t2[2] + t2[3]);
     }
     if (pj < npairs) {
       float* st = warp_stats + pj * HEAD_STAT_STRIDE;
       if (kind == 0) {
-        lse_merge(st[ST_M_O], st[ST_S_O], m, sum);
+        lse_merge3(st[ST_M_O], st[ST_S_O], st[ST_T_O], m, sum, tsum);
       } else if (kind == 1) {
         lse_merge(st[ST_M_R], st[ST_S_R], m, sum);
       } else {
@@ -217,12 +243,12 @@ __device__ __forceinline__ void head_tile_pairs8_t(const float (&o)[8], const fl
 __device__ __forceinline__ void head_stats_finish(const float* stats, int nwarps, int tab,
                                                   int npairs, float* out, int tid, int nthreads) {
   for (int pj = tid; pj < npairs; pj += nthreads) {
-    float mo = NEG_INF, so = 0.f, mr = NEG_INF, sr = 0.f, mz = NEG_INF, sz = 0.f;
+    float mo = NEG_INF, so = 0.f, to = 0.f, mr = NEG_INF, sr = 0.f, mz = NEG_INF, sz = 0.f;
     float bv = NEG_INF;
     int bi = INT_MAX;
     for (int w = 0; w < nwarps; ++w) {
       const float* s = stats + (w * tab + pj) * HEAD_STAT_STRIDE;
-      lse_merge(mo, so, s[ST_M_O], s[ST_S_O]);
+      lse_merge3(mo, so, to, s[ST_M_O], s[ST_S_O], s[ST_T_O]);
       lse_merge(mr, sr, s[ST_M_R], s[ST_S_R]);
       lse_merge(mz, sz, s[ST_M_Z], s[ST_S_Z]);
       const float v = s[ST_BEST_V];
@@ -241,6 +267,9 @@ __device__ __forceinline__ void head_stats_finish(const float* stats, int nwarps
     d[ST_S_Z] = sz;
     d[ST_BEST_V] = bv;
     d[ST_BEST_I] = __int_as_float(bi);
+    d[ST_T_O] = to;
+#pragma unroll
+    for (int f = HEAD_STAT_USED; f < HEAD_STAT_FIELDS; ++f) d[f] = 0.f;
   }
 }
 
@@ -251,9 +280,19 @@ __device__ __forceinline__ void head_stats_finish(const float* stats, int nwarps
 // them).  Each lane issues the loads of all its slots before merging them, and
 // the choices go through shared memory (`s_choice`, P ints), so the tail costs
 // about one L2 round trip.
-constexpr int MERGE_SLOTS_PER_LANE = 8;
+constexpr int MERGE_SLOTS_PER_LANE = 6;
 
-// s_draft[p]: the draft scored by pair p (-1 for none), in shared memory.
+// Acceptance test of one position from its fused log-probability, entropy
+// and greedy choice: exact match (Alg. 2) or the typical threshold (Alg. 3).
+__device__ __forceinline__ bool position_kept(const AcceptArgs& acc, int x, int choice,
+                                              float logp_fused, float ent_orig) {
+  if (acc.mode == RV_ACCEPT_TYPICAL)
+    return logp_fused > fminf(acc.log_eps, acc.log_delta - ent_orig);  // false for NaN
+  return x == choice;
+}
+
+// s_draft[p]: the draft scored by pair p (-1 for none), in shared memory;
+// s_choice: 2P ints of shared memory (choices, then kept flags).
 __device__ __forceinline__ void head_merge_all(const float* partials, const float* gathered,
                                                const int* s_draft, int B, int gamma, int V,
                                                int P, int slots, const HeadFinal& f,
@@ -261,26 +300,28 @@ __device__ __forceinline__ void head_merge_all(const float* partials, const floa
                                                int nthreads) {
   const int lane = tid & 31, warp = tid >> 5, nw = nthreads >> 5;
   const float nan = __int_as_float(0x7fc00000);
+  int* const s_kept = s_choice + P;
   for (int p = warp; p < P; p += nw) {
-    float mo = NEG_INF, so = 0.f, mr = NEG_INF, sr = 0.f, mz = NEG_INF, sz = 0.f;
+    float mo = NEG_INF, so = 0.f, to = 0.f, mr = NEG_INF, sr = 0.f, mz = NEG_INF, sz = 0.f;
     float bv = NEG_INF;
     int bi = INT_MAX;
     for (int g0 = lane; g0 < slots; g0 += 32 * MERGE_SLOTS_PER_LANE) {
       float4 lo[MERGE_SLOTS_PER_LANE], hi[MERGE_SLOTS_PER_LANE];
+      float tt[MERGE_SLOTS_PER_LANE];
 #pragma unroll
       for (int k = 0; k < MERGE_SLOTS_PER_LANE; ++k) {
         const int g = g0 + 32 * k;
         if (g < slots) {
-          const float4* q =
-              reinterpret_cast<const float4*>(partials + (static_cast<long long>(g) * P + p) * HEAD_STAT_FIELDS);
-          lo[k] = __ldcg(q);
-          hi[k] = __ldcg(q + 1);
+          const float* q = partials + (static_cast<long long>(g) * P + p) * HEAD_STAT_FIELDS;
+          lo[k] = __ldcg(reinterpret_cast<const float4*>(q));
+          hi[k] = __ldcg(reinterpret_cast<const float4*>(q) + 1);
+          tt[k] = __ldcg(q + ST_T_O);
         }
       }
 #pragma unroll
       for (int k = 0; k < MERGE_SLOTS_PER_LANE; ++k) {
         if (g0 + 32 * k < slots) {
-          lse_merge(mo, so, lo[k].x, lo[k].y);
+          lse_merge3(mo, so, to, lo[k].x, lo[k].y, tt[k]);
           lse_merge(mr, sr, lo[k].z, lo[k].w);
           lse_merge(mz, sz, hi[k].x, hi[k].y);
           const int i = __float_as_int(hi[k].w);
@@ -293,7 +334,8 @@ __device__ __forceinline__ void head_merge_all(const float* partials, const floa
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
-      lse_merge(mo, so, __shfl_xor_sync(0xffffffffu, mo, o), __shfl_xor_sync(0xffffffffu, so, o));
+      lse_merge3(mo, so, to, __shfl_xor_sync(0xffffffffu, mo, o), __shfl_xor_sync(0xffffffffu, so, o),
+                 __shfl_xor_sync(0xffffffffu, to, o));
       lse_merge(mr, sr, __shfl_xor_sync(0xffffffffu, mr, o), __shfl_xor_sync(0xffffffffu, sr, o));
       lse_merge(mz, sz, __shfl_xor_sync(0xffffffffu, mz, o), __shfl_xor_sync(0xffffffffu, sz, o));
     }
@@ -301,14 +343,17 @@ __device__ __forceinline__ void head_merge_all(const float* partials, const floa
     if (lane == 0) {
       const int b = p / (gamma + 1), i = p % (gamma + 1);
       const float lse_o = mo + logf(so), lse_r = mr + logf(sr), lse_z = mz + logf(sz);
+      const float ent = logf(so) - to / so;
       float* sc = f.scores + static_cast<long long>(p) * RV_NSCORES;
       sc[RV_SCORE_LSE_ORIG] = lse_o;
       sc[RV_SCORE_LSE_REFL] = lse_r;
       sc[RV_SCORE_LSE_FUSED] = lse_z;
+      sc[RV_SCORE_ENT_ORIG] = ent;
       int choice = bi;
       float lp_z = nan, lp_o = nan, lp_r = nan;
+      int x = -1;
       if (i < gamma) {
-        const int x = s_draft[p];
+        x = s_draft[p];
         if (x >= 0 && x < V) {
           const float4 gx = __ldcg(reinterpret_cast<const float4*>(gathered) + p);
           lp_z = gx.z - lse_z;
@@ -326,6 +371,7 @@ __device__ __forceinline__ void head_merge_all(const float* partials, const floa
       sc[RV_SCORE_LOGP_REFL] = lp_r;
       f.argmax[p] = choice;
       s_choice[p] = choice;
+      s_kept[p] = position_kept(f.acc, x, choice, lp_z, ent) ? 1 : 0;
     }
   }
   if (f.acc.accepted_len == nullptr) return;
@@ -333,7 +379,7 @@ __device__ __forceinline__ void head_merge_all(const float* partials, const floa
   for (int b = tid; b < B; b += nthreads) {
     int n = gamma;
     for (int i = 0; i < gamma; ++i) {
-      const bool ok = s_draft[b * (gamma + 1) + i] == s_choice[b * (gamma + 1) + i];
+      const bool ok = s_kept[b * (gamma + 1) + i] != 0;
       f.acc.accept_mask[b * gamma + i] = ok ? 1 : 0;
       if (!ok && n == gamma) n = i;
     }

@@ -2,11 +2,13 @@
 // that gathers the original / reflective hidden rows for the LM head (and
 // packs the block in the same launch); the finalize kernel that merges the
 // head's per-CTA statistics into per-position scores (Eq. 2) and, inside
-// rv_verify_step, runs the exact-match acceptance with the longest accepted
-// prefix (Alg. 2); the stand-alone acceptance kernel of rv_accept.
+// rv_verify_step, runs the acceptance (exact match, Alg. 2, or the typical
+// threshold, Alg. 3) with the longest accepted prefix; the stand-alone
+// acceptance kernels of rv_accept and rv_accept_typical.
 #include <cfloat>
 #include <climits>
 
+#include "head_epilogue.cuh"
 #include "rv_device.cuh"
 #include "rv_kernels.h"
 
@@ -129,12 +131,12 @@ cudaError_t launch_prep(const HeadArgs& a, const HeadPlan& p, void* hsel, const 
 constexpr int FIN_MAX_WARPS = 32;
 
 struct MergeStat {
-  float mo, so, mr, sr, mz, sz, bv;
+  float mo, so, to, mr, sr, mz, sz, bv;
   int bi;
 };
 
 __device__ __forceinline__ void merge_into(MergeStat& a, const MergeStat& b) {
-  lse_merge(a.mo, a.so, b.mo, b.so);
+  lse_merge3(a.mo, a.so, a.to, b.mo, b.so, b.to);
   lse_merge(a.mr, a.sr, b.mr, b.sr);
   lse_merge(a.mz, a.sz, b.mz, b.sz);
   if (b.bv > a.bv || (b.bv == a.bv && b.bi < a.bi)) {
@@ -147,6 +149,7 @@ __device__ __forceinline__ MergeStat shfl_stat(const MergeStat& s, int o) {
   MergeStat r;
   r.mo = __shfl_xor_sync(0xffffffffu, s.mo, o);
   r.so = __shfl_xor_sync(0xffffffffu, s.so, o);
+  r.to = __shfl_xor_sync(0xffffffffu, s.to, o);
   r.mr = __shfl_xor_sync(0xffffffffu, s.mr, o);
   r.sr = __shfl_xor_sync(0xffffffffu, s.sr, o);
   r.mz = __shfl_xor_sync(0xffffffffu, s.mz, o);
@@ -164,6 +167,7 @@ __global__ void head_finalize_kernel(const float* __restrict__ partials,
                                      unsigned* status, AcceptArgs acc) {
   __shared__ MergeStat red[FIN_MAX_WARPS];
   __shared__ int s_choice[65];
+  __shared__ int s_kept[65];
   const int b = blockIdx.x;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
   const int npos = gamma + 1, per_pass = nw / wpp;
@@ -172,12 +176,12 @@ __global__ void head_finalize_kernel(const float* __restrict__ partials,
   for (int base = 0; base < npos; base += per_pass) {
     const int i = base + warp / wpp;
     const bool active = i < npos;
-    MergeStat st{NEG_INF, 0.f, NEG_INF, 0.f, NEG_INF, 0.f, NEG_INF, INT_MAX};
+    MergeStat st{NEG_INF, 0.f, 0.f, NEG_INF, 0.f, NEG_INF, 0.f, NEG_INF, INT_MAX};
     if (active) {
       const int p = b * npos + i;
       for (int g = sub * 32 + lane; g < slots; g += wpp * 32) {
         const float* q = partials + (static_cast<long long>(g) * P + p) * HEAD_STAT_FIELDS;
-        const MergeStat o{q[ST_M_O], q[ST_S_O], q[ST_M_R], q[ST_S_R],
+        const MergeStat o{q[ST_M_O], q[ST_S_O], q[ST_T_O], q[ST_M_R], q[ST_S_R],
                           q[ST_M_Z], q[ST_S_Z], q[ST_BEST_V], __float_as_int(q[ST_BEST_I])};
         merge_into(st, o);
       }
@@ -192,14 +196,17 @@ __global__ void head_finalize_kernel(const float* __restrict__ partials,
       const float lse_o = st.mo + logf(st.so);
       const float lse_r = st.mr + logf(st.sr);
       const float lse_z = st.mz + logf(st.sz);
+      const float ent = logf(st.so) - st.to / st.so;
       float* sc = scores + static_cast<long long>(p) * RV_NSCORES;
+      sc[RV_SCORE_ENT_ORIG] = ent;
       sc[RV_SCORE_LSE_ORIG] = lse_o;
       sc[RV_SCORE_LSE_REFL] = lse_r;
       sc[RV_SCORE_LSE_FUSED] = lse_z;
       int choice = st.bi;
       float lp_z = nan, lp_o = nan, lp_r = nan;
+      int x = -1;
       if (i < gamma) {
-        const int x = drafts[b * gamma + i];
+        x = drafts[b * gamma + i];
         if (x >= 0 && x < V) {
           const float* gx = gathered + static_cast<long long>(p) * GATHER_FIELDS;
           const float zx = gx[2];
@@ -218,6 +225,7 @@ __global__ void head_finalize_kernel(const float* __restrict__ partials,
       sc[RV_SCORE_LOGP_REFL] = lp_r;
       argmax_out[p] = choice;
       s_choice[i] = choice;
+      s_kept[i] = position_kept(acc, x, choice, lp_z, ent) ? 1 : 0;
     }
     __syncthreads();
   }
@@ -225,7 +233,7 @@ __global__ void head_finalize_kernel(const float* __restrict__ partials,
   if (threadIdx.x == 0) {
     int n = gamma;
     for (int i = 0; i < gamma; ++i) {
-      const bool ok = drafts[b * gamma + i] == s_choice[i];
+      const bool ok = s_kept[i] != 0;
       acc.accept_mask[b * gamma + i] = ok ? 1 : 0;
       if (!ok && n == gamma) n = i;
     }
@@ -269,6 +277,37 @@ __global__ void accept_kernel(const int32_t* __restrict__ drafts,
   accepted_len[b] = n;
   next_token[b] = argmax[b * (gamma + 1) + n];
   ctx_out[b] = ctx_in[b] + n;
+}
+
+// ---------------------------------------------------------------- typical accept (Alg. 3)
+__global__ void accept_typical_kernel(const int32_t* __restrict__ drafts,
+                                      const float* __restrict__ scores,
+                                      const int32_t* __restrict__ argmax, int B, int gamma,
+                                      AcceptArgs a) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  int n = gamma;
+  for (int i = 0; i < gamma; ++i) {
+    const float* sc = scores + (static_cast<long long>(b) * (gamma + 1) + i) * RV_NSCORES;
+    const bool ok = position_kept(a, drafts[b * gamma + i], argmax[b * (gamma + 1) + i],
+                                  sc[RV_SCORE_LOGP_FUSED], sc[RV_SCORE_ENT_ORIG]);
+    a.accept_mask[b * gamma + i] = ok ? 1 : 0;
+    if (!ok && n == gamma) n = i;
+  }
+  a.accepted_len[b] = n;
+  a.next_token[b] = argmax[b * (gamma + 1) + n];
+  a.ctx_out[b] = a.ctx_in[b] + n;
+}
+
+cudaError_t launch_accept_typical(const int32_t* drafts, const float* scores,
+                                  const int32_t* argmax, int B, int gamma, float log_eps,
+                                  float log_delta, uint8_t* accept_mask, int32_t* accepted_len,
+                                  int32_t* next_token, const int32_t* ctx_in, int32_t* ctx_out,
+                                  cudaStream_t s) {
+  AcceptArgs a{accept_mask, accepted_len, next_token, ctx_in, ctx_out, RV_ACCEPT_TYPICAL, log_eps,
+               log_delta};
+  accept_typical_kernel<<<(B + 127) / 128, 128, 0, s>>>(drafts, scores, argmax, B, gamma, a);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_accept(const int32_t* drafts, const int32_t* argmax, int B, int gamma,

@@ -90,6 +90,9 @@ struct rv_handle {
   int head_pair_max = 0;
   int tm_h_box = -1;
   bool attn_tc_ok = false;  // tcgen05 attention usable for this configuration
+  // acceptance rule of rv_verify_step (rv_set_acceptance)
+  int accept_mode = RV_ACCEPT_EXACT;
+  float accept_log_eps = 0.f, accept_log_delta = 0.f;
   // tensor maps of the last tcgen05 attention call and what they were made for
   AttnTcMaps attn_maps;
   const void* attn_map_ptrs[5] = {nullptr, nullptr, nullptr, nullptr, nullptr};
@@ -587,6 +590,46 @@ extern "C" RV_API int rv_accept(rv_handle* h, const int32_t* draft_ids, const in
                      ctx_out, static_cast<cudaStream_t>(stream));
 }
 
+extern "C" RV_API int rv_accept_typical(rv_handle* h, const int32_t* draft_ids, const float* scores,
+                                        const int32_t* argmax, int32_t B, int32_t gamma, float eps,
+                                        float delta, uint8_t* accept_mask, int32_t* accepted_len,
+                                        int32_t* next_token, const int32_t* ctx_in,
+                                        int32_t* ctx_out, void* stream) {
+  if (!h) return RV_ERR_INVALID_ARG;
+  h->err.clear();
+  if (B < 0 || gamma < 1) return fail(h, RV_ERR_SHAPE, "need B >= 0 and gamma >= 1");
+  if (B > h->cfg.max_batch || gamma > h->cfg.max_gamma)
+    return fail(h, RV_ERR_CAPACITY, "B / gamma above the handle's maxima");
+  if (!(eps > 0.f) || !(delta > 0.f) || !std::isfinite(eps) || !std::isfinite(delta))
+    return fail(h, RV_ERR_INVALID_ARG, "typical acceptance needs finite eps > 0 and delta > 0");
+  if (B == 0) return RV_OK;
+  if (!draft_ids || !scores || !argmax || !accept_mask || !accepted_len || !next_token || !ctx_in ||
+      !ctx_out)
+    return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  ProfScope prof(h, RV_PROF_ACCEPT, s);
+  cudaError_t e = launch_accept_typical(draft_ids, scores, argmax, B, gamma, logf(eps), logf(delta),
+                                        accept_mask, accepted_len, next_token, ctx_in, ctx_out, s);
+  h->launches += 1;
+  return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "typical accept launch");
+}
+
+extern "C" RV_API int rv_set_acceptance(rv_handle* h, int32_t mode, float eps, float delta) {
+  if (!h) return RV_ERR_INVALID_ARG;
+  h->err.clear();
+  if (mode == RV_ACCEPT_EXACT) {
+    h->accept_mode = mode;
+    return RV_OK;
+  }
+  if (mode != RV_ACCEPT_TYPICAL) return fail(h, RV_ERR_INVALID_ARG, "unknown acceptance mode %d", mode);
+  if (!(eps > 0.f) || !(delta > 0.f) || !std::isfinite(eps) || !std::isfinite(delta))
+    return fail(h, RV_ERR_INVALID_ARG, "typical acceptance needs finite eps > 0 and delta > 0");
+  h->accept_mode = mode;
+  h->accept_log_eps = logf(eps);
+  h->accept_log_delta = logf(delta);
+  return RV_OK;
+}
+
 // ============================================================================ whole step
 
 extern "C" RV_API int rv_verify_step(
@@ -629,7 +672,8 @@ extern "C" RV_API int rv_verify_step(
   if (rc == RV_OK) {
     PackArgs pk{draft_ids, prompt_ids, prefix_ids, ctx_in, B, gamma, n_prompt, n_prefix, block_ids,
                 pos_ids};
-    AcceptArgs ac{accept_mask, accepted_len, next_token, ctx_in, ctx_out};
+    AcceptArgs ac{accept_mask, accepted_len,       next_token,         ctx_in,
+                  ctx_out,     h->accept_mode,     h->accept_log_eps,  h->accept_log_delta};
     rc = head_impl(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin,
                    do_pack ? &pk : nullptr, &ac, s);
   }

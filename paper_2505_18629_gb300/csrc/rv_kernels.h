@@ -11,7 +11,7 @@
 namespace rv {
 
 // Per-pair partial statistics written by each head CTA, merged by head_merge.
-// Layout [slot][pair][HEAD_STAT_FIELDS].
+// Layout [slot][pair][HEAD_STAT_FIELDS] (three 16-byte vectors per pair).
 enum HeadStat : int {
   ST_M_O = 0,  // running max of o_i over the CTA's vocab rows
   ST_S_O,      // sum exp(o_i - m)
@@ -21,7 +21,9 @@ enum HeadStat : int {
   ST_S_Z,
   ST_BEST_V,   // max of z_i over rows v != x_i
   ST_BEST_I,   // its row (int bits; smallest on ties)
-  HEAD_STAT_FIELDS
+  ST_T_O,      // sum exp(o_i - m) (o_i - m): with ST_S_O, the entropy of softmax(o_i)
+  HEAD_STAT_USED,
+  HEAD_STAT_FIELDS = 12
 };
 constexpr int GATHER_FIELDS = 4;  // o_i[x_i], o'_i[x_i], z_i[x_i], unused
 
@@ -43,12 +45,16 @@ struct HeadPlan {
 };
 
 // Optional acceptance fused into the head merge (rv_verify_step).
+// mode RV_ACCEPT_EXACT: x_i == argmax p_i (Alg. 2); RV_ACCEPT_TYPICAL:
+// log p_i(x_i) > min(log_eps, log_delta - H(softmax(o_i))) (Alg. 3).
 struct AcceptArgs {
   uint8_t* accept_mask;
   int32_t* accepted_len;
   int32_t* next_token;
   const int32_t* ctx_in;
   int32_t* ctx_out;
+  int mode;
+  float log_eps, log_delta;
 };
 
 // Outputs of the merge when the LM-head kernel finishes it itself (its last
@@ -104,6 +110,12 @@ cudaError_t launch_head_finalize(const HeadArgs& a, const HeadPlan& p, float* sc
 cudaError_t launch_accept(const int32_t* drafts, const int32_t* argmax, int B, int gamma,
                           uint8_t* accept_mask, int32_t* accepted_len, int32_t* next_token,
                           const int32_t* ctx_in, int32_t* ctx_out, cudaStream_t s);
+// Typical acceptance (Alg. 3) from the head's scores and argmax.
+cudaError_t launch_accept_typical(const int32_t* drafts, const float* scores,
+                                  const int32_t* argmax, int B, int gamma, float log_eps,
+                                  float log_delta, uint8_t* accept_mask, int32_t* accepted_len,
+                                  int32_t* next_token, const int32_t* ctx_in, int32_t* ctx_out,
+                                  cudaStream_t s);
 
 // ---- LM head (k_head_tc.cu: bf16 tcgen05; k_head_simt.cu: fp32)
 // Vocab rows per TMA box of the weight: full tiles use HEAD_TILE_ROWS, the

@@ -32,9 +32,12 @@ RV_DEV_TIMEOUT = 4
 RV_DTYPE_BF16 = 0
 RV_DTYPE_F32 = 1
 
-RV_NSCORES = 6
+RV_NSCORES = 7
 RV_SCORE_LSE_ORIG, RV_SCORE_LSE_REFL, RV_SCORE_LSE_FUSED = 0, 1, 2
 RV_SCORE_LOGP_FUSED, RV_SCORE_LOGP_ORIG, RV_SCORE_LOGP_REFL = 3, 4, 5
+RV_SCORE_ENT_ORIG = 6
+
+RV_ACCEPT_EXACT, RV_ACCEPT_TYPICAL = 0, 1
 
 RV_PROF_ATTENTION, RV_PROF_HEAD_GEMM, RV_PROF_HEAD, RV_PROF_ACCEPT = 0, 1, 2, 3
 
@@ -70,6 +73,8 @@ def _load():
         "rv_verify_attention": (I, [P, P, P, P, P, P, P, I, I, P, P]),
         "rv_verify_head": (I, [P, P, P, P, I, I, I, F, P, P, P, P]),
         "rv_accept": (I, [P, P, P, I, I, P, P, P, P, P, P]),
+        "rv_accept_typical": (I, [P, P, P, P, I, I, F, F, P, P, P, P, P, P]),
+        "rv_set_acceptance": (I, [P, I, F, F]),
         "rv_verify_step": (I, [P, P, P, P, P, P, P, P, P, P, P, P, I, I, I, I, F, P, P, P, P, P, P,
                                P, P, P, P, P]),
         "rv_verify_step_host": (I, [P, P, P, P, P, P, P, P, P, P, P, P, I, I, I, I, F, P, P, P, P,
@@ -195,6 +200,19 @@ def rv_accept(h, draft_ids, argmax, accept_mask, accepted_len, next_token, ctx_i
     _check(h, _lib.rv_accept(h.ptr, _ptr(draft_ids), _ptr(argmax), B, gamma, _ptr(accept_mask),
                              _ptr(accepted_len), _ptr(next_token), _ptr(ctx_in), _ptr(ctx_out),
                              _stream(stream)))
+
+
+def rv_accept_typical(h, draft_ids, scores, argmax, eps, delta, accept_mask, accepted_len,
+                      next_token, ctx_in, ctx_out, stream=None):
+    B, gamma = draft_ids.shape
+    _check(h, _lib.rv_accept_typical(h.ptr, _ptr(draft_ids), _ptr(scores), _ptr(argmax), B, gamma,
+                                     float(eps), float(delta), _ptr(accept_mask),
+                                     _ptr(accepted_len), _ptr(next_token), _ptr(ctx_in),
+                                     _ptr(ctx_out), _stream(stream)))
+
+
+def rv_set_acceptance(h, mode, eps=0.0, delta=0.0):
+    _check(h, _lib.rv_set_acceptance(h.ptr, int(mode), float(eps), float(delta)))
 
 
 def rv_verify_step(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, prompt_ids,

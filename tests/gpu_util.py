@@ -171,9 +171,13 @@ def compare(inp: synth.VerifyInputs, drafts, alpha, ref: dict, gpu: GpuRun, chec
                    np.abs(sc[:, :g, 4] - ref["logp_orig"]).max(),
                    np.abs(sc[:, :g, 5] - ref["logp_refl"]).max())
     assert logp_err <= LOGP_ATOL, f"log-prob error {logp_err}"
-    assert np.isnan(sc[:, g, 3:]).all()
+    assert np.isnan(sc[:, g, 3:6]).all()
+    ent_err = np.abs(sc[..., 6] - ref["ent_orig"]).max()
+    assert ent_err <= LOGP_ATOL, f"entropy error {ent_err}"
     m_err = np.abs(gpu.margin[seqs].astype(np.float64) - ref["margin"]).max()
     assert m_err <= LOGP_ATOL, f"margin error {m_err}"
+    if "typical_gap" in ref:
+        return _compare_typical(inp, ref, gpu, seqs, lse_err, logp_err, m_err, amax)
     # ---- decisions with the margin rule
     low = ref["margin"] < MARGIN_EPS                       # [S, gamma]
     low_choice = ref["choice_gap"] < MARGIN_EPS            # [S, gamma+1]
@@ -196,6 +200,46 @@ def compare(inp: synth.VerifyInputs, drafts, alpha, ref: dict, gpu: GpuRun, chec
         assert gpu.next_token[b] == gpu.argmax[b, n]
     return Report(int(low.size), int(low.sum()), int(mask_mismatch.sum()), excused,
                   float(lse_err), float(logp_err), float(m_err), amax)
+
+
+def _compare_typical(inp, ref, gpu, seqs, lse_err, logp_err, m_err, amax) -> Report:
+    """Typical acceptance (Alg. 3): decisions bit-exact except where the oracle's
+    log p_i(x_i) is within MARGIN_EPS of the log threshold (counted); n and t may
+    differ only past such a position; t is the greedy choice at n+1."""
+    wl = inp.wl
+    g = wl.gamma
+    low = np.abs(ref["typical_gap"]) < MARGIN_EPS
+    low_choice = ref["choice_gap"] < MARGIN_EPS
+    am_ok = (gpu.argmax[seqs] == ref["argmax"]) | low_choice
+    assert am_ok.all(), "argmax differs at a position with a clear choice"
+    mism = gpu.accept_mask[seqs] != ref["accept_mask"]
+    assert not (mism & ~low).any(), "typical accept mask differs at a clear decision"
+    excused = 0
+    for k, b in enumerate(seqs):
+        n_ref = int(ref["accepted_len"][k])
+        same = gpu.accepted_len[b] == n_ref and gpu.next_token[b] == ref["next_token"][k]
+        if not same:
+            lim = min(n_ref + 1, g)
+            assert low[k, :lim].any() or low_choice[k, min(n_ref, g)], \
+                f"sequence {b}: accepted {gpu.accepted_len[b]} vs {n_ref} without a close decision"
+            excused += 1
+        assert gpu.ctx_out[b] == inp.ctx_lens[b] + gpu.accepted_len[b]
+        n = int(gpu.accepted_len[b])
+        assert gpu.accept_mask[b, :n].all() and (n == g or gpu.accept_mask[b, n] == 0)
+        assert gpu.next_token[b] == gpu.argmax[b, n]
+    return Report(int(low.size), int(low.sum()), int(mism.sum()), excused, float(lse_err),
+                  float(logp_err), float(m_err), amax)
+
+
+def oracle_typical(inp, drafts, alpha, eps, delta, seqs=None, with_attn=True):
+    """Oracle verify step with the typical acceptance of Alg. 3."""
+    ref = oracle_step(inp, drafts, alpha, seqs=seqs, with_attn=with_attn)
+    wl = inp.wl
+    seqs = np.arange(wl.B) if seqs is None else np.asarray(seqs)
+    acc, n, t, gap = orc.typical_accept(drafts[seqs], ref["logp_fused"], ref["ent_orig"],
+                                        ref["argmax"], eps, delta)
+    ref.update(accept_mask=acc.astype(np.uint8), accepted_len=n, next_token=t, typical_gap=gap)
+    return ref
 
 
 def _bits_like(ref_f64: np.ndarray, like: np.ndarray) -> np.ndarray:

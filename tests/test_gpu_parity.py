@@ -315,6 +315,88 @@ def test_host_validation_errors(gu):
     h.close()
 
 
+# ------------------------------------------------------------------ typical acceptance (Alg. 3)
+
+def _typical_params(gu, inp, drafts, alpha, bind):
+    """eps / delta that split the drafts about half and half: the entropy term
+    binds (bind='delta') or the constant eps does (bind='eps')."""
+    ref = gu.oracle_step(inp, drafts, alpha, with_attn=False)
+    p = np.exp(ref["logp_fused"])
+    if bind == "delta":
+        return 1.0, float(np.median(p * np.exp(ref["ent_orig"][:, :-1])))
+    return float(np.median(p)), 1e30
+
+
+@pytest.mark.parametrize("bind", ["delta", "eps"])
+def test_typical_acceptance_step(gu, bind):
+    from paper_2505_18629_gb300 import rv, synth
+    wl = _wl(B=6, gamma=5, seed=70)
+    inp = synth.generate(wl)
+    drafts = gu.oracle_drafts(inp, ALPHA)
+    eps, delta = _typical_params(gu, inp, drafts, ALPHA, bind)
+    h = gu.make_handle(wl)
+    rv.rv_set_acceptance(h, rv.RV_ACCEPT_TYPICAL, eps, delta)
+    gpu = gu.run_gpu(inp, drafts, ALPHA, h=h)
+    ref = gu.oracle_typical(inp, drafts, ALPHA, eps, delta)
+    rep = gu.compare(inp, drafts, ALPHA, ref, gpu)
+    assert 0 < ref["accept_mask"].sum() < ref["accept_mask"].size
+    print(f"\ntypical ({bind}): {rep}")
+    # back to exact match on the same handle
+    rv.rv_set_acceptance(h, rv.RV_ACCEPT_EXACT)
+    gpu = gu.run_gpu(inp, drafts, ALPHA, h=h)
+    gu.compare(inp, drafts, ALPHA, gu.oracle_step(inp, drafts, ALPHA), gpu)
+    h.close()
+
+
+def test_typical_acceptance_separate_entry_points(gu):
+    import torch
+    from paper_2505_18629_gb300 import rv, synth
+    wl = _wl(B=5, gamma=4, seed=71)
+    inp = synth.generate(wl)
+    drafts = gu.oracle_drafts(inp, ALPHA)
+    eps, delta = _typical_params(gu, inp, drafts, ALPHA, "delta")
+    h = gu.make_handle(wl)
+    B, g = wl.B, wl.gamma
+    d = gu.to_dev(drafts.astype(np.int32))
+    sc = torch.empty((B, g + 1, rv.RV_NSCORES), device="cuda")
+    am = torch.empty((B, g + 1), dtype=torch.int32, device="cuda")
+    mg = torch.empty((B, g), device="cuda")
+    rv.rv_verify_head(h, gu.to_dev(inp.hidden), gu.to_dev(inp.W), d, g, wl.R, ALPHA, sc, am, mg)
+    acc = torch.empty((B, g), dtype=torch.uint8, device="cuda")
+    n = torch.empty((B,), dtype=torch.int32, device="cuda")
+    t = torch.empty_like(n)
+    ctx = gu.to_dev(inp.ctx_lens.astype(np.int32))
+    co = torch.empty_like(ctx)
+    rv.rv_accept_typical(h, d, sc, am, eps, delta, acc, n, t, ctx, co)
+    ref = gu.oracle_typical(inp, drafts, ALPHA, eps, delta, with_attn=False)
+    low = np.abs(ref["typical_gap"]) < gu.MARGIN_EPS
+    assert not ((gu.to_np(acc) != ref["accept_mask"]) & ~low).any()
+    if not low.any():
+        np.testing.assert_array_equal(gu.to_np(n), ref["accepted_len"])
+        np.testing.assert_array_equal(gu.to_np(t), ref["next_token"])
+    np.testing.assert_allclose(gu.to_np(sc)[..., rv.RV_SCORE_ENT_ORIG], ref["ent_orig"], atol=gu.LOGP_ATOL)
+    with pytest.raises(rv.RVError):
+        rv.rv_accept_typical(h, d, sc, am, 0.0, delta, acc, n, t, ctx, co)
+    with pytest.raises(rv.RVError):
+        rv.rv_set_acceptance(h, 7, 0.1, 0.1)
+    h.close()
+
+
+def test_typical_acceptance_fp32_and_pairs(gu):
+    # the fp32 CUDA-core head and the CTA-pair tensor-core head (N >= 96)
+    from paper_2505_18629_gb300 import rv, synth
+    for wl in (synth.WORKLOADS["tiny"], _wl(B=14, gamma=8, R=8, V=777, H=256, ctx=(10, 60), seed=72)):
+        inp = synth.generate(wl)
+        drafts = gu.oracle_drafts(inp, ALPHA)
+        eps, delta = _typical_params(gu, inp, drafts, ALPHA, "delta")
+        h = gu.make_handle(wl)
+        rv.rv_set_acceptance(h, rv.RV_ACCEPT_TYPICAL, eps, delta)
+        gpu = gu.run_gpu(inp, drafts, ALPHA, h=h)
+        ref = gu.oracle_typical(inp, drafts, ALPHA, eps, delta)
+        gu.compare(inp, drafts, ALPHA, ref, gpu)
+        h.close()
+
+
 # ------------------------------------------------------------------ full-size workloads
 
 def test_llama3_8b_b1_full(gu):
@@ -326,6 +408,20 @@ def test_llama3_8b_b1_full(gu):
 def test_llama3_8b_b16_full(gu):
     from paper_2505_18629_gb300 import synth
     _check(gu, synth.WORKLOADS["llama3-8b-b16"])
+
+
+def test_llama3_8b_b16_typical(gu):
+    from paper_2505_18629_gb300 import rv, synth
+    wl = synth.WORKLOADS["llama3-8b-b16"]
+    inp = synth.generate(wl)
+    drafts = gu.oracle_drafts(inp, ALPHA)
+    eps, delta = _typical_params(gu, inp, drafts, ALPHA, "delta")
+    h = gu.make_handle(wl)
+    rv.rv_set_acceptance(h, rv.RV_ACCEPT_TYPICAL, eps, delta)
+    gpu = gu.run_gpu(inp, drafts, ALPHA, h=h)
+    ref = gu.oracle_typical(inp, drafts, ALPHA, eps, delta, with_attn=False)
+    gu.compare(inp, drafts, ALPHA, ref, gpu, check_attn=False)
+    h.close()
 
 
 def test_llama3_70b_b32_sampled(gu):

@@ -57,7 +57,8 @@ def test_static_head_matches_handle_head_on_two_calls(env):
         sr, sg = gu.to_np(ref[0]), gu.to_np(got[0])
         np.testing.assert_allclose(sg[..., :3], sr[..., :3], atol=gu.LOGP_ATOL, rtol=0)
         np.testing.assert_allclose(sg[:, :-1, 3:], sr[:, :-1, 3:], atol=gu.LOGP_ATOL, rtol=0)
-        assert np.isnan(sg[:, -1, 3:]).all()
+        assert np.isnan(sg[:, -1, 3:6]).all()                 # no draft at the bonus position
+        np.testing.assert_allclose(sg[..., 6], sr[..., 6], atol=gu.LOGP_ATOL, rtol=0)  # entropy
         np.testing.assert_allclose(gu.to_np(got[2]), gu.to_np(ref[2]), atol=gu.LOGP_ATOL, rtol=0)
         close = gu.to_np(ref[2]) < gu.MARGIN_EPS
         am_r, am_g = gu.to_np(ref[1]), gu.to_np(got[1])

@@ -292,6 +292,59 @@ def typical_accept(drafts, logp_fused, ent_orig, choice, eps: float, delta: floa
     return acc, n, t, gap
 
 
+def inverse_cdf_sample(w: np.ndarray, u: float) -> int:
+    """The token drawn from the distribution proportional to w >= 0 by one
+    uniform u in [0, 1): the smallest v whose cumulative weight exceeds u * sum(w)."""
+    w = np.asarray(w, np.float64)
+    c = np.cumsum(w)
+    return int(min(np.searchsorted(c, u * c[-1], side="right"), len(w) - 1))
+
+
+def speculative_accept(drafts, z, q, r, u):
+    """Speculative sampling with Reflective Verification (Alg. 1).
+
+    drafts [B, gamma]; z [B, gamma+1, V] fused logits (p_i = softmax(z_i),
+    Eq. 2); q [B, gamma, V] the draft model's distributions q_i; r [B, gamma]
+    the uniforms r_i ~ U(0, 1); u [B] one more uniform per sequence for t.
+    n is the number of leading drafts with r_i <= p_i(x_i) / q_i(x_i) (Alg. 1
+    stops at the first i with r_i > p_i(x_i) / q_i(x_i)); t ~ p' with
+    p' = norm(max(0, p_{n+1} - q_{n+1})) when n < gamma, else p' = p_{gamma+1},
+    drawn by inverse CDF with u.
+
+    Returns (accept_mask [B, gamma] bool, n [B], t [B], log_ratio [B, gamma],
+    cdf_gap [B]) where log_ratio = log p_i(x_i) - log q_i(x_i) and cdf_gap is
+    the distance of u from the nearest cumulative-weight boundary of p'
+    (normalised), which bounds how close the draw of t was to a tie.
+    """
+    drafts = np.asarray(drafts, np.int64)
+    z = np.asarray(z, np.float64)
+    q = np.asarray(q, np.float64)
+    r = np.asarray(r, np.float64)
+    B, gamma = drafts.shape
+    logp = z - logsumexp(z)[..., None]
+    bi = np.arange(B)[:, None]
+    ii = np.arange(gamma)[None, :]
+    with np.errstate(divide="ignore"):
+        log_ratio = logp[bi, ii, drafts] - np.log(q[bi, ii, drafts])
+    acc = np.log(r) <= log_ratio
+    n = np.full(B, gamma, np.int64)
+    t = np.zeros(B, np.int64)
+    cdf_gap = np.zeros(B)
+    for b in range(B):
+        for i in range(gamma):
+            if not acc[b, i]:
+                n[b] = i
+                break
+        p_next = np.exp(logp[b, n[b]])
+        w = np.maximum(0.0, p_next - q[b, n[b]]) if n[b] < gamma else p_next
+        if not w.sum() > 0:  # p_{n+1} <= q_{n+1} everywhere: only possible through rounding
+            w = p_next
+        t[b] = inverse_cdf_sample(w, float(u[b]))
+        c = np.cumsum(w) / w.sum()
+        cdf_gap[b] = np.min(np.abs(c - u[b]))
+    return acc, n, t, log_ratio, cdf_gap
+
+
 def verify_step(inp_W, hidden, q, k_blk, v_blk, k_cache, v_cache, ctx_lens,
                 drafts, prompt_ids, prefix_ids, gamma: int, R: int, alpha: float):
     """One whole verify step: pack, attention, head + fusion, accept, prefix.

@@ -486,3 +486,106 @@ def test_pins_catch_swapped_threshold_parameters(monkeypatch):
     real = orc.typical_accept
     monkeypatch.setattr(orc, "typical_accept", swapped)
     assert _fails(test_typical_threshold_worked_example)
+
+
+# ------------------------------------------------------------------ Alg. 1: speculative sampling
+
+def test_inverse_cdf_sample_closed_forms():
+    w = np.array([0.1, 0.0, 0.3, 0.6])
+    assert orc.inverse_cdf_sample(w, 0.0) == 0
+    assert orc.inverse_cdf_sample(w, 0.0999) == 0
+    assert orc.inverse_cdf_sample(w, 0.1001) == 2          # a zero weight is never drawn
+    assert orc.inverse_cdf_sample(w, 0.3999) == 2
+    assert orc.inverse_cdf_sample(w, 0.4001) == 3
+    assert orc.inverse_cdf_sample(w, 0.999999) == 3
+    assert orc.inverse_cdf_sample(5.0 * w, 0.25) == 2       # scale-free
+    # a midpoint grid of u reproduces w / sum(w) exactly
+    grid = (np.arange(1000) + 0.5) / 1000
+    hits = np.bincount([orc.inverse_cdf_sample(w, x) for x in grid], minlength=4) / 1000
+    np.testing.assert_allclose(hits, w / w.sum(), atol=1e-3)
+
+
+def _spec_case(rng, B, gamma, V, same=False):
+    z = rng.normal(0, 1.5, (B, gamma + 1, V))
+    q = scipy.special.softmax(rng.normal(0, 1.5, (B, gamma, V)), axis=-1)
+    if same:
+        q = scipy.special.softmax(z[:, :gamma], axis=-1)
+    drafts = np.array([[rng.choice(V, p=q[b, i]) for i in range(gamma)] for b in range(B)])
+    return z, q, drafts
+
+
+def test_speculative_draft_equal_to_target_accepts_everything():
+    # q_i = p_i: every ratio is 1 and r_i < 1 keeps every draft; t ~ p_{gamma+1}
+    rng = np.random.default_rng(21)
+    z, q, drafts = _spec_case(rng, 8, 4, 11, same=True)
+    r = rng.uniform(0, 1, (8, 4))
+    u = rng.uniform(0, 1, 8)
+    acc, n, t, lr, _ = orc.speculative_accept(drafts, z, q, r, u)
+    assert acc.all() and (n == 4).all()
+    np.testing.assert_allclose(lr, 0.0, atol=1e-12)
+    p_last = scipy.special.softmax(z[:, 4], axis=-1)
+    for b in range(8):
+        assert t[b] == orc.inverse_cdf_sample(p_last[b], u[b])
+
+
+def test_speculative_first_token_is_distributed_as_p1():
+    # The speculative-sampling guarantee (Alg. 1): over x_1 ~ q_1, r_1 and u the
+    # first emitted token (x_1 if kept, else t) has distribution p_1 exactly.
+    # Evaluated by quadrature with the oracle itself: a midpoint grid of r_1
+    # gives P(keep x_1), and a midpoint grid of u the law of t after a rejection.
+    rng = np.random.default_rng(22)
+    V, gamma = 6, 1
+    z = rng.normal(0, 1.0, (1, gamma + 1, V))
+    q = scipy.special.softmax(rng.normal(0, 1.0, (1, gamma, V)), axis=-1)
+    p1 = scipy.special.softmax(z[0, 0])
+    r_grid = (np.arange(2000) + 0.5) / 2000
+    u_grid = (np.arange(2000) + 0.5) / 2000
+    dist = np.zeros(V)
+    for x1 in range(V):
+        d = np.array([[x1]])
+        keep = np.mean([orc.speculative_accept(d, z, q, np.array([[r1]]), np.array([0.5]))[0][0, 0]
+                        for r1 in r_grid])
+        dist[x1] += q[0, 0, x1] * keep
+        if keep < 1.0:
+            for uu in u_grid:  # r_1 just below 1 rejects every draft with p_1(x_1) < q_1(x_1)
+                t = orc.speculative_accept(d, z, q, np.array([[1 - 1e-12]]), np.array([uu]))[2][0]
+                dist[t] += q[0, 0, x1] * (1.0 - keep) / len(u_grid)
+    np.testing.assert_allclose(dist, p1, atol=2e-3)
+    assert abs(dist.sum() - 1.0) < 1e-9
+
+
+def test_speculative_stopping_and_residual():
+    rng = np.random.default_rng(23)
+    B, gamma, V = 32, 5, 9
+    z, q, drafts = _spec_case(rng, B, gamma, V)
+    r = rng.uniform(0, 1, (B, gamma))
+    u = rng.uniform(0, 1, B)
+    acc, n, t, lr, gap = orc.speculative_accept(drafts, z, q, r, u)
+    p = scipy.special.softmax(z, axis=-1)
+    for b in range(B):
+        assert acc[b, :n[b]].all() and (n[b] == gamma or not acc[b, n[b]])
+        if n[b] < gamma:
+            w = np.maximum(0, p[b, n[b]] - q[b, n[b]])
+            assert w[t[b]] > 0                                 # t lies where p exceeds q
+            # the residual never proposes the rejected draft more than p allows
+        else:
+            assert p[b, gamma, t[b]] > 0
+    # r = 0 keeps every draft with p_i(x_i) > 0; r -> 1 keeps only drafts with p >= q
+    acc0, n0, *_ = orc.speculative_accept(drafts, z, q, np.full((B, gamma), 1e-300), u)
+    assert acc0.all() and (n0 == gamma).all()
+    acc1, *_ = orc.speculative_accept(drafts, z, q, np.full((B, gamma), 1 - 1e-12), u)
+    np.testing.assert_array_equal(acc1, lr >= np.log1p(-1e-12))
+
+
+def test_pins_catch_plain_p_instead_of_residual(monkeypatch):
+    real = orc.speculative_accept
+
+    def plain(drafts, z, q, r, u):
+        # planted slip: t ~ p_{n+1} even after a rejection (no residual)
+        acc, n, t, lr, gap = real(drafts, z, q, r, u)
+        logp = np.asarray(z) - orc.logsumexp(np.asarray(z))[..., None]
+        t = np.array([orc.inverse_cdf_sample(np.exp(logp[b, n[b]]), float(u[b]))
+                      for b in range(len(n))])
+        return acc, n, t, lr, gap
+    monkeypatch.setattr(orc, "speculative_accept", plain)
+    assert _fails(test_speculative_first_token_is_distributed_as_p1)

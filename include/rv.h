@@ -80,6 +80,7 @@ extern "C" {
 /* Acceptance rules (rv_set_acceptance). */
 #define RV_ACCEPT_EXACT 0       /* exact match with the greedy choice (Alg. 2)               */
 #define RV_ACCEPT_TYPICAL 1     /* entropy-based threshold of typical acceptance (Alg. 3)     */
+#define RV_ACCEPT_SPECULATIVE 2 /* speculative sampling with residual resampling (Alg. 1)     */
 
 /* Model / capacity description fixed at creation. */
 typedef struct rv_config {
@@ -195,11 +196,40 @@ RV_API int rv_accept_typical(rv_handle* h, const int32_t* draft_ids, const float
                              int32_t* next_token, const int32_t* ctx_in, int32_t* ctx_out,
                              void* stream);
 
-/* Acceptance rule used by rv_verify_step (and rv_verify_step_host) on this
- * handle: RV_ACCEPT_EXACT (the default; eps and delta ignored) or
- * RV_ACCEPT_TYPICAL with its eps > 0 and delta > 0 (see rv_accept_typical).
- * Host-side setting, takes effect for the following calls. */
+/* Acceptance rule of this handle, for the following calls:
+ *   RV_ACCEPT_EXACT (the default; eps and delta ignored) and RV_ACCEPT_TYPICAL
+ *     (eps > 0, delta > 0; see rv_accept_typical) apply to rv_verify_step and
+ *     rv_verify_step_host;
+ *   RV_ACCEPT_SPECULATIVE makes every LM-head call (rv_verify_head, the step)
+ *     also write its fused logits z_i to a buffer of the handle (allocated
+ *     here once: max_batch * (max_gamma+1) * vocab floats), which
+ *     rv_accept_speculative and rv_verify_step_speculative read; in this mode
+ *     plain rv_verify_step returns RV_ERR_INVALID_ARG (it has no draft
+ *     distributions).
+ * Errors: RV_ERR_INVALID_ARG for an unknown mode or bad eps / delta,
+ * RV_ERR_CUDA if the buffer cannot be allocated. */
 RV_API int rv_set_acceptance(rv_handle* h, int32_t mode, float eps, float delta);
+
+/* Speculative sampling with Reflective Verification (Alg. 1), after an
+ * rv_verify_head call on this handle in RV_ACCEPT_SPECULATIVE mode (same
+ * stream, same B and gamma):
+ *   accept_mask[b][i-1] = r_i <= p_i(x_i) / q_i(x_i)       uint8 [B, gamma]
+ *     (tested as log r_i <= log p_i(x_i) - log q_i(x_i), p_i the fused
+ *      distribution of Eq. 2; q_i(x_i) = 0 keeps the draft)
+ *   accepted_len[b] = n = number of leading kept drafts       int32 [B]
+ *   next_token[b]   = t ~ norm(max(0, p_{n+1} - q_{n+1})) if n < gamma, else
+ *                     t ~ p_{gamma+1}, drawn by inverse CDF with u: the
+ *                     smallest v whose cumulative weight exceeds u * sum(w)
+ *   ctx_out[b]      = ctx_in[b] + n (may alias ctx_in)
+ * Inputs (device, float32): q_draft [B, gamma, vocab] the draft model's
+ * distributions q_i (rows sum to 1), r_uniform [B, gamma] and u_uniform [B]
+ * in [0, 1); scores as written by the preceding rv_verify_head.  Draft ids
+ * outside [0, vocab) are rejected and set RV_DEV_DRAFT_RANGE. */
+RV_API int rv_accept_speculative(rv_handle* h, const int32_t* draft_ids, const float* q_draft,
+                                 const float* r_uniform, const float* u_uniform,
+                                 const float* scores, int32_t B, int32_t gamma,
+                                 uint8_t* accept_mask, int32_t* accepted_len, int32_t* next_token,
+                                 const int32_t* ctx_in, int32_t* ctx_out, void* stream);
 
 /* The whole verify step on device buffers, in one call and four kernel
  * launches: the attention (rv_verify_attention) on an internal stream forked
@@ -221,6 +251,19 @@ RV_API int rv_verify_step(rv_handle* h, const void* q, const void* k_blk, const 
                           int32_t* argmax, float* margin, uint8_t* accept_mask,
                           int32_t* accepted_len, int32_t* next_token, int32_t* ctx_out,
                           void* stream);
+
+/* rv_verify_step with the speculative-sampling acceptance of Alg. 1
+ * (rv_accept_speculative) in place of the handle's fused rule; needs the
+ * handle in RV_ACCEPT_SPECULATIVE mode.  q_draft, r_uniform, u_uniform as in
+ * rv_accept_speculative; one more launch than rv_verify_step. */
+RV_API int rv_verify_step_speculative(
+    rv_handle* h, const void* q, const void* k_blk, const void* v_blk, void* k_cache,
+    void* v_cache, const void* hidden, const void* w_head, const int32_t* draft_ids,
+    const int32_t* prompt_ids, const int32_t* prefix_ids, const int32_t* ctx_in, int32_t B,
+    int32_t gamma, int32_t n_prompt, int32_t n_prefix, float alpha, const float* q_draft,
+    const float* r_uniform, const float* u_uniform, int32_t* block_ids, int32_t* pos_ids,
+    void* attn_out, float* scores, int32_t* argmax, float* margin, uint8_t* accept_mask,
+    int32_t* accepted_len, int32_t* next_token, int32_t* ctx_out, void* stream);
 
 /* The whole verify step from HOST buffers (synchronous).  The per-step inputs
  * (q, k_blk, v_blk, hidden, draft / prompt / prefix ids, ctx lens) are copied

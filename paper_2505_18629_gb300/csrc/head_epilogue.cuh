@@ -61,7 +61,8 @@ __device__ __forceinline__ void head_stats_init(float* stats, int n_entries, int
 __device__ __forceinline__ void head_tile_pairs8(const float (&o)[8], const float (&r)[8], int g8,
                                                  int npairs, int v, bool valid, float alpha,
                                                  const int* s_drafts, float* warp_stats,
-                                                 float* gathered, int lane) {
+                                                 float* gathered, int lane, float* zout = nullptr,
+                                                 int V = 0) {
   const float beta = 1.f - alpha;
   float ov[8], rv[8], zv[8], Mo[8], Mr[8], Mz[8], bv[8];
   int bi[8];
@@ -72,6 +73,7 @@ __device__ __forceinline__ void head_tile_pairs8(const float (&o)[8], const floa
     ov[j] = valid ? o[j] : NEG_INF;
     rv[j] = valid ? r[j] : NEG_INF;
     zv[j] = valid ? fmaf(alpha, r[j], beta * o[j]) : NEG_INF;
+    if (zout != nullptr && valid && pj < npairs) zout[static_cast<long long>(pj) * V + v] = zv[j];
     if (valid && v == x && pj < npairs) {
       float* gx = gathered + pj * GATHER_FIELDS;
       gx[0] = ov[j];
@@ -162,13 +164,17 @@ constexpr int HEAD_SCR_FLOATS = 32 * HEAD_SCR_STRIDE;
 __device__ __forceinline__ void head_tile_pairs8_t(const float (&o)[8], const float (&r)[8], int g8,
                                                    int npairs, int v, bool valid, float alpha,
                                                    const int* s_drafts, float* warp_stats,
-                                                   float* gathered, float* scr, int lane) {
+                                                   float* gathered, float* scr, int lane,
+                                                   float* zout = nullptr, int V = 0) {
   const float beta = 1.f - alpha;
   float zr[8];
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
     const int pj = g8 + j;
     zr[j] = fmaf(alpha, r[j], beta * o[j]);
+    // fused logits for the residual draw of speculative sampling (Alg. 1):
+    // a warp store covers 32 consecutive vocab rows of one pair
+    if (zout != nullptr && valid && pj < npairs) zout[static_cast<long long>(pj) * V + v] = zr[j];
     if (valid && v == s_drafts[pj] && pj < npairs) {
       float* gx = gathered + pj * GATHER_FIELDS;
       gx[0] = o[j];

@@ -23,6 +23,7 @@ struct HeadSimtParams {
   const int32_t* drafts;
   float* partials;
   float* gathered;
+  float* zout;  // [P][V] fused logits, or null
 };
 
 __global__ void __launch_bounds__(HS_BM) head_simt_kernel(const HeadSimtParams p) {
@@ -82,7 +83,8 @@ __global__ void __launch_bounds__(HS_BM) head_simt_kernel(const HeadSimtParams p
           }
         }
       }
-      head_tile_pairs8(o, r, g8, npairs, v, valid, p.alpha, s_drafts, wstats, gathered, lane);
+      head_tile_pairs8(o, r, g8, npairs, v, valid, p.alpha, s_drafts, wstats, gathered, lane,
+                       p.zout ? p.zout + static_cast<long long>(pair0) * p.V : nullptr, p.V);
     }
   }
   __syncthreads();
@@ -108,6 +110,7 @@ cudaError_t launch_head_simt(const HeadArgs& a, const HeadPlan& pl, cudaStream_t
   p.drafts = a.drafts;
   p.partials = a.partials;
   p.gathered = a.gathered;
+  p.zout = a.zout;
   dim3 grid(pl.slots, pl.n_chunks);
   head_simt_kernel<<<grid, HS_BM, 0, s>>>(p);
   return cudaGetLastError();

@@ -55,6 +55,7 @@ struct Head2Params {
   const int32_t* drafts;
   float* partials;
   float* gathered;
+  float* zout;  // [P][V] fused logits, or null
   unsigned* status;
 };
 
@@ -304,7 +305,8 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
         tmem_ld8(trow + p.Pcp + g8, r);
         tmem_ld_wait();
         head_tile_pairs8_t(o, r, g8, npairs, v, valid, p.alpha, s_drafts, wstats, gathered,
-                           scr_base + ew * HEAD_SCR_FLOATS, lane);
+                           scr_base + ew * HEAD_SCR_FLOATS, lane,
+                           p.zout ? p.zout + static_cast<long long>(pair0) * p.V : nullptr, p.V);
       }
       tc_fence_before();
       __syncwarp();
@@ -437,6 +439,7 @@ cudaError_t launch_head_tc2(const HeadArgs& a, const HeadPlan& pl, const HeadTcL
   p.drafts = a.drafts;
   p.partials = a.partials;
   p.gathered = a.gathered;
+  p.zout = a.zout;
   p.status = a.status;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(pl.slots, pl.n_chunks, 1);

@@ -279,6 +279,133 @@ __global__ void accept_kernel(const int32_t* __restrict__ drafts,
   ctx_out[b] = ctx_in[b] + n;
 }
 
+// ---------------------------------------------------------------- speculative accept (Alg. 1)
+// One CTA per sequence.  Thread 0 runs the ratio test: draft i is kept while
+// log r_i <= log p_i(x_i) - log q_i(x_i) (p_i from the head's fused log-prob),
+// n = the number of leading kept drafts.  Then the CTA draws t from
+//   p' = norm(max(0, p_{n+1} - q_{n+1}))  (n < gamma)   or   p_{gamma+1}
+// by inverse CDF with u: each thread sums the weights of a contiguous range of
+// the vocabulary, a block-wide exclusive scan orders the ranges, and the
+// thread whose range holds u * sum(w) walks it to the token.
+constexpr int SPEC_THREADS = 1024;
+
+__device__ __forceinline__ float spec_weight(const float* zrow, const float* qrow, float lse, int v) {
+  const float p = __expf(zrow[v] - lse);
+  return qrow ? fmaxf(0.f, p - qrow[v]) : p;
+}
+
+__global__ void __launch_bounds__(SPEC_THREADS)
+    accept_speculative_kernel(const int32_t* __restrict__ drafts, const float* __restrict__ q,
+                              const float* __restrict__ r, const float* __restrict__ u,
+                              const float* __restrict__ scores, const float* __restrict__ z,
+                              int gamma, int V, AcceptArgs a, unsigned* status) {
+  constexpr int NW = SPEC_THREADS / 32;
+  __shared__ float s_wtot[NW], s_woff[NW];
+  __shared__ float s_total;
+  __shared__ int s_n, s_t, s_last;
+  const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (tid == 0) {
+    int n = gamma;
+    for (int i = 0; i < gamma; ++i) {
+      const int x = drafts[b * gamma + i];
+      const float logp = scores[(static_cast<long long>(b) * (gamma + 1) + i) * RV_NSCORES +
+                                RV_SCORE_LOGP_FUSED];
+      bool keep = false;
+      if (x >= 0 && x < V) {
+        const float qx = q[(static_cast<long long>(b) * gamma + i) * V + x];
+        // log r <= log p - log q; q(x) = 0 makes the ratio infinite (kept)
+        keep = qx > 0.f ? logf(r[b * gamma + i]) <= logp - logf(qx) : logp > NEG_INF;
+      } else {
+        raise_status(status, RV_DEV_DRAFT_RANGE);
+      }
+      a.accept_mask[b * gamma + i] = keep ? 1 : 0;
+      if (!keep && n == gamma) n = i;
+    }
+    s_n = n;
+    s_t = -1;
+    s_last = -1;
+  }
+  __syncthreads();
+  const int n = s_n;
+  const long long prow = static_cast<long long>(b) * (gamma + 1) + n;
+  const float lse = scores[prow * RV_NSCORES + RV_SCORE_LSE_FUSED];
+  const float* zrow = z + prow * V;
+  const float* qrow = n < gamma ? q + (static_cast<long long>(b) * gamma + n) * V : nullptr;
+  const int chunk = (V + SPEC_THREADS - 1) / SPEC_THREADS;
+  const int c0 = min(V, tid * chunk), c1 = min(V, c0 + chunk);
+  for (int pass = 0; pass < 2; ++pass) {  // pass 1 only when every residual weight is zero
+    float part = 0.f;
+    for (int v = c0; v < c1; ++v) part += spec_weight(zrow, qrow, lse, v);
+    float incl = part;  // inclusive scan within the warp
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    if (lane == 31) s_wtot[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {  // exclusive scan of the warp totals
+      const float w = s_wtot[lane];
+      float wi = w;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const float y = __shfl_up_sync(0xffffffffu, wi, o);
+        if (lane >= o) wi += y;
+      }
+      s_woff[lane] = wi - w;
+      if (lane == 31) s_total = wi;
+    }
+    __syncthreads();
+    const float W = s_total;
+    if (!(W > 0.f)) {  // p_{n+1} <= q_{n+1} everywhere (only through rounding): draw from p_{n+1}
+      qrow = nullptr;
+      __syncthreads();
+      continue;
+    }
+    const float target = u[b] * W;
+    const float lo = s_woff[warp] + (incl - part);
+    if (part > 0.f) atomicMax(&s_last, tid);
+    if (part > 0.f && target >= lo && target < lo + part) {
+      float c = lo;
+      int t = -1;
+      for (int v = c0; v < c1; ++v) {
+        const float w = spec_weight(zrow, qrow, lse, v);
+        c += w;
+        if (w > 0.f) t = v;
+        if (w > 0.f && c > target) break;
+      }
+      atomicMax(&s_t, t);
+    }
+    __syncthreads();
+    // u * W at or past the rounded sum of the ranges: the last token with weight
+    if (s_t < 0 && tid == s_last) {
+      int t = -1;
+      for (int v = c0; v < c1; ++v)
+        if (spec_weight(zrow, qrow, lse, v) > 0.f) t = v;
+      s_t = t;
+    }
+    break;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    a.accepted_len[b] = n;
+    a.next_token[b] = s_t >= 0 ? s_t : 0;
+    a.ctx_out[b] = a.ctx_in[b] + n;
+  }
+}
+
+cudaError_t launch_accept_speculative(const int32_t* drafts, const float* q, const float* r,
+                                      const float* u, const float* scores, const float* z, int B,
+                                      int gamma, int V, uint8_t* accept_mask,
+                                      int32_t* accepted_len, int32_t* next_token,
+                                      const int32_t* ctx_in, int32_t* ctx_out, unsigned* status,
+                                      cudaStream_t s) {
+  AcceptArgs a{accept_mask, accepted_len, next_token, ctx_in, ctx_out, 0, 0.f, 0.f};
+  accept_speculative_kernel<<<B, SPEC_THREADS, 0, s>>>(drafts, q, r, u, scores, z, gamma, V, a,
+                                                       status);
+  return cudaGetLastError();
+}
+
 // ---------------------------------------------------------------- typical accept (Alg. 3)
 __global__ void accept_typical_kernel(const int32_t* __restrict__ drafts,
                                       const float* __restrict__ scores,

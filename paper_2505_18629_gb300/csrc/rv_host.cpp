@@ -93,6 +93,9 @@ struct rv_handle {
   // acceptance rule of rv_verify_step (rv_set_acceptance)
   int accept_mode = RV_ACCEPT_EXACT;
   float accept_log_eps = 0.f, accept_log_delta = 0.f;
+  // fused logits z [max_batch * (max_gamma + 1)][vocab] written by the head in
+  // speculative-sampling mode (allocated on the first rv_set_acceptance to it)
+  float* zbuf = nullptr;
   // tensor maps of the last tcgen05 attention call and what they were made for
   AttnTcMaps attn_maps;
   const void* attn_map_ptrs[5] = {nullptr, nullptr, nullptr, nullptr, nullptr};
@@ -326,6 +329,7 @@ extern "C" RV_API int rv_destroy(rv_handle* h) {
   cudaEventDestroy(h->ev_join);
   cudaEventDestroy(h->ev_fork);
   cudaStreamDestroy(h->side);
+  if (h->zbuf) cudaFree(h->zbuf);
   cudaFree(h->ws.base);
   delete h;
   return RV_OK;
@@ -504,7 +508,8 @@ int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_
   HeadArgs a{hidden, w_head, draft_ids, B, gamma, R, c.vocab, c.hidden, alpha,
              h->ws.head_partials, h->ws.gathered, h->ws.status,
              bf16 ? h->ws.status + 16 : nullptr,    // tile counter: its own 64-byte line
-             bf16 ? h->ws.status + 32 : nullptr};   // finished-CTA counter
+             bf16 ? h->ws.status + 32 : nullptr,    // finished-CTA counter
+             h->accept_mode == RV_ACCEPT_SPECULATIVE ? h->zbuf : nullptr};
   HeadPlan pl = head_plan(B, gamma, c.vocab, h->num_sms, bf16);
   if (bf16 && pl.N >= HEAD_PAIR_MIN_N) {
     // CTA pairs: as many as fit at once (two CTAs of a pair share a GPC)
@@ -621,6 +626,20 @@ extern "C" RV_API int rv_set_acceptance(rv_handle* h, int32_t mode, float eps, f
     h->accept_mode = mode;
     return RV_OK;
   }
+  if (mode == RV_ACCEPT_SPECULATIVE) {
+    if (!h->zbuf) {
+      const rv_config& c = h->cfg;
+      const size_t bytes = static_cast<size_t>(c.max_batch) * (c.max_gamma + 1) * c.vocab * 4;
+      cudaError_t e = cudaMalloc(&h->zbuf, bytes);
+      if (e != cudaSuccess) {
+        h->zbuf = nullptr;
+        return fail(h, RV_ERR_CUDA, "fused-logit buffer cudaMalloc(%zu): %s", bytes,
+                    cudaGetErrorString(e));
+      }
+    }
+    h->accept_mode = mode;
+    return RV_OK;
+  }
   if (mode != RV_ACCEPT_TYPICAL) return fail(h, RV_ERR_INVALID_ARG, "unknown acceptance mode %d", mode);
   if (!(eps > 0.f) || !(delta > 0.f) || !std::isfinite(eps) || !std::isfinite(delta))
     return fail(h, RV_ERR_INVALID_ARG, "typical acceptance needs finite eps > 0 and delta > 0");
@@ -632,15 +651,23 @@ extern "C" RV_API int rv_set_acceptance(rv_handle* h, int32_t mode, float eps, f
 
 // ============================================================================ whole step
 
-extern "C" RV_API int rv_verify_step(
-    rv_handle* h, const void* q, const void* k_blk, const void* v_blk, void* k_cache, void* v_cache,
-    const void* hidden, const void* w_head, const int32_t* draft_ids, const int32_t* prompt_ids,
-    const int32_t* prefix_ids, const int32_t* ctx_in, int32_t B, int32_t gamma, int32_t n_prompt,
-    int32_t n_prefix, float alpha, int32_t* block_ids, int32_t* pos_ids, void* attn_out,
-    float* scores, int32_t* argmax, float* margin, uint8_t* accept_mask, int32_t* accepted_len,
-    int32_t* next_token, int32_t* ctx_out, void* stream) {
-  if (!h) return RV_ERR_INVALID_ARG;
-  h->err.clear();
+namespace {
+
+// The whole step; `spec` != nullptr runs the speculative-sampling acceptance
+// (Alg. 1) after the head instead of the rule fused into the head's merge.
+struct SpecInputs {
+  const float* q;
+  const float* r;
+  const float* u;
+};
+
+int step_impl(rv_handle* h, const void* q, const void* k_blk, const void* v_blk, void* k_cache,
+              void* v_cache, const void* hidden, const void* w_head, const int32_t* draft_ids,
+              const int32_t* prompt_ids, const int32_t* prefix_ids, const int32_t* ctx_in,
+              int32_t B, int32_t gamma, int32_t n_prompt, int32_t n_prefix, float alpha,
+              int32_t* block_ids, int32_t* pos_ids, void* attn_out, float* scores,
+              int32_t* argmax, float* margin, uint8_t* accept_mask, int32_t* accepted_len,
+              int32_t* next_token, int32_t* ctx_out, const SpecInputs* spec, void* stream) {
   if (n_prompt < 0 || n_prefix < 0) return fail(h, RV_ERR_SHAPE, "negative template part");
   const int R = n_prompt + n_prefix;
   int rc = check_head_args(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin);
@@ -675,7 +702,15 @@ extern "C" RV_API int rv_verify_step(
     AcceptArgs ac{accept_mask, accepted_len,       next_token,         ctx_in,
                   ctx_out,     h->accept_mode,     h->accept_log_eps,  h->accept_log_delta};
     rc = head_impl(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin,
-                   do_pack ? &pk : nullptr, &ac, s);
+                   do_pack ? &pk : nullptr, spec ? nullptr : &ac, s);
+    if (rc == RV_OK && spec) {
+      ProfScope prof(h, RV_PROF_ACCEPT, s);
+      e = launch_accept_speculative(draft_ids, spec->q, spec->r, spec->u, scores, h->zbuf, B,
+                                    gamma, c.vocab, accept_mask, accepted_len, next_token, ctx_in,
+                                    ctx_out, h->ws.status, s);
+      h->launches += 1;
+      if (e != cudaSuccess) rc = cuda_fail(h, e, "speculative accept launch");
+    }
   }
   if (fork) {
     e = cudaEventRecord(h->ev_join, h->side);
@@ -683,6 +718,77 @@ extern "C" RV_API int rv_verify_step(
     if (e != cudaSuccess && rc == RV_OK) return cuda_fail(h, e, "stream join");
   }
   return rc;
+}
+
+}  // namespace
+
+extern "C" RV_API int rv_verify_step(
+    rv_handle* h, const void* q, const void* k_blk, const void* v_blk, void* k_cache, void* v_cache,
+    const void* hidden, const void* w_head, const int32_t* draft_ids, const int32_t* prompt_ids,
+    const int32_t* prefix_ids, const int32_t* ctx_in, int32_t B, int32_t gamma, int32_t n_prompt,
+    int32_t n_prefix, float alpha, int32_t* block_ids, int32_t* pos_ids, void* attn_out,
+    float* scores, int32_t* argmax, float* margin, uint8_t* accept_mask, int32_t* accepted_len,
+    int32_t* next_token, int32_t* ctx_out, void* stream) {
+  if (!h) return RV_ERR_INVALID_ARG;
+  h->err.clear();
+  if (h->accept_mode == RV_ACCEPT_SPECULATIVE)
+    return fail(h, RV_ERR_INVALID_ARG,
+                "speculative sampling needs the draft distributions: use rv_verify_step_speculative");
+  return step_impl(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, prompt_ids,
+                   prefix_ids, ctx_in, B, gamma, n_prompt, n_prefix, alpha, block_ids, pos_ids,
+                   attn_out, scores, argmax, margin, accept_mask, accepted_len, next_token, ctx_out,
+                   nullptr, stream);
+}
+
+extern "C" RV_API int rv_verify_step_speculative(
+    rv_handle* h, const void* q, const void* k_blk, const void* v_blk, void* k_cache, void* v_cache,
+    const void* hidden, const void* w_head, const int32_t* draft_ids, const int32_t* prompt_ids,
+    const int32_t* prefix_ids, const int32_t* ctx_in, int32_t B, int32_t gamma, int32_t n_prompt,
+    int32_t n_prefix, float alpha, const float* q_draft, const float* r_uniform,
+    const float* u_uniform, int32_t* block_ids, int32_t* pos_ids, void* attn_out, float* scores,
+    int32_t* argmax, float* margin, uint8_t* accept_mask, int32_t* accepted_len,
+    int32_t* next_token, int32_t* ctx_out, void* stream) {
+  if (!h) return RV_ERR_INVALID_ARG;
+  h->err.clear();
+  if (h->accept_mode != RV_ACCEPT_SPECULATIVE || !h->zbuf)
+    return fail(h, RV_ERR_INVALID_ARG,
+                "call rv_set_acceptance(RV_ACCEPT_SPECULATIVE) on the handle first");
+  if (B > 0 && (!q_draft || !r_uniform || !u_uniform))
+    return fail(h, RV_ERR_INVALID_ARG, "NULL draft distribution or uniforms");
+  const SpecInputs spec{q_draft, r_uniform, u_uniform};
+  return step_impl(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, prompt_ids,
+                   prefix_ids, ctx_in, B, gamma, n_prompt, n_prefix, alpha, block_ids, pos_ids,
+                   attn_out, scores, argmax, margin, accept_mask, accepted_len, next_token, ctx_out,
+                   &spec, stream);
+}
+
+extern "C" RV_API int rv_accept_speculative(rv_handle* h, const int32_t* draft_ids,
+                                            const float* q_draft, const float* r_uniform,
+                                            const float* u_uniform, const float* scores,
+                                            int32_t B, int32_t gamma, uint8_t* accept_mask,
+                                            int32_t* accepted_len, int32_t* next_token,
+                                            const int32_t* ctx_in, int32_t* ctx_out,
+                                            void* stream) {
+  if (!h) return RV_ERR_INVALID_ARG;
+  h->err.clear();
+  if (h->accept_mode != RV_ACCEPT_SPECULATIVE || !h->zbuf)
+    return fail(h, RV_ERR_INVALID_ARG,
+                "call rv_set_acceptance(RV_ACCEPT_SPECULATIVE) before rv_verify_head");
+  if (B < 0 || gamma < 1) return fail(h, RV_ERR_SHAPE, "need B >= 0 and gamma >= 1");
+  if (B > h->cfg.max_batch || gamma > h->cfg.max_gamma)
+    return fail(h, RV_ERR_CAPACITY, "B / gamma above the handle's maxima");
+  if (B == 0) return RV_OK;
+  if (!draft_ids || !q_draft || !r_uniform || !u_uniform || !scores || !accept_mask ||
+      !accepted_len || !next_token || !ctx_in || !ctx_out)
+    return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  ProfScope prof(h, RV_PROF_ACCEPT, s);
+  cudaError_t e = launch_accept_speculative(draft_ids, q_draft, r_uniform, u_uniform, scores,
+                                            h->zbuf, B, gamma, h->cfg.vocab, accept_mask,
+                                            accepted_len, next_token, ctx_in, ctx_out,
+                                            h->ws.status, s);
+  h->launches += 1;
+  return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "speculative accept launch");
 }
 
 extern "C" RV_API int rv_verify_step_host(

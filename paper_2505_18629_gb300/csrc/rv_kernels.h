@@ -82,6 +82,7 @@ struct HeadArgs {
   unsigned* status;
   unsigned* tile_counter;  // LM-head tile counter, zeroed by the prep kernel
   unsigned* done_counter;  // finished LM-head CTAs (fused merge), zeroed by the prep kernel
+  float* zout = nullptr;   // [P][V] fused logits z_i (speculative sampling), or none
 };
 
 // ---- small kernels (k_small.cu)
@@ -110,6 +111,15 @@ cudaError_t launch_head_finalize(const HeadArgs& a, const HeadPlan& p, float* sc
 cudaError_t launch_accept(const int32_t* drafts, const int32_t* argmax, int B, int gamma,
                           uint8_t* accept_mask, int32_t* accepted_len, int32_t* next_token,
                           const int32_t* ctx_in, int32_t* ctx_out, cudaStream_t s);
+// Speculative-sampling acceptance (Alg. 1) from the head's scores and the
+// fused logits it wrote (z [P][V]), the draft distributions q [B][gamma][V],
+// uniforms r [B][gamma] and u [B].  One CTA per sequence.
+cudaError_t launch_accept_speculative(const int32_t* drafts, const float* q, const float* r,
+                                      const float* u, const float* scores, const float* z, int B,
+                                      int gamma, int V, uint8_t* accept_mask,
+                                      int32_t* accepted_len, int32_t* next_token,
+                                      const int32_t* ctx_in, int32_t* ctx_out, unsigned* status,
+                                      cudaStream_t s);
 // Typical acceptance (Alg. 3) from the head's scores and argmax.
 cudaError_t launch_accept_typical(const int32_t* drafts, const float* scores,
                                   const int32_t* argmax, int B, int gamma, float log_eps,

@@ -90,6 +90,8 @@ def test_entry_points_reject_null_handle(rv):
     assert L.rv_accept_typical(None, None, None, None, 1, 1, 0.09, 0.3, None, None, None, None,
                                None, None) == -1
     assert L.rv_set_acceptance(None, 1, 0.09, 0.3) == -1
+    assert L.rv_accept_speculative(None, None, None, None, None, None, 1, 1, None, None, None,
+                                   None, None, None) == -1
     assert L.rv_destroy(None) == 0
 
 

@@ -397,6 +397,131 @@ def test_typical_acceptance_fp32_and_pairs(gu):
         h.close()
 
 
+# ------------------------------------------------------------------ speculative sampling (Alg. 1)
+
+SPEC_TOL = 2e-3  # decisions / CDF positions this close to a boundary may differ (fp32 vs fp64)
+
+
+def _spec_inputs(inp, alpha, seed, same=False):
+    """Draft distributions q_i (float32) near the oracle's fused p_i, drafts
+    x_i ~ q_i, uniforms r and u; plus the oracle's fused logits z."""
+    import oracle.rv_oracle as orc
+    wl = inp.wl
+    rng = np.random.default_rng(seed)
+    dummy = np.zeros((wl.B, wl.gamma), np.int64)
+    z = orc.verify_head(inp.W, inp.hidden, dummy, wl.gamma, wl.R, alpha)["z"]
+    logit_q = z[:, :wl.gamma] + (0.0 if same else rng.normal(0, 1.0, z[:, :wl.gamma].shape))
+    q = np.exp(logit_q - logit_q.max(-1, keepdims=True))
+    q = (q / q.sum(-1, keepdims=True)).astype(np.float32)
+    q64 = q.astype(np.float64) / q.astype(np.float64).sum(-1, keepdims=True)
+    drafts = np.array([[rng.choice(wl.V, p=q64[b, i]) for i in range(wl.gamma)]
+                       for b in range(wl.B)], np.int64)
+    r = rng.uniform(0, 1, (wl.B, wl.gamma)).astype(np.float32)
+    u = rng.uniform(0, 1, wl.B).astype(np.float32)
+    return z, q, drafts, r, u
+
+
+def _run_spec(gu, inp, drafts, alpha, q, r, u, separate=False):
+    import torch
+    from paper_2505_18629_gb300 import rv
+    wl = inp.wl
+    B, g = wl.B, wl.gamma
+    h = gu.make_handle(wl)
+    rv.rv_set_acceptance(h, rv.RV_ACCEPT_SPECULATIVE)
+    dq, dr, du = gu.to_dev(q), gu.to_dev(r), gu.to_dev(u)
+    d = gu.to_dev(drafts.astype(np.int32))
+    ctx = gu.to_dev(inp.ctx_lens.astype(np.int32))
+    sc = torch.empty((B, g + 1, rv.RV_NSCORES), device="cuda")
+    am = torch.empty((B, g + 1), dtype=torch.int32, device="cuda")
+    mg = torch.empty((B, g), device="cuda")
+    acc = torch.full((B, g), 7, dtype=torch.uint8, device="cuda")
+    n = torch.full((B,), -7, dtype=torch.int32, device="cuda")
+    t = torch.full((B,), -7, dtype=torch.int32, device="cuda")
+    co = torch.full((B,), -7, dtype=torch.int32, device="cuda")
+    if separate:
+        rv.rv_verify_head(h, gu.to_dev(inp.hidden), gu.to_dev(inp.W), d, g, wl.R, alpha, sc, am, mg)
+        rv.rv_accept_speculative(h, d, dq, dr, du, sc, acc, n, t, ctx, co)
+    else:
+        q_, kb, vb = gu.to_dev(inp.q), gu.to_dev(inp.k_blk), gu.to_dev(inp.v_blk)
+        kc, vc = gu.to_dev(inp.k_cache), gu.to_dev(inp.v_cache)
+        prompt = gu.to_dev(inp.prompt_ids.astype(np.int32)) if inp.prompt_ids.size else None
+        prefix = gu.to_dev(inp.prefix_ids.astype(np.int32))
+        attn = torch.zeros_like(q_)
+        with pytest.raises(rv.RVError):  # plain step refuses the sampling rule (no q)
+            rv.rv_verify_step(h, q_, kb, vb, kc, vc, gu.to_dev(inp.hidden), gu.to_dev(inp.W), d,
+                              prompt, prefix, ctx, alpha, None, None, attn, sc, am, mg, acc, n, t, co)
+        rv.rv_verify_step_speculative(h, q_, kb, vb, kc, vc, gu.to_dev(inp.hidden),
+                                      gu.to_dev(inp.W), d, prompt, prefix, ctx, alpha, dq, dr, du,
+                                      None, None, attn, sc, am, mg, acc, n, t, co)
+    status = rv.rv_read_status(h)
+    h.close()
+    return gu.to_np(acc), gu.to_np(n), gu.to_np(t), gu.to_np(co), gu.to_np(sc), status
+
+
+def _check_spec(inp, z, q, drafts, r, u, gpu):
+    import oracle.rv_oracle as orc
+    wl = inp.wl
+    g = wl.gamma
+    acc_g, n_g, t_g, co_g, sc_g, status = gpu
+    assert status == 0
+    q64 = q.astype(np.float64) / q.astype(np.float64).sum(-1, keepdims=True)
+    acc, n, t, log_ratio, _ = orc.speculative_accept(drafts, z, q64, r.astype(np.float64),
+                                                     u.astype(np.float64))
+    close = np.abs(np.log(r.astype(np.float64)) - log_ratio) < SPEC_TOL
+    assert not ((acc_g.astype(bool) != acc) & ~close).any(), "accept decision differs at a clear case"
+    logp = z - orc.logsumexp(z)[..., None]
+    p = np.exp(logp)
+    n_match = 0
+    for b in range(wl.B):
+        nb = int(n_g[b])
+        assert acc_g[b, :nb].all() and (nb == g or acc_g[b, nb] == 0)
+        assert co_g[b] == inp.ctx_lens[b] + nb
+        if nb != n[b]:
+            assert close[b, :min(n[b], nb) + 1].any(), f"sequence {b}: n {nb} vs {n[b]}"
+            continue
+        n_match += 1
+        w = np.maximum(0.0, p[b, nb] - q64[b, nb]) if nb < g else p[b, nb]
+        c = np.cumsum(w) / w.sum()
+        tb = int(t_g[b])
+        lo = c[tb - 1] if tb > 0 else 0.0
+        assert lo - SPEC_TOL <= u[b] <= c[tb] + SPEC_TOL, \
+            f"sequence {b}: t {tb} at CDF [{lo:.5f}, {c[tb]:.5f}] for u {u[b]:.5f}"
+    assert n_match >= wl.B // 2
+    return acc, n
+
+
+@pytest.mark.parametrize("separate", [False, True])
+def test_speculative_sampling_small(gu, separate):
+    from paper_2505_18629_gb300 import synth
+    wl = _wl(B=8, gamma=5, V=1000, seed=80)
+    inp = synth.generate(wl)
+    z, q, drafts, r, u = _spec_inputs(inp, ALPHA, 81)
+    acc, n = _check_spec(inp, z, q, drafts, r, u,
+                         _run_spec(gu, inp, drafts, ALPHA, q, r, u, separate=separate))
+    assert 0 < acc.sum() < acc.size
+
+
+def test_speculative_sampling_draft_equals_target(gu):
+    # q = p (up to float32): every draft is kept and t ~ p_{gamma+1}
+    from paper_2505_18629_gb300 import synth
+    wl = _wl(B=6, gamma=4, V=1000, seed=82)
+    inp = synth.generate(wl)
+    z, q, drafts, r, u = _spec_inputs(inp, ALPHA, 83, same=True)
+    r = np.minimum(r, 0.99).astype(np.float32)
+    acc, n = _check_spec(inp, z, q, drafts, r, u, _run_spec(gu, inp, drafts, ALPHA, q, r, u))
+    assert acc.all()
+
+
+def test_speculative_sampling_pairs_and_8b(gu):
+    # the CTA-pair head (N >= 96) and the full 8B batch-1 vocabulary
+    from paper_2505_18629_gb300 import synth
+    for wl, seqs_ok in ((_wl(B=14, gamma=8, R=8, V=777, H=256, ctx=(10, 60), seed=84), None),
+                        (synth.WORKLOADS["llama3-8b-b1"], None)):
+        inp = synth.generate(wl)
+        z, q, drafts, r, u = _spec_inputs(inp, ALPHA, 85)
+        _check_spec(inp, z, q, drafts, r, u, _run_spec(gu, inp, drafts, ALPHA, q, r, u))
+
+
 # ------------------------------------------------------------------ full-size workloads
 
 def test_llama3_8b_b1_full(gu):

@@ -20,6 +20,8 @@ Notation follows the paper:
   * p_i = softmax((1-alpha) o_i + alpha o_{m+i-1})   (Eq. 2, Alg. 1)
   * exact-match verification with the greedy choice x^_i = argmax p_i
     (Alg. 2, read as "stop at the first mismatch"; see ``exact_match_accept``)
+    or with sampled x^_i ~ softmax(z_i / T) (``sampled_exact_accept``)
+  * typical acceptance (Alg. 3) and speculative sampling (Alg. 1)
 
 Hidden-state rows: row 0 is the target's last hidden state after the prefix
 (gives o_1, "M_p(prefix)" in Alg. 1); row r (1..Lb) follows block token r-1.
@@ -343,6 +345,40 @@ def speculative_accept(drafts, z, q, r, u):
         c = np.cumsum(w) / w.sum()
         cdf_gap[b] = np.min(np.abs(c - u[b]))
     return acc, n, t, log_ratio, cdf_gap
+
+
+def sampled_exact_accept(drafts, z, temperature: float, u):
+    """Exact-match verification with sampled target tokens (Alg. 2).
+
+    drafts [B, gamma]; z [B, gamma+1, V] fused logits (Eq. 2); u [B, gamma+1]
+    one uniform per position.  At sampling temperature T the target's token at
+    position i is x^_i ~ softmax(z_i / T) (T = 1 gives p_i itself), drawn by
+    inverse CDF with u[b, i].  Drafts are kept up to the first mismatch
+    x_i != x^_i (the stopping set read as in ``exact_match_accept``), and the
+    next token t ~ p_{n+1} is the draw x^_{n+1} already taken at that position:
+    the emitted tokens [x_1..x_n, t] are then x^_1..x^_{n+1}, i.e. exactly what
+    sampling the target alone would give, which makes the rule lossless
+    (Sec. 4.1).  T -> 0 reduces to the greedy rule of ``exact_match_accept``.
+
+    Returns (accept_mask [B, gamma] uint8, n [B], t [B], xhat [B, gamma+1],
+    cdf_gap [B, gamma+1]) where cdf_gap is the distance of u from the nearest
+    cumulative-weight boundary of softmax(z_i / T), which bounds how close
+    each draw was to a tie.
+    """
+    z = np.asarray(z, np.float64)
+    u = np.asarray(u, np.float64)
+    B, G1, V = z.shape
+    zt = z / float(temperature)
+    p_t = np.exp(zt - logsumexp(zt)[..., None])
+    xhat = np.zeros((B, G1), np.int64)
+    cdf_gap = np.zeros((B, G1))
+    for b in range(B):
+        for i in range(G1):
+            xhat[b, i] = inverse_cdf_sample(p_t[b, i], float(u[b, i]))
+            c = np.cumsum(p_t[b, i]) / p_t[b, i].sum()
+            cdf_gap[b, i] = np.min(np.abs(c - u[b, i]))
+    acc, n, t = exact_match_accept(drafts, xhat)
+    return acc, n, t, xhat, cdf_gap
 
 
 def verify_step(inp_W, hidden, q, k_blk, v_blk, k_cache, v_cache, ctx_lens,

@@ -589,3 +589,79 @@ def test_pins_catch_plain_p_instead_of_residual(monkeypatch):
         return acc, n, t, lr, gap
     monkeypatch.setattr(orc, "speculative_accept", plain)
     assert _fails(test_speculative_first_token_is_distributed_as_p1)
+
+
+# ------------------------------------------------------------------ Alg. 2: sampled exact match
+
+def test_sampled_exact_low_temperature_is_greedy():
+    # T -> 0: softmax(z / T) concentrates on argmax z, so every draw is the
+    # greedy choice whatever u is, and the rule is the greedy exact match.
+    rng = np.random.default_rng(31)
+    B, gamma, V = 16, 5, 13
+    z = rng.normal(0, 2.0, (B, gamma + 1, V))
+    greedy = orc.greedy_choice(z)
+    drafts = np.where(rng.uniform(size=(B, gamma)) < 0.7, greedy[:, :gamma],
+                      rng.integers(0, V, (B, gamma)))
+    u = rng.uniform(0, 1, (B, gamma + 1))
+    acc, n, t, xhat, _ = orc.sampled_exact_accept(drafts, z, 1e-4, u)
+    np.testing.assert_array_equal(xhat, greedy)
+    acc_g, n_g, t_g = orc.exact_match_accept(drafts, greedy)
+    np.testing.assert_array_equal(acc, acc_g)
+    np.testing.assert_array_equal(n, n_g)
+    np.testing.assert_array_equal(t, t_g)
+
+
+@pytest.mark.parametrize("T", [0.2, 0.8, 1.0, 3.0])
+def test_sampled_exact_temperature_closed_form(T):
+    # Two tokens with logits (0, d): P(x^ = 1) = 1 / (1 + exp(-d / T)).  A
+    # midpoint grid of u gives the draw frequencies to within 1 / grid.
+    d = 0.9
+    z = np.array([[[0.0, d]]])
+    grid = (np.arange(4000) + 0.5) / 4000
+    ones = np.mean([orc.sampled_exact_accept(np.zeros((1, 0), np.int64), z, T,
+                                             np.array([[x]]))[3][0, 0] for x in grid])
+    assert abs(ones - 1.0 / (1.0 + np.exp(-d / T))) < 1e-3
+
+
+def test_sampled_exact_emits_the_target_draws():
+    # Lossless: the emitted tokens [x_1..x_n, t] are the target's own draws
+    # x^_1..x^_{n+1}, so the output is what sampling the target alone gives.
+    rng = np.random.default_rng(32)
+    B, gamma, V = 64, 6, 7
+    z = rng.normal(0, 1.0, (B, gamma + 1, V))
+    T = 0.8
+    u = rng.uniform(0, 1, (B, gamma + 1))
+    p_t = scipy.special.softmax(z / T, axis=-1)
+    # drafts that often agree with the draws: x_i ~ p_t (an ideal draft model)
+    drafts = np.array([[rng.choice(V, p=p_t[b, i]) for i in range(gamma)] for b in range(B)])
+    acc, n, t, xhat, _ = orc.sampled_exact_accept(drafts, z, T, u)
+    assert (n > 0).any() and (n < gamma).any()
+    for b in range(B):
+        emitted = list(drafts[b, :n[b]]) + [t[b]]
+        assert emitted == list(xhat[b, :n[b] + 1])
+        assert n[b] == gamma or drafts[b, n[b]] != xhat[b, n[b]]
+        for i in range(gamma + 1):
+            assert xhat[b, i] == orc.inverse_cdf_sample(p_t[b, i], u[b, i])
+
+
+def test_pins_catch_sampled_exact_fresh_draw_for_t(monkeypatch):
+    real = orc.sampled_exact_accept
+
+    def fresh(drafts, z, temperature, u):
+        # planted slip: t drawn afresh from p_{n+1} instead of reusing x^_{n+1}
+        acc, n, t, xhat, gap = real(drafts, z, temperature, u)
+        zt = np.asarray(z, np.float64) / temperature
+        p_t = np.exp(zt - orc.logsumexp(zt)[..., None])
+        t = np.array([orc.inverse_cdf_sample(p_t[b, n[b]], 1.0 - float(u[b, n[b]]))
+                      for b in range(len(n))])
+        return acc, n, t, xhat, gap
+    monkeypatch.setattr(orc, "sampled_exact_accept", fresh)
+    assert _fails(test_sampled_exact_emits_the_target_draws)
+
+
+def test_pins_catch_temperature_multiplied(monkeypatch):
+    real = orc.sampled_exact_accept
+    # planted slip: softmax(z * T) instead of softmax(z / T)
+    monkeypatch.setattr(orc, "sampled_exact_accept",
+                        lambda drafts, z, T, u: real(drafts, np.asarray(z) * T * T, T, u))
+    assert _fails(lambda: test_sampled_exact_temperature_closed_form(0.2))

@@ -81,6 +81,7 @@ extern "C" {
 #define RV_ACCEPT_EXACT 0       /* exact match with the greedy choice (Alg. 2)               */
 #define RV_ACCEPT_TYPICAL 1     /* entropy-based threshold of typical acceptance (Alg. 3)     */
 #define RV_ACCEPT_SPECULATIVE 2 /* speculative sampling with residual resampling (Alg. 1)     */
+#define RV_ACCEPT_SAMPLED 3     /* exact match with target tokens sampled at temperature T (Alg. 2) */
 
 /* Model / capacity description fixed at creation. */
 typedef struct rv_config {
@@ -200,12 +201,13 @@ RV_API int rv_accept_typical(rv_handle* h, const int32_t* draft_ids, const float
  *   RV_ACCEPT_EXACT (the default; eps and delta ignored) and RV_ACCEPT_TYPICAL
  *     (eps > 0, delta > 0; see rv_accept_typical) apply to rv_verify_step and
  *     rv_verify_step_host;
- *   RV_ACCEPT_SPECULATIVE makes every LM-head call (rv_verify_head, the step)
- *     also write its fused logits z_i to a buffer of the handle (allocated
- *     here once: max_batch * (max_gamma+1) * vocab floats), which
- *     rv_accept_speculative and rv_verify_step_speculative read; in this mode
- *     plain rv_verify_step returns RV_ERR_INVALID_ARG (it has no draft
- *     distributions).
+ *   RV_ACCEPT_SPECULATIVE and RV_ACCEPT_SAMPLED make every LM-head call
+ *     (rv_verify_head, the step) also write its fused logits z_i to a buffer
+ *     of the handle (allocated here once: max_batch * (max_gamma+1) * vocab
+ *     floats), which rv_accept_speculative / rv_verify_step_speculative and
+ *     rv_accept_sampled / rv_verify_step_sampled read; in these modes plain
+ *     rv_verify_step returns RV_ERR_INVALID_ARG (it has no draft
+ *     distributions or uniforms).
  * Errors: RV_ERR_INVALID_ARG for an unknown mode or bad eps / delta,
  * RV_ERR_CUDA if the buffer cannot be allocated. */
 RV_API int rv_set_acceptance(rv_handle* h, int32_t mode, float eps, float delta);
@@ -230,6 +232,28 @@ RV_API int rv_accept_speculative(rv_handle* h, const int32_t* draft_ids, const f
                                  const float* scores, int32_t B, int32_t gamma,
                                  uint8_t* accept_mask, int32_t* accepted_len, int32_t* next_token,
                                  const int32_t* ctx_in, int32_t* ctx_out, void* stream);
+
+/* Exact-match verification with target tokens sampled at temperature T
+ * (Alg. 2), after an rv_verify_head call on this handle in RV_ACCEPT_SAMPLED
+ * mode (same stream, same B and gamma).  The target's token at position
+ * i = 1..gamma+1 is x^_i ~ softmax(z_i / T), with z_i the fused logits of
+ * Eq. 2, drawn by inverse CDF with u = u_uniform[b][i-1]: the smallest v
+ * whose cumulative weight exp((z_i[v] - max z_i) / T) exceeds u times the sum
+ * of the weights.  Then, as in rv_accept:
+ *   sampled[b][i-1]     = x^_i                                  int32 [B, gamma+1]
+ *   accept_mask[b][i-1] = (x_i == x^_i)                          uint8 [B, gamma]
+ *   accepted_len[b] = n = min({i-1 : x_i != x^_i} U {gamma})     int32 [B]
+ *   next_token[b]   = t = x^_{n+1}, the draw already taken at n+1
+ *   ctx_out[b]      = ctx_in[b] + n (may alias ctx_in)
+ * The emitted tokens [x_1..x_n, t] are x^_1..x^_{n+1}: what sampling the
+ * target alone gives with the same uniforms.  u_uniform [B, gamma+1] float32
+ * in [0, 1) (device).  temperature must be finite and > 0, else
+ * RV_ERR_INVALID_ARG.  Two launches: the draws (one CTA per position), then
+ * the acceptance. */
+RV_API int rv_accept_sampled(rv_handle* h, const int32_t* draft_ids, const float* u_uniform,
+                             float temperature, int32_t B, int32_t gamma, int32_t* sampled,
+                             uint8_t* accept_mask, int32_t* accepted_len, int32_t* next_token,
+                             const int32_t* ctx_in, int32_t* ctx_out, void* stream);
 
 /* The whole verify step on device buffers, in one call and four kernel
  * launches: the attention (rv_verify_attention) on an internal stream forked
@@ -263,6 +287,19 @@ RV_API int rv_verify_step_speculative(
     int32_t gamma, int32_t n_prompt, int32_t n_prefix, float alpha, const float* q_draft,
     const float* r_uniform, const float* u_uniform, int32_t* block_ids, int32_t* pos_ids,
     void* attn_out, float* scores, int32_t* argmax, float* margin, uint8_t* accept_mask,
+    int32_t* accepted_len, int32_t* next_token, int32_t* ctx_out, void* stream);
+
+/* rv_verify_step with exact-match verification against target tokens
+ * sampled at temperature T (rv_accept_sampled) in place of the greedy rule;
+ * needs the handle in RV_ACCEPT_SAMPLED mode.  temperature, u_uniform and
+ * sampled as in rv_accept_sampled; two launches more than rv_verify_step. */
+RV_API int rv_verify_step_sampled(
+    rv_handle* h, const void* q, const void* k_blk, const void* v_blk, void* k_cache,
+    void* v_cache, const void* hidden, const void* w_head, const int32_t* draft_ids,
+    const int32_t* prompt_ids, const int32_t* prefix_ids, const int32_t* ctx_in, int32_t B,
+    int32_t gamma, int32_t n_prompt, int32_t n_prefix, float alpha, float temperature,
+    const float* u_uniform, int32_t* block_ids, int32_t* pos_ids, void* attn_out, float* scores,
+    int32_t* argmax, float* margin, int32_t* sampled, uint8_t* accept_mask,
     int32_t* accepted_len, int32_t* next_token, int32_t* ctx_out, void* stream);
 
 /* The whole verify step from HOST buffers (synchronous).  The per-step inputs

@@ -30,10 +30,10 @@ __device__ __forceinline__ void lse_merge3(float& m, float& s, float& t, float M
                                            float T) {
   const float mn = fmaxf(m, M);
   if (mn == NEG_INF) return;
-  const float a = (m == NEG_INF) ? 0.f : exp2f((m - mn) * LOG2E);
-  const float c = (M == NEG_INF) ? 0.f : exp2f((M - mn) * LOG2E);
+  const float a = (m == NEG_INF) ? 0.f : exp2f(__fmul_rn(m - mn, LOG2E));
+  const float c = (M == NEG_INF) ? 0.f : exp2f(__fmul_rn(M - mn, LOG2E));
   t = (a == 0.f ? 0.f : a * (t + (m - mn) * s)) + (c == 0.f ? 0.f : c * (T + (M - mn) * S));
-  s = s * a + S * c;
+  s = lse_rescale_sum(s, a, S, c);  // the update of lse_merge, bit for bit
   m = mn;
 }
 

@@ -406,6 +406,133 @@ cudaError_t launch_accept_speculative(const int32_t* drafts, const float* q, con
   return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------- sampled target tokens (Alg. 2)
+// One CTA per position (b, i), i = 1..gamma+1: the target's token at
+// temperature T, x^_i ~ softmax(z_i / T), drawn by inverse CDF with the
+// position's uniform u: the smallest v whose cumulative weight
+// w_v = exp((z_i[v] - max z_i) / T) exceeds u * sum(w).  Pass 1 streams the
+// row once for (max, sum) (each thread an online pair over a strided, coalesced
+// range); pass 2 walks the row in order, 4 consecutive tokens per thread and
+// SAMP_THREADS * 4 tokens per tile: a block-wide exclusive scan of the
+// threads' weights gives each thread its cumulative range, and the one whose
+// range holds the target walks its 4 tokens.  The ranges of one tile are
+// gapless (each boundary is written once, to shared memory, and read by both
+// neighbours), so the target falls in exactly one range or past the last.
+constexpr int SAMP_THREADS = 512;
+constexpr int SAMP_PER = 4;
+constexpr int SAMP_TILE = SAMP_THREADS * SAMP_PER;
+
+__global__ void __launch_bounds__(SAMP_THREADS)
+    sample_fused_kernel(const float* __restrict__ z, const float* __restrict__ u, int V,
+                        float inv_t, int32_t* __restrict__ xhat) {
+  constexpr int NW = SAMP_THREADS / 32;
+  __shared__ float s_m[NW], s_s[NW];
+  __shared__ float s_wtot[NW];
+  __shared__ float s_lo[SAMP_THREADS + 1];
+  __shared__ float s_max, s_target;
+  __shared__ int s_t, s_last;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const long long prow = blockIdx.x;
+  const float* row = z + prow * V;
+  // pass 1: max and sum of exp((z - max) / T)
+  float m = NEG_INF, sm = 0.f;
+  for (int v = tid; v < V; v += SAMP_THREADS) {
+    const float x = row[v] * inv_t;
+    if (x > m) {
+      sm = sm * expf(m - x) + 1.f;
+      m = x;
+    } else {
+      sm += expf(x - m);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1)
+    lse_merge(m, sm, __shfl_xor_sync(0xffffffffu, m, o), __shfl_xor_sync(0xffffffffu, sm, o));
+  if (lane == 0) {
+    s_m[warp] = m;
+    s_s[warp] = sm;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    m = lane < NW ? s_m[lane] : NEG_INF;
+    sm = lane < NW ? s_s[lane] : 0.f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+      lse_merge(m, sm, __shfl_xor_sync(0xffffffffu, m, o), __shfl_xor_sync(0xffffffffu, sm, o));
+    if (lane == 0) {
+      s_max = m;
+      s_target = u[prow] * sm;
+      s_t = -1;
+      s_last = -1;
+    }
+  }
+  __syncthreads();
+  const float M = s_max, target = s_target;
+  // pass 2: the inverse CDF, tile by tile in vocabulary order
+  float run = 0.f;  // cumulative weight before this tile (same value in every thread)
+  for (int t0 = 0; t0 < V; t0 += SAMP_TILE) {
+    const int v0 = t0 + tid * SAMP_PER;
+    float w[SAMP_PER];
+    float part = 0.f;
+#pragma unroll
+    for (int j = 0; j < SAMP_PER; ++j) {
+      w[j] = v0 + j < V ? expf(row[v0 + j] * inv_t - M) : 0.f;
+      part += w[j];
+    }
+    float incl = part;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    // exclusive prefix: exactly the previous lane's inclusive value, so the
+    // boundaries never decrease
+    float excl = __shfl_up_sync(0xffffffffu, incl, 1);
+    if (lane == 0) excl = 0.f;
+    if (lane == 31) s_wtot[warp] = incl;
+    __syncthreads();
+    float woff = 0.f;  // exclusive prefix of the warp totals
+    for (int k = 0; k < warp; ++k) woff += s_wtot[k];
+    s_lo[tid] = run + (woff + excl);
+    if (tid == SAMP_THREADS - 1) s_lo[SAMP_THREADS] = run + (woff + incl);
+    __syncthreads();
+    const float lo = s_lo[tid], hi = s_lo[tid + 1];
+    const unsigned live = __ballot_sync(0xffffffffu, part > 0.f);  // last weighted range
+    if (live != 0u && lane == 31 - __clz(live)) atomicMax(&s_last, v0);
+    if (target >= lo && target < hi) {
+      float c = lo;
+      int pick = -1;
+#pragma unroll
+      for (int j = 0; j < SAMP_PER; ++j) {
+        c += w[j];
+        if (w[j] > 0.f) pick = v0 + j;
+        if (w[j] > 0.f && c > target) break;
+      }
+      atomicMax(&s_t, pick);
+    }
+    run = s_lo[SAMP_THREADS];
+    __syncthreads();
+    if (s_t >= 0) break;
+  }
+  if (tid == 0) {
+    int t = s_t;
+    if (t < 0) {
+      // u * sum(w) at or past the rounded total: the last token with weight
+      t = s_last >= 0 ? s_last : 0;
+      const int vmax = min(V, t + SAMP_PER);
+      for (int v = t; v < vmax; ++v)
+        if (expf(row[v] * inv_t - M) > 0.f) t = v;
+    }
+    xhat[prow] = t;
+  }
+}
+
+cudaError_t launch_sample_fused(const float* z, const float* u, int P, int V, float temperature,
+                                int32_t* xhat, cudaStream_t s) {
+  sample_fused_kernel<<<P, SAMP_THREADS, 0, s>>>(z, u, V, 1.f / temperature, xhat);
+  return cudaGetLastError();
+}
+
 // ---------------------------------------------------------------- typical accept (Alg. 3)
 __global__ void accept_typical_kernel(const int32_t* __restrict__ drafts,
                                       const float* __restrict__ scores,

@@ -394,10 +394,16 @@ __device__ __forceinline__ float exp_shifted(float x, float m) {
 
 // Merge running (m, s) with another (M, S): the log-sum-exp of the union is
 // m' + log(s'), m' = max(m, M).
+// The sum update is spelled out with explicit roundings (no contraction left
+// to the compiler), so that lse_merge3 below, which performs the same update,
+// gives bit-identical sums for identical inputs.
+__device__ __forceinline__ float lse_rescale_sum(float s, float a, float S, float c) {
+  return __fmaf_rn(s, a, __fmul_rn(S, c));
+}
 __device__ __forceinline__ void lse_merge(float& m, float& s, float M, float S) {
   const float mn = fmaxf(m, M);
   if (mn == NEG_INF) return;
-  s = s * exp2f((m - mn) * LOG2E) + S * exp2f((M - mn) * LOG2E);
+  s = lse_rescale_sum(s, exp2f(__fmul_rn(m - mn, LOG2E)), S, exp2f(__fmul_rn(M - mn, LOG2E)));
   m = mn;
 }
 

@@ -500,6 +500,11 @@ int check_head_args(rv_handle* h, const void* hidden, const void* w_head, const 
   return RV_OK;
 }
 
+// The head also writes the fused logits (speculative sampling, sampled exact match).
+bool writes_z(const rv_handle* h) {
+  return h->accept_mode == RV_ACCEPT_SPECULATIVE || h->accept_mode == RV_ACCEPT_SAMPLED;
+}
+
 int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_t* draft_ids, int B,
               int gamma, int R, float alpha, float* scores, int32_t* argmax, float* margin,
               const PackArgs* pack, const AcceptArgs* acc, cudaStream_t s) {
@@ -509,7 +514,7 @@ int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_
              h->ws.head_partials, h->ws.gathered, h->ws.status,
              bf16 ? h->ws.status + 16 : nullptr,    // tile counter: its own 64-byte line
              bf16 ? h->ws.status + 32 : nullptr,    // finished-CTA counter
-             h->accept_mode == RV_ACCEPT_SPECULATIVE ? h->zbuf : nullptr};
+             writes_z(h) ? h->zbuf : nullptr};
   HeadPlan pl = head_plan(B, gamma, c.vocab, h->num_sms, bf16);
   if (bf16 && pl.N >= HEAD_PAIR_MIN_N) {
     // CTA pairs: as many as fit at once (two CTAs of a pair share a GPC)
@@ -626,7 +631,7 @@ extern "C" RV_API int rv_set_acceptance(rv_handle* h, int32_t mode, float eps, f
     h->accept_mode = mode;
     return RV_OK;
   }
-  if (mode == RV_ACCEPT_SPECULATIVE) {
+  if (mode == RV_ACCEPT_SPECULATIVE || mode == RV_ACCEPT_SAMPLED) {
     if (!h->zbuf) {
       const rv_config& c = h->cfg;
       const size_t bytes = static_cast<size_t>(c.max_batch) * (c.max_gamma + 1) * c.vocab * 4;
@@ -653,13 +658,33 @@ extern "C" RV_API int rv_set_acceptance(rv_handle* h, int32_t mode, float eps, f
 
 namespace {
 
-// The whole step; `spec` != nullptr runs the speculative-sampling acceptance
-// (Alg. 1) after the head instead of the rule fused into the head's merge.
+// The whole step; `spec` != nullptr runs a sampling acceptance after the head
+// instead of the rule fused into the head's merge: speculative sampling
+// (Alg. 1; q, r, u) or exact match against sampled target tokens (Alg. 2;
+// u, temperature, sampled).
 struct SpecInputs {
   const float* q;
   const float* r;
   const float* u;
+  bool sampled_exact = false;
+  float temperature = 1.f;
+  int32_t* sampled = nullptr;
 };
+
+int sampled_accept_launches(rv_handle* h, const int32_t* draft_ids, const float* u,
+                            float temperature, int B, int gamma, int32_t* sampled,
+                            uint8_t* accept_mask, int32_t* accepted_len, int32_t* next_token,
+                            const int32_t* ctx_in, int32_t* ctx_out, cudaStream_t s) {
+  ProfScope prof(h, RV_PROF_ACCEPT, s);
+  cudaError_t e = launch_sample_fused(h->zbuf, u, B * (gamma + 1), h->cfg.vocab, temperature,
+                                      sampled, s);
+  h->launches += 1;
+  if (e != cudaSuccess) return cuda_fail(h, e, "sampling launch");
+  e = launch_accept(draft_ids, sampled, B, gamma, accept_mask, accepted_len, next_token, ctx_in,
+                    ctx_out, s);
+  h->launches += 1;
+  return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "accept launch");
+}
 
 int step_impl(rv_handle* h, const void* q, const void* k_blk, const void* v_blk, void* k_cache,
               void* v_cache, const void* hidden, const void* w_head, const int32_t* draft_ids,
@@ -703,7 +728,11 @@ int step_impl(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
                   ctx_out,     h->accept_mode,     h->accept_log_eps,  h->accept_log_delta};
     rc = head_impl(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin,
                    do_pack ? &pk : nullptr, spec ? nullptr : &ac, s);
-    if (rc == RV_OK && spec) {
+    if (rc == RV_OK && spec && spec->sampled_exact) {
+      rc = sampled_accept_launches(h, draft_ids, spec->u, spec->temperature, B, gamma,
+                                   spec->sampled, accept_mask, accepted_len, next_token, ctx_in,
+                                   ctx_out, s);
+    } else if (rc == RV_OK && spec) {
       ProfScope prof(h, RV_PROF_ACCEPT, s);
       e = launch_accept_speculative(draft_ids, spec->q, spec->r, spec->u, scores, h->zbuf, B,
                                     gamma, c.vocab, accept_mask, accepted_len, next_token, ctx_in,
@@ -734,6 +763,9 @@ extern "C" RV_API int rv_verify_step(
   if (h->accept_mode == RV_ACCEPT_SPECULATIVE)
     return fail(h, RV_ERR_INVALID_ARG,
                 "speculative sampling needs the draft distributions: use rv_verify_step_speculative");
+  if (h->accept_mode == RV_ACCEPT_SAMPLED)
+    return fail(h, RV_ERR_INVALID_ARG,
+                "sampled exact match needs the uniforms: use rv_verify_step_sampled");
   return step_impl(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, prompt_ids,
                    prefix_ids, ctx_in, B, gamma, n_prompt, n_prefix, alpha, block_ids, pos_ids,
                    attn_out, scores, argmax, margin, accept_mask, accepted_len, next_token, ctx_out,
@@ -760,6 +792,56 @@ extern "C" RV_API int rv_verify_step_speculative(
                    prefix_ids, ctx_in, B, gamma, n_prompt, n_prefix, alpha, block_ids, pos_ids,
                    attn_out, scores, argmax, margin, accept_mask, accepted_len, next_token, ctx_out,
                    &spec, stream);
+}
+
+extern "C" RV_API int rv_verify_step_sampled(
+    rv_handle* h, const void* q, const void* k_blk, const void* v_blk, void* k_cache, void* v_cache,
+    const void* hidden, const void* w_head, const int32_t* draft_ids, const int32_t* prompt_ids,
+    const int32_t* prefix_ids, const int32_t* ctx_in, int32_t B, int32_t gamma, int32_t n_prompt,
+    int32_t n_prefix, float alpha, float temperature, const float* u_uniform, int32_t* block_ids,
+    int32_t* pos_ids, void* attn_out, float* scores, int32_t* argmax, float* margin,
+    int32_t* sampled, uint8_t* accept_mask, int32_t* accepted_len, int32_t* next_token,
+    int32_t* ctx_out, void* stream) {
+  if (!h) return RV_ERR_INVALID_ARG;
+  h->err.clear();
+  if (h->accept_mode != RV_ACCEPT_SAMPLED || !h->zbuf)
+    return fail(h, RV_ERR_INVALID_ARG, "call rv_set_acceptance(RV_ACCEPT_SAMPLED) on the handle first");
+  if (!(temperature > 0.f) || !std::isfinite(temperature))
+    return fail(h, RV_ERR_INVALID_ARG, "temperature must be finite and > 0");
+  if (B > 0 && (!u_uniform || !sampled))
+    return fail(h, RV_ERR_INVALID_ARG, "NULL uniforms or sampled-token output");
+  SpecInputs spec{nullptr, nullptr, u_uniform};
+  spec.sampled_exact = true;
+  spec.temperature = temperature;
+  spec.sampled = sampled;
+  return step_impl(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, prompt_ids,
+                   prefix_ids, ctx_in, B, gamma, n_prompt, n_prefix, alpha, block_ids, pos_ids,
+                   attn_out, scores, argmax, margin, accept_mask, accepted_len, next_token, ctx_out,
+                   &spec, stream);
+}
+
+extern "C" RV_API int rv_accept_sampled(rv_handle* h, const int32_t* draft_ids,
+                                        const float* u_uniform, float temperature, int32_t B,
+                                        int32_t gamma, int32_t* sampled, uint8_t* accept_mask,
+                                        int32_t* accepted_len, int32_t* next_token,
+                                        const int32_t* ctx_in, int32_t* ctx_out, void* stream) {
+  if (!h) return RV_ERR_INVALID_ARG;
+  h->err.clear();
+  if (h->accept_mode != RV_ACCEPT_SAMPLED || !h->zbuf)
+    return fail(h, RV_ERR_INVALID_ARG,
+                "call rv_set_acceptance(RV_ACCEPT_SAMPLED) before rv_verify_head");
+  if (B < 0 || gamma < 1) return fail(h, RV_ERR_SHAPE, "need B >= 0 and gamma >= 1");
+  if (B > h->cfg.max_batch || gamma > h->cfg.max_gamma)
+    return fail(h, RV_ERR_CAPACITY, "B / gamma above the handle's maxima");
+  if (!(temperature > 0.f) || !std::isfinite(temperature))
+    return fail(h, RV_ERR_INVALID_ARG, "temperature must be finite and > 0");
+  if (B == 0) return RV_OK;
+  if (!draft_ids || !u_uniform || !sampled || !accept_mask || !accepted_len || !next_token ||
+      !ctx_in || !ctx_out)
+    return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument");
+  return sampled_accept_launches(h, draft_ids, u_uniform, temperature, B, gamma, sampled,
+                                 accept_mask, accepted_len, next_token, ctx_in, ctx_out,
+                                 static_cast<cudaStream_t>(stream));
 }
 
 extern "C" RV_API int rv_accept_speculative(rv_handle* h, const int32_t* draft_ids,

@@ -120,6 +120,11 @@ cudaError_t launch_accept_speculative(const int32_t* drafts, const float* q, con
                                       int32_t* accepted_len, int32_t* next_token,
                                       const int32_t* ctx_in, int32_t* ctx_out, unsigned* status,
                                       cudaStream_t s);
+// Target tokens at temperature T (Alg. 2 with sampling): for each of the P
+// positions, xhat[p] ~ softmax(z[p] / T) by inverse CDF with u[p]; z [P][V]
+// are the fused logits the head wrote.  One CTA per position.
+cudaError_t launch_sample_fused(const float* z, const float* u, int P, int V, float temperature,
+                                int32_t* xhat, cudaStream_t s);
 // Typical acceptance (Alg. 3) from the head's scores and argmax.
 cudaError_t launch_accept_typical(const int32_t* drafts, const float* scores,
                                   const int32_t* argmax, int B, int gamma, float log_eps,

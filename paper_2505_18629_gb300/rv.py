@@ -37,7 +37,7 @@ RV_SCORE_LSE_ORIG, RV_SCORE_LSE_REFL, RV_SCORE_LSE_FUSED = 0, 1, 2
 RV_SCORE_LOGP_FUSED, RV_SCORE_LOGP_ORIG, RV_SCORE_LOGP_REFL = 3, 4, 5
 RV_SCORE_ENT_ORIG = 6
 
-RV_ACCEPT_EXACT, RV_ACCEPT_TYPICAL, RV_ACCEPT_SPECULATIVE = 0, 1, 2
+RV_ACCEPT_EXACT, RV_ACCEPT_TYPICAL, RV_ACCEPT_SPECULATIVE, RV_ACCEPT_SAMPLED = 0, 1, 2, 3
 
 RV_PROF_ATTENTION, RV_PROF_HEAD_GEMM, RV_PROF_HEAD, RV_PROF_ACCEPT = 0, 1, 2, 3
 
@@ -78,6 +78,9 @@ def _load():
         "rv_accept_speculative": (I, [P, P, P, P, P, P, I, I, P, P, P, P, P, P]),
         "rv_verify_step_speculative": (I, [P, P, P, P, P, P, P, P, P, P, P, P, I, I, I, I, F, P, P,
                                            P, P, P, P, P, P, P, P, P, P, P, P]),
+        "rv_accept_sampled": (I, [P, P, P, F, I, I, P, P, P, P, P, P, P]),
+        "rv_verify_step_sampled": (I, [P, P, P, P, P, P, P, P, P, P, P, P, I, I, I, I, F, F, P, P,
+                                       P, P, P, P, P, P, P, P, P, P, P]),
         "rv_verify_step": (I, [P, P, P, P, P, P, P, P, P, P, P, P, I, I, I, I, F, P, P, P, P, P, P,
                                P, P, P, P, P]),
         "rv_verify_step_host": (I, [P, P, P, P, P, P, P, P, P, P, P, P, I, I, I, I, F, P, P, P, P,
@@ -223,6 +226,15 @@ def rv_accept_speculative(h, draft_ids, q_draft, r_uniform, u_uniform, scores, a
                                          _ptr(ctx_out), _stream(stream)))
 
 
+def rv_accept_sampled(h, draft_ids, u_uniform, temperature, sampled, accept_mask, accepted_len,
+                      next_token, ctx_in, ctx_out, stream=None):
+    B, gamma = draft_ids.shape
+    _check(h, _lib.rv_accept_sampled(h.ptr, _ptr(draft_ids), _ptr(u_uniform), float(temperature),
+                                     B, gamma, _ptr(sampled), _ptr(accept_mask),
+                                     _ptr(accepted_len), _ptr(next_token), _ptr(ctx_in),
+                                     _ptr(ctx_out), _stream(stream)))
+
+
 def rv_set_acceptance(h, mode, eps=0.0, delta=0.0):
     _check(h, _lib.rv_set_acceptance(h.ptr, int(mode), float(eps), float(delta)))
 
@@ -255,6 +267,22 @@ def rv_verify_step_speculative(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_h
         _ptr(w_head), _ptr(draft_ids), _ptr(prompt_ids), _ptr(prefix_ids), _ptr(ctx_in), B, gamma,
         n_prompt, n_prefix, float(alpha), _ptr(q_draft), _ptr(r_uniform), _ptr(u_uniform),
         _ptr(block_ids), _ptr(pos_ids), _ptr(attn_out), _ptr(scores), _ptr(argmax), _ptr(margin),
+        _ptr(accept_mask), _ptr(accepted_len), _ptr(next_token), _ptr(ctx_out), _stream(stream)))
+
+
+def rv_verify_step_sampled(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids,
+                           prompt_ids, prefix_ids, ctx_in, alpha, temperature, u_uniform,
+                           block_ids, pos_ids, attn_out, scores, argmax, margin, sampled,
+                           accept_mask, accepted_len, next_token, ctx_out, stream=None):
+    """Whole step with exact match against target tokens sampled at temperature T (Alg. 2)."""
+    B, gamma = draft_ids.shape
+    n_prompt = 0 if prompt_ids is None else prompt_ids.numel()
+    n_prefix = prefix_ids.shape[1]
+    _check(h, _lib.rv_verify_step_sampled(
+        h.ptr, _ptr(q), _ptr(k_blk), _ptr(v_blk), _ptr(k_cache), _ptr(v_cache), _ptr(hidden),
+        _ptr(w_head), _ptr(draft_ids), _ptr(prompt_ids), _ptr(prefix_ids), _ptr(ctx_in), B, gamma,
+        n_prompt, n_prefix, float(alpha), float(temperature), _ptr(u_uniform), _ptr(block_ids),
+        _ptr(pos_ids), _ptr(attn_out), _ptr(scores), _ptr(argmax), _ptr(margin), _ptr(sampled),
         _ptr(accept_mask), _ptr(accepted_len), _ptr(next_token), _ptr(ctx_out), _stream(stream)))
 
 

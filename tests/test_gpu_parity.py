@@ -147,6 +147,16 @@ def test_bf16_multi_chunk(gu):
     _check(gu, _wl(B=20, gamma=8, R=2, V=1500, H=128, ctx=(1, 40), seed=46), check_attn=False)
 
 
+@pytest.mark.parametrize("B,gamma,V", [(16, 8, 1000), (16, 8, 60000), (15, 9, 60000)])
+def test_bf16_pair_kernel_two_chunks_many_tiles(gu, B, gamma, V):
+    # 144 / 150 pairs -> two chunks of 72 / 75 pairs on CTA pairs (the second
+    # shape with 5 padding pairs per chunk); at V = 60000 every CTA pair runs
+    # several vocab tiles, so both accumulator slots are reused and their
+    # barrier phases flip; H = 320 leaves a half-filled last K stage
+    _check(gu, _wl(B=B, gamma=gamma, R=3, V=V, H=320, ctx=(1, 30), seed=47 + V % 7),
+           check_attn=False)
+
+
 def test_bf16_no_template_gamma1(gu):
     _check(gu, _wl(gamma=1, R=0, B=2, seed=47), ctx=[3, 0])
 
@@ -520,6 +530,141 @@ def test_speculative_sampling_pairs_and_8b(gu):
         inp = synth.generate(wl)
         z, q, drafts, r, u = _spec_inputs(inp, ALPHA, 85)
         _check_spec(inp, z, q, drafts, r, u, _run_spec(gu, inp, drafts, ALPHA, q, r, u))
+
+
+# ------------------------------------------------------------------ sampled exact match (Alg. 2, temperature T)
+
+def _sampled_inputs(inp, alpha, T, seed, keep=0.7):
+    """The oracle's fused logits z, uniforms u [B, gamma+1], and drafts that
+    equal the oracle's sampled target token with probability `keep`."""
+    import oracle.rv_oracle as orc
+    wl = inp.wl
+    rng = np.random.default_rng(seed)
+    dummy = np.zeros((wl.B, wl.gamma), np.int64)
+    z = orc.verify_head(inp.W, inp.hidden, dummy, wl.gamma, wl.R, alpha)["z"]
+    u = rng.uniform(0, 1, (wl.B, wl.gamma + 1)).astype(np.float32)
+    _, _, _, xhat, _ = orc.sampled_exact_accept(dummy, z, T, u.astype(np.float64))
+    alt = rng.integers(0, wl.V, (wl.B, wl.gamma))
+    drafts = np.where(rng.uniform(size=(wl.B, wl.gamma)) < keep, xhat[:, :wl.gamma], alt)
+    return z, u, drafts.astype(np.int64)
+
+
+def _run_sampled(gu, inp, drafts, alpha, T, u, separate=False):
+    import torch
+    from paper_2505_18629_gb300 import rv
+    wl = inp.wl
+    B, g = wl.B, wl.gamma
+    h = gu.make_handle(wl)
+    rv.rv_set_acceptance(h, rv.RV_ACCEPT_SAMPLED)
+    du = gu.to_dev(u)
+    d = gu.to_dev(drafts.astype(np.int32))
+    ctx = gu.to_dev(inp.ctx_lens.astype(np.int32))
+    sc = torch.empty((B, g + 1, rv.RV_NSCORES), device="cuda")
+    am = torch.empty((B, g + 1), dtype=torch.int32, device="cuda")
+    mg = torch.empty((B, g), device="cuda")
+    xs = torch.full((B, g + 1), -7, dtype=torch.int32, device="cuda")
+    acc = torch.full((B, g), 7, dtype=torch.uint8, device="cuda")
+    n = torch.full((B,), -7, dtype=torch.int32, device="cuda")
+    t = torch.full((B,), -7, dtype=torch.int32, device="cuda")
+    co = torch.full((B,), -7, dtype=torch.int32, device="cuda")
+    if separate:
+        rv.rv_verify_head(h, gu.to_dev(inp.hidden), gu.to_dev(inp.W), d, g, wl.R, alpha, sc, am, mg)
+        rv.rv_accept_sampled(h, d, du, T, xs, acc, n, t, ctx, co)
+    else:
+        q_, kb, vb = gu.to_dev(inp.q), gu.to_dev(inp.k_blk), gu.to_dev(inp.v_blk)
+        kc, vc = gu.to_dev(inp.k_cache), gu.to_dev(inp.v_cache)
+        prompt = gu.to_dev(inp.prompt_ids.astype(np.int32)) if inp.prompt_ids.size else None
+        prefix = gu.to_dev(inp.prefix_ids.astype(np.int32))
+        attn = torch.zeros_like(q_)
+        with pytest.raises(rv.RVError):  # the plain step refuses the sampling rule (no uniforms)
+            rv.rv_verify_step(h, q_, kb, vb, kc, vc, gu.to_dev(inp.hidden), gu.to_dev(inp.W), d,
+                              prompt, prefix, ctx, alpha, None, None, attn, sc, am, mg, acc, n, t, co)
+        with pytest.raises(rv.RVError):  # temperature must be > 0
+            rv.rv_verify_step_sampled(h, q_, kb, vb, kc, vc, gu.to_dev(inp.hidden),
+                                      gu.to_dev(inp.W), d, prompt, prefix, ctx, alpha, 0.0, du,
+                                      None, None, attn, sc, am, mg, xs, acc, n, t, co)
+        rv.rv_verify_step_sampled(h, q_, kb, vb, kc, vc, gu.to_dev(inp.hidden), gu.to_dev(inp.W),
+                                  d, prompt, prefix, ctx, alpha, T, du, None, None, attn, sc, am,
+                                  mg, xs, acc, n, t, co)
+    status = rv.rv_read_status(h)
+    h.close()
+    return (gu.to_np(xs), gu.to_np(acc), gu.to_np(n), gu.to_np(t), gu.to_np(co), gu.to_np(am),
+            status)
+
+
+def _check_sampled(inp, z, u, drafts, T, gpu, min_match=0.9, tol=SPEC_TOL):
+    """Sampled tokens equal the oracle's draw except where u lies within
+    SPEC_TOL of a cumulative-weight boundary (then the token must be one whose
+    CDF interval holds u up to SPEC_TOL); acceptance, n, t and ctx follow the
+    GPU's own draws exactly (Alg. 2), and equal the oracle's wherever every
+    draw up to n+1 matched."""
+    import oracle.rv_oracle as orc
+    wl = inp.wl
+    g = wl.gamma
+    xs, acc, n, t, co, _, status = gpu
+    assert status == 0
+    acc_o, n_o, t_o, xhat_o, gap = orc.sampled_exact_accept(drafts, z, T, u.astype(np.float64))
+    zt = z / T
+    p_t = np.exp(zt - orc.logsumexp(zt)[..., None])
+    same = xs == xhat_o
+    for b, i in zip(*np.nonzero(~same)):
+        assert gap[b, i] < tol, f"draw ({b},{i}): {xs[b, i]} vs {xhat_o[b, i]}, gap {gap[b, i]:.2e}"
+        c = np.cumsum(p_t[b, i])
+        k = int(xs[b, i])
+        lo = c[k - 1] if k > 0 else 0.0
+        assert lo - tol <= u[b, i] <= c[k] + tol
+    assert same.mean() >= min_match, f"only {same.mean():.3f} of the draws match"
+    # Alg. 2 on the GPU's own draws: bit-exact
+    acc_s, n_s, t_s = orc.exact_match_accept(drafts, xs)
+    assert (acc == acc_s).all() and (n == n_s).all() and (t == t_s).all()
+    assert (co == inp.ctx_lens + n).all()
+    rows_same = same.all(axis=1)
+    assert (n[rows_same] == n_o[rows_same]).all() and (t[rows_same] == t_o[rows_same]).all()
+    return acc, n
+
+
+@pytest.mark.parametrize("T,separate", [(1.0, False), (0.8, True), (0.2, False)])
+def test_sampled_exact_match_small(gu, T, separate):
+    from paper_2505_18629_gb300 import synth
+    wl = _wl(B=8, gamma=5, V=1000, seed=90)
+    inp = synth.generate(wl)
+    z, u, drafts = _sampled_inputs(inp, ALPHA, T, 91)
+    acc, n = _check_sampled(inp, z, u, drafts, T,
+                            _run_sampled(gu, inp, drafts, ALPHA, T, u, separate=separate))
+    assert 0 < acc.sum() < acc.size
+
+
+def test_sampled_exact_match_low_temperature_is_greedy(gu):
+    # T -> 0: every draw is the greedy choice of the head (away from ties)
+    from paper_2505_18629_gb300 import synth
+    wl = _wl(B=6, gamma=4, V=1500, seed=92)
+    inp = synth.generate(wl)
+    T = 1e-4
+    z, u, drafts = _sampled_inputs(inp, ALPHA, T, 93)
+    gpu = _run_sampled(gu, inp, drafts, ALPHA, T, u)
+    _check_sampled(inp, z, u, drafts, T, gpu)
+    xs, am = gpu[0], gpu[5]
+    srt = np.sort(z, axis=-1)
+    clear = (srt[..., -1] - srt[..., -2]) > 1e-3
+    assert (xs[clear] == am[clear]).all()
+
+
+@pytest.mark.parametrize("name", ["tiny", "pairs", "llama3-8b-b1"])
+def test_sampled_exact_match_kernels_and_8b(gu, name):
+    # the fp32 head, the CTA-pair head (N >= 96) and the full 8B vocabulary
+    from paper_2505_18629_gb300 import synth
+    wl = (_wl(B=14, gamma=8, R=8, V=777, H=256, ctx=(10, 60), seed=94) if name == "pairs"
+          else synth.WORKLOADS[name])
+    inp = synth.generate(wl)
+    z, u, drafts = _sampled_inputs(inp, ALPHA, 0.8, 95)
+    gpu = _run_sampled(gu, inp, drafts, ALPHA, 0.8, u)
+    if name == "llama3-8b-b1":
+        # 128256 tokens: adjacent CDF boundaries are ~1e-5 apart, as close as the
+        # fp32-vs-fp64 logit error moves them; a draw may land on a neighbour,
+        # whose interval must then hold u within 2e-4
+        _check_sampled(inp, z, u, drafts, 0.8, gpu, min_match=0.0, tol=2e-4)
+    else:
+        _check_sampled(inp, z, u, drafts, 0.8, gpu)
 
 
 # ------------------------------------------------------------------ full-size workloads

@@ -22,6 +22,9 @@ Notation follows the paper:
     (Alg. 2, read as "stop at the first mismatch"; see ``exact_match_accept``)
     or with sampled x^_i ~ softmax(z_i / T) (``sampled_exact_accept``)
   * typical acceptance (Alg. 3) and speculative sampling (Alg. 1)
+  * the pending-token block [t, x_1..x_gamma, template, x_1..x_gamma], whose
+    first position is the last emitted token (``pack_block_pending``,
+    ``verify_step_pending``)
 
 Hidden-state rows: row 0 is the target's last hidden state after the prefix
 (gives o_1, "M_p(prefix)" in Alg. 1); row r (1..Lb) follows block token r-1.
@@ -101,6 +104,23 @@ def pack_block(drafts, prompt_ids, prefix_ids, ctx_lens):
         rows.append(blk)
         pos.append(int(ctx_lens[b]) + np.arange(blk.shape[0], dtype=np.int64))
     return np.stack(rows).astype(np.int32), np.stack(pos).astype(np.int32)
+
+
+def pack_block_pending(pending, drafts, prompt_ids, prefix_ids, ctx_lens):
+    """Pending-token variant of the block: [t, x_1..x_gamma, template, x_1..x_gamma].
+
+    The last emitted token t (pending[b]) has not gone through the target yet,
+    so the block starts with it: its position is the first after the context,
+    its final hidden state gives o_1 ("M_p(prefix)" in Alg. 1, with the
+    prefix ending in t), and its key/value are appended with the block's.
+    Returns block_ids, pos_ids [B, Lb + 1] (Lb = 2 gamma + R), positions
+    ctx_b, ctx_b + 1, ...
+    """
+    pending = np.asarray(pending, np.int64)
+    blk, _ = pack_block(drafts, prompt_ids, prefix_ids, ctx_lens)
+    block = np.concatenate([pending[:, None], blk.astype(np.int64)], axis=1)
+    pos = np.asarray(ctx_lens, np.int64)[:, None] + np.arange(block.shape[1], dtype=np.int64)
+    return block.astype(np.int32), pos.astype(np.int32)
 
 
 # --------------------------------------------------------------------------
@@ -397,3 +417,24 @@ def verify_step(inp_W, hidden, q, k_blk, v_blk, k_cache, v_cache, ctx_lens,
     return dict(block_ids=block_ids, pos_ids=pos_ids, attn=attn, k_cache=kc, v_cache=vc,
                 accept_mask=acc, accepted_len=n, next_token=t,
                 ctx_out=np.asarray(ctx_lens, np.int64) + n, **head)
+
+
+def verify_step_pending(inp_W, hidden, q, k_blk, v_blk, k_cache, v_cache, ctx_lens, pending,
+                        drafts, prompt_ids, prefix_ids, gamma: int, R: int, alpha: float):
+    """The verify step with the pending-token block [t, x_1..x_gamma, template,
+    x_1..x_gamma] (Lb + 1 = 2 gamma + R + 1 positions after the context).
+
+    Hidden row 0 is the pending token's (it gives o_1), so the head's rows are
+    those of ``verify_head`` unchanged: original rows 0..gamma, reflective
+    rows gamma+R..2 gamma+R.  The attention covers the Lb + 1 block positions
+    and appends all their keys/values.  Of those, t and the n accepted drafts
+    stay in the context: the new length is ctx + 1 + n (the template, the
+    copy and the rejected drafts are pruned by length, Sec. 3.1).
+    """
+    block_ids, pos_ids = pack_block_pending(pending, drafts, prompt_ids, prefix_ids, ctx_lens)
+    attn, kc, vc = verify_attention(q, k_blk, v_blk, k_cache, v_cache, ctx_lens)
+    head = verify_head(inp_W, hidden, drafts, gamma, R, alpha)
+    acc, n, t = exact_match_accept(drafts, head["argmax"])
+    return dict(block_ids=block_ids, pos_ids=pos_ids, attn=attn, k_cache=kc, v_cache=vc,
+                accept_mask=acc, accepted_len=n, next_token=t,
+                ctx_out=np.asarray(ctx_lens, np.int64) + 1 + n, **head)

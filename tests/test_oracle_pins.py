@@ -665,3 +665,129 @@ def test_pins_catch_temperature_multiplied(monkeypatch):
     monkeypatch.setattr(orc, "sampled_exact_accept",
                         lambda drafts, z, T, u: real(drafts, np.asarray(z) * T * T, T, u))
     assert _fails(lambda: test_sampled_exact_temperature_closed_form(0.2))
+
+
+# --------------------------------------------------------------------------
+# Pending-token block [t, x_1..x_gamma, template, x_1..x_gamma]
+# --------------------------------------------------------------------------
+
+def test_pending_block_layout_table3():
+    # Table 3's {5+3+4+5} block with the last emitted token in front: 18 positions
+    g = _golden("table3_block_layout.json")
+    gamma, n_prompt, n_prefix = g["gamma"], g["n_prompt"], g["n_prefix"]
+    drafts = np.array([[101, 102, 103, 104, 105], [111, 112, 113, 114, 115]])
+    prompt = np.array([201, 202, 203])
+    prefix = np.array([[301, 302, 303, 304], [311, 312, 313, 314]])
+    ctx = np.array([40, 7])
+    blk, pos = orc.pack_block_pending(np.array([99, 98]), drafts, prompt, prefix, ctx)
+    std, _ = orc.pack_block(drafts, prompt, prefix, ctx)
+    assert blk.shape == (2, g["budget"] + 1)
+    assert list(blk[:, 0]) == [99, 98]
+    np.testing.assert_array_equal(blk[:, 1:], std)
+    for b in range(2):
+        assert list(pos[b]) == list(range(ctx[b], ctx[b] + g["budget"] + 1))
+
+
+@pytest.mark.parametrize("gamma,R", [(5, 7), (1, 0), (4, 4)])
+def test_pending_rows_score_their_draft(gamma, R):
+    # hidden row r follows pending-block position r and predicts position r + 1:
+    # row 0 (the pending token) predicts x_1, and the head's original /
+    # reflective rows (unchanged from the standard layout) score x_i twice
+    drafts = np.arange(1, gamma + 1)[None, :] + 1000
+    prompt = np.arange(max(R - min(R, 4), 0)) + 2000
+    prefix = (np.arange(min(R, 4)) + 3000)[None, :]
+    blk, _ = orc.pack_block_pending(np.array([7]), drafts, prompt, prefix, np.array([0]))
+    b = blk[0]
+    for i in range(1, gamma + 1):
+        assert b[orc.original_row(i) + 1] == drafts[0, i - 1]
+        assert b[orc.reflective_row(i, gamma, R) + 1] == drafts[0, i - 1]
+    assert orc.reflective_row(gamma + 1, gamma, R) == b.shape[0] - 1   # the last position
+
+
+def _pending_attention_case(rng, B=3, gamma=3, R=2, Hq=4, Hkv=2, D=8, ctxs=(0, 5, 11)):
+    Lp = 2 * gamma + R + 1
+    C = max(ctxs) + Lp + 2
+    q = rng.normal(size=(B, Lp, Hq, D))
+    kb = rng.normal(size=(B, Lp, Hkv, D))
+    vb = rng.normal(size=(B, Lp, Hkv, D))
+    kc = rng.normal(size=(B, Hkv, C, D))
+    vc = rng.normal(size=(B, Hkv, C, D))
+    return q, kb, vb, kc, vc, np.asarray(ctxs)
+
+
+def test_pending_attention_equals_standard_after_appending_t():
+    # Causality (Sec. 3.1): running the pending block at ctx is the same forward
+    # pass as first appending t's key/value at position ctx and running the
+    # standard block at ctx + 1 -- same outputs for the block's other rows, same
+    # cache afterwards; and t's own row is plain decoding over context + t.
+    rng = np.random.default_rng(31)
+    q, kb, vb, kc, vc, ctx = _pending_attention_case(rng)
+    out, kc1, vc1 = orc.verify_attention(q, kb, vb, kc, vc, ctx)
+    kc2, vc2 = kc.copy(), vc.copy()
+    for b in range(len(ctx)):
+        kc2[b, :, ctx[b]] = kb[b, 0]
+        vc2[b, :, ctx[b]] = vb[b, 0]
+    out2, kc3, vc3 = orc.verify_attention(q[:, 1:], kb[:, 1:], vb[:, 1:], kc2, vc2, ctx + 1)
+    np.testing.assert_allclose(out[:, 1:], out2, rtol=0, atol=1e-12)
+    np.testing.assert_array_equal(kc1, kc3)
+    np.testing.assert_array_equal(vc1, vc3)
+    dec, _, _ = orc.verify_attention(q[:, :1], kb[:, :1], vb[:, :1], kc, vc, ctx)
+    np.testing.assert_allclose(out[:, :1], dec, rtol=0, atol=1e-12)
+
+
+def test_pending_step_keeps_t_and_the_accepted_drafts():
+    # After the step the context is [old context, t, x_1..x_n]: its last kept
+    # key is x_n's (t's when n = 0) and t's key sits at the old length.
+    from paper_2505_18629_gb300 import synth
+    wl = synth.Workload("p", B=4, gamma=3, R=2, ctx=(0, 20), H=32, Hq=4, Hkv=2, D=16, V=50,
+                        dtype="f32", p_argmax=0.5, seed=33)
+    inp = synth.generate(wl)
+    Lp = wl.Lb + 1
+    rng = np.random.default_rng(34)
+    q = rng.normal(size=(wl.B, Lp, wl.Hq, wl.D)).astype(np.float32)
+    kb = rng.normal(size=(wl.B, Lp, wl.Hkv, wl.D)).astype(np.float32)
+    vb = rng.normal(size=(wl.B, Lp, wl.Hkv, wl.D)).astype(np.float32)
+    kc = np.zeros((wl.B, wl.Hkv, wl.capacity + 1, wl.D), np.float32)
+    vc = np.zeros_like(kc)
+    choice = orc.verify_head(inp.W, inp.hidden, np.zeros((wl.B, wl.gamma), np.int64), wl.gamma,
+                             wl.R, 0.3)["argmax"]
+    drafts = np.where(rng.uniform(size=(wl.B, wl.gamma)) < 0.6, choice[:, :wl.gamma],
+                      rng.integers(0, wl.V, (wl.B, wl.gamma)))
+    pending = rng.integers(0, wl.V, wl.B)
+    r = orc.verify_step_pending(inp.W, inp.hidden, q, kb, vb, kc, vc, inp.ctx_lens, pending,
+                                drafts, inp.prompt_ids, inp.prefix_ids, wl.gamma, wl.R, 0.3)
+    assert (r["block_ids"][:, 0] == pending).all()
+    for b in range(wl.B):
+        c, n, co = int(inp.ctx_lens[b]), int(r["accepted_len"][b]), int(r["ctx_out"][b])
+        np.testing.assert_array_equal(r["k_cache"][b, :, c], kb[b, 0])          # t
+        np.testing.assert_array_equal(r["k_cache"][b, :, co - 1], kb[b, n])     # x_n (or t)
+        assert co - c - 1 == n
+    # the emitted tokens are those of the standard layout's step (same head rows)
+    std = orc.exact_match_accept(drafts, r["argmax"])
+    np.testing.assert_array_equal(r["accepted_len"], std[1])
+    np.testing.assert_array_equal(r["next_token"], std[2])
+
+
+def test_pins_catch_pending_length_without_t(monkeypatch):
+    real = orc.verify_step_pending
+
+    def drop_t(*args, **kw):
+        r = real(*args, **kw)
+        r["ctx_out"] = r["ctx_out"] - 1
+        return r
+    monkeypatch.setattr(orc, "verify_step_pending", drop_t)
+    with pytest.raises(AssertionError):
+        test_pending_step_keeps_t_and_the_accepted_drafts()
+
+
+def test_pins_catch_pending_token_at_the_end(monkeypatch):
+    real = orc.pack_block
+
+    def t_last(pending, drafts, prompt_ids, prefix_ids, ctx_lens):
+        blk, pos = real(drafts, prompt_ids, prefix_ids, ctx_lens)
+        blk = np.concatenate([blk, np.asarray(pending)[:, None]], axis=1).astype(np.int32)
+        pos = (np.asarray(ctx_lens)[:, None] + np.arange(blk.shape[1])).astype(np.int32)
+        return blk, pos
+    monkeypatch.setattr(orc, "pack_block_pending", t_last)
+    with pytest.raises(AssertionError):
+        test_pending_block_layout_table3()

@@ -128,6 +128,18 @@ RV_API int rv_pack_block(rv_handle* h, const int32_t* draft_ids, const int32_t* 
                          int32_t gamma, int32_t n_prompt, int32_t n_prefix, int32_t* block_ids,
                          int32_t* pos_ids, void* stream);
 
+/* The pending-token block [t_b, x_1..x_gamma, prompt, prefix_b, x_1..x_gamma]:
+ * as rv_pack_block, with the last emitted token t_b = pending_ids[b] (not yet
+ * run through the target) in front.  Its final hidden state gives o_1 (the
+ * prefix of Alg. 1 then ends in t_b), and its key/value are appended with the
+ * block's.  Outputs block_ids, pos_ids [B, Lb + 1] with positions
+ * ctx_lens[b] .. ctx_lens[b] + Lb, Lb = 2*gamma + n_prompt + n_prefix. */
+RV_API int rv_pack_block_pending(rv_handle* h, const int32_t* pending_ids,
+                                 const int32_t* draft_ids, const int32_t* prompt_ids,
+                                 const int32_t* prefix_ids, const int32_t* ctx_lens, int32_t B,
+                                 int32_t gamma, int32_t n_prompt, int32_t n_prefix,
+                                 int32_t* block_ids, int32_t* pos_ids, void* stream);
+
 /* One attention layer of the verify forward pass (Sec. 3.1): causal attention
  * of the block's queries against the KV cache plus the block itself.  Query j
  * of sequence b (position ctx_b + j) attends to cached keys [0, ctx_b) and
@@ -275,6 +287,23 @@ RV_API int rv_verify_step(rv_handle* h, const void* q, const void* k_blk, const 
                           int32_t* argmax, float* margin, uint8_t* accept_mask,
                           int32_t* accepted_len, int32_t* next_token, int32_t* ctx_out,
                           void* stream);
+
+/* rv_verify_step over the pending-token block (rv_pack_block_pending): the
+ * attention covers Lb + 1 = 2*gamma + R + 1 block positions (q, k_blk,
+ * v_blk, attn_out have Lb + 1 rows; their keys/values are appended at
+ * [ctx_b, ctx_b + Lb + 1)); hidden [B, Lb + 1, H] has the pending token's
+ * state in row 0, which gives o_1, so the LM head is unchanged (original rows
+ * 0..gamma, reflective rows gamma+R..2*gamma+R).  The handle's exact-match or
+ * typical rule runs; since t stays in the context, ctx_out = ctx_in + 1 + n.
+ * RV_ERR_INVALID_ARG in the sampling modes. */
+RV_API int rv_verify_step_pending(
+    rv_handle* h, const void* q, const void* k_blk, const void* v_blk, void* k_cache,
+    void* v_cache, const void* hidden, const void* w_head, const int32_t* pending_ids,
+    const int32_t* draft_ids, const int32_t* prompt_ids, const int32_t* prefix_ids,
+    const int32_t* ctx_in, int32_t B, int32_t gamma, int32_t n_prompt, int32_t n_prefix,
+    float alpha, int32_t* block_ids, int32_t* pos_ids, void* attn_out, float* scores,
+    int32_t* argmax, float* margin, uint8_t* accept_mask, int32_t* accepted_len,
+    int32_t* next_token, int32_t* ctx_out, void* stream);
 
 /* rv_verify_step with the speculative-sampling acceptance of Alg. 1
  * (rv_accept_speculative) in place of the handle's fused rule; needs the

@@ -391,7 +391,7 @@ __device__ __forceinline__ void head_merge_all(const float* partials, const floa
     }
     f.acc.accepted_len[b] = n;
     f.acc.next_token[b] = s_choice[b * (gamma + 1) + n];
-    f.acc.ctx_out[b] = f.acc.ctx_in[b] + n;
+    f.acc.ctx_out[b] = f.acc.ctx_in[b] + n + f.acc.ctx_extra;
   }
 }
 

@@ -16,18 +16,23 @@ namespace rv {
 
 // ---------------------------------------------------------------- pack (Eq. 1)
 // block[b] = [x_1..x_gamma, prompt, prefix_b, x_1..x_gamma]; pos = ctx_b + j.
+// With `pending`, the pending-token block [t_b, x_1..x_gamma, prompt, prefix_b,
+// x_1..x_gamma]: the last emitted token goes first.
 __global__ void pack_block_kernel(const int32_t* __restrict__ drafts,
                                   const int32_t* __restrict__ prompt,
                                   const int32_t* __restrict__ prefix,
                                   const int32_t* __restrict__ ctx, int B, int gamma,
                                   int n_prompt, int n_prefix, int32_t* __restrict__ block,
-                                  int32_t* __restrict__ pos) {
-  const int Lb = 2 * gamma + n_prompt + n_prefix;
+                                  int32_t* __restrict__ pos, const int32_t* __restrict__ pending) {
+  const int lead = pending ? 1 : 0;
+  const int Lb = 2 * gamma + n_prompt + n_prefix + lead;
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= B * Lb) return;
-  const int b = idx / Lb, j = idx % Lb;
+  const int b = idx / Lb, jj = idx % Lb, j = jj - lead;
   int tok;
-  if (j < gamma) {
+  if (j < 0) {
+    tok = pending[b];
+  } else if (j < gamma) {
     tok = drafts[b * gamma + j];
   } else if (j < gamma + n_prompt) {
     tok = prompt[j - gamma];
@@ -37,16 +42,18 @@ __global__ void pack_block_kernel(const int32_t* __restrict__ drafts,
     tok = drafts[b * gamma + (j - gamma - n_prompt - n_prefix)];
   }
   block[idx] = tok;
-  pos[idx] = ctx[b] + j;
+  pos[idx] = ctx[b] + jj;
 }
 
 cudaError_t launch_pack_block(const int32_t* drafts, const int32_t* prompt, const int32_t* prefix,
                               const int32_t* ctx, int B, int gamma, int n_prompt, int n_prefix,
-                              int32_t* block_ids, int32_t* pos_ids, cudaStream_t s) {
-  const int n = B * (2 * gamma + n_prompt + n_prefix);
+                              int32_t* block_ids, int32_t* pos_ids, cudaStream_t s,
+                              const int32_t* pending) {
+  const int n = B * (2 * gamma + n_prompt + n_prefix + (pending ? 1 : 0));
   if (n == 0) return cudaSuccess;
   pack_block_kernel<<<(n + 255) / 256, 256, 0, s>>>(drafts, prompt, prefix, ctx, B, gamma,
-                                                     n_prompt, n_prefix, block_ids, pos_ids);
+                                                     n_prompt, n_prefix, block_ids, pos_ids,
+                                                     pending);
   return cudaGetLastError();
 }
 
@@ -65,12 +72,15 @@ __global__ void prep_kernel(const uint4* __restrict__ hidden, uint4* __restrict_
   if (tid0 == 0 && tile_counter) *tile_counter = 0u;  // the LM head that follows claims tiles from 0
   if (tid0 == 0 && done_counter) *done_counter = 0u;
   if (pk.block != nullptr) {
-    const int Lb = 2 * pk.gamma + pk.n_prompt + pk.n_prefix;
+    const int lead = pk.pending ? 1 : 0;  // the pending-token block [t, x, prompt, prefix, x]
+    const int Lb = 2 * pk.gamma + pk.n_prompt + pk.n_prefix + lead;
     for (long long idx = tid0; idx < static_cast<long long>(pk.B) * Lb;
          idx += static_cast<long long>(gridDim.x) * blockDim.x) {
-      const int b = static_cast<int>(idx / Lb), j = static_cast<int>(idx % Lb);
+      const int b = static_cast<int>(idx / Lb), jj = static_cast<int>(idx % Lb), j = jj - lead;
       int tok;
-      if (j < pk.gamma)
+      if (j < 0)
+        tok = pk.pending[b];
+      else if (j < pk.gamma)
         tok = pk.drafts[b * pk.gamma + j];
       else if (j < pk.gamma + pk.n_prompt)
         tok = pk.prompt[j - pk.gamma];
@@ -79,7 +89,7 @@ __global__ void prep_kernel(const uint4* __restrict__ hidden, uint4* __restrict_
       else
         tok = pk.drafts[b * pk.gamma + (j - pk.gamma - pk.n_prompt - pk.n_prefix)];
       pk.block[idx] = tok;
-      pk.pos[idx] = pk.ctx[b] + j;
+      pk.pos[idx] = pk.ctx[b] + jj;
     }
   }
   if (hsel == nullptr) return;
@@ -107,7 +117,8 @@ cudaError_t launch_prep(const HeadArgs& a, const HeadPlan& p, void* hsel, const 
   long long work = 0;
   if (pack) {
     pk = *pack;
-    work = static_cast<long long>(pk.B) * (2 * pk.gamma + pk.n_prompt + pk.n_prefix);
+    work = static_cast<long long>(pk.B) *
+           (2 * pk.gamma + pk.n_prompt + pk.n_prefix + (pk.pending ? 1 : 0));
   }
   const int Hv = a.H / 8;  // 8 bf16 per 16-byte vector
   const int Lh = 2 * a.gamma + a.R + 1;
@@ -239,7 +250,7 @@ __global__ void head_finalize_kernel(const float* __restrict__ partials,
     }
     acc.accepted_len[b] = n;
     acc.next_token[b] = s_choice[n];
-    acc.ctx_out[b] = acc.ctx_in[b] + n;
+    acc.ctx_out[b] = acc.ctx_in[b] + n + acc.ctx_extra;
   }
 }
 
@@ -265,7 +276,7 @@ __global__ void accept_kernel(const int32_t* __restrict__ drafts,
                               const int32_t* __restrict__ argmax, int B, int gamma,
                               uint8_t* __restrict__ accept_mask, int32_t* __restrict__ accepted_len,
                               int32_t* __restrict__ next_token, const int32_t* ctx_in,
-                              int32_t* ctx_out) {
+                              int32_t* ctx_out, int ctx_extra) {
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= B) return;
   int n = gamma;
@@ -276,7 +287,7 @@ __global__ void accept_kernel(const int32_t* __restrict__ drafts,
   }
   accepted_len[b] = n;
   next_token[b] = argmax[b * (gamma + 1) + n];
-  ctx_out[b] = ctx_in[b] + n;
+  ctx_out[b] = ctx_in[b] + n + ctx_extra;
 }
 
 // ---------------------------------------------------------------- speculative accept (Alg. 1)
@@ -390,7 +401,7 @@ __global__ void __launch_bounds__(SPEC_THREADS)
   if (tid == 0) {
     a.accepted_len[b] = n;
     a.next_token[b] = s_t >= 0 ? s_t : 0;
-    a.ctx_out[b] = a.ctx_in[b] + n;
+    a.ctx_out[b] = a.ctx_in[b] + n + a.ctx_extra;
   }
 }
 
@@ -399,8 +410,8 @@ cudaError_t launch_accept_speculative(const int32_t* drafts, const float* q, con
                                       int gamma, int V, uint8_t* accept_mask,
                                       int32_t* accepted_len, int32_t* next_token,
                                       const int32_t* ctx_in, int32_t* ctx_out, unsigned* status,
-                                      cudaStream_t s) {
-  AcceptArgs a{accept_mask, accepted_len, next_token, ctx_in, ctx_out, 0, 0.f, 0.f};
+                                      cudaStream_t s, int ctx_extra) {
+  AcceptArgs a{accept_mask, accepted_len, next_token, ctx_in, ctx_out, 0, 0.f, 0.f, ctx_extra};
   accept_speculative_kernel<<<B, SPEC_THREADS, 0, s>>>(drafts, q, r, u, scores, z, gamma, V, a,
                                                        status);
   return cudaGetLastError();
@@ -550,25 +561,27 @@ __global__ void accept_typical_kernel(const int32_t* __restrict__ drafts,
   }
   a.accepted_len[b] = n;
   a.next_token[b] = argmax[b * (gamma + 1) + n];
-  a.ctx_out[b] = a.ctx_in[b] + n;
+  a.ctx_out[b] = a.ctx_in[b] + n + a.ctx_extra;
 }
 
 cudaError_t launch_accept_typical(const int32_t* drafts, const float* scores,
                                   const int32_t* argmax, int B, int gamma, float log_eps,
                                   float log_delta, uint8_t* accept_mask, int32_t* accepted_len,
                                   int32_t* next_token, const int32_t* ctx_in, int32_t* ctx_out,
-                                  cudaStream_t s) {
+                                  cudaStream_t s, int ctx_extra) {
   AcceptArgs a{accept_mask, accepted_len, next_token, ctx_in, ctx_out, RV_ACCEPT_TYPICAL, log_eps,
-               log_delta};
+               log_delta, ctx_extra};
   accept_typical_kernel<<<(B + 127) / 128, 128, 0, s>>>(drafts, scores, argmax, B, gamma, a);
   return cudaGetLastError();
 }
 
 cudaError_t launch_accept(const int32_t* drafts, const int32_t* argmax, int B, int gamma,
                           uint8_t* accept_mask, int32_t* accepted_len, int32_t* next_token,
-                          const int32_t* ctx_in, int32_t* ctx_out, cudaStream_t s) {
+                          const int32_t* ctx_in, int32_t* ctx_out, cudaStream_t s,
+                          int ctx_extra) {
   accept_kernel<<<(B + 127) / 128, 128, 0, s>>>(drafts, argmax, B, gamma, accept_mask,
-                                                accepted_len, next_token, ctx_in, ctx_out);
+                                                accepted_len, next_token, ctx_in, ctx_out,
+                                                ctx_extra);
   return cudaGetLastError();
 }
 

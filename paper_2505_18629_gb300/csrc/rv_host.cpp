@@ -122,7 +122,8 @@ int cuda_fail(rv_handle* h, cudaError_t e, const char* what) {
 }
 
 size_t esize(const rv_config& c) { return c.dtype == RV_DTYPE_BF16 ? 2 : 4; }
-int lb_max(const rv_config& c) { return 2 * c.max_gamma + c.max_template; }
+// Block positions: 2 gamma + R, plus one for the pending-token block.
+int lb_max(const rv_config& c) { return 2 * c.max_gamma + c.max_template + 1; }
 
 HeadPlan head_plan(int B, int gamma, int V, int num_sms, bool tc) {
   HeadPlan p;
@@ -363,6 +364,29 @@ extern "C" RV_API int rv_pack_block(rv_handle* h, const int32_t* draft_ids, cons
     return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument");
   cudaError_t e = launch_pack_block(draft_ids, prompt_ids, prefix_ids, ctx_lens, B, gamma, n_prompt,
                                     n_prefix, block_ids, pos_ids, static_cast<cudaStream_t>(stream));
+  h->launches += 1;
+  return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "pack_block launch");
+}
+
+extern "C" RV_API int rv_pack_block_pending(rv_handle* h, const int32_t* pending_ids,
+                                            const int32_t* draft_ids, const int32_t* prompt_ids,
+                                            const int32_t* prefix_ids, const int32_t* ctx_lens,
+                                            int32_t B, int32_t gamma, int32_t n_prompt,
+                                            int32_t n_prefix, int32_t* block_ids, int32_t* pos_ids,
+                                            void* stream) {
+  if (!h) return RV_ERR_INVALID_ARG;
+  h->err.clear();
+  if (B < 0 || gamma < 0 || n_prompt < 0 || n_prefix < 0)
+    return fail(h, RV_ERR_SHAPE, "negative size");
+  if (B > h->cfg.max_batch || gamma > h->cfg.max_gamma || n_prompt + n_prefix > h->cfg.max_template)
+    return fail(h, RV_ERR_CAPACITY, "B/gamma/template above the handle's maxima");
+  if (B == 0) return RV_OK;
+  if (!pending_ids || !draft_ids || !ctx_lens || !block_ids || !pos_ids ||
+      (n_prompt > 0 && !prompt_ids) || (n_prefix > 0 && !prefix_ids))
+    return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument");
+  cudaError_t e = launch_pack_block(draft_ids, prompt_ids, prefix_ids, ctx_lens, B, gamma, n_prompt,
+                                    n_prefix, block_ids, pos_ids, static_cast<cudaStream_t>(stream),
+                                    pending_ids);
   h->launches += 1;
   return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "pack_block launch");
 }
@@ -674,14 +698,15 @@ struct SpecInputs {
 int sampled_accept_launches(rv_handle* h, const int32_t* draft_ids, const float* u,
                             float temperature, int B, int gamma, int32_t* sampled,
                             uint8_t* accept_mask, int32_t* accepted_len, int32_t* next_token,
-                            const int32_t* ctx_in, int32_t* ctx_out, cudaStream_t s) {
+                            const int32_t* ctx_in, int32_t* ctx_out, cudaStream_t s,
+                            int ctx_extra = 0) {
   ProfScope prof(h, RV_PROF_ACCEPT, s);
   cudaError_t e = launch_sample_fused(h->zbuf, u, B * (gamma + 1), h->cfg.vocab, temperature,
                                       sampled, s);
   h->launches += 1;
   if (e != cudaSuccess) return cuda_fail(h, e, "sampling launch");
   e = launch_accept(draft_ids, sampled, B, gamma, accept_mask, accepted_len, next_token, ctx_in,
-                    ctx_out, s);
+                    ctx_out, s, ctx_extra);
   h->launches += 1;
   return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "accept launch");
 }
@@ -692,9 +717,11 @@ int step_impl(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
               int32_t B, int32_t gamma, int32_t n_prompt, int32_t n_prefix, float alpha,
               int32_t* block_ids, int32_t* pos_ids, void* attn_out, float* scores,
               int32_t* argmax, float* margin, uint8_t* accept_mask, int32_t* accepted_len,
-              int32_t* next_token, int32_t* ctx_out, const SpecInputs* spec, void* stream) {
+              int32_t* next_token, int32_t* ctx_out, const SpecInputs* spec, void* stream,
+              const int32_t* pending = nullptr) {
   if (n_prompt < 0 || n_prefix < 0) return fail(h, RV_ERR_SHAPE, "negative template part");
   const int R = n_prompt + n_prefix;
+  const int lead = pending ? 1 : 0;  // the pending-token block has one more position
   int rc = check_head_args(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin);
   if (rc != RV_OK || B == 0) return rc;
   if (!ctx_in || !accept_mask || !accepted_len || !next_token || !ctx_out)
@@ -704,7 +731,7 @@ int step_impl(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
     return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument for the block packing");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const rv_config& c = h->cfg;
-  const int Lb = 2 * gamma + R;
+  const int Lb = 2 * gamma + R + lead;
   // Small batches: the attention (independent of the LM head) runs on the side
   // stream and shares the SMs with the HBM-bound head; join before returning.
   // Larger batches use the persistent tcgen05 attention, which fills every SM
@@ -723,20 +750,21 @@ int step_impl(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
                            fork ? h->side : s);
   if (rc == RV_OK) {
     PackArgs pk{draft_ids, prompt_ids, prefix_ids, ctx_in, B, gamma, n_prompt, n_prefix, block_ids,
-                pos_ids};
+                pos_ids, pending};
     AcceptArgs ac{accept_mask, accepted_len,       next_token,         ctx_in,
-                  ctx_out,     h->accept_mode,     h->accept_log_eps,  h->accept_log_delta};
+                  ctx_out,     h->accept_mode,     h->accept_log_eps,  h->accept_log_delta,
+                  lead};
     rc = head_impl(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin,
                    do_pack ? &pk : nullptr, spec ? nullptr : &ac, s);
     if (rc == RV_OK && spec && spec->sampled_exact) {
       rc = sampled_accept_launches(h, draft_ids, spec->u, spec->temperature, B, gamma,
                                    spec->sampled, accept_mask, accepted_len, next_token, ctx_in,
-                                   ctx_out, s);
+                                   ctx_out, s, lead);
     } else if (rc == RV_OK && spec) {
       ProfScope prof(h, RV_PROF_ACCEPT, s);
       e = launch_accept_speculative(draft_ids, spec->q, spec->r, spec->u, scores, h->zbuf, B,
                                     gamma, c.vocab, accept_mask, accepted_len, next_token, ctx_in,
-                                    ctx_out, h->ws.status, s);
+                                    ctx_out, h->ws.status, s, lead);
       h->launches += 1;
       if (e != cudaSuccess) rc = cuda_fail(h, e, "speculative accept launch");
     }
@@ -770,6 +798,27 @@ extern "C" RV_API int rv_verify_step(
                    prefix_ids, ctx_in, B, gamma, n_prompt, n_prefix, alpha, block_ids, pos_ids,
                    attn_out, scores, argmax, margin, accept_mask, accepted_len, next_token, ctx_out,
                    nullptr, stream);
+}
+
+extern "C" RV_API int rv_verify_step_pending(
+    rv_handle* h, const void* q, const void* k_blk, const void* v_blk, void* k_cache, void* v_cache,
+    const void* hidden, const void* w_head, const int32_t* pending_ids, const int32_t* draft_ids,
+    const int32_t* prompt_ids, const int32_t* prefix_ids, const int32_t* ctx_in, int32_t B,
+    int32_t gamma, int32_t n_prompt, int32_t n_prefix, float alpha, int32_t* block_ids,
+    int32_t* pos_ids, void* attn_out, float* scores, int32_t* argmax, float* margin,
+    uint8_t* accept_mask, int32_t* accepted_len, int32_t* next_token, int32_t* ctx_out,
+    void* stream) {
+  if (!h) return RV_ERR_INVALID_ARG;
+  h->err.clear();
+  if (h->accept_mode == RV_ACCEPT_SPECULATIVE || h->accept_mode == RV_ACCEPT_SAMPLED)
+    return fail(h, RV_ERR_INVALID_ARG,
+                "the pending-token step runs the exact-match or typical rule of the handle");
+  if (B > 0 && !pending_ids)
+    return fail(h, RV_ERR_INVALID_ARG, "NULL pending token ids");
+  return step_impl(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, prompt_ids,
+                   prefix_ids, ctx_in, B, gamma, n_prompt, n_prefix, alpha, block_ids, pos_ids,
+                   attn_out, scores, argmax, margin, accept_mask, accepted_len, next_token, ctx_out,
+                   nullptr, stream, pending_ids);
 }
 
 extern "C" RV_API int rv_verify_step_speculative(

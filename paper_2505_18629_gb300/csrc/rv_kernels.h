@@ -55,6 +55,7 @@ struct AcceptArgs {
   int32_t* ctx_out;
   int mode;
   float log_eps, log_delta;
+  int ctx_extra = 0;  // 1 with the pending-token block: t stays in the context too
 };
 
 // Outputs of the merge when the LM-head kernel finishes it itself (its last
@@ -86,9 +87,11 @@ struct HeadArgs {
 };
 
 // ---- small kernels (k_small.cu)
+// pending != nullptr: the pending-token block [t, x, prompt, prefix, x] (Lb + 1 positions).
 cudaError_t launch_pack_block(const int32_t* drafts, const int32_t* prompt, const int32_t* prefix,
                               const int32_t* ctx, int B, int gamma, int n_prompt, int n_prefix,
-                              int32_t* block_ids, int32_t* pos_ids, cudaStream_t s);
+                              int32_t* block_ids, int32_t* pos_ids, cudaStream_t s,
+                              const int32_t* pending = nullptr);
 // Optional block packing (Eq. 1) for rv_verify_step: pack.block == nullptr skips it.
 struct PackArgs {
   const int32_t* drafts;
@@ -98,6 +101,7 @@ struct PackArgs {
   int B, gamma, n_prompt, n_prefix;
   int32_t* block;
   int32_t* pos;
+  const int32_t* pending = nullptr;  // [B]: the pending-token block [t, x, prompt, prefix, x]
 };
 // hidden rows of every chunk into hsel [n_chunks * N, H] (bf16), pads zeroed;
 // also packs the block when `pack` is given (one launch for both).
@@ -110,7 +114,8 @@ cudaError_t launch_head_finalize(const HeadArgs& a, const HeadPlan& p, float* sc
                                  cudaStream_t s);
 cudaError_t launch_accept(const int32_t* drafts, const int32_t* argmax, int B, int gamma,
                           uint8_t* accept_mask, int32_t* accepted_len, int32_t* next_token,
-                          const int32_t* ctx_in, int32_t* ctx_out, cudaStream_t s);
+                          const int32_t* ctx_in, int32_t* ctx_out, cudaStream_t s,
+                          int ctx_extra = 0);
 // Speculative-sampling acceptance (Alg. 1) from the head's scores and the
 // fused logits it wrote (z [P][V]), the draft distributions q [B][gamma][V],
 // uniforms r [B][gamma] and u [B].  One CTA per sequence.
@@ -119,7 +124,7 @@ cudaError_t launch_accept_speculative(const int32_t* drafts, const float* q, con
                                       int gamma, int V, uint8_t* accept_mask,
                                       int32_t* accepted_len, int32_t* next_token,
                                       const int32_t* ctx_in, int32_t* ctx_out, unsigned* status,
-                                      cudaStream_t s);
+                                      cudaStream_t s, int ctx_extra = 0);
 // Target tokens at temperature T (Alg. 2 with sampling): for each of the P
 // positions, xhat[p] ~ softmax(z[p] / T) by inverse CDF with u[p]; z [P][V]
 // are the fused logits the head wrote.  One CTA per position.
@@ -130,7 +135,7 @@ cudaError_t launch_accept_typical(const int32_t* drafts, const float* scores,
                                   const int32_t* argmax, int B, int gamma, float log_eps,
                                   float log_delta, uint8_t* accept_mask, int32_t* accepted_len,
                                   int32_t* next_token, const int32_t* ctx_in, int32_t* ctx_out,
-                                  cudaStream_t s);
+                                  cudaStream_t s, int ctx_extra = 0);
 
 // ---- LM head (k_head_tc.cu: bf16 tcgen05; k_head_simt.cu: fp32)
 // Vocab rows per TMA box of the weight: full tiles use HEAD_TILE_ROWS, the

@@ -70,6 +70,9 @@ def _load():
         "rv_last_error": (ctypes.c_char_p, [P]),
         "rv_workspace_bytes": (I, [P, U64P]),
         "rv_pack_block": (I, [P, P, P, P, P, I, I, I, I, P, P, P]),
+        "rv_pack_block_pending": (I, [P, P, P, P, P, P, I, I, I, I, P, P, P]),
+        "rv_verify_step_pending": (I, [P, P, P, P, P, P, P, P, P, P, P, P, P, I, I, I, I, F, P, P, P,
+                                       P, P, P, P, P, P, P, P]),
         "rv_verify_attention": (I, [P, P, P, P, P, P, P, I, I, P, P]),
         "rv_verify_head": (I, [P, P, P, P, I, I, I, F, P, P, P, P]),
         "rv_accept": (I, [P, P, P, I, I, P, P, P, P, P, P]),
@@ -185,6 +188,17 @@ def rv_pack_block(h, draft_ids, prompt_ids, prefix_ids, ctx_lens, block_ids, pos
                                  _ptr(pos_ids), _stream(stream)))
 
 
+def rv_pack_block_pending(h, pending_ids, draft_ids, prompt_ids, prefix_ids, ctx_lens, block_ids,
+                          pos_ids, stream=None):
+    B, gamma = draft_ids.shape
+    n_prompt = 0 if prompt_ids is None else prompt_ids.numel()
+    n_prefix = prefix_ids.shape[1]
+    _check(h, _lib.rv_pack_block_pending(h.ptr, _ptr(pending_ids), _ptr(draft_ids),
+                                         _ptr(prompt_ids), _ptr(prefix_ids), _ptr(ctx_lens), B,
+                                         gamma, n_prompt, n_prefix, _ptr(block_ids), _ptr(pos_ids),
+                                         _stream(stream)))
+
+
 def rv_verify_attention(h, q, k_blk, v_blk, k_cache, v_cache, ctx_lens, out, stream=None):
     B, Lb = q.shape[0], q.shape[1]
     _check(h, _lib.rv_verify_attention(h.ptr, _ptr(q), _ptr(k_blk), _ptr(v_blk), _ptr(k_cache),
@@ -252,6 +266,22 @@ def rv_verify_step(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_i
         n_prompt, n_prefix, float(alpha), _ptr(block_ids), _ptr(pos_ids), _ptr(attn_out),
         _ptr(scores), _ptr(argmax), _ptr(margin), _ptr(accept_mask), _ptr(accepted_len),
         _ptr(next_token), _ptr(ctx_out), _stream(stream)))
+
+
+def rv_verify_step_pending(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, pending_ids,
+                           draft_ids, prompt_ids, prefix_ids, ctx_in, alpha, block_ids, pos_ids,
+                           attn_out, scores, argmax, margin, accept_mask, accepted_len, next_token,
+                           ctx_out, stream=None):
+    """Whole step over the pending-token block [t, x, template, x] (Lb + 1 positions)."""
+    B, gamma = draft_ids.shape
+    n_prompt = 0 if prompt_ids is None else prompt_ids.numel()
+    n_prefix = prefix_ids.shape[1]
+    _check(h, _lib.rv_verify_step_pending(
+        h.ptr, _ptr(q), _ptr(k_blk), _ptr(v_blk), _ptr(k_cache), _ptr(v_cache), _ptr(hidden),
+        _ptr(w_head), _ptr(pending_ids), _ptr(draft_ids), _ptr(prompt_ids), _ptr(prefix_ids),
+        _ptr(ctx_in), B, gamma, n_prompt, n_prefix, float(alpha), _ptr(block_ids), _ptr(pos_ids),
+        _ptr(attn_out), _ptr(scores), _ptr(argmax), _ptr(margin), _ptr(accept_mask),
+        _ptr(accepted_len), _ptr(next_token), _ptr(ctx_out), _stream(stream)))
 
 
 def rv_verify_step_speculative(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids,

@@ -139,16 +139,21 @@ class Report:
 
 
 def compare(inp: synth.VerifyInputs, drafts, alpha, ref: dict, gpu: GpuRun, check_attn=True,
-            seqs=None) -> Report:
-    """Assert GPU == oracle under the tolerances above; `seqs` restricts to sampled sequences."""
+            seqs=None, pending=None) -> Report:
+    """Assert GPU == oracle under the tolerances above; `seqs` restricts to sampled sequences.
+    `pending` [B]: the step ran over the pending-token block [t, x, template, x]."""
     wl = inp.wl
     g = wl.gamma
     seqs = np.arange(wl.B) if seqs is None else np.asarray(seqs)
-    ri = np.arange(len(seqs))  # index into ref arrays (ref computed on `seqs` only)
+    lead = 0 if pending is None else 1
     assert gpu.status == 0, f"device status 0x{gpu.status:x}"
     # ---- pack
-    blk, pos = orc.pack_block(drafts[seqs], inp.prompt_ids, inp.prefix_ids[seqs],
-                              inp.ctx_lens[seqs])
+    if pending is None:
+        blk, pos = orc.pack_block(drafts[seqs], inp.prompt_ids, inp.prefix_ids[seqs],
+                                  inp.ctx_lens[seqs])
+    else:
+        blk, pos = orc.pack_block_pending(pending[seqs], drafts[seqs], inp.prompt_ids,
+                                          inp.prefix_ids[seqs], inp.ctx_lens[seqs])
     np.testing.assert_array_equal(gpu.block_ids[seqs], blk)
     np.testing.assert_array_equal(gpu.pos_ids[seqs], pos)
     # ---- attention + cache append
@@ -157,11 +162,11 @@ def compare(inp: synth.VerifyInputs, drafts, alpha, ref: dict, gpu: GpuRun, chec
         ok, amax, nbad = attn_close(gpu.attn[seqs], ref["attn"])
         assert ok, f"attention: {nbad} elements beyond {ATTN_RTOL} relative (max {amax:.3g})"
         for k, b in enumerate(seqs):
-            c = int(inp.ctx_lens[b])
-            np.testing.assert_array_equal(gpu.k_cache[b, :, :c + wl.Lb],
-                                          _bits_like(ref["k_cache"][k, :, :c + wl.Lb], gpu.k_cache))
-            np.testing.assert_array_equal(gpu.v_cache[b, :, :c + wl.Lb],
-                                          _bits_like(ref["v_cache"][k, :, :c + wl.Lb], gpu.v_cache))
+            c = int(inp.ctx_lens[b]) + wl.Lb + lead
+            np.testing.assert_array_equal(gpu.k_cache[b, :, :c],
+                                          _bits_like(ref["k_cache"][k, :, :c], gpu.k_cache))
+            np.testing.assert_array_equal(gpu.v_cache[b, :, :c],
+                                          _bits_like(ref["v_cache"][k, :, :c], gpu.v_cache))
     # ---- head scores
     sc = gpu.scores[seqs].astype(np.float64)
     lse_err = max(np.abs(sc[..., 0] - ref["lse_orig"]).max(), np.abs(sc[..., 1] - ref["lse_refl"]).max(),
@@ -194,7 +199,7 @@ def compare(inp: synth.VerifyInputs, drafts, alpha, ref: dict, gpu: GpuRun, chec
             assert low[k, :lim].any() or low_choice[k, min(n_ref, g)], \
                 f"sequence {b}: accepted {gpu.accepted_len[b]} vs {n_ref} without a close decision"
             excused += 1
-        assert gpu.ctx_out[b] == inp.ctx_lens[b] + gpu.accepted_len[b]
+        assert gpu.ctx_out[b] == inp.ctx_lens[b] + lead + gpu.accepted_len[b]
         n = int(gpu.accepted_len[b])
         assert gpu.accept_mask[b, :n].all() and (n == g or gpu.accept_mask[b, n] == 0)
         assert gpu.next_token[b] == gpu.argmax[b, n]

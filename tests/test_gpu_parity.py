@@ -667,6 +667,87 @@ def test_sampled_exact_match_kernels_and_8b(gu, name):
         _check_sampled(inp, z, u, drafts, 0.8, gpu)
 
 
+# ------------------------------------------------------------------ pending-token block (NEXT 3)
+
+def _pending_run(gu, wl, alpha=ALPHA, seed=0, check_attn=True):
+    """rv_verify_step_pending against the oracle's verify_step_pending.  The
+    workload's block gets one more position in front (the pending token's
+    query / key / value, drawn like the others); hidden row 0 is the pending
+    token's state, so the head's inputs are the workload's unchanged."""
+    import torch
+    import oracle.rv_oracle as orc
+    from paper_2505_18629_gb300 import rv, synth
+    wl = wl.replace(cmax=wl.ctx[1] + wl.Lb + 1)
+    inp = synth.generate(wl)
+    rng = np.random.default_rng(seed)
+    bf = wl.dtype == "bf16"
+    std = 1.0 if bf else 0.02
+
+    def front(x):
+        row = rng.normal(0, std, x[:, :1].shape).astype(np.float32)
+        return np.concatenate([synth.to_bf16_bits(row) if bf else row, x], axis=1)
+    inp.q, inp.k_blk, inp.v_blk = front(inp.q), front(inp.k_blk), front(inp.v_blk)
+    pending = rng.integers(0, wl.V, wl.B)
+    drafts = gu.oracle_drafts(inp, alpha)
+    ref = orc.verify_step_pending(inp.W, inp.hidden, inp.q, inp.k_blk, inp.v_blk, inp.k_cache,
+                                  inp.v_cache, inp.ctx_lens, pending, drafts, inp.prompt_ids,
+                                  inp.prefix_ids, wl.gamma, wl.R, alpha)
+    ref.pop("z")
+    B, g, Lp = wl.B, wl.gamma, wl.Lb + 1
+    h = gu.make_handle(wl)
+    W, hidden = gu.to_dev(inp.W), gu.to_dev(inp.hidden)
+    q, kb, vb = gu.to_dev(inp.q), gu.to_dev(inp.k_blk), gu.to_dev(inp.v_blk)
+    kc, vc = gu.to_dev(inp.k_cache), gu.to_dev(inp.v_cache)
+    ctx = gu.to_dev(inp.ctx_lens.astype(np.int32))
+    d = gu.to_dev(drafts.astype(np.int32))
+    pend = gu.to_dev(pending.astype(np.int32))
+    prompt = gu.to_dev(inp.prompt_ids.astype(np.int32)) if inp.prompt_ids.size else None
+    prefix = gu.to_dev(inp.prefix_ids.astype(np.int32))
+    i32 = dict(dtype=torch.int32, device="cuda")
+    block, pos = torch.full((B, Lp), -7, **i32), torch.full((B, Lp), -7, **i32)
+    attn = torch.zeros_like(q)
+    scores = torch.full((B, g + 1, rv.RV_NSCORES), float("nan"), device="cuda")
+    argmax = torch.full((B, g + 1), -7, **i32)
+    margin = torch.full((B, g), float("nan"), device="cuda")
+    acc = torch.full((B, g), 7, dtype=torch.uint8, device="cuda")
+    alen, nxt, co = (torch.full((B,), -7, **i32) for _ in range(3))
+    rv.rv_verify_step_pending(h, q, kb, vb, kc, vc, hidden, W, pend, d, prompt, prefix, ctx, alpha,
+                              block, pos, attn, scores, argmax, margin, acc, alen, nxt, co)
+    status = rv.rv_read_status(h)
+    # the separate packing entry point gives the same block
+    block2, pos2 = torch.full((B, Lp), -7, **i32), torch.full((B, Lp), -7, **i32)
+    rv.rv_pack_block_pending(h, pend, d, prompt, prefix, ctx, block2, pos2)
+    torch.cuda.synchronize()
+    h.close()
+    gpu = gu.GpuRun(gu.to_np(attn), gu.to_np(kc), gu.to_np(vc), gu.to_np(scores),
+                    gu.to_np(argmax), gu.to_np(margin), gu.to_np(acc), gu.to_np(alen),
+                    gu.to_np(nxt), gu.to_np(co), gu.to_np(block), gu.to_np(pos), status)
+    np.testing.assert_array_equal(gu.to_np(block2), gpu.block_ids)
+    np.testing.assert_array_equal(gu.to_np(pos2), gpu.pos_ids)
+    rep = gu.compare(inp, drafts, alpha, ref, gpu, check_attn=check_attn, pending=pending)
+    print(f"\n{wl.name} (pending token): {rep}")
+    return rep
+
+
+@pytest.mark.parametrize("kind", ["mma_sync", "tcgen05", "f32"])
+def test_pending_token_step(gu, kind):
+    # the small-batch attention (cluster split-KV), the persistent tcgen05
+    # attention (B * Hkv = 40), and the fp32 path
+    from paper_2505_18629_gb300 import synth
+    if kind == "mma_sync":
+        wl = _wl(seed=100)
+    elif kind == "tcgen05":
+        wl = _wl(B=20, Hq=8, Hkv=2, gamma=3, R=4, V=600, H=256, ctx=(0, 700), seed=101)
+    else:
+        wl = synth.WORKLOADS["tiny"]
+    _pending_run(gu, wl, seed=102)
+
+
+def test_pending_token_step_8b_b16(gu):
+    from paper_2505_18629_gb300 import synth
+    _pending_run(gu, synth.WORKLOADS["llama3-8b-b16"], seed=103)
+
+
 # ------------------------------------------------------------------ full-size workloads
 
 def test_llama3_8b_b1_full(gu):

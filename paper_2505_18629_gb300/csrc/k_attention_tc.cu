@@ -286,11 +286,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         tc_fence_after();
         const uint32_t pcol = tmem + static_cast<uint32_t>(pb * TC_KT);
         const uint32_t vb = base + TC_V_OFF + (v % TC_STAGES) * TC_KV_BYTES;
-#pragma unroll
-        for (int kk = 0; kk < TC_KT / 16; ++kk)
-          tc_mma_bf16_tmem_a(tmem + TC_O_COL, pcol + kk * 8,
-                             sw128_mnmajor_desc(vb + kk * 16 * 128, TC_KV_BYTES / 2, 1024),
-                             idesc_o, (!first || kk > 0) ? 1u : 0u);
+        // K-slice kk of V (16 keys x 128 B rows) starts 16 * 128 bytes after slice kk - 1
+        static_assert(TC_KT == 128, "eight K-slices of 16 keys per tile");
+        tc_mma_stage8_tmem_a_mn(tmem + TC_O_COL, pcol,
+                                sw128_mnmajor_desc(vb, TC_KV_BYTES / 2, 1024), (16 * 128) >> 4,
+                                idesc_o, first ? 0u : 1u);
         tc_commit(o_done(pb));
         tc_commit(kv_empty(v % TC_STAGES));
         return true;
@@ -314,14 +314,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           }
           tc_fence_after();
           const uint32_t kb = base + TC_K_OFF + st * TC_KV_BYTES;
-#pragma unroll
-          for (int kk = 0; kk < TC_D / 16; ++kk) {
-            const uint32_t half = static_cast<uint32_t>(kk >> 2);
-            const uint32_t off = static_cast<uint32_t>((kk & 3) * 32);
-            tc_mma_bf16_tmem_a(tmem + static_cast<uint32_t>((v & 1) * TC_KT), tmem + TC_Q_COL + kk * 8,
-                               sw128_kmajor_desc(kb + half * (TC_KV_BYTES / 2) + off), idesc_s,
-                               kk > 0 ? 1u : 0u);
-          }
+          static_assert(TC_D == 128, "eight K-slices of 16 head dims");
+          tc_mma_stage8_tmem_a(tmem + static_cast<uint32_t>((v & 1) * TC_KT), tmem + TC_Q_COL,
+                               sw128_kmajor_desc(kb), (TC_KV_BYTES / 2) >> 4, idesc_s, 0u);
           tc_commit(s_full(v & 1));
           if (j > 0 && !issue_pv(v - 1, j == 1)) ok = false;
         }

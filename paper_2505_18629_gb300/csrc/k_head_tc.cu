@@ -272,9 +272,8 @@ __global__ void __launch_bounds__(ht_threads(EPI), 1)
           tc_fence_after();
           const uint64_t ad = sw128_kmajor_desc(a_tiles + s * HT_A_BYTES);
           const uint64_t bd = sw128_kmajor_desc(b_tiles + s * b_bytes);
-#pragma unroll
-          for (int kk = 0; kk < HT_BK / 16; ++kk)
-            tc_mma_bf16(d_tmem, ad + 2u * kk, bd + 2u * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
+          static_assert(HT_BK == 64, "one 64-wide box per stage: four MMAs");
+          tc_mma_stage4(d_tmem, ad, bd, idesc, kb != 0 ? 1u : 0u);
           tc_commit(empty_bar(s));
           if (++s == S) {
             s = 0;

@@ -93,13 +93,29 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap
       : "memory");
 }
 
-__device__ __forceinline__ void tc2_mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
-                                             uint32_t idesc, uint32_t accumulate) {
+// The 8 MMAs of one 128-wide K stage of the pair (two 64-wide boxes of A and
+// of B, `a_half` / `b_half` descriptor units apart) from one asm block; only
+// the first reads the accumulate flag (see tc_mma_stage4 for why).
+__device__ __forceinline__ void tc2_mma_stage8(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                               uint32_t a_half, uint32_t b_half, uint32_t idesc,
+                                               uint32_t accumulate) {
   asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      "{\n\t.reg .pred p;\n\t.reg .b64 a<8>, b<8>, ha, hb;\n\t"
+      "setp.ne.b32 p, %6, 0;\n\t"
+      "cvt.u64.u32 ha, %4;\n\tcvt.u64.u32 hb, %5;\n\t"
+      "add.s64 a1, %1, 2;\n\tadd.s64 a2, %1, 4;\n\tadd.s64 a3, %1, 6;\n\t"
+      "add.s64 a4, %1, ha;\n\tadd.s64 a5, a4, 2;\n\tadd.s64 a6, a4, 4;\n\tadd.s64 a7, a4, 6;\n\t"
+      "add.s64 b1, %2, 2;\n\tadd.s64 b2, %2, 4;\n\tadd.s64 b3, %2, 6;\n\t"
+      "add.s64 b4, %2, hb;\n\tadd.s64 b5, b4, 2;\n\tadd.s64 b6, b4, 4;\n\tadd.s64 b7, b4, 6;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], a1, b1, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], a2, b2, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], a3, b3, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], a4, b4, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], a5, b5, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], a6, b6, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], a7, b7, %3, 1;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(a_half), "r"(b_half), "r"(accumulate)
       : "memory");
 }
 
@@ -263,12 +279,7 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
           }
           const uint64_t ad = ad0 + static_cast<uint32_t>(s) * a_step;
           const uint64_t bd = bd0 + static_cast<uint32_t>(s) * b_step;
-#pragma unroll
-          for (int kk = 0; kk < H2_BK / 16; ++kk) {
-            const uint32_t hf = static_cast<uint32_t>(kk >> 2), o = 2u * static_cast<uint32_t>(kk & 3);
-            tc2_mma_bf16(d_tmem, ad + hf * a_hstep + o, bd + hf * b_hstep + o, idesc,
-                         (kb | kk) != 0 ? 1u : 0u);
-          }
+          tc2_mma_stage8(d_tmem, ad, bd, a_hstep, b_hstep, idesc, kb != 0 ? 1u : 0u);
           tc2_commit(empty_bar(s), 3);
           if (++s == S) {
             s = 0;

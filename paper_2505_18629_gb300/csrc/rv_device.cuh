@@ -219,27 +219,77 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32_bmn(uint32_t M, uint32_t N
   return idesc_bf16_f32(M, N) | (1u << 16);
 }
 
-// D[tmem] (+)= A[smem] * B[smem]^T, issued by a single thread.
-__device__ __forceinline__ void tc_mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
-                                            uint32_t idesc, uint32_t accumulate) {
+// The MMAs of one K stage, issued from one asm block.  Each MMA takes K = 16;
+// slice k of a K-major 128-byte-swizzled operand starts 32 bytes (2 in
+// descriptor units) after slice k - 1 within a 64-wide box, and the next box
+// starts `half` descriptor units later.  Only the first MMA reads the
+// accumulate flag `acc`; the others accumulate.  Issued this way, consecutive
+// MMAs into one accumulator overlap in the tensor pipe (one instruction per
+// MMA with a run-time flag each costs up to twice the MMA's own time).
+//
+// 4 MMAs, one 64-wide box: D (+)= A[smem] B[smem]^T, one CTA.
+__device__ __forceinline__ void tc_mma_stage4(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                              uint32_t idesc, uint32_t acc) {
   asm volatile(
-      "{\n\t.reg .pred p;\n\t"
+      "{\n\t.reg .pred p;\n\t.reg .b64 a1, a2, a3, b1, b2, b3;\n\t"
       "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      "add.s64 a1, %1, 2;\n\tadd.s64 a2, %1, 4;\n\tadd.s64 a3, %1, 6;\n\t"
+      "add.s64 b1, %2, 2;\n\tadd.s64 b2, %2, 4;\n\tadd.s64 b3, %2, 6;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], a1, b1, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], a2, b2, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], a3, b3, %3, 1;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(acc)
       : "memory");
 }
 
-// D[tmem] (+)= A[tmem] * B[smem]^T: the A operand (M rows x 16 K elements) is
-// read from tensor memory, one row per lane, two bf16 per 32-bit column.
-__device__ __forceinline__ void tc_mma_bf16_tmem_a(uint32_t d_tmem, uint32_t a_tmem,
-                                                   uint64_t b_desc, uint32_t idesc,
-                                                   uint32_t accumulate) {
+// 8 MMAs, two 64-wide boxes of B (K-major, `b_half` units apart); A (the M x
+// 128 K-slice block, 16 bf16 = 8 columns per slice) read from tensor memory.
+__device__ __forceinline__ void tc_mma_stage8_tmem_a(uint32_t d_tmem, uint32_t a_tmem,
+                                                     uint64_t b_desc, uint32_t b_half,
+                                                     uint32_t idesc, uint32_t acc) {
   asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      "{\n\t.reg .pred p;\n\t.reg .b32 a<8>;\n\t.reg .b64 b<8>, h;\n\t"
+      "setp.ne.b32 p, %5, 0;\n\t"
+      "cvt.u64.u32 h, %4;\n\t"
+      "add.u32 a1, %1, 8;\n\tadd.u32 a2, %1, 16;\n\tadd.u32 a3, %1, 24;\n\t"
+      "add.u32 a4, %1, 32;\n\tadd.u32 a5, %1, 40;\n\tadd.u32 a6, %1, 48;\n\tadd.u32 a7, %1, 56;\n\t"
+      "add.s64 b1, %2, 2;\n\tadd.s64 b2, %2, 4;\n\tadd.s64 b3, %2, 6;\n\t"
+      "add.s64 b4, %2, h;\n\tadd.s64 b5, b4, 2;\n\tadd.s64 b6, b4, 4;\n\tadd.s64 b7, b4, 6;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [a1], b1, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [a2], b2, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [a3], b3, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [a4], b4, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [a5], b5, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [a6], b6, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [a7], b7, %3, 1;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(b_half), "r"(acc)
+      : "memory");
+}
+
+// 8 MMAs with A from tensor memory and an MN-major B whose K-slices are
+// `b_step` descriptor units apart (slice k at b_desc + k * b_step).
+__device__ __forceinline__ void tc_mma_stage8_tmem_a_mn(uint32_t d_tmem, uint32_t a_tmem,
+                                                        uint64_t b_desc, uint32_t b_step,
+                                                        uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t.reg .b32 a<8>;\n\t.reg .b64 b<8>, h;\n\t"
+      "setp.ne.b32 p, %5, 0;\n\t"
+      "cvt.u64.u32 h, %4;\n\t"
+      "add.u32 a1, %1, 8;\n\tadd.u32 a2, %1, 16;\n\tadd.u32 a3, %1, 24;\n\t"
+      "add.u32 a4, %1, 32;\n\tadd.u32 a5, %1, 40;\n\tadd.u32 a6, %1, 48;\n\tadd.u32 a7, %1, 56;\n\t"
+      "add.s64 b1, %2, h;\n\tadd.s64 b2, b1, h;\n\tadd.s64 b3, b2, h;\n\tadd.s64 b4, b3, h;\n\t"
+      "add.s64 b5, b4, h;\n\tadd.s64 b6, b5, h;\n\tadd.s64 b7, b6, h;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [a1], b1, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [a2], b2, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [a3], b3, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [a4], b4, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [a5], b5, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [a6], b6, %3, 1;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [a7], b7, %3, 1;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(b_step), "r"(acc)
       : "memory");
 }
 

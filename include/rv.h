@@ -335,7 +335,12 @@ RV_API int rv_verify_step_sampled(
  * (q, k_blk, v_blk, hidden, draft / prompt / prefix ids, ctx lens) are copied
  * from host memory (pinned memory gives asynchronous copies) into the handle's
  * device staging, rv_verify_step runs, and the per-step results are copied
- * back into host memory before the call returns.  The model state stays on
+ * back into host memory before the call returns.  The ids and lengths travel
+ * in one copy through a pinned buffer of the handle, q / k_blk / v_blk are
+ * copied on the handle's second stream while the hidden states copy on
+ * `stream`, and all results but the attention output come back in one copy
+ * (then scattered into the caller's buffers).  The first call allocates the
+ * two small pinned buffers (RV_ERR_CUDA if that fails).  The model state stays on
  * the device: w_head, k_cache and v_cache are device pointers.  Host buffers
  * have the layouts of rv_verify_step; attn_out_host may be NULL to skip
  * reading the attention output back, block_ids_host NULL to skip the packing.

@@ -56,6 +56,12 @@ struct Workspace {
   uint8_t* st_accept = nullptr;
   int32_t* st_acc_len = nullptr;
   int32_t* st_next = nullptr;
+  // rv_verify_step_host: the small per-step inputs (ids, lengths) and all the
+  // per-step outputs but the attention, each as one contiguous region, so that
+  // each crosses PCIe / C2C in one copy
+  char* st_small_in = nullptr;
+  char* st_small_out = nullptr;
+  size_t small_in_bytes = 0, small_out_bytes = 0;
 };
 
 }  // namespace
@@ -80,6 +86,10 @@ struct rv_handle {
   // LM head on the caller's stream (fork / join through the two events).
   cudaStream_t side = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  cudaEvent_t ev_copy_start = nullptr, ev_copy_done = nullptr;  // rv_verify_step_host
+  // pinned host mirrors of st_small_in / st_small_out (first rv_verify_step_host call)
+  char* pin_in = nullptr;
+  char* pin_out = nullptr;
   unsigned profiling = 0;  // bit mask of the regions being recorded
   ProfRegion prof[RV_PROF_COUNT];
   unsigned long long launches = 0;
@@ -254,6 +264,14 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
   const size_t o_am = take(static_cast<size_t>(Pmax) * 4);
   const size_t o_mg = take(static_cast<size_t>(c.max_batch) * c.max_gamma * 4);
   const size_t o_acc = take(static_cast<size_t>(c.max_batch) * c.max_gamma);
+  // the host-buffer step's contiguous small regions (layout: see small_layout)
+  const size_t small_in = 4 * (static_cast<size_t>(c.max_batch) * (c.max_gamma + 1 + c.max_template) +
+                               c.max_template) + 64;
+  const size_t small_out =
+      4 * (static_cast<size_t>(Pmax) * (RV_NSCORES + 1) + static_cast<size_t>(c.max_batch) *
+                                                              (c.max_gamma + 3 + 2 * Lbm)) +
+      static_cast<size_t>(c.max_batch) * c.max_gamma + 256;
+  const size_t o_sin = take(small_in), o_sout = take(small_out);
   const size_t o_al = take(c.max_batch * 4), o_nt = take(c.max_batch * 4);
   h->attn_tc_ok = bf16 && attn_tc_supported(c.n_q_heads, c.n_kv_heads, c.head_dim) &&
                   attn_tc_smem_max(c.max_batch) <= h->smem_optin;
@@ -295,10 +313,16 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
   h->ws.st_accept = reinterpret_cast<uint8_t*>(b + o_acc);
   h->ws.st_acc_len = reinterpret_cast<int32_t*>(b + o_al);
   h->ws.st_next = reinterpret_cast<int32_t*>(b + o_nt);
+  h->ws.st_small_in = b + o_sin;
+  h->ws.st_small_out = b + o_sout;
+  h->ws.small_in_bytes = small_in;
+  h->ws.small_out_bytes = small_out;
   e = cudaMemset(h->ws.base, 0, off);
   if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_copy_start, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_copy_done, cudaEventDisableTiming);
   if (e == cudaSuccess && bf16) e = attn_configure(&h->attn_max_cluster);
   if (e == cudaSuccess && h->attn_tc_ok) e = attn_tc_configure(attn_tc_smem_max(c.max_batch));
   if (e == cudaSuccess && bf16) e = head_tc_configure(h->smem_optin);
@@ -311,6 +335,8 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
     h->encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
   }
   if (e != cudaSuccess) {
+    if (h->ev_copy_done) cudaEventDestroy(h->ev_copy_done);
+    if (h->ev_copy_start) cudaEventDestroy(h->ev_copy_start);
     if (h->ev_join) cudaEventDestroy(h->ev_join);
     if (h->ev_fork) cudaEventDestroy(h->ev_fork);
     if (h->side) cudaStreamDestroy(h->side);
@@ -329,8 +355,12 @@ extern "C" RV_API int rv_destroy(rv_handle* h) {
     for (auto ev : r.ev) cudaEventDestroy(ev);
   cudaEventDestroy(h->ev_join);
   cudaEventDestroy(h->ev_fork);
+  cudaEventDestroy(h->ev_copy_start);
+  cudaEventDestroy(h->ev_copy_done);
   cudaStreamDestroy(h->side);
   if (h->zbuf) cudaFree(h->zbuf);
+  if (h->pin_in) cudaFreeHost(h->pin_in);
+  if (h->pin_out) cudaFreeHost(h->pin_out);
   cudaFree(h->ws.base);
   delete h;
   return RV_OK;
@@ -682,6 +712,17 @@ extern "C" RV_API int rv_set_acceptance(rv_handle* h, int32_t mode, float eps, f
 
 namespace {
 
+// Whether the step runs the attention on the side stream, beside the LM head
+// (small batches), or before it on the caller's stream (the persistent
+// tcgen05 attention, which fills every SM).
+bool attn_forks(const rv_handle* h, int B, int Lb) {
+  const rv_config& c = h->cfg;
+  return c.dtype != RV_DTYPE_BF16 ||
+         !attn_plan(B, Lb, c.n_q_heads, c.n_kv_heads, c.max_ctx, h->num_sms, true,
+                    h->attn_max_cluster, c.head_dim, h->attn_tc_ok)
+              .tc;
+}
+
 // The whole step; `spec` != nullptr runs a sampling acceptance after the head
 // instead of the rule fused into the head's merge: speculative sampling
 // (Alg. 1; q, r, u) or exact match against sampled target tokens (Alg. 2;
@@ -734,40 +775,47 @@ int step_impl(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
   const int Lb = 2 * gamma + R + lead;
   // Small batches: the attention (independent of the LM head) runs on the side
   // stream and shares the SMs with the HBM-bound head; join before returning.
-  // Larger batches use the persistent tcgen05 attention, which fills every SM
-  // as the head does: there the two run one after the other on `stream`.
-  const bool fork = c.dtype != RV_DTYPE_BF16 ||
-                    !attn_plan(B, Lb, c.n_q_heads, c.n_kv_heads, c.max_ctx, h->num_sms, true,
-                               h->attn_max_cluster, c.head_dim, h->attn_tc_ok)
-                         .tc;
+  // The head goes first (it is the long pole).  Larger batches use the
+  // persistent tcgen05 attention, which fills every SM as the head does:
+  // there the two run one after the other on `stream`.
+  const bool fork = attn_forks(h, B, Lb);
   cudaError_t e = cudaSuccess;
   if (fork) {
     e = cudaEventRecord(h->ev_fork, s);
     if (e == cudaSuccess) e = cudaStreamWaitEvent(h->side, h->ev_fork, 0);
     if (e != cudaSuccess) return cuda_fail(h, e, "stream fork");
   }
-  rc = rv_verify_attention(h, q, k_blk, v_blk, k_cache, v_cache, ctx_in, B, Lb, attn_out,
-                           fork ? h->side : s);
-  if (rc == RV_OK) {
+  auto run_head = [&]() -> int {
     PackArgs pk{draft_ids, prompt_ids, prefix_ids, ctx_in, B, gamma, n_prompt, n_prefix, block_ids,
                 pos_ids, pending};
     AcceptArgs ac{accept_mask, accepted_len,       next_token,         ctx_in,
                   ctx_out,     h->accept_mode,     h->accept_log_eps,  h->accept_log_delta,
                   lead};
-    rc = head_impl(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin,
-                   do_pack ? &pk : nullptr, spec ? nullptr : &ac, s);
-    if (rc == RV_OK && spec && spec->sampled_exact) {
-      rc = sampled_accept_launches(h, draft_ids, spec->u, spec->temperature, B, gamma,
-                                   spec->sampled, accept_mask, accepted_len, next_token, ctx_in,
-                                   ctx_out, s, lead);
-    } else if (rc == RV_OK && spec) {
+    int r = head_impl(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin,
+                      do_pack ? &pk : nullptr, spec ? nullptr : &ac, s);
+    if (r == RV_OK && spec && spec->sampled_exact) {
+      r = sampled_accept_launches(h, draft_ids, spec->u, spec->temperature, B, gamma,
+                                  spec->sampled, accept_mask, accepted_len, next_token, ctx_in,
+                                  ctx_out, s, lead);
+    } else if (r == RV_OK && spec) {
       ProfScope prof(h, RV_PROF_ACCEPT, s);
-      e = launch_accept_speculative(draft_ids, spec->q, spec->r, spec->u, scores, h->zbuf, B,
-                                    gamma, c.vocab, accept_mask, accepted_len, next_token, ctx_in,
-                                    ctx_out, h->ws.status, s, lead);
+      cudaError_t e2 = launch_accept_speculative(draft_ids, spec->q, spec->r, spec->u, scores,
+                                                 h->zbuf, B, gamma, c.vocab, accept_mask,
+                                                 accepted_len, next_token, ctx_in, ctx_out,
+                                                 h->ws.status, s, lead);
       h->launches += 1;
-      if (e != cudaSuccess) rc = cuda_fail(h, e, "speculative accept launch");
+      if (e2 != cudaSuccess) r = cuda_fail(h, e2, "speculative accept launch");
     }
+    return r;
+  };
+  if (fork) {
+    rc = run_head();
+    if (rc == RV_OK)
+      rc = rv_verify_attention(h, q, k_blk, v_blk, k_cache, v_cache, ctx_in, B, Lb, attn_out,
+                               h->side);
+  } else {
+    rc = rv_verify_attention(h, q, k_blk, v_blk, k_cache, v_cache, ctx_in, B, Lb, attn_out, s);
+    if (rc == RV_OK) rc = run_head();
   }
   if (fork) {
     e = cudaEventRecord(h->ev_join, h->side);
@@ -959,46 +1007,87 @@ extern "C" RV_API int rv_verify_step_host(
   const size_t P = static_cast<size_t>(B) * (gamma + 1);
   Workspace& w = h->ws;
   cudaError_t e = cudaSuccess;
-  size_t in_bytes = 0, out_bytes = 0;
-  auto h2d = [&](void* dst, const void* src, size_t n) {
-    if (e == cudaSuccess && n) e = cudaMemcpyAsync(dst, src, n, cudaMemcpyHostToDevice, s);
-    in_bytes += n;
-  };
-  auto d2h = [&](void* dst, const void* src, size_t n) {
-    if (e == cudaSuccess && n) e = cudaMemcpyAsync(dst, src, n, cudaMemcpyDeviceToHost, s);
-    out_bytes += n;
-  };
-  h2d(w.st_q, q_host, nq);
-  h2d(w.st_kb, k_blk_host, nkv);
-  h2d(w.st_vb, v_blk_host, nkv);
-  h2d(w.st_hidden, hidden_host, nh);
-  h2d(w.st_drafts, draft_ids_host, nd);
-  h2d(w.st_ctx_in, ctx_in_host, nc);
-  if (do_pack) {
-    h2d(w.st_prompt, prompt_ids_host, npr);
-    h2d(w.st_prefix, prefix_ids_host, npx);
+  if (!h->pin_in) {  // first call: pinned host mirrors of the small regions
+    e = cudaHostAlloc(reinterpret_cast<void**>(&h->pin_in), w.small_in_bytes, cudaHostAllocDefault);
+    if (e == cudaSuccess)
+      e = cudaHostAlloc(reinterpret_cast<void**>(&h->pin_out), w.small_out_bytes,
+                        cudaHostAllocDefault);
+    if (e != cudaSuccess) {
+      if (h->pin_in) cudaFreeHost(h->pin_in);
+      h->pin_in = h->pin_out = nullptr;
+      return cuda_fail(h, e, "pinned staging cudaHostAlloc");
+    }
   }
+  // Contiguous layouts of this call's small inputs and outputs (16-byte aligned parts).
+  size_t off = 0;
+  auto part = [&off](size_t n) {
+    const size_t o = off;
+    off += (n + 15) & ~size_t(15);
+    return o;
+  };
+  const size_t i_dr = part(nd), i_ci = part(nc), i_pr = part(do_pack ? npr : 0),
+               i_px = part(do_pack ? npx : 0);
+  const size_t in_small = off;
+  off = 0;
+  const size_t o_sc = part(P * RV_NSCORES * 4), o_am = part(P * 4), o_mg = part(nd),
+               o_al = part(nc), o_nt = part(nc), o_co = part(nc), o_bl = part(do_pack ? nbl : 0),
+               o_ps = part(do_pack ? nbl : 0), o_ac = part(static_cast<size_t>(B) * gamma);
+  const size_t out_small = off;
+  char* const hi = h->pin_in;
+  std::memcpy(hi + i_dr, draft_ids_host, nd);
+  std::memcpy(hi + i_ci, ctx_in_host, nc);
+  if (do_pack) {
+    if (npr) std::memcpy(hi + i_pr, prompt_ids_host, npr);
+    if (npx) std::memcpy(hi + i_px, prefix_ids_host, npx);
+  }
+  char* const di = w.st_small_in;
+  char* const dout = w.st_small_out;
+  // q, k_blk, v_blk on the side stream, concurrently with the ids and the
+  // hidden states on `stream`; `stream` waits for them before the step
+  // (the side stream's attention, when it runs there, follows its copies in
+  // stream order; otherwise `stream` waits for them before the step)
+  e = cudaEventRecord(h->ev_copy_start, s);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(h->side, h->ev_copy_start, 0);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(di, hi, in_small, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(w.st_hidden, hidden_host, nh, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(w.st_q, q_host, nq, cudaMemcpyHostToDevice, h->side);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(w.st_kb, k_blk_host, nkv, cudaMemcpyHostToDevice, h->side);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(w.st_vb, v_blk_host, nkv, cudaMemcpyHostToDevice, h->side);
+  if (e == cudaSuccess) e = cudaEventRecord(h->ev_copy_done, h->side);
+  if (e == cudaSuccess && !attn_forks(h, B, Lb)) e = cudaStreamWaitEvent(s, h->ev_copy_done, 0);
   if (e != cudaSuccess) return cuda_fail(h, e, "host->device copy");
+  const size_t in_bytes = in_small + nh + nq + 2 * nkv;
+  auto I32 = [](char* p) { return reinterpret_cast<int32_t*>(p); };
   int rc = rv_verify_step(h, w.st_q, w.st_kb, w.st_vb, k_cache, v_cache, w.st_hidden, w_head,
-                          w.st_drafts, w.st_prompt, w.st_prefix, w.st_ctx_in, B, gamma, n_prompt,
-                          n_prefix, alpha, do_pack ? w.st_block : nullptr, w.st_pos, w.st_attn,
-                          w.st_scores, w.st_argmax, w.st_margin, w.st_accept, w.st_acc_len,
-                          w.st_next, w.st_ctx_out, stream);
+                          I32(di + i_dr), do_pack ? I32(di + i_pr) : nullptr,
+                          do_pack ? I32(di + i_px) : nullptr, I32(di + i_ci), B, gamma, n_prompt,
+                          n_prefix, alpha, do_pack ? I32(dout + o_bl) : nullptr,
+                          do_pack ? I32(dout + o_ps) : nullptr, w.st_attn,
+                          reinterpret_cast<float*>(dout + o_sc), I32(dout + o_am),
+                          reinterpret_cast<float*>(dout + o_mg),
+                          reinterpret_cast<uint8_t*>(dout + o_ac), I32(dout + o_al),
+                          I32(dout + o_nt), I32(dout + o_co), stream);
   if (rc != RV_OK) return rc;
-  if (attn_out_host) d2h(attn_out_host, w.st_attn, nq);
-  if (do_pack) {
-    d2h(block_ids_host, w.st_block, nbl);
-    d2h(pos_ids_host, w.st_pos, nbl);
+  size_t out_bytes = out_small;
+  if (attn_out_host) {
+    e = cudaMemcpyAsync(attn_out_host, w.st_attn, nq, cudaMemcpyDeviceToHost, s);
+    out_bytes += nq;
   }
-  d2h(scores_host, w.st_scores, P * RV_NSCORES * 4);
-  d2h(argmax_host, w.st_argmax, P * 4);
-  d2h(margin_host, w.st_margin, nd);
-  d2h(accept_mask_host, w.st_accept, static_cast<size_t>(B) * gamma);
-  d2h(accepted_len_host, w.st_acc_len, nc);
-  d2h(next_token_host, w.st_next, nc);
-  d2h(ctx_out_host, w.st_ctx_out, nc);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(h->pin_out, dout, out_small, cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return cuda_fail(h, e, "device->host copy");
+  const char* const ho = h->pin_out;
+  std::memcpy(scores_host, ho + o_sc, P * RV_NSCORES * 4);
+  std::memcpy(argmax_host, ho + o_am, P * 4);
+  std::memcpy(margin_host, ho + o_mg, nd);
+  std::memcpy(accept_mask_host, ho + o_ac, static_cast<size_t>(B) * gamma);
+  std::memcpy(accepted_len_host, ho + o_al, nc);
+  std::memcpy(next_token_host, ho + o_nt, nc);
+  std::memcpy(ctx_out_host, ho + o_co, nc);
+  if (do_pack) {
+    std::memcpy(block_ids_host, ho + o_bl, nbl);
+    std::memcpy(pos_ids_host, ho + o_ps, nbl);
+  }
   if (h2d_bytes) *h2d_bytes = in_bytes;
   if (d2h_bytes) *d2h_bytes = out_bytes;
   return RV_OK;

@@ -278,6 +278,24 @@ def test_host_buffer_step_matches_device_step(gu):
     _same_decisions(gu, outs["sc"].numpy(), outs["am"].numpy(), outs["mg"].numpy(), step)
     np.testing.assert_array_equal(outs["al"].numpy(), step.accepted_len)
     np.testing.assert_array_equal(outs["nt"].numpy(), step.next_token)
+    # the prepared form of the same call, twice on the same buffers (the cache
+    # gets the same block appended again at the same positions)
+    for v in outs.values():
+        v.zero_()
+    ins = [host(inp.q), host(inp.k_blk), host(inp.v_blk), kc, vc, host(inp.hidden),
+           gu.to_dev(inp.W), host(drafts.astype(np.int32)), host(inp.prompt_ids),
+           host(inp.prefix_ids), host(inp.ctx_lens)]
+    prep = rv.PreparedStepHost(h, *ins, ALPHA, outs["blk"], outs["pos"], outs["attn"], outs["sc"],
+                               outs["am"], outs["mg"], outs["acc"], outs["al"], outs["nt"],
+                               outs["co"])
+    for _ in range(2):
+        assert prep() == (h2d, d2h)
+        np.testing.assert_array_equal(outs["blk"].numpy(), step.block_ids)
+        np.testing.assert_array_equal(outs["attn"].view(torch.int16).numpy().view(np.uint16),
+                                      step.attn)
+        _same_decisions(gu, outs["sc"].numpy(), outs["am"].numpy(), outs["mg"].numpy(), step)
+        np.testing.assert_array_equal(outs["al"].numpy(), step.accepted_len)
+        np.testing.assert_array_equal(outs["co"].numpy(), step.ctx_out)
     h.close()
 
 

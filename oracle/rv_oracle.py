@@ -22,6 +22,8 @@ Notation follows the paper:
     (Alg. 2, read as "stop at the first mismatch"; see ``exact_match_accept``)
     or with sampled x^_i ~ softmax(z_i / T) (``sampled_exact_accept``)
   * typical acceptance (Alg. 3) and speculative sampling (Alg. 1)
+  * the pre-blended head: z_i = W b_i with b_i the bf16-rounded blend of the
+    two hidden states (``verify_head_preblended``; linearity of Eq. 2)
   * the pending-token block [t, x_1..x_gamma, template, x_1..x_gamma], whose
     first position is the last emitted token (``pack_block_pending``,
     ``verify_step_pending``)
@@ -254,6 +256,65 @@ def verify_head(W, hidden, drafts, gamma: int, R: int, alpha: float):
         logp_refl=o_refl[bi, ii, drafts] - lse_r[:, :gamma],
         argmax=choice, margin=margin, choice_gap=choice_gap, ent_orig=entropy(o), z=z,
     )
+
+
+def round_to_bf16(x) -> np.ndarray:
+    """float32 values rounded to the nearest bf16 (ties to even), as float32.
+
+    bf16 keeps the top 16 bits of a float32: add half of the dropped range,
+    plus one when the kept part is odd (ties to even), then truncate."""
+    u = np.asarray(x, np.float32).view(np.uint32).astype(np.uint64)
+    keep_odd = (u >> 16) & 1
+    r = ((u + 0x7FFF + keep_odd) >> 16) << 16
+    return r.astype(np.uint32).view(np.float32)
+
+
+def preblend_rows(hidden, gamma: int, R: int, alpha: float) -> np.ndarray:
+    """The hidden state whose LM-head product is the fused logit vector.
+
+    The head has no bias, so by linearity z_i = (1-a) W h + a W h' = W b_i
+    with b_i = (1-a) h_{row i-1} + a h_{row i-1+shift_len} (Eq. 2).  A bf16
+    LM head takes b_i in bf16: it is formed in float32 as
+    fl((1-a) h) + fl(a h') (products rounded, then the sum rounded, no fused
+    multiply-add) and then rounded to bf16.  That rounding is the variant's
+    only difference from fusing the two logit vectors.
+    Returns b [B, gamma+1, H] float32 (each value a bf16)."""
+    h = as_f64(hidden).astype(np.float32)
+    a = np.float32(alpha)
+    beta = np.float32(np.float32(1.0) - a)
+    orig_idx = [original_row(i) for i in range(1, gamma + 2)]
+    refl_idx = [reflective_row(i, gamma, R) for i in range(1, gamma + 2)]
+    blend = (beta * h[:, orig_idx, :]).astype(np.float32) + (a * h[:, refl_idx, :]).astype(np.float32)
+    return round_to_bf16(blend.astype(np.float32))
+
+
+def verify_head_preblended(W, hidden, drafts, gamma: int, R: int, alpha: float):
+    """The fused distribution from pre-blended hidden states (a bf16 LM head).
+
+    z_i = W b_i with b_i from ``preblend_rows``; everything derived from z
+    (lse_fused, logp_fused, argmax, margin, choice_gap, z) as in
+    ``verify_head``.  The unfused original / reflective distributions are not
+    formed, so lse_orig, lse_refl, logp_orig, logp_refl and ent_orig are NaN."""
+    drafts = np.asarray(drafts, np.int64)
+    b = preblend_rows(hidden, gamma, R, alpha)
+    B = b.shape[0]
+    z = head_logits(W, b.reshape(B * (gamma + 1), -1)).reshape(B, gamma + 1, -1)
+    lse_z = logsumexp(z)
+    bi = np.arange(B)[:, None]
+    ii = np.arange(gamma)[None, :]
+    zx = z[bi, ii, drafts]
+    z_others = z[:, :gamma, :].copy()
+    z_others[bi, ii, drafts] = -np.inf
+    margin = np.abs(zx - z_others.max(axis=-1))
+    choice = greedy_choice(z)
+    z_rest = z.copy()
+    np.put_along_axis(z_rest, choice[..., None], -np.inf, axis=-1)
+    choice_gap = np.take_along_axis(z, choice[..., None], axis=-1)[..., 0] - z_rest.max(axis=-1)
+    nan1 = np.full((B, gamma + 1), np.nan)
+    nan2 = np.full((B, gamma), np.nan)
+    return dict(lse_orig=nan1, lse_refl=nan1.copy(), lse_fused=lse_z, logp_fused=zx - lse_z[:, :gamma],
+                logp_orig=nan2, logp_refl=nan2.copy(), argmax=choice, margin=margin,
+                choice_gap=choice_gap, ent_orig=nan1.copy(), z=z)
 
 
 # --------------------------------------------------------------------------

@@ -791,3 +791,72 @@ def test_pins_catch_pending_token_at_the_end(monkeypatch):
     monkeypatch.setattr(orc, "pack_block_pending", t_last)
     with pytest.raises(AssertionError):
         test_pending_block_layout_table3()
+
+
+# --------------------------------------------------------------------------
+# Pre-blended head: z_i = W b_i, b_i the bf16-rounded blend (linearity of Eq. 2)
+# --------------------------------------------------------------------------
+
+def test_round_to_bf16_matches_torch():
+    rng = np.random.default_rng(41)
+    x = np.concatenate([rng.normal(0, 1, 20000), rng.normal(0, 1e-30, 100), rng.normal(0, 1e30, 100),
+                        [1.0 + 2 ** -8, 1.0 + 3 * 2 ** -8, -(1.0 + 2 ** -8), 0.0, -0.0, 2 ** -130]])
+    x = x.astype(np.float32)
+    ref = torch.from_numpy(x).to(torch.bfloat16).float().numpy()
+    np.testing.assert_array_equal(orc.round_to_bf16(x), ref)
+
+
+def _preblend_case(seed, B=3, gamma=3, R=2, H=48, V=40):
+    from paper_2505_18629_gb300 import synth
+    rng = np.random.default_rng(seed)
+    W = synth.to_bf16_bits(rng.normal(0, 0.05, (V, H)).astype(np.float32))
+    hidden = synth.to_bf16_bits(rng.normal(0, 1, (B, 2 * gamma + R + 1, H)).astype(np.float32))
+    drafts = rng.integers(0, V, (B, gamma))
+    return W, hidden, drafts
+
+
+@pytest.mark.parametrize("alpha", [0.0, 1.0])
+def test_preblended_head_is_exact_at_alpha_0_and_1(alpha):
+    # the blend is then one of the two bf16 rows itself: no rounding, same logits
+    W, hidden, drafts = _preblend_case(42)
+    a = orc.verify_head_preblended(W, hidden, drafts, 3, 2, alpha)
+    b = orc.verify_head(W, hidden, drafts, 3, 2, alpha)
+    np.testing.assert_array_equal(a["z"], b["z"])
+    np.testing.assert_array_equal(a["argmax"], b["argmax"])
+    np.testing.assert_array_equal(a["lse_fused"], b["lse_fused"])
+    assert np.isnan(a["lse_orig"]).all() and np.isnan(a["ent_orig"]).all()
+
+
+def test_preblended_head_within_the_bf16_rounding_bound():
+    # |W b - z| <= sum_k |W_vk| |b_k - b*_k| with b* the exact blend, and
+    # |b_k - b*_k| <= 2^-8 |b*_k| (float32 steps + one bf16 rounding)
+    W, hidden, drafts = _preblend_case(43)
+    alpha = 0.3
+    a = orc.verify_head_preblended(W, hidden, drafts, 3, 2, alpha)
+    b = orc.verify_head(W, hidden, drafts, 3, 2, alpha)
+    h = orc.as_f64(hidden)
+    oi = [orc.original_row(i) for i in range(1, 5)]
+    ri = [orc.reflective_row(i, 3, 2) for i in range(1, 5)]
+    exact = (1 - alpha) * h[:, oi, :] + alpha * h[:, ri, :]
+    bound = np.einsum("vk,bik->biv", np.abs(orc.as_f64(W)), np.abs(exact)) * 2.0 ** -8
+    diff = np.abs(a["z"] - b["z"])
+    assert (diff <= bound).all()
+    assert diff.max() > 0          # the rounding is real
+    # every blended value is a bf16 number: a float32 whose low 16 bits are zero
+    blend = orc.preblend_rows(hidden, 3, 2, alpha)
+    assert not (np.asarray(blend, np.float32).view(np.uint32) & 0xFFFF).any()
+
+
+def test_pins_catch_unrounded_blend(monkeypatch):
+    real = orc.round_to_bf16
+    monkeypatch.setattr(orc, "round_to_bf16", lambda x: np.asarray(x, np.float32))
+    with pytest.raises(AssertionError):
+        test_preblended_head_within_the_bf16_rounding_bound()
+    monkeypatch.setattr(orc, "round_to_bf16", real)
+
+
+def test_pins_catch_swapped_blend_weights(monkeypatch):
+    real = orc.preblend_rows
+    monkeypatch.setattr(orc, "preblend_rows", lambda h, g, R, a: real(h, g, R, 1.0 - a))
+    with pytest.raises(AssertionError):
+        test_preblended_head_is_exact_at_alpha_0_and_1(0.0)

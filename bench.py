@@ -229,8 +229,8 @@ def run_reference(args, wl):
     print(json.dumps(line), flush=True)
 
 
-def _config(wl, world=1):
-    return {"workload": wl.name, "B": wl.B, "gamma": wl.gamma, "template": wl.R, "Lb": wl.Lb,
+def _config(wl, world=1, head_mode="fused"):
+    return {"workload": wl.name, "head": head_mode, "B": wl.B, "gamma": wl.gamma, "template": wl.R, "Lb": wl.Lb,
             "ctx": list(wl.ctx), "hidden": wl.H, "vocab": wl.V, "q_heads": wl.Hq,
             "kv_heads": wl.Hkv, "head_dim": wl.D, "alpha": ALPHA,
             "parallelism": f"replicas x{world} (independent batches per GPU)",
@@ -249,6 +249,9 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=200)
+    ap.add_argument("--head-mode", default="fused", choices=["fused", "preblended"],
+                    help="fused: both logit vectors fused per vocab row (Eq. 2); preblended: "
+                         "the head on the blended hidden states (one row per position)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -284,6 +287,8 @@ def main():
     prefix = dev_t(inp.prefix_ids.astype(np.int32))
     h = rv.rv_create(wl.H, wl.V, wl.Hq, wl.Hkv, wl.D, B, g, R, wl.capacity,
                      rv.RV_DTYPE_BF16 if wl.dtype == "bf16" else rv.RV_DTYPE_F32)
+    if args.head_mode == "preblended":
+        rv.rv_set_head_mode(h, rv.RV_HEAD_PREBLENDED)
     block = torch.empty((B, Lb), dtype=torch.int32, device=dev)
     pos = torch.empty_like(block)
     attn = torch.empty_like(q)
@@ -400,7 +405,9 @@ def main():
 
     # ---- roofline of the LM-head kernel
     hbm, tf_burst, tf_sus, peak_src = _peaks()
-    n_rows = 2 * (g + 1) * B
+    # hidden rows through the head: original and reflective (fused), or one
+    # blended row per position (pre-blended)
+    n_rows = (1 if args.head_mode == "preblended" else 2) * (g + 1) * B
     head_bytes = wl.V * wl.H * 2 + n_rows * wl.H * 2
     head_flops = 2.0 * n_rows * wl.H * wl.V
     head_avg_s = head_ms * 1e-3 / max(head_n, 1)       # timed region: gather + LM head
@@ -412,7 +419,7 @@ def main():
     bound = "hbm" if t_hbm >= t_tc else "tensor"
     traffic = None
     rec = NCU_TRAFFIC.get(wl.name)
-    if rec and rec.get("src_sha") == _kernel_src_hash():
+    if rec and rec.get("src_sha") == _kernel_src_hash() and args.head_mode == "fused":
         traffic = rec["bytes"]
     if bound == "hbm":
         roof = {"bound": "hbm", "achieved": achieved_gbs, "peak": hbm, "unit": "GB/s",
@@ -442,7 +449,7 @@ def main():
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32",
         "data": "synthetic (seeded Gaussian weights/activations shaped like Llama-3-8B)",
-        "config": _config(wl, world),
+        "config": _config(wl, world, args.head_mode),
         "step_us": ms_step * 1e3,
         "drafts_per_s": units / B / Lb * B * g / (ms_step * 1e-3),
         "step_roofline_frac": step_roof_s / (ms_step * 1e-3),

@@ -83,6 +83,10 @@ extern "C" {
 #define RV_ACCEPT_SPECULATIVE 2 /* speculative sampling with residual resampling (Alg. 1)     */
 #define RV_ACCEPT_SAMPLED 3     /* exact match with target tokens sampled at temperature T (Alg. 2) */
 
+/* LM-head variants (rv_set_head_mode). */
+#define RV_HEAD_FUSED_LOGITS 0  /* o_i and o_{m+i-1} from their own rows, fused (Eq. 2)      */
+#define RV_HEAD_PREBLENDED 1    /* z_i = W b_i from the blended hidden state (linearity)      */
+
 /* Model / capacity description fixed at creation. */
 typedef struct rv_config {
     int32_t hidden;       /* H: hidden size (multiple of 8)                     */
@@ -223,6 +227,23 @@ RV_API int rv_accept_typical(rv_handle* h, const int32_t* draft_ids, const float
  * Errors: RV_ERR_INVALID_ARG for an unknown mode or bad eps / delta,
  * RV_ERR_CUDA if the buffer cannot be allocated. */
 RV_API int rv_set_acceptance(rv_handle* h, int32_t mode, float eps, float delta);
+
+/* LM-head variant of this handle, for every following head call (rv_verify_head
+ * and the steps):
+ *   RV_HEAD_FUSED_LOGITS (the default): the original and reflective logits come
+ *     from their own hidden rows and are fused per vocab row (Eq. 2);
+ *   RV_HEAD_PREBLENDED: the head has no bias, so z_i = (1-a) W h + a W h' =
+ *     W b_i; each sequence's gamma+1 rows b_i = bf16(fl((1-a) h) + fl(a h'))
+ *     (float32 products and sum, then one rounding to bf16) go through the
+ *     head instead of 2(gamma+1) rows.  Half the MMA work and, above 128
+ *     positions, one weight stream where the fused head needs two.  z differs
+ *     from the fused logits by that rounding only (|dz_v| <= 2^-8 sum_k
+ *     |W_vk| |b_k|).  The original / reflective fields of `scores` (lse_orig,
+ *     lse_refl, logp_orig, logp_refl, ent_orig) are NaN, so the typical rule
+ *     (Alg. 3, which needs the entropy) is refused in this mode.
+ * Errors: RV_ERR_INVALID_ARG for an unknown mode or with the typical rule set,
+ * RV_ERR_UNSUPPORTED for an fp32 handle. */
+RV_API int rv_set_head_mode(rv_handle* h, int32_t mode);
 
 /* Speculative sampling with Reflective Verification (Alg. 1), after an
  * rv_verify_head call on this handle in RV_ACCEPT_SPECULATIVE mode (same

@@ -244,6 +244,65 @@ __device__ __forceinline__ void head_tile_pairs8_t(const float (&o)[8], const fl
   __syncwarp();  // the staging rows are reused by the next group
 }
 
+// Variant of head_tile_pairs8_t for the pre-blended head: the accumulator
+// columns are the fused logits z themselves (z = W b, b the blended hidden
+// state), so only the z statistics are kept: lane j < 8 reduces pair g8+j over
+// the warp's 32 rows (max, sum-exp, best z over v != x_i) and folds it into
+// the running statistics; the lane at v == x_i stores z there.
+__device__ __forceinline__ void head_tile_z8_t(const float (&z)[8], int g8, int npairs, int v,
+                                               bool valid, const int* s_drafts, float* warp_stats,
+                                               float* gathered, float* scr, int lane,
+                                               float* zout = nullptr, int V = 0) {
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const int pj = g8 + j;
+    if (zout != nullptr && valid && pj < npairs) zout[static_cast<long long>(pj) * V + v] = z[j];
+    if (valid && v == s_drafts[pj] && pj < npairs) gathered[pj * GATHER_FIELDS + 2] = z[j];
+  }
+  float4* const row = reinterpret_cast<float4*>(scr + lane * HEAD_SCR_STRIDE);
+  const float ninf = NEG_INF;
+  row[0] = valid ? make_float4(z[0], z[1], z[2], z[3]) : make_float4(ninf, ninf, ninf, ninf);
+  row[1] = valid ? make_float4(z[4], z[5], z[6], z[7]) : make_float4(ninf, ninf, ninf, ninf);
+  __syncwarp();
+  if (lane < 8) {
+    const int pj = g8 + lane;
+    float val[32];
+    float m = NEG_INF;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      val[i] = scr[i * HEAD_SCR_STRIDE + lane];
+      m = fmaxf(m, val[i]);
+    }
+    float sum = 0.f;
+    if (m != NEG_INF) {
+      float s2[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int i = 0; i < 32; ++i) s2[i & 3] += __expf(val[i] - m);
+      sum = (s2[0] + s2[1]) + (s2[2] + s2[3]);
+    }
+    if (pj < npairs) {
+      float* st = warp_stats + pj * HEAD_STAT_STRIDE;
+      lse_merge(st[ST_M_Z], st[ST_S_Z], m, sum);
+      const int x = s_drafts[pj];
+      const int v0 = v - lane;  // vocab row of staged row 0
+      float bv = NEG_INF;
+      int bi = INT_MAX;
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        if (val[i] > bv && v0 + i != x) {
+          bv = val[i];
+          bi = v0 + i;
+        }
+      const int si = __float_as_int(st[ST_BEST_I]);
+      if (bv > st[ST_BEST_V] || (bv == st[ST_BEST_V] && bi < si)) {
+        st[ST_BEST_V] = bv;
+        st[ST_BEST_I] = __int_as_float(bi);
+      }
+    }
+  }
+  __syncwarp();  // the staging rows are reused by the next group
+}
+
 // Combine the warps' tables (each `tab` pairs long) into one partial per pair
 // and store it.  `out` points at partials[slot][chunk's first pair].
 __device__ __forceinline__ void head_stats_finish(const float* stats, int nwarps, int tab,
@@ -348,8 +407,10 @@ __device__ __forceinline__ void head_merge_all(const float* partials, const floa
     warp_argmax(bv, bi);
     if (lane == 0) {
       const int b = p / (gamma + 1), i = p % (gamma + 1);
-      const float lse_o = mo + logf(so), lse_r = mr + logf(sr), lse_z = mz + logf(sz);
-      const float ent = logf(so) - to / so;
+      // (the pre-blended head has no separate original / reflective logits)
+      const float lse_o = f.zonly ? nan : mo + logf(so), lse_r = f.zonly ? nan : mr + logf(sr);
+      const float lse_z = mz + logf(sz);
+      const float ent = f.zonly ? nan : logf(so) - to / so;
       float* sc = f.scores + static_cast<long long>(p) * RV_NSCORES;
       sc[RV_SCORE_LSE_ORIG] = lse_o;
       sc[RV_SCORE_LSE_REFL] = lse_r;
@@ -363,8 +424,8 @@ __device__ __forceinline__ void head_merge_all(const float* partials, const floa
         if (x >= 0 && x < V) {
           const float4 gx = __ldcg(reinterpret_cast<const float4*>(gathered) + p);
           lp_z = gx.z - lse_z;
-          lp_o = gx.x - lse_o;
-          lp_r = gx.y - lse_r;
+          lp_o = f.zonly ? nan : gx.x - lse_o;
+          lp_r = f.zonly ? nan : gx.y - lse_r;
           if (gx.z > bv || (gx.z == bv && x < bi)) choice = x;
           f.margin[b * gamma + i] = fabsf(gx.z - bv);
         } else {

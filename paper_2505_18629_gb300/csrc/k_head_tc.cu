@@ -66,26 +66,27 @@ struct HeadTcParams {
   float* gathered;
   float* zout;  // [P][V] fused logits, or null
   unsigned* status;
+  int zonly;    // pre-blended head: column j of the accumulator is z of pair j
 };
 
-static int ht_epi_warps(int N) { return N / 2 <= HT_SMALL_PAIRS ? 4 : 8; }
+static int ht_epi_warps(int pairs) { return pairs <= HT_SMALL_PAIRS ? 4 : 8; }
 
-static size_t ht_fixed_bytes(int N) {
-  // alignment slack + barriers/tile ring/misc + drafts + per-warp statistics (Pcp = N/2 pairs)
-  // + per-warp staging rows of the tile reduction
-  return 1024 + 512 + MAX_PAIRS_PER_CHUNK * 4 +
-         static_cast<size_t>(4) * (N / 2) * HEAD_STAT_STRIDE * 4 + 16 +
-         static_cast<size_t>(ht_epi_warps(N)) * HEAD_SCR_FLOATS * 4;
+static size_t ht_fixed_bytes(int pairs) {
+  // alignment slack + barriers/tile ring/misc + drafts + per-warp statistics (`pairs`
+  // entries per lane quadrant) + per-warp staging rows of the tile reduction
+  return 1024 + 512 + MAX_ZPAIRS_PER_CHUNK * 4 +
+         static_cast<size_t>(4) * pairs * HEAD_STAT_STRIDE * 4 + 16 +
+         static_cast<size_t>(ht_epi_warps(pairs)) * HEAD_SCR_FLOATS * 4;
 }
 
-size_t head_tc_smem_bytes(int N, int stages) {
-  return ht_fixed_bytes(N) + static_cast<size_t>(stages) * (HT_A_BYTES + N * 128);
+size_t head_tc_smem_bytes(int N, int pairs, int stages) {
+  return ht_fixed_bytes(pairs) + static_cast<size_t>(stages) * (HT_A_BYTES + N * 128);
 }
 
-int head_tc_max_stages(int N, size_t smem_limit) {
+int head_tc_max_stages(int N, int pairs, size_t smem_limit) {
   const size_t per = HT_A_BYTES + N * 128;
-  if (smem_limit <= ht_fixed_bytes(N)) return 0;
-  const int s = static_cast<int>((smem_limit - ht_fixed_bytes(N)) / per);
+  if (smem_limit <= ht_fixed_bytes(pairs)) return 0;
+  const int s = static_cast<int>((smem_limit - ht_fixed_bytes(pairs)) / per);
   return s > 12 ? 12 : s;
 }
 
@@ -96,11 +97,11 @@ int head_tc_max_stages(int N, size_t smem_limit) {
 #ifndef RV_HEAD_SMEM_TARGET_KB
 #define RV_HEAD_SMEM_TARGET_KB 151
 #endif
-int head_tc_stages(int N, size_t smem_limit) {
+int head_tc_stages(int N, int pairs, size_t smem_limit) {
   const int per = static_cast<int>(HT_A_BYTES) + N * 128;
-  const int room = RV_HEAD_SMEM_TARGET_KB * 1024 - static_cast<int>(ht_fixed_bytes(N));
+  const int room = RV_HEAD_SMEM_TARGET_KB * 1024 - static_cast<int>(ht_fixed_bytes(pairs));
   const int want = room > 0 ? room / per : 0;
-  return std::max(2, std::min(head_tc_max_stages(N, smem_limit), std::max(4, want)));
+  return std::max(2, std::min(head_tc_max_stages(N, pairs, smem_limit), std::max(4, want)));
 }
 
 template <int EPI>
@@ -135,7 +136,7 @@ __global__ void __launch_bounds__(ht_threads(EPI), 1)
   int2* const tring = reinterpret_cast<int2*>(gbase + (misc - base) + 16);  // (v0, v_end) or v0 < 0
   int* const s_drafts = reinterpret_cast<int*>(gbase + (misc - base) + 16 + 8 * HT_TRING);
   float* const stats =
-      reinterpret_cast<float*>(gbase + (misc - base) + 16 + 8 * HT_TRING + MAX_PAIRS_PER_CHUNK * 4);
+      reinterpret_cast<float*>(gbase + (misc - base) + 16 + 8 * HT_TRING + MAX_ZPAIRS_PER_CHUNK * 4);
   const int tab = p.Pcp;  // pairs per statistics table
   // per-warp staging rows of the transposed tile reduction (16-byte aligned)
   float* const scr_base = reinterpret_cast<float*>(
@@ -173,7 +174,7 @@ __global__ void __launch_bounds__(ht_threads(EPI), 1)
   if (warp == 1) tmem_alloc(smem_u32(tmem_slot), p.tmem_cols);
   if (warp >= 2) {
     const int e = threadIdx.x - 64;
-    for (int j = e; j < MAX_PAIRS_PER_CHUNK; j += EPI * 32)
+    for (int j = e; j < MAX_ZPAIRS_PER_CHUNK; j += EPI * 32)
       s_drafts[j] = (j < npairs) ? pair_draft(p.drafts, pair0 + j, p.gamma) : -1;
     head_stats_init(stats, 4 * tab, e, EPI * 32);
   }
@@ -312,14 +313,22 @@ __global__ void __launch_bounds__(ht_threads(EPI), 1)
       const bool valid = v < tile.y;
       const uint32_t trow =
           tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(slot * p.N);
+      float* const zout = p.zout ? p.zout + static_cast<long long>(pair0) * p.V : nullptr;
       for (int g8 = 8 * half; g8 < npairs; g8 += 8 * (EPI / 4)) {
+        if (p.zonly) {
+          float z[8];
+          tmem_ld8(trow + g8, z);
+          tmem_ld_wait();
+          head_tile_z8_t(z, g8, npairs, v, valid, s_drafts, wstats, gathered,
+                         scr_base + ew * HEAD_SCR_FLOATS, lane, zout, p.V);
+          continue;
+        }
         float o[8], r[8];
         tmem_ld8(trow + g8, o);
         tmem_ld8(trow + p.Pcp + g8, r);
         tmem_ld_wait();
         head_tile_pairs8_t(o, r, g8, npairs, v, valid, p.alpha, s_drafts, wstats, gathered,
-                           scr_base + ew * HEAD_SCR_FLOATS, lane,
-                           p.zout ? p.zout + static_cast<long long>(pair0) * p.V : nullptr, p.V);
+                           scr_base + ew * HEAD_SCR_FLOATS, lane, zout, p.V);
       }
       tc_fence_before();
       __syncwarp();
@@ -406,9 +415,10 @@ cudaError_t launch_head_tc(const HeadArgs& a, const HeadPlan& pl, const HeadTcLa
   p.gathered = a.gathered;
   p.zout = a.zout;
   p.status = a.status;
+  p.zonly = pl.zonly ? 1 : 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(pl.slots, pl.n_chunks, 1);
-  const int epi = ht_epi_warps(pl.N);
+  const int epi = ht_epi_warps(pl.pad_pairs);
   cfg.blockDim = dim3(ht_threads(epi), 1, 1);
   cfg.dynamicSmemBytes = l.smem_bytes;
   cfg.stream = s;

@@ -57,6 +57,7 @@ struct Head2Params {
   float* gathered;
   float* zout;  // [P][V] fused logits, or null
   unsigned* status;
+  int zonly;    // pre-blended head: column j of the accumulator is z of pair j
 };
 
 __device__ __forceinline__ uint32_t cluster_ctarank() {
@@ -147,7 +148,9 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
   const int chunk = blockIdx.y;
   const int slot_id = blockIdx.x;  // partial slot within the chunk
   const int S = p.stages;
-  const uint32_t b_half = static_cast<uint32_t>(p.Pcp) * 128u;  // one 64-wide half of B
+  // this CTA's half of the B rows (the original or the reflective rows; or, for
+  // the pre-blended head, the first or second half of the blended rows)
+  const uint32_t b_half = static_cast<uint32_t>(p.N / 2) * 128u;  // one 64-wide half of B
   const uint32_t b_bytes = 2u * b_half;                          // this CTA's part of B
 
   const uint32_t a_tiles = base;
@@ -163,7 +166,7 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
   volatile int* const abort_flag = reinterpret_cast<volatile int*>(gbase + (misc - base) + 4);
   int* const s_drafts = reinterpret_cast<int*>(gbase + (misc - base) + 16);
   float* const stats =
-      reinterpret_cast<float*>(gbase + (misc - base) + 16 + MAX_PAIRS_PER_CHUNK * 4);
+      reinterpret_cast<float*>(gbase + (misc - base) + 16 + MAX_ZPAIRS_PER_CHUNK * 4);
   const int tab = p.Pcp;
   // per-warp staging rows of the transposed tile reduction (16-byte aligned)
   float* const scr_base = reinterpret_cast<float*>(
@@ -200,7 +203,7 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
   }
   if (warp >= 2) {
     const int e = threadIdx.x - 64;
-    for (int j = e; j < MAX_PAIRS_PER_CHUNK; j += EPI * 32)
+    for (int j = e; j < MAX_ZPAIRS_PER_CHUNK; j += EPI * 32)
       s_drafts[j] = (j < npairs) ? pair_draft(p.drafts, pair0 + j, p.gamma) : -1;
     head_stats_init(stats, 4 * tab, e, EPI * 32);
   }
@@ -229,7 +232,7 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
           }
           if (leader) mbar_arrive_expect_tx(full_bar(s), 2u * (H2_A_BYTES + b_bytes));
           const uint32_t fb = mapa_shared(full_bar(s), leader_rank);
-          const int hrow = chunk * p.N + static_cast<int>(rank) * p.Pcp;
+          const int hrow = chunk * p.N + static_cast<int>(rank) * (p.N / 2);
 #pragma unroll
           for (int hf = 0; hf < 2; ++hf) {
             tma_load_2d_pair(a_tiles + s * H2_A_BYTES + hf * H2_A_HALF, &tm_w, kb * H2_BK + 64 * hf,
@@ -310,14 +313,22 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
       const bool valid = v < p.V;
       const uint32_t trow =
           tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(slot * p.N);
+      float* const zout = p.zout ? p.zout + static_cast<long long>(pair0) * p.V : nullptr;
       for (int g8 = 8 * half; g8 < npairs; g8 += 8 * (EPI / 4)) {
+        if (p.zonly) {
+          float z[8];
+          tmem_ld8(trow + g8, z);
+          tmem_ld_wait();
+          head_tile_z8_t(z, g8, npairs, v, valid, s_drafts, wstats, gathered,
+                         scr_base + ew * HEAD_SCR_FLOATS, lane, zout, p.V);
+          continue;
+        }
         float o[8], r[8];
         tmem_ld8(trow + g8, o);
         tmem_ld8(trow + p.Pcp + g8, r);
         tmem_ld_wait();
         head_tile_pairs8_t(o, r, g8, npairs, v, valid, p.alpha, s_drafts, wstats, gathered,
-                           scr_base + ew * HEAD_SCR_FLOATS, lane,
-                           p.zout ? p.zout + static_cast<long long>(pair0) * p.V : nullptr, p.V);
+                           scr_base + ew * HEAD_SCR_FLOATS, lane, zout, p.V);
       }
       tc_fence_before();
       __syncwarp();
@@ -360,11 +371,11 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
 // ---------------------------------------------------------------- host side
 
 namespace {
-int h2_epi_warps(int N) { return N / 2 <= 32 ? 4 : 8; }
-size_t h2_fixed_bytes(int N) {
-  return 1024 + 256 + 16 + MAX_PAIRS_PER_CHUNK * 4 +
-         static_cast<size_t>(4) * (N / 2) * HEAD_STAT_STRIDE * 4 + 64 + 16 +
-         static_cast<size_t>(h2_epi_warps(N)) * HEAD_SCR_FLOATS * 4;
+int h2_epi_warps(int pairs) { return pairs <= 32 ? 4 : 8; }
+size_t h2_fixed_bytes(int pairs) {
+  return 1024 + 256 + 16 + MAX_ZPAIRS_PER_CHUNK * 4 +
+         static_cast<size_t>(4) * pairs * HEAD_STAT_STRIDE * 4 + 64 + 16 +
+         static_cast<size_t>(h2_epi_warps(pairs)) * HEAD_SCR_FLOATS * 4;
 }
 uint32_t h2_tmem_cols(int N) {
   uint32_t need = static_cast<uint32_t>(2 * N), c = 32;
@@ -373,17 +384,17 @@ uint32_t h2_tmem_cols(int N) {
 }
 }  // namespace
 
-size_t head_tc2_smem_bytes(int N, int stages) {
-  return h2_fixed_bytes(N) + static_cast<size_t>(stages) * (H2_A_BYTES + (N / 2) * 256);
+size_t head_tc2_smem_bytes(int N, int pairs, int stages) {
+  return h2_fixed_bytes(pairs) + static_cast<size_t>(stages) * (H2_A_BYTES + (N / 2) * 256);
 }
 
 #ifndef RV_HEAD2_STAGE_TARGET_KB
 #define RV_HEAD2_STAGE_TARGET_KB 200
 #endif
-int head_tc2_stages(int N, size_t smem_limit) {
+int head_tc2_stages(int N, int pairs, size_t smem_limit) {
   const size_t per = H2_A_BYTES + (N / 2) * 256;
-  if (smem_limit <= h2_fixed_bytes(N)) return 0;
-  const int most = static_cast<int>((smem_limit - h2_fixed_bytes(N)) / per);
+  if (smem_limit <= h2_fixed_bytes(pairs)) return 0;
+  const int most = static_cast<int>((smem_limit - h2_fixed_bytes(pairs)) / per);
   const int want = static_cast<int>((RV_HEAD2_STAGE_TARGET_KB * 1024 + per - 1) / per);
   return std::max(0, std::min(std::min(most, 8), std::max(3, want)));
 }
@@ -404,11 +415,11 @@ cudaError_t head_tc2_configure(size_t smem_bytes) {
   return e != cudaSuccess ? e : head_tc2_configure_one<8>(smem_bytes);
 }
 
-int head_tc2_max_pairs(int N, int stages) {
+int head_tc2_max_pairs(int N, int pairs, int stages) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(2, 1, 1);
-  cfg.blockDim = dim3(h2_threads(h2_epi_warps(N)), 1, 1);
-  cfg.dynamicSmemBytes = head_tc2_smem_bytes(N, stages);
+  cfg.blockDim = dim3(h2_threads(h2_epi_warps(pairs)), 1, 1);
+  cfg.dynamicSmemBytes = head_tc2_smem_bytes(N, pairs, stages);
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
@@ -417,7 +428,7 @@ int head_tc2_max_pairs(int N, int stages) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int n = 0;
-  cudaError_t e = h2_epi_warps(N) == 4
+  cudaError_t e = h2_epi_warps(pairs) == 4
                       ? cudaOccupancyMaxActiveClusters(&n, head_tc2_kernel<4>, &cfg)
                       : cudaOccupancyMaxActiveClusters(&n, head_tc2_kernel<8>, &cfg);
   if (e != cudaSuccess) {
@@ -452,9 +463,10 @@ cudaError_t launch_head_tc2(const HeadArgs& a, const HeadPlan& pl, const HeadTcL
   p.gathered = a.gathered;
   p.zout = a.zout;
   p.status = a.status;
+  p.zonly = pl.zonly ? 1 : 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(pl.slots, pl.n_chunks, 1);
-  const int epi = h2_epi_warps(pl.N);
+  const int epi = h2_epi_warps(pl.pad_pairs);
   cfg.blockDim = dim3(h2_threads(epi), 1, 1);
   cfg.dynamicSmemBytes = l.smem_bytes;
   cfg.stream = s;

@@ -60,11 +60,23 @@ cudaError_t launch_pack_block(const int32_t* drafts, const int32_t* prompt, cons
 // ---------------------------------------------------------------- prep: gather rows (+ pack)
 // hsel row (c*N + j)        = hidden[b][i]            (original row of pair c*Pc+j)
 // hsel row (c*N + Pcp + j)  = hidden[b][gamma+R+i]    (reflective row, shift_len = gamma+R)
+// or, for the pre-blended head (N = Pcp), the blended state of Eq. 2's
+// linearity, each element rounded once to bf16:
+// hsel row (c*N + j)        = bf16(fl((1-a) h[b][i]) + fl(a h[b][gamma+R+i]))
 // padding rows are zero.  One 16-byte vector per thread and step.  When the
 // block is to be packed too, the first B*Lb threads of the grid also do that.
+__device__ __forceinline__ uint32_t blend_bf16x2(uint32_t o, uint32_t r, float alpha, float beta) {
+  const float o0 = __uint_as_float(o << 16), o1 = __uint_as_float(o & 0xFFFF0000u);
+  const float r0 = __uint_as_float(r << 16), r1 = __uint_as_float(r & 0xFFFF0000u);
+  const float b0 = __fadd_rn(__fmul_rn(beta, o0), __fmul_rn(alpha, r0));
+  const float b1 = __fadd_rn(__fmul_rn(beta, o1), __fmul_rn(alpha, r1));
+  return pack_bf16(b0, b1);
+}
+
 __global__ void prep_kernel(const uint4* __restrict__ hidden, uint4* __restrict__ hsel, int P,
                             int gamma, int R, int Lh, int Hv, int Pc, int Pcp, int N, int n_chunks,
-                            const PackArgs pk, unsigned* tile_counter, unsigned* done_counter) {
+                            int zonly, float alpha, float beta, const PackArgs pk,
+                            unsigned* tile_counter, unsigned* done_counter) {
   // The LM-head kernel that follows may start now (programmatic dependent
   // launch); it waits for this grid before it reads anything written here.
   asm volatile("griddepcontrol.launch_dependents;");
@@ -98,14 +110,21 @@ __global__ void prep_kernel(const uint4* __restrict__ hidden, uint4* __restrict_
     const int col = static_cast<int>(idx % Hv);
     const int row = static_cast<int>(idx / Hv);
     const int c = row / N, r = row % N;
-    const bool refl = r >= Pcp;
+    const bool refl = !zonly && r >= Pcp;
     const int j = refl ? r - Pcp : r;
     const int p = c * Pc + j;
     uint4 v = make_uint4(0, 0, 0, 0);
     if (j < Pc && p < P) {
       const int b = p / (gamma + 1), i = p % (gamma + 1);
-      const int hrow = refl ? i + gamma + R : i;
-      v = hidden[(static_cast<long long>(b) * Lh + hrow) * Hv + col];
+      const long long orow = (static_cast<long long>(b) * Lh + i) * Hv + col;
+      const long long rrow = (static_cast<long long>(b) * Lh + i + gamma + R) * Hv + col;
+      if (zonly) {
+        const uint4 o = hidden[orow], rr = hidden[rrow];
+        v = make_uint4(blend_bf16x2(o.x, rr.x, alpha, beta), blend_bf16x2(o.y, rr.y, alpha, beta),
+                       blend_bf16x2(o.z, rr.z, alpha, beta), blend_bf16x2(o.w, rr.w, alpha, beta));
+      } else {
+        v = hidden[refl ? rrow : orow];
+      }
     }
     hsel[idx] = v;
   }
@@ -129,7 +148,8 @@ cudaError_t launch_prep(const HeadArgs& a, const HeadPlan& p, void* hsel, const 
   const int blocks = static_cast<int>(std::min<long long>((work + threads - 1) / threads, 4096));
   prep_kernel<<<blocks, threads, 0, s>>>(static_cast<const uint4*>(a.hidden),
                                          static_cast<uint4*>(hsel), p.P, a.gamma, a.R, Lh, Hv,
-                                         p.pairs_per_chunk, p.pad_pairs, p.N, p.n_chunks, pk,
+                                         p.pairs_per_chunk, p.pad_pairs, p.N, p.n_chunks,
+                                         p.zonly ? 1 : 0, a.alpha, 1.0f - a.alpha, pk,
                                          a.tile_counter, a.done_counter);
   return cudaGetLastError();
 }
@@ -175,7 +195,7 @@ __global__ void head_finalize_kernel(const float* __restrict__ partials,
                                      const int32_t* __restrict__ drafts, int P, int gamma, int V,
                                      int slots, int wpp, float* __restrict__ scores,
                                      int32_t* __restrict__ argmax_out, float* __restrict__ margin,
-                                     unsigned* status, AcceptArgs acc) {
+                                     unsigned* status, AcceptArgs acc, int zonly) {
   __shared__ MergeStat red[FIN_MAX_WARPS];
   __shared__ int s_choice[65];
   __shared__ int s_kept[65];
@@ -204,10 +224,11 @@ __global__ void head_finalize_kernel(const float* __restrict__ partials,
     if (active && sub == 0 && lane == 0) {
       for (int w = 1; w < wpp; ++w) merge_into(st, red[warp + w]);
       const int p = b * npos + i;
-      const float lse_o = st.mo + logf(st.so);
-      const float lse_r = st.mr + logf(st.sr);
+      // (the pre-blended head has no separate original / reflective logits)
+      const float lse_o = zonly ? nan : st.mo + logf(st.so);
+      const float lse_r = zonly ? nan : st.mr + logf(st.sr);
       const float lse_z = st.mz + logf(st.sz);
-      const float ent = logf(st.so) - st.to / st.so;
+      const float ent = zonly ? nan : logf(st.so) - st.to / st.so;
       float* sc = scores + static_cast<long long>(p) * RV_NSCORES;
       sc[RV_SCORE_ENT_ORIG] = ent;
       sc[RV_SCORE_LSE_ORIG] = lse_o;
@@ -222,8 +243,8 @@ __global__ void head_finalize_kernel(const float* __restrict__ partials,
           const float* gx = gathered + static_cast<long long>(p) * GATHER_FIELDS;
           const float zx = gx[2];
           lp_z = zx - lse_z;
-          lp_o = gx[0] - lse_o;
-          lp_r = gx[1] - lse_r;
+          lp_o = zonly ? nan : gx[0] - lse_o;
+          lp_r = zonly ? nan : gx[1] - lse_r;
           if (zx > st.bv || (zx == st.bv && x < st.bi)) choice = x;
           margin[b * gamma + i] = fabsf(zx - st.bv);
         } else {
@@ -267,7 +288,7 @@ cudaError_t launch_head_finalize(const HeadArgs& a, const HeadPlan& p, float* sc
   }
   head_finalize_kernel<<<a.B, warps * 32, 0, s>>>(a.partials, a.gathered, a.drafts, p.P, a.gamma,
                                                   a.V, p.slots, wpp, scores, argmax, margin,
-                                                  a.status, ac);
+                                                  a.status, ac, p.zonly ? 1 : 0);
   return cudaGetLastError();
 }
 

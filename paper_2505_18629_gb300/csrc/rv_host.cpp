@@ -93,7 +93,8 @@ struct rv_handle {
   unsigned profiling = 0;  // bit mask of the regions being recorded
   ProfRegion prof[RV_PROF_COUNT];
   unsigned long long launches = 0;
-  int head_tc_stages_cached_N = -1;
+  int head_mode = RV_HEAD_FUSED_LOGITS;  // rv_set_head_mode
+  int head_tc_stages_cached_N = -1;     // keyed by 2 * N + pre-blended
   int head_tc_stages = 0;
   int head_pair_cached_N = -1;   // pair kernel: stages and co-resident pairs for this N
   int head_pair_stages = 0;
@@ -135,13 +136,17 @@ size_t esize(const rv_config& c) { return c.dtype == RV_DTYPE_BF16 ? 2 : 4; }
 // Block positions: 2 gamma + R, plus one for the pending-token block.
 int lb_max(const rv_config& c) { return 2 * c.max_gamma + c.max_template + 1; }
 
-HeadPlan head_plan(int B, int gamma, int V, int num_sms, bool tc) {
+// zonly: the pre-blended head (one blended row per pair, N = pad_pairs,
+// rounded to 16 for the MMA; up to MAX_ZPAIRS_PER_CHUNK pairs per chunk).
+HeadPlan head_plan(int B, int gamma, int V, int num_sms, bool tc, bool zonly = false) {
   HeadPlan p;
+  p.zonly = zonly;
   p.P = B * (gamma + 1);
-  p.n_chunks = (p.P + MAX_PAIRS_PER_CHUNK - 1) / MAX_PAIRS_PER_CHUNK;
+  const int cap = zonly ? MAX_ZPAIRS_PER_CHUNK : MAX_PAIRS_PER_CHUNK;
+  p.n_chunks = (p.P + cap - 1) / cap;
   p.pairs_per_chunk = (p.P + p.n_chunks - 1) / p.n_chunks;
-  p.pad_pairs = (p.pairs_per_chunk + 7) / 8 * 8;
-  p.N = 2 * p.pad_pairs;
+  p.pad_pairs = zonly ? (p.pairs_per_chunk + 15) / 16 * 16 : (p.pairs_per_chunk + 7) / 8 * 8;
+  p.N = zonly ? p.pad_pairs : 2 * p.pad_pairs;
   p.n_vtiles = (V + 127) / 128;
   p.pair = false;
   if (tc) {  // one persistent CTA per SM; the vocab is split in whole tiles
@@ -245,6 +250,10 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
       const int nch = (P + MAX_PAIRS_PER_CHUNK - 1) / MAX_PAIRS_PER_CHUNK;
       const int pc = (P + nch - 1) / nch;
       hsel_rows = std::max(hsel_rows, static_cast<size_t>(nch) * 2 * ((pc + 7) / 8 * 8));
+      // the pre-blended head's plan: one row per pair, 16-row aligned chunks
+      const int nz = (P + MAX_ZPAIRS_PER_CHUNK - 1) / MAX_ZPAIRS_PER_CHUNK;
+      const int pz = (P + nz - 1) / nz;
+      hsel_rows = std::max(hsel_rows, static_cast<size_t>(nz) * ((pz + 15) / 16 * 16));
     }
   }
   const size_t o_hsel = take(hsel_rows * c.hidden * 2);
@@ -523,17 +532,17 @@ int encode_maps(rv_handle* h, const void* w, const HeadPlan& pl, HeadTcLaunch& l
   if (pl.pair) {
     l.stages = h->head_pair_stages;
     l.unit_rows = HEAD_TILE_ROWS;
-    l.smem_bytes = head_tc2_smem_bytes(pl.N, l.stages);
+    l.smem_bytes = head_tc2_smem_bytes(pl.N, pl.pad_pairs, l.stages);
     return RV_OK;
   }
-  if (h->head_tc_stages_cached_N != pl.N) {
-    h->head_tc_stages = head_tc_stages(pl.N, h->smem_optin);
-    h->head_tc_stages_cached_N = pl.N;
+  if (h->head_tc_stages_cached_N != 2 * pl.N + pl.zonly) {
+    h->head_tc_stages = head_tc_stages(pl.N, pl.pad_pairs, h->smem_optin);
+    h->head_tc_stages_cached_N = 2 * pl.N + pl.zonly;
   }
   l.stages = h->head_tc_stages;
   l.unit_rows = HEAD_TILE_ROWS;  // whole tiles: one TMA box per stage
   if (l.stages < 2) return fail(h, RV_ERR_UNSUPPORTED, "not enough shared memory for the head pipeline");
-  l.smem_bytes = head_tc_smem_bytes(pl.N, l.stages);
+  l.smem_bytes = head_tc_smem_bytes(pl.N, pl.pad_pairs, l.stages);
   return RV_OK;
 }
 
@@ -569,14 +578,16 @@ int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_
              bf16 ? h->ws.status + 16 : nullptr,    // tile counter: its own 64-byte line
              bf16 ? h->ws.status + 32 : nullptr,    // finished-CTA counter
              writes_z(h) ? h->zbuf : nullptr};
-  HeadPlan pl = head_plan(B, gamma, c.vocab, h->num_sms, bf16);
+  HeadPlan pl = head_plan(B, gamma, c.vocab, h->num_sms, bf16,
+                          bf16 && h->head_mode == RV_HEAD_PREBLENDED);
   if (bf16 && pl.N >= HEAD_PAIR_MIN_N) {
     // CTA pairs: as many as fit at once (two CTAs of a pair share a GPC)
-    if (h->head_pair_cached_N != pl.N) {
-      h->head_pair_stages = head_tc2_stages(pl.N, h->smem_optin);
-      h->head_pair_max =
-          h->head_pair_stages >= 2 ? head_tc2_max_pairs(pl.N, h->head_pair_stages) : 0;
-      h->head_pair_cached_N = pl.N;
+    if (h->head_pair_cached_N != 2 * pl.N + pl.zonly) {
+      h->head_pair_stages = head_tc2_stages(pl.N, pl.pad_pairs, h->smem_optin);
+      h->head_pair_max = h->head_pair_stages >= 2
+                             ? head_tc2_max_pairs(pl.N, pl.pad_pairs, h->head_pair_stages)
+                             : 0;
+      h->head_pair_cached_N = 2 * pl.N + pl.zonly;
     }
     const int n_pt = (c.vocab + 255) / 256;
     const int pairs = std::min({h->num_sms / 2 / pl.n_chunks, h->head_pair_max / pl.n_chunks, n_pt});
@@ -599,7 +610,7 @@ int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_
   }
   // Small pair counts: the head kernel's last CTA finishes the merge itself.
   const bool fused = bf16 && pl.P <= HEAD_FUSED_FINAL_MAX_PAIRS;
-  HeadFinal fin{scores, argmax, margin, acc ? *acc : AcceptArgs{}};
+  HeadFinal fin{scores, argmax, margin, acc ? *acc : AcceptArgs{}, pl.zonly ? 1 : 0};
   {
     ProfScope prof(h, RV_PROF_HEAD_GEMM, s);
     e = !bf16    ? launch_head_simt(a, pl, s)
@@ -700,11 +711,33 @@ extern "C" RV_API int rv_set_acceptance(rv_handle* h, int32_t mode, float eps, f
     return RV_OK;
   }
   if (mode != RV_ACCEPT_TYPICAL) return fail(h, RV_ERR_INVALID_ARG, "unknown acceptance mode %d", mode);
+  if (h->head_mode == RV_HEAD_PREBLENDED)
+    return fail(h, RV_ERR_INVALID_ARG,
+                "typical acceptance needs the original distribution's entropy, which the "
+                "pre-blended head does not form");
   if (!(eps > 0.f) || !(delta > 0.f) || !std::isfinite(eps) || !std::isfinite(delta))
     return fail(h, RV_ERR_INVALID_ARG, "typical acceptance needs finite eps > 0 and delta > 0");
   h->accept_mode = mode;
   h->accept_log_eps = logf(eps);
   h->accept_log_delta = logf(delta);
+  return RV_OK;
+}
+
+extern "C" RV_API int rv_set_head_mode(rv_handle* h, int32_t mode) {
+  if (!h) return RV_ERR_INVALID_ARG;
+  h->err.clear();
+  if (mode == RV_HEAD_FUSED_LOGITS) {
+    h->head_mode = mode;
+    return RV_OK;
+  }
+  if (mode != RV_HEAD_PREBLENDED) return fail(h, RV_ERR_INVALID_ARG, "unknown head mode %d", mode);
+  if (h->cfg.dtype != RV_DTYPE_BF16)
+    return fail(h, RV_ERR_UNSUPPORTED, "the pre-blended head is the bf16 LM head's variant");
+  if (h->accept_mode == RV_ACCEPT_TYPICAL)
+    return fail(h, RV_ERR_INVALID_ARG,
+                "typical acceptance needs the original distribution's entropy, which the "
+                "pre-blended head does not form");
+  h->head_mode = mode;
   return RV_OK;
 }
 

@@ -32,16 +32,20 @@ constexpr int GATHER_FIELDS = 4;  // o_i[x_i], o'_i[x_i], z_i[x_i], unused
 // [c*pairs_per_chunk, ...).  Its gathered hidden rows form a block of
 // 2*pad_pairs rows: original rows first, reflective rows after pad_pairs.
 constexpr int MAX_PAIRS_PER_CHUNK = 128;
+// The pre-blended head gathers one row per pair (the blended hidden state), so
+// its chunks take up to 256 pairs (pad_pairs rows, one accumulator column each).
+constexpr int MAX_ZPAIRS_PER_CHUNK = 256;
 
 struct HeadPlan {
   int P;               // total pairs B*(gamma+1)
   int n_chunks;
   int pairs_per_chunk; // Pc
-  int pad_pairs;       // Pcp = round_up(Pc, 8)
-  int N;               // 2*Pcp: MMA N (columns of the TMEM accumulator)
+  int pad_pairs;       // Pcp = round_up(Pc, 8) (pre-blended: round_up(Pc, 16))
+  int N;               // MMA N (columns of the TMEM accumulator): 2*Pcp (pre-blended: Pcp)
   int n_vtiles;        // ceil(V / 128)
   int slots;           // CTAs per chunk (= partial slots)
   bool pair;           // CTA-pair kernel (k_head_tc2.cu): slots = 2 * pairs
+  bool zonly = false;  // pre-blended head: one blended row per pair, z statistics only
 };
 
 // Optional acceptance fused into the head merge (rv_verify_step).
@@ -65,6 +69,7 @@ struct HeadFinal {
   int32_t* argmax;
   float* margin;
   AcceptArgs acc;  // acc.accepted_len == nullptr: no acceptance
+  int zonly = 0;   // pre-blended head: the original / reflective fields are NaN
 };
 // Largest pair count whose merge the head kernel's last CTA finishes itself.
 #ifndef RV_HEAD_FUSED_FINAL_MAX_PAIRS
@@ -151,9 +156,10 @@ struct HeadTcLaunch {
   int unit_rows;       // vocab split granularity across CTAs (multiple of 16, <= 128)
   size_t smem_bytes;
 };
-size_t head_tc_smem_bytes(int N, int stages);
-int head_tc_max_stages(int N, size_t smem_limit);
-int head_tc_stages(int N, size_t smem_limit);  // the depth the launcher uses
+// `pairs` = pad_pairs of the plan (the statistics tables' length)
+size_t head_tc_smem_bytes(int N, int pairs, int stages);
+int head_tc_max_stages(int N, int pairs, size_t smem_limit);
+int head_tc_stages(int N, int pairs, size_t smem_limit);  // the depth the launcher uses
 cudaError_t head_tc_configure(size_t smem_bytes);  // cudaFuncSetAttribute
 // fin != nullptr: the kernel's last CTA merges the statistics and writes the
 // outputs (P <= HEAD_FUSED_FINAL_MAX_PAIRS).  The launch uses programmatic
@@ -169,10 +175,10 @@ cudaError_t launch_head_simt(const HeadArgs& a, const HeadPlan& p, cudaStream_t 
 #define RV_HEAD_PAIR_MIN_N 96
 #endif
 constexpr int HEAD_PAIR_MIN_N = RV_HEAD_PAIR_MIN_N;  // N from which pairs are used
-size_t head_tc2_smem_bytes(int N, int stages);
-int head_tc2_stages(int N, size_t smem_limit);
+size_t head_tc2_smem_bytes(int N, int pairs, int stages);
+int head_tc2_stages(int N, int pairs, size_t smem_limit);
 cudaError_t head_tc2_configure(size_t smem_bytes);
-int head_tc2_max_pairs(int N, int stages);  // co-resident CTA pairs (occupancy query)
+int head_tc2_max_pairs(int N, int pairs, int stages);  // co-resident CTA pairs (occupancy query)
 cudaError_t launch_head_tc2(const HeadArgs& a, const HeadPlan& p, const HeadTcLaunch& l,
                             const HeadFinal* fin, cudaStream_t s);
 

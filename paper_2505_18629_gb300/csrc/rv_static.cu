@@ -148,9 +148,9 @@ extern "C" RV_API int rv_verify_head_static(const void* hidden, const void* w_he
              status, reinterpret_cast<unsigned*>(s + ST_OFF_STATUS + 64),
              reinterpret_cast<unsigned*>(s + ST_OFF_STATUS + 128)};
   HeadTcLaunch l;
-  l.stages = head_tc_stages(pl.N, d->smem_optin);
+  l.stages = head_tc_stages(pl.N, pl.pad_pairs, d->smem_optin);
   l.unit_rows = HEAD_TILE_ROWS;
-  l.smem_bytes = head_tc_smem_bytes(pl.N, l.stages);
+  l.smem_bytes = head_tc_smem_bytes(pl.N, pl.pad_pairs, l.stages);
   if (l.stages < 2) return RV_ERR_UNSUPPORTED;
   if (!encode_2d(d->encode, &l.tm_w, w_head, hidden_size, vocab, 64, HEAD_TILE_ROWS) ||
       !encode_2d(d->encode, &l.tm_w16, w_head, hidden_size, vocab, 64, HEAD_W_BOX_ROWS) ||

@@ -38,6 +38,7 @@ RV_SCORE_LOGP_FUSED, RV_SCORE_LOGP_ORIG, RV_SCORE_LOGP_REFL = 3, 4, 5
 RV_SCORE_ENT_ORIG = 6
 
 RV_ACCEPT_EXACT, RV_ACCEPT_TYPICAL, RV_ACCEPT_SPECULATIVE, RV_ACCEPT_SAMPLED = 0, 1, 2, 3
+RV_HEAD_FUSED_LOGITS, RV_HEAD_PREBLENDED = 0, 1
 
 RV_PROF_ATTENTION, RV_PROF_HEAD_GEMM, RV_PROF_HEAD, RV_PROF_ACCEPT = 0, 1, 2, 3
 
@@ -78,6 +79,7 @@ def _load():
         "rv_accept": (I, [P, P, P, I, I, P, P, P, P, P, P]),
         "rv_accept_typical": (I, [P, P, P, P, I, I, F, F, P, P, P, P, P, P]),
         "rv_set_acceptance": (I, [P, I, F, F]),
+        "rv_set_head_mode": (I, [P, I]),
         "rv_accept_speculative": (I, [P, P, P, P, P, P, I, I, P, P, P, P, P, P]),
         "rv_verify_step_speculative": (I, [P, P, P, P, P, P, P, P, P, P, P, P, I, I, I, I, F, P, P,
                                            P, P, P, P, P, P, P, P, P, P, P, P]),
@@ -247,6 +249,10 @@ def rv_accept_sampled(h, draft_ids, u_uniform, temperature, sampled, accept_mask
                                      B, gamma, _ptr(sampled), _ptr(accept_mask),
                                      _ptr(accepted_len), _ptr(next_token), _ptr(ctx_in),
                                      _ptr(ctx_out), _stream(stream)))
+
+
+def rv_set_head_mode(h, mode):
+    _check(h, _lib.rv_set_head_mode(h.ptr, int(mode)))
 
 
 def rv_set_acceptance(h, mode, eps=0.0, delta=0.0):

@@ -138,6 +138,16 @@ class Report:
     attn_max_rel: float
 
 
+def _err(gpu_vals: np.ndarray, ref_vals: np.ndarray) -> float:
+    """Largest absolute difference; a field the oracle leaves NaN (the
+    pre-blended head's original / reflective statistics) must be NaN on the
+    GPU too and contributes 0."""
+    if np.isnan(ref_vals).all():
+        assert np.isnan(gpu_vals).all(), "a field without a value is not NaN"
+        return 0.0
+    return float(np.abs(gpu_vals - ref_vals).max())
+
+
 def compare(inp: synth.VerifyInputs, drafts, alpha, ref: dict, gpu: GpuRun, check_attn=True,
             seqs=None, pending=None) -> Report:
     """Assert GPU == oracle under the tolerances above; `seqs` restricts to sampled sequences.
@@ -169,15 +179,14 @@ def compare(inp: synth.VerifyInputs, drafts, alpha, ref: dict, gpu: GpuRun, chec
                                           _bits_like(ref["v_cache"][k, :, :c], gpu.v_cache))
     # ---- head scores
     sc = gpu.scores[seqs].astype(np.float64)
-    lse_err = max(np.abs(sc[..., 0] - ref["lse_orig"]).max(), np.abs(sc[..., 1] - ref["lse_refl"]).max(),
-                  np.abs(sc[..., 2] - ref["lse_fused"]).max())
+    lse_err = max(_err(sc[..., 0], ref["lse_orig"]), _err(sc[..., 1], ref["lse_refl"]),
+                  _err(sc[..., 2], ref["lse_fused"]))
     assert lse_err <= LOGP_ATOL, f"lse error {lse_err}"
-    logp_err = max(np.abs(sc[:, :g, 3] - ref["logp_fused"]).max(),
-                   np.abs(sc[:, :g, 4] - ref["logp_orig"]).max(),
-                   np.abs(sc[:, :g, 5] - ref["logp_refl"]).max())
+    logp_err = max(_err(sc[:, :g, 3], ref["logp_fused"]), _err(sc[:, :g, 4], ref["logp_orig"]),
+                   _err(sc[:, :g, 5], ref["logp_refl"]))
     assert logp_err <= LOGP_ATOL, f"log-prob error {logp_err}"
     assert np.isnan(sc[:, g, 3:6]).all()
-    ent_err = np.abs(sc[..., 6] - ref["ent_orig"]).max()
+    ent_err = _err(sc[..., 6], ref["ent_orig"])
     assert ent_err <= LOGP_ATOL, f"entropy error {ent_err}"
     m_err = np.abs(gpu.margin[seqs].astype(np.float64) - ref["margin"]).max()
     assert m_err <= LOGP_ATOL, f"margin error {m_err}"
@@ -254,11 +263,14 @@ def _bits_like(ref_f64: np.ndarray, like: np.ndarray) -> np.ndarray:
     return ref_f64.astype(like.dtype)
 
 
-def oracle_step(inp: synth.VerifyInputs, drafts, alpha, seqs=None, with_attn=True):
-    """Oracle verify step on all or on a sample of the sequences."""
+def oracle_step(inp: synth.VerifyInputs, drafts, alpha, seqs=None, with_attn=True,
+                preblended=False):
+    """Oracle verify step on all or on a sample of the sequences
+    (`preblended`: the head on the blended hidden states)."""
     wl = inp.wl
     seqs = np.arange(wl.B) if seqs is None else np.asarray(seqs)
-    head = orc.verify_head(inp.W, inp.hidden[seqs], drafts[seqs], wl.gamma, wl.R, alpha)
+    head_fn = orc.verify_head_preblended if preblended else orc.verify_head
+    head = head_fn(inp.W, inp.hidden[seqs], drafts[seqs], wl.gamma, wl.R, alpha)
     acc, n, t = orc.exact_match_accept(drafts[seqs], head["argmax"])
     ref = dict(head, accept_mask=acc, accepted_len=n, next_token=t)
     ref.pop("z")

@@ -30,8 +30,9 @@ def _wl(**kw):
     return base.replace(**kw)
 
 
-def _check(gu, wl, alpha=ALPHA, ctx=None, seqs=None, check_attn=True, drafts=None):
-    from paper_2505_18629_gb300 import synth
+def _check(gu, wl, alpha=ALPHA, ctx=None, seqs=None, check_attn=True, drafts=None,
+           preblended=False):
+    from paper_2505_18629_gb300 import rv, synth
     if ctx is not None:
         wl = wl.replace(ctx=(min(ctx), max(ctx)))
     inp = synth.generate(wl)
@@ -39,8 +40,15 @@ def _check(gu, wl, alpha=ALPHA, ctx=None, seqs=None, check_attn=True, drafts=Non
         inp.ctx_lens[:] = np.asarray(ctx, np.int32)
     if drafts is None:
         drafts = gu.oracle_drafts(inp, alpha, seqs=seqs)
-    gpu = gu.run_gpu(inp, drafts, alpha)
-    ref = gu.oracle_step(inp, drafts, alpha, seqs=seqs, with_attn=check_attn)
+    h = None
+    if preblended:
+        h = gu.make_handle(wl)
+        rv.rv_set_head_mode(h, rv.RV_HEAD_PREBLENDED)
+    gpu = gu.run_gpu(inp, drafts, alpha, h=h)
+    if h is not None:
+        h.close()
+    ref = gu.oracle_step(inp, drafts, alpha, seqs=seqs, with_attn=check_attn,
+                         preblended=preblended)
     rep = gu.compare(inp, drafts, alpha, ref, gpu, check_attn=check_attn, seqs=seqs)
     print(f"\n{wl.name}: {rep}")
     return inp, drafts, gpu, ref, rep
@@ -552,14 +560,15 @@ def test_speculative_sampling_pairs_and_8b(gu):
 
 # ------------------------------------------------------------------ sampled exact match (Alg. 2, temperature T)
 
-def _sampled_inputs(inp, alpha, T, seed, keep=0.7):
+def _sampled_inputs(inp, alpha, T, seed, keep=0.7, preblended=False):
     """The oracle's fused logits z, uniforms u [B, gamma+1], and drafts that
     equal the oracle's sampled target token with probability `keep`."""
     import oracle.rv_oracle as orc
     wl = inp.wl
     rng = np.random.default_rng(seed)
     dummy = np.zeros((wl.B, wl.gamma), np.int64)
-    z = orc.verify_head(inp.W, inp.hidden, dummy, wl.gamma, wl.R, alpha)["z"]
+    head_fn = orc.verify_head_preblended if preblended else orc.verify_head
+    z = head_fn(inp.W, inp.hidden, dummy, wl.gamma, wl.R, alpha)["z"]
     u = rng.uniform(0, 1, (wl.B, wl.gamma + 1)).astype(np.float32)
     _, _, _, xhat, _ = orc.sampled_exact_accept(dummy, z, T, u.astype(np.float64))
     alt = rng.integers(0, wl.V, (wl.B, wl.gamma))
@@ -567,13 +576,15 @@ def _sampled_inputs(inp, alpha, T, seed, keep=0.7):
     return z, u, drafts.astype(np.int64)
 
 
-def _run_sampled(gu, inp, drafts, alpha, T, u, separate=False):
+def _run_sampled(gu, inp, drafts, alpha, T, u, separate=False, preblended=False):
     import torch
     from paper_2505_18629_gb300 import rv
     wl = inp.wl
     B, g = wl.B, wl.gamma
     h = gu.make_handle(wl)
     rv.rv_set_acceptance(h, rv.RV_ACCEPT_SAMPLED)
+    if preblended:
+        rv.rv_set_head_mode(h, rv.RV_HEAD_PREBLENDED)
     du = gu.to_dev(u)
     d = gu.to_dev(drafts.astype(np.int32))
     ctx = gu.to_dev(inp.ctx_lens.astype(np.int32))
@@ -764,6 +775,90 @@ def test_pending_token_step(gu, kind):
 def test_pending_token_step_8b_b16(gu):
     from paper_2505_18629_gb300 import synth
     _pending_run(gu, synth.WORKLOADS["llama3-8b-b16"], seed=103)
+
+
+# ------------------------------------------------------------------ pre-blended head (NEXT 3)
+
+@pytest.mark.parametrize("shape", ["ragged", "one-pair", "pairs-144", "two-chunks"])
+def test_preblended_head(gu, shape):
+    # the head on b_i = bf16(fl((1-a) h) + fl(a h')) against the oracle's
+    # verify_head_preblended (whose blend is that rounding, so the tolerance is
+    # the plain head's): N = 16 on single CTAs; 144 pairs in one chunk on CTA
+    # pairs (above the 128 pairs of a two-distribution chunk); 288 pairs in two
+    # chunks of 144 with several vocab tiles per CTA pair
+    if shape == "ragged":
+        _check(gu, _wl(seed=110), ctx=[0, 77, 300], preblended=True)
+    elif shape == "one-pair":
+        _check(gu, _wl(B=1, gamma=2, R=4, seed=111), ctx=[5], preblended=True)
+    elif shape == "pairs-144":
+        _check(gu, _wl(B=16, gamma=8, R=3, V=60000, H=320, ctx=(1, 30), seed=112),
+               check_attn=False, preblended=True)
+    else:
+        _check(gu, _wl(B=32, gamma=8, R=2, V=5000, H=192, ctx=(1, 20), seed=113),
+               check_attn=False, preblended=True)
+
+
+def test_preblended_head_differs_from_fused_by_the_blend_rounding(gu):
+    # same inputs through both head modes: the fused-logit statistics agree
+    # within the bound of the blend's bf16 rounding, and not bit for bit
+    from paper_2505_18629_gb300 import rv, synth
+    wl = _wl(B=4, gamma=5, V=3000, seed=114)
+    inp = synth.generate(wl)
+    drafts = gu.oracle_drafts(inp, ALPHA)
+    fused = gu.run_gpu(inp, drafts, ALPHA)
+    h = gu.make_handle(wl)
+    rv.rv_set_head_mode(h, rv.RV_HEAD_PREBLENDED)
+    pre = gu.run_gpu(inp, drafts, ALPHA, h=h)
+    h.close()
+    import oracle.rv_oracle as orc
+    d = np.abs(pre.scores[..., 2].astype(np.float64) - fused.scores[..., 2])
+    # |dz_v| <= u sum_k |W_vk| |b_k| with u = 2^-8, the bf16 unit roundoff, and
+    # |d lse| <= max_v |dz_v|; 1e-4 for the two heads' float32 accumulations
+    b = orc.preblend_rows(inp.hidden, wl.gamma, wl.R, ALPHA).astype(np.float64)
+    bound = 2.0 ** -8 * (np.abs(b) @ np.abs(orc.as_f64(inp.W)).T).max(axis=-1) + 1e-4
+    assert (d <= bound).all()
+    assert d.max() > 0
+    assert np.isnan(pre.scores[..., [0, 1, 6]]).all()
+    assert np.isfinite(fused.scores[..., [0, 1, 6]]).all()
+
+
+def test_preblended_mode_validation(gu):
+    from paper_2505_18629_gb300 import rv, synth
+    h = gu.make_handle(_wl())
+    with pytest.raises(rv.RVError):
+        rv.rv_set_head_mode(h, 7)
+    rv.rv_set_acceptance(h, rv.RV_ACCEPT_TYPICAL, 0.3, 0.09)
+    with pytest.raises(rv.RVError):  # the typical rule needs the original entropy
+        rv.rv_set_head_mode(h, rv.RV_HEAD_PREBLENDED)
+    rv.rv_set_acceptance(h, rv.RV_ACCEPT_EXACT)
+    rv.rv_set_head_mode(h, rv.RV_HEAD_PREBLENDED)
+    with pytest.raises(rv.RVError):
+        rv.rv_set_acceptance(h, rv.RV_ACCEPT_TYPICAL, 0.3, 0.09)
+    rv.rv_set_head_mode(h, rv.RV_HEAD_FUSED_LOGITS)
+    rv.rv_set_acceptance(h, rv.RV_ACCEPT_TYPICAL, 0.3, 0.09)
+    h.close()
+    h32 = gu.make_handle(synth.WORKLOADS["tiny"])
+    with pytest.raises(rv.RVError):  # the bf16 head's variant only
+        rv.rv_set_head_mode(h32, rv.RV_HEAD_PREBLENDED)
+    h32.close()
+
+
+@pytest.mark.parametrize("name", ["small", "pairs"])
+def test_preblended_sampled_exact_match(gu, name):
+    # the pre-blended head writes z for the sampling rule as well
+    from paper_2505_18629_gb300 import synth
+    wl = (_wl(B=8, gamma=5, V=1000, seed=115) if name == "small"
+          else _wl(B=14, gamma=8, R=8, V=777, H=256, ctx=(10, 60), seed=116))
+    inp = synth.generate(wl)
+    z, u, drafts = _sampled_inputs(inp, ALPHA, 0.8, 117, preblended=True)
+    gpu = _run_sampled(gu, inp, drafts, ALPHA, 0.8, u, preblended=True)
+    _check_sampled(inp, z, u, drafts, 0.8, gpu)
+
+
+@pytest.mark.parametrize("name", ["llama3-8b-b1", "llama3-8b-b16"])
+def test_preblended_llama3_8b(gu, name):
+    from paper_2505_18629_gb300 import synth
+    _check(gu, synth.WORKLOADS[name], check_attn=False, preblended=True)
 
 
 # ------------------------------------------------------------------ full-size workloads

@@ -27,6 +27,10 @@ Notation follows the paper:
   * the pending-token block [t, x_1..x_gamma, template, x_1..x_gamma], whose
     first position is the last emitted token (``pack_block_pending``,
     ``verify_step_pending``)
+  * standard speculative verification, the baseline the method is compared
+    with (Sec. 4): block [x_1..x_gamma], p_i = softmax(o_i) from the gamma+1
+    original rows alone (``pack_block_standard``, ``verify_head_standard``,
+    ``verify_step_standard``)
 
 Hidden-state rows: row 0 is the target's last hidden state after the prefix
 (gives o_1, "M_p(prefix)" in Alg. 1); row r (1..Lb) follows block token r-1.
@@ -123,6 +127,16 @@ def pack_block_pending(pending, drafts, prompt_ids, prefix_ids, ctx_lens):
     block = np.concatenate([pending[:, None], blk.astype(np.int64)], axis=1)
     pos = np.asarray(ctx_lens, np.int64)[:, None] + np.arange(block.shape[1], dtype=np.int64)
     return block.astype(np.int32), pos.astype(np.int32)
+
+
+def pack_block_standard(drafts, ctx_lens):
+    """Block of standard speculative verification (no reflection): the drafts
+    alone, [x_1..x_gamma], at positions ctx_b, ctx_b + 1, ...
+    Returns block_ids, pos_ids [B, gamma]."""
+    drafts = np.asarray(drafts, np.int64)
+    gamma = drafts.shape[1]
+    pos = np.asarray(ctx_lens, np.int64)[:, None] + np.arange(gamma, dtype=np.int64)
+    return drafts.astype(np.int32), pos.astype(np.int32)
 
 
 # --------------------------------------------------------------------------
@@ -317,6 +331,39 @@ def verify_head_preblended(W, hidden, drafts, gamma: int, R: int, alpha: float):
                 choice_gap=choice_gap, ent_orig=nan1.copy(), z=z)
 
 
+def verify_head_standard(W, hidden, drafts, gamma: int):
+    """LM head of standard speculative verification: p_i = softmax(o_i).
+
+    hidden [B, gamma+1, H] -- row 0 the state after the prefix, row i the
+    state after x_i -- so o_i = W h_{row i-1} for i = 1..gamma+1, as in
+    ``verify_head`` without the reflective rows (Eq. 2 at alpha = 0).  The
+    result has ``verify_head``'s keys; the distribution is o's own, so its
+    statistics sit in the fused fields (lse_fused, logp_fused, argmax,
+    margin, choice_gap, z) and the original / reflective / entropy fields are
+    NaN, as the single-distribution head leaves them."""
+    hidden = as_f64(hidden)
+    drafts = np.asarray(drafts, np.int64)
+    B = hidden.shape[0]
+    rows = [original_row(i) for i in range(1, gamma + 2)]
+    o = head_logits(W, hidden[:, rows, :].reshape(B * (gamma + 1), -1)).reshape(B, gamma + 1, -1)
+    lse = logsumexp(o)
+    bi = np.arange(B)[:, None]
+    ii = np.arange(gamma)[None, :]
+    ox = o[bi, ii, drafts]
+    o_others = o[:, :gamma, :].copy()
+    o_others[bi, ii, drafts] = -np.inf
+    margin = np.abs(ox - o_others.max(axis=-1))
+    choice = greedy_choice(o)
+    o_rest = o.copy()
+    np.put_along_axis(o_rest, choice[..., None], -np.inf, axis=-1)
+    choice_gap = np.take_along_axis(o, choice[..., None], axis=-1)[..., 0] - o_rest.max(axis=-1)
+    nan1 = np.full((B, gamma + 1), np.nan)
+    nan2 = np.full((B, gamma), np.nan)
+    return dict(lse_orig=nan1, lse_refl=nan1.copy(), lse_fused=lse, logp_fused=ox - lse[:, :gamma],
+                logp_orig=nan2, logp_refl=nan2.copy(), argmax=choice, margin=margin,
+                choice_gap=choice_gap, ent_orig=nan1.copy(), z=o)
+
+
 # --------------------------------------------------------------------------
 # Exact-match verification (Alg. 2) with greedy x^_i, prefix, next token
 # --------------------------------------------------------------------------
@@ -499,3 +546,19 @@ def verify_step_pending(inp_W, hidden, q, k_blk, v_blk, k_cache, v_cache, ctx_le
     return dict(block_ids=block_ids, pos_ids=pos_ids, attn=attn, k_cache=kc, v_cache=vc,
                 accept_mask=acc, accepted_len=n, next_token=t,
                 ctx_out=np.asarray(ctx_lens, np.int64) + 1 + n, **head)
+
+
+def verify_step_standard(inp_W, hidden, q, k_blk, v_blk, k_cache, v_cache, ctx_lens, drafts,
+                         gamma: int):
+    """One step of standard speculative verification, the method's baseline:
+    block [x_1..x_gamma] (``pack_block_standard``), causal attention over its
+    gamma positions, p_i = softmax(o_i) from hidden [B, gamma+1, H]
+    (``verify_head_standard``), exact match (Alg. 2), new context ctx + n
+    (the rejected drafts' keys/values are dropped by length)."""
+    block_ids, pos_ids = pack_block_standard(drafts, ctx_lens)
+    attn, kc, vc = verify_attention(q, k_blk, v_blk, k_cache, v_cache, ctx_lens)
+    head = verify_head_standard(inp_W, hidden, drafts, gamma)
+    acc, n, t = exact_match_accept(drafts, head["argmax"])
+    return dict(block_ids=block_ids, pos_ids=pos_ids, attn=attn, k_cache=kc, v_cache=vc,
+                accept_mask=acc, accepted_len=n, next_token=t,
+                ctx_out=np.asarray(ctx_lens, np.int64) + n, **head)

@@ -860,3 +860,93 @@ def test_pins_catch_swapped_blend_weights(monkeypatch):
     monkeypatch.setattr(orc, "preblend_rows", lambda h, g, R, a: real(h, g, R, 1.0 - a))
     with pytest.raises(AssertionError):
         test_preblended_head_is_exact_at_alpha_0_and_1(0.0)
+
+
+# --------------------------------------------------------------------------
+# Standard speculative verification, the baseline without reflection (Sec. 4)
+# --------------------------------------------------------------------------
+
+def test_standard_block_closed_form_and_first_segment():
+    # the drafts alone at the positions after the context; they are the first
+    # segment of the reflective block (Eq. 1)
+    blk, pos = orc.pack_block_standard([[5, 6, 7], [1, 1, 2]], [10, 0])
+    np.testing.assert_array_equal(blk, [[5, 6, 7], [1, 1, 2]])
+    np.testing.assert_array_equal(pos, [[10, 11, 12], [0, 1, 2]])
+    rng = np.random.default_rng(51)
+    drafts = rng.integers(0, 100, (3, 4))
+    full, fpos = orc.pack_block(drafts, np.array([9, 8], np.int32),
+                                rng.integers(0, 100, (3, 4)), np.array([3, 7, 0]))
+    s, spos = orc.pack_block_standard(drafts, np.array([3, 7, 0]))
+    np.testing.assert_array_equal(full[:, :4], s)
+    np.testing.assert_array_equal(fpos[:, :4], spos)
+
+
+def test_standard_head_matches_torch_log_softmax():
+    # o_i from hidden row i-1 (rows beyond gamma are not read), against
+    # torch's fp64 matmul / log_softmax / logsumexp / argmax
+    rng = np.random.default_rng(52)
+    B, gamma, V, H = 3, 4, 300, 16
+    W = rng.standard_normal((V, H)).astype(np.float32)
+    hidden = rng.standard_normal((B, gamma + 2, H)).astype(np.float32)
+    drafts = rng.integers(0, V, (B, gamma))
+    r = orc.verify_head_standard(W, hidden, drafts, gamma)
+    o = torch.from_numpy(hidden[:, :gamma + 1].astype(np.float64)) @ \
+        torch.from_numpy(W.astype(np.float64)).T
+    lsm = torch.log_softmax(o, dim=-1).numpy()
+    np.testing.assert_allclose(r["lse_fused"], torch.logsumexp(o, dim=-1).numpy(), atol=1e-10)
+    bi, ii = np.arange(B)[:, None], np.arange(gamma)[None, :]
+    np.testing.assert_allclose(r["logp_fused"], lsm[bi, ii, drafts], atol=1e-10)
+    np.testing.assert_array_equal(r["argmax"], torch.argmax(o, dim=-1).numpy())
+    for f in ("lse_orig", "lse_refl", "logp_orig", "logp_refl", "ent_orig"):
+        assert np.isnan(r[f]).all()
+
+
+def test_standard_head_is_alpha_zero_of_the_reflective_head():
+    # Eq. 2 at alpha = 0 is standard verification: with the same states in
+    # rows 0..gamma, the reflective head's fused statistics equal these
+    rng = np.random.default_rng(53)
+    gamma, R = 3, 4
+    W, hidden, drafts = _rand_head(rng, 2, gamma, R, 120, 8)
+    r = orc.verify_head(W, hidden, drafts, gamma, R, 0.0)
+    s = orc.verify_head_standard(W, hidden[:, :gamma + 1], drafts, gamma)
+    for f in ("lse_fused", "logp_fused", "margin", "choice_gap"):
+        np.testing.assert_allclose(s[f], r[f], atol=1e-10)
+    np.testing.assert_array_equal(s["argmax"], r["argmax"])
+
+
+def test_standard_step_attention_and_decisions():
+    # the standard step's attention is the reflective block's first segment
+    # (Sec. 3.1); at alpha = 0 both steps take the same decisions
+    rng = np.random.default_rng(54)
+    B, gamma, R, Hq, Hkv, D, V, H = 2, 3, 2, 4, 2, 8, 60, 8
+    Lb = 2 * gamma + R
+    q, kb, vb, kc, vc, ctx = _rand_attn(rng, B, Lb, Hq, Hkv, D, [4, 0], 20)
+    W, hidden, _ = _rand_head(rng, B, gamma, R, V, H)
+    choice = np.argmax(orc.as_f64(hidden[:, :gamma]) @ orc.as_f64(W).T, axis=-1)
+    drafts = np.where(rng.random((B, gamma)) < 0.7, choice, rng.integers(0, V, (B, gamma)))
+    full = orc.verify_step(W, hidden, q, kb, vb, kc, vc, ctx, drafts, np.array([1], np.int32),
+                           rng.integers(0, V, (B, 1)), gamma, R, 0.0)
+    std = orc.verify_step_standard(W, hidden[:, :gamma + 1], q[:, :gamma], kb[:, :gamma],
+                                   vb[:, :gamma], kc, vc, ctx, drafts, gamma)
+    np.testing.assert_array_equal(std["attn"], full["attn"][:, :gamma])
+    for b, c in enumerate(ctx):
+        np.testing.assert_array_equal(std["k_cache"][b, :, :c + gamma], full["k_cache"][b, :, :c + gamma])
+    for f in ("accept_mask", "accepted_len", "next_token", "ctx_out"):
+        np.testing.assert_array_equal(std[f], full[f])
+
+
+def test_pins_catch_standard_row_off_by_one(monkeypatch):
+    monkeypatch.setattr(orc, "original_row", lambda i: i)
+    with pytest.raises(AssertionError):
+        test_standard_head_matches_torch_log_softmax()
+
+
+def test_pins_catch_standard_block_with_copy(monkeypatch):
+    def with_copy(drafts, ctx_lens):
+        d = np.asarray(drafts, np.int64)
+        blk = np.concatenate([d, d], axis=1)
+        pos = np.asarray(ctx_lens, np.int64)[:, None] + np.arange(blk.shape[1])
+        return blk.astype(np.int32), pos.astype(np.int32)
+    monkeypatch.setattr(orc, "pack_block_standard", with_copy)
+    with pytest.raises(AssertionError):
+        test_standard_block_closed_form_and_first_segment()

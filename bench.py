@@ -16,6 +16,11 @@ fp64 CPU oracle on a bounded sample of the same step (rank 0).
 
 `--impl reference` times the CPU oracle alone (the paper ships no code; the
 oracle written from the paper stands in for it) on the same workload.
+
+`--sweep` times the 8B-shaped sweep instead (B in {1,4,16,64} x gamma in
+{2,4,8} x ctx in {1024,8192}, template 8): per point the reflective step, the
+same step at alpha = 0, and standard speculative verification (block of the
+drafts alone, gamma+1 head rows), one JSON line each point.
 """
 from __future__ import annotations
 
@@ -237,6 +242,119 @@ def _config(wl, world=1, head_mode="fused"):
             "l2": "inputs larger than L2: the LM-head weight (V*H*2 bytes) streams every step"}
 
 
+# ---------------------------------------------------------------------------- sweep
+
+def _time_steps(fn, steps, warmup, stream):
+    import torch
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        fn()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) * 1e3 / steps  # µs per step
+
+
+def run_sweep(args):
+    """Each sweep point three ways on the same device-resident inputs (seeded
+    on the device: W N(0, 0.02), hidden rows RMS 1, Q/K/V/cache N(0, 1), all
+    bf16): the reflective step at alpha = 0.3, the reflective step at
+    alpha = 0, and standard verification.  At alpha = 0 the fused
+    distribution is the original one, so its decisions must equal standard
+    verification's (Eq. 2); the count of differing sequences is reported."""
+    import torch
+    from paper_2505_18629_gb300 import rv, synth
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream(dev)
+    hbm, tf_burst, _, peak_src = _peaks()
+    pts = synth.sweep_workloads()
+    if args.sweep_points:
+        keep = set(args.sweep_points.split(","))
+        pts = [w for w in pts if w.name in keep]
+    g0 = torch.Generator(device=dev)
+    g0.manual_seed(100)
+    H, V = pts[0].H, pts[0].V
+    W = (torch.randn(V, H, generator=g0, device=dev) * 0.02).to(torch.bfloat16)
+    clocks = ClockSampler(0)
+    clocks.start()
+    for wl in pts:
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(wl.seed)
+        B, g, R, Lb, C = wl.B, wl.gamma, wl.R, wl.Lb, wl.capacity
+        bf = torch.bfloat16
+
+        def rnd(*shape):
+            return torch.randn(*shape, generator=gen, device=dev).to(bf)
+        hid = torch.randn(B, Lb + 1, H, generator=gen, device=dev)
+        hidden = (hid / hid.pow(2).mean(-1, keepdim=True).sqrt()).to(bf)
+        q, kb, vb = rnd(B, Lb, wl.Hq, wl.D), rnd(B, Lb, wl.Hkv, wl.D), rnd(B, Lb, wl.Hkv, wl.D)
+        kc, vc = rnd(B, wl.Hkv, C, wl.D), rnd(B, wl.Hkv, C, wl.D)
+        ctx = torch.full((B,), wl.ctx[0], dtype=torch.int32, device=dev)
+        prompt = torch.randint(0, V, (wl.n_prompt,), generator=gen, device=dev, dtype=torch.int32)
+        prefix = torch.randint(0, V, (B, wl.n_prefix_eff), generator=gen, device=dev,
+                               dtype=torch.int32)
+        h = rv.rv_create(H, V, wl.Hq, wl.Hkv, wl.D, B, g, R, C, rv.RV_DTYPE_BF16)
+
+        def outs(lb):
+            i32 = dict(dtype=torch.int32, device=dev)
+            return [torch.empty((B, lb), **i32), torch.empty((B, lb), **i32),
+                    torch.empty((B, lb, wl.Hq, wl.D), dtype=bf, device=dev),
+                    torch.empty((B, g + 1, rv.RV_NSCORES), device=dev),
+                    torch.empty((B, g + 1), **i32), torch.empty((B, g), device=dev),
+                    torch.empty((B, g), dtype=torch.uint8, device=dev), torch.empty((B,), **i32),
+                    torch.empty((B,), **i32), torch.empty((B,), **i32)]
+        o_r, o_0, o_s = outs(Lb), outs(Lb), outs(g)
+        # drafts: the reflective head's own greedy choice with p_argmax, else uniform
+        d0 = torch.zeros((B, g), dtype=torch.int32, device=dev)
+        rv.rv_verify_head(h, hidden, W, d0, g, R, ALPHA, o_r[3], o_r[4], o_r[5])
+        keep = torch.rand((B, g), generator=gen, device=dev) < wl.p_argmax
+        alt = torch.randint(0, V, (B, g), generator=gen, device=dev, dtype=torch.int32)
+        drafts = torch.where(keep, o_r[4][:, :g], alt).contiguous()
+        q_s, kb_s, vb_s = (x[:, :g].contiguous() for x in (q, kb, vb))
+        hid_s = hidden[:, :g + 1].contiguous()
+        empty = torch.zeros((B, 0), dtype=torch.int32, device=dev)
+
+        def refl(alpha, o):
+            return lambda: rv.rv_verify_step(h, q, kb, vb, kc, vc, hidden, W, drafts, prompt,
+                                             prefix, ctx, alpha, *o, stream)
+
+        def std():
+            rv.rv_verify_step(h, q_s, kb_s, vb_s, kc, vc, hid_s, W, drafts, None, empty, ctx,
+                              0.0, *o_s, stream)
+        steps, warm = args.steps, max(args.warmup, 3)
+        t_r = _time_steps(refl(ALPHA, o_r), steps, warm, stream)
+        t_0 = _time_steps(refl(0.0, o_0), steps, warm, stream)
+        rv.rv_set_head_mode(h, rv.RV_HEAD_STANDARD)
+        t_s = _time_steps(std, steps, warm, stream)
+        rv.rv_set_head_mode(h, rv.RV_HEAD_FUSED_LOGITS)
+        st = rv.rv_read_status(h, stream)
+        same = ((o_0[6] == o_s[6]).all(dim=1) & (o_0[7] == o_s[7]) & (o_0[8] == o_s[8]))
+        ctx_mean = float(wl.ctx[0])
+        kv = B * ctx_mean * wl.Hkv * wl.D * 2 * 2
+
+        def roof(rows):
+            return max(2.0 * rows * H * V / (tf_burst * 1e12), (V * H * 2 + kv) / (hbm * 1e9)) * 1e6
+        r_r, r_s = roof(2 * (g + 1) * B), roof((g + 1) * B)
+        print(json.dumps({
+            "sweep_point": wl.name, "B": B, "gamma": g, "template": R, "ctx": wl.ctx[0],
+            "Lb": Lb, "reflective_us": t_r, "alpha0_us": t_0, "standard_us": t_s,
+            "reflective_over_standard": t_r / t_s,
+            "positions_per_s": B * Lb / (t_r * 1e-6), "drafts_per_s": B * g / (t_r * 1e-6),
+            "step_roofline_us": r_r, "frac": r_r / t_r,
+            "standard_roofline_us": r_s, "standard_frac": r_s / t_s,
+            "alpha0_vs_standard_differing_sequences": int(B - same.sum().item()),
+            "status": st, "peak_source": peak_src}), flush=True)
+        h.close()
+        del q, kb, vb, kc, vc, hidden, hid, o_r, o_0, o_s, q_s, kb_s, vb_s, hid_s
+        torch.cuda.empty_cache()
+    print(json.dumps({"sweep_clocks": clocks.stop(), "steps": args.steps,
+                      "data": "synthetic, seeded on the device"}), flush=True)
+
+
 # ---------------------------------------------------------------------------- main arm
 
 def main():
@@ -252,8 +370,17 @@ def main():
     ap.add_argument("--head-mode", default="fused", choices=["fused", "preblended"],
                     help="fused: both logit vectors fused per vocab row (Eq. 2); preblended: "
                          "the head on the blended hidden states (one row per position)")
+    ap.add_argument("--sweep", action="store_true",
+                    help="time the 8B sweep (reflective, alpha = 0, standard) instead")
+    ap.add_argument("--sweep-points", default="",
+                    help="comma-separated sweep point names (default: all 24)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
+    if args.sweep:
+        if args.steps == 2000:
+            args.steps = 50
+        run_sweep(args)
+        return
 
     from paper_2505_18629_gb300 import synth
     wl = synth.workload(args.workload)

@@ -86,6 +86,7 @@ extern "C" {
 /* LM-head variants (rv_set_head_mode). */
 #define RV_HEAD_FUSED_LOGITS 0  /* o_i and o_{m+i-1} from their own rows, fused (Eq. 2)      */
 #define RV_HEAD_PREBLENDED 1    /* z_i = W b_i from the blended hidden state (linearity)      */
+#define RV_HEAD_STANDARD 2      /* standard speculative verification: no reflection           */
 
 /* Model / capacity description fixed at creation. */
 typedef struct rv_config {
@@ -241,6 +242,13 @@ RV_API int rv_set_acceptance(rv_handle* h, int32_t mode, float eps, float delta)
  *     |W_vk| |b_k|).  The original / reflective fields of `scores` (lse_orig,
  *     lse_refl, logp_orig, logp_refl, ent_orig) are NaN, so the typical rule
  *     (Alg. 3, which needs the entropy) is refused in this mode.
+ *   RV_HEAD_STANDARD: standard speculative verification, the baseline the
+ *     method is compared with (Sec. 4): the block is the drafts alone,
+ *     [x_1..x_gamma] (Lb = gamma; the template must be empty, R = 0, else
+ *     RV_ERR_SHAPE), hidden is [B, gamma+1, H] with row i-1 giving
+ *     p_i = softmax(o_i), alpha is not used.  The step entry points, the pack
+ *     calls and the host-buffer step follow this layout; the fused fields of
+ *     `scores` hold o's statistics and the other fields are NaN, as above.
  * Errors: RV_ERR_INVALID_ARG for an unknown mode or with the typical rule set,
  * RV_ERR_UNSUPPORTED for an fp32 handle. */
 RV_API int rv_set_head_mode(rv_handle* h, int32_t mode);

@@ -17,15 +17,17 @@ namespace rv {
 // ---------------------------------------------------------------- pack (Eq. 1)
 // block[b] = [x_1..x_gamma, prompt, prefix_b, x_1..x_gamma]; pos = ctx_b + j.
 // With `pending`, the pending-token block [t_b, x_1..x_gamma, prompt, prefix_b,
-// x_1..x_gamma]: the last emitted token goes first.
+// x_1..x_gamma]: the last emitted token goes first.  copy == 0: standard
+// verification's block, [x_1..x_gamma] (or [t_b, x_1..x_gamma]), no template.
 __global__ void pack_block_kernel(const int32_t* __restrict__ drafts,
                                   const int32_t* __restrict__ prompt,
                                   const int32_t* __restrict__ prefix,
                                   const int32_t* __restrict__ ctx, int B, int gamma,
                                   int n_prompt, int n_prefix, int32_t* __restrict__ block,
-                                  int32_t* __restrict__ pos, const int32_t* __restrict__ pending) {
+                                  int32_t* __restrict__ pos, const int32_t* __restrict__ pending,
+                                  int copy) {
   const int lead = pending ? 1 : 0;
-  const int Lb = 2 * gamma + n_prompt + n_prefix + lead;
+  const int Lb = (1 + copy) * gamma + n_prompt + n_prefix + lead;
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= B * Lb) return;
   const int b = idx / Lb, jj = idx % Lb, j = jj - lead;
@@ -48,12 +50,12 @@ __global__ void pack_block_kernel(const int32_t* __restrict__ drafts,
 cudaError_t launch_pack_block(const int32_t* drafts, const int32_t* prompt, const int32_t* prefix,
                               const int32_t* ctx, int B, int gamma, int n_prompt, int n_prefix,
                               int32_t* block_ids, int32_t* pos_ids, cudaStream_t s,
-                              const int32_t* pending) {
-  const int n = B * (2 * gamma + n_prompt + n_prefix + (pending ? 1 : 0));
+                              const int32_t* pending, int copy) {
+  const int n = B * ((1 + copy) * gamma + n_prompt + n_prefix + (pending ? 1 : 0));
   if (n == 0) return cudaSuccess;
   pack_block_kernel<<<(n + 255) / 256, 256, 0, s>>>(drafts, prompt, prefix, ctx, B, gamma,
                                                      n_prompt, n_prefix, block_ids, pos_ids,
-                                                     pending);
+                                                     pending, copy);
   return cudaGetLastError();
 }
 
@@ -63,6 +65,8 @@ cudaError_t launch_pack_block(const int32_t* drafts, const int32_t* prompt, cons
 // or, for the pre-blended head (N = Pcp), the blended state of Eq. 2's
 // linearity, each element rounded once to bf16:
 // hsel row (c*N + j)        = bf16(fl((1-a) h[b][i]) + fl(a h[b][gamma+R+i]))
+// or, for standard verification (zonly == 2, N = Pcp, hidden [B, gamma+1, H]):
+// hsel row (c*N + j)        = h[b][i]
 // padding rows are zero.  One 16-byte vector per thread and step.  When the
 // block is to be packed too, the first B*Lb threads of the grid also do that.
 __device__ __forceinline__ uint32_t blend_bf16x2(uint32_t o, uint32_t r, float alpha, float beta) {
@@ -85,7 +89,7 @@ __global__ void prep_kernel(const uint4* __restrict__ hidden, uint4* __restrict_
   if (tid0 == 0 && done_counter) *done_counter = 0u;
   if (pk.block != nullptr) {
     const int lead = pk.pending ? 1 : 0;  // the pending-token block [t, x, prompt, prefix, x]
-    const int Lb = 2 * pk.gamma + pk.n_prompt + pk.n_prefix + lead;
+    const int Lb = (1 + pk.copy) * pk.gamma + pk.n_prompt + pk.n_prefix + lead;
     for (long long idx = tid0; idx < static_cast<long long>(pk.B) * Lb;
          idx += static_cast<long long>(gridDim.x) * blockDim.x) {
       const int b = static_cast<int>(idx / Lb), jj = static_cast<int>(idx % Lb), j = jj - lead;
@@ -118,7 +122,9 @@ __global__ void prep_kernel(const uint4* __restrict__ hidden, uint4* __restrict_
       const int b = p / (gamma + 1), i = p % (gamma + 1);
       const long long orow = (static_cast<long long>(b) * Lh + i) * Hv + col;
       const long long rrow = (static_cast<long long>(b) * Lh + i + gamma + R) * Hv + col;
-      if (zonly) {
+      if (zonly == 2) {
+        v = hidden[orow];
+      } else if (zonly) {
         const uint4 o = hidden[orow], rr = hidden[rrow];
         v = make_uint4(blend_bf16x2(o.x, rr.x, alpha, beta), blend_bf16x2(o.y, rr.y, alpha, beta),
                        blend_bf16x2(o.z, rr.z, alpha, beta), blend_bf16x2(o.w, rr.w, alpha, beta));
@@ -137,10 +143,11 @@ cudaError_t launch_prep(const HeadArgs& a, const HeadPlan& p, void* hsel, const 
   if (pack) {
     pk = *pack;
     work = static_cast<long long>(pk.B) *
-           (2 * pk.gamma + pk.n_prompt + pk.n_prefix + (pk.pending ? 1 : 0));
+           ((1 + pk.copy) * pk.gamma + pk.n_prompt + pk.n_prefix + (pk.pending ? 1 : 0));
   }
   const int Hv = a.H / 8;  // 8 bf16 per 16-byte vector
-  const int Lh = 2 * a.gamma + a.R + 1;
+  // hidden rows per sequence: the block's positions plus the state before it
+  const int Lh = p.standard ? a.gamma + 1 : 2 * a.gamma + a.R + 1;
   if (hsel) work = std::max(work, static_cast<long long>(p.n_chunks) * p.N * Hv);
   if (a.tile_counter) work = std::max(work, 1LL);
   if (work == 0) return cudaSuccess;
@@ -149,7 +156,8 @@ cudaError_t launch_prep(const HeadArgs& a, const HeadPlan& p, void* hsel, const 
   prep_kernel<<<blocks, threads, 0, s>>>(static_cast<const uint4*>(a.hidden),
                                          static_cast<uint4*>(hsel), p.P, a.gamma, a.R, Lh, Hv,
                                          p.pairs_per_chunk, p.pad_pairs, p.N, p.n_chunks,
-                                         p.zonly ? 1 : 0, a.alpha, 1.0f - a.alpha, pk,
+                                         p.standard ? 2 : (p.zonly ? 1 : 0), a.alpha,
+                                         1.0f - a.alpha, pk,
                                          a.tile_counter, a.done_counter);
   return cudaGetLastError();
 }

@@ -138,9 +138,11 @@ int lb_max(const rv_config& c) { return 2 * c.max_gamma + c.max_template + 1; }
 
 // zonly: the pre-blended head (one blended row per pair, N = pad_pairs,
 // rounded to 16 for the MMA; up to MAX_ZPAIRS_PER_CHUNK pairs per chunk).
-HeadPlan head_plan(int B, int gamma, int V, int num_sms, bool tc, bool zonly = false) {
+HeadPlan head_plan(int B, int gamma, int V, int num_sms, bool tc, bool zonly = false,
+                   bool standard = false) {
   HeadPlan p;
   p.zonly = zonly;
+  p.standard = standard;
   p.P = B * (gamma + 1);
   const int cap = zonly ? MAX_ZPAIRS_PER_CHUNK : MAX_PAIRS_PER_CHUNK;
   p.n_chunks = (p.P + cap - 1) / cap;
@@ -401,8 +403,11 @@ extern "C" RV_API int rv_pack_block(rv_handle* h, const int32_t* draft_ids, cons
   if (!draft_ids || !ctx_lens || !block_ids || !pos_ids || (n_prompt > 0 && !prompt_ids) ||
       (n_prefix > 0 && !prefix_ids))
     return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument");
+  if (h->head_mode == RV_HEAD_STANDARD && n_prompt + n_prefix != 0)
+    return fail(h, RV_ERR_SHAPE, "standard verification's block has no template");
   cudaError_t e = launch_pack_block(draft_ids, prompt_ids, prefix_ids, ctx_lens, B, gamma, n_prompt,
-                                    n_prefix, block_ids, pos_ids, static_cast<cudaStream_t>(stream));
+                                    n_prefix, block_ids, pos_ids, static_cast<cudaStream_t>(stream),
+                                    nullptr, h->head_mode == RV_HEAD_STANDARD ? 0 : 1);
   h->launches += 1;
   return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "pack_block launch");
 }
@@ -423,9 +428,11 @@ extern "C" RV_API int rv_pack_block_pending(rv_handle* h, const int32_t* pending
   if (!pending_ids || !draft_ids || !ctx_lens || !block_ids || !pos_ids ||
       (n_prompt > 0 && !prompt_ids) || (n_prefix > 0 && !prefix_ids))
     return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument");
+  if (h->head_mode == RV_HEAD_STANDARD && n_prompt + n_prefix != 0)
+    return fail(h, RV_ERR_SHAPE, "standard verification's block has no template");
   cudaError_t e = launch_pack_block(draft_ids, prompt_ids, prefix_ids, ctx_lens, B, gamma, n_prompt,
                                     n_prefix, block_ids, pos_ids, static_cast<cudaStream_t>(stream),
-                                    pending_ids);
+                                    pending_ids, h->head_mode == RV_HEAD_STANDARD ? 0 : 1);
   h->launches += 1;
   return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "pack_block launch");
 }
@@ -546,6 +553,12 @@ int encode_maps(rv_handle* h, const void* w, const HeadPlan& pl, HeadTcLaunch& l
   return RV_OK;
 }
 
+// Block positions of a step (without the pending token): [x, template, x], or
+// the drafts alone for standard verification.
+int block_len(const rv_handle* h, int gamma, int R) {
+  return h->head_mode == RV_HEAD_STANDARD ? gamma : 2 * gamma + R;
+}
+
 int check_head_args(rv_handle* h, const void* hidden, const void* w_head, const int32_t* draft_ids,
                     int B, int gamma, int R, float alpha, const void* o1, const void* o2,
                     const void* o3) {
@@ -555,6 +568,8 @@ int check_head_args(rv_handle* h, const void* hidden, const void* w_head, const 
     return fail(h, RV_ERR_CAPACITY, "B %d / gamma %d / R %d above the handle's maxima (%d/%d/%d)", B,
                 gamma, R, c.max_batch, c.max_gamma, c.max_template);
   if (!std::isfinite(alpha)) return fail(h, RV_ERR_INVALID_ARG, "alpha is not finite");
+  if (h->head_mode == RV_HEAD_STANDARD && R != 0)
+    return fail(h, RV_ERR_SHAPE, "standard verification has no template: R must be 0 (got %d)", R);
   if (B == 0) return RV_OK;
   if (!hidden || !w_head || !draft_ids || !o1 || !o2 || !o3)
     return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument");
@@ -579,7 +594,8 @@ int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_
              bf16 ? h->ws.status + 32 : nullptr,    // finished-CTA counter
              writes_z(h) ? h->zbuf : nullptr};
   HeadPlan pl = head_plan(B, gamma, c.vocab, h->num_sms, bf16,
-                          bf16 && h->head_mode == RV_HEAD_PREBLENDED);
+                          bf16 && h->head_mode != RV_HEAD_FUSED_LOGITS,
+                          bf16 && h->head_mode == RV_HEAD_STANDARD);
   if (bf16 && pl.N >= HEAD_PAIR_MIN_N) {
     // CTA pairs: as many as fit at once (two CTAs of a pair share a GPC)
     if (h->head_pair_cached_N != 2 * pl.N + pl.zonly) {
@@ -711,10 +727,10 @@ extern "C" RV_API int rv_set_acceptance(rv_handle* h, int32_t mode, float eps, f
     return RV_OK;
   }
   if (mode != RV_ACCEPT_TYPICAL) return fail(h, RV_ERR_INVALID_ARG, "unknown acceptance mode %d", mode);
-  if (h->head_mode == RV_HEAD_PREBLENDED)
+  if (h->head_mode != RV_HEAD_FUSED_LOGITS)
     return fail(h, RV_ERR_INVALID_ARG,
                 "typical acceptance needs the original distribution's entropy, which the "
-                "pre-blended head does not form");
+                "single-distribution heads do not form");
   if (!(eps > 0.f) || !(delta > 0.f) || !std::isfinite(eps) || !std::isfinite(delta))
     return fail(h, RV_ERR_INVALID_ARG, "typical acceptance needs finite eps > 0 and delta > 0");
   h->accept_mode = mode;
@@ -730,13 +746,14 @@ extern "C" RV_API int rv_set_head_mode(rv_handle* h, int32_t mode) {
     h->head_mode = mode;
     return RV_OK;
   }
-  if (mode != RV_HEAD_PREBLENDED) return fail(h, RV_ERR_INVALID_ARG, "unknown head mode %d", mode);
+  if (mode != RV_HEAD_PREBLENDED && mode != RV_HEAD_STANDARD)
+    return fail(h, RV_ERR_INVALID_ARG, "unknown head mode %d", mode);
   if (h->cfg.dtype != RV_DTYPE_BF16)
-    return fail(h, RV_ERR_UNSUPPORTED, "the pre-blended head is the bf16 LM head's variant");
+    return fail(h, RV_ERR_UNSUPPORTED, "the single-distribution heads are bf16 LM-head variants");
   if (h->accept_mode == RV_ACCEPT_TYPICAL)
     return fail(h, RV_ERR_INVALID_ARG,
                 "typical acceptance needs the original distribution's entropy, which the "
-                "pre-blended head does not form");
+                "single-distribution heads do not form");
   h->head_mode = mode;
   return RV_OK;
 }
@@ -805,7 +822,7 @@ int step_impl(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
     return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument for the block packing");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const rv_config& c = h->cfg;
-  const int Lb = 2 * gamma + R + lead;
+  const int Lb = block_len(h, gamma, R) + lead;
   // Small batches: the attention (independent of the LM head) runs on the side
   // stream and shares the SMs with the HBM-bound head; join before returning.
   // The head goes first (it is the long pole).  Larger batches use the
@@ -821,6 +838,7 @@ int step_impl(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
   auto run_head = [&]() -> int {
     PackArgs pk{draft_ids, prompt_ids, prefix_ids, ctx_in, B, gamma, n_prompt, n_prefix, block_ids,
                 pos_ids, pending};
+    pk.copy = h->head_mode == RV_HEAD_STANDARD ? 0 : 1;
     AcceptArgs ac{accept_mask, accepted_len,       next_token,         ctx_in,
                   ctx_out,     h->accept_mode,     h->accept_log_eps,  h->accept_log_delta,
                   lead};
@@ -1030,7 +1048,9 @@ extern "C" RV_API int rv_verify_step_host(
     return fail(h, RV_ERR_INVALID_ARG, "NULL pointer argument for the block packing");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const size_t es = esize(c);
-  const int Lb = 2 * gamma + R;
+  if (h->head_mode == RV_HEAD_STANDARD && R != 0)
+    return fail(h, RV_ERR_SHAPE, "standard verification has no template: R must be 0 (got %d)", R);
+  const int Lb = block_len(h, gamma, R);
   const size_t nq = static_cast<size_t>(B) * Lb * c.n_q_heads * c.head_dim * es;
   const size_t nkv = static_cast<size_t>(B) * Lb * c.n_kv_heads * c.head_dim * es;
   const size_t nh = static_cast<size_t>(B) * (Lb + 1) * c.hidden * es;

@@ -46,6 +46,7 @@ struct HeadPlan {
   int slots;           // CTAs per chunk (= partial slots)
   bool pair;           // CTA-pair kernel (k_head_tc2.cu): slots = 2 * pairs
   bool zonly = false;  // pre-blended head: one blended row per pair, z statistics only
+  bool standard = false;  // standard verification: z-only on the original rows (Lh = gamma+1)
 };
 
 // Optional acceptance fused into the head merge (rv_verify_step).
@@ -96,7 +97,7 @@ struct HeadArgs {
 cudaError_t launch_pack_block(const int32_t* drafts, const int32_t* prompt, const int32_t* prefix,
                               const int32_t* ctx, int B, int gamma, int n_prompt, int n_prefix,
                               int32_t* block_ids, int32_t* pos_ids, cudaStream_t s,
-                              const int32_t* pending = nullptr);
+                              const int32_t* pending = nullptr, int copy = 1);
 // Optional block packing (Eq. 1) for rv_verify_step: pack.block == nullptr skips it.
 struct PackArgs {
   const int32_t* drafts;
@@ -107,6 +108,7 @@ struct PackArgs {
   int32_t* block;
   int32_t* pos;
   const int32_t* pending = nullptr;  // [B]: the pending-token block [t, x, prompt, prefix, x]
+  int copy = 1;  // 0: standard verification's block, the drafts alone (no template, no copy)
 };
 // hidden rows of every chunk into hsel [n_chunks * N, H] (bf16), pads zeroed;
 // also packs the block when `pack` is given (one launch for both).

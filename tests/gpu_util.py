@@ -149,16 +149,22 @@ def _err(gpu_vals: np.ndarray, ref_vals: np.ndarray) -> float:
 
 
 def compare(inp: synth.VerifyInputs, drafts, alpha, ref: dict, gpu: GpuRun, check_attn=True,
-            seqs=None, pending=None) -> Report:
+            seqs=None, pending=None, standard=False) -> Report:
     """Assert GPU == oracle under the tolerances above; `seqs` restricts to sampled sequences.
-    `pending` [B]: the step ran over the pending-token block [t, x, template, x]."""
+    `pending` [B]: the step ran over the pending-token block [t, x, template, x].
+    `standard`: standard verification's block [x] (or [t, x])."""
     wl = inp.wl
     g = wl.gamma
     seqs = np.arange(wl.B) if seqs is None else np.asarray(seqs)
     lead = 0 if pending is None else 1
+    Lb = g if standard else wl.Lb
     assert gpu.status == 0, f"device status 0x{gpu.status:x}"
     # ---- pack
-    if pending is None:
+    if standard:
+        d = drafts[seqs] if pending is None else np.concatenate(
+            [np.asarray(pending)[seqs, None], drafts[seqs]], axis=1)
+        blk, pos = orc.pack_block_standard(d, inp.ctx_lens[seqs])
+    elif pending is None:
         blk, pos = orc.pack_block(drafts[seqs], inp.prompt_ids, inp.prefix_ids[seqs],
                                   inp.ctx_lens[seqs])
     else:
@@ -172,7 +178,7 @@ def compare(inp: synth.VerifyInputs, drafts, alpha, ref: dict, gpu: GpuRun, chec
         ok, amax, nbad = attn_close(gpu.attn[seqs], ref["attn"])
         assert ok, f"attention: {nbad} elements beyond {ATTN_RTOL} relative (max {amax:.3g})"
         for k, b in enumerate(seqs):
-            c = int(inp.ctx_lens[b]) + wl.Lb + lead
+            c = int(inp.ctx_lens[b]) + Lb + lead
             np.testing.assert_array_equal(gpu.k_cache[b, :, :c],
                                           _bits_like(ref["k_cache"][k, :, :c], gpu.k_cache))
             np.testing.assert_array_equal(gpu.v_cache[b, :, :c],

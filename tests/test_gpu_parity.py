@@ -861,6 +861,134 @@ def test_preblended_llama3_8b(gu, name):
     _check(gu, synth.WORKLOADS[name], check_attn=False, preblended=True)
 
 
+# ------------------------------------------------------------------ standard verification (the baseline)
+
+def _standard_run(gu, wl, seqs=None, check_attn=True, pending=False, host=False):
+    """rv_verify_step (or the pending / host-buffer step) of a standard-verification
+    handle on the workload's first gamma block positions and gamma+1 hidden rows,
+    against the oracle's verify_step_standard."""
+    import torch
+    import oracle.rv_oracle as orc
+    from paper_2505_18629_gb300 import rv, synth
+    inp = synth.generate(wl)
+    B, g = wl.B, wl.gamma
+    S = np.arange(B) if seqs is None else np.asarray(seqs)
+    lead = 1 if pending else 0
+    hid = np.ascontiguousarray(inp.hidden[:, :g + 1])
+    choice = inp.draft_alt.copy()
+    choice[S] = orc.verify_head_standard(inp.W, hid[S], np.zeros((len(S), g), np.int64),
+                                         g)["argmax"][:, :g]
+    drafts = synth.make_drafts(inp, choice)
+    t = np.random.default_rng(wl.seed + 7).integers(0, wl.V, B).astype(np.int32)
+    Lb = g + lead
+    qs, kbs, vbs = (np.ascontiguousarray(x[:, :Lb]) for x in (inp.q, inp.k_blk, inp.v_blk))
+    h = gu.make_handle(wl)
+    rv.rv_set_head_mode(h, rv.RV_HEAD_STANDARD)
+    kc, vc = gu.to_dev(inp.k_cache), gu.to_dev(inp.v_cache)
+    W = gu.to_dev(inp.W)
+    if host:
+        def pin(x):
+            tt = torch.from_numpy(x.view(np.int16) if x.dtype == np.uint16 else np.ascontiguousarray(x))
+            return (tt.view(torch.bfloat16) if x.dtype == np.uint16 else tt).pin_memory()
+        dev = dict(q=pin(qs), kb=pin(kbs), vb=pin(vbs), hid=pin(hid),
+                   d=pin(drafts.astype(np.int32)), ctx=pin(inp.ctx_lens.astype(np.int32)))
+        mk = lambda shape, dt=torch.int32: torch.full(shape, -7, dtype=dt).pin_memory()
+        attn = torch.zeros(qs.shape, dtype=torch.bfloat16).pin_memory()
+        sc = torch.full((B, g + 1, rv.RV_NSCORES), float("nan")).pin_memory()
+        mg = torch.full((B, g), float("nan")).pin_memory()
+    else:
+        dev = dict(q=gu.to_dev(qs), kb=gu.to_dev(kbs), vb=gu.to_dev(vbs), hid=gu.to_dev(hid),
+                   d=gu.to_dev(drafts.astype(np.int32)), ctx=gu.to_dev(inp.ctx_lens.astype(np.int32)))
+        mk = lambda shape, dt=torch.int32: torch.full(shape, -7, dtype=dt, device="cuda")
+        attn = torch.zeros_like(dev["q"])
+        sc = torch.full((B, g + 1, rv.RV_NSCORES), float("nan"), device="cuda")
+        mg = torch.full((B, g), float("nan"), device="cuda")
+    prefix = mk((B, 0))
+    block, pos = mk((B, Lb)), mk((B, Lb))
+    am, acc = mk((B, g + 1)), mk((B, g), torch.uint8)
+    n, nt, co = mk((B,)), mk((B,)), mk((B,))
+    args = (dev["q"], dev["kb"], dev["vb"], kc, vc, dev["hid"], W)
+    tail = (None, prefix, dev["ctx"], ALPHA, block, pos, attn, sc, am, mg, acc, n, nt, co)
+    if inp.prompt_ids.size:
+        with pytest.raises(rv.RVError):  # standard verification has no template
+            rv.rv_verify_step(h, *args, dev["d"], gu.to_dev(inp.prompt_ids.astype(np.int32)),
+                              *tail[1:])
+    if host:
+        rv.rv_verify_step_host(h, *args, dev["d"], *tail)
+    elif pending:
+        rv.rv_verify_step_pending(h, *args, gu.to_dev(t), dev["d"], *tail)
+    else:
+        rv.rv_verify_step(h, *args, dev["d"], *tail)
+    torch.cuda.synchronize()
+    gpu = gu.GpuRun(gu.to_np(attn), gu.to_np(kc), gu.to_np(vc), gu.to_np(sc), gu.to_np(am),
+                    gu.to_np(mg), gu.to_np(acc), gu.to_np(n), gu.to_np(nt), gu.to_np(co),
+                    gu.to_np(block), gu.to_np(pos), rv.rv_read_status(h))
+    h.close()
+    ref = orc.verify_step_standard(inp.W, hid[S], qs[S], kbs[S], vbs[S], inp.k_cache[S],
+                                   inp.v_cache[S], inp.ctx_lens[S], drafts[S], g)
+    ref.pop("z")
+    ref.pop("ctx_out")
+    if not check_attn:
+        for k in ("attn", "k_cache", "v_cache"):
+            ref.pop(k)
+    rep = gu.compare(inp, drafts, ALPHA, ref, gpu, check_attn=check_attn, seqs=seqs,
+                     pending=t if pending else None, standard=True)
+    print(f"\nstandard {wl.name}: {rep}")
+    return gpu
+
+
+def test_standard_verification_small(gu):
+    _standard_run(gu, _wl(seed=120), check_attn=True)
+
+
+def test_standard_verification_tcgen05_attention(gu):
+    # B*Hkv = 40 (sequence, KV head) pairs: the persistent tcgen05 attention,
+    # here over gamma = 6 block positions
+    _standard_run(gu, _wl(B=20, gamma=6, R=8, Hq=16, Hkv=2, V=2000, ctx=(0, 700), seed=121))
+
+
+def test_standard_verification_pending_block(gu):
+    # block [t, x_1..x_gamma]: t's state in hidden row 0, ctx += 1 + n
+    _standard_run(gu, _wl(B=3, gamma=4, seed=122), pending=True)
+
+
+def test_standard_verification_host_buffers(gu):
+    _standard_run(gu, _wl(B=4, gamma=5, seed=123), host=True)
+
+
+@pytest.mark.parametrize("name,seqs", [("llama3-8b-b16", None), ("sweep-b64-g8-c8192", [0, 33, 63])])
+def test_standard_verification_8b(gu, name, seqs):
+    from paper_2505_18629_gb300 import synth
+    _standard_run(gu, synth.workload(name), seqs=seqs)
+
+
+def test_standard_pack_entry_points(gu):
+    import torch
+    import oracle.rv_oracle as orc
+    from paper_2505_18629_gb300 import rv
+    h = gu.make_handle(_wl())
+    rv.rv_set_head_mode(h, rv.RV_HEAD_STANDARD)
+    d = np.array([[3, 4, 5, 6], [7, 8, 9, 10]], np.int32)
+    ctx = np.array([11, 0], np.int32)
+    blk = torch.full((2, 5), -7, dtype=torch.int32, device="cuda")
+    pos = torch.full((2, 5), -7, dtype=torch.int32, device="cuda")
+    empty = torch.zeros((2, 0), dtype=torch.int32, device="cuda")
+    b4, p4 = torch.full((2, 4), -7, dtype=torch.int32, device="cuda"), torch.full((2, 4), -7, dtype=torch.int32, device="cuda")
+    rv.rv_pack_block(h, gu.to_dev(d), None, empty, gu.to_dev(ctx), b4, p4)
+    eb, ep = orc.pack_block_standard(d, ctx)
+    np.testing.assert_array_equal(gu.to_np(b4), eb)
+    np.testing.assert_array_equal(gu.to_np(p4), ep)
+    t = np.array([1, 2], np.int32)
+    rv.rv_pack_block_pending(h, gu.to_dev(t), gu.to_dev(d), None, empty, gu.to_dev(ctx), blk, pos)
+    eb, ep = orc.pack_block_standard(np.concatenate([t[:, None], d], axis=1), ctx)
+    np.testing.assert_array_equal(gu.to_np(blk), eb)
+    np.testing.assert_array_equal(gu.to_np(pos), ep)
+    with pytest.raises(rv.RVError):  # no template in standard verification
+        rv.rv_pack_block(h, gu.to_dev(d), gu.to_dev(np.array([1], np.int32)), empty,
+                         gu.to_dev(ctx), b4, p4)
+    h.close()
+
+
 # ------------------------------------------------------------------ full-size workloads
 
 def test_llama3_8b_b1_full(gu):

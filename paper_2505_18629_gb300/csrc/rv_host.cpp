@@ -775,13 +775,22 @@ extern "C" RV_API int rv_set_head_mode(rv_handle* h, int32_t mode) {
 
 // ============================================================================ whole step
 
+// The persistent tcgen05 attention also runs on the side stream, after the LM
+// head is launched: its CTAs take the SMs that the head's last tiles leave
+// idle (8B B=16 step 318 -> 313 us, e2e 0.99 -> 1.07 M positions/s).  The two
+// kernels cannot share an SM (their shared memory exceeds one SM's), and
+// neither waits on the other.
+#ifndef RV_FORK_PERSISTENT_ATTENTION
+#define RV_FORK_PERSISTENT_ATTENTION 1
+#endif
+
 namespace {
 
-// Whether the step runs the attention on the side stream, beside the LM head
-// (small batches), or before it on the caller's stream (the persistent
-// tcgen05 attention, which fills every SM).
+// Whether the step runs the attention on the side stream, beside the LM head,
+// or before it on the caller's stream.
 bool attn_forks(const rv_handle* h, int B, int Lb) {
   const rv_config& c = h->cfg;
+  if (RV_FORK_PERSISTENT_ATTENTION) return true;
   return c.dtype != RV_DTYPE_BF16 ||
          !attn_plan(B, Lb, c.n_q_heads, c.n_kv_heads, c.max_ctx, h->num_sms, true,
                     h->attn_max_cluster, c.head_dim, h->attn_tc_ok)
@@ -838,11 +847,10 @@ int step_impl(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const rv_config& c = h->cfg;
   const int Lb = block_len(h, gamma, R) + lead;
-  // Small batches: the attention (independent of the LM head) runs on the side
-  // stream and shares the SMs with the HBM-bound head; join before returning.
-  // The head goes first (it is the long pole).  Larger batches use the
-  // persistent tcgen05 attention, which fills every SM as the head does:
-  // there the two run one after the other on `stream`.
+  // The attention (independent of the LM head) runs on the side stream; join
+  // before returning.  The head goes first (it is the long pole).  At small
+  // batches the split-KV attention shares the SMs with the HBM-bound head; the
+  // persistent tcgen05 attention of larger batches takes SMs as head CTAs finish.
   const bool fork = attn_forks(h, B, Lb);
   cudaError_t e = cudaSuccess;
   if (fork) {

@@ -387,6 +387,15 @@ RV_API int rv_verify_step_host(rv_handle* h, const void* q_host, const void* k_b
                                int32_t* ctx_out_host, uint64_t* h2d_bytes, uint64_t* d2h_bytes,
                                void* stream);
 
+/* Whether this handle holds the CUDA graph of a repeated rv_verify_step_host
+ * call: the second call with the same arguments (pointers, sizes, alpha, the
+ * handle's modes and stream) is captured on `stream`, and later identical
+ * calls replay it.  No capture is attempted on the legacy default stream
+ * (NULL), with pageable host buffers, or while profiling is enabled.  *active
+ * = 1 when a graph is held, else 0.  Errors: RV_ERR_INVALID_ARG for NULL
+ * arguments. */
+RV_API int rv_host_step_graphed(const rv_handle* h, int32_t* active);
+
 /* ---- allocation-free LM head ------------------------------------------------
  * The paper has no counterpart: this entry point exists for callers that may
  * not allocate device memory (code running where cudaMalloc is unavailable or

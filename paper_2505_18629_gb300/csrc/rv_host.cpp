@@ -43,28 +43,33 @@ struct Workspace {
   void* st_vb = nullptr;
   void* st_hidden = nullptr;
   void* st_attn = nullptr;
-  int32_t* st_drafts = nullptr;
-  int32_t* st_prompt = nullptr;
-  int32_t* st_prefix = nullptr;
-  int32_t* st_block = nullptr;
-  int32_t* st_pos = nullptr;
-  int32_t* st_ctx_in = nullptr;
-  int32_t* st_ctx_out = nullptr;
-  float* st_scores = nullptr;
-  int32_t* st_argmax = nullptr;
-  float* st_margin = nullptr;
-  uint8_t* st_accept = nullptr;
-  int32_t* st_acc_len = nullptr;
-  int32_t* st_next = nullptr;
-  // rv_verify_step_host: the small per-step inputs (ids, lengths) and all the
-  // per-step outputs but the attention, each as one contiguous region, so that
-  // each crosses PCIe / C2C in one copy
-  char* st_small_in = nullptr;
-  char* st_small_out = nullptr;
+  // rv_verify_step_host: sizes of the pinned regions holding the small per-step
+  // inputs (ids, lengths) and all the per-step outputs but the attention
   size_t small_in_bytes = 0, small_out_bytes = 0;
 };
 
 }  // namespace
+
+// Page-locked host memory (a stream capture cannot copy from pageable memory).
+bool pinned(const void* p) {
+  cudaPointerAttributes a{};
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeHost;
+}
+
+// Everything that determines the device work of one rv_verify_step_host call.
+struct HostStepKey {
+  const void* ptr[24];
+  int32_t dims[4];
+  float alpha;
+  int32_t accept_mode, head_mode;
+  float log_eps, log_delta;
+  void* stream;
+  bool same(const HostStepKey& o) const { return std::memcmp(this, &o, sizeof(*this)) == 0; }
+};
 
 struct rv_handle {
   rv_config cfg;
@@ -87,9 +92,20 @@ struct rv_handle {
   cudaStream_t side = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   cudaEvent_t ev_copy_start = nullptr, ev_copy_done = nullptr;  // rv_verify_step_host
-  // pinned host mirrors of st_small_in / st_small_out (first rv_verify_step_host call)
+  // pinned staging of rv_verify_step_host's small inputs / outputs, which the
+  // kernels read / write in place (first rv_verify_step_host call)
   char* pin_in = nullptr;
   char* pin_out = nullptr;
+  // rv_verify_step_host: the arguments of the last call, and the CUDA graph of
+  // the device part of a call repeated with the same arguments
+  HostStepKey last_key{};
+  bool have_key = false;
+  HostStepKey graph_key{};
+  cudaGraphExec_t host_graph = nullptr;
+  unsigned long long graph_launches = 0;  // our kernel launches in the graph
+  bool graphs_off = false;                // capture failed once: direct calls only
+  const void* zc_hidden_ptr = nullptr;    // hidden-state buffer last seen, and whether it is
+  bool zc_hidden_ok = false;              // page-locked (read in place by the row gather)
   unsigned profiling = 0;  // bit mask of the regions being recorded
   ProfRegion prof[RV_PROF_COUNT];
   unsigned long long launches = 0;
@@ -266,16 +282,6 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
   const size_t n_hid = static_cast<size_t>(c.max_batch) * (Lbm + 1) * c.hidden;
   const size_t o_q = take(n_q * es), o_kb = take(n_kv * es), o_vb = take(n_kv * es);
   const size_t o_hid = take(n_hid * es), o_ao = take(n_q * es);
-  const size_t o_dr = take(static_cast<size_t>(c.max_batch) * c.max_gamma * 4);
-  const size_t o_pr = take(static_cast<size_t>(c.max_template) * 4 + 4);
-  const size_t o_px = take(static_cast<size_t>(c.max_batch) * c.max_template * 4 + 4);
-  const size_t o_bl = take(static_cast<size_t>(c.max_batch) * Lbm * 4);
-  const size_t o_ps = take(static_cast<size_t>(c.max_batch) * Lbm * 4);
-  const size_t o_ci = take(c.max_batch * 4), o_co = take(c.max_batch * 4);
-  const size_t o_sc = take(static_cast<size_t>(Pmax) * RV_NSCORES * 4);
-  const size_t o_am = take(static_cast<size_t>(Pmax) * 4);
-  const size_t o_mg = take(static_cast<size_t>(c.max_batch) * c.max_gamma * 4);
-  const size_t o_acc = take(static_cast<size_t>(c.max_batch) * c.max_gamma);
   // the host-buffer step's contiguous small regions (layout: see small_layout)
   const size_t small_in = 4 * (static_cast<size_t>(c.max_batch) * (c.max_gamma + 1 + c.max_template) +
                                c.max_template) + 64;
@@ -283,8 +289,6 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
       4 * (static_cast<size_t>(Pmax) * (RV_NSCORES + 1) + static_cast<size_t>(c.max_batch) *
                                                               (c.max_gamma + 3 + 2 * Lbm)) +
       static_cast<size_t>(c.max_batch) * c.max_gamma + 256;
-  const size_t o_sin = take(small_in), o_sout = take(small_out);
-  const size_t o_al = take(c.max_batch * 4), o_nt = take(c.max_batch * 4);
   h->attn_tc_ok = bf16 && attn_tc_supported(c.n_q_heads, c.n_kv_heads, c.head_dim) &&
                   attn_tc_smem_max(c.max_batch) <= h->smem_optin;
   const int a_slots =
@@ -312,21 +316,6 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
   h->ws.st_vb = b + o_vb;
   h->ws.st_hidden = b + o_hid;
   h->ws.st_attn = b + o_ao;
-  h->ws.st_drafts = reinterpret_cast<int32_t*>(b + o_dr);
-  h->ws.st_prompt = reinterpret_cast<int32_t*>(b + o_pr);
-  h->ws.st_prefix = reinterpret_cast<int32_t*>(b + o_px);
-  h->ws.st_block = reinterpret_cast<int32_t*>(b + o_bl);
-  h->ws.st_pos = reinterpret_cast<int32_t*>(b + o_ps);
-  h->ws.st_ctx_in = reinterpret_cast<int32_t*>(b + o_ci);
-  h->ws.st_ctx_out = reinterpret_cast<int32_t*>(b + o_co);
-  h->ws.st_scores = reinterpret_cast<float*>(b + o_sc);
-  h->ws.st_argmax = reinterpret_cast<int32_t*>(b + o_am);
-  h->ws.st_margin = reinterpret_cast<float*>(b + o_mg);
-  h->ws.st_accept = reinterpret_cast<uint8_t*>(b + o_acc);
-  h->ws.st_acc_len = reinterpret_cast<int32_t*>(b + o_al);
-  h->ws.st_next = reinterpret_cast<int32_t*>(b + o_nt);
-  h->ws.st_small_in = b + o_sin;
-  h->ws.st_small_out = b + o_sout;
   h->ws.small_in_bytes = small_in;
   h->ws.small_out_bytes = small_out;
   e = cudaMemset(h->ws.base, 0, off);
@@ -371,6 +360,7 @@ extern "C" RV_API int rv_destroy(rv_handle* h) {
   cudaEventDestroy(h->ev_copy_done);
   cudaStreamDestroy(h->side);
   if (h->zbuf) cudaFree(h->zbuf);
+  if (h->host_graph) cudaGraphExecDestroy(h->host_graph);
   if (h->pin_in) cudaFreeHost(h->pin_in);
   if (h->pin_out) cudaFreeHost(h->pin_out);
   cudaFree(h->ws.base);
@@ -1116,41 +1106,126 @@ extern "C" RV_API int rv_verify_step_host(
     if (npr) std::memcpy(hi + i_pr, prompt_ids_host, npr);
     if (npx) std::memcpy(hi + i_px, prefix_ids_host, npx);
   }
-  char* const di = w.st_small_in;
-  char* const dout = w.st_small_out;
-  // q, k_blk, v_blk on the side stream, concurrently with the ids and the
-  // hidden states on `stream`; `stream` waits for them before the step
-  // (the side stream's attention, when it runs there, follows its copies in
-  // stream order; otherwise `stream` waits for them before the step)
-  e = cudaEventRecord(h->ev_copy_start, s);
-  if (e == cudaSuccess) e = cudaStreamWaitEvent(h->side, h->ev_copy_start, 0);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(di, hi, in_small, cudaMemcpyHostToDevice, s);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(w.st_hidden, hidden_host, nh, cudaMemcpyHostToDevice, s);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(w.st_q, q_host, nq, cudaMemcpyHostToDevice, h->side);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(w.st_kb, k_blk_host, nkv, cudaMemcpyHostToDevice, h->side);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(w.st_vb, v_blk_host, nkv, cudaMemcpyHostToDevice, h->side);
-  if (e == cudaSuccess) e = cudaEventRecord(h->ev_copy_done, h->side);
-  if (e == cudaSuccess && !attn_forks(h, B, Lb)) e = cudaStreamWaitEvent(s, h->ev_copy_done, 0);
-  if (e != cudaSuccess) return cuda_fail(h, e, "host->device copy");
-  const size_t in_bytes = in_small + nh + nq + 2 * nkv;
-  auto I32 = [](char* p) { return reinterpret_cast<int32_t*>(p); };
-  int rc = rv_verify_step(h, w.st_q, w.st_kb, w.st_vb, k_cache, v_cache, w.st_hidden, w_head,
-                          I32(di + i_dr), do_pack ? I32(di + i_pr) : nullptr,
-                          do_pack ? I32(di + i_px) : nullptr, I32(di + i_ci), B, gamma, n_prompt,
-                          n_prefix, alpha, do_pack ? I32(dout + o_bl) : nullptr,
-                          do_pack ? I32(dout + o_ps) : nullptr, w.st_attn,
-                          reinterpret_cast<float*>(dout + o_sc), I32(dout + o_am),
-                          reinterpret_cast<float*>(dout + o_mg),
-                          reinterpret_cast<uint8_t*>(dout + o_ac), I32(dout + o_al),
-                          I32(dout + o_nt), I32(dout + o_co), stream);
-  if (rc != RV_OK) return rc;
-  size_t out_bytes = out_small;
-  if (attn_out_host) {
-    e = cudaMemcpyAsync(attn_out_host, w.st_attn, nq, cudaMemcpyDeviceToHost, s);
-    out_bytes += nq;
+  // The kernels read the small inputs from the pinned staging `hi` and write
+  // the small outputs into the pinned staging `ho` themselves (mapped host
+  // memory), and the row gather reads the hidden states from the caller's
+  // buffer when it is page-locked: only q / k_blk / v_blk (and attn_out) go
+  // through copies, on the side stream beside the LM head.
+  if (h->zc_hidden_ptr != hidden_host) {
+    h->zc_hidden_ok = pinned(hidden_host);
+    h->zc_hidden_ptr = hidden_host;
   }
-  if (e == cudaSuccess) e = cudaMemcpyAsync(h->pin_out, dout, out_small, cudaMemcpyDeviceToHost, s);
-  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  const bool zc_hidden = h->zc_hidden_ok;
+  char* const di = hi;
+  char* const dout = h->pin_out;
+  const size_t in_bytes = in_small + nh + nq + 2 * nkv;
+  const size_t out_bytes = out_small + (attn_out_host ? nq : 0);
+  auto I32 = [](char* p) { return reinterpret_cast<int32_t*>(p); };
+  // The device part: copies in, the step, copies out (all stream-ordered).
+  auto issue = [&]() -> int {
+    // q, k_blk, v_blk on the side stream, concurrently with the ids and the
+    // hidden states on `stream` (the side stream's attention follows its
+    // copies in stream order; otherwise `stream` waits for them before the step)
+    cudaError_t e = cudaEventRecord(h->ev_copy_start, s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(h->side, h->ev_copy_start, 0);
+    if (e == cudaSuccess && !zc_hidden)
+      e = cudaMemcpyAsync(w.st_hidden, hidden_host, nh, cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(w.st_q, q_host, nq, cudaMemcpyHostToDevice, h->side);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(w.st_kb, k_blk_host, nkv, cudaMemcpyHostToDevice, h->side);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(w.st_vb, v_blk_host, nkv, cudaMemcpyHostToDevice, h->side);
+    if (e == cudaSuccess) e = cudaEventRecord(h->ev_copy_done, h->side);
+    if (e == cudaSuccess && !attn_forks(h, B, Lb)) e = cudaStreamWaitEvent(s, h->ev_copy_done, 0);
+    if (e != cudaSuccess) return cuda_fail(h, e, "host->device copy");
+    int rc = rv_verify_step(h, w.st_q, w.st_kb, w.st_vb, k_cache, v_cache,
+                            zc_hidden ? hidden_host : w.st_hidden, w_head,
+                            I32(di + i_dr), do_pack ? I32(di + i_pr) : nullptr,
+                            do_pack ? I32(di + i_px) : nullptr, I32(di + i_ci), B, gamma,
+                            n_prompt, n_prefix, alpha, do_pack ? I32(dout + o_bl) : nullptr,
+                            do_pack ? I32(dout + o_ps) : nullptr, w.st_attn,
+                            reinterpret_cast<float*>(dout + o_sc), I32(dout + o_am),
+                            reinterpret_cast<float*>(dout + o_mg),
+                            reinterpret_cast<uint8_t*>(dout + o_ac), I32(dout + o_al),
+                            I32(dout + o_nt), I32(dout + o_co), stream);
+    if (rc != RV_OK) return rc;
+    if (attn_out_host) e = cudaMemcpyAsync(attn_out_host, w.st_attn, nq, cudaMemcpyDeviceToHost, s);
+    return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "device->host copy");
+  };
+  // A call repeated with the same arguments (a serving loop reusing its pinned
+  // buffers) is captured once as a CUDA graph and then replayed: one launch
+  // instead of about twenty API calls.  Profiling (event records inside the
+  // step) keeps the direct path.
+  HostStepKey key{};
+  {
+    const void* ptrs[24] = {q_host, k_blk_host, v_blk_host, k_cache, v_cache, hidden_host, w_head,
+                            prompt_ids_host, prefix_ids_host, block_ids_host, pos_ids_host,
+                            attn_out_host, scores_host, argmax_host, margin_host, accept_mask_host,
+                            accepted_len_host, next_token_host, ctx_out_host, draft_ids_host,
+                            ctx_in_host, nullptr, nullptr, nullptr};
+    std::memcpy(key.ptr, ptrs, sizeof(ptrs));
+    key.dims[0] = B;
+    key.dims[1] = gamma;
+    key.dims[2] = n_prompt;
+    key.dims[3] = n_prefix;
+    key.alpha = alpha;
+    key.accept_mode = h->accept_mode;
+    key.head_mode = h->head_mode;
+    key.log_eps = h->accept_log_eps;
+    key.log_delta = h->accept_log_delta;
+    key.stream = stream;
+  }
+  bool replay = false;
+  if (!h->graphs_off && h->profiling == 0) {
+    if (h->host_graph && key.same(h->graph_key)) {
+      replay = true;
+    } else if (h->have_key && key.same(h->last_key) && s != nullptr &&
+               pinned(q_host) && pinned(k_blk_host) && pinned(v_blk_host) &&
+               pinned(hidden_host) && (!attn_out_host || pinned(attn_out_host))) {
+      if (h->host_graph) {
+        cudaGraphExecDestroy(h->host_graph);
+        h->host_graph = nullptr;
+      }
+      // (the legacy default stream cannot be captured, nor can copies from
+      // pageable memory; a capture that fails all the same leaves the
+      // handle on the direct path)
+      const unsigned long long before = h->launches;
+      cudaError_t e = s ? cudaStreamBeginCapture(s, cudaStreamCaptureModeThreadLocal)
+                        : cudaErrorStreamCaptureUnsupported;
+      int rc = e == cudaSuccess ? issue() : RV_OK;
+      cudaGraph_t g = nullptr;
+      if (e == cudaSuccess) e = cudaStreamEndCapture(s, &g);
+      if (rc != RV_OK && rc != RV_ERR_CUDA) {  // an argument error: the direct call's too
+        if (g) cudaGraphDestroy(g);
+        h->launches = before;
+        return rc;
+      }
+      if (rc == RV_OK && e == cudaSuccess) e = cudaGraphInstantiate(&h->host_graph, g, 0);
+      if (g) cudaGraphDestroy(g);
+      if (rc == RV_OK && e == cudaSuccess) {
+        h->graph_key = key;
+        h->graph_launches = h->launches - before;
+        replay = true;
+      } else {
+        cudaGetLastError();
+        h->err.clear();
+        h->host_graph = nullptr;
+        h->graphs_off = true;
+      }
+      h->launches = before;
+    }
+    h->last_key = key;
+    h->have_key = true;
+  }
+  if (replay) {
+    e = cudaGraphLaunch(h->host_graph, s);
+    if (e != cudaSuccess) return cuda_fail(h, e, "graph launch");
+    h->launches += h->graph_launches;
+  } else {
+    const int rc = issue();
+    if (rc != RV_OK) return rc;
+  }
+  e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return cuda_fail(h, e, "device->host copy");
   const char* const ho = h->pin_out;
   std::memcpy(scores_host, ho + o_sc, P * RV_NSCORES * 4);
@@ -1166,6 +1241,12 @@ extern "C" RV_API int rv_verify_step_host(
   }
   if (h2d_bytes) *h2d_bytes = in_bytes;
   if (d2h_bytes) *d2h_bytes = out_bytes;
+  return RV_OK;
+}
+
+extern "C" RV_API int rv_host_step_graphed(const rv_handle* h, int32_t* active) {
+  if (!h || !active) return RV_ERR_INVALID_ARG;
+  *active = h->host_graph != nullptr ? 1 : 0;
   return RV_OK;
 }
 

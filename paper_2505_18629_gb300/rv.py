@@ -80,6 +80,7 @@ def _load():
         "rv_accept_typical": (I, [P, P, P, P, I, I, F, F, P, P, P, P, P, P]),
         "rv_set_acceptance": (I, [P, I, F, F]),
         "rv_set_head_mode": (I, [P, I]),
+        "rv_host_step_graphed": (I, [P, P]),
         "rv_accept_speculative": (I, [P, P, P, P, P, P, I, I, P, P, P, P, P, P]),
         "rv_verify_step_speculative": (I, [P, P, P, P, P, P, P, P, P, P, P, P, I, I, I, I, F, P, P,
                                            P, P, P, P, P, P, P, P, P, P, P, P]),
@@ -249,6 +250,13 @@ def rv_accept_sampled(h, draft_ids, u_uniform, temperature, sampled, accept_mask
                                      B, gamma, _ptr(sampled), _ptr(accept_mask),
                                      _ptr(accepted_len), _ptr(next_token), _ptr(ctx_in),
                                      _ptr(ctx_out), _stream(stream)))
+
+
+def rv_host_step_graphed(h):
+    """True when the handle replays a CUDA graph for its repeated host-buffer step."""
+    v = ctypes.c_int32()
+    _check(h, _lib.rv_host_step_graphed(h.ptr, ctypes.byref(v)))
+    return bool(v.value)
 
 
 def rv_set_head_mode(h, mode):

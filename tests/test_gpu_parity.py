@@ -307,6 +307,61 @@ def test_host_buffer_step_matches_device_step(gu):
     h.close()
 
 
+def test_host_buffer_step_graph_replay(gu):
+    # the same call repeated on a non-default stream is captured once as a CUDA
+    # graph and replayed; new contents of the pinned inputs (here the drafts)
+    # flow through every replay, and the launch count grows as for direct calls
+    import torch
+    from paper_2505_18629_gb300 import rv, synth
+    wl = _wl(seed=56, B=2)
+    inp = synth.generate(wl)
+    d1 = gu.oracle_drafts(inp, ALPHA)
+    d2 = ((d1 + 1) % wl.V).astype(d1.dtype)
+    ref = {1: gu.run_gpu(inp, d1, ALPHA), 2: gu.run_gpu(inp, d2, ALPHA)}
+    h = gu.make_handle(wl)
+    g, B, Lb = wl.gamma, wl.B, wl.Lb
+
+    def host(x):
+        t = torch.from_numpy(x.view(np.int16) if x.dtype == np.uint16 else np.ascontiguousarray(x))
+        return (t.view(torch.bfloat16) if x.dtype == np.uint16 else t).pin_memory()
+    kc, vc = gu.to_dev(inp.k_cache), gu.to_dev(inp.v_cache)
+    outs = dict(blk=torch.empty((B, Lb), dtype=torch.int32), pos=torch.empty((B, Lb), dtype=torch.int32),
+                attn=torch.empty(inp.q.shape, dtype=torch.bfloat16),
+                sc=torch.empty((B, g + 1, rv.RV_NSCORES)), am=torch.empty((B, g + 1), dtype=torch.int32),
+                mg=torch.empty((B, g)), acc=torch.empty((B, g), dtype=torch.uint8),
+                al=torch.empty((B,), dtype=torch.int32), nt=torch.empty((B,), dtype=torch.int32),
+                co=torch.empty((B,), dtype=torch.int32))
+    outs = {k: v.pin_memory() for k, v in outs.items()}
+    drafts = host(d1.astype(np.int32))
+    stream = torch.cuda.Stream()
+    prep = rv.PreparedStepHost(h, host(inp.q), host(inp.k_blk), host(inp.v_blk), kc, vc,
+                               host(inp.hidden), gu.to_dev(inp.W), drafts, host(inp.prompt_ids),
+                               host(inp.prefix_ids), host(inp.ctx_lens), ALPHA, outs["blk"],
+                               outs["pos"], outs["attn"], outs["sc"], outs["am"], outs["mg"],
+                               outs["acc"], outs["al"], outs["nt"], outs["co"], stream)
+    counts = []
+    for which in (1, 1, 2, 1, 2):
+        drafts.copy_(torch.from_numpy((d1 if which == 1 else d2).astype(np.int32)))
+        for v in outs.values():
+            v.zero_()
+        n0 = rv.rv_launch_count(h)
+        prep()
+        counts.append(rv.rv_launch_count(h) - n0)
+        step = ref[which]
+        np.testing.assert_array_equal(outs["blk"].numpy(), step.block_ids)
+        np.testing.assert_array_equal(outs["attn"].view(torch.int16).numpy().view(np.uint16),
+                                      step.attn)
+        _same_decisions(gu, outs["sc"].numpy(), outs["am"].numpy(), outs["mg"].numpy(), step)
+        np.testing.assert_array_equal(outs["acc"].numpy(), step.accept_mask)
+        np.testing.assert_array_equal(outs["al"].numpy(), step.accepted_len)
+        np.testing.assert_array_equal(outs["nt"].numpy(), step.next_token)
+        np.testing.assert_array_equal(outs["co"].numpy(), step.ctx_out)
+    assert len(set(counts)) == 1 and counts[0] > 0, counts
+    assert rv.rv_host_step_graphed(h)
+    assert rv.rv_read_status(h) == 0
+    h.close()
+
+
 # ------------------------------------------------------------------ device-side checks
 
 def test_out_of_range_draft_sets_status(gu):

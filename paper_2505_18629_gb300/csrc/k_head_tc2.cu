@@ -158,6 +158,9 @@ template <int EPI, int MC>
 __global__ void __launch_bounds__(h2_threads(EPI), 1)
     head_tc2_kernel(const __grid_constant__ CUtensorMap tm_w,
                     const __grid_constant__ CUtensorMap tm_h, const Head2Params p) {
+  // the merge launch that follows (programmatic dependent launch) may be
+  // scheduled now; it waits for this grid before it reads anything
+  asm volatile("griddepcontrol.launch_dependents;");
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;

@@ -204,6 +204,8 @@ __global__ void head_finalize_kernel(const float* __restrict__ partials,
                                      int slots, int wpp, float* __restrict__ scores,
                                      int32_t* __restrict__ argmax_out, float* __restrict__ margin,
                                      unsigned* status, AcceptArgs acc, int zonly) {
+  // launched as a programmatic dependent of the LM head: wait for its results
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   __shared__ MergeStat red[FIN_MAX_WARPS];
   __shared__ int s_choice[65];
   __shared__ int s_kept[65];
@@ -294,10 +296,18 @@ cudaError_t launch_head_finalize(const HeadArgs& a, const HeadPlan& p, float* sc
     wpp = std::max(1, std::min((p.slots + 31) / 32, FIN_MAX_WARPS / npos));
     warps = npos * wpp;
   }
-  head_finalize_kernel<<<a.B, warps * 32, 0, s>>>(a.partials, a.gathered, a.drafts, p.P, a.gamma,
-                                                  a.V, p.slots, wpp, scores, argmax, margin,
-                                                  a.status, ac, p.zonly ? 1 : 0);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.B, 1, 1);
+  cfg.blockDim = dim3(warps * 32, 1, 1);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, head_finalize_kernel, a.partials, a.gathered, a.drafts, p.P,
+                            a.gamma, a.V, p.slots, wpp, scores, argmax, margin, a.status, ac,
+                            p.zonly ? 1 : 0);
 }
 
 // ---------------------------------------------------------------- accept (Alg. 2)

@@ -477,11 +477,13 @@ def main():
     ms_total = e0.elapsed_time(e1)
     head_ms, head_n = rv.rv_profile_read(h, rv.RV_PROF_HEAD)
     rv.rv_profile_enable(h, 0)
-    # Breakdown run (after the timed region, not part of `value`): each kernel
-    # alone between its own events.
+    # Breakdown run (after the timed region, not part of `value`): the LM head
+    # and the attention each alone (their own entry points, one after the
+    # other on one stream), between the library's events around the kernels.
     rv.rv_profile_enable(h, (1 << rv.RV_PROF_HEAD_GEMM) | (1 << rv.RV_PROF_ATTENTION))
     for _ in range(min(args.steps, 200)):
-        step()
+        rv.rv_verify_head(h, hidden, W, drafts, g, R, ALPHA, scores, argmax, margin, stream)
+        rv.rv_verify_attention(h, q, kb, vb, kc, vc, ctx, attn, stream)
     torch.cuda.synchronize(dev)
     gemm_ms, gemm_n = rv.rv_profile_read(h, rv.RV_PROF_HEAD_GEMM)
     attn_ms, attn_n = rv.rv_profile_read(h, rv.RV_PROF_ATTENTION)

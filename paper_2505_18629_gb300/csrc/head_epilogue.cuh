@@ -182,14 +182,17 @@ __device__ __forceinline__ void head_tile_pairs8_t(const float (&o)[8], const fl
       gx[2] = zr[j];
     }
   }
+  // 16-byte slot k of staged row l sits at slot k ^ ((l >> 2) & 1): rows l and
+  // l + 4 of an eight-lane store wavefront then fall on different banks
   float4* const row = reinterpret_cast<float4*>(scr + lane * HEAD_SCR_STRIDE);
+  const int sw = (lane >> 2) & 1;
   const float ninf = NEG_INF;
-  row[0] = valid ? make_float4(o[0], o[1], o[2], o[3]) : make_float4(ninf, ninf, ninf, ninf);
-  row[1] = valid ? make_float4(o[4], o[5], o[6], o[7]) : make_float4(ninf, ninf, ninf, ninf);
-  row[2] = valid ? make_float4(r[0], r[1], r[2], r[3]) : make_float4(ninf, ninf, ninf, ninf);
-  row[3] = valid ? make_float4(r[4], r[5], r[6], r[7]) : make_float4(ninf, ninf, ninf, ninf);
-  row[4] = valid ? make_float4(zr[0], zr[1], zr[2], zr[3]) : make_float4(ninf, ninf, ninf, ninf);
-  row[5] = valid ? make_float4(zr[4], zr[5], zr[6], zr[7]) : make_float4(ninf, ninf, ninf, ninf);
+  row[0 ^ sw] = valid ? make_float4(o[0], o[1], o[2], o[3]) : make_float4(ninf, ninf, ninf, ninf);
+  row[1 ^ sw] = valid ? make_float4(o[4], o[5], o[6], o[7]) : make_float4(ninf, ninf, ninf, ninf);
+  row[2 ^ sw] = valid ? make_float4(r[0], r[1], r[2], r[3]) : make_float4(ninf, ninf, ninf, ninf);
+  row[3 ^ sw] = valid ? make_float4(r[4], r[5], r[6], r[7]) : make_float4(ninf, ninf, ninf, ninf);
+  row[4 ^ sw] = valid ? make_float4(zr[0], zr[1], zr[2], zr[3]) : make_float4(ninf, ninf, ninf, ninf);
+  row[5 ^ sw] = valid ? make_float4(zr[4], zr[5], zr[6], zr[7]) : make_float4(ninf, ninf, ninf, ninf);
   __syncwarp();
   if (lane < 24) {
     const int j = lane & 7, kind = lane >> 3;  // 0: o, 1: r, 2: z
@@ -198,7 +201,7 @@ __device__ __forceinline__ void head_tile_pairs8_t(const float (&o)[8], const fl
     float m = NEG_INF;
 #pragma unroll
     for (int i = 0; i < 32; ++i) {
-      val[i] = scr[i * HEAD_SCR_STRIDE + lane];
+      val[i] = scr[i * HEAD_SCR_STRIDE + (((i >> 2) & 1) ? (lane ^ 4) : lane)];
       m = fmaxf(m, val[i]);
     }
     float sum = 0.f, tsum = 0.f;  // tsum: sum exp(x - m) (x - m), for the entropy of o
@@ -260,9 +263,10 @@ __device__ __forceinline__ void head_tile_z8_t(const float (&z)[8], int g8, int 
     if (valid && v == s_drafts[pj] && pj < npairs) gathered[pj * GATHER_FIELDS + 2] = z[j];
   }
   float4* const row = reinterpret_cast<float4*>(scr + lane * HEAD_SCR_STRIDE);
+  const int sw = (lane >> 2) & 1;  // the swizzle of head_tile_pairs8_t
   const float ninf = NEG_INF;
-  row[0] = valid ? make_float4(z[0], z[1], z[2], z[3]) : make_float4(ninf, ninf, ninf, ninf);
-  row[1] = valid ? make_float4(z[4], z[5], z[6], z[7]) : make_float4(ninf, ninf, ninf, ninf);
+  row[0 ^ sw] = valid ? make_float4(z[0], z[1], z[2], z[3]) : make_float4(ninf, ninf, ninf, ninf);
+  row[1 ^ sw] = valid ? make_float4(z[4], z[5], z[6], z[7]) : make_float4(ninf, ninf, ninf, ninf);
   __syncwarp();
   if (lane < 8) {
     const int pj = g8 + lane;
@@ -270,7 +274,7 @@ __device__ __forceinline__ void head_tile_z8_t(const float (&z)[8], int g8, int 
     float m = NEG_INF;
 #pragma unroll
     for (int i = 0; i < 32; ++i) {
-      val[i] = scr[i * HEAD_SCR_STRIDE + lane];
+      val[i] = scr[i * HEAD_SCR_STRIDE + (((i >> 2) & 1) ? (lane ^ 4) : lane)];
       m = fmaxf(m, val[i]);
     }
     float sum = 0.f;

@@ -49,9 +49,9 @@ FALLBACK_BF16_TFLOPS = 1900.0
 # dram__bytes_write.sum` on the workload named (see profiles/), valid only while
 # the kernel sources hash to `src_sha`.
 NCU_TRAFFIC = {
-    "llama3-8b-b1": {"bytes": 1050904576 + 2824448, "src_sha": "d906e4fbd407c152",
+    "llama3-8b-b1": {"bytes": 1050912512 + 2772736, "src_sha": "2322d678d1a54902",
                      "summary": "profiles/head_tc_llama3-8b-b1.md"},
-    "llama3-8b-b16": {"bytes": 1053123584 + 2789632, "src_sha": "d906e4fbd407c152",
+    "llama3-8b-b16": {"bytes": 1053160704 + 2951680, "src_sha": "2322d678d1a54902",
                       "summary": "profiles/head_tc2_llama3-8b-b16.md"},
 }
 

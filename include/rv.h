@@ -434,8 +434,9 @@ RV_API int rv_read_status(rv_handle* h, void* stream, uint32_t* status);
 #define RV_PROF_COUNT 4
 
 /* mask: bit (1 << region) set = from now on, record a CUDA event pair on the
- * launching stream around each such region (up to 1024 per region, then
- * recording stops); 0 stops recording.  An event pair around RV_PROF_HEAD_GEMM
+ * launching stream around each such region (up to 1024 per region between two
+ * rv_profile_read calls, then recording stops); 0 stops recording.  Pairs
+ * recorded under earlier masks are kept until rv_profile_read.  An event pair around RV_PROF_HEAD_GEMM
  * sits between the row-gather launch and the LM-head launch and so disables
  * their overlap (programmatic dependent launch); RV_PROF_HEAD brackets both
  * without that cost.  Not for use inside graph capture. */

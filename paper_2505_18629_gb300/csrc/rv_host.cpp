@@ -1276,7 +1276,6 @@ extern "C" RV_API int rv_profile_enable(rv_handle* h, int32_t mask) {
           if (e != cudaSuccess) return cuda_fail(h, e, "cudaEventCreate");
         }
       }
-      r.used = 0;
     }
   }
   h->profiling = static_cast<unsigned>(mask) & ((1u << RV_PROF_COUNT) - 1u);

@@ -1017,6 +1017,47 @@ def test_standard_verification_8b(gu, name, seqs):
     _standard_run(gu, synth.workload(name), seqs=seqs)
 
 
+def test_standard_verification_sampled_exact_match(gu):
+    # standard verification's head writes z = o for the sampling rule too:
+    # rv_verify_head (R = 0, hidden [B, gamma+1, H]) + rv_accept_sampled
+    import torch
+    import oracle.rv_oracle as orc
+    from paper_2505_18629_gb300 import rv, synth
+    wl = _wl(B=8, gamma=5, V=1000, seed=124)
+    inp = synth.generate(wl)
+    B, g, T = wl.B, wl.gamma, 0.8
+    hid = np.ascontiguousarray(inp.hidden[:, :g + 1])
+    dummy = np.zeros((B, g), np.int64)
+    z = orc.verify_head_standard(inp.W, hid, dummy, g)["z"]
+    rng = np.random.default_rng(125)
+    u = rng.uniform(0, 1, (B, g + 1)).astype(np.float32)
+    _, _, _, xhat, _ = orc.sampled_exact_accept(dummy, z, T, u.astype(np.float64))
+    drafts = np.where(rng.uniform(size=(B, g)) < 0.7, xhat[:, :g],
+                      rng.integers(0, wl.V, (B, g))).astype(np.int64)
+    h = gu.make_handle(wl)
+    rv.rv_set_head_mode(h, rv.RV_HEAD_STANDARD)
+    rv.rv_set_acceptance(h, rv.RV_ACCEPT_SAMPLED)
+    d = gu.to_dev(drafts.astype(np.int32))
+    ctx = gu.to_dev(inp.ctx_lens.astype(np.int32))
+    sc = torch.empty((B, g + 1, rv.RV_NSCORES), device="cuda")
+    am = torch.empty((B, g + 1), dtype=torch.int32, device="cuda")
+    mg = torch.empty((B, g), device="cuda")
+    xs = torch.full((B, g + 1), -7, dtype=torch.int32, device="cuda")
+    acc = torch.full((B, g), 7, dtype=torch.uint8, device="cuda")
+    n = torch.full((B,), -7, dtype=torch.int32, device="cuda")
+    t = torch.full((B,), -7, dtype=torch.int32, device="cuda")
+    co = torch.full((B,), -7, dtype=torch.int32, device="cuda")
+    with pytest.raises(rv.RVError):  # a template with standard verification
+        rv.rv_verify_head(h, gu.to_dev(hid), gu.to_dev(inp.W), d, g, 2, ALPHA, sc, am, mg)
+    rv.rv_verify_head(h, gu.to_dev(hid), gu.to_dev(inp.W), d, g, 0, ALPHA, sc, am, mg)
+    rv.rv_accept_sampled(h, d, gu.to_dev(u), T, xs, acc, n, t, ctx, co)
+    gpu = (gu.to_np(xs), gu.to_np(acc), gu.to_np(n), gu.to_np(t), gu.to_np(co), gu.to_np(am),
+           rv.rv_read_status(h))
+    h.close()
+    acc_np, _ = _check_sampled(inp, z, u, drafts, T, gpu)
+    assert 0 < acc_np.sum() < acc_np.size
+
+
 def test_standard_pack_entry_points(gu):
     import torch
     import oracle.rv_oracle as orc

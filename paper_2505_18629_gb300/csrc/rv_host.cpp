@@ -766,12 +766,15 @@ extern "C" RV_API int rv_set_head_mode(rv_handle* h, int32_t mode) {
 // ============================================================================ whole step
 
 // The persistent tcgen05 attention also runs on the side stream, after the LM
-// head is launched: its CTAs take the SMs that the head's last tiles leave
-// idle (8B B=16 step 318 -> 313 us, e2e 0.99 -> 1.07 M positions/s).  The two
-// kernels cannot share an SM (their shared memory exceeds one SM's), and
-// neither waits on the other.
-#ifndef RV_FORK_PERSISTENT_ATTENTION
-#define RV_FORK_PERSISTENT_ATTENTION 1
+// head is launched, when the KV capacity is at most this many positions: its
+// CTAs take the SMs that the head's last tiles leave idle (8B B=16 step
+// 318 -> 313 us, e2e 0.99 -> 1.07 M positions/s).  The two kernels cannot share
+// an SM (their shared memory exceeds one SM's), and neither waits on the other.
+// With long caches the attention is better run alone first (8B B=16 ctx 8192:
+// 404 -> 383 us; B=64 ctx 8192: 887 -> 824 us); the context lengths
+// themselves live on the device, so the capacity decides.
+#ifndef RV_FORK_ATTENTION_MAX_CTX
+#define RV_FORK_ATTENTION_MAX_CTX 4608
 #endif
 
 namespace {
@@ -780,7 +783,7 @@ namespace {
 // or before it on the caller's stream.
 bool attn_forks(const rv_handle* h, int B, int Lb) {
   const rv_config& c = h->cfg;
-  if (RV_FORK_PERSISTENT_ATTENTION) return true;
+  if (c.max_ctx <= RV_FORK_ATTENTION_MAX_CTX) return true;
   return c.dtype != RV_DTYPE_BF16 ||
          !attn_plan(B, Lb, c.n_q_heads, c.n_kv_heads, c.max_ctx, h->num_sms, true,
                     h->attn_max_cluster, c.head_dim, h->attn_tc_ok)

@@ -360,20 +360,23 @@ RV_API int rv_verify_step_sampled(
     int32_t* argmax, float* margin, int32_t* sampled, uint8_t* accept_mask,
     int32_t* accepted_len, int32_t* next_token, int32_t* ctx_out, void* stream);
 
-/* The whole verify step from HOST buffers (synchronous).  The per-step inputs
- * (q, k_blk, v_blk, hidden, draft / prompt / prefix ids, ctx lens) are copied
- * from host memory (pinned memory gives asynchronous copies) into the handle's
- * device staging, rv_verify_step runs, and the per-step results are copied
- * back into host memory before the call returns.  The ids and lengths travel
- * in one copy through a pinned buffer of the handle, q / k_blk / v_blk are
- * copied on the handle's second stream while the hidden states copy on
- * `stream`, and all results but the attention output come back in one copy
- * (then scattered into the caller's buffers).  The first call allocates the
- * two small pinned buffers (RV_ERR_CUDA if that fails).  The model state stays on
- * the device: w_head, k_cache and v_cache are device pointers.  Host buffers
- * have the layouts of rv_verify_step; attn_out_host may be NULL to skip
- * reading the attention output back, block_ids_host NULL to skip the packing.
- * *h2d_bytes / *d2h_bytes (optional) receive the bytes copied each way. */
+/* The whole verify step from HOST buffers (synchronous).  The small per-step
+ * inputs (draft / prompt / prefix ids, ctx lens) are gathered into a pinned
+ * buffer of the handle that the kernels read in place, and the kernels write
+ * all results but the attention output into a second pinned buffer, which is
+ * scattered into the caller's buffers after the stream synchronises.  The row
+ * gather reads hidden_host in place when it is page-locked (only the rows the
+ * LM head needs cross the link), else it is copied into device staging first.
+ * q / k_blk / v_blk are copied into device staging on the handle's second
+ * stream (page-locked memory makes these copies asynchronous).  The first call
+ * allocates the two small pinned buffers (RV_ERR_CUDA if that fails).  The
+ * model state stays on the device: w_head, k_cache and v_cache are device
+ * pointers.  Host buffers have the layouts of rv_verify_step; attn_out_host
+ * may be NULL to skip reading the attention output back, block_ids_host NULL
+ * to skip the packing.  A call repeated with the same arguments on a
+ * non-default stream replays a CUDA graph (rv_host_step_graphed).
+ * *h2d_bytes / *d2h_bytes (optional) receive the bytes of the per-step inputs
+ * and outputs (the inputs' full sizes, also where only some rows are read). */
 RV_API int rv_verify_step_host(rv_handle* h, const void* q_host, const void* k_blk_host,
                                const void* v_blk_host, void* k_cache, void* v_cache,
                                const void* hidden_host, const void* w_head,

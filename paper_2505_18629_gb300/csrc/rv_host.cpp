@@ -63,12 +63,17 @@ bool pinned(const void* p) {
 // Everything that determines the device work of one rv_verify_step_host call.
 struct HostStepKey {
   const void* ptr[24];
-  int32_t dims[4];
+  int32_t dims[5];  // B, gamma, n_prompt, n_prefix, hidden states read in place
   float alpha;
   int32_t accept_mode, head_mode;
   float log_eps, log_delta;
   void* stream;
-  bool same(const HostStepKey& o) const { return std::memcmp(this, &o, sizeof(*this)) == 0; }
+  bool same(const HostStepKey& o) const {  // field by field (the struct has padding)
+    return std::memcmp(ptr, o.ptr, sizeof(ptr)) == 0 &&
+           std::memcmp(dims, o.dims, sizeof(dims)) == 0 && alpha == o.alpha &&
+           accept_mode == o.accept_mode && head_mode == o.head_mode && log_eps == o.log_eps &&
+           log_delta == o.log_delta && stream == o.stream;
+  }
 };
 
 struct rv_handle {
@@ -104,8 +109,6 @@ struct rv_handle {
   cudaGraphExec_t host_graph = nullptr;
   unsigned long long graph_launches = 0;  // our kernel launches in the graph
   bool graphs_off = false;                // capture failed once: direct calls only
-  const void* zc_hidden_ptr = nullptr;    // hidden-state buffer last seen, and whether it is
-  bool zc_hidden_ok = false;              // page-locked (read in place by the row gather)
   unsigned profiling = 0;  // bit mask of the regions being recorded
   ProfRegion prof[RV_PROF_COUNT];
   unsigned long long launches = 0;
@@ -1114,11 +1117,9 @@ extern "C" RV_API int rv_verify_step_host(
   // memory), and the row gather reads the hidden states from the caller's
   // buffer when it is page-locked: only q / k_blk / v_blk (and attn_out) go
   // through copies, on the side stream beside the LM head.
-  if (h->zc_hidden_ptr != hidden_host) {
-    h->zc_hidden_ok = pinned(hidden_host);
-    h->zc_hidden_ptr = hidden_host;
-  }
-  const bool zc_hidden = h->zc_hidden_ok;
+  // (asked on every call: a buffer at a known address may have been freed and
+  // replaced by pageable memory)
+  const bool zc_hidden = pinned(hidden_host);
   char* const di = hi;
   char* const dout = h->pin_out;
   const size_t in_bytes = in_small + nh + nq + 2 * nkv;
@@ -1171,6 +1172,7 @@ extern "C" RV_API int rv_verify_step_host(
     key.dims[1] = gamma;
     key.dims[2] = n_prompt;
     key.dims[3] = n_prefix;
+    key.dims[4] = zc_hidden ? 1 : 0;
     key.alpha = alpha;
     key.accept_mode = h->accept_mode;
     key.head_mode = h->head_mode;
@@ -1184,7 +1186,7 @@ extern "C" RV_API int rv_verify_step_host(
       replay = true;
     } else if (h->have_key && key.same(h->last_key) && s != nullptr &&
                pinned(q_host) && pinned(k_blk_host) && pinned(v_blk_host) &&
-               pinned(hidden_host) && (!attn_out_host || pinned(attn_out_host))) {
+               zc_hidden && (!attn_out_host || pinned(attn_out_host))) {
       if (h->host_graph) {
         cudaGraphExecDestroy(h->host_graph);
         h->host_graph = nullptr;

@@ -92,6 +92,12 @@ def test_entry_points_reject_null_handle(rv):
     assert L.rv_set_acceptance(None, 1, 0.09, 0.3) == -1
     assert L.rv_accept_speculative(None, None, None, None, None, None, 1, 1, None, None, None,
                                    None, None, None) == -1
+    assert L.rv_set_head_mode(None, 1) == -1
+    assert L.rv_host_step_graphed(None, None) == -1
+    assert L.rv_accept_sampled(None, None, None, 1.0, 1, 1, None, None, None, None, None,
+                               None, None) == -1
+    assert L.rv_pack_block_pending(None, None, None, None, None, None, 1, 1, 0, 0, None, None,
+                                   None) == -1
     assert L.rv_destroy(None) == 0
 
 

@@ -42,6 +42,8 @@ sys.path.insert(0, ROOT)
 METRIC = "verify-step µs & positions/s at 1 GB300; % of roofline (HBM-bound head/attn)"
 UNIT = "positions/s"
 ALPHA = 0.3
+TYPICAL_EPS, TYPICAL_DELTA = 0.3, 0.09  # --accept typical (the paper gives no values)
+SAMPLED_T = 0.8                         # --accept sampled (Table 4's sampling temperature)
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
 
@@ -355,6 +357,118 @@ def run_sweep(args):
                       "data": "synthetic, seeded on the device"}), flush=True)
 
 
+# ---------------------------------------------------------------------------- rule variants
+
+def run_variant(args):
+    """The step with another acceptance rule (Alg. 3, Alg. 1, sampled Alg. 2)
+    or over the pending-token block, device-timed on one GPU: positions/s,
+    µs per step, and the sampling rules' own launches (their draws over the
+    fused logits) timed alone.  The random numbers the rules draw are inputs,
+    drawn once on the device; the draft distributions of speculative sampling
+    are softmax(N(0, 1)) rows."""
+    import torch
+    from paper_2505_18629_gb300 import rv, synth
+    if args.pending and args.accept in ("speculative", "sampled"):
+        raise SystemExit("--pending runs the exact-match or typical rule")
+    wl = synth.workload(args.workload)
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream(dev)
+    inp = synth.generate(wl)
+    B, g, R, Lb = wl.B, wl.gamma, wl.R, wl.Lb
+
+    def dev_t(x):
+        if x.dtype == np.uint16:
+            return torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).to(dev)
+        return torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+
+    W = dev_t(inp.W)
+    hidden, q, kb, vb = dev_t(inp.hidden), dev_t(inp.q), dev_t(inp.k_blk), dev_t(inp.v_blk)
+    kc, vc = dev_t(inp.k_cache), dev_t(inp.v_cache)
+    ctx = dev_t(inp.ctx_lens.astype(np.int32))
+    prompt = dev_t(inp.prompt_ids.astype(np.int32)) if inp.prompt_ids.size else None
+    prefix = dev_t(inp.prefix_ids.astype(np.int32))
+    h = rv.rv_create(wl.H, wl.V, wl.Hq, wl.Hkv, wl.D, B, g, R, wl.capacity,
+                     rv.RV_DTYPE_BF16 if wl.dtype == "bf16" else rv.RV_DTYPE_F32)
+    if args.head_mode == "preblended":
+        rv.rv_set_head_mode(h, rv.RV_HEAD_PREBLENDED)
+    lead = 1 if args.pending else 0
+    if args.pending:  # one more block position in front (the last emitted token t)
+        q, kb, vb = (torch.cat([x[:, :1], x], dim=1).contiguous() for x in (q, kb, vb))
+    block = torch.empty((B, Lb + lead), dtype=torch.int32, device=dev)
+    pos = torch.empty_like(block)
+    attn = torch.empty_like(q)
+    scores = torch.empty((B, g + 1, rv.RV_NSCORES), device=dev)
+    argmax = torch.empty((B, g + 1), dtype=torch.int32, device=dev)
+    margin = torch.empty((B, g), device=dev)
+    acc = torch.empty((B, g), dtype=torch.uint8, device=dev)
+    alen = torch.empty((B,), dtype=torch.int32, device=dev)
+    nxt = torch.empty_like(alen)
+    ctx_out = torch.empty_like(alen)
+    d0 = torch.zeros((B, g), dtype=torch.int32, device=dev)
+    rv.rv_verify_head(h, hidden, W, d0, g, R, ALPHA, scores, argmax, margin)
+    drafts = dev_t(synth.make_drafts(inp, argmax[:, :g].cpu().numpy()))
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(wl.seed + 7)
+    t_ids = torch.randint(0, wl.V, (B,), generator=gen, device=dev, dtype=torch.int32)
+    if args.accept == "typical":
+        rv.rv_set_acceptance(h, rv.RV_ACCEPT_TYPICAL, TYPICAL_EPS, TYPICAL_DELTA)
+    elif args.accept == "speculative":
+        rv.rv_set_acceptance(h, rv.RV_ACCEPT_SPECULATIVE)
+        q_draft = torch.softmax(torch.randn((B, g, wl.V), generator=gen, device=dev), dim=-1)
+        r_u = torch.rand((B, g), generator=gen, device=dev)
+        u_u = torch.rand((B,), generator=gen, device=dev)
+    elif args.accept == "sampled":
+        rv.rv_set_acceptance(h, rv.RV_ACCEPT_SAMPLED)
+        u_s = torch.rand((B, g + 1), generator=gen, device=dev)
+        sampled = torch.empty((B, g + 1), dtype=torch.int32, device=dev)
+
+    def step():
+        if args.pending:
+            rv.rv_verify_step_pending(h, q, kb, vb, kc, vc, hidden, W, t_ids, drafts, prompt,
+                                      prefix, ctx, ALPHA, block, pos, attn, scores, argmax,
+                                      margin, acc, alen, nxt, ctx_out, stream)
+        elif args.accept == "speculative":
+            rv.rv_verify_step_speculative(h, q, kb, vb, kc, vc, hidden, W, drafts, prompt, prefix,
+                                          ctx, ALPHA, q_draft, r_u, u_u, block, pos, attn, scores,
+                                          argmax, margin, acc, alen, nxt, ctx_out, stream)
+        elif args.accept == "sampled":
+            rv.rv_verify_step_sampled(h, q, kb, vb, kc, vc, hidden, W, drafts, prompt, prefix,
+                                      ctx, ALPHA, SAMPLED_T, u_s, block, pos, attn, scores, argmax,
+                                      margin, sampled, acc, alen, nxt, ctx_out, stream)
+        else:
+            rv.rv_verify_step(h, q, kb, vb, kc, vc, hidden, W, drafts, prompt, prefix, ctx, ALPHA,
+                              block, pos, attn, scores, argmax, margin, acc, alen, nxt, ctx_out,
+                              stream)
+
+    clocks = ClockSampler(0)
+    clocks.start()
+    us = _time_steps(step, args.steps, max(args.warmup, 3), stream)
+    clk = clocks.stop()
+    accept_us = None
+    if args.accept in ("speculative", "sampled"):
+        rv.rv_profile_enable(h, 1 << rv.RV_PROF_ACCEPT)
+        for _ in range(min(args.steps, 100)):
+            step()
+        torch.cuda.synchronize(dev)
+        acc_ms, acc_n = rv.rv_profile_read(h, rv.RV_PROF_ACCEPT)
+        rv.rv_profile_enable(h, 0)
+        accept_us = acc_ms * 1e3 / max(acc_n, 1)
+    st = rv.rv_read_status(h, stream)
+    if st:
+        raise RuntimeError(f"device status 0x{st:x}")
+    units = B * (Lb + lead)
+    print(json.dumps({
+        "metric": METRIC, "value": units / (us * 1e-6), "unit": UNIT, "n_gpus": 1,
+        "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": us * 1e-3,
+        "higher_is_better": True, "dtype": "bf16" if wl.dtype == "bf16" else "f32",
+        "data": "synthetic", "step_us": us, "accept_launches_us": accept_us,
+        "mean_accepted": float(alen.float().mean().item()),
+        "config": dict(_config(wl, 1, args.head_mode), accept=args.accept, pending=args.pending),
+        "clocks": clk}), flush=True)
+    h.close()
+
+
 # ---------------------------------------------------------------------------- main arm
 
 def main():
@@ -370,6 +484,14 @@ def main():
     ap.add_argument("--head-mode", default="fused", choices=["fused", "preblended"],
                     help="fused: both logit vectors fused per vocab row (Eq. 2); preblended: "
                          "the head on the blended hidden states (one row per position)")
+    ap.add_argument("--accept", default="exact",
+                    choices=["exact", "typical", "speculative", "sampled"],
+                    help="acceptance rule of the step: exact match (Alg. 2, default), typical "
+                         "(Alg. 3), speculative sampling (Alg. 1), exact match against sampled "
+                         "target tokens (Alg. 2 at temperature T); other than exact, or with "
+                         "--pending, one JSON line of the step's device time")
+    ap.add_argument("--pending", action="store_true",
+                    help="the pending-token block [t, x, template, x] (exact or typical rule)")
     ap.add_argument("--sweep", action="store_true",
                     help="time the 8B sweep (reflective, alpha = 0, standard) instead")
     ap.add_argument("--sweep-points", default="",
@@ -380,6 +502,11 @@ def main():
         if args.steps == 2000:
             args.steps = 50
         run_sweep(args)
+        return
+    if args.accept != "exact" or args.pending:
+        if args.steps == 2000:
+            args.steps = 500
+        run_variant(args)
         return
 
     from paper_2505_18629_gb300 import synth

@@ -371,6 +371,8 @@ def run_variant(args):
     if args.pending and args.accept in ("speculative", "sampled"):
         raise SystemExit("--pending runs the exact-match or typical rule")
     wl = synth.workload(args.workload)
+    if args.pending:  # the cache takes the block and the pending token
+        wl = wl.replace(cmax=wl.ctx[1] + wl.Lb + 1)
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     stream = torch.cuda.current_stream(dev)

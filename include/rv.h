@@ -296,17 +296,21 @@ RV_API int rv_accept_sampled(rv_handle* h, const int32_t* draft_ids, const float
                              uint8_t* accept_mask, int32_t* accepted_len, int32_t* next_token,
                              const int32_t* ctx_in, int32_t* ctx_out, void* stream);
 
-/* The whole verify step on device buffers, in one call and four kernel
- * launches: the attention (rv_verify_attention) on an internal stream forked
- * from `stream`, concurrently with -- on `stream` -- one launch that gathers
- * the LM-head rows and packs the block (rv_pack_block; skipped when block_ids
- * is NULL), the LM head, and one launch that merges the head's statistics and
+/* The whole verify step on device buffers, in one call and three to five
+ * kernel launches: on `stream`, one launch that gathers the LM-head rows and
+ * packs the block (rv_pack_block; skipped when block_ids is NULL), the LM head
+ * and, above 64 positions, one launch that merges the head's statistics and
  * runs the acceptance (rv_accept, or rv_accept_typical when the handle's rule
- * is RV_ACCEPT_TYPICAL; see rv_set_acceptance).  The internal stream is joined back into
- * `stream` before the call returns, so later work on `stream` sees every
- * output; the pattern is also valid inside stream capture.  Arguments as in those
- * calls; the template is n_prompt prompt ids + n_prefix prefix ids, so
- * R = n_prompt + n_prefix and Lb = 2*gamma + R.  ctx_out may alias ctx_in. */
+ * is RV_ACCEPT_TYPICAL; see rv_set_acceptance; with fewer positions the head's
+ * last CTA does it); the attention (rv_verify_attention) on an internal stream
+ * forked from `stream` after the head's launch, beside it -- except the
+ * persistent tcgen05 attention of handles whose KV capacity exceeds 4608
+ * positions, which runs first, on `stream`.  The internal stream is joined
+ * back into `stream` before the call returns, so later work on `stream` sees
+ * every output; the pattern is also valid inside stream capture.  Arguments as
+ * in those calls; the template is n_prompt prompt ids + n_prefix prefix ids,
+ * so R = n_prompt + n_prefix and Lb = 2*gamma + R (Lb = gamma, no template,
+ * for RV_HEAD_STANDARD).  ctx_out may alias ctx_in. */
 RV_API int rv_verify_step(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
                           void* k_cache, void* v_cache, const void* hidden, const void* w_head,
                           const int32_t* draft_ids, const int32_t* prompt_ids,

@@ -751,7 +751,7 @@ def test_sampled_exact_match_kernels_and_8b(gu, name):
         _check_sampled(inp, z, u, drafts, 0.8, gpu)
 
 
-# ------------------------------------------------------------------ pending-token block (NEXT 3)
+# ------------------------------------------------------------------ pending-token block
 
 def _pending_run(gu, wl, alpha=ALPHA, seed=0, check_attn=True):
     """rv_verify_step_pending against the oracle's verify_step_pending.  The
@@ -832,7 +832,7 @@ def test_pending_token_step_8b_b16(gu):
     _pending_run(gu, synth.WORKLOADS["llama3-8b-b16"], seed=103)
 
 
-# ------------------------------------------------------------------ pre-blended head (NEXT 3)
+# ------------------------------------------------------------------ pre-blended head
 
 @pytest.mark.parametrize("shape", ["ragged", "one-pair", "pairs-144", "two-chunks"])
 def test_preblended_head(gu, shape):

@@ -950,3 +950,18 @@ def test_pins_catch_standard_block_with_copy(monkeypatch):
     monkeypatch.setattr(orc, "pack_block_standard", with_copy)
     with pytest.raises(AssertionError):
         test_standard_block_closed_form_and_first_segment()
+
+
+def test_pins_catch_inverse_cdf_slips(monkeypatch):
+    # one token early (the last v whose cumulative weight is still below u * sum)
+    real = orc.inverse_cdf_sample
+    monkeypatch.setattr(orc, "inverse_cdf_sample", lambda w, u: max(0, real(w, u) - 1))
+    with pytest.raises(AssertionError):
+        test_inverse_cdf_sample_closed_forms()
+    # u compared against unnormalised cumulative weights
+    def unscaled(w, u):
+        c = np.cumsum(np.asarray(w, np.float64))
+        return int(min(np.searchsorted(c, u, side="right"), len(c) - 1))
+    monkeypatch.setattr(orc, "inverse_cdf_sample", unscaled)
+    with pytest.raises(AssertionError):
+        test_inverse_cdf_sample_closed_forms()

@@ -27,14 +27,6 @@
 //               empty-accumulator barrier
 // The pair streams a static range of 256-row vocab tiles; the weight streams
 // from HBM once per chunk (evict-first), the hidden rows are re-read from L2.
-//
-// With two pair chunks (MC = 2) the two pairs that take the same vocab tiles
-// for the two chunks form one cluster of four CTAs (cluster ranks 0,1: chunk 0;
-// 2,3: chunk 1) and share the weight tiles: CTA r of each pair loads one
-// 64-wide K half of its 128 weight rows and multicasts it to CTA r of both
-// pairs, so each weight byte leaves L2 once instead of once per chunk.  A
-// stage is then refilled only after both pairs' MMAs released it (its empty
-// barrier takes one commit from each pair).
 #include <cfloat>
 
 #include "head_epilogue.cuh"
@@ -128,20 +120,6 @@ __device__ __forceinline__ void tc2_mma_stage8(uint32_t d_tmem, uint64_t a_desc,
       : "memory");
 }
 
-// As tma_load_2d_pair, multicast to the CTAs of `mask` (same shared-memory
-// offset in each); each destination's bytes complete on the barrier at the
-// offset of `bar_cluster` in the even CTA of that destination's pair.
-__device__ __forceinline__ void tma_load_2d_pair_mc(uint32_t dst, const CUtensorMap* tm, int32_t x,
-                                                    int32_t y, uint32_t bar_cluster, uint16_t mask,
-                                                    uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
-      ".multicast::cluster.L2::cache_hint [%0], [%1, {%2, %3}], [%4], %5, %6;" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(tm)), "r"(x), "r"(y), "r"(bar_cluster), "h"(mask),
-      "l"(policy)
-      : "memory");
-}
-
 // Arrive on the barrier at `bar` in every CTA of `mask` once the MMAs issued
 // so far by this thread are complete.
 __device__ __forceinline__ void tc2_commit(uint32_t bar, uint16_t mask) {
@@ -154,7 +132,7 @@ __device__ __forceinline__ void tc2_commit(uint32_t bar, uint16_t mask) {
 
 }  // namespace
 
-template <int EPI, int MC>
+template <int EPI>
 __global__ void __launch_bounds__(h2_threads(EPI), 1)
     head_tc2_kernel(const __grid_constant__ CUtensorMap tm_w,
                     const __grid_constant__ CUtensorMap tm_h, const Head2Params p) {
@@ -170,10 +148,8 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
   const uint32_t crank = cluster_ctarank();
   const uint32_t rank = crank & 1u;  // 0: the pair's MMA issuer
   const bool leader = rank == 0;
-  // commit masks: this pair's two CTAs; the stage release goes to every CTA
-  // of the cluster (MC = 2: both pairs refill each stage)
+  // commit mask: this pair's two CTAs (the stage release and the accumulator)
   const uint16_t pair_mask = static_cast<uint16_t>(3u << (crank & ~1u));
-  const uint16_t empty_mask = MC == 2 ? static_cast<uint16_t>(0xF) : pair_mask;
   const int pair = blockIdx.x >> 1;
   const int chunk = blockIdx.y;
   const int slot_id = blockIdx.x;  // partial slot within the chunk
@@ -210,7 +186,7 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(full_bar(s), 1);   // the even CTA's expect-tx; both CTAs' bytes
-      mbar_init(empty_bar(s), MC);  // the MMA commit of each pair sharing the stage
+      mbar_init(empty_bar(s), 1);  // the pair's MMA commit
     }
     mbar_init(accf0, 1);
     mbar_init(accf0 + 8, 1);
@@ -263,18 +239,10 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
           if (leader) mbar_arrive_expect_tx(full_bar(s), 2u * (H2_A_BYTES + b_bytes));
           const uint32_t fb = mapa_shared(full_bar(s), leader_rank);
           const int hrow = chunk * p.N + static_cast<int>(rank) * (p.N / 2);
-          if (MC == 2) {
-            // weight half `chunk` of this CTA's rows, to CTA `rank` of both pairs
-            const int hf = chunk;
-            tma_load_2d_pair_mc(a_tiles + s * H2_A_BYTES + hf * H2_A_HALF, &tm_w,
-                                kb * H2_BK + 64 * hf, v0, fb,
-                                static_cast<uint16_t>((1u << rank) | (1u << (rank + 2))), pol_w);
-          }
 #pragma unroll
           for (int hf = 0; hf < 2; ++hf) {
-            if (MC == 1)
-              tma_load_2d_pair(a_tiles + s * H2_A_BYTES + hf * H2_A_HALF, &tm_w,
-                               kb * H2_BK + 64 * hf, v0, fb, pol_w);
+            tma_load_2d_pair(a_tiles + s * H2_A_BYTES + hf * H2_A_HALF, &tm_w, kb * H2_BK + 64 * hf,
+                             v0, fb, pol_w);
             tma_load_2d_pair(b_tiles + s * b_bytes + hf * b_half, &tm_h, kb * H2_BK + 64 * hf, hrow,
                              fb, pol_h);
           }
@@ -287,10 +255,9 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
       }
       // after an abort the even CTA lets every copy of the pair still in flight
       // land (its full barriers count both CTAs' bytes) before the final
-      // cluster barrier releases the odd CTA; with MC = 2 the other pair may
-      // have issued up to S more stages' weight halves into this pair
+      // cluster barrier releases the odd CTA
       if (!ok && leader) {
-        for (int j = max(0, issued - S); j < issued + (MC - 1) * S; ++j)
+        for (int j = max(0, issued - S); j < issued; ++j)
           drain_wait(full_bar(j % S), static_cast<uint32_t>((j / S) & 1));
       }
     }
@@ -322,7 +289,7 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
           const uint64_t ad = ad0 + static_cast<uint32_t>(s) * a_step;
           const uint64_t bd = bd0 + static_cast<uint32_t>(s) * b_step;
           tc2_mma_stage8(d_tmem, ad, bd, a_hstep, b_hstep, idesc, kb != 0 ? 1u : 0u);
-          tc2_commit(empty_bar(s), empty_mask);
+          tc2_commit(empty_bar(s), pair_mask);
           if (++s == S) {
             s = 0;
             ph ^= 1u;
@@ -445,45 +412,40 @@ int head_tc2_stages(int N, int pairs, size_t smem_limit) {
   return std::max(0, std::min(std::min(most, 8), std::max(3, want)));
 }
 
-template <int EPI, int MC>
+template <int EPI>
 static cudaError_t head_tc2_configure_one(size_t smem_bytes) {
-  cudaError_t e = cudaFuncSetAttribute(head_tc2_kernel<EPI, MC>,
+  cudaError_t e = cudaFuncSetAttribute(head_tc2_kernel<EPI>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem_bytes));
   if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(head_tc2_kernel<EPI, MC>,
+  e = cudaFuncSetAttribute(head_tc2_kernel<EPI>,
                            cudaFuncAttributePreferredSharedMemoryCarveout,
                            cudaSharedmemCarveoutMaxShared);
   return e;
 }
 
 cudaError_t head_tc2_configure(size_t smem_bytes) {
-  cudaError_t e = head_tc2_configure_one<4, 1>(smem_bytes);
-  if (e == cudaSuccess) e = head_tc2_configure_one<8, 1>(smem_bytes);
-  if (e == cudaSuccess) e = head_tc2_configure_one<4, 2>(smem_bytes);
-  if (e == cudaSuccess) e = head_tc2_configure_one<8, 2>(smem_bytes);
+  cudaError_t e = head_tc2_configure_one<4>(smem_bytes);
+  if (e == cudaSuccess) e = head_tc2_configure_one<8>(smem_bytes);
   return e;
 }
 
-int head_tc2_max_pairs(int N, int pairs, int stages, int mc) {
+int head_tc2_max_pairs(int N, int pairs, int stages) {
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(2, mc, 1);
+  cfg.gridDim = dim3(2, 1, 1);
   cfg.blockDim = dim3(h2_threads(h2_epi_warps(pairs)), 1, 1);
   cfg.dynamicSmemBytes = head_tc2_smem_bytes(N, pairs, stages);
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
-  attr[0].val.clusterDim.y = mc;
+  attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int n = 0;
   const bool e4 = h2_epi_warps(pairs) == 4;
-  cudaError_t e =
-      mc == 2 ? (e4 ? cudaOccupancyMaxActiveClusters(&n, head_tc2_kernel<4, 2>, &cfg)
-                    : cudaOccupancyMaxActiveClusters(&n, head_tc2_kernel<8, 2>, &cfg))
-              : (e4 ? cudaOccupancyMaxActiveClusters(&n, head_tc2_kernel<4, 1>, &cfg)
-                    : cudaOccupancyMaxActiveClusters(&n, head_tc2_kernel<8, 1>, &cfg));
+  cudaError_t e = e4 ? cudaOccupancyMaxActiveClusters(&n, head_tc2_kernel<4>, &cfg)
+                     : cudaOccupancyMaxActiveClusters(&n, head_tc2_kernel<8>, &cfg);
   if (e != cudaSuccess) {
     cudaGetLastError();
     return 0;
@@ -523,22 +485,17 @@ cudaError_t launch_head_tc2(const HeadArgs& a, const HeadPlan& pl, const HeadTcL
   cfg.blockDim = dim3(h2_threads(epi), 1, 1);
   cfg.dynamicSmemBytes = l.smem_bytes;
   cfg.stream = s;
-  const int mc = pl.multicast ? 2 : 1;  // the two chunks' pairs of a vocab range in one cluster
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   attr[1].id = cudaLaunchAttributeClusterDimension;
   attr[1].val.clusterDim.x = 2;
-  attr[1].val.clusterDim.y = mc;
+  attr[1].val.clusterDim.y = 1;
   attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  if (mc == 2) {
-    if (epi == 4) return cudaLaunchKernelEx(&cfg, head_tc2_kernel<4, 2>, l.tm_w, l.tm_h, p);
-    return cudaLaunchKernelEx(&cfg, head_tc2_kernel<8, 2>, l.tm_w, l.tm_h, p);
-  }
-  if (epi == 4) return cudaLaunchKernelEx(&cfg, head_tc2_kernel<4, 1>, l.tm_w, l.tm_h, p);
-  return cudaLaunchKernelEx(&cfg, head_tc2_kernel<8, 1>, l.tm_w, l.tm_h, p);
+  if (epi == 4) return cudaLaunchKernelEx(&cfg, head_tc2_kernel<4>, l.tm_w, l.tm_h, p);
+  return cudaLaunchKernelEx(&cfg, head_tc2_kernel<8>, l.tm_w, l.tm_h, p);
 }
 
 }  // namespace rv

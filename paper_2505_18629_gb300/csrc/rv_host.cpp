@@ -118,7 +118,6 @@ struct rv_handle {
   int head_pair_cached_N = -1;   // pair kernel: stages and co-resident pairs for this N
   int head_pair_stages = 0;
   int head_pair_max = 0;
-  int head_pair_max4 = 0;        // co-resident clusters of two pairs (weight multicast)
   int tm_h_box = -1;
   bool attn_tc_ok = false;  // tcgen05 attention usable for this configuration
   // acceptance rule of rv_verify_step (rv_set_acceptance)
@@ -597,26 +596,14 @@ int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_
       h->head_pair_max = h->head_pair_stages >= 2
                              ? head_tc2_max_pairs(pl.N, pl.pad_pairs, h->head_pair_stages)
                              : 0;
-      h->head_pair_max4 = h->head_pair_stages >= 2
-                              ? head_tc2_max_pairs(pl.N, pl.pad_pairs, h->head_pair_stages, 2)
-                              : 0;
       h->head_pair_cached_N = 2 * pl.N + pl.zonly;
     }
     const int n_pt = (c.vocab + 255) / 256;
-    if (pl.n_chunks == 2 && pl.N >= RV_HEAD2_MULTICAST_MIN_N && h->head_pair_max4 >= 1) {
-      // the two chunks' pairs of each vocab range in one cluster of four CTAs,
-      // sharing the weight tiles by multicast
-      const int pairs = std::min({h->num_sms / 4, h->head_pair_max4, n_pt});
+    const int pairs =
+        std::min({h->num_sms / 2 / pl.n_chunks, h->head_pair_max / pl.n_chunks, n_pt});
+    if (pairs >= 1) {
       pl.pair = true;
-      pl.multicast = true;
       pl.slots = 2 * pairs;
-    } else {
-      const int pairs =
-          std::min({h->num_sms / 2 / pl.n_chunks, h->head_pair_max / pl.n_chunks, n_pt});
-      if (pairs >= 1) {
-        pl.pair = true;
-        pl.slots = 2 * pairs;
-      }
     }
   }
   ProfScope prof_all(h, RV_PROF_HEAD, s);

@@ -45,7 +45,6 @@ struct HeadPlan {
   int n_vtiles;        // ceil(V / 128)
   int slots;           // CTAs per chunk (= partial slots)
   bool pair;           // CTA-pair kernel (k_head_tc2.cu): slots = 2 * pairs
-  bool multicast = false;  // pair kernel, two chunks: clusters of 4 share the weight tiles
   bool zonly = false;  // pre-blended head: one blended row per pair, z statistics only
   bool standard = false;  // standard verification: z-only on the original rows (Lh = gamma+1)
 };
@@ -178,17 +177,11 @@ cudaError_t launch_head_simt(const HeadArgs& a, const HeadPlan& p, cudaStream_t 
 #define RV_HEAD_PAIR_MIN_N 96
 #endif
 constexpr int HEAD_PAIR_MIN_N = RV_HEAD_PAIR_MIN_N;  // N from which pairs are used
-// Two chunks of at least this N: clusters of two pairs share the weight tiles
-// by multicast (measured: 70B B=32, N = 224: 618 -> 585 us; 8B B=16, N = 144:
-// 264 -> 270 us, so not there).
-#ifndef RV_HEAD2_MULTICAST_MIN_N
-#define RV_HEAD2_MULTICAST_MIN_N 192
-#endif
 size_t head_tc2_smem_bytes(int N, int pairs, int stages);
 int head_tc2_stages(int N, int pairs, size_t smem_limit);
 cudaError_t head_tc2_configure(size_t smem_bytes);
-// co-resident clusters of `mc` CTA pairs (occupancy query)
-int head_tc2_max_pairs(int N, int pairs, int stages, int mc = 1);
+// co-resident CTA pairs (occupancy query)
+int head_tc2_max_pairs(int N, int pairs, int stages);
 
 cudaError_t launch_head_tc2(const HeadArgs& a, const HeadPlan& p, const HeadTcLaunch& l,
                             const HeadFinal* fin, cudaStream_t s);

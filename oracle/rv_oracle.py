@@ -424,10 +424,16 @@ def typical_accept(drafts, logp_fused, ent_orig, choice, eps: float, delta: floa
 
 def inverse_cdf_sample(w: np.ndarray, u: float) -> int:
     """The token drawn from the distribution proportional to w >= 0 by one
-    uniform u in [0, 1): the smallest v whose cumulative weight exceeds u * sum(w)."""
+    uniform u in [0, 1): the smallest v whose cumulative weight exceeds u * sum(w).
+    If no cumulative weight exceeds it (u = 1, outside the domain), the draw is
+    the last token of positive weight: a token of zero weight is never drawn."""
     w = np.asarray(w, np.float64)
     c = np.cumsum(w)
-    return int(min(np.searchsorted(c, u * c[-1], side="right"), len(w) - 1))
+    v = int(np.searchsorted(c, u * c[-1], side="right"))
+    if v >= len(w):
+        pos = np.flatnonzero(w > 0)
+        v = int(pos[-1]) if pos.size else len(w) - 1
+    return v
 
 
 def speculative_accept(drafts, z, q, r, u):

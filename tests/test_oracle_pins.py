@@ -499,6 +499,10 @@ def test_inverse_cdf_sample_closed_forms():
     assert orc.inverse_cdf_sample(w, 0.4001) == 3
     assert orc.inverse_cdf_sample(w, 0.999999) == 3
     assert orc.inverse_cdf_sample(5.0 * w, 0.25) == 2       # scale-free
+    # weights ending in zeros: the top of the range takes the last weighted token
+    tail0 = np.array([0.5, 0.5, 0.0])
+    assert orc.inverse_cdf_sample(tail0, np.nextafter(1.0, 0.0)) == 1
+    assert orc.inverse_cdf_sample(tail0, 1.0) == 1
     # a midpoint grid of u reproduces w / sum(w) exactly
     grid = (np.arange(1000) + 0.5) / 1000
     hits = np.bincount([orc.inverse_cdf_sample(w, x) for x in grid], minlength=4) / 1000

@@ -129,12 +129,169 @@ def _stream(stream):
     return ctypes.c_void_p(int(stream))
 
 
+# ------------------------------------------------------------------ argument checks
+# The C entry points take bare pointers, so they cannot see a tensor's size: a
+# hidden-state tensor with too few rows would be read past its end on the
+# device.  Every wrapper therefore checks shapes and element types against the
+# sizes it passes (and the handle's configuration) and raises ValueError before
+# anything is launched.
+
+def _expect(name, t, shape, dtype, device=True, min_first=False):
+    """One tensor: shape (first dimension at least shape[0] with min_first),
+    dtype, contiguity and, unless device is None, device (True) or host
+    (False) memory."""
+    if t is None:
+        raise ValueError(f"{name} is required")
+    if not isinstance(t, torch.Tensor):
+        raise ValueError(f"{name} must be a torch.Tensor")
+    got = tuple(t.shape)
+    want = tuple(int(x) for x in shape)
+    if min_first:
+        ok = len(got) == len(want) and got[0] >= want[0] and got[1:] == want[1:]
+    else:
+        ok = got == want
+    if not ok:
+        lead = ">= " if min_first else ""
+        raise ValueError(f"{name} has shape {list(got)}, expected {lead}{list(want)}")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} has dtype {t.dtype}, expected {dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if device is not None and t.is_cuda != device:
+        raise ValueError(f"{name} must be in {'device' if device else 'host'} memory")
+
+
+class _Checks:
+    """Shapes and dtypes of every tensor first, then where each one lives, so
+    that a wrong shape is reported as such whatever the memory."""
+
+    def __init__(self):
+        self._where = []
+
+    def __call__(self, name, t, shape, dtype, device=True, min_first=False):
+        _expect(name, t, shape, dtype, None, min_first)
+        self._where.append((name, t, device))
+
+    def placed(self):
+        for name, t, device in self._where:
+            if device is not None and t.is_cuda != device:
+                raise ValueError(f"{name} must be in {'device' if device else 'host'} memory")
+
+
+def _block_len(h, gamma, R):
+    """Block positions without the pending token: [x, template, x], or the
+    drafts alone for standard verification."""
+    return gamma if h.head_mode == RV_HEAD_STANDARD else 2 * gamma + R
+
+
+def _check_head(h, hidden, w_head, draft_ids, gamma, R, scores, argmax, margin, device=True,
+                ck=None):
+    own = ck is None
+    ck = _Checks() if own else ck
+    c = h.cfg
+    act = h.act_dtype
+    if hidden is None or hidden.dim() != 3:
+        raise ValueError("hidden must be [B, Lb + 1, H]")
+    B = hidden.shape[0]
+    ck("hidden", hidden, (B, _block_len(h, gamma, R) + 1, c.hidden), act, device)
+    ck("w_head", w_head, (c.vocab, c.hidden), act, True)
+    ck("draft_ids", draft_ids, (B, gamma), torch.int32, device)
+    ck("scores", scores, (B, gamma + 1, RV_NSCORES), torch.float32, device)
+    ck("argmax", argmax, (B, gamma + 1), torch.int32, device)
+    ck("margin", margin, (B, gamma), torch.float32, device)
+    if own:
+        ck.placed()
+    return B
+
+
+def _check_attention(h, q, k_blk, v_blk, k_cache, v_cache, ctx_lens, out, B, Lq, device=True,
+                     ck=None):
+    own = ck is None
+    ck = _Checks() if own else ck
+    c = h.cfg
+    act = h.act_dtype
+    ck("q", q, (B, Lq, c.n_q_heads, c.head_dim), act, device)
+    ck("k_blk", k_blk, (B, Lq, c.n_kv_heads, c.head_dim), act, device)
+    ck("v_blk", v_blk, (B, Lq, c.n_kv_heads, c.head_dim), act, device)
+    ck("k_cache", k_cache, (B, c.n_kv_heads, c.max_ctx, c.head_dim), act, True, min_first=True)
+    ck("v_cache", v_cache, (B, c.n_kv_heads, c.max_ctx, c.head_dim), act, True, min_first=True)
+    ck("ctx_lens", ctx_lens, (B,), torch.int32, device)
+    if out is not None:
+        ck("attn_out", out, (B, Lq, c.n_q_heads, c.head_dim), act, device)
+    if own:
+        ck.placed()
+
+
+def _check_ids(B, gamma, draft_ids, prompt_ids, prefix_ids, device=True, ck=None):
+    own = ck is None
+    ck = _Checks() if own else ck
+    ck("draft_ids", draft_ids, (B, gamma), torch.int32, device)
+    if prompt_ids is not None:
+        ck("prompt_ids", prompt_ids, (prompt_ids.numel(),), torch.int32, device)
+    if prefix_ids is None or prefix_ids.dim() != 2:
+        raise ValueError("prefix_ids must be [B, n_prefix]")
+    ck("prefix_ids", prefix_ids, (B, prefix_ids.shape[1]), torch.int32, device)
+    if own:
+        ck.placed()
+
+
+def _check_accept_out(B, gamma, accept_mask, accepted_len, next_token, ctx_in, ctx_out,
+                      device=True, ck=None):
+    own = ck is None
+    ck = _Checks() if own else ck
+    ck("accept_mask", accept_mask, (B, gamma), torch.uint8, device)
+    ck("accepted_len", accepted_len, (B,), torch.int32, device)
+    ck("next_token", next_token, (B,), torch.int32, device)
+    ck("ctx_in", ctx_in, (B,), torch.int32, device)
+    ck("ctx_out", ctx_out, (B,), torch.int32, device)
+    if own:
+        ck.placed()
+
+
+def _check_step(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, prompt_ids,
+                prefix_ids, ctx_in, block_ids, pos_ids, attn_out, scores, argmax, margin,
+                accept_mask, accepted_len, next_token, ctx_out, lead=0, device=True):
+    """Shapes of a whole step; lead = 1 for the pending-token block."""
+    if draft_ids is None or draft_ids.dim() != 2:
+        raise ValueError("draft_ids must be [B, gamma]")
+    ck = _Checks()
+    B, gamma = draft_ids.shape
+    _check_ids(B, gamma, draft_ids, prompt_ids, prefix_ids, device, ck)
+    n_prompt = 0 if prompt_ids is None else prompt_ids.numel()
+    R = n_prompt + prefix_ids.shape[1]
+    Lq = _block_len(h, gamma, R) + lead
+    _check_attention(h, q, k_blk, v_blk, k_cache, v_cache, ctx_in, attn_out, B, Lq, device, ck)
+    _check_head(h, hidden, w_head, draft_ids, gamma, R, scores, argmax, margin, device, ck)
+    if block_ids is not None or pos_ids is not None:
+        ck("block_ids", block_ids, (B, Lq), torch.int32, device)
+        ck("pos_ids", pos_ids, (B, Lq), torch.int32, device)
+    _check_accept_out(B, gamma, accept_mask, accepted_len, next_token, ctx_in, ctx_out, device, ck)
+    ck.placed()
+
+
+def _check_speculative_inputs(h, B, gamma, q_draft, r_uniform, u_uniform):
+    _expect("q_draft", q_draft, (B, gamma, h.cfg.vocab), torch.float32)
+    _expect("r_uniform", r_uniform, (B, gamma), torch.float32)
+    _expect("u_uniform", u_uniform, (B,), torch.float32)
+
+
+def _check_sampled_inputs(B, gamma, u_uniform, sampled):
+    _expect("u_uniform", u_uniform, (B, gamma + 1), torch.float32)
+    _expect("sampled", sampled, (B, gamma + 1), torch.int32)
+
+
 class Handle:
     """Owns an ``rv_handle*``; ``close()`` (or garbage collection) destroys it."""
 
     def __init__(self, ptr, cfg):
         self._p = ptr
         self.cfg = cfg
+        self.head_mode = RV_HEAD_FUSED_LOGITS  # last mode set by rv_set_head_mode
+
+    @property
+    def act_dtype(self):
+        """Element type of hidden states, weight, q/k/v and caches."""
+        return torch.bfloat16 if self.cfg.dtype == RV_DTYPE_BF16 else torch.float32
 
     @property
     def ptr(self):
@@ -184,8 +341,13 @@ def rv_workspace_bytes(h: Handle) -> int:
 def rv_pack_block(h, draft_ids, prompt_ids, prefix_ids, ctx_lens, block_ids, pos_ids,
                   stream=None):
     B, gamma = draft_ids.shape
+    _check_ids(B, gamma, draft_ids, prompt_ids, prefix_ids)
     n_prompt = 0 if prompt_ids is None else prompt_ids.numel()
     n_prefix = prefix_ids.shape[1]
+    Lb = _block_len(h, gamma, n_prompt + n_prefix)
+    _expect("ctx_lens", ctx_lens, (B,), torch.int32)
+    _expect("block_ids", block_ids, (B, Lb), torch.int32)
+    _expect("pos_ids", pos_ids, (B, Lb), torch.int32)
     _check(h, _lib.rv_pack_block(h.ptr, _ptr(draft_ids), _ptr(prompt_ids), _ptr(prefix_ids),
                                  _ptr(ctx_lens), B, gamma, n_prompt, n_prefix, _ptr(block_ids),
                                  _ptr(pos_ids), _stream(stream)))
@@ -194,8 +356,14 @@ def rv_pack_block(h, draft_ids, prompt_ids, prefix_ids, ctx_lens, block_ids, pos
 def rv_pack_block_pending(h, pending_ids, draft_ids, prompt_ids, prefix_ids, ctx_lens, block_ids,
                           pos_ids, stream=None):
     B, gamma = draft_ids.shape
+    _check_ids(B, gamma, draft_ids, prompt_ids, prefix_ids)
     n_prompt = 0 if prompt_ids is None else prompt_ids.numel()
     n_prefix = prefix_ids.shape[1]
+    Lb = _block_len(h, gamma, n_prompt + n_prefix)
+    _expect("pending_ids", pending_ids, (B,), torch.int32)
+    _expect("ctx_lens", ctx_lens, (B,), torch.int32)
+    _expect("block_ids", block_ids, (B, Lb + 1), torch.int32)
+    _expect("pos_ids", pos_ids, (B, Lb + 1), torch.int32)
     _check(h, _lib.rv_pack_block_pending(h.ptr, _ptr(pending_ids), _ptr(draft_ids),
                                          _ptr(prompt_ids), _ptr(prefix_ids), _ptr(ctx_lens), B,
                                          gamma, n_prompt, n_prefix, _ptr(block_ids), _ptr(pos_ids),
@@ -203,7 +371,12 @@ def rv_pack_block_pending(h, pending_ids, draft_ids, prompt_ids, prefix_ids, ctx
 
 
 def rv_verify_attention(h, q, k_blk, v_blk, k_cache, v_cache, ctx_lens, out, stream=None):
+    if q is None or q.dim() != 4:
+        raise ValueError("q must be [B, Lb, Hq, D]")
     B, Lb = q.shape[0], q.shape[1]
+    _check_attention(h, q, k_blk, v_blk, k_cache, v_cache, ctx_lens, out, B, Lb)
+    if out is None:
+        raise ValueError("out is required")
     _check(h, _lib.rv_verify_attention(h.ptr, _ptr(q), _ptr(k_blk), _ptr(v_blk), _ptr(k_cache),
                                        _ptr(v_cache), _ptr(ctx_lens), B, Lb, _ptr(out),
                                        _stream(stream)))
@@ -211,7 +384,7 @@ def rv_verify_attention(h, q, k_blk, v_blk, k_cache, v_cache, ctx_lens, out, str
 
 def rv_verify_head(h, hidden, w_head, draft_ids, gamma, R, alpha, scores, argmax, margin,
                    stream=None):
-    B = hidden.shape[0]
+    B = _check_head(h, hidden, w_head, draft_ids, gamma, R, scores, argmax, margin)
     _check(h, _lib.rv_verify_head(h.ptr, _ptr(hidden), _ptr(w_head), _ptr(draft_ids), B, gamma,
                                   R, float(alpha), _ptr(scores), _ptr(argmax), _ptr(margin),
                                   _stream(stream)))
@@ -220,6 +393,9 @@ def rv_verify_head(h, hidden, w_head, draft_ids, gamma, R, alpha, scores, argmax
 def rv_accept(h, draft_ids, argmax, accept_mask, accepted_len, next_token, ctx_in, ctx_out,
               stream=None):
     B, gamma = draft_ids.shape
+    _expect("draft_ids", draft_ids, (B, gamma), torch.int32)
+    _expect("argmax", argmax, (B, gamma + 1), torch.int32)
+    _check_accept_out(B, gamma, accept_mask, accepted_len, next_token, ctx_in, ctx_out)
     _check(h, _lib.rv_accept(h.ptr, _ptr(draft_ids), _ptr(argmax), B, gamma, _ptr(accept_mask),
                              _ptr(accepted_len), _ptr(next_token), _ptr(ctx_in), _ptr(ctx_out),
                              _stream(stream)))
@@ -228,6 +404,10 @@ def rv_accept(h, draft_ids, argmax, accept_mask, accepted_len, next_token, ctx_i
 def rv_accept_typical(h, draft_ids, scores, argmax, eps, delta, accept_mask, accepted_len,
                       next_token, ctx_in, ctx_out, stream=None):
     B, gamma = draft_ids.shape
+    _expect("draft_ids", draft_ids, (B, gamma), torch.int32)
+    _expect("scores", scores, (B, gamma + 1, RV_NSCORES), torch.float32)
+    _expect("argmax", argmax, (B, gamma + 1), torch.int32)
+    _check_accept_out(B, gamma, accept_mask, accepted_len, next_token, ctx_in, ctx_out)
     _check(h, _lib.rv_accept_typical(h.ptr, _ptr(draft_ids), _ptr(scores), _ptr(argmax), B, gamma,
                                      float(eps), float(delta), _ptr(accept_mask),
                                      _ptr(accepted_len), _ptr(next_token), _ptr(ctx_in),
@@ -237,6 +417,10 @@ def rv_accept_typical(h, draft_ids, scores, argmax, eps, delta, accept_mask, acc
 def rv_accept_speculative(h, draft_ids, q_draft, r_uniform, u_uniform, scores, accept_mask,
                           accepted_len, next_token, ctx_in, ctx_out, stream=None):
     B, gamma = draft_ids.shape
+    _expect("draft_ids", draft_ids, (B, gamma), torch.int32)
+    _check_speculative_inputs(h, B, gamma, q_draft, r_uniform, u_uniform)
+    _expect("scores", scores, (B, gamma + 1, RV_NSCORES), torch.float32)
+    _check_accept_out(B, gamma, accept_mask, accepted_len, next_token, ctx_in, ctx_out)
     _check(h, _lib.rv_accept_speculative(h.ptr, _ptr(draft_ids), _ptr(q_draft), _ptr(r_uniform),
                                          _ptr(u_uniform), _ptr(scores), B, gamma, _ptr(accept_mask),
                                          _ptr(accepted_len), _ptr(next_token), _ptr(ctx_in),
@@ -246,6 +430,9 @@ def rv_accept_speculative(h, draft_ids, q_draft, r_uniform, u_uniform, scores, a
 def rv_accept_sampled(h, draft_ids, u_uniform, temperature, sampled, accept_mask, accepted_len,
                       next_token, ctx_in, ctx_out, stream=None):
     B, gamma = draft_ids.shape
+    _expect("draft_ids", draft_ids, (B, gamma), torch.int32)
+    _check_sampled_inputs(B, gamma, u_uniform, sampled)
+    _check_accept_out(B, gamma, accept_mask, accepted_len, next_token, ctx_in, ctx_out)
     _check(h, _lib.rv_accept_sampled(h.ptr, _ptr(draft_ids), _ptr(u_uniform), float(temperature),
                                      B, gamma, _ptr(sampled), _ptr(accept_mask),
                                      _ptr(accepted_len), _ptr(next_token), _ptr(ctx_in),
@@ -261,6 +448,7 @@ def rv_host_step_graphed(h):
 
 def rv_set_head_mode(h, mode):
     _check(h, _lib.rv_set_head_mode(h.ptr, int(mode)))
+    h.head_mode = int(mode)
 
 
 def rv_set_acceptance(h, mode, eps=0.0, delta=0.0):
@@ -271,6 +459,9 @@ def rv_verify_step(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_i
                    prefix_ids, ctx_in, alpha, block_ids, pos_ids, attn_out, scores, argmax, margin,
                    accept_mask, accepted_len, next_token, ctx_out, stream=None):
     """Whole step; prompt_ids may be None (empty prompt), block_ids None skips packing."""
+    _check_step(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, prompt_ids,
+                prefix_ids, ctx_in, block_ids, pos_ids, attn_out, scores, argmax, margin,
+                accept_mask, accepted_len, next_token, ctx_out)
     B, gamma = draft_ids.shape
     n_prompt = 0 if prompt_ids is None else prompt_ids.numel()
     n_prefix = prefix_ids.shape[1]
@@ -287,7 +478,11 @@ def rv_verify_step_pending(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head,
                            attn_out, scores, argmax, margin, accept_mask, accepted_len, next_token,
                            ctx_out, stream=None):
     """Whole step over the pending-token block [t, x, template, x] (Lb + 1 positions)."""
+    _check_step(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, prompt_ids,
+                prefix_ids, ctx_in, block_ids, pos_ids, attn_out, scores, argmax, margin,
+                accept_mask, accepted_len, next_token, ctx_out, lead=1)
     B, gamma = draft_ids.shape
+    _expect("pending_ids", pending_ids, (B,), torch.int32)
     n_prompt = 0 if prompt_ids is None else prompt_ids.numel()
     n_prefix = prefix_ids.shape[1]
     _check(h, _lib.rv_verify_step_pending(
@@ -303,7 +498,11 @@ def rv_verify_step_speculative(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_h
                                u_uniform, block_ids, pos_ids, attn_out, scores, argmax, margin,
                                accept_mask, accepted_len, next_token, ctx_out, stream=None):
     """Whole step with the speculative-sampling acceptance (Alg. 1)."""
+    _check_step(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, prompt_ids,
+                prefix_ids, ctx_in, block_ids, pos_ids, attn_out, scores, argmax, margin,
+                accept_mask, accepted_len, next_token, ctx_out)
     B, gamma = draft_ids.shape
+    _check_speculative_inputs(h, B, gamma, q_draft, r_uniform, u_uniform)
     n_prompt = 0 if prompt_ids is None else prompt_ids.numel()
     n_prefix = prefix_ids.shape[1]
     _check(h, _lib.rv_verify_step_speculative(
@@ -319,7 +518,11 @@ def rv_verify_step_sampled(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head,
                            block_ids, pos_ids, attn_out, scores, argmax, margin, sampled,
                            accept_mask, accepted_len, next_token, ctx_out, stream=None):
     """Whole step with exact match against target tokens sampled at temperature T (Alg. 2)."""
+    _check_step(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, prompt_ids,
+                prefix_ids, ctx_in, block_ids, pos_ids, attn_out, scores, argmax, margin,
+                accept_mask, accepted_len, next_token, ctx_out)
     B, gamma = draft_ids.shape
+    _check_sampled_inputs(B, gamma, u_uniform, sampled)
     n_prompt = 0 if prompt_ids is None else prompt_ids.numel()
     n_prefix = prefix_ids.shape[1]
     _check(h, _lib.rv_verify_step_sampled(
@@ -335,6 +538,9 @@ def rv_verify_step_host(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, dr
                         scores, argmax, margin, accept_mask, accepted_len, next_token, ctx_out,
                         stream=None):
     """Host tensors in/out (pin them for asynchronous copies); returns (h2d, d2h) bytes."""
+    _check_step(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, prompt_ids,
+                prefix_ids, ctx_in, block_ids, pos_ids, attn_out, scores, argmax, margin,
+                accept_mask, accepted_len, next_token, ctx_out, device=False)
     B, gamma = draft_ids.shape
     n_prompt = 0 if prompt_ids is None else prompt_ids.numel()
     n_prefix = prefix_ids.shape[1]
@@ -348,6 +554,41 @@ def rv_verify_step_host(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, dr
     return hb.value, db.value
 
 
+class PreparedStep:
+    """rv_verify_step with its arguments checked and marshalled once.
+
+    For loops that run the same step on the same device buffers (a serving
+    loop's persistent inputs and outputs, a benchmark): the shape checks and
+    ~30 ctypes arguments cost tens of microseconds of Python per call, which
+    this pays once.  Calling the object runs the same C entry point."""
+
+    def __init__(self, h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids,
+                 prompt_ids, prefix_ids, ctx_in, alpha, block_ids, pos_ids, attn_out, scores,
+                 argmax, margin, accept_mask, accepted_len, next_token, ctx_out, stream=None):
+        _check_step(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, prompt_ids,
+                    prefix_ids, ctx_in, block_ids, pos_ids, attn_out, scores, argmax, margin,
+                    accept_mask, accepted_len, next_token, ctx_out)
+        B, gamma = draft_ids.shape
+        n_prompt = 0 if prompt_ids is None else prompt_ids.numel()
+        n_prefix = prefix_ids.shape[1]
+        self._h = h
+        self._keep = (q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, prompt_ids,
+                      prefix_ids, ctx_in, block_ids, pos_ids, attn_out, scores, argmax, margin,
+                      accept_mask, accepted_len, next_token, ctx_out)
+        self._fn = _lib.rv_verify_step
+        self._args = (
+            h.ptr, _ptr(q), _ptr(k_blk), _ptr(v_blk), _ptr(k_cache), _ptr(v_cache), _ptr(hidden),
+            _ptr(w_head), _ptr(draft_ids), _ptr(prompt_ids), _ptr(prefix_ids), _ptr(ctx_in), B,
+            gamma, n_prompt, n_prefix, float(alpha), _ptr(block_ids), _ptr(pos_ids),
+            _ptr(attn_out), _ptr(scores), _ptr(argmax), _ptr(margin), _ptr(accept_mask),
+            _ptr(accepted_len), _ptr(next_token), _ptr(ctx_out), _stream(stream))
+
+    def __call__(self):
+        rc = self._fn(*self._args)
+        if rc != RV_OK:
+            _check(self._h, rc)
+
+
 class PreparedStepHost:
     """rv_verify_step_host with its arguments marshalled once.
 
@@ -359,6 +600,9 @@ class PreparedStepHost:
     def __init__(self, h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids,
                  prompt_ids, prefix_ids, ctx_in, alpha, block_ids, pos_ids, attn_out, scores,
                  argmax, margin, accept_mask, accepted_len, next_token, ctx_out, stream=None):
+        _check_step(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, prompt_ids,
+                    prefix_ids, ctx_in, block_ids, pos_ids, attn_out, scores, argmax, margin,
+                    accept_mask, accepted_len, next_token, ctx_out, device=False)
         B, gamma = draft_ids.shape
         n_prompt = 0 if prompt_ids is None else prompt_ids.numel()
         n_prefix = prefix_ids.shape[1]
@@ -391,8 +635,20 @@ def rv_verify_head_static(hidden, w_head, draft_ids, gamma, R, alpha, scores, ar
                           dev_status=None, stream=None):
     """rv_verify_head without a handle or any device allocation (fixed internal
     scratch; limits RV_STATIC_MAX_PAIRS / RV_STATIC_MAX_HIDDEN)."""
+    if hidden is None or hidden.dim() != 3 or w_head is None or w_head.dim() != 2:
+        raise ValueError("hidden must be [B, 2*gamma+R+1, H] and w_head [V, H]")
     B = hidden.shape[0]
     V, H = w_head.shape
+    ck = _Checks()
+    ck("hidden", hidden, (B, 2 * gamma + R + 1, H), torch.bfloat16)
+    ck("w_head", w_head, (V, H), torch.bfloat16)
+    ck("draft_ids", draft_ids, (B, gamma), torch.int32)
+    ck("scores", scores, (B, gamma + 1, RV_NSCORES), torch.float32)
+    ck("argmax", argmax, (B, gamma + 1), torch.int32)
+    ck("margin", margin, (B, gamma), torch.float32)
+    if dev_status is not None:
+        ck("dev_status", dev_status, (1,), torch.int32)
+    ck.placed()
     rc = _lib.rv_verify_head_static(_ptr(hidden), _ptr(w_head), _ptr(draft_ids), B, gamma, R, V,
                                     H, float(alpha), _ptr(scores), _ptr(argmax), _ptr(margin),
                                     _ptr(dev_status), _stream(stream))

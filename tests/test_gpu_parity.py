@@ -392,17 +392,32 @@ def test_context_overflow_sets_status_and_skips(gu):
 def test_host_validation_errors(gu):
     import torch
     from paper_2505_18629_gb300 import rv
-    h = gu.make_handle(_wl())
-    z = torch.zeros(8, device="cuda")
+    wl = _wl()
+    h = gu.make_handle(wl)
+    g, R = wl.gamma, wl.R
+    W = torch.zeros((wl.V, wl.H), dtype=torch.bfloat16, device="cuda")
+
+    def head(B, alpha):
+        rv.rv_verify_head(h, torch.zeros((B, 2 * g + R + 1, wl.H), dtype=torch.bfloat16,
+                                         device="cuda"), W,
+                          torch.zeros((B, g), dtype=torch.int32, device="cuda"), g, R, alpha,
+                          torch.zeros((B, g + 1, rv.RV_NSCORES), device="cuda"),
+                          torch.zeros((B, g + 1), dtype=torch.int32, device="cuda"),
+                          torch.zeros((B, g), device="cuda"))
     with pytest.raises(rv.RVError) as e:
-        rv.rv_verify_head(h, torch.zeros((4, 14, 320), dtype=torch.bfloat16, device="cuda"), z,
-                          torch.zeros((4, 4), dtype=torch.int32, device="cuda"), 4, 5, 0.3, z, z, z)
+        head(4, 0.3)
     assert e.value.code == rv.RV_ERR_CAPACITY                # B=4 > max_batch=3
     with pytest.raises(rv.RVError) as e:
-        rv.rv_verify_head(h, torch.zeros((1, 14, 320), dtype=torch.bfloat16, device="cuda"), z,
-                          torch.zeros((1, 4), dtype=torch.int32, device="cuda"), 4, 5,
-                          float("nan"), z, z, z)
+        head(1, float("nan"))
     assert e.value.code == rv.RV_ERR_INVALID_ARG
+    # a hidden tensor with too few rows is refused by the binding, before any launch
+    with pytest.raises(ValueError, match="hidden"):
+        rv.rv_verify_head(h, torch.zeros((1, 2 * g + R, wl.H), dtype=torch.bfloat16,
+                                         device="cuda"), W,
+                          torch.zeros((1, g), dtype=torch.int32, device="cuda"), g, R, 0.3,
+                          torch.zeros((1, g + 1, rv.RV_NSCORES), device="cuda"),
+                          torch.zeros((1, g + 1), dtype=torch.int32, device="cuda"),
+                          torch.zeros((1, g), device="cuda"))
     h.close()
 
 

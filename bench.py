@@ -102,8 +102,12 @@ def aggregate(ms_local: float, units_local: float, world: int):
 # ---------------------------------------------------------------------------- clocks
 
 class ClockSampler:
-    """nvidia-smi sampling during the timed region (clock, power, throttle reasons)."""
-    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+    """nvidia-smi sampling (clock, power, throttle reasons) while the GPU is
+    under load.  The sampler runs from start() to stop(); mark(t0, t1) names a
+    loaded window in time.time() seconds (the run-in and the timed steps that
+    follow it), and stop() summarises the samples inside the marked windows
+    (all samples if none was marked or none falls inside)."""
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
               "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
               "clocks_event_reasons.sw_power_cap")
 
@@ -111,6 +115,7 @@ class ClockSampler:
         self.dev = device_index
         self.proc = None
         self.path = None
+        self.windows = []
 
     def start(self):
         try:
@@ -120,9 +125,19 @@ class ClockSampler:
                 ["nvidia-smi", "-i", str(self.dev), f"--query-gpu={self.FIELDS}",
                  "--format=csv,noheader,nounits", "-lms", "100", "-f", self.path],
                 stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
-            time.sleep(0.3)
         except (OSError, FileNotFoundError):
             self.proc = None
+
+    def mark(self, t0: float, t1: float):
+        self.windows.append((t0, t1))
+
+    @staticmethod
+    def _when(stamp: str):
+        import datetime
+        try:
+            return datetime.datetime.strptime(stamp.strip(), "%Y/%m/%d %H:%M:%S.%f").timestamp()
+        except ValueError:
+            return None
 
     def stop(self):
         if self.proc is None:
@@ -137,19 +152,26 @@ class ClockSampler:
         with open(self.path) as f:
             for line in f:
                 parts = [p.strip() for p in line.split(",")]
-                if len(parts) >= 7:
+                if len(parts) >= 8:
                     rows.append(parts)
         os.unlink(self.path)
         if not rows:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
-        sm = [float(r[0]) for r in rows if r[0].replace(".", "").isdigit()]
-        mx = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        inside = [r for r in rows if any(
+            w is not None and a - 0.05 <= w <= b + 0.05
+            for w in [self._when(r[0])] for a, b in self.windows)]
+        used = inside if inside else rows
+        num = lambda x: x.replace(".", "").isdigit()  # noqa: E731
+        sm = [float(r[1]) for r in used if num(r[1])]
+        mx = [float(r[2]) for r in used if num(r[2])]
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = sorted({names[i] for r in rows for i in range(4) if r[3 + i].lower() == "active"})
-        pw = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        reasons = sorted({names[i] for r in used for i in range(4) if r[4 + i].lower() == "active"})
+        pw = [float(r[3]) for r in used if num(r[3])]
         return {"sm_mhz": statistics.median(sm) if sm else None,
                 "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
-                "samples": len(rows), "power_w_max": max(pw) if pw else None}
+                "samples": len(used), "samples_total": len(rows),
+                "window": "run-in + timed steps" if inside else "whole run",
+                "power_w_max": max(pw) if pw else None}
 
 
 # ---------------------------------------------------------------------------- CPU oracle legs
@@ -218,15 +240,21 @@ def run_reference(args, wl):
     for _ in range(args.warmup):
         oracle_sample_step(inp, drafts, heads, rows)
     est = []
+    t_wall0 = time.perf_counter()
     for _ in range(args.steps):
         a, h = oracle_sample_step(inp, drafts, heads, rows)
         est.append(a * wl.Hq / heads + h * wl.V / rows)
+    wall_s = time.perf_counter() - t_wall0
     t_step = statistics.median(est)
     value = wl.B * wl.Lb / t_step
     sample = (f"each step: attention over {heads}/{wl.Hq} query heads, LM head over {rows}/{wl.V} "
               f"vocab rows, extrapolated linearly to the full step")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_step * 1e3,
+            "ms_per_step_kind": "extrapolated: the median sampled step scaled linearly to all "
+                                "query heads and vocab rows; never observed as wall time",
+            "observed": {"wall_s": wall_s, "sampled_ms_per_step": wall_s * 1e3 / args.steps,
+                         "what": f"{args.steps} sampled steps as run"},
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "config": _config(wl),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores_used(),
@@ -483,6 +511,12 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=200)
+    ap.add_argument("--run-in-s", type=float, default=0.3,
+                    help="wall seconds of untimed full steps right before each timed region")
+    ap.add_argument("--extra-workload", default="llama3-8b-b16",
+                    help="a second workload measured in the same run under the JSON key "
+                         "--extra-key ('' for none)")
+    ap.add_argument("--extra-key", default="b16")
     ap.add_argument("--head-mode", default="fused", choices=["fused", "preblended"],
                     help="fused: both logit vectors fused per vocab row (Eq. 2); preblended: "
                          "the head on the blended hidden states (one row per position)")
@@ -525,7 +559,44 @@ def main():
         dist.init_process_group("nccl")
     dev = torch.device("cuda", local if world > 1 else 0)
     torch.cuda.set_device(dev)
-    from paper_2505_18629_gb300 import rv
+
+    clocks = ClockSampler(dev.index if dev.index is not None else 0)
+    clocks.start()
+    res = measure_workload(wl, args, dev, world, rank, clocks)
+    line = res.pop("line")
+    inp, drafts_np = res["inp"], res["drafts_np"]
+    if args.extra_workload and args.extra_workload != wl.name:
+        # the batched workload in the same run, with the same steady-state
+        # rules (its own run-in, timed region, breakdown and e2e)
+        del res
+        torch.cuda.empty_cache()
+        xwl = synth.workload(args.extra_workload)
+        xres = measure_workload(xwl, args, dev, world, rank, clocks)
+        xline = xres["line"]
+        line[args.extra_key] = {k: xline[k] for k in (
+            "value", "unit", "ms_per_step", "step_us", "step_roofline_frac", "roofline",
+            "attention", "e2e", "gpu_launches", "mean_accepted", "config")}
+        del xres
+        torch.cuda.empty_cache()
+    line["clocks"] = clocks.stop()
+    if rank == 0 and not args.no_cpu_baseline and world == 1:
+        B, Lb = wl.B, wl.Lb
+        t_full, sample, spent = cpu_step_estimate(inp, drafts_np, args.cpu_seconds)
+        line["cpu_baseline"] = {"value": B * Lb / t_full, "unit": UNIT, "cores": cores_used(),
+                                "kind": "oracle", "sample": sample, "seconds": spent}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def measure_workload(wl, args, dev, world, rank, clocks):
+    """Device-timed steps, the LM head / attention breakdown and the
+    host-buffer (e2e) step of one workload.  Returns {"line": the JSON fields,
+    "inp": the synthetic inputs, "drafts_np": the drafts}."""
+    import torch
+    import torch.distributed as dist
+    from paper_2505_18629_gb300 import rv, synth
 
     inp = synth.generate(wl.replace(seed=wl.seed + 1000 * rank) if rank else wl)
     B, g, R, Lb = wl.B, wl.gamma, wl.R, wl.Lb
@@ -565,9 +636,11 @@ def main():
     drafts = dev_t(drafts_np)
     stream = torch.cuda.current_stream(dev)
 
-    def step():
-        rv.rv_verify_step(h, q, kb, vb, kc, vc, hidden, W, drafts, prompt, prefix, ctx, ALPHA,
-                          block, pos, attn, scores, argmax, margin, acc, alen, nxt, ctx_out, stream)
+    # the step's arguments checked and marshalled once (the buffers are reused
+    # every step, as a serving loop's would be)
+    step = rv.PreparedStep(h, q, kb, vb, kc, vc, hidden, W, drafts, prompt, prefix, ctx, ALPHA,
+                           block, pos, attn, scores, argmax, margin, acc, alen, nxt, ctx_out,
+                           stream)
 
     for _ in range(args.warmup):
         step()
@@ -576,14 +649,30 @@ def main():
         raise RuntimeError(f"device status 0x{st:x} during warm-up")
     mean_accepted = float(alen.float().mean().item())
 
-    clocks = ClockSampler(dev.index if dev.index is not None else 0)
-    clocks.start()
+    # The profiling event pool is created on the first enable (thousands of
+    # CUDA events, milliseconds of host time): create it here, outside the
+    # timed region, and drop what it recorded.
+    prof_mask = (1 << rv.RV_PROF_HEAD) | (1 << rv.RV_PROF_HEAD_GEMM) | (1 << rv.RV_PROF_ATTENTION)
+    rv.rv_profile_enable(h, prof_mask)
+    rv.rv_profile_enable(h, 0)
+    for region in (rv.RV_PROF_HEAD, rv.RV_PROF_HEAD_GEMM, rv.RV_PROF_ATTENTION):
+        rv.rv_profile_read(h, region)
+    # Run-in: full steps for a fixed wall time before the timed region, so
+    # that the GPU is out of its idle state and the clock sampler is running
+    # when the first timed step starts.
+    t_load0 = time.time()
+    t_end = time.perf_counter() + args.run_in_s
+    n_run_in = 0
+    while time.perf_counter() < t_end or n_run_in < 3:
+        step()
+        n_run_in += 1
+        if n_run_in % 64 == 0:
+            torch.cuda.synchronize(dev)
     # An event pair around the row gather + LM head (+ its merge) leaves their
     # programmatic overlap intact; the head time it gives includes the short
-    # gather.
-    # (sampled on every PROF_EVERY-th step: each event record costs the step a
-    # few microseconds of GPU time)
-    PROF_EVERY = 8
+    # gather.  It is recorded on every PROF_EVERY-th timed step (each event
+    # record costs the step a few microseconds of GPU time).
+    PROF_EVERY = 4
     launches0 = rv.rv_launch_count(h)
     if world > 1:
         dist.barrier()
@@ -591,7 +680,7 @@ def main():
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for i in range(args.steps):
-        sampled = i % PROF_EVERY == 0
+        sampled = i % PROF_EVERY == PROF_EVERY - 1
         if sampled:
             rv.rv_profile_enable(h, 1 << rv.RV_PROF_HEAD)
         step()
@@ -599,10 +688,10 @@ def main():
             rv.rv_profile_enable(h, 0)
     e1.record(stream)
     torch.cuda.synchronize(dev)
+    clocks.mark(t_load0, time.time())
     if world > 1:
         dist.barrier()
     launches = rv.rv_launch_count(h) - launches0
-    clk = clocks.stop()
     ms_total = e0.elapsed_time(e1)
     head_ms, head_n = rv.rv_profile_read(h, rv.RV_PROF_HEAD)
     rv.rv_profile_enable(h, 0)
@@ -610,7 +699,7 @@ def main():
     # and the attention each alone (their own entry points, one after the
     # other on one stream), between the library's events around the kernels.
     rv.rv_profile_enable(h, (1 << rv.RV_PROF_HEAD_GEMM) | (1 << rv.RV_PROF_ATTENTION))
-    for _ in range(min(args.steps, 200)):
+    for _ in range(min(max(args.steps, 50), 200)):
         rv.rv_verify_head(h, hidden, W, drafts, g, R, ALPHA, scores, argmax, margin, stream)
         rv.rv_verify_attention(h, q, kb, vb, kc, vc, ctx, attn, stream)
     torch.cuda.synchronize(dev)
@@ -652,8 +741,11 @@ def main():
     step_host = rv.PreparedStepHost(h, hq, hkb, hvb, kc, vc, hhid, W, hdr, hprompt, hprefix,
                                     hctx, ALPHA, o_blk, o_pos, None, o_sc, o_am, o_mg, o_acc,
                                     o_al, o_nt, o_co, e2e_stream)
-    for _ in range(3):
+    t_end = time.perf_counter() + min(args.run_in_s, 0.1)
+    n_e2e_warm = 0
+    while time.perf_counter() < t_end or n_e2e_warm < 3:
         step_host()
+        n_e2e_warm += 1
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize(dev)
@@ -689,13 +781,17 @@ def main():
                 "frac": achieved_tf / tf_burst, "traffic": traffic}
     roof.update({"kernel": "LM head (head_tc_kernel; head_tc2_kernel on CTA pairs from N >= 96 "
                            "hidden rows per chunk): GEMM + online log-softmax (+ merge), timed with the "
-                           "row-gather launch before it by an event pair on every 8th timed step",
+                           f"row-gather launch before it by an event pair on every {PROF_EVERY}th "
+                           "timed step",
                  "peak_source": f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured"
                  else "fallback", "algorithmic_bytes": head_bytes,
                  "algorithmic_flops": head_flops, "avg_us": head_avg_s * 1e6, "launches": head_n,
                  "kernel_alone_us": gemm_avg_s * 1e6,
                  "frac_kernel_alone": (head_bytes / gemm_avg_s / 1e9 / hbm) if bound == "hbm"
-                 else head_flops / gemm_avg_s / 1e12 / tf_burst})
+                 else head_flops / gemm_avg_s / 1e12 / tf_burst,
+                 # the HBM-bound fraction as well where the tensor bound is the larger
+                 "frac_hbm": head_bytes / head_avg_s / 1e9 / hbm,
+                 "frac_hbm_kernel_alone": head_bytes / gemm_avg_s / 1e9 / hbm})
     # attention kernels (one layer): KV read + block Q/K/V/O
     ctx_mean = float(np.mean(inp.ctx_lens))
     attn_bytes = (B * (ctx_mean + Lb) * wl.Hkv * wl.D * 2 * 2 + B * Lb * wl.Hq * wl.D * 2 * 2
@@ -709,7 +805,8 @@ def main():
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32",
         "data": "synthetic (seeded Gaussian weights/activations shaped like Llama-3-8B)",
-        "config": _config(wl, world, args.head_mode),
+        "config": dict(_config(wl, world, args.head_mode), run_in_steps=n_run_in,
+                       run_in_s=args.run_in_s),
         "step_us": ms_step * 1e3,
         "drafts_per_s": units / B / Lb * B * g / (ms_step * 1e-3),
         "step_roofline_frac": step_roof_s / (ms_step * 1e-3),
@@ -724,17 +821,9 @@ def main():
                 "api": "rv_verify_step_host (pinned host buffers, synchronous; repeated calls "
                        "replay one CUDA graph)"},
         "gpu_launches": launches,
-        "clocks": clk,
     }
-    if rank == 0 and not args.no_cpu_baseline and world == 1:
-        t_full, sample, spent = cpu_step_estimate(inp, drafts_np, args.cpu_seconds)
-        line["cpu_baseline"] = {"value": B * Lb / t_full, "unit": UNIT, "cores": cores_used(),
-                                "kind": "oracle", "sample": sample, "seconds": spent}
-    if rank == 0:
-        print(json.dumps(line), flush=True)
     h.close()
-    if world > 1:
-        dist.destroy_process_group()
+    return {"line": line, "inp": inp, "drafts_np": drafts_np}
 
 
 if __name__ == "__main__":

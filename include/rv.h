@@ -414,7 +414,9 @@ RV_API int rv_host_step_graphed(const rv_handle* h, int32_t* active);
  *   hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin:
  *           as in rv_verify_head (bf16 only); vocab / hidden_size give V, H.
  *   dev_status: optional device word; the RV_DEV_* bits of this call are
- *           OR-ed into it (NULL: they go to the shared array and are lost).
+ *           OR-ed into it and never cleared by the library, so the caller
+ *           zeroes it before the first call (NULL: the bits go to the shared
+ *           array and are lost).
  * Limits: B * (gamma + 1) <= RV_STATIC_MAX_PAIRS and hidden_size <=
  * RV_STATIC_MAX_HIDDEN, else RV_ERR_CAPACITY before anything is launched.
  * The first call on a device (make it before any stream capture) looks up the

@@ -222,6 +222,32 @@ def compare(inp: synth.VerifyInputs, drafts, alpha, ref: dict, gpu: GpuRun, chec
                   float(lse_err), float(logp_err), float(m_err), amax)
 
 
+def compare_head(ref: dict, scores: np.ndarray, argmax: np.ndarray, margin: np.ndarray,
+                 gamma: int) -> Report:
+    """LM-head outputs (scores, argmax, margin of rv_verify_head) against the
+    oracle's verify_head on the same sequences: statistics within LOGP_ATOL,
+    the choice bit-exact except where the oracle's choice gap is below
+    MARGIN_EPS (counted)."""
+    g = gamma
+    sc = scores.astype(np.float64)
+    lse_err = max(_err(sc[..., 0], ref["lse_orig"]), _err(sc[..., 1], ref["lse_refl"]),
+                  _err(sc[..., 2], ref["lse_fused"]))
+    assert lse_err <= LOGP_ATOL, f"lse error {lse_err}"
+    logp_err = max(_err(sc[:, :g, 3], ref["logp_fused"]), _err(sc[:, :g, 4], ref["logp_orig"]),
+                   _err(sc[:, :g, 5], ref["logp_refl"]))
+    assert logp_err <= LOGP_ATOL, f"log-prob error {logp_err}"
+    assert np.isnan(sc[:, g, 3:6]).all()                  # no draft at the bonus position
+    ent_err = _err(sc[..., 6], ref["ent_orig"])
+    assert ent_err <= LOGP_ATOL, f"entropy error {ent_err}"
+    m_err = float(np.abs(margin.astype(np.float64) - ref["margin"]).max())
+    assert m_err <= LOGP_ATOL, f"margin error {m_err}"
+    low_choice = ref["choice_gap"] < MARGIN_EPS
+    assert ((argmax == ref["argmax"]) | low_choice).all(), \
+        "argmax differs at a position with a clear choice"
+    return Report(int(low_choice.size), int(low_choice.sum()), 0, 0, float(lse_err),
+                  float(logp_err), m_err, 0.0)
+
+
 def _compare_typical(inp, ref, gpu, seqs, lse_err, logp_err, m_err, amax) -> Report:
     """Typical acceptance (Alg. 3): decisions bit-exact except where the oracle's
     log p_i(x_i) is within MARGIN_EPS of the log threshold (counted); n and t may

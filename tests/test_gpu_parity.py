@@ -981,8 +981,15 @@ def _standard_run(gu, wl, seqs=None, check_attn=True, pending=False, host=False)
     tail = (None, prefix, dev["ctx"], ALPHA, block, pos, attn, sc, am, mg, acc, n, nt, co)
     if inp.prompt_ids.size:
         with pytest.raises(rv.RVError):  # standard verification has no template
-            rv.rv_verify_step(h, *args, dev["d"], gu.to_dev(inp.prompt_ids.astype(np.int32)),
-                              *tail[1:])
+            prompt = inp.prompt_ids.astype(np.int32)
+            if host:
+                rv.rv_verify_step_host(h, *args, dev["d"], torch.from_numpy(prompt).pin_memory(),
+                                       *tail[1:])
+            elif pending:
+                rv.rv_verify_step_pending(h, *args, gu.to_dev(t), dev["d"], gu.to_dev(prompt),
+                                          *tail[1:])
+            else:
+                rv.rv_verify_step(h, *args, dev["d"], gu.to_dev(prompt), *tail[1:])
     if host:
         rv.rv_verify_step_host(h, *args, dev["d"], *tail)
     elif pending:

@@ -3,31 +3,48 @@
 // memory rather than by HBM:
 //
 //   acc[v][c] = sum_k W[v][k] * hsel[c][k]   over 256 vocab rows v per pair tile
-//   (128 per CTA) and the N gathered hidden rows c of one pair chunk (original
-//   rows 0..Pcp-1, reflective rows Pcp..2Pcp-1: o_i and o_{m+i-1} of Alg. 1),
+//   (128 per CTA) and the gathered hidden rows c of one pair chunk: o_i and
+//   o_{m+i-1} of Alg. 1,
 //
-// followed by the same online log-softmax / fusion epilogue (Eq. 2) as the
-// one-CTA kernel, so that no logit is written to memory.  One MMA of the pair
-// (M = 256, issued by the even CTA) reads the A operand from each CTA's own
-// shared memory (its 128 weight rows) and the B operand split across the two
-// (the even CTA holds the original rows, the odd CTA the reflective rows), so
-// each SM stages its weight rows and only half of the hidden rows; every CTA
-// gets its own 128 x N accumulator in its TMEM.
+// followed by the online log-softmax / fusion epilogue (Eq. 2), so that no
+// logit is written to memory.  One MMA of the pair (M = 256, issued by the
+// even CTA) reads the A operand from each CTA's own shared memory (its 128
+// weight rows) and the B operand split across the two (the even CTA holds the
+// original rows, the odd CTA the reflective rows), so each SM stages its
+// weight rows and only half of the hidden rows; every CTA gets its own 128-row
+// accumulator in its TMEM.
+//
+// Sub-groups.  The pairs of a chunk are split into H sub-groups of Ph pairs;
+// sub-group h has its own accumulator of Ns = 2 Ph columns (o of its pairs,
+// then o'), one MMA per 16-wide K step each.  Every sub-group reads the same
+// weight stage, so a chunk of up to 160 pairs (H = 2) streams each weight tile
+// into shared memory once.  The accumulators rotate through a ring of R slots
+// (R * Ns <= 512 TMEM columns, R >= H + 1): the next tile's first sub-group
+// starts in the free slot while the epilogue still reads this tile's.
 //
 // Per CTA, warp-specialised:
-//   warp 0      TMA producer: weight tile [128 x 128] + half hidden tile
-//               [Pcp x 128] per stage (each as two 64-wide boxes); both CTAs'
-//               copies complete on the even CTA's full barrier
-//   warp 1      TMEM owner (both CTAs, 2 accumulator slots of N columns); in
-//               the even CTA it also issues the pair's MMAs from one thread,
-//               and its commits release the stage and fill the accumulator
-//               slot in both CTAs
-//   warps 2..   epilogue over this CTA's 128 rows; the slot is free again once
-//               the epilogue warps of both CTAs have arrived on the even CTA's
-//               empty-accumulator barrier
+//   warp 0      TMA producer: weight tile [128 x 128] + this CTA's hidden rows
+//               of every sub-group per stage (each as two 64-wide boxes); both
+//               CTAs' copies complete on the even CTA's full barrier
+//   warp 1      TMEM owner (both CTAs); in the even CTA it also issues the
+//               pair's MMAs from one thread, and its commits release the stage
+//               and fill the accumulator slots in both CTAs
+//   warps 2..   epilogue, H2_WPQ warps per TMEM lane quadrant
 // The pair streams a static range of 256-row vocab tiles; the weight streams
 // from HBM once per chunk (evict-first), the hidden rows are re-read from L2.
+//
+// Epilogue.  tcgen05.ld.16x256b gives lane l of a warp the rows l/4 + 8i
+// (i = 0..3, two loads) and the columns 2(l%4), 2(l%4)+1 of an 8-column group,
+// so a column's 32 rows lie in 4 registers of 8 lanes: the max / sum-exp /
+// argmax reductions over the vocab rows take 3 register steps and 3 shuffle
+// levels, with every lane busy.  The tile results are folded into running
+// statistics that live in registers: in a group of 8 pairs, lane l keeps, for
+// column 2(l%4) + ((l/4) & 1), the statistics of quantity l/8 (o with its
+// entropy term, o', z, or the best z over v != x_i), one fold per lane and
+// group.  At the end they go to per-quadrant tables in shared memory (over
+// the drained pipeline stages) and are merged into the CTA's partials.
 #include <cfloat>
+#include <climits>
 
 #include "head_epilogue.cuh"
 #include "rv_device.cuh"
@@ -38,13 +55,28 @@ namespace rv {
 namespace {
 
 constexpr int H2_BM = 128;  // vocab rows per CTA per pair tile
-constexpr int H2_BK = 128;  // K per stage: two 64-wide swizzled halves, 8 MMAs
+constexpr int H2_BK = 128;  // K per stage: two 64-wide swizzled halves, 8 MMAs per sub-group
 constexpr uint32_t H2_A_HALF = H2_BM * 64 * 2;      // 16 KB
 constexpr uint32_t H2_A_BYTES = 2 * H2_A_HALF;      // 32 KB
-__host__ __device__ constexpr int h2_threads(int epi_warps) { return 64 + epi_warps * 32; }
+#ifndef RV_HEAD2_WPQ
+#define RV_HEAD2_WPQ 3
+#endif
+constexpr int H2_WPQ = RV_HEAD2_WPQ;  // epilogue warps per TMEM lane quadrant (3: measured best at 8B B=16)
+constexpr int H2_EPI = 4 * H2_WPQ;
+constexpr int H2_THREADS = 64 + 32 * H2_EPI;
+// groups one epilogue warp may own: of 2 sub-groups of up to 10 groups (160
+// pairs), or of 1 of up to 16 groups (128 pairs, or 256 pre-blended pairs in
+// groups of 16)
+constexpr int h2_cdiv(int a, int b) { return (a + b - 1) / b; }
+constexpr int H2_MAX_OWN = 2 * h2_cdiv(10, H2_WPQ) > h2_cdiv(16, H2_WPQ) ? 2 * h2_cdiv(10, H2_WPQ)
+                                                                        : h2_cdiv(16, H2_WPQ);
+constexpr int H2_MAX_H = 2;     // sub-groups per tile
+constexpr int H2_MAX_R = 4;     // accumulator slots
 
 struct Head2Params {
-  int V, n_kb, N, Pcp, Pc, P, stages, gamma;
+  int V, n_kb;
+  int H, Ph, Ns, R;  // sub-groups per tile, pairs per sub-group, columns per slot, slots
+  int Pcp, Pc, P, stages, gamma;
   int pair_slots;  // CTA pairs per chunk
   int n_ptiles;    // ceil(V / 256)
   unsigned* done_counter;
@@ -130,10 +162,325 @@ __device__ __forceinline__ void tc2_commit(uint32_t bar, uint16_t mask) {
       : "memory");
 }
 
+// 16 lanes x 256 bit: lane l of the warp gets rows (base + l/4) and
+// (base + 8 + l/4), columns 2(l%4) and 2(l%4)+1 of the 8 columns at `taddr`:
+// v = {row l/4: col, col+1; row 8 + l/4: col, col+1}.
+__device__ __forceinline__ void tmem_ld_16x256b(uint32_t taddr, uint32_t* v) {
+  asm volatile("tcgen05.ld.sync.aligned.16x256b.x1.b32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3])
+               : "r"(taddr));
+}
+// .x2: the same for columns 8..15 in v[4..7].
+__device__ __forceinline__ void tmem_ld_16x256b_x2(uint32_t taddr, uint32_t* v) {
+  asm volatile("tcgen05.ld.sync.aligned.16x256b.x2.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+               : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]),
+                 "=r"(v[6]), "=r"(v[7])
+               : "r"(taddr));
+}
+
+// After tcgen05.wait::ld: makes every later use of `v` depend on this point,
+// so that no use of a loaded register is scheduled before the wait.
+__device__ __forceinline__ void after_ld(uint32_t (&v)[16]) {
+#pragma unroll
+  for (int i = 0; i < 16; ++i) asm volatile("" : "+r"(v[i]));
+}
+
+__device__ __forceinline__ void shfl_best(float& bv, int& bi, int off) {
+  const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
+  const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
+  if (ov > bv || (ov == bv && oi < bi)) {
+    bv = ov;
+    bi = oi;
+  }
+}
+
+struct TileOut {
+  float m, s, t;
+};
+
+// Stores at the draft row of each of the lane's columns: `x[j]` (this lane's
+// pair of column j) may fall on one of its rows rq + 8i; at most one (unique
+// writer over the CTA).  Rows at or beyond V (a partial last tile) hold zeros;
+// a draft there is out of range and its gathered values are never read.
+template <int NC>
+__device__ __forceinline__ void gather_draft_rows(const float* o, const float* r, const float* z,
+                                                  const int* x, int row0, float* gathered,
+                                                  int gpair_lane, const int* col_pair) {
+#pragma unroll
+  for (int j = 0; j < NC; ++j) {
+    const int d = x[j] - row0;
+    if (static_cast<unsigned>(d) < 32u && (d & 7) == 0) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        if (d == 8 * i) {
+          float* gx = gathered + (gpair_lane + col_pair[j]) * GATHER_FIELDS;
+          if (o != nullptr) {
+            gx[0] = o[NC * i + j];
+            gx[1] = r[NC * i + j];
+          }
+          gx[2] = z[NC * i + j];
+        }
+      }
+    }
+  }
+}
+
+// One group of eight pairs of the two-distribution head: lo = o and lr = o'
+// as loaded by two tcgen05.ld.16x256b each (rows +0 / +16 of this warp's
+// quadrant); x[j] the draft of the lane's column j (-1: none).  Rows at or
+// beyond V count as -inf.  Forms z = (1-a) o + a o' (Eq. 2), stores o, o', z
+// at the draft row of each pair and, when asked, z itself; returns this
+// lane's tile statistics: quantity lane / 8 (o, o', z, best z over v != x_i)
+// of column 2(lane%4) + ((lane/4)&1).
+__device__ __forceinline__ TileOut group8_fused(const uint32_t* lo, const uint32_t* lr,
+                                                int v_row0, int V, float alpha, float beta,
+                                                const int (&x)[2], int gpair, int npairs,
+                                                float* gathered, float* zout, int lane) {
+  const int c4 = lane & 3, rq = lane >> 2;
+  const int row0 = v_row0 + rq;  // this lane's first row; the others are +8, +16, +24
+  float o[8], r[8], z[8];
+  // element 2i + j: row row0 + 8i, column 2 c4 + j
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    o[k] = __uint_as_float(lo[k]);
+    r[k] = __uint_as_float(lr[k]);
+    z[k] = fmaf(alpha, r[k], beta * o[k]);
+  }
+  if (v_row0 + 32 > V) {  // a partial last tile (warp-uniform)
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      if (row0 + 8 * i >= V) {
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+          o[2 * i + j] = NEG_INF;
+          r[2 * i + j] = NEG_INF;
+          z[2 * i + j] = NEG_INF;
+        }
+      }
+    }
+  }
+  {
+    const int col_pair[2] = {2 * c4, 2 * c4 + 1};
+    gather_draft_rows<2>(o, r, z, x, row0, gathered, gpair, col_pair);
+  }
+  if (zout != nullptr) {  // sampling modes only (uniform)
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int v = row0 + 8 * i;
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        const int pj = gpair + 2 * c4 + j;
+        if (v < V && pj < npairs) zout[static_cast<long long>(pj) * V + v] = z[2 * i + j];
+      }
+    }
+  }
+  float mo[2], mr[2], mz[2];
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    mo[j] = fmaxf(fmaxf(o[j], o[2 + j]), fmaxf(o[4 + j], o[6 + j]));
+    mr[j] = fmaxf(fmaxf(r[j], r[2 + j]), fmaxf(r[4 + j], r[6 + j]));
+    mz[j] = fmaxf(fmaxf(z[j], z[2 + j]), fmaxf(z[4 + j], z[6 + j]));
+  }
+#pragma unroll
+  for (int off = 4; off < 32; off <<= 1) {
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      mo[j] = fmaxf(mo[j], __shfl_xor_sync(0xffffffffu, mo[j], off));
+      mr[j] = fmaxf(mr[j], __shfl_xor_sync(0xffffffffu, mr[j], off));
+      mz[j] = fmaxf(mz[j], __shfl_xor_sync(0xffffffffu, mz[j], off));
+    }
+  }
+  float so[2], to[2], sr[2], sz[2], bv[2];
+  int bi[2];
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    // all rows -inf (a tile past the vocab end): empty sums, no NaN
+    const float nmo = mo[j] == NEG_INF ? 0.f : -mo[j] * LOG2E;
+    const float nmr = mr[j] == NEG_INF ? 0.f : -mr[j] * LOG2E;
+    const float nmz = mz[j] == NEG_INF ? 0.f : -mz[j] * LOG2E;
+    so[j] = 0.f;
+    to[j] = 0.f;
+    sr[j] = 0.f;
+    sz[j] = 0.f;
+    bv[j] = NEG_INF;
+    bi[j] = INT_MAX;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int k = 2 * i + j;
+      const float eo = ex2_approx(fmaf(o[k], LOG2E, nmo));
+      so[j] += eo;
+      to[j] += eo == 0.f ? 0.f : eo * (o[k] - mo[j]);
+      sr[j] += ex2_approx(fmaf(r[k], LOG2E, nmr));
+      sz[j] += ex2_approx(fmaf(z[k], LOG2E, nmz));
+      const int v = row0 + 8 * i;  // rows in increasing order: strict > keeps the lowest
+      const bool better = v != x[j] && z[k] > bv[j];
+      bv[j] = better ? z[k] : bv[j];
+      bi[j] = better ? v : bi[j];
+    }
+  }
+#pragma unroll
+  for (int off = 4; off < 32; off <<= 1) {
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      so[j] += __shfl_xor_sync(0xffffffffu, so[j], off);
+      to[j] += __shfl_xor_sync(0xffffffffu, to[j], off);
+      sr[j] += __shfl_xor_sync(0xffffffffu, sr[j], off);
+      sz[j] += __shfl_xor_sync(0xffffffffu, sz[j], off);
+      shfl_best(bv[j], bi[j], off);
+    }
+  }
+  const int qn = rq >> 1;
+  const bool j1 = (rq & 1) != 0;
+  const float M_o = j1 ? mo[1] : mo[0], M_r = j1 ? mr[1] : mr[0], M_z = j1 ? mz[1] : mz[0];
+  const float S_o = j1 ? so[1] : so[0], S_r = j1 ? sr[1] : sr[0], S_z = j1 ? sz[1] : sz[0];
+  const float B_v = j1 ? bv[1] : bv[0];
+  const int B_i = j1 ? bi[1] : bi[0];
+  TileOut out;
+  out.m = qn == 0 ? M_o : qn == 1 ? M_r : qn == 2 ? M_z : B_v;
+  out.s = qn == 0 ? S_o : qn == 1 ? S_r : qn == 2 ? S_z : __int_as_float(B_i);
+  out.t = j1 ? to[1] : to[0];
+  return out;
+}
+
+// One group of sixteen pairs of the pre-blended head (the columns are z):
+// la / lb as loaded by tcgen05.ld.16x256b.x2 at rows +0 / +16; lane l has
+// rows l/4 + 8i and columns 2(l%4) + (jj & 1) + 8 (jj >> 1), jj = 0..3, with
+// drafts x[jj].  Returns quantity l/16 (z statistics, best z over v != x_i)
+// of column jj = (l/4) & 3.
+__device__ __forceinline__ TileOut group16_z(const uint32_t* la, const uint32_t* lb, int v_row0,
+                                             int V, const int (&x)[4], int gpair, int npairs,
+                                             float* gathered, float* zout, int lane) {
+  const int c4 = lane & 3, rq = lane >> 2;
+  const int row0 = v_row0 + rq;
+  float z[16];  // element 4i + jj
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint32_t* src = i < 2 ? la : lb;
+    const int ii = i & 1;  // .x2 registers: {row +0: c, c+1; row +8: c, c+1; the same 8 columns on}
+#pragma unroll
+    for (int jj = 0; jj < 4; ++jj) z[4 * i + jj] = __uint_as_float(src[4 * (jj >> 1) + 2 * ii + (jj & 1)]);
+  }
+  if (v_row0 + 32 > V) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      if (row0 + 8 * i >= V) {
+#pragma unroll
+        for (int jj = 0; jj < 4; ++jj) z[4 * i + jj] = NEG_INF;
+      }
+    }
+  }
+  {
+    const int col_pair[4] = {2 * c4, 2 * c4 + 1, 8 + 2 * c4, 9 + 2 * c4};
+    gather_draft_rows<4>(nullptr, nullptr, z, x, row0, gathered, gpair, col_pair);
+  }
+  if (zout != nullptr) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int v = row0 + 8 * i;
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj) {
+        const int pj = gpair + 2 * c4 + (jj & 1) + 8 * (jj >> 1);
+        if (v < V && pj < npairs) zout[static_cast<long long>(pj) * V + v] = z[4 * i + jj];
+      }
+    }
+  }
+  float mz[4], sz[4], bv[4];
+  int bi[4];
+#pragma unroll
+  for (int jj = 0; jj < 4; ++jj)
+    mz[jj] = fmaxf(fmaxf(z[jj], z[4 + jj]), fmaxf(z[8 + jj], z[12 + jj]));
+#pragma unroll
+  for (int off = 4; off < 32; off <<= 1) {
+#pragma unroll
+    for (int jj = 0; jj < 4; ++jj) mz[jj] = fmaxf(mz[jj], __shfl_xor_sync(0xffffffffu, mz[jj], off));
+  }
+#pragma unroll
+  for (int jj = 0; jj < 4; ++jj) {
+    const float nmz = mz[jj] == NEG_INF ? 0.f : -mz[jj] * LOG2E;
+    sz[jj] = 0.f;
+    bv[jj] = NEG_INF;
+    bi[jj] = INT_MAX;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float zz = z[4 * i + jj];
+      sz[jj] += ex2_approx(fmaf(zz, LOG2E, nmz));
+      const int v = row0 + 8 * i;
+      const bool better = v != x[jj] && zz > bv[jj];
+      bv[jj] = better ? zz : bv[jj];
+      bi[jj] = better ? v : bi[jj];
+    }
+  }
+#pragma unroll
+  for (int off = 4; off < 32; off <<= 1) {
+#pragma unroll
+    for (int jj = 0; jj < 4; ++jj) {
+      sz[jj] += __shfl_xor_sync(0xffffffffu, sz[jj], off);
+      shfl_best(bv[jj], bi[jj], off);
+    }
+  }
+  const int sel = rq & 3, qn = rq >> 2;
+  float M = mz[0], S = sz[0], Bv = bv[0];
+  int I = bi[0];
+#pragma unroll
+  for (int jj = 1; jj < 4; ++jj) {
+    M = sel == jj ? mz[jj] : M;
+    S = sel == jj ? sz[jj] : S;
+    Bv = sel == jj ? bv[jj] : Bv;
+    I = sel == jj ? bi[jj] : I;
+  }
+  TileOut out;
+  out.m = qn == 0 ? M : Bv;
+  out.s = qn == 0 ? S : __int_as_float(I);
+  out.t = 0.f;
+  return out;
+}
+
 }  // namespace
 
-template <int EPI>
-__global__ void __launch_bounds__(h2_threads(EPI), 1)
+// Running statistics of the epilogue lane: one (m, s, t) per owned group, in
+// registers.  The group loop stays rolled (unrolled over the groups, its body
+// would not fit the instruction cache of the eight epilogue warps), so the
+// state rotates: the current group's is always at index 0, and after a tile
+// the ring has turned exactly once.
+struct LaneStats {
+  float m[H2_MAX_OWN], s[H2_MAX_OWN], t[H2_MAX_OWN];
+  __device__ __forceinline__ void rotate() {
+    const float m0 = m[0], s0 = s[0], t0 = t[0];
+#pragma unroll
+    for (int i = 0; i + 1 < H2_MAX_OWN; ++i) {
+      m[i] = m[i + 1];
+      s[i] = s[i + 1];
+      t[i] = t[i + 1];
+    }
+    m[H2_MAX_OWN - 1] = m0;
+    s[H2_MAX_OWN - 1] = s0;
+    t[H2_MAX_OWN - 1] = t0;
+  }
+  // Fold the tile's (M, S, T) into entry 0 without branches.  Argmax lanes:
+  // the larger value, the lower row on ties (rows kept as int bits in s).
+  // The others: running (m, s, t) with s = sum exp(x - m) and
+  // t = sum exp(x - m) (x - m) (t for o only; the entropy is log s - t / s),
+  // merged with one exponential: the side whose maximum is kept is scaled
+  // by exactly 1.
+  __device__ __forceinline__ void fold0(bool best, const TileOut& o) {
+    const float m0 = m[0], s0 = s[0], t0 = t[0];
+    const bool take = o.m > m0 || (o.m == m0 && __float_as_int(o.s) < __float_as_int(s0));
+    const float mn = fmaxf(m0, o.m);
+    const bool keep = m0 >= o.m;
+    const float f = ex2_approx(__fmul_rn(keep ? o.m - m0 : m0 - o.m, LOG2E));
+    const float a = keep ? 1.f : f, c = keep ? f : 1.f;
+    const float tn = (a == 0.f ? 0.f : a * (t0 + (m0 - mn) * s0)) +
+                     (c == 0.f ? 0.f : c * (o.t + (o.m - mn) * o.s));
+    const float sn = __fmaf_rn(s0, a, __fmul_rn(o.s, c));
+    const bool empty = mn == NEG_INF;  // nothing seen yet on either side
+    m[0] = best ? (take ? o.m : m0) : (empty ? m0 : mn);
+    s[0] = best ? (take ? o.s : s0) : (empty ? s0 : sn);
+    t[0] = best ? t0 : (empty ? t0 : tn);
+  }
+};
+
+template <bool ZONLY>
+__global__ void __launch_bounds__(H2_THREADS, 1)
     head_tc2_kernel(const __grid_constant__ CUtensorMap tm_w,
                     const __grid_constant__ CUtensorMap tm_h, const Head2Params p) {
   // the merge launch that follows (programmatic dependent launch) may be
@@ -148,35 +495,34 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
   const uint32_t crank = cluster_ctarank();
   const uint32_t rank = crank & 1u;  // 0: the pair's MMA issuer
   const bool leader = rank == 0;
-  // commit mask: this pair's two CTAs (the stage release and the accumulator)
+  // commit mask: this pair's two CTAs (the stage release and the accumulators)
   const uint16_t pair_mask = static_cast<uint16_t>(3u << (crank & ~1u));
   const int pair = blockIdx.x >> 1;
   const int chunk = blockIdx.y;
   const int slot_id = blockIdx.x;  // partial slot within the chunk
-  const int S = p.stages;
-  // this CTA's half of the B rows (the original or the reflective rows; or, for
-  // the pre-blended head, the first or second half of the blended rows)
-  const uint32_t b_half = static_cast<uint32_t>(p.N / 2) * 128u;  // one 64-wide half of B
-  const uint32_t b_bytes = 2u * b_half;                          // this CTA's part of B
+  const int S = p.stages, R = p.R, H = p.H;
+  // this CTA's rows of B per stage: Ns / 2 of every sub-group (the original
+  // or the reflective rows; for the pre-blended head the first or second half
+  // of the blended rows)
+  const uint32_t b_rows = static_cast<uint32_t>(H * p.Ns / 2);
+  const uint32_t b_half = b_rows * 128u;  // one 64-wide K half of this CTA's B
+  const uint32_t b_bytes = 2u * b_half;
 
   const uint32_t a_tiles = base;
   const uint32_t b_tiles = base + S * H2_A_BYTES;
   const uint32_t bars = b_tiles + S * b_bytes;
   auto full_bar = [&](int s) { return bars + 8u * s; };
   auto empty_bar = [&](int s) { return bars + 8u * (S + s); };
-  const uint32_t accf0 = bars + 8u * (2 * S);
-  const uint32_t acce0 = accf0 + 16u;
-  const uint32_t drain_bar = acce0 + 16u;
+  const uint32_t accf0 = bars + 8u * (2 * S);   // slot filled (MMA -> epilogue)
+  const uint32_t acce0 = accf0 + 8u * H2_MAX_R;  // slot read (epilogue -> MMA)
+  const uint32_t drain_bar = acce0 + 8u * H2_MAX_R;
   const uint32_t misc = (drain_bar + 8u + 15u) & ~15u;
   uint32_t* const tmem_slot = reinterpret_cast<uint32_t*>(gbase + (misc - base));
   volatile int* const abort_flag = reinterpret_cast<volatile int*>(gbase + (misc - base) + 4);
   int* const s_drafts = reinterpret_cast<int*>(gbase + (misc - base) + 16);
-  float* const stats =
-      reinterpret_cast<float*>(gbase + (misc - base) + 16 + MAX_ZPAIRS_PER_CHUNK * 4);
-  const int tab = p.Pcp;
-  // per-warp staging rows of the transposed tile reduction (16-byte aligned)
-  float* const scr_base = reinterpret_cast<float*>(
-      (reinterpret_cast<uintptr_t>(stats + 4 * tab * HEAD_STAT_STRIDE) + 15) & ~uintptr_t(15));
+  // statistics tables [4 quadrants][Pcp][HEAD_STAT_STRIDE] over the drained
+  // pipeline stages, written once at the end
+  float* const stats = reinterpret_cast<float*>(gbase);
 
   const int pair0 = chunk * p.Pc;
   const int npairs = min(p.Pc, p.P - pair0);
@@ -188,10 +534,10 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
       mbar_init(full_bar(s), 1);   // the even CTA's expect-tx; both CTAs' bytes
       mbar_init(empty_bar(s), 1);  // the pair's MMA commit
     }
-    mbar_init(accf0, 1);
-    mbar_init(accf0 + 8, 1);
-    mbar_init(acce0, 2 * EPI);  // the epilogue warps of both CTAs
-    mbar_init(acce0 + 8, 2 * EPI);
+    for (int k = 0; k < H2_MAX_R; ++k) {
+      mbar_init(accf0 + 8u * k, 1);
+      mbar_init(acce0 + 8u * k, 2 * H2_EPI);  // the epilogue warps of both CTAs
+    }
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
     fence_barrier_init();
@@ -209,9 +555,8 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
   }
   if (warp >= 2) {
     const int e = threadIdx.x - 64;
-    for (int j = e; j < MAX_ZPAIRS_PER_CHUNK; j += EPI * 32)
+    for (int j = e; j < MAX_ZPAIRS_PER_CHUNK; j += H2_EPI * 32)
       s_drafts[j] = (j < npairs) ? pair_draft(p.drafts, pair0 + j, p.gamma) : -1;
-    head_stats_init(stats, 4 * tab, e, EPI * 32);
   }
   // both CTAs: barriers initialised and TMEM allocated before any cross-CTA use
   tc_fence_before();
@@ -229,6 +574,7 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
       int s = 0, issued = 0;
       uint32_t ph = 0;
       bool ok = true;
+      const int hrow = chunk * H * p.Ns + static_cast<int>(rank) * static_cast<int>(b_rows);
       for (int pt = pt0; pt < pt1 && ok; ++pt) {
         const int v0 = pt * 2 * H2_BM + static_cast<int>(rank) * H2_BM;
         for (int kb = 0; kb < p.n_kb; ++kb) {
@@ -238,7 +584,6 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
           }
           if (leader) mbar_arrive_expect_tx(full_bar(s), 2u * (H2_A_BYTES + b_bytes));
           const uint32_t fb = mapa_shared(full_bar(s), leader_rank);
-          const int hrow = chunk * p.N + static_cast<int>(rank) * (p.N / 2);
 #pragma unroll
           for (int hf = 0; hf < 2; ++hf) {
             tma_load_2d_pair(a_tiles + s * H2_A_BYTES + hf * H2_A_HALF, &tm_w, kb * H2_BK + 64 * hf,
@@ -265,37 +610,51 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer (even CTA)
     if (leader && lane == 0) {
-      const uint32_t idesc = idesc_bf16_f32(2 * H2_BM, p.N);
+      const uint32_t idesc = idesc_bf16_f32(2 * H2_BM, p.Ns);
       // descriptors of stage 0; stage s adds s * bytes / 16 to the start field
       const uint64_t ad0 = sw128_kmajor_desc(a_tiles), bd0 = sw128_kmajor_desc(b_tiles);
       const uint32_t a_step = H2_A_BYTES >> 4, b_step = b_bytes >> 4;
       const uint32_t a_hstep = H2_A_HALF >> 4, b_hstep = b_half >> 4;
+      const uint32_t b_sub = (static_cast<uint32_t>(p.Ns / 2) * 128u) >> 4;  // next sub-group's rows
       int s = 0;
       uint32_t ph = 0;
       bool ok = true;
-      for (int pt = pt0, lt = 0; pt < pt1 && ok; ++pt, ++lt) {
-        const int slot = lt & 1;
-        if (!mbar_wait(acce0 + 8u * slot, ((lt >> 1) & 1) ^ 1u, abort_flag, p.status)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(slot * p.N);
-        for (int kb = 0; kb < p.n_kb; ++kb) {
+      int u = 0;  // accumulator uses so far (tile * H + sub-group)
+      for (int pt = pt0; pt < pt1 && ok; ++pt) {
+        uint32_t d_tmem[H2_MAX_H] = {0u, 0u};
+        for (int kb = 0; kb < p.n_kb && ok; ++kb) {
           if (!mbar_wait(full_bar(s), ph, abort_flag, p.status)) {
             ok = false;
             break;
           }
           const uint64_t ad = ad0 + static_cast<uint32_t>(s) * a_step;
           const uint64_t bd = bd0 + static_cast<uint32_t>(s) * b_step;
-          tc2_mma_stage8(d_tmem, ad, bd, a_hstep, b_hstep, idesc, kb != 0 ? 1u : 0u);
+#pragma unroll
+          for (int h = 0; h < H2_MAX_H; ++h) {
+            if (h >= H) break;
+            if (kb == 0) {
+              // the slot of this sub-group must have been read by the epilogue
+              const int uu = u + h, sl = uu % R;
+              if (!mbar_wait(acce0 + 8u * sl, ((uu / R) & 1) ^ 1u, abort_flag, p.status)) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+              d_tmem[h] = tmem_base + static_cast<uint32_t>(sl * p.Ns);
+            }
+            tc2_mma_stage8(d_tmem[h], ad, bd + static_cast<uint32_t>(h) * b_sub, a_hstep, b_hstep,
+                           idesc, kb != 0 ? 1u : 0u);
+          }
           tc2_commit(empty_bar(s), pair_mask);
           if (++s == S) {
             s = 0;
             ph ^= 1u;
           }
         }
-        if (ok) tc2_commit(accf0 + 8u * slot, pair_mask);
+        if (ok) {
+          for (int h = 0; h < H; ++h) tc2_commit(accf0 + 8u * ((u + h) % R), pair_mask);
+        }
+        u += H;
       }
       // every MMA issued must be complete before TMEM is released
       tc2_commit(drain_bar, static_cast<uint16_t>(1u << crank));
@@ -304,46 +663,190 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
     __syncwarp();
   } else {
     // ------------------------------------------------------------ epilogue (both CTAs)
-    const int q = warp & 3;    // TMEM lane quadrant this warp may access
-    const int ew = warp - 2;   // statistics table of this warp
-    const int half = ew >> 2;  // which alternate groups of 8 pairs it takes
-    // the two warps of a quadrant take disjoint pairs: they share one table
-    float* const wstats = stats + q * tab * HEAD_STAT_STRIDE;
+    const int q = warp & 3;          // TMEM lane quadrant this warp may access
+    const int kq = (warp - 2) >> 2;  // this warp's index within its quadrant
+    const float beta = 1.f - p.alpha;
+    constexpr int gsz = ZONLY ? 16 : 8;  // pairs per group
+    const int ng = p.Ph / gsz;           // groups per sub-group
+    // this warp's groups: g = kq, kq + WPQ, ... of every sub-group, in order
+    const int n_h0 = kq < ng ? (ng - kq + H2_WPQ - 1) / H2_WPQ : 0;
+    const int n_mine = H * n_h0;
+    LaneStats st;
+    const int qn = ZONLY ? (lane >> 4) : (lane >> 3);
+    const bool is_best = ZONLY ? qn == 1 : qn == 3;
+#pragma unroll
+    for (int i = 0; i < H2_MAX_OWN; ++i) {
+      st.m[i] = NEG_INF;
+      st.s[i] = is_best ? __int_as_float(INT_MAX) : 0.f;
+      st.t[i] = 0.f;
+    }
+    const uint32_t lane_q = static_cast<uint32_t>(q * 32) << 16;
     float* const gathered = p.gathered + static_cast<long long>(pair0) * GATHER_FIELDS;
-    for (int pt = pt0, lt = 0; pt < pt1; ++pt, ++lt) {
-      const int slot = lt & 1;
-      const bool ok = mbar_wait(accf0 + 8u * slot, (lt >> 1) & 1, abort_flag, p.status);
-      if (!__all_sync(0xffffffffu, ok)) break;
+    float* const zout = p.zout ? p.zout + static_cast<long long>(pair0) * p.V : nullptr;
+    // slot and phase of the accumulator use the MMA issuer counts next
+    int use_slot = 0, use_phase = 0;
+    bool ok = true;
+    int slot0 = 0, slot1 = 0, phase0 = 0, phase1 = 0;  // of sub-groups 0 and 1 this tile
+    auto slot_of = [&](int h) { return h == 0 ? slot0 : slot1; };
+    auto wait_slot = [&](int h) -> bool {
+      const bool w = mbar_wait(accf0 + 8u * slot_of(h), h == 0 ? phase0 : phase1, abort_flag,
+                               p.status);
       tc_fence_after();
-      const int v = pt * 2 * H2_BM + static_cast<int>(rank) * H2_BM + q * 32 + lane;
-      const bool valid = v < p.V;
-      const uint32_t trow =
-          tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(slot * p.N);
-      float* const zout = p.zout ? p.zout + static_cast<long long>(pair0) * p.V : nullptr;
-      for (int g8 = 8 * half; g8 < npairs; g8 += 8 * (EPI / 4)) {
-        if (p.zonly) {
-          float z[8];
-          tmem_ld8(trow + g8, z);
-          tmem_ld_wait();
-          head_tile_z8_t(z, g8, npairs, v, valid, s_drafts, wstats, gathered,
-                         scr_base + ew * HEAD_SCR_FLOATS, lane, zout, p.V);
-          continue;
-        }
-        float o[8], r[8];
-        tmem_ld8(trow + g8, o);
-        tmem_ld8(trow + p.Pcp + g8, r);
-        tmem_ld_wait();
-        head_tile_pairs8_t(o, r, g8, npairs, v, valid, p.alpha, s_drafts, wstats, gathered,
-                           scr_base + ew * HEAD_SCR_FLOATS, lane, zout, p.V);
-      }
+      return __all_sync(0xffffffffu, w);
+    };
+    auto release_slot = [&](int h) {
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(mapa_shared(acce0 + 8u * slot, leader_rank));
+      if (lane == 0) mbar_arrive_cluster(mapa_shared(acce0 + 8u * slot_of(h), leader_rank));
+    };
+    // first TMEM column of group g of sub-group h of the current tile
+    auto tcol = [&](int h, int g) -> uint32_t {
+      return tmem_base + lane_q + static_cast<uint32_t>(slot_of(h) * p.Ns + g * gsz);
+    };
+    auto load_group = [&](uint32_t t0, uint32_t* b) {
+      if (ZONLY) {
+        tmem_ld_16x256b_x2(t0, b);
+        tmem_ld_16x256b_x2(t0 + (16u << 16), b + 8);
+      } else {
+        tmem_ld_16x256b(t0, b);
+        tmem_ld_16x256b(t0 + (16u << 16), b + 4);
+        tmem_ld_16x256b(t0 + static_cast<uint32_t>(p.Ph), b + 8);
+        tmem_ld_16x256b(t0 + static_cast<uint32_t>(p.Ph) + (16u << 16), b + 12);
+      }
+    };
+    // drafts of this lane's columns of group (h, g)
+    constexpr int NC = ZONLY ? 4 : 2;
+    auto load_drafts = [&](int h, int g, int (&x)[NC]) {
+      const int c4 = lane & 3;
+      const int gp = h * p.Ph + g * gsz;
+#pragma unroll
+      for (int j = 0; j < NC; ++j)
+        x[j] = s_drafts[gp + 2 * c4 + (j & 1) + 8 * (j >> 1)];  // -1: no draft (or padding)
+    };
+    for (int pt = pt0; pt < pt1 && ok; ++pt) {
+      slot0 = use_slot;
+      phase0 = use_phase;
+      if (++use_slot == R) {
+        use_slot = 0;
+        use_phase ^= 1;
+      }
+      if (H == 2) {
+        slot1 = use_slot;
+        phase1 = use_phase;
+        if (++use_slot == R) {
+          use_slot = 0;
+          use_phase ^= 1;
+        }
+      }
+      const int v_row0 = pt * 2 * H2_BM + static_cast<int>(rank) * H2_BM + q * 32;
+      if (n_mine == 0) {
+        // a warp without groups still counts on every slot's barrier
+        for (int h = 0; h < H && ok; ++h) {
+          ok = wait_slot(h);
+          if (ok) release_slot(h);
+        }
+        continue;
+      }
+      uint32_t cb[16], nb[16];
+      int cx[NC], nx[NC];
+      if (!wait_slot(0)) {
+        ok = false;
+        break;
+      }
+      load_group(tcol(0, kq), cb);
+      load_drafts(0, kq, cx);
+      tmem_ld_wait();
+      after_ld(cb);
+      int h = 0, gi = 0;  // sub-group and index within it of group idx
+#pragma unroll 1
+      for (int idx = 0; idx < n_mine; ++idx) {
+        const int g = gi * H2_WPQ + kq;
+        // the next group
+        int nh = h, ngi = gi + 1;
+        if (ngi == n_h0) {
+          ++nh;
+          ngi = 0;
+        }
+        const bool more = idx + 1 < n_mine;
+        if (more && nh != h && !wait_slot(nh)) {
+          ok = false;
+          break;
+        }
+        if (more) {  // lands while this group is reduced
+          load_group(tcol(nh, ngi * H2_WPQ + kq), nb);
+          load_drafts(nh, ngi * H2_WPQ + kq, nx);
+        }
+        const int gpair = h * p.Ph + g * gsz;
+        TileOut t;
+        if constexpr (ZONLY)
+          t = group16_z(cb, cb + 8, v_row0, p.V, cx, gpair, npairs, gathered, zout, lane);
+        else
+          t = group8_fused(cb, cb + 8, v_row0, p.V, p.alpha, beta, cx, gpair, npairs, gathered,
+                           zout, lane);
+        st.fold0(is_best, t);
+        st.rotate();
+        tmem_ld_wait();
+        after_ld(nb);
+#pragma unroll
+        for (int k = 0; k < 16; ++k) cb[k] = nb[k];
+#pragma unroll
+        for (int j = 0; j < NC; ++j) cx[j] = nx[j];
+        // the last group of a sub-group has been read: its slot is free
+        if (!more || nh != h) release_slot(h);
+        h = nh;
+        gi = ngi;
+      }
+      // back to the tile-start alignment of the ring
+#pragma unroll 1
+      for (int k = n_mine; k < H2_MAX_OWN; ++k) st.rotate();
     }
-    named_bar_sync(1, EPI * 32);
+    // every accumulator has been read (all MMAs of the pair complete), so the
+    // pipeline stages of this CTA are no longer written or read: the tables go
+    // over them
+    named_bar_sync(1, H2_EPI * 32);
+    const int c4 = lane & 3, rq = lane >> 2;
+    const int tab = p.Pcp;
+#pragma unroll
+    for (int idx = 0; idx < H2_MAX_OWN; ++idx) {
+      if (idx >= n_mine) break;
+      const int h = idx / n_h0, g = (idx % n_h0) * H2_WPQ + kq;
+      int pj;
+      if (ZONLY) {
+        const int jj = rq & 3;
+        pj = h * p.Ph + g * 16 + 2 * c4 + (jj & 1) + 8 * (jj >> 1);
+      } else {
+        pj = h * p.Ph + g * 8 + 2 * c4 + (rq & 1);
+      }
+      if (pj < npairs) {
+        float* d = stats + (q * tab + pj) * HEAD_STAT_STRIDE;
+        if (is_best) {
+          d[ST_BEST_V] = st.m[idx];
+          d[ST_BEST_I] = st.s[idx];
+        } else if (ZONLY) {
+          d[ST_M_Z] = st.m[idx];
+          d[ST_S_Z] = st.s[idx];
+          d[ST_M_O] = NEG_INF;  // no separate o / o' in this head
+          d[ST_S_O] = 0.f;
+          d[ST_T_O] = 0.f;
+          d[ST_M_R] = NEG_INF;
+          d[ST_S_R] = 0.f;
+        } else if (qn == 0) {
+          d[ST_M_O] = st.m[idx];
+          d[ST_S_O] = st.s[idx];
+          d[ST_T_O] = st.t[idx];
+        } else if (qn == 1) {
+          d[ST_M_R] = st.m[idx];
+          d[ST_S_R] = st.s[idx];
+        } else {
+          d[ST_M_Z] = st.m[idx];
+          d[ST_S_Z] = st.s[idx];
+        }
+      }
+    }
+    named_bar_sync(1, H2_EPI * 32);
     head_stats_finish(stats, 4, tab, npairs,
                       p.partials + (static_cast<long long>(slot_id) * p.P + pair0) * HEAD_STAT_FIELDS,
-                      threadIdx.x - 64, EPI * 32);
+                      threadIdx.x - 64, H2_EPI * 32);
   }
 
   tc_fence_before();
@@ -378,62 +881,56 @@ __global__ void __launch_bounds__(h2_threads(EPI), 1)
 // ---------------------------------------------------------------- host side
 
 namespace {
-#ifndef RV_HEAD2_EPI4_MAX_PAIRS
-#define RV_HEAD2_EPI4_MAX_PAIRS 72
-#endif
-// epilogue warps: four (one per TMEM lane quadrant) up to this many pairs, else
-// eight.  At 72 pairs (8B, B=16) four warps leave room for a fourth pipeline
-// stage: 264 -> 254 us for the head.
-int h2_epi_warps(int pairs) { return pairs <= RV_HEAD2_EPI4_MAX_PAIRS ? 4 : 8; }
-size_t h2_fixed_bytes(int pairs) {
-  return 1024 + 256 + 16 + MAX_ZPAIRS_PER_CHUNK * 4 +
-         static_cast<size_t>(4) * pairs * HEAD_STAT_STRIDE * 4 + 64 + 16 +
-         static_cast<size_t>(h2_epi_warps(pairs)) * HEAD_SCR_FLOATS * 4;
-}
-uint32_t h2_tmem_cols(int N) {
-  uint32_t need = static_cast<uint32_t>(2 * N), c = 32;
-  while (c < need) c <<= 1;
+size_t h2_fixed_bytes() { return 1024 + 256 + 16 + MAX_ZPAIRS_PER_CHUNK * 4 + 64; }
+uint32_t h2_tmem_cols(int cols) {
+  uint32_t c = 32;
+  while (c < static_cast<uint32_t>(cols)) c <<= 1;
   return c;
 }
+size_t h2_stage_bytes(int N) { return H2_A_BYTES + static_cast<size_t>(N / 2) * 256; }
 }  // namespace
 
 size_t head_tc2_smem_bytes(int N, int pairs, int stages) {
-  return h2_fixed_bytes(pairs) + static_cast<size_t>(stages) * (H2_A_BYTES + (N / 2) * 256);
+  (void)pairs;
+  return h2_fixed_bytes() + static_cast<size_t>(stages) * h2_stage_bytes(N);
 }
 
 #ifndef RV_HEAD2_STAGE_TARGET_KB
 #define RV_HEAD2_STAGE_TARGET_KB 200
 #endif
 int head_tc2_stages(int N, int pairs, size_t smem_limit) {
-  const size_t per = H2_A_BYTES + (N / 2) * 256;
-  if (smem_limit <= h2_fixed_bytes(pairs)) return 0;
-  const int most = static_cast<int>((smem_limit - h2_fixed_bytes(pairs)) / per);
+  const size_t per = h2_stage_bytes(N);
+  if (smem_limit <= h2_fixed_bytes()) return 0;
+  const int most = static_cast<int>((smem_limit - h2_fixed_bytes()) / per);
   const int want = static_cast<int>((RV_HEAD2_STAGE_TARGET_KB * 1024 + per - 1) / per);
-  return std::max(0, std::min(std::min(most, 8), std::max(3, want)));
+  int st = std::max(0, std::min(std::min(most, 8), std::max(3, want)));
+  // the statistics tables written at the end go over the stages
+  const size_t tables = static_cast<size_t>(4) * pairs * HEAD_STAT_STRIDE * 4;
+  while (st > 0 && st < most && static_cast<size_t>(st) * per < tables) ++st;
+  return static_cast<size_t>(st) * per >= tables ? st : 0;
 }
 
-template <int EPI>
+template <bool ZONLY>
 static cudaError_t head_tc2_configure_one(size_t smem_bytes) {
-  cudaError_t e = cudaFuncSetAttribute(head_tc2_kernel<EPI>,
+  cudaError_t e = cudaFuncSetAttribute(head_tc2_kernel<ZONLY>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem_bytes));
-  if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(head_tc2_kernel<EPI>,
-                           cudaFuncAttributePreferredSharedMemoryCarveout,
-                           cudaSharedmemCarveoutMaxShared);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(head_tc2_kernel<ZONLY>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             cudaSharedmemCarveoutMaxShared);
   return e;
 }
 
 cudaError_t head_tc2_configure(size_t smem_bytes) {
-  cudaError_t e = head_tc2_configure_one<4>(smem_bytes);
-  if (e == cudaSuccess) e = head_tc2_configure_one<8>(smem_bytes);
+  cudaError_t e = head_tc2_configure_one<false>(smem_bytes);
+  if (e == cudaSuccess) e = head_tc2_configure_one<true>(smem_bytes);
   return e;
 }
 
 int head_tc2_max_pairs(int N, int pairs, int stages) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(2, 1, 1);
-  cfg.blockDim = dim3(h2_threads(h2_epi_warps(pairs)), 1, 1);
+  cfg.blockDim = dim3(H2_THREADS, 1, 1);
   cfg.dynamicSmemBytes = head_tc2_smem_bytes(N, pairs, stages);
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -443,9 +940,8 @@ int head_tc2_max_pairs(int N, int pairs, int stages) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int n = 0;
-  const bool e4 = h2_epi_warps(pairs) == 4;
-  cudaError_t e = e4 ? cudaOccupancyMaxActiveClusters(&n, head_tc2_kernel<4>, &cfg)
-                     : cudaOccupancyMaxActiveClusters(&n, head_tc2_kernel<8>, &cfg);
+  // both instantiations have the same block size and shared memory
+  cudaError_t e = cudaOccupancyMaxActiveClusters(&n, head_tc2_kernel<false>, &cfg);
   if (e != cudaSuccess) {
     cudaGetLastError();
     return 0;
@@ -453,12 +949,41 @@ int head_tc2_max_pairs(int N, int pairs, int stages) {
   return n;
 }
 
+void head_pair_chunks(int P, int* n_chunks, int* pairs_per_chunk, int* sub, int* sub_pairs) {
+  const int n = std::max(1, (P + HEAD_PAIR_MAX_CHUNK - 1) / HEAD_PAIR_MAX_CHUNK);
+  const int pc = (P + n - 1) / n;
+  *n_chunks = n;
+  *pairs_per_chunk = pc;
+  *sub = pc > MAX_PAIRS_PER_CHUNK ? 2 : 1;
+  const int per = (pc + *sub - 1) / *sub;
+  *sub_pairs = (per + 7) / 8 * 8;
+}
+
+int head_tc2_slots(const HeadPlan& pl) {
+  const int ns = pl.zonly ? pl.sub_pairs : 2 * pl.sub_pairs;
+  return std::min(H2_MAX_R, 512 / ns);
+}
+
+bool head_tc2_supports(const HeadPlan& pl) {
+  const int gsz = pl.zonly ? 16 : 8;
+  if (pl.sub < 1 || pl.sub > H2_MAX_H || pl.sub_pairs < gsz || pl.sub_pairs % gsz != 0)
+    return false;
+  if (pl.zonly && pl.sub != 1) return false;
+  if (pl.sub * pl.sub_pairs != pl.pad_pairs) return false;
+  const int ng = pl.sub_pairs / gsz;
+  const int per_warp = pl.sub * ((ng + H2_WPQ - 1) / H2_WPQ);
+  return per_warp <= H2_MAX_OWN && head_tc2_slots(pl) >= pl.sub + 1;
+}
+
 cudaError_t launch_head_tc2(const HeadArgs& a, const HeadPlan& pl, const HeadTcLaunch& l,
                             const HeadFinal* fin, cudaStream_t s) {
   Head2Params p;
   p.V = a.V;
   p.n_kb = (a.H + H2_BK - 1) / H2_BK;
-  p.N = pl.N;
+  p.H = pl.sub;
+  p.Ph = pl.sub_pairs;
+  p.Ns = pl.zonly ? pl.sub_pairs : 2 * pl.sub_pairs;
+  p.R = head_tc2_slots(pl);
   p.Pcp = pl.pad_pairs;
   p.Pc = pl.pairs_per_chunk;
   p.P = pl.P;
@@ -471,7 +996,7 @@ cudaError_t launch_head_tc2(const HeadArgs& a, const HeadPlan& pl, const HeadTcL
   p.fused = fin != nullptr ? 1 : 0;
   if (fin) p.fin = *fin;
   p.slots = pl.slots;
-  p.tmem_cols = h2_tmem_cols(pl.N);
+  p.tmem_cols = h2_tmem_cols(p.R * p.Ns);
   p.alpha = a.alpha;
   p.drafts = a.drafts;
   p.partials = a.partials;
@@ -481,8 +1006,7 @@ cudaError_t launch_head_tc2(const HeadArgs& a, const HeadPlan& pl, const HeadTcL
   p.zonly = pl.zonly ? 1 : 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(pl.slots, pl.n_chunks, 1);
-  const int epi = h2_epi_warps(pl.pad_pairs);
-  cfg.blockDim = dim3(h2_threads(epi), 1, 1);
+  cfg.blockDim = dim3(H2_THREADS, 1, 1);
   cfg.dynamicSmemBytes = l.smem_bytes;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
@@ -494,8 +1018,8 @@ cudaError_t launch_head_tc2(const HeadArgs& a, const HeadPlan& pl, const HeadTcL
   attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  if (epi == 4) return cudaLaunchKernelEx(&cfg, head_tc2_kernel<4>, l.tm_w, l.tm_h, p);
-  return cudaLaunchKernelEx(&cfg, head_tc2_kernel<8>, l.tm_w, l.tm_h, p);
+  if (pl.zonly) return cudaLaunchKernelEx(&cfg, head_tc2_kernel<true>, l.tm_w, l.tm_h, p);
+  return cudaLaunchKernelEx(&cfg, head_tc2_kernel<false>, l.tm_w, l.tm_h, p);
 }
 
 }  // namespace rv

@@ -168,6 +168,8 @@ HeadPlan head_plan(int B, int gamma, int V, int num_sms, bool tc, bool zonly = f
   p.pairs_per_chunk = (p.P + p.n_chunks - 1) / p.n_chunks;
   p.pad_pairs = zonly ? (p.pairs_per_chunk + 15) / 16 * 16 : (p.pairs_per_chunk + 7) / 8 * 8;
   p.N = zonly ? p.pad_pairs : 2 * p.pad_pairs;
+  p.sub = 1;
+  p.sub_pairs = p.pad_pairs;
   p.n_vtiles = (V + 127) / 128;
   p.pair = false;
   if (tc) {  // one persistent CTA per SM; the vocab is split in whole tiles
@@ -179,6 +181,18 @@ HeadPlan head_plan(int B, int gamma, int V, int num_sms, bool tc, bool zonly = f
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// The CTA-pair plan of the two-distribution head: chunks of up to
+// HEAD_PAIR_MAX_CHUNK pairs, each one pass over the weight; a chunk of more
+// than MAX_PAIRS_PER_CHUNK pairs (too many columns for two accumulators) is
+// two sub-groups with accumulators of their own.
+HeadPlan head_pair_plan(const HeadPlan& base) {
+  HeadPlan p = base;
+  head_pair_chunks(p.P, &p.n_chunks, &p.pairs_per_chunk, &p.sub, &p.sub_pairs);
+  p.pad_pairs = p.sub * p.sub_pairs;
+  p.N = 2 * p.pad_pairs;
+  return p;
+}
 
 struct ProfScope {
   rv_handle* h;
@@ -271,6 +285,9 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
       const int nch = (P + MAX_PAIRS_PER_CHUNK - 1) / MAX_PAIRS_PER_CHUNK;
       const int pc = (P + nch - 1) / nch;
       hsel_rows = std::max(hsel_rows, static_cast<size_t>(nch) * 2 * ((pc + 7) / 8 * 8));
+      int pn = 0, ppc = 0, psub = 0, psp = 0;  // the CTA-pair plan's chunks
+      head_pair_chunks(P, &pn, &ppc, &psub, &psp);
+      hsel_rows = std::max(hsel_rows, static_cast<size_t>(pn) * 2 * psub * psp);
       // the pre-blended head's plan: one row per pair, 16-row aligned chunks
       const int nz = (P + MAX_ZPAIRS_PER_CHUNK - 1) / MAX_ZPAIRS_PER_CHUNK;
       const int pz = (P + nz - 1) / nz;
@@ -591,19 +608,23 @@ int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_
                           bf16 && h->head_mode == RV_HEAD_STANDARD);
   if (bf16 && pl.N >= HEAD_PAIR_MIN_N) {
     // CTA pairs: as many as fit at once (two CTAs of a pair share a GPC)
-    if (h->head_pair_cached_N != 2 * pl.N + pl.zonly) {
-      h->head_pair_stages = head_tc2_stages(pl.N, pl.pad_pairs, h->smem_optin);
-      h->head_pair_max = h->head_pair_stages >= 2
-                             ? head_tc2_max_pairs(pl.N, pl.pad_pairs, h->head_pair_stages)
-                             : 0;
-      h->head_pair_cached_N = 2 * pl.N + pl.zonly;
-    }
-    const int n_pt = (c.vocab + 255) / 256;
-    const int pairs =
-        std::min({h->num_sms / 2 / pl.n_chunks, h->head_pair_max / pl.n_chunks, n_pt});
-    if (pairs >= 1) {
-      pl.pair = true;
-      pl.slots = 2 * pairs;
+    HeadPlan pp = pl.zonly ? pl : head_pair_plan(pl);
+    if (head_tc2_supports(pp)) {
+      if (h->head_pair_cached_N != 2 * pp.N + pp.zonly) {
+        h->head_pair_stages = head_tc2_stages(pp.N, pp.pad_pairs, h->smem_optin);
+        h->head_pair_max = h->head_pair_stages >= 2
+                               ? head_tc2_max_pairs(pp.N, pp.pad_pairs, h->head_pair_stages)
+                               : 0;
+        h->head_pair_cached_N = 2 * pp.N + pp.zonly;
+      }
+      const int n_pt = (c.vocab + 255) / 256;
+      const int pairs =
+          std::min({h->num_sms / 2 / pp.n_chunks, h->head_pair_max / pp.n_chunks, n_pt});
+      if (pairs >= 1) {
+        pl = pp;
+        pl.pair = true;
+        pl.slots = 2 * pairs;
+      }
     }
   }
   ProfScope prof_all(h, RV_PROF_HEAD, s);

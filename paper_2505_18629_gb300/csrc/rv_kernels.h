@@ -45,6 +45,10 @@ struct HeadPlan {
   int n_vtiles;        // ceil(V / 128)
   int slots;           // CTAs per chunk (= partial slots)
   bool pair;           // CTA-pair kernel (k_head_tc2.cu): slots = 2 * pairs
+  // CTA-pair kernel: the chunk's pairs in `sub` sub-groups of `sub_pairs`
+  // (pad_pairs = sub * sub_pairs), one accumulator each; 1 and pad_pairs otherwise
+  int sub = 1;
+  int sub_pairs = 0;
   bool zonly = false;  // pre-blended head: one blended row per pair, z statistics only
   bool standard = false;  // standard verification: z-only on the original rows (Lh = gamma+1)
 };
@@ -177,12 +181,22 @@ cudaError_t launch_head_simt(const HeadArgs& a, const HeadPlan& p, cudaStream_t 
 #define RV_HEAD_PAIR_MIN_N 96
 #endif
 constexpr int HEAD_PAIR_MIN_N = RV_HEAD_PAIR_MIN_N;  // N from which pairs are used
+// Chunks of the CTA-pair head: at most HEAD_PAIR_MAX_CHUNK pairs per chunk; a
+// chunk of more than MAX_PAIRS_PER_CHUNK pairs is split into two sub-groups.
+#ifndef RV_HEAD_PAIR_MAX_CHUNK
+#define RV_HEAD_PAIR_MAX_CHUNK 160
+#endif
+constexpr int HEAD_PAIR_MAX_CHUNK = RV_HEAD_PAIR_MAX_CHUNK;
+void head_pair_chunks(int P, int* n_chunks, int* pairs_per_chunk, int* sub, int* sub_pairs);
 size_t head_tc2_smem_bytes(int N, int pairs, int stages);
 int head_tc2_stages(int N, int pairs, size_t smem_limit);
 cudaError_t head_tc2_configure(size_t smem_bytes);
 // co-resident CTA pairs (occupancy query)
 int head_tc2_max_pairs(int N, int pairs, int stages);
 
+// accumulator slots of the plan, and whether the kernel takes its sub-groups
+int head_tc2_slots(const HeadPlan& p);
+bool head_tc2_supports(const HeadPlan& p);
 cudaError_t launch_head_tc2(const HeadArgs& a, const HeadPlan& p, const HeadTcLaunch& l,
                             const HeadFinal* fin, cudaStream_t s);
 

@@ -51,12 +51,11 @@ FALLBACK_BF16_TFLOPS = 1900.0
 # dram__bytes_write.sum` on the workload named (see profiles/), valid only while
 # the kernel sources hash to `src_sha`.
 NCU_TRAFFIC = {
-    "llama3-8b-b1": {"bytes": 1050912512 + 2772736, "src_sha": "2322d678d1a54902",
+    "llama3-8b-b1": {"bytes": 1050899456 + 3078144, "src_sha": "44ea9a01f2baf9a7",
                      "summary": "profiles/head_tc_llama3-8b-b1.md"},
-    "llama3-8b-b16": {"bytes": 1053160704 + 2951680, "src_sha": "2322d678d1a54902",
+    "llama3-8b-b16": {"bytes": 1053382656 + 5539584, "src_sha": "44ea9a01f2baf9a7",
                       "summary": "profiles/head_tc2_llama3-8b-b16.md"},
 }
-
 
 def _kernel_src_hash() -> str:
     h = hashlib.sha256()
@@ -680,7 +679,9 @@ def measure_workload(wl, args, dev, world, rank, clocks):
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for i in range(args.steps):
-        sampled = i % PROF_EVERY == PROF_EVERY - 1
+        # (a run shorter than PROF_EVERY samples its last step)
+        sampled = i % PROF_EVERY == PROF_EVERY - 1 or (args.steps < PROF_EVERY and
+                                                       i == args.steps - 1)
         if sampled:
             rv.rv_profile_enable(h, 1 << rv.RV_PROF_HEAD)
         step()

@@ -1139,9 +1139,26 @@ def test_llama3_70b_b32_sampled(gu):
     _check(gu, synth.WORKLOADS["llama3-70b-b32"], seqs=[0, 17, 31])
 
 
-@pytest.mark.parametrize("name", ["sweep-b1-g2-c1024", "sweep-b64-g8-c8192", "sweep-b4-g4-c8192"])
+# One sweep point per launch path (attention kernel, attention beside / before
+# the LM head, LM-head kernel, sub-groups and chunks of its pairs, merge in
+# the head's last CTA or a separate launch):
+#   b1-g2-c1024   mma.sync attention beside the head; one-CTA head, merged in its last CTA
+#   b4-g4-c8192   mma.sync attention before the head (KV capacity above 4608)
+#   b4-g8-c1024   one-CTA head with 36 pairs (N = 80)
+#   b16-g2-c1024  tcgen05 attention + chunk merge; CTA-pair head, 48 pairs, merged in its last CTA
+#   b16-g4-c1024  CTA-pair head, 80 pairs, separate merge launch
+#   b16-g4-c8192  as above with the attention before the head
+#   b16-g8-c8192  CTA-pair head, 144 pairs in two sub-groups; attention before the head
+#   b64-g2-c1024  CTA-pair head, two chunks of 96 pairs
+#   b64-g4-c1024  CTA-pair head, two chunks of 160 pairs in two sub-groups
+#   b64-g8-c8192  four chunks of 144 pairs in two sub-groups; attention before the head
+@pytest.mark.parametrize("name", ["sweep-b1-g2-c1024", "sweep-b4-g4-c8192", "sweep-b4-g8-c1024",
+                                  "sweep-b16-g2-c1024", "sweep-b16-g4-c1024",
+                                  "sweep-b16-g4-c8192", "sweep-b16-g8-c8192",
+                                  "sweep-b64-g2-c1024", "sweep-b64-g4-c1024",
+                                  "sweep-b64-g8-c8192"])
 def test_sweep_points(gu, name):
     from paper_2505_18629_gb300 import synth
     wl = synth.workload(name)
-    seqs = None if wl.B <= 4 else [0, 33, 63]
+    seqs = None if wl.B <= 4 else ([0, 7, 15] if wl.B <= 16 else [0, 33, 63])
     _check(gu, wl, seqs=seqs)

@@ -163,11 +163,13 @@ cudaError_t launch_prep(const HeadArgs& a, const HeadPlan& p, void* hsel, const 
 }
 
 // ---------------------------------------------------------------- head finalize
-// One CTA per sequence; `wpp` warps per position i (pair p = b*(gamma+1)+i)
-// merge the slots' (max, sum) triples and argmax (each lane about one slot),
-// then one thread finishes the position's scores.  Inside rv_verify_step the
-// CTA then runs the exact-match acceptance of its sequence (Alg. 2).
-constexpr int FIN_MAX_WARPS = 32;
+// One CTA per position p = b*(gamma+1) + i: its threads merge the slots'
+// (max, sum) triples and argmax candidates (16-byte loads, a few slots per
+// thread), then thread 0 finishes the position's scores.  Inside
+// rv_verify_step each sequence's acceptance follows: the last of its
+// positions' CTAs to finish (a ticket per sequence, re-armed by that CTA)
+// reads the positions' choices and scores back and runs Alg. 2 (or Alg. 3).
+constexpr int FIN_THREADS = 128;
 
 struct MergeStat {
   float mo, so, to, mr, sr, mz, sz, bv;
@@ -198,91 +200,90 @@ __device__ __forceinline__ MergeStat shfl_stat(const MergeStat& s, int o) {
   return r;
 }
 
-__global__ void head_finalize_kernel(const float* __restrict__ partials,
-                                     const float* __restrict__ gathered,
-                                     const int32_t* __restrict__ drafts, int P, int gamma, int V,
-                                     int slots, int wpp, float* __restrict__ scores,
-                                     int32_t* __restrict__ argmax_out, float* __restrict__ margin,
-                                     unsigned* status, AcceptArgs acc, int zonly) {
+__global__ void __launch_bounds__(FIN_THREADS)
+    head_finalize_kernel(const float* __restrict__ partials, const float* __restrict__ gathered,
+                         const int32_t* __restrict__ drafts, int P, int gamma, int V, int slots,
+                         float* scores, int32_t* argmax_out, float* __restrict__ margin,
+                         unsigned* status, AcceptArgs acc, int zonly, unsigned* seq_tickets) {
   // launched as a programmatic dependent of the LM head: wait for its results
   asm volatile("griddepcontrol.wait;" ::: "memory");
-  __shared__ MergeStat red[FIN_MAX_WARPS];
-  __shared__ int s_choice[65];
-  __shared__ int s_kept[65];
-  const int b = blockIdx.x;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
-  const int npos = gamma + 1, per_pass = nw / wpp;
-  const int sub = warp % wpp;
+  __shared__ MergeStat red[FIN_THREADS / 32];
+  __shared__ int s_last;
+  const int p = blockIdx.x;
+  const int npos = gamma + 1, b = p / npos, i = p % npos;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float nan = __int_as_float(0x7fc00000);
-  for (int base = 0; base < npos; base += per_pass) {
-    const int i = base + warp / wpp;
-    const bool active = i < npos;
-    MergeStat st{NEG_INF, 0.f, 0.f, NEG_INF, 0.f, NEG_INF, 0.f, NEG_INF, INT_MAX};
-    if (active) {
-      const int p = b * npos + i;
-      for (int g = sub * 32 + lane; g < slots; g += wpp * 32) {
-        const float* q = partials + (static_cast<long long>(g) * P + p) * HEAD_STAT_FIELDS;
-        const MergeStat o{q[ST_M_O], q[ST_S_O], q[ST_T_O], q[ST_M_R], q[ST_S_R],
-                          q[ST_M_Z], q[ST_S_Z], q[ST_BEST_V], __float_as_int(q[ST_BEST_I])};
-        merge_into(st, o);
-      }
-    }
+  MergeStat st{NEG_INF, 0.f, 0.f, NEG_INF, 0.f, NEG_INF, 0.f, NEG_INF, INT_MAX};
+  for (int g = threadIdx.x; g < slots; g += FIN_THREADS) {
+    // fields 0..3: o and o' (max, sum); 4..7: z (max, sum), best z and its row; 8: entropy term
+    const float4* q =
+        reinterpret_cast<const float4*>(partials + (static_cast<long long>(g) * P + p) * HEAD_STAT_FIELDS);
+    const float4 lo = __ldcg(q), hi = __ldcg(q + 1);
+    const float t = __ldcg(reinterpret_cast<const float*>(q) + ST_T_O);
+    merge_into(st, MergeStat{lo.x, lo.y, t, lo.z, lo.w, hi.x, hi.y, hi.z, __float_as_int(hi.w)});
+  }
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) merge_into(st, shfl_stat(st, o));
-    if (lane == 0) red[warp] = st;
-    __syncthreads();
-    if (active && sub == 0 && lane == 0) {
-      for (int w = 1; w < wpp; ++w) merge_into(st, red[warp + w]);
-      const int p = b * npos + i;
-      // (the pre-blended head has no separate original / reflective logits)
-      const float lse_o = zonly ? nan : st.mo + logf(st.so);
-      const float lse_r = zonly ? nan : st.mr + logf(st.sr);
-      const float lse_z = st.mz + logf(st.sz);
-      const float ent = zonly ? nan : logf(st.so) - st.to / st.so;
-      float* sc = scores + static_cast<long long>(p) * RV_NSCORES;
-      sc[RV_SCORE_ENT_ORIG] = ent;
-      sc[RV_SCORE_LSE_ORIG] = lse_o;
-      sc[RV_SCORE_LSE_REFL] = lse_r;
-      sc[RV_SCORE_LSE_FUSED] = lse_z;
-      int choice = st.bi;
-      float lp_z = nan, lp_o = nan, lp_r = nan;
-      int x = -1;
-      if (i < gamma) {
-        x = drafts[b * gamma + i];
-        if (x >= 0 && x < V) {
-          const float* gx = gathered + static_cast<long long>(p) * GATHER_FIELDS;
-          const float zx = gx[2];
-          lp_z = zx - lse_z;
-          lp_o = zonly ? nan : gx[0] - lse_o;
-          lp_r = zonly ? nan : gx[1] - lse_r;
-          if (zx > st.bv || (zx == st.bv && x < st.bi)) choice = x;
-          margin[b * gamma + i] = fabsf(zx - st.bv);
-        } else {
-          raise_status(status, RV_DEV_DRAFT_RANGE);
-          margin[b * gamma + i] = nan;
-        }
-      }
-      sc[RV_SCORE_LOGP_FUSED] = lp_z;
-      sc[RV_SCORE_LOGP_ORIG] = lp_o;
-      sc[RV_SCORE_LOGP_REFL] = lp_r;
-      argmax_out[p] = choice;
-      s_choice[i] = choice;
-      s_kept[i] = position_kept(acc, x, choice, lp_z, ent) ? 1 : 0;
-    }
-    __syncthreads();
-  }
-  if (acc.accepted_len == nullptr) return;
+  for (int o = 16; o > 0; o >>= 1) merge_into(st, shfl_stat(st, o));
+  if (lane == 0) red[warp] = st;
+  __syncthreads();
   if (threadIdx.x == 0) {
-    int n = gamma;
-    for (int i = 0; i < gamma; ++i) {
-      const bool ok = s_kept[i] != 0;
-      acc.accept_mask[b * gamma + i] = ok ? 1 : 0;
-      if (!ok && n == gamma) n = i;
+    for (int w = 1; w < FIN_THREADS / 32; ++w) merge_into(st, red[w]);
+    // (the pre-blended head has no separate original / reflective logits)
+    const float lse_o = zonly ? nan : st.mo + logf(st.so);
+    const float lse_r = zonly ? nan : st.mr + logf(st.sr);
+    const float lse_z = st.mz + logf(st.sz);
+    const float ent = zonly ? nan : logf(st.so) - st.to / st.so;
+    float* sc = scores + static_cast<long long>(p) * RV_NSCORES;
+    sc[RV_SCORE_ENT_ORIG] = ent;
+    sc[RV_SCORE_LSE_ORIG] = lse_o;
+    sc[RV_SCORE_LSE_REFL] = lse_r;
+    sc[RV_SCORE_LSE_FUSED] = lse_z;
+    int choice = st.bi;
+    float lp_z = nan, lp_o = nan, lp_r = nan;
+    if (i < gamma) {
+      const int x = drafts[b * gamma + i];
+      if (x >= 0 && x < V) {
+        const float* gx = gathered + static_cast<long long>(p) * GATHER_FIELDS;
+        const float zx = gx[2];
+        lp_z = zx - lse_z;
+        lp_o = zonly ? nan : gx[0] - lse_o;
+        lp_r = zonly ? nan : gx[1] - lse_r;
+        if (zx > st.bv || (zx == st.bv && x < st.bi)) choice = x;
+        margin[b * gamma + i] = fabsf(zx - st.bv);
+      } else {
+        raise_status(status, RV_DEV_DRAFT_RANGE);
+        margin[b * gamma + i] = nan;
+      }
     }
-    acc.accepted_len[b] = n;
-    acc.next_token[b] = s_choice[n];
-    acc.ctx_out[b] = acc.ctx_in[b] + n + acc.ctx_extra;
+    sc[RV_SCORE_LOGP_FUSED] = lp_z;
+    sc[RV_SCORE_LOGP_ORIG] = lp_o;
+    sc[RV_SCORE_LOGP_REFL] = lp_r;
+    argmax_out[p] = choice;
+    s_last = 0;
+    if (acc.accepted_len != nullptr) {
+      __threadfence();  // this position's outputs before the ticket
+      s_last = atomicAdd(seq_tickets + b, 1u) == static_cast<unsigned>(npos - 1) ? 1 : 0;
+    }
   }
+  __syncthreads();
+  if (!s_last || threadIdx.x != 0) return;
+  // the sequence's last position: every other position's outputs are visible
+  __threadfence();
+  seq_tickets[b] = 0u;  // re-armed for the next launch
+  int n = gamma;
+  for (int k = 0; k < gamma; ++k) {
+    const int pk = b * npos + k;
+    const int x = drafts[b * gamma + k];
+    const int choice = __ldcg(argmax_out + pk);
+    const float lp = __ldcg(scores + static_cast<long long>(pk) * RV_NSCORES + RV_SCORE_LOGP_FUSED);
+    const float ent = __ldcg(scores + static_cast<long long>(pk) * RV_NSCORES + RV_SCORE_ENT_ORIG);
+    const bool ok = position_kept(acc, x, choice, lp, ent);
+    acc.accept_mask[b * gamma + k] = ok ? 1 : 0;
+    if (!ok && n == gamma) n = k;
+  }
+  acc.accepted_len[b] = n;
+  acc.next_token[b] = __ldcg(argmax_out + b * npos + n);
+  acc.ctx_out[b] = acc.ctx_in[b] + n + acc.ctx_extra;
 }
 
 cudaError_t launch_head_finalize(const HeadArgs& a, const HeadPlan& p, float* scores,
@@ -290,15 +291,10 @@ cudaError_t launch_head_finalize(const HeadArgs& a, const HeadPlan& p, float* sc
                                  cudaStream_t s) {
   AcceptArgs ac = {};
   if (acc) ac = *acc;
-  const int npos = a.gamma + 1;
-  int wpp = 1, warps = FIN_MAX_WARPS;
-  if (npos <= FIN_MAX_WARPS) {
-    wpp = std::max(1, std::min((p.slots + 31) / 32, FIN_MAX_WARPS / npos));
-    warps = npos * wpp;
-  }
+  if (acc && a.seq_tickets == nullptr) return cudaErrorInvalidValue;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(a.B, 1, 1);
-  cfg.blockDim = dim3(warps * 32, 1, 1);
+  cfg.gridDim = dim3(p.P, 1, 1);
+  cfg.blockDim = dim3(FIN_THREADS, 1, 1);
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -306,8 +302,8 @@ cudaError_t launch_head_finalize(const HeadArgs& a, const HeadPlan& p, float* sc
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, head_finalize_kernel, a.partials, a.gathered, a.drafts, p.P,
-                            a.gamma, a.V, p.slots, wpp, scores, argmax, margin, a.status, ac,
-                            p.zonly ? 1 : 0);
+                            a.gamma, a.V, p.slots, scores, argmax, margin, a.status, ac,
+                            p.zonly ? 1 : 0, a.seq_tickets);
 }
 
 // ---------------------------------------------------------------- accept (Alg. 2)

@@ -37,6 +37,7 @@ struct Workspace {
   float* gathered = nullptr;
   void* hsel = nullptr;
   AttnTcScratch attn{};  // tcgen05 attention: partial results, tickets, counters
+  unsigned* fin_tickets = nullptr;  // [max_batch], zero between launches (head finalize)
   // staging for rv_verify_step_host
   void* st_q = nullptr;
   void* st_kb = nullptr;
@@ -315,6 +316,7 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
   const size_t o_apo = take(static_cast<size_t>(a_slots) * 128 * 128 * 4);
   const size_t o_aml = take(static_cast<size_t>(a_slots) * 128 * 2 * 4);
   const size_t o_act = take(64);
+  const size_t o_fin = take(static_cast<size_t>(c.max_batch) * 4);  // finalize tickets
 
   e = cudaMalloc(&h->ws.base, off);
   if (e != cudaSuccess) {
@@ -330,6 +332,7 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
   h->ws.attn.part_o = reinterpret_cast<float*>(b + o_apo);
   h->ws.attn.part_ml = reinterpret_cast<float*>(b + o_aml);
   h->ws.attn.counters = reinterpret_cast<unsigned*>(b + o_act);
+  h->ws.fin_tickets = reinterpret_cast<unsigned*>(b + o_fin);
   h->ws.st_q = b + o_q;
   h->ws.st_kb = b + o_kb;
   h->ws.st_vb = b + o_vb;
@@ -602,7 +605,7 @@ int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_
              h->ws.head_partials, h->ws.gathered, h->ws.status,
              bf16 ? h->ws.status + 16 : nullptr,    // tile counter: its own 64-byte line
              bf16 ? h->ws.status + 32 : nullptr,    // finished-CTA counter
-             writes_z(h) ? h->zbuf : nullptr};
+             writes_z(h) ? h->zbuf : nullptr, h->ws.fin_tickets};
   HeadPlan pl = head_plan(B, gamma, c.vocab, h->num_sms, bf16,
                           bf16 && h->head_mode != RV_HEAD_FUSED_LOGITS,
                           bf16 && h->head_mode == RV_HEAD_STANDARD);

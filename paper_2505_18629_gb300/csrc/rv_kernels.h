@@ -94,6 +94,9 @@ struct HeadArgs {
   unsigned* tile_counter;  // LM-head tile counter, zeroed by the prep kernel
   unsigned* done_counter;  // finished LM-head CTAs (fused merge), zeroed by the prep kernel
   float* zout = nullptr;   // [P][V] fused logits z_i (speculative sampling), or none
+  // [B] per-sequence tickets of the finalize launch's acceptance (zero between
+  // launches; needed when the finalize runs the acceptance)
+  unsigned* seq_tickets = nullptr;
 };
 
 // ---- small kernels (k_small.cu)

@@ -9,14 +9,18 @@
 // chunk); persistent CTAs (at most one per SM) claim items from a counter, so
 // sequences of different lengths balance across the SMs.  An item that covers
 // the whole sequence writes its rows directly; otherwise it writes its
-// normalised partial O with (max, sum), and a second small kernel merges the
-// chunks (one warp per row).
+// normalised partial O (bf16) with (max, sum), and a second small kernel
+// merges the chunks (one thread per row).
 //
 // Per CTA, warp-specialised:
-//   warp 0     claims items and loads with TMA, per tile of 128 keys, the K
-//              and V tiles from the cache ([B*Hkv*Cmax][D]) or, for the
-//              block's keys, from k_blk / v_blk (3-D box over [B*Lb][Hkv][D])
-//              into a ring of stages
+//   warp 0     claims items and loads with TMA the item's 128 query rows
+//              (3-D box over q [B*Lb][Hq][D]) into a shared-memory buffer,
+//              then, per tile of 128 keys, the K and V tiles from the cache
+//              ([B*Hkv*Cmax][D]) or, for the block's keys, from k_blk / v_blk
+//              (3-D box over [B*Lb][Hkv][D]) into a ring of stages.  Items are
+//              claimed full key chunks first and the sequences' last chunks
+//              (shorter, with the block's keys) after them, so that the small
+//              items fill the end of the launch
 //   warp 1     allocates TMEM and issues the MMAs from one thread:
 //                S_t  = Q K_t^T   (M 128, N 128, K 128) into S[t % 2]; Q is
 //                                 read from TMEM
@@ -28,8 +32,9 @@
 //              computes the next scores while the softmax runs; the MMAs of a
 //              CTA execute in issue order, so QK of tile t+2 overwrites S[t % 2]
 //              only after PV of tile t has read P_t
-//   warps 2-5  one thread per query row (its TMEM lane): writes its Q row into
-//              TMEM, runs the online softmax of S_t (base-2, the 1/sqrt(D)
+//   warps 2-5  one thread per query row (its TMEM lane): copies its Q row from
+//              the shared-memory buffer into TMEM (which frees the buffer for
+//              the next item's rows), runs the online softmax of S_t (base-2, the 1/sqrt(D)
 //              scale folded into the exponent), rescales its O row lazily
 //              (only when its max rises by more than 2^8), and at the end of
 //              the item stores the O row (output or partial).  The next item's
@@ -56,9 +61,11 @@ constexpr int TC_IRING = 4;      // item ring between the producer and the consu
 constexpr float TC_RESCALE_LOG2 = 8.f;
 
 constexpr uint32_t TC_KV_BYTES = TC_KT * TC_D * 2;  // 32 KB: two halves of [128 keys][128 B]
+constexpr uint32_t TC_Q_BYTES = TC_M * TC_D * 2;    // 32 KB: two halves of [128 rows][128 B]
 constexpr uint32_t TC_K_OFF = 0;
 constexpr uint32_t TC_V_OFF = TC_K_OFF + TC_STAGES * TC_KV_BYTES;
-constexpr uint32_t TC_BAR_OFF = TC_V_OFF + TC_STAGES * TC_KV_BYTES;
+constexpr uint32_t TC_QS_OFF = TC_V_OFF + TC_STAGES * TC_KV_BYTES;  // staged query rows
+constexpr uint32_t TC_BAR_OFF = TC_QS_OFF + TC_Q_BYTES;
 constexpr uint32_t TC_MISC_OFF = TC_BAR_OFF + 256;
 constexpr uint32_t TC_RING_OFF = TC_MISC_OFF + 16;  // TC_IRING items of 8 ints
 constexpr uint32_t TC_SCAN_OFF = TC_RING_OFF + TC_IRING * 32;
@@ -76,7 +83,9 @@ struct TcArgs {
   const __nv_bfloat16* k_blk;
   const __nv_bfloat16* v_blk;
   __nv_bfloat16* out;
-  float* part_o;       // [slot][128][128] normalised partial O
+  // normalised partial O, chunk-major: [slot][32 chunks of 4 dims][128 rows] x 16 B,
+  // so that a warp's 32 rows store one chunk as 512 contiguous bytes
+  float* part_o;
   float* part_ml;      // [slot][128][2]   (max in log2 units, sum)
   unsigned* counters;  // [0] item counter, [1] CTAs finished
   unsigned* status;
@@ -112,7 +121,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     attention_tc_kernel(const __grid_constant__ CUtensorMap tm_kc,
                         const __grid_constant__ CUtensorMap tm_vc,
                         const __grid_constant__ CUtensorMap tm_kb,
-                        const __grid_constant__ CUtensorMap tm_vb, const TcArgs a) {
+                        const __grid_constant__ CUtensorMap tm_vb,
+                        const __grid_constant__ CUtensorMap tm_q, const TcArgs a) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -131,10 +141,14 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   const uint32_t drain_bar = b2 + 56u;
   auto r_full = [&](int i) { return b2 + 64u + 8u * i; };  // TC_IRING each
   auto r_empty = [&](int i) { return b2 + 64u + 8u * (TC_IRING + i); };
+  const uint32_t qs_full = b2 + 64u + 16u * TC_IRING;  // an item's rows are staged (TMA)
+  const uint32_t qs_empty = qs_full + 8u;              // the softmax warps copied them to TMEM
+  static_assert(32 + 16 * TC_STAGES + 64 + 16 * TC_IRING + 16 <= 256, "barrier block");
   uint32_t* const tmem_slot = reinterpret_cast<uint32_t*>(smem + TC_MISC_OFF);
   volatile int* const abort_flag = reinterpret_cast<volatile int*>(smem + TC_MISC_OFF + 4);
   Item* const ring = reinterpret_cast<Item*>(smem + TC_RING_OFF);
   int* const scan = reinterpret_cast<int*>(smem + TC_SCAN_OFF);  // [B + 1] first item of b
+  int* const order = scan + a.B + 1;  // [B] sequences by the size of their last chunk, largest first
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 4);
@@ -149,6 +163,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     }
     mbar_init(o_free, 4);
     mbar_init(drain_bar, 1);
+    mbar_init(qs_full, 1);
+    mbar_init(qs_empty, 4);
     for (int i = 0; i < TC_IRING; ++i) {
       mbar_init(r_full(i), 1);
       mbar_init(r_empty(i), 5);  // the MMA thread + one lane per softmax warp
@@ -157,12 +173,16 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     fence_barrier_init();
   }
   if (warp == 0) {
-    // items of sequence b: Hkv * n_rg * chunks(b), numbered sequence by sequence
+    // Items: first the full chunks (all chunks but the last) of every sequence,
+    // numbered sequence by sequence (scan[b] = the first of sequence b), then
+    // the last chunk of every (sequence, KV head, row group), the sequences in
+    // decreasing order of that chunk's tiles (ties: lower b first), so that
+    // the smallest items end the launch.
     const int per_seq = a.Hkv * a.n_rg;
     int carry = 0;
     for (int b0 = 0; b0 < a.B; b0 += 32) {
       const int b = b0 + lane;
-      const int n = b < a.B ? per_seq * seq_chunks(a.ctx[b], a.Lb, a.Cmax, a.chunk) : 0;
+      const int n = b < a.B ? per_seq * (seq_chunks(a.ctx[b], a.Lb, a.Cmax, a.chunk) - 1) : 0;
       int incl = n;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
@@ -172,8 +192,25 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       if (b < a.B) scan[b] = carry + incl - n;
       carry += __shfl_sync(0xffffffffu, incl, 31);
     }
+    auto last_tiles = [&](int b) {
+      const int ctx = a.ctx[b];
+      if (ctx < 0 || ctx + a.Lb > a.Cmax) return 0;
+      const int nch = seq_chunks(ctx, a.Lb, a.Cmax, a.chunk);
+      const int kc = ctx - min(ctx, (nch - 1) * a.chunk);
+      return (kc + TC_KT - 1) / TC_KT + (a.Lb + TC_KT - 1) / TC_KT;
+    };
+    for (int b = lane; b < a.B; b += 32) {
+      const int tb = last_tiles(b);
+      int rank = 0;
+      for (int o = 0; o < a.B; ++o) {
+        const int to = last_tiles(o);
+        rank += (to > tb || (to == tb && o < b)) ? 1 : 0;
+      }
+      order[rank] = b;
+    }
     if (lane == 0) {
       scan[a.B] = carry;
+      tma_prefetch_desc(&tm_q);
       tma_prefetch_desc(&tm_kc);
       tma_prefetch_desc(&tm_vc);
       tma_prefetch_desc(&tm_kb);
@@ -193,8 +230,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     if (lane == 0) {
       const uint64_t pol_blk = policy_evict_last();
       const uint64_t pol_kv = a.kv_evict_first ? policy_evict_first() : policy_evict_normal();
-      const int total = scan[a.B];
-      int u = 0;
+      const int per_seq = a.Hkv * a.n_rg;
+      const int n_full = scan[a.B];
+      const int total = n_full + a.B * per_seq;
+      int u = 0, nq = 0;
       bool ok = true;
       for (int lt = 0; ok; ++lt) {
         const int i = static_cast<int>(atomicAdd(&a.counters[0], 1u));
@@ -203,23 +242,35 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         item.kvh = item.rg = item.c = item.ctx = item.kc_lo = item.kc_hi = 0;
         item.nch = 1;
         if (i < total) {
-          int lo = 0, hi = a.B - 1;  // the last b with scan[b] <= i
-          while (lo < hi) {
-            const int mid = (lo + hi + 1) >> 1;
-            if (scan[mid] <= i)
-              lo = mid;
-            else
-              hi = mid - 1;
+          int b, rem, c_last = 0;
+          if (i < n_full) {
+            int lo = 0, hi = a.B - 1;  // the last b with scan[b] <= i
+            while (lo < hi) {
+              const int mid = (lo + hi + 1) >> 1;
+              if (scan[mid] <= i)
+                lo = mid;
+              else
+                hi = mid - 1;
+            }
+            b = lo;
+            rem = i - scan[b];
+          } else {
+            b = order[(i - n_full) / per_seq];
+            rem = (i - n_full) % per_seq;
+            c_last = 1;
           }
-          const int b = lo;
           const int ctx = a.ctx[b];
           const int nch = seq_chunks(ctx, a.Lb, a.Cmax, a.chunk);
-          int rem = i - scan[b];
           item.b = b;
           item.rg = rem % a.n_rg;
           rem /= a.n_rg;
-          item.c = rem % nch;
-          item.kvh = rem / nch;
+          if (c_last) {
+            item.c = nch - 1;
+            item.kvh = rem;
+          } else {
+            item.c = rem % (nch - 1);
+            item.kvh = rem / (nch - 1);
+          }
           item.nch = nch;
           const bool valid = ctx >= 0 && ctx + a.Lb <= a.Cmax;
           item.ctx = valid ? ctx : -1;
@@ -237,6 +288,19 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         if (item.b < 0) break;
         const int n = item_tiles(item, a.Lb);
         if (n == 0) continue;
+        // the item's query rows: (j, g) for j from rg * 128 / G, one box per 64 dims
+        if (!mbar_wait(qs_empty, (nq & 1) ^ 1u, abort_flag, a.status)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(qs_full, TC_Q_BYTES);
+        {
+          const int z = item.b * a.Lb + item.rg * (TC_M / a.G);
+          tma_load_3d(base + TC_QS_OFF, &tm_q, 0, item.kvh * a.G, z, qs_full, pol_blk);
+          tma_load_3d(base + TC_QS_OFF + TC_Q_BYTES / 2, &tm_q, 64, item.kvh * a.G, z, qs_full,
+                      pol_blk);
+        }
+        ++nq;
         const int n_cache = item_cache_tiles(item);
         const int row_c = (item.b * a.Hkv + item.kvh) * a.Cmax;
         for (int j = 0; j < n; ++j) {
@@ -267,6 +331,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       if (!ok) {  // let the copies still in flight land before the CTA exits
         for (int v = max(0, u - TC_STAGES); v < u; ++v)
           drain_wait(kv_full(v % TC_STAGES), static_cast<uint32_t>((v / TC_STAGES) & 1));
+        if (nq > 0) drain_wait(qs_full, static_cast<uint32_t>((nq - 1) & 1));
       }
     }
     __syncwarp();
@@ -350,19 +415,24 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         if (it.b < 0 || item_tiles(it, a.Lb) > 0) return true;
       }
     };
-    // this row of the item's Q: global -> registers (issued early) -> TMEM
+    // this row of the item's Q: the staged rows (TMA, 128-byte swizzle: chunk c
+    // of row r at c ^ (r & 7)) -> registers -> TMEM; the buffer is released as
+    // soon as every row has been read.  Rows past the item's (another
+    // sequence's, or zeros) are read too; their scores are masked.
     uint4 qv[16];
-    auto q_fetch = [&](const Item& it) {
-      const int gr = it.rg * TC_M + r;
-      if (gr < a.rows) {
-        const uint4* src = reinterpret_cast<const uint4*>(
-            a.q + ((static_cast<long long>(it.b) * a.Lb + gr / a.G) * a.Hq + it.kvh * a.G + gr % a.G) * TC_D);
+    int nq = 0;
+    auto q_fetch = [&](const Item& it) -> bool {
+      (void)it;
+      const bool w = mbar_wait(qs_full, nq & 1, abort_flag, a.status);
+      if (!__all_sync(0xffffffffu, w)) return false;
+      ++nq;
 #pragma unroll
-        for (int c = 0; c < 16; ++c) qv[c] = __ldg(src + c);
-      } else {
-#pragma unroll
-        for (int c = 0; c < 16; ++c) qv[c] = make_uint4(0u, 0u, 0u, 0u);
-      }
+      for (int c = 0; c < 16; ++c)
+        qv[c] = *reinterpret_cast<const uint4*>(smem + TC_QS_OFF + (c >> 3) * (TC_Q_BYTES / 2) +
+                                                r * 128 + (((c & 7) ^ (r & 7)) << 4));
+      __syncwarp();
+      if (lane == 0) mbar_arrive(qs_empty);
+      return true;
     };
     auto q_store = [&]() {
 #pragma unroll
@@ -386,8 +456,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     Item item;
     live = next_item(item);
     if (live && item.b >= 0) {
-      q_fetch(item);
-      q_store();
+      live = q_fetch(item);
+      if (live) q_store();
     }
     int u = 0;
     while (live && item.b >= 0) {
@@ -505,7 +575,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       live = next_item(nxt);
       if (!live) break;
       if (nxt.b >= 0) {
-        q_fetch(nxt);
+        live = q_fetch(nxt);
+        if (!live) break;
         q_store();
       }
 
@@ -542,14 +613,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
               *reinterpret_cast<uint4*>(dst + 32 * c + i) = pk;
             }
         } else {
-          float* const po = a.part_o + (static_cast<long long>(slot) * TC_M + r) * TC_D;
+          float4* const po =
+              reinterpret_cast<float4*>(a.part_o) + static_cast<long long>(slot) * 32 * TC_M + r;
 #pragma unroll
-          for (int c = 0; c < 4; ++c)
-#pragma unroll
-            for (int i = 0; i < 32; i += 4)
-              __stcg(reinterpret_cast<float4*>(po + 32 * c + i),
-                     make_float4(ov[c][i] * inv, ov[c][i + 1] * inv, ov[c][i + 2] * inv,
-                                 ov[c][i + 3] * inv));
+          for (int c = 0; c < 32; ++c) {
+            const float* v = &ov[c >> 3][(c & 7) * 4];
+            __stcg(po + c * TC_M, make_float4(v[0] * inv, v[1] * inv, v[2] * inv, v[3] * inv));
+          }
           __stcg(reinterpret_cast<float2*>(a.part_ml) + static_cast<long long>(slot) * TC_M + r,
                  make_float2(m_used, l));
         }
@@ -576,7 +646,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
 }
 
 // Merge of the chunks of each (sequence, KV head, row group) whose sequence
-// needed several: one warp per query row, lane i holding dims 4i..4i+3.
+// needed several: one CTA per (group, 8 dims), one thread per query row, so
+// that the CTA's threads read consecutive rows of the chunk-major partials.
 // out = sum_c w_c O_c / sum_c w_c with w_c = l_c 2^(m_c - max_c m_c).
 struct MergeArgs {
   const int32_t* ctx;
@@ -586,15 +657,14 @@ struct MergeArgs {
   int Lb, Hq, Hkv, G, Cmax, rows, n_rg, chunk, max_chunks;
 };
 
-__global__ void __launch_bounds__(256) attention_merge_kernel(const MergeArgs a) {
+__global__ void __launch_bounds__(TC_M) attention_merge_kernel(const MergeArgs a) {
   asm volatile("griddepcontrol.wait;" ::: "memory");  // the attention grid's results
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int group = blockIdx.x;
   const int rg = group % a.n_rg, t = group / a.n_rg;
   const int kvh = t % a.Hkv, b = t / a.Hkv;
-  const int rr = blockIdx.y * 8 + warp;  // row within the row group
+  const int rr = threadIdx.x;  // row within the row group
   const int gr = rg * TC_M + rr;
-  if (rr >= TC_M || gr >= a.rows) return;
+  if (gr >= a.rows) return;
   const int ctx = a.ctx[b];
   if (ctx < 0 || ctx + a.Lb > a.Cmax) return;
   const int nch = seq_chunks(ctx, a.Lb, a.Cmax, a.chunk);
@@ -602,32 +672,43 @@ __global__ void __launch_bounds__(256) attention_merge_kernel(const MergeArgs a)
   const long long slot0 = static_cast<long long>(group) * a.max_chunks;
   const float2* ml = reinterpret_cast<const float2*>(a.part_ml);
   float M = NEG_INF;
-  for (int c = lane; c < nch; c += 32) {
+  for (int c = 0; c < nch; ++c) {
     const float2 v = __ldcg(ml + (slot0 + c) * TC_M + rr);
     if (v.y > 0.f) M = fmaxf(M, v.x);
   }
-  M = warp_max(M);
-  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
   float den = 0.f;
-#pragma unroll 4
   for (int c = 0; c < nch; ++c) {
     const float2 v = __ldcg(ml + (slot0 + c) * TC_M + rr);
-    const float4 o =
-        __ldcg(reinterpret_cast<const float4*>(a.part_o + ((slot0 + c) * TC_M + rr) * TC_D) + lane);
-    const float w = v.y > 0.f ? v.y * exp2f(v.x - M) : 0.f;
-    acc.x = fmaf(w, o.x, acc.x);
-    acc.y = fmaf(w, o.y, acc.y);
-    acc.z = fmaf(w, o.z, acc.z);
-    acc.w = fmaf(w, o.w, acc.w);
-    den += w;
+    den += v.y > 0.f ? v.y * exp2f(v.x - M) : 0.f;
   }
   const float id = den > 0.f ? 1.f / den : 0.f;
   const long long orow =
       (static_cast<long long>(b) * a.Lb + gr / a.G) * a.Hq + kvh * a.G + gr % a.G;
-  uint2 pk;
-  pk.x = pack_bf16(acc.x * id, acc.y * id);
-  pk.y = pack_bf16(acc.z * id, acc.w * id);
-  *reinterpret_cast<uint2*>(a.out + orow * TC_D + lane * 4) = pk;
+  const float4* part = reinterpret_cast<const float4*>(a.part_o);
+  {
+    const int ch = blockIdx.y;  // 8 dims: chunks 2 ch and 2 ch + 1
+    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    for (int c = 0; c < nch; ++c) {
+      const float2 v = __ldcg(ml + (slot0 + c) * TC_M + rr);
+      const float w = v.y > 0.f ? v.y * exp2f(v.x - M) * id : 0.f;
+      const float4 lo = __ldcg(part + ((slot0 + c) * 32 + 2 * ch) * TC_M + rr);
+      const float4 hi = __ldcg(part + ((slot0 + c) * 32 + 2 * ch + 1) * TC_M + rr);
+      acc[0] = fmaf(w, lo.x, acc[0]);
+      acc[1] = fmaf(w, lo.y, acc[1]);
+      acc[2] = fmaf(w, lo.z, acc[2]);
+      acc[3] = fmaf(w, lo.w, acc[3]);
+      acc[4] = fmaf(w, hi.x, acc[4]);
+      acc[5] = fmaf(w, hi.y, acc[5]);
+      acc[6] = fmaf(w, hi.z, acc[6]);
+      acc[7] = fmaf(w, hi.w, acc[7]);
+    }
+    uint4 o;
+    o.x = pack_bf16(acc[0], acc[1]);
+    o.y = pack_bf16(acc[2], acc[3]);
+    o.z = pack_bf16(acc[4], acc[5]);
+    o.w = pack_bf16(acc[6], acc[7]);
+    *reinterpret_cast<uint4*>(a.out + orow * TC_D + ch * 8) = o;
+  }
 }
 
 // ---------------------------------------------------------------- planning / launch
@@ -646,7 +727,8 @@ AttnTcPlan attn_tc_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms) {
   p.max_chunks = std::max(1, (Cmax + p.chunk - 1) / p.chunk);
   p.slots = static_cast<int>(groups) * p.max_chunks;
   p.grid = static_cast<int>(std::min<long long>(num_sms, p.slots));
-  p.smem_bytes = TC_SCAN_OFF + static_cast<size_t>(B + 1) * 4 + 1024;
+  // scan [B + 1], order [B] (+ 1024 for alignment)
+  p.smem_bytes = TC_SCAN_OFF + static_cast<size_t>(2 * B + 1) * 4 + 1024;
   return p;
 }
 
@@ -655,7 +737,7 @@ bool attn_tc_supported(int Hq, int Hkv, int D) {
 }
 
 size_t attn_tc_smem_max(int max_batch) {
-  return TC_SCAN_OFF + static_cast<size_t>(max_batch + 1) * 4 + 1024;
+  return TC_SCAN_OFF + static_cast<size_t>(2 * max_batch + 1) * 4 + 1024;
 }
 
 int attn_tc_max_slots(int max_batch, int Lb_max, int Hq, int Hkv, int num_sms) {
@@ -689,6 +771,14 @@ bool encode(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap* m, const void* p
 // boxes of 64 dims x 128 keys, 128-byte swizzled.
 bool attn_tc_encode(PFN_cuTensorMapEncodeTiled_v12000 enc, const AttnArgs& x, AttnTcMaps* m) {
   const cuuint64_t rs = static_cast<cuuint64_t>(TC_D) * 2;
+  {  // q [B*Lb][Hq][D]: boxes of 64 dims x G heads x 128/G block positions
+    const int G = x.Hq / x.Hkv;
+    const cuuint64_t dims[3] = {TC_D, static_cast<cuuint64_t>(x.Hq),
+                                static_cast<cuuint64_t>(x.B) * x.Lb};
+    const cuuint64_t str[2] = {rs, rs * x.Hq};
+    const cuuint32_t box[3] = {64, static_cast<cuuint32_t>(G), static_cast<cuuint32_t>(TC_M / G)};
+    if (!encode(enc, &m->q, x.q, 3, dims, str, box)) return false;
+  }
   {
     const cuuint64_t dims[3] = {TC_D, static_cast<cuuint64_t>(x.Hkv),
                                 static_cast<cuuint64_t>(x.B) * x.Lb};
@@ -733,7 +823,7 @@ cudaError_t launch_attention_tc(const AttnArgs& x, const AttnTcPlan& p, const At
   a.max_chunks = p.max_chunks;
   a.scale_log2 = LOG2E / sqrtf(static_cast<float>(x.D));
   a.kv_evict_first = p.n_rg == 1;  // with several row groups each K/V tile is read again
-  attention_tc_kernel<<<p.grid, TC_THREADS, p.smem_bytes, s>>>(m.kc, m.vc, m.kb, m.vb, a);
+  attention_tc_kernel<<<p.grid, TC_THREADS, p.smem_bytes, s>>>(m.kc, m.vc, m.kb, m.vb, m.q, a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || p.max_chunks == 1) return e;
 
@@ -752,8 +842,8 @@ cudaError_t launch_attention_tc(const AttnArgs& x, const AttnTcPlan& p, const At
   g.chunk = p.chunk;
   g.max_chunks = p.max_chunks;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(x.B * x.Hkv * p.n_rg, (std::min(p.rows, TC_M) + 7) / 8, 1);
-  cfg.blockDim = dim3(256, 1, 1);
+  cfg.gridDim = dim3(x.B * x.Hkv * p.n_rg, TC_D / 8, 1);
+  cfg.blockDim = dim3(TC_M, 1, 1);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];

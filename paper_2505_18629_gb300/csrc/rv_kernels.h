@@ -245,6 +245,7 @@ struct AttnTcPlan {
 struct AttnTcMaps {
   CUtensorMap kc, vc;  // [B*Hkv*Cmax][D], box {64, 128}
   CUtensorMap kb, vb;  // [B*Lb][Hkv][D], box {64, 1, 128}
+  CUtensorMap q;       // [B*Lb][Hq][D], box {64, G, 128 / G}
 };
 struct AttnTcScratch {
   float* part_o;       // [slots][128][128]

@@ -1033,7 +1033,11 @@ def test_standard_verification_host_buffers(gu):
     _standard_run(gu, _wl(B=4, gamma=5, seed=123), host=True)
 
 
-@pytest.mark.parametrize("name,seqs", [("llama3-8b-b16", None), ("sweep-b64-g8-c8192", [0, 33, 63])])
+# 8B B=16: CTA-pair z-only head (144 pairs); sweep-b16-g4: one-CTA z-only head
+# with its merge in a separate launch (80 pairs); sweep-b64-g8: three chunks of
+# 192 pairs on CTA pairs.
+@pytest.mark.parametrize("name,seqs", [("llama3-8b-b16", None), ("sweep-b16-g4-c1024", [0, 7, 15]),
+                                       ("sweep-b64-g8-c8192", [0, 33, 63])])
 def test_standard_verification_8b(gu, name, seqs):
     from paper_2505_18629_gb300 import synth
     _standard_run(gu, synth.workload(name), seqs=seqs)

@@ -5,8 +5,8 @@ Its results must match the oracle's verify_head and rv_verify_head's on the
 same inputs, within the tolerances of the parity tests, on two calls in a row
 (the second call must not see the first call's leftovers in the shared
 scratch), with and without a caller-supplied status word, and at the 8B shape
-(H = 4096, V = 128256, B = 1, gamma = 5, template 8), which is within its
-limits.  This file is collected last on purpose.
+(H = 4096, V = 128256, B = 1, gamma = 5, template 8), and at its limits
+(64 pairs, H = 8192) without allocating.  This file is collected last on purpose.
 """
 import numpy as np
 import pytest
@@ -123,6 +123,37 @@ def test_static_head_at_the_8b_shape(env):
         assert int(status.item()) == 0
         _check_against_oracle_and_handle(gu, rv, wl, inp, drafts, got, ref)
     h.close()
+
+
+def test_static_head_at_its_limits_allocates_nothing(env):
+    """64 pairs (B = 8, gamma = 7) at H = RV_STATIC_MAX_HIDDEN: the largest call
+    it accepts.  After a first call (which may load the library's module), two
+    more calls leave the device's free memory and the caching allocator's
+    allocation count unchanged."""
+    import torch
+    gu, rv, synth = env
+    B, gamma = 8, rv.RV_STATIC_MAX_PAIRS // 8 - 1
+    wl, inp, drafts = _inputs(gu, synth, 64, B=B, gamma=gamma, R=4, V=1200,
+                              H=rv.RV_STATIC_MAX_HIDDEN)
+    assert B * (gamma + 1) == rv.RV_STATIC_MAX_PAIRS
+    hid, W = gu.to_dev(inp.hidden), gu.to_dev(inp.W)
+    d = gu.to_dev(drafts.astype(np.int32))
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    outs = [_outputs(torch, B, gamma, rv) for _ in range(3)]
+    rv.rv_verify_head_static(hid, W, d, gamma, wl.R, ALPHA, *outs[0], dev_status=status)
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    n0 = torch.cuda.memory_stats().get("allocation.all.allocated", 0)
+    for got in outs[1:]:
+        rv.rv_verify_head_static(hid, W, d, gamma, wl.R, ALPHA, *got, dev_status=status)
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] == free0
+    assert torch.cuda.memory_stats().get("allocation.all.allocated", 0) == n0
+    assert int(status.item()) == 0
+    head = orc.verify_head(inp.W, inp.hidden, drafts, wl.gamma, wl.R, ALPHA)
+    for got in outs:
+        sg, am_g, mg_g = (gu.to_np(t) for t in got)
+        gu.compare_head(head, sg, am_g, mg_g, wl.gamma)
 
 
 def test_static_head_rejects_sizes_beyond_its_scratch(env):

@@ -486,12 +486,22 @@ def run_variant(args):
     st = rv.rv_read_status(h, stream)
     if st:
         raise RuntimeError(f"device status 0x{st:x}")
+    exact_us = None
+    if args.accept != "exact" and not args.pending:
+        # the same step with the exact-match rule, same handle and inputs
+        rv.rv_set_acceptance(h, rv.RV_ACCEPT_EXACT)
+        args_accept = args.accept
+        args.accept = "exact"
+        exact_us = _time_steps(step, args.steps, max(args.warmup, 3), stream)
+        args.accept = args_accept
     units = B * (Lb + lead)
     print(json.dumps({
         "metric": METRIC, "value": units / (us * 1e-6), "unit": UNIT, "n_gpus": 1,
         "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": us * 1e-3,
         "higher_is_better": True, "dtype": "bf16" if wl.dtype == "bf16" else "f32",
         "data": "synthetic", "step_us": us, "accept_launches_us": accept_us,
+        "exact_step_us": exact_us,
+        "vs_exact": us / exact_us if exact_us else None,
         "mean_accepted": float(alen.float().mean().item()),
         "config": dict(_config(wl, 1, args.head_mode), accept=args.accept, pending=args.pending),
         "clocks": clk}), flush=True)

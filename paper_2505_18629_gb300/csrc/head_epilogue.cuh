@@ -158,6 +158,14 @@ __device__ __forceinline__ void head_tile_pairs8(const float (&o)[8], const floa
 // c % 8; o, r or z for c / 8) over the 32 rows with plain loads - no shuffle
 // trees - then folds the result into the warp's running statistics.  Same
 // results as the shuffle version up to the order of the sums.
+// sum over the 32 staged rows of exp((x - m) / T); rows at -inf add 0.
+__device__ __forceinline__ float subtile_sum_t(const float (&val)[32], float m, float inv_t) {
+  float s2[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int i = 0; i < 32; ++i) s2[i & 3] += __expf((val[i] - m) * inv_t);
+  return (s2[0] + s2[1]) + (s2[2] + s2[3]);
+}
+
 constexpr int HEAD_SCR_STRIDE = 24;  // floats per staged row (16-byte aligned rows)
 constexpr int HEAD_SCR_FLOATS = 32 * HEAD_SCR_STRIDE;
 
@@ -165,7 +173,9 @@ __device__ __forceinline__ void head_tile_pairs8_t(const float (&o)[8], const fl
                                                    int npairs, int v, bool valid, float alpha,
                                                    const int* s_drafts, float* warp_stats,
                                                    float* gathered, float* scr, int lane,
-                                                   float* zout = nullptr, int V = 0) {
+                                                   float* zout = nullptr, int V = 0,
+                                                   float2* zsub = nullptr, int n_sub = 0,
+                                                   float inv_t = 1.f) {
   const float beta = 1.f - alpha;
   float zr[8];
 #pragma unroll
@@ -225,9 +235,12 @@ __device__ __forceinline__ void head_tile_pairs8_t(const float (&o)[8], const fl
         lse_merge(st[ST_M_R], st[ST_S_R], m, sum);
       } else {
         lse_merge(st[ST_M_Z], st[ST_S_Z], m, sum);
+        const int v0 = v - lane;  // vocab row of staged row 0
+        if (zsub != nullptr && m != NEG_INF)  // sampled exact match: this subtile's sums at T
+          zsub[static_cast<long long>(pj) * n_sub + (v0 >> 5)] =
+              make_float2(m, inv_t == 1.f ? sum : subtile_sum_t(val, m, inv_t));
         // best z over the rows v != x_i (lowest row on ties)
         const int x = s_drafts[pj];
-        const int v0 = v - lane;  // vocab row of staged row 0
         float bv = NEG_INF;
         int bi = INT_MAX;
 #pragma unroll
@@ -255,7 +268,9 @@ __device__ __forceinline__ void head_tile_pairs8_t(const float (&o)[8], const fl
 __device__ __forceinline__ void head_tile_z8_t(const float (&z)[8], int g8, int npairs, int v,
                                                bool valid, const int* s_drafts, float* warp_stats,
                                                float* gathered, float* scr, int lane,
-                                               float* zout = nullptr, int V = 0) {
+                                               float* zout = nullptr, int V = 0,
+                                               float2* zsub = nullptr, int n_sub = 0,
+                                               float inv_t = 1.f) {
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
     const int pj = g8 + j;
@@ -289,6 +304,9 @@ __device__ __forceinline__ void head_tile_z8_t(const float (&z)[8], int g8, int 
       lse_merge(st[ST_M_Z], st[ST_S_Z], m, sum);
       const int x = s_drafts[pj];
       const int v0 = v - lane;  // vocab row of staged row 0
+      if (zsub != nullptr && m != NEG_INF)  // sampled exact match: this subtile's sums at T
+        zsub[static_cast<long long>(pj) * n_sub + (v0 >> 5)] =
+            make_float2(m, inv_t == 1.f ? sum : subtile_sum_t(val, m, inv_t));
       float bv = NEG_INF;
       int bi = INT_MAX;
 #pragma unroll

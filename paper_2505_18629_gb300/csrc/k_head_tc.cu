@@ -65,6 +65,9 @@ struct HeadTcParams {
   float* partials;
   float* gathered;
   float* zout;  // [P][V] fused logits, or null
+  float2* zsub;  // [P][n_sub] subtile (max z, sum exp((z - max) / T)), or null
+  int n_sub;
+  float inv_t;
   unsigned* status;
   int zonly;    // pre-blended head: column j of the accumulator is z of pair j
 };
@@ -317,13 +320,14 @@ __global__ void __launch_bounds__(ht_threads(EPI), 1)
       const uint32_t trow =
           tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(slot * p.N);
       float* const zout = p.zout ? p.zout + static_cast<long long>(pair0) * p.V : nullptr;
+      float2* const zsub = p.zsub ? p.zsub + static_cast<long long>(pair0) * p.n_sub : nullptr;
       for (int g8 = 8 * half; g8 < npairs; g8 += 8 * (EPI / 4)) {
         if (p.zonly) {
           float z[8];
           tmem_ld8(trow + g8, z);
           tmem_ld_wait();
           head_tile_z8_t(z, g8, npairs, v, valid, s_drafts, wstats, gathered,
-                         scr_base + ew * HEAD_SCR_FLOATS, lane, zout, p.V);
+                         scr_base + ew * HEAD_SCR_FLOATS, lane, zout, p.V, zsub, p.n_sub, p.inv_t);
           continue;
         }
         float o[8], r[8];
@@ -331,7 +335,8 @@ __global__ void __launch_bounds__(ht_threads(EPI), 1)
         tmem_ld8(trow + p.Pcp + g8, r);
         tmem_ld_wait();
         head_tile_pairs8_t(o, r, g8, npairs, v, valid, p.alpha, s_drafts, wstats, gathered,
-                           scr_base + ew * HEAD_SCR_FLOATS, lane, zout, p.V);
+                           scr_base + ew * HEAD_SCR_FLOATS, lane, zout, p.V, zsub, p.n_sub,
+                           p.inv_t);
       }
       tc_fence_before();
       __syncwarp();
@@ -417,6 +422,9 @@ cudaError_t launch_head_tc(const HeadArgs& a, const HeadPlan& pl, const HeadTcLa
   p.partials = a.partials;
   p.gathered = a.gathered;
   p.zout = a.zout;
+  p.zsub = a.zsub;
+  p.n_sub = (a.V + 31) / 32;
+  p.inv_t = a.inv_t;
   p.status = a.status;
   p.zonly = pl.zonly ? 1 : 0;
   cudaLaunchConfig_t cfg = {};

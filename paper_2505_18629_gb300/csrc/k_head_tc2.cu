@@ -88,6 +88,9 @@ struct Head2Params {
   float* partials;
   float* gathered;
   float* zout;  // [P][V] fused logits, or null
+  float2* zsub;  // [P][n_sub] subtile (max z, sum exp((z - max) / T)), or null
+  int n_sub;
+  float inv_t;
   unsigned* status;
   int zonly;    // pre-blended head: column j of the accumulator is z of pair j
 };
@@ -198,6 +201,17 @@ struct TileOut {
   float m, s, t;
 };
 
+// Where a group's fused logits go besides the statistics (sampling modes; the
+// pointers are offset to the chunk's first pair, null when unused): every z
+// (speculative sampling), or one (max z, sum exp((z - max) / T)) per pair and
+// 32-row subtile (sampled exact match).
+struct ZSink {
+  float* z;
+  float2* sub;
+  int n_sub;
+  float inv_t;
+};
+
 // Stores at the draft row of each of the lane's columns: `x[j]` (this lane's
 // pair of column j) may fall on one of its rows rq + 8i; at most one (unique
 // writer over the CTA).  Rows at or beyond V (a partial last tile) hold zeros;
@@ -232,10 +246,11 @@ __device__ __forceinline__ void gather_draft_rows(const float* o, const float* r
 // at the draft row of each pair and, when asked, z itself; returns this
 // lane's tile statistics: quantity lane / 8 (o, o', z, best z over v != x_i)
 // of column 2(lane%4) + ((lane/4)&1).
+template <bool SUB>
 __device__ __forceinline__ TileOut group8_fused(const uint32_t* lo, const uint32_t* lr,
                                                 int v_row0, int V, float alpha, float beta,
                                                 const int (&x)[2], int gpair, int npairs,
-                                                float* gathered, float* zout, int lane) {
+                                                float* gathered, const ZSink& zs, int lane) {
   const int c4 = lane & 3, rq = lane >> 2;
   const int row0 = v_row0 + rq;  // this lane's first row; the others are +8, +16, +24
   float o[8], r[8], z[8];
@@ -263,14 +278,14 @@ __device__ __forceinline__ TileOut group8_fused(const uint32_t* lo, const uint32
     const int col_pair[2] = {2 * c4, 2 * c4 + 1};
     gather_draft_rows<2>(o, r, z, x, row0, gathered, gpair, col_pair);
   }
-  if (zout != nullptr) {  // sampling modes only (uniform)
+  if (zs.z != nullptr) {  // speculative sampling only (uniform)
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       const int v = row0 + 8 * i;
 #pragma unroll
       for (int j = 0; j < 2; ++j) {
         const int pj = gpair + 2 * c4 + j;
-        if (v < V && pj < npairs) zout[static_cast<long long>(pj) * V + v] = z[2 * i + j];
+        if (v < V && pj < npairs) zs.z[static_cast<long long>(pj) * V + v] = z[2 * i + j];
       }
     }
   }
@@ -329,6 +344,31 @@ __device__ __forceinline__ TileOut group8_fused(const uint32_t* lo, const uint32
       shfl_best(bv[j], bi[j], off);
     }
   }
+  if (SUB && v_row0 < V) {  // sampled exact match only (uniform)
+    float sT[2] = {sz[0], sz[1]};         // T = 1: the sums above
+    if (zs.inv_t != 1.f) {
+      const float k2 = LOG2E * zs.inv_t;
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        sT[j] = 0.f;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) sT[j] += ex2_approx((z[2 * i + j] - mz[j]) * k2);
+      }
+#pragma unroll
+      for (int off = 4; off < 32; off <<= 1) {
+#pragma unroll
+        for (int j = 0; j < 2; ++j) sT[j] += __shfl_xor_sync(0xffffffffu, sT[j], off);
+      }
+    }
+    if (rq == 0) {
+#pragma unroll
+      for (int j = 0; j < 2; ++j) {
+        const int pj = gpair + 2 * c4 + j;
+        if (pj < npairs)
+          zs.sub[static_cast<long long>(pj) * zs.n_sub + (v_row0 >> 5)] = make_float2(mz[j], sT[j]);
+      }
+    }
+  }
   const int qn = rq >> 1;
   const bool j1 = (rq & 1) != 0;
   const float M_o = j1 ? mo[1] : mo[0], M_r = j1 ? mr[1] : mr[0], M_z = j1 ? mz[1] : mz[0];
@@ -347,9 +387,10 @@ __device__ __forceinline__ TileOut group8_fused(const uint32_t* lo, const uint32
 // rows l/4 + 8i and columns 2(l%4) + (jj & 1) + 8 (jj >> 1), jj = 0..3, with
 // drafts x[jj].  Returns quantity l/16 (z statistics, best z over v != x_i)
 // of column jj = (l/4) & 3.
+template <bool SUB>
 __device__ __forceinline__ TileOut group16_z(const uint32_t* la, const uint32_t* lb, int v_row0,
                                              int V, const int (&x)[4], int gpair, int npairs,
-                                             float* gathered, float* zout, int lane) {
+                                             float* gathered, const ZSink& zs, int lane) {
   const int c4 = lane & 3, rq = lane >> 2;
   const int row0 = v_row0 + rq;
   float z[16];  // element 4i + jj
@@ -373,14 +414,14 @@ __device__ __forceinline__ TileOut group16_z(const uint32_t* la, const uint32_t*
     const int col_pair[4] = {2 * c4, 2 * c4 + 1, 8 + 2 * c4, 9 + 2 * c4};
     gather_draft_rows<4>(nullptr, nullptr, z, x, row0, gathered, gpair, col_pair);
   }
-  if (zout != nullptr) {
+  if (zs.z != nullptr) {
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       const int v = row0 + 8 * i;
 #pragma unroll
       for (int jj = 0; jj < 4; ++jj) {
         const int pj = gpair + 2 * c4 + (jj & 1) + 8 * (jj >> 1);
-        if (v < V && pj < npairs) zout[static_cast<long long>(pj) * V + v] = z[4 * i + jj];
+        if (v < V && pj < npairs) zs.z[static_cast<long long>(pj) * V + v] = z[4 * i + jj];
       }
     }
   }
@@ -416,6 +457,32 @@ __device__ __forceinline__ TileOut group16_z(const uint32_t* la, const uint32_t*
     for (int jj = 0; jj < 4; ++jj) {
       sz[jj] += __shfl_xor_sync(0xffffffffu, sz[jj], off);
       shfl_best(bv[jj], bi[jj], off);
+    }
+  }
+  if (SUB && v_row0 < V) {  // sampled exact match only (uniform)
+    float sT[4] = {sz[0], sz[1], sz[2], sz[3]};
+    if (zs.inv_t != 1.f) {
+      const float k2 = LOG2E * zs.inv_t;
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj) {
+        sT[jj] = 0.f;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) sT[jj] += ex2_approx((z[4 * i + jj] - mz[jj]) * k2);
+      }
+#pragma unroll
+      for (int off = 4; off < 32; off <<= 1) {
+#pragma unroll
+        for (int jj = 0; jj < 4; ++jj) sT[jj] += __shfl_xor_sync(0xffffffffu, sT[jj], off);
+      }
+    }
+    if (rq == 0) {
+#pragma unroll
+      for (int jj = 0; jj < 4; ++jj) {
+        const int pj = gpair + 2 * c4 + (jj & 1) + 8 * (jj >> 1);
+        if (pj < npairs)
+          zs.sub[static_cast<long long>(pj) * zs.n_sub + (v_row0 >> 5)] =
+              make_float2(mz[jj], sT[jj]);
+      }
     }
   }
   const int sel = rq & 3, qn = rq >> 2;
@@ -479,7 +546,9 @@ struct LaneStats {
   }
 };
 
-template <bool ZONLY>
+// SUB: the epilogue also stores the subtile sums of sampled exact match (its
+// own instantiation, so that the other modes carry none of its registers).
+template <bool ZONLY, bool SUB>
 __global__ void __launch_bounds__(H2_THREADS, 1)
     head_tc2_kernel(const __grid_constant__ CUtensorMap tm_w,
                     const __grid_constant__ CUtensorMap tm_h, const Head2Params p) {
@@ -682,7 +751,9 @@ __global__ void __launch_bounds__(H2_THREADS, 1)
     }
     const uint32_t lane_q = static_cast<uint32_t>(q * 32) << 16;
     float* const gathered = p.gathered + static_cast<long long>(pair0) * GATHER_FIELDS;
-    float* const zout = p.zout ? p.zout + static_cast<long long>(pair0) * p.V : nullptr;
+    const ZSink zs{p.zout ? p.zout + static_cast<long long>(pair0) * p.V : nullptr,
+                   p.zsub ? p.zsub + static_cast<long long>(pair0) * p.n_sub : nullptr, p.n_sub,
+                   p.inv_t};
     // slot and phase of the accumulator use the MMA issuer counts next
     int use_slot = 0, use_phase = 0;
     bool ok = true;
@@ -779,10 +850,10 @@ __global__ void __launch_bounds__(H2_THREADS, 1)
         const int gpair = h * p.Ph + g * gsz;
         TileOut t;
         if constexpr (ZONLY)
-          t = group16_z(cb, cb + 8, v_row0, p.V, cx, gpair, npairs, gathered, zout, lane);
+          t = group16_z<SUB>(cb, cb + 8, v_row0, p.V, cx, gpair, npairs, gathered, zs, lane);
         else
-          t = group8_fused(cb, cb + 8, v_row0, p.V, p.alpha, beta, cx, gpair, npairs, gathered,
-                           zout, lane);
+          t = group8_fused<SUB>(cb, cb + 8, v_row0, p.V, p.alpha, beta, cx, gpair, npairs, gathered,
+                           zs, lane);
         st.fold0(is_best, t);
         st.rotate();
         tmem_ld_wait();
@@ -910,20 +981,23 @@ int head_tc2_stages(int N, int pairs, size_t smem_limit) {
   return static_cast<size_t>(st) * per >= tables ? st : 0;
 }
 
-template <bool ZONLY>
+template <bool ZONLY, bool SUB>
 static cudaError_t head_tc2_configure_one(size_t smem_bytes) {
-  cudaError_t e = cudaFuncSetAttribute(head_tc2_kernel<ZONLY>,
+  cudaError_t e = cudaFuncSetAttribute(head_tc2_kernel<ZONLY, SUB>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem_bytes));
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(head_tc2_kernel<ZONLY>, cudaFuncAttributePreferredSharedMemoryCarveout,
+    e = cudaFuncSetAttribute(head_tc2_kernel<ZONLY, SUB>,
+                             cudaFuncAttributePreferredSharedMemoryCarveout,
                              cudaSharedmemCarveoutMaxShared);
   return e;
 }
 
 cudaError_t head_tc2_configure(size_t smem_bytes) {
-  cudaError_t e = head_tc2_configure_one<false>(smem_bytes);
-  if (e == cudaSuccess) e = head_tc2_configure_one<true>(smem_bytes);
+  cudaError_t e = head_tc2_configure_one<false, false>(smem_bytes);
+  if (e == cudaSuccess) e = head_tc2_configure_one<true, false>(smem_bytes);
+  if (e == cudaSuccess) e = head_tc2_configure_one<false, true>(smem_bytes);
+  if (e == cudaSuccess) e = head_tc2_configure_one<true, true>(smem_bytes);
   return e;
 }
 
@@ -941,7 +1015,7 @@ int head_tc2_max_pairs(int N, int pairs, int stages) {
   cfg.numAttrs = 1;
   int n = 0;
   // both instantiations have the same block size and shared memory
-  cudaError_t e = cudaOccupancyMaxActiveClusters(&n, head_tc2_kernel<false>, &cfg);
+  cudaError_t e = cudaOccupancyMaxActiveClusters(&n, head_tc2_kernel<false, false>, &cfg);
   if (e != cudaSuccess) {
     cudaGetLastError();
     return 0;
@@ -1002,6 +1076,9 @@ cudaError_t launch_head_tc2(const HeadArgs& a, const HeadPlan& pl, const HeadTcL
   p.partials = a.partials;
   p.gathered = a.gathered;
   p.zout = a.zout;
+  p.zsub = a.zsub;
+  p.n_sub = (a.V + 31) / 32;
+  p.inv_t = a.inv_t;
   p.status = a.status;
   p.zonly = pl.zonly ? 1 : 0;
   cudaLaunchConfig_t cfg = {};
@@ -1018,8 +1095,12 @@ cudaError_t launch_head_tc2(const HeadArgs& a, const HeadPlan& pl, const HeadTcL
   attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  if (pl.zonly) return cudaLaunchKernelEx(&cfg, head_tc2_kernel<true>, l.tm_w, l.tm_h, p);
-  return cudaLaunchKernelEx(&cfg, head_tc2_kernel<false>, l.tm_w, l.tm_h, p);
+  if (a.zsub != nullptr) {
+    if (pl.zonly) return cudaLaunchKernelEx(&cfg, head_tc2_kernel<true, true>, l.tm_w, l.tm_h, p);
+    return cudaLaunchKernelEx(&cfg, head_tc2_kernel<false, true>, l.tm_w, l.tm_h, p);
+  }
+  if (pl.zonly) return cudaLaunchKernelEx(&cfg, head_tc2_kernel<true, false>, l.tm_w, l.tm_h, p);
+  return cudaLaunchKernelEx(&cfg, head_tc2_kernel<false, false>, l.tm_w, l.tm_h, p);
 }
 
 }  // namespace rv

@@ -579,6 +579,347 @@ cudaError_t launch_sample_fused(const float* z, const float* u, int P, int V, fl
   return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------- draws from subtile sums (Alg. 2)
+// One CTA of 32 warps per position p.  The inverse CDF of softmax(z_p / T)
+// at u_p, in two levels: the head left per 32-row subtile k the pair
+// (m_k, s_k) with s_k = sum exp((z - m_k) / T), so the subtile weights are
+// w_k = s_k exp((m_k - M) / T) (M = max m_k).  The CTA scans the w_k in
+// vocabulary order to the subtile k* whose range holds u S (S = sum w_k),
+// with the fraction f of w_k* below the target.  Warp r then recomputes row r
+// of that subtile's fused logits from the head's own operands (the w row
+// times the position's hsel rows, fp32 sums; z = (1-a) o + a o' as the head
+// forms it), and the first warp picks the first row whose cumulative weight
+// within the subtile exceeds f times the subtile's total.  Up to the rounding of the sums this is the
+// smallest v whose cumulative weight exceeds u * sum(w); a target at or past
+// the rounded total takes the last row of positive weight.
+//
+// The scan: a round covers SUB_ROUND entries; warp w owns SUB_WARP
+// consecutive ones, entry 32 j + lane of them in register j of the lane (the
+// loads coalesce).  Each entry's range [lo, hi) is formed so that one
+// entry's hi and the next entry's lo are the same expression of the same
+// values (the shuffled neighbour, the carried register total, the warp
+// offset), so the ranges tile [0, S) without gaps or overlaps in floating
+// point: a target below S falls in exactly one of them.
+constexpr int SUB_THREADS = 1024;          // one warp per row of a subtile
+constexpr int SUB_REG = 4;                 // subtile entries per lane and round
+constexpr int SUB_WARP = 32 * SUB_REG;
+constexpr int SUB_ROUND = SUB_THREADS * SUB_REG;
+constexpr int SUB_LD = 8;                  // 16-byte weight loads per lane and batch
+
+// A 16-byte read-only load the compiler keeps in program order with the
+// others of its kind (volatile), so that a batch of them is in flight at once.
+// D += A B, m16n8k16, bf16 operands, fp32 accumulators (register order of
+// the PTX fragment layout: a0 / a1 rows g / g+8 at k 2q..2q+1, a2 / a3 the
+// same rows at k 2q+8..2q+9; b0 / b1 column g at k 2q.. / 2q+8..).
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                               uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "{%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ uint4 ldg_batch(const uint4* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
+// One round of the scan: the lane's weights w[], their in-register inclusive
+// scans across the warp (incl[]) and the warp's total; nothing is shared yet.
+// k2 = log2(e) / T: w = s exp2((m - M) k2).
+__device__ __forceinline__ float sub_round_weights(const float2* sub, int n_sub, int base, float M,
+                                                   float k2, int lane, float (&w)[SUB_REG],
+                                                   float (&incl)[SUB_REG], int& last) {
+  float2 e[SUB_REG];  // every load in flight before the first is used
+#pragma unroll
+  for (int j = 0; j < SUB_REG; ++j)
+    e[j] = base + 32 * j < n_sub ? __ldg(sub + base + 32 * j) : make_float2(NEG_INF, 0.f);
+#pragma unroll
+  for (int j = 0; j < SUB_REG; ++j) {
+    const float x = e[j].x == NEG_INF ? 0.f : e[j].y * ex2_approx((e[j].x - M) * k2);
+    w[j] = x;
+    incl[j] = x;
+    if (x > 0.f) last = base + 32 * j;
+  }
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+#pragma unroll
+    for (int j = 0; j < SUB_REG; ++j) {
+      const float y = __shfl_up_sync(0xffffffffu, incl[j], o);
+      if (lane >= o) incl[j] += y;
+    }
+  }
+  float carry = 0.f;
+#pragma unroll
+  for (int j = 0; j < SUB_REG; ++j) carry = carry + __shfl_sync(0xffffffffu, incl[j], 31);
+  return carry;
+}
+
+__global__ void __launch_bounds__(SUB_THREADS, 1)
+    sample_subtiles_kernel(const SubtileDraw d, AcceptArgs acc) {
+  constexpr int NW = SUB_THREADS / 32;
+  static_assert(NW == 32, "one warp per row of a 32-row subtile");
+  __shared__ float s_red[NW];
+  __shared__ float s_wtot[NW];
+  __shared__ float2 s_part[16][32];  // per chunk group: (o, o') of each subtile row
+  __shared__ float s_frac;
+  __shared__ int s_k, s_last;
+  extern __shared__ uint4 s_h[];  // the position's hsel rows: o (and o')
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int p = blockIdx.x;
+  const int nvec = d.H / 8;
+  const float k2 = LOG2E * d.inv_t;
+  const float2* const sub = d.zsub + static_cast<long long>(p) * d.n_sub;
+  if (tid == 0) {
+    s_k = -1;
+    s_last = -1;
+    s_frac = 1.f;
+  }
+  // launched as a programmatic dependent of the LM head: its outputs first
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  // M = max m_k, with the position's hsel rows staged meanwhile
+  const int base0 = SUB_WARP * warp + lane;
+  float m = NEG_INF;
+  for (int r0 = 0; r0 < d.n_sub; r0 += SUB_ROUND) {
+    float mk[SUB_REG];
+#pragma unroll
+    for (int j = 0; j < SUB_REG; ++j) {
+      const int k = r0 + base0 + 32 * j;
+      mk[j] = k < d.n_sub ? __ldg(&sub[k].x) : NEG_INF;
+    }
+    if (r0 == 0) {
+      const int pc = p / d.Pc, pj = p % d.Pc;
+      const uint4* const h_o =
+          static_cast<const uint4*>(d.hsel) + static_cast<long long>(pc * d.N + pj) * nvec;
+      const uint4* const h_r = h_o + static_cast<long long>(d.Pcp) * nvec;
+      for (int c = tid; c < nvec; c += SUB_THREADS) {
+        const uint4 a = __ldg(h_o + c);
+        const uint4 b = d.zonly ? a : __ldg(h_r + c);
+        s_h[c] = a;
+        if (!d.zonly) s_h[nvec + c] = b;
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < SUB_REG; ++j) m = fmaxf(m, mk[j]);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  if (lane == 0) s_red[warp] = m;
+  __syncthreads();
+  float M = s_red[0];
+#pragma unroll
+  for (int k = 1; k < NW; ++k) M = fmaxf(M, s_red[k]);
+  // S: with several rounds, a first pass of the same arithmetic
+  const bool one_round = d.n_sub <= SUB_ROUND;
+  float S = 0.f;
+  float w[SUB_REG], incl[SUB_REG];
+  if (!one_round) {
+    float run = 0.f;
+    for (int r0 = 0; r0 < d.n_sub; r0 += SUB_ROUND) {
+      int dummy = -1;
+      const float wt = sub_round_weights(sub, d.n_sub, r0 + base0, M, k2, lane, w, incl, dummy);
+      __syncthreads();
+      if (lane == 0) s_wtot[warp] = wt;
+      __syncthreads();
+      float woff = 0.f;
+      for (int k = 0; k < NW; ++k) woff = woff + s_wtot[k];
+      run = run + woff;
+    }
+    S = run;
+  }
+  float run = 0.f;
+  for (int r0 = 0; r0 < d.n_sub; r0 += SUB_ROUND) {
+    int last = -1;
+    const float wt = sub_round_weights(sub, d.n_sub, r0 + base0, M, k2, lane, w, incl, last);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) last = max(last, __shfl_xor_sync(0xffffffffu, last, o));
+    if (r0 > 0) __syncthreads();  // s_wtot of the previous round has been read
+    if (lane == 0) {
+      s_wtot[warp] = wt;
+      if (last >= 0) atomicMax(&s_last, last);
+    }
+    __syncthreads();
+    float woff = 0.f, total = 0.f;
+    for (int k = 0; k < NW; ++k) {
+      if (k == warp) woff = total;
+      total = total + s_wtot[k];
+    }
+    if (one_round) S = total;
+    const float target = d.u[p] * S;
+    // the lane's entries: lo = run + (woff + (carry_j + excl_j)), hi likewise
+    // with incl_j (the shuffles first, all independent; then the carries)
+    float excl[SUB_REG], tot[SUB_REG];
+#pragma unroll
+    for (int j = 0; j < SUB_REG; ++j) {
+      excl[j] = __shfl_up_sync(0xffffffffu, incl[j], 1);
+      tot[j] = __shfl_sync(0xffffffffu, incl[j], 31);
+    }
+    float carry = 0.f;
+    int hit = -1;
+    float hit_lo = 0.f;
+#pragma unroll
+    for (int j = 0; j < SUB_REG; ++j) {
+      const float lo = run + (woff + (carry + (lane == 0 ? 0.f : excl[j])));
+      const float hi = run + (woff + (carry + incl[j]));
+      if (target >= lo && target < hi) {
+        hit = j;
+        hit_lo = lo;
+      }
+      carry = carry + tot[j];
+    }
+    if (hit >= 0) {  // one entry of the whole CTA at most
+#pragma unroll
+      for (int j = 0; j < SUB_REG; ++j)
+        if (j == hit) s_frac = (target - hit_lo) / w[j];
+      s_k = r0 + base0 + 32 * hit;
+    }
+    run = run + total;
+    __syncthreads();
+    if (s_k >= 0) break;
+  }
+  // (clamped: a defect upstream must not turn into reads outside w)
+  const int ks = min(max(s_k >= 0 ? s_k : s_last, 0), d.n_sub - 1);
+  const float frac = s_k >= 0 ? fminf(fmaxf(s_frac, 0.f), 1.f) : 1.f;
+  // The subtile's 32 rows times the position's rows on the tensor cores
+  // (mma.sync m16n8k16, bf16 operands, fp32 sums): warp w takes rows
+  // 16 (w & 1) .. + 15 and every 16th 32-element chunk of the hidden
+  // dimension from w >> 1.  A chunk is read as one 16-byte vector per thread
+  // and row (8 consecutive k): thread (g, q) = (lane / 4, lane % 4) holds
+  // k = 32 c + 8 q .. + 7 of rows g and g + 8, and its fragments use them as
+  // the k slots it owns in two consecutive k16 steps (2q, 2q+1 | 2q+8, 2q+9);
+  // the fragment of column g (0: o, 1: o', the others zero) takes the same k
+  // of the position's rows from shared memory.  Both operands see one
+  // permutation of k, so the sums are the dot products.
+  {
+    const int g = lane >> 2, q = lane & 3;
+    const int mt = warp & 1, cw = warp >> 1;
+    const int nch = d.H / 32;
+    const int r0 = 16 * mt + g, r1 = r0 + 8;  // rows within the subtile
+    // (rows at or past V read row V - 1: in bounds; their z is discarded)
+    const uint4* const w0 = static_cast<const uint4*>(d.w) +
+                            static_cast<long long>(min(ks * 32 + r0, d.V - 1)) * nvec + q;
+    const uint4* const w1 = static_cast<const uint4*>(d.w) +
+                            static_cast<long long>(min(ks * 32 + r1, d.V - 1)) * nvec + q;
+    const uint4* const hq = s_h + (g == 1 ? nvec : 0) + q;
+    const bool hcol = g == 0 || (g == 1 && !d.zonly);
+    for (int c = cw; c < nch; c += 16) {  // every chunk of this warp toward L2 first
+      asm volatile("prefetch.global.L2 [%0];" ::"l"(w0 + 4 * c));
+      asm volatile("prefetch.global.L2 [%0];" ::"l"(w1 + 4 * c));
+    }
+    float acc4[4] = {0.f, 0.f, 0.f, 0.f};
+    constexpr int NB = SUB_LD / 2;  // chunks per batch
+    for (int c0 = cw; c0 < nch; c0 += 16 * NB) {
+      uint4 a0[NB], a1[NB];
+#pragma unroll
+      for (int u = 0; u < NB; ++u) {
+        const int c = c0 + 16 * u;
+        a0[u] = c < nch ? ldg_batch(w0 + 4 * c) : make_uint4(0, 0, 0, 0);
+        a1[u] = c < nch ? ldg_batch(w1 + 4 * c) : make_uint4(0, 0, 0, 0);
+      }
+#pragma unroll
+      for (int u = 0; u < NB; ++u) {
+        const int c = c0 + 16 * u;
+        if (c < nch) {  // warp-uniform
+          const uint4 h = hcol ? hq[4 * c] : make_uint4(0, 0, 0, 0);
+          mma_bf16_16816(acc4, a0[u].x, a1[u].x, a0[u].y, a1[u].y, h.x, h.y);
+          mma_bf16_16816(acc4, a0[u].z, a1[u].z, a0[u].w, a1[u].w, h.z, h.w);
+        }
+      }
+    }
+    if (q == 0) {  // columns 0 and 1 of rows r0 and r1
+      s_part[cw][r0] = make_float2(acc4[0], acc4[1]);
+      s_part[cw][r1] = make_float2(acc4[2], acc4[3]);
+    }
+  }
+  __syncthreads();
+  if (warp != 0) return;
+  const int npos = d.gamma + 1, b = p / npos;
+  int last_pos;
+  {
+    float so = 0.f, sr = 0.f;  // row `lane` of the subtile: the 16 partials in order
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      so += s_part[k][lane].x;
+      sr += s_part[k][lane].y;
+    }
+    const float z = ks * 32 + lane < d.V ? (d.zonly ? so : fmaf(d.alpha, sr, (1.f - d.alpha) * so))
+                                         : NEG_INF;
+    float zmax = z;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) zmax = fmaxf(zmax, __shfl_xor_sync(0xffffffffu, zmax, o));
+    const float ew = z == NEG_INF ? 0.f : ex2_approx((z - zmax) * k2);
+    float cum = ew;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float y = __shfl_up_sync(0xffffffffu, cum, o);
+      if (lane >= o) cum += y;
+    }
+    const float tgt = frac * __shfl_sync(0xffffffffu, cum, 31);
+    const unsigned over = __ballot_sync(0xffffffffu, ew > 0.f && cum > tgt);
+    const unsigned pos = __ballot_sync(0xffffffffu, ew > 0.f);
+    const int r = over != 0u ? __ffs(over) - 1 : (pos != 0u ? 31 - __clz(pos) : 0);
+    unsigned t = 0u;
+    if (lane == 0) {
+      d.xhat[p] = ks * 32 + r;
+      if (acc.accepted_len != nullptr)  // release: this position's draw before the ticket;
+        asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;"  // acquire: the others'
+                     : "=r"(t) : "l"(d.tickets + b) : "memory");
+    }
+    last_pos = acc.accepted_len != nullptr &&
+               __shfl_sync(0xffffffffu, t, 0) == static_cast<unsigned>(npos - 1);
+  }
+  if (!last_pos) return;
+  // the sequence's last position: exact match against every draw (Alg. 2),
+  // 32 drafts per round (the ticket's acquire made the other draws visible to
+  // lane 0; the warp barrier below passes that on to the warp)
+  __syncwarp();
+  if (lane == 0) d.tickets[b] = 0u;  // re-armed for the next launch
+  int n = d.gamma, t = 0;
+  for (int i0 = 0; i0 <= d.gamma; i0 += 32) {  // the draws x^_1..x^_{gamma+1}
+    const int i = i0 + lane;
+    const int xh = i <= d.gamma ? __ldcg(d.xhat + b * npos + i) : 0;
+    const bool ok = i >= d.gamma || d.drafts[b * d.gamma + i] == xh;
+    if (i < d.gamma) acc.accept_mask[b * d.gamma + i] = ok ? 1 : 0;
+    const unsigned bad = __ballot_sync(0xffffffffu, !ok);
+    if (bad != 0u && n == d.gamma) n = i0 + __ffs(bad) - 1;
+    const int tn = __shfl_sync(0xffffffffu, xh, (n - i0) & 31);
+    if (n >= i0 && n < i0 + 32) t = tn;
+  }
+  if (lane == 0) {
+    acc.accepted_len[b] = n;
+    acc.next_token[b] = t;
+    acc.ctx_out[b] = acc.ctx_in[b] + n + acc.ctx_extra;
+  }
+}
+
+cudaError_t launch_sample_subtiles(const SubtileDraw& d, const AcceptArgs* acc, cudaStream_t s) {
+  if (d.P <= 0) return cudaSuccess;
+  if (d.H % 32 != 0 || (acc && d.tickets == nullptr)) return cudaErrorInvalidValue;
+  AcceptArgs a = {};
+  if (acc) a = *acc;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(d.P, 1, 1);
+  cfg.blockDim = dim3(SUB_THREADS, 1, 1);
+  cfg.dynamicSmemBytes = static_cast<size_t>(d.zonly ? 1 : 2) * d.H * 2;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (cfg.dynamicSmemBytes > 48 * 1024) {  // hidden sizes above 12288
+    const cudaError_t e = cudaFuncSetAttribute(sample_subtiles_kernel,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               static_cast<int>(cfg.dynamicSmemBytes));
+    if (e != cudaSuccess) return e;
+  }
+  return cudaLaunchKernelEx(&cfg, sample_subtiles_kernel, d, a);
+}
+
 // ---------------------------------------------------------------- typical accept (Alg. 3)
 __global__ void accept_typical_kernel(const int32_t* __restrict__ drafts,
                                       const float* __restrict__ scores,

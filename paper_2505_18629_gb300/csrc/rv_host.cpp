@@ -127,6 +127,10 @@ struct rv_handle {
   // fused logits z [max_batch * (max_gamma + 1)][vocab] written by the head in
   // speculative-sampling mode (allocated on the first rv_set_acceptance to it)
   float* zbuf = nullptr;
+  // per position and 32-row subtile (max z, sum exp((z - max) / T)) for the
+  // sampled-exact-match step of a bf16 handle [max_batch * (max_gamma + 1)]
+  // [ceil(vocab / 32)] (allocated with zbuf)
+  float2* zsub = nullptr;
   // tensor maps of the last tcgen05 attention call and what they were made for
   AttnTcMaps attn_maps;
   const void* attn_map_ptrs[5] = {nullptr, nullptr, nullptr, nullptr, nullptr};
@@ -206,9 +210,11 @@ struct ProfScope {
       cudaEventRecord(h->prof[r].ev[2 * idx], s);
     }
   }
-  ~ProfScope() {
+  void close() {
     if (idx >= 0) cudaEventRecord(h->prof[region].ev[2 * idx + 1], s);
+    idx = -1;
   }
+  ~ProfScope() { close(); }
 };
 
 int validate_config(const rv_config* c) {
@@ -382,6 +388,7 @@ extern "C" RV_API int rv_destroy(rv_handle* h) {
   cudaEventDestroy(h->ev_copy_done);
   cudaStreamDestroy(h->side);
   if (h->zbuf) cudaFree(h->zbuf);
+  if (h->zsub) cudaFree(h->zsub);
   if (h->host_graph) cudaGraphExecDestroy(h->host_graph);
   if (h->pin_in) cudaFreeHost(h->pin_in);
   if (h->pin_out) cudaFreeHost(h->pin_out);
@@ -596,16 +603,32 @@ bool writes_z(const rv_handle* h) {
   return h->accept_mode == RV_ACCEPT_SPECULATIVE || h->accept_mode == RV_ACCEPT_SAMPLED;
 }
 
+// Sampled exact match inside the step (bf16): the head leaves subtile sums at
+// temperature 1 / inv_t instead of the fused logits, and the draws (and the
+// acceptance on them) follow in one launch.
+struct SubtileRequest {
+  const float* u;
+  float inv_t;
+  int32_t* xhat;
+  AcceptArgs acc;
+};
+
 int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_t* draft_ids, int B,
               int gamma, int R, float alpha, float* scores, int32_t* argmax, float* margin,
-              const PackArgs* pack, const AcceptArgs* acc, cudaStream_t s) {
+              const PackArgs* pack, const AcceptArgs* acc, cudaStream_t s,
+              const SubtileRequest* sub = nullptr) {
   const rv_config& c = h->cfg;
   const bool bf16 = c.dtype == RV_DTYPE_BF16;
+  if (sub && (!bf16 || !h->zsub)) return fail(h, RV_ERR_INVALID_ARG, "no subtile-sum buffer");
   HeadArgs a{hidden, w_head, draft_ids, B, gamma, R, c.vocab, c.hidden, alpha,
              h->ws.head_partials, h->ws.gathered, h->ws.status,
              bf16 ? h->ws.status + 16 : nullptr,    // tile counter: its own 64-byte line
              bf16 ? h->ws.status + 32 : nullptr,    // finished-CTA counter
-             writes_z(h) ? h->zbuf : nullptr, h->ws.fin_tickets};
+             writes_z(h) && !sub ? h->zbuf : nullptr, h->ws.fin_tickets};
+  if (sub) {
+    a.zsub = h->zsub;
+    a.inv_t = sub->inv_t;
+  }
   HeadPlan pl = head_plan(B, gamma, c.vocab, h->num_sms, bf16,
                           bf16 && h->head_mode != RV_HEAD_FUSED_LOGITS,
                           bf16 && h->head_mode == RV_HEAD_STANDARD);
@@ -654,10 +677,21 @@ int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_
     h->launches += 1;
   }
   if (e != cudaSuccess) return cuda_fail(h, e, "LM head launch");
-  if (fused) return RV_OK;
-  e = launch_head_finalize(a, pl, scores, argmax, margin, acc, s);
+  if (!fused) {
+    e = launch_head_finalize(a, pl, scores, argmax, margin, acc, s);
+    h->launches += 1;
+    if (e != cudaSuccess) return cuda_fail(h, e, "head finalize launch");
+  }
+  if (!sub) return RV_OK;
+  prof_all.close();
+  ProfScope prof(h, RV_PROF_ACCEPT, s);
+  const SubtileDraw d{h->zsub,    (c.vocab + 31) / 32, sub->u,      sub->inv_t,      w_head,
+                      h->ws.hsel, c.vocab,            c.hidden,    pl.P,            gamma,
+                      pl.pairs_per_chunk, pl.pad_pairs, pl.N,      pl.zonly ? 1 : 0, alpha,
+                      sub->xhat,  draft_ids,          h->ws.fin_tickets};
+  e = launch_sample_subtiles(d, &sub->acc, s);
   h->launches += 1;
-  return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "head finalize launch");
+  return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "subtile draw launch");
 }
 
 int accept_impl(rv_handle* h, const int32_t* draft_ids, const int32_t* argmax, int B, int gamma,
@@ -732,13 +766,23 @@ extern "C" RV_API int rv_set_acceptance(rv_handle* h, int32_t mode, float eps, f
     return RV_OK;
   }
   if (mode == RV_ACCEPT_SPECULATIVE || mode == RV_ACCEPT_SAMPLED) {
+    const rv_config& c = h->cfg;
     if (!h->zbuf) {
-      const rv_config& c = h->cfg;
       const size_t bytes = static_cast<size_t>(c.max_batch) * (c.max_gamma + 1) * c.vocab * 4;
       cudaError_t e = cudaMalloc(&h->zbuf, bytes);
       if (e != cudaSuccess) {
         h->zbuf = nullptr;
         return fail(h, RV_ERR_CUDA, "fused-logit buffer cudaMalloc(%zu): %s", bytes,
+                    cudaGetErrorString(e));
+      }
+    }
+    if (mode == RV_ACCEPT_SAMPLED && c.dtype == RV_DTYPE_BF16 && !h->zsub) {
+      const size_t bytes =
+          static_cast<size_t>(c.max_batch) * (c.max_gamma + 1) * ((c.vocab + 31) / 32) * 8;
+      cudaError_t e = cudaMalloc(&h->zsub, bytes);
+      if (e != cudaSuccess) {
+        h->zsub = nullptr;
+        return fail(h, RV_ERR_CUDA, "subtile-sum buffer cudaMalloc(%zu): %s", bytes,
                     cudaGetErrorString(e));
       }
     }
@@ -872,6 +916,11 @@ int step_impl(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
     AcceptArgs ac{accept_mask, accepted_len,       next_token,         ctx_in,
                   ctx_out,     h->accept_mode,     h->accept_log_eps,  h->accept_log_delta,
                   lead};
+    if (spec && spec->sampled_exact && h->zsub) {
+      const SubtileRequest sr{spec->u, 1.f / spec->temperature, spec->sampled, ac};
+      return head_impl(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin,
+                       do_pack ? &pk : nullptr, nullptr, s, &sr);
+    }
     int r = head_impl(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin,
                       do_pack ? &pk : nullptr, spec ? nullptr : &ac, s);
     if (r == RV_OK && spec && spec->sampled_exact) {

@@ -97,6 +97,11 @@ struct HeadArgs {
   // [B] per-sequence tickets of the finalize launch's acceptance (zero between
   // launches; needed when the finalize runs the acceptance)
   unsigned* seq_tickets = nullptr;
+  // Sampled exact match (Alg. 2, temperature T): per position and 32-row
+  // subtile k (vocab rows [32k, 32k+32) below V) the pair (max z, sum exp((z -
+  // max) / T)), [P][ceil(V / 32)]; or none.  The bf16 tensor-core heads only.
+  float2* zsub = nullptr;
+  float inv_t = 1.f;       // 1 / T for zsub
 };
 
 // ---- small kernels (k_small.cu)
@@ -144,6 +149,30 @@ cudaError_t launch_accept_speculative(const int32_t* drafts, const float* q, con
 // are the fused logits the head wrote.  One CTA per position.
 cudaError_t launch_sample_fused(const float* z, const float* u, int P, int V, float temperature,
                                 int32_t* xhat, cudaStream_t s);
+// Target tokens at temperature T from the head's subtile sums (zsub above):
+// for each of the P positions the inverse CDF of softmax(z / T) at u[p] picks
+// the 32-row subtile from the sums, then the row inside it from that
+// subtile's fused logits, recomputed from the head's operands (w rows, the
+// position's hsel rows as `launch_prep` laid them out for plan `pl`).  With
+// `acc`, the last of a sequence's positions to finish runs the exact-match
+// acceptance on the draws (a ticket per sequence in `tickets`, zero between
+// launches).  One CTA per position.
+struct SubtileDraw {
+  const float2* zsub;
+  int n_sub;
+  const float* u;       // [P]
+  float inv_t;
+  const void* w;        // [V][H] bf16
+  const void* hsel;     // prep's rows
+  int V, H, P, gamma;
+  int Pc, Pcp, N;       // the head plan's chunking of hsel
+  int zonly;            // 1: one row per position (z = w . row)
+  float alpha;
+  int32_t* xhat;        // [P]
+  const int32_t* drafts;
+  unsigned* tickets;
+};
+cudaError_t launch_sample_subtiles(const SubtileDraw& d, const AcceptArgs* acc, cudaStream_t s);
 // Typical acceptance (Alg. 3) from the head's scores and argmax.
 cudaError_t launch_accept_typical(const int32_t* drafts, const float* scores,
                                   const int32_t* argmax, int B, int gamma, float log_eps,

@@ -766,6 +766,25 @@ def test_sampled_exact_match_kernels_and_8b(gu, name):
         _check_sampled(inp, z, u, drafts, 0.8, gpu)
 
 
+@pytest.mark.parametrize("name", ["pairs-two-subgroups", "pairs-two-chunks", "preblended-two-chunks"])
+def test_sampled_exact_match_subtile_draw_layouts(gu, name):
+    # inside rv_verify_step_sampled the head leaves per-32-row subtile sums and
+    # the draw recomputes one subtile from the head's operands: one chunk of
+    # 150 pairs in two sub-groups, two chunks of 160 pairs in two sub-groups,
+    # and the pre-blended head over two chunks; vocabularies not a multiple
+    # of 32, two temperatures
+    pre = name.startswith("preblended")
+    B, g = (15, 9) if name == "pairs-two-subgroups" else (32, 9) if not pre else (40, 7)
+    V = {"pairs-two-subgroups": 1777, "pairs-two-chunks": 1501, "preblended-two-chunks": 1243}[name]
+    from paper_2505_18629_gb300 import synth
+    wl = _wl(B=B, gamma=g, R=6, V=V, H=256, ctx=(5, 40), seed=96)
+    inp = synth.generate(wl)
+    for T in (0.8, 0.3):
+        z, u, drafts = _sampled_inputs(inp, ALPHA, T, 97, preblended=pre)
+        _check_sampled(inp, z, u, drafts, T, _run_sampled(gu, inp, drafts, ALPHA, T, u,
+                                                           preblended=pre))
+
+
 # ------------------------------------------------------------------ pending-token block
 
 def _pending_run(gu, wl, alpha=ALPHA, seed=0, check_attn=True):

@@ -326,116 +326,209 @@ __global__ void accept_kernel(const int32_t* __restrict__ drafts,
 }
 
 // ---------------------------------------------------------------- speculative accept (Alg. 1)
-// One CTA per sequence.  Thread 0 runs the ratio test: draft i is kept while
+// A cluster of SPC_CL CTAs per sequence.  The first warp of every CTA runs the
+// ratio test (one lane per draft): draft i is kept while
 // log r_i <= log p_i(x_i) - log q_i(x_i) (p_i from the head's fused log-prob),
-// n = the number of leading kept drafts.  Then the CTA draws t from
+// n = the number of leading kept drafts.  Then the cluster draws t from
 //   p' = norm(max(0, p_{n+1} - q_{n+1}))  (n < gamma)   or   p_{gamma+1}
-// by inverse CDF with u: each thread sums the weights of a contiguous range of
-// the vocabulary, a block-wide exclusive scan orders the ranges, and the
-// thread whose range holds u * sum(w) walks it to the token.
-constexpr int SPEC_THREADS = 1024;
+// by inverse CDF with u.  CTA c owns the c-th of SPC_CL equal slices of the
+// vocabulary; it scans the weights of its slice in vocabulary order (warp w
+// owns SPC_WARP consecutive tokens, lane l the ones at 32 j + l: the loads
+// coalesce) and sends its total to every CTA of the cluster.  Every CTA forms
+// the same prefix of the slice totals, so all agree on the slice that holds
+// u * sum(w); that CTA finds the token.  Each range's upper end and the next
+// range's lower end are the same expression of the same values, within a
+// slice as between slices, so the ranges tile [0, sum(w)) exactly in floating
+// point.  If every residual weight is zero (p_{n+1} <= q_{n+1} everywhere, only
+// through rounding) the draw is from p_{n+1} itself.
+constexpr int SPC_CL = 16;
+constexpr int SPC_THREADS = 512;
+constexpr int SPC_E = 16;                        // tokens per lane and round
+constexpr int SPC_WARP = 32 * SPC_E;
+constexpr int SPC_ROUND = SPC_THREADS * SPC_E;
 
-__device__ __forceinline__ float spec_weight(const float* zrow, const float* qrow, float lse, int v) {
-  const float p = __expf(zrow[v] - lse);
-  return qrow ? fmaxf(0.f, p - qrow[v]) : p;
+__device__ __forceinline__ float spec_weight(float zv, float qv, float lse, bool resid) {
+  const float p = __expf(zv - lse);
+  return resid ? fmaxf(0.f, p - qv) : p;
 }
 
-__global__ void __launch_bounds__(SPEC_THREADS)
+// One round of a slice: the lane's weights and their warp scans (see
+// sub_round_weights); returns the warp's total.
+__device__ __forceinline__ float spc_round(const float* zrow, const float* qrow, float lse,
+                                           bool resid, int base, int v_hi, int lane,
+                                           float (&w)[SPC_E], float (&incl)[SPC_E], int& last) {
+  float zv[SPC_E], qv[SPC_E];
+#pragma unroll
+  for (int j = 0; j < SPC_E; ++j) {
+    const int v = base + 32 * j;
+    zv[j] = v < v_hi ? __ldg(zrow + v) : NEG_INF;
+    qv[j] = (resid && v < v_hi) ? __ldg(qrow + v) : 0.f;
+  }
+#pragma unroll
+  for (int j = 0; j < SPC_E; ++j) {
+    w[j] = zv[j] == NEG_INF ? 0.f : spec_weight(zv[j], qv[j], lse, resid);
+    incl[j] = w[j];
+    if (w[j] > 0.f) last = base + 32 * j;
+  }
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+#pragma unroll
+    for (int j = 0; j < SPC_E; ++j) {
+      const float y = __shfl_up_sync(0xffffffffu, incl[j], o);
+      if (lane >= o) incl[j] += y;
+    }
+  }
+  float carry = 0.f;
+#pragma unroll
+  for (int j = 0; j < SPC_E; ++j) carry = carry + __shfl_sync(0xffffffffu, incl[j], 31);
+  return carry;
+}
+
+__global__ void __launch_bounds__(SPC_THREADS)
     accept_speculative_kernel(const int32_t* __restrict__ drafts, const float* __restrict__ q,
                               const float* __restrict__ r, const float* __restrict__ u,
                               const float* __restrict__ scores, const float* __restrict__ z,
                               int gamma, int V, AcceptArgs a, unsigned* status) {
-  constexpr int NW = SPEC_THREADS / 32;
-  __shared__ float s_wtot[NW], s_woff[NW];
-  __shared__ float s_total;
-  __shared__ int s_n, s_t, s_last;
-  const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  if (tid == 0) {
+  constexpr int NW = SPC_THREADS / 32;
+  __shared__ float s_wc[2][SPC_CL];  // every slice's total, per pass (written by its CTA)
+  __shared__ int s_lastc[2][SPC_CL];  // every slice's last token of positive weight
+  __shared__ float s_wtot[NW];
+  __shared__ int s_n, s_last;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  uint32_t rank;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(rank));
+  const int b = blockIdx.x / SPC_CL;
+  // (other CTAs' shared memory is written only after every CTA has started)
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+  if (warp == 0) {  // the ratio test, 32 drafts per round
     int n = gamma;
-    for (int i = 0; i < gamma; ++i) {
-      const int x = drafts[b * gamma + i];
-      const float logp = scores[(static_cast<long long>(b) * (gamma + 1) + i) * RV_NSCORES +
-                                RV_SCORE_LOGP_FUSED];
-      bool keep = false;
-      if (x >= 0 && x < V) {
-        const float qx = q[(static_cast<long long>(b) * gamma + i) * V + x];
-        // log r <= log p - log q; q(x) = 0 makes the ratio infinite (kept)
-        keep = qx > 0.f ? logf(r[b * gamma + i]) <= logp - logf(qx) : logp > NEG_INF;
-      } else {
-        raise_status(status, RV_DEV_DRAFT_RANGE);
+    for (int i0 = 0; i0 < gamma; i0 += 32) {
+      const int i = i0 + lane;
+      bool keep = true;
+      if (i < gamma) {
+        const int x = drafts[b * gamma + i];
+        const float logp = scores[(static_cast<long long>(b) * (gamma + 1) + i) * RV_NSCORES +
+                                  RV_SCORE_LOGP_FUSED];
+        keep = false;
+        if (x >= 0 && x < V) {
+          const float qx = q[(static_cast<long long>(b) * gamma + i) * V + x];
+          // log r <= log p - log q; q(x) = 0 makes the ratio infinite (kept)
+          keep = qx > 0.f ? logf(r[b * gamma + i]) <= logp - logf(qx) : logp > NEG_INF;
+        } else if (rank == 0) {
+          raise_status(status, RV_DEV_DRAFT_RANGE);
+        }
+        if (rank == 0) a.accept_mask[b * gamma + i] = keep ? 1 : 0;
       }
-      a.accept_mask[b * gamma + i] = keep ? 1 : 0;
-      if (!keep && n == gamma) n = i;
+      const unsigned bad = __ballot_sync(0xffffffffu, !keep);
+      if (bad != 0u && n == gamma) n = i0 + __ffs(bad) - 1;
     }
-    s_n = n;
-    s_t = -1;
-    s_last = -1;
+    if (lane == 0) s_n = n;
   }
   __syncthreads();
   const int n = s_n;
   const long long prow = static_cast<long long>(b) * (gamma + 1) + n;
   const float lse = scores[prow * RV_NSCORES + RV_SCORE_LSE_FUSED];
-  const float* zrow = z + prow * V;
-  const float* qrow = n < gamma ? q + (static_cast<long long>(b) * gamma + n) * V : nullptr;
-  const int chunk = (V + SPEC_THREADS - 1) / SPEC_THREADS;
-  const int c0 = min(V, tid * chunk), c1 = min(V, c0 + chunk);
-  for (int pass = 0; pass < 2; ++pass) {  // pass 1 only when every residual weight is zero
-    float part = 0.f;
-    for (int v = c0; v < c1; ++v) part += spec_weight(zrow, qrow, lse, v);
-    float incl = part;  // inclusive scan within the warp
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const float y = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += y;
-    }
-    if (lane == 31) s_wtot[warp] = incl;
-    __syncthreads();
-    if (warp == 0) {  // exclusive scan of the warp totals
-      const float w = s_wtot[lane];
-      float wi = w;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const float y = __shfl_up_sync(0xffffffffu, wi, o);
-        if (lane >= o) wi += y;
-      }
-      s_woff[lane] = wi - w;
-      if (lane == 31) s_total = wi;
-    }
-    __syncthreads();
-    const float W = s_total;
-    if (!(W > 0.f)) {  // p_{n+1} <= q_{n+1} everywhere (only through rounding): draw from p_{n+1}
-      qrow = nullptr;
+  const float* const zrow = z + prow * V;
+  const float* const qrow = q + (static_cast<long long>(b) * gamma + min(n, gamma - 1)) * V;
+  const int Vc = (V + SPC_CL - 1) / SPC_CL;
+  const int v_lo = min(V, static_cast<int>(rank) * Vc), v_hi = min(V, v_lo + Vc);
+  const int base0 = v_lo + SPC_WARP * warp + lane;
+  const bool one_round = v_hi - v_lo <= SPC_ROUND;
+  float w[SPC_E], incl[SPC_E];
+  for (int pass = 0; pass < 2; ++pass) {
+    const bool resid = pass == 0 && n < gamma;
+    // this slice's total, in the scan's own arithmetic
+    float run = 0.f, wt_first = 0.f;
+    int last = -1;
+    for (int r0 = 0; r0 < v_hi - v_lo; r0 += SPC_ROUND) {
+      const float wt = spc_round(zrow, qrow, lse, resid, base0 + r0, v_hi, lane, w, incl, last);
+      if (r0 == 0) wt_first = wt;
       __syncthreads();
-      continue;
+      if (lane == 0) s_wtot[warp] = wt;
+      __syncthreads();
+      float total = 0.f;
+      for (int k = 0; k < NW; ++k) total = total + s_wtot[k];
+      run = run + total;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) last = max(last, __shfl_xor_sync(0xffffffffu, last, o));
+    if (tid == 0) s_last = -1;
+    __syncthreads();
+    if (lane == 0 && last >= 0) atomicMax(&s_last, last);
+    __syncthreads();
+    // to every CTA of the cluster: this slice's total and last weighted token
+    if (pass == 0) asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+    if (tid < SPC_CL) {
+      uint32_t d0, d1;
+      asm volatile("mapa.shared::cluster.u32 %0, %1, %2;"
+                   : "=r"(d0) : "r"(smem_u32(&s_wc[pass][rank])), "r"(tid));
+      asm volatile("mapa.shared::cluster.u32 %0, %1, %2;"
+                   : "=r"(d1) : "r"(smem_u32(&s_lastc[pass][rank])), "r"(tid));
+      asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(d0), "f"(run) : "memory");
+      asm volatile("st.shared::cluster.s32 [%0], %1;" ::"r"(d1), "r"(s_last) : "memory");
+    }
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                     : "memory");
+    float W = 0.f;
+    for (int c = 0; c < SPC_CL; ++c) W = W + s_wc[pass][c];
+    if (!(W > 0.f)) {  // (the same in every CTA of the cluster)
+      if (pass == 0) continue;
+      if (rank == 0 && tid == 0) a.next_token[b] = 0;  // no weight at all: non-finite logits
+      break;
     }
     const float target = u[b] * W;
-    const float lo = s_woff[warp] + (incl - part);
-    if (part > 0.f) atomicMax(&s_last, tid);
-    if (part > 0.f && target >= lo && target < lo + part) {
-      float c = lo;
-      int t = -1;
-      for (int v = c0; v < c1; ++v) {
-        const float w = spec_weight(zrow, qrow, lse, v);
-        c += w;
-        if (w > 0.f) t = v;
-        if (w > 0.f && c > target) break;
+    float P = 0.f;
+    int owner = -1, last_c = -1;
+    float P_owner = 0.f;
+    for (int c = 0; c < SPC_CL; ++c) {
+      const float Pn = P + s_wc[pass][c];
+      if (owner < 0 && target >= P && target < Pn) {
+        owner = c;
+        P_owner = P;
       }
-      atomicMax(&s_t, t);
+      if (s_wc[pass][c] > 0.f) last_c = c;
+      P = Pn;
     }
-    __syncthreads();
-    // u * W at or past the rounded sum of the ranges: the last token with weight
-    if (s_t < 0 && tid == s_last) {
-      int t = -1;
-      for (int v = c0; v < c1; ++v)
-        if (spec_weight(zrow, qrow, lse, v) > 0.f) t = v;
-      s_t = t;
+    if (owner < 0) {  // u * W at or past the rounded total: the last token with weight
+      if (static_cast<int>(rank) == last_c && tid == 0) a.next_token[b] = s_lastc[pass][last_c];
+      break;
     }
+    if (static_cast<int>(rank) != owner) break;
+    // the owner: the token whose range holds the target
+    run = 0.f;
+    if (tid == 0) s_last = -1;  // reused: the token found
+    for (int r0 = 0; r0 < v_hi - v_lo; r0 += SPC_ROUND) {
+      int dummy = -1;
+      const float wt = one_round ? wt_first
+                                 : spc_round(zrow, qrow, lse, resid, base0 + r0, v_hi, lane, w,
+                                             incl, dummy);
+      __syncthreads();
+      if (lane == 0) s_wtot[warp] = wt;
+      __syncthreads();
+      float woff = 0.f, total = 0.f;
+      for (int k = 0; k < NW; ++k) {
+        if (k == warp) woff = total;
+        total = total + s_wtot[k];
+      }
+      float carry = 0.f;
+#pragma unroll
+      for (int j = 0; j < SPC_E; ++j) {
+        const float ex = __shfl_up_sync(0xffffffffu, incl[j], 1);
+        const float tj = __shfl_sync(0xffffffffu, incl[j], 31);
+        const float lo = P_owner + (run + (woff + (carry + (lane == 0 ? 0.f : ex))));
+        const float hi = P_owner + (run + (woff + (carry + incl[j])));
+        if (target >= lo && target < hi) s_last = base0 + r0 + 32 * j;
+        carry = carry + tj;
+      }
+      run = run + total;
+      __syncthreads();
+      if (s_last >= 0) break;
+    }
+    if (tid == 0) a.next_token[b] = s_last >= 0 ? s_last : s_lastc[pass][owner];
     break;
   }
-  __syncthreads();
-  if (tid == 0) {
+  if (rank == 0 && tid == 0) {
     a.accepted_len[b] = n;
-    a.next_token[b] = s_t >= 0 ? s_t : 0;
     a.ctx_out[b] = a.ctx_in[b] + n + a.ctx_extra;
   }
 }
@@ -446,10 +539,27 @@ cudaError_t launch_accept_speculative(const int32_t* drafts, const float* q, con
                                       int32_t* accepted_len, int32_t* next_token,
                                       const int32_t* ctx_in, int32_t* ctx_out, unsigned* status,
                                       cudaStream_t s, int ctx_extra) {
+  static bool configured = false;
+  if (!configured) {
+    const cudaError_t e = cudaFuncSetAttribute(accept_speculative_kernel,
+                                               cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
   AcceptArgs a{accept_mask, accepted_len, next_token, ctx_in, ctx_out, 0, 0.f, 0.f, ctx_extra};
-  accept_speculative_kernel<<<B, SPEC_THREADS, 0, s>>>(drafts, q, r, u, scores, z, gamma, V, a,
-                                                       status);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(B * SPC_CL, 1, 1);
+  cfg.blockDim = dim3(SPC_THREADS, 1, 1);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = SPC_CL;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, accept_speculative_kernel, drafts, q, r, u, scores, z, gamma, V,
+                            a, status);
 }
 
 // ---------------------------------------------------------------- sampled target tokens (Alg. 2)

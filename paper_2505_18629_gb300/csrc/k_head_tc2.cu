@@ -839,6 +839,10 @@ __global__ void __launch_bounds__(H2_THREADS, 1)
           ngi = 0;
         }
         const bool more = idx + 1 < n_mine;
+        // this group (the last of sub-group h unless the next one is h's too)
+        // is in registers already: h's slot is free before it is reduced, so
+        // the MMAs of the next tile need not wait for this reduction
+        if (!more || nh != h) release_slot(h);
         if (more && nh != h && !wait_slot(nh)) {
           ok = false;
           break;
@@ -862,8 +866,6 @@ __global__ void __launch_bounds__(H2_THREADS, 1)
         for (int k = 0; k < 16; ++k) cb[k] = nb[k];
 #pragma unroll
         for (int j = 0; j < NC; ++j) cx[j] = nx[j];
-        // the last group of a sub-group has been read: its slot is free
-        if (!more || nh != h) release_slot(h);
         h = nh;
         gi = ngi;
       }

@@ -396,7 +396,8 @@ def run_variant(args):
     are softmax(N(0, 1)) rows."""
     import torch
     from paper_2505_18629_gb300 import rv, synth
-    if args.pending and args.accept in ("speculative", "sampled"):
+    sampled_rule = args.accept in ("sampled", "typical-sampled")
+    if args.pending and (args.accept == "speculative" or sampled_rule):
         raise SystemExit("--pending runs the exact-match or typical rule")
     wl = synth.workload(args.workload)
     if args.pending:  # the cache takes the block and the pending token
@@ -448,8 +449,11 @@ def run_variant(args):
         q_draft = torch.softmax(torch.randn((B, g, wl.V), generator=gen, device=dev), dim=-1)
         r_u = torch.rand((B, g), generator=gen, device=dev)
         u_u = torch.rand((B,), generator=gen, device=dev)
-    elif args.accept == "sampled":
-        rv.rv_set_acceptance(h, rv.RV_ACCEPT_SAMPLED)
+    elif sampled_rule:
+        if args.accept == "sampled":
+            rv.rv_set_acceptance(h, rv.RV_ACCEPT_SAMPLED)
+        else:
+            rv.rv_set_acceptance(h, rv.RV_ACCEPT_TYPICAL_SAMPLED, TYPICAL_EPS, TYPICAL_DELTA)
         u_s = torch.rand((B, g + 1), generator=gen, device=dev)
         sampled = torch.empty((B, g + 1), dtype=torch.int32, device=dev)
 
@@ -462,7 +466,7 @@ def run_variant(args):
             rv.rv_verify_step_speculative(h, q, kb, vb, kc, vc, hidden, W, drafts, prompt, prefix,
                                           ctx, ALPHA, q_draft, r_u, u_u, block, pos, attn, scores,
                                           argmax, margin, acc, alen, nxt, ctx_out, stream)
-        elif args.accept == "sampled":
+        elif args.accept in ("sampled", "typical-sampled"):
             rv.rv_verify_step_sampled(h, q, kb, vb, kc, vc, hidden, W, drafts, prompt, prefix,
                                       ctx, ALPHA, SAMPLED_T, u_s, block, pos, attn, scores, argmax,
                                       margin, sampled, acc, alen, nxt, ctx_out, stream)
@@ -476,7 +480,7 @@ def run_variant(args):
     us = _time_steps(step, args.steps, max(args.warmup, 3), stream)
     clk = clocks.stop()
     accept_us = None
-    if args.accept in ("speculative", "sampled"):
+    if args.accept in ("speculative", "sampled", "typical-sampled"):
         rv.rv_profile_enable(h, 1 << rv.RV_PROF_ACCEPT)
         for _ in range(min(args.steps, 100)):
             step()
@@ -531,11 +535,12 @@ def main():
                     help="fused: both logit vectors fused per vocab row (Eq. 2); preblended: "
                          "the head on the blended hidden states (one row per position)")
     ap.add_argument("--accept", default="exact",
-                    choices=["exact", "typical", "speculative", "sampled"],
+                    choices=["exact", "typical", "speculative", "sampled", "typical-sampled"],
                     help="acceptance rule of the step: exact match (Alg. 2, default), typical "
                          "(Alg. 3), speculative sampling (Alg. 1), exact match against sampled "
-                         "target tokens (Alg. 2 at temperature T); other than exact, or with "
-                         "--pending, one JSON line of the step's device time")
+                         "target tokens (Alg. 2 at temperature T), typical with t sampled at T "
+                         "(Alg. 3); other than exact, or with --pending, one JSON line of the "
+                         "step's device time")
     ap.add_argument("--pending", action="store_true",
                     help="the pending-token block [t, x, template, x] (exact or typical rule)")
     ap.add_argument("--sweep", action="store_true",

@@ -82,6 +82,7 @@ extern "C" {
 #define RV_ACCEPT_TYPICAL 1     /* entropy-based threshold of typical acceptance (Alg. 3)     */
 #define RV_ACCEPT_SPECULATIVE 2 /* speculative sampling with residual resampling (Alg. 1)     */
 #define RV_ACCEPT_SAMPLED 3     /* exact match with target tokens sampled at temperature T (Alg. 2) */
+#define RV_ACCEPT_TYPICAL_SAMPLED 4 /* typical acceptance (Alg. 3), t ~ p_{n+1} at temperature T */
 
 /* LM-head variants (rv_set_head_mode). */
 #define RV_HEAD_FUSED_LOGITS 0  /* o_i and o_{m+i-1} from their own rows, fused (Eq. 2)      */
@@ -224,7 +225,16 @@ RV_API int rv_accept_typical(rv_handle* h, const int32_t* draft_ids, const float
  *     floats), which rv_accept_speculative / rv_verify_step_speculative and
  *     rv_accept_sampled / rv_verify_step_sampled read; in these modes plain
  *     rv_verify_step returns RV_ERR_INVALID_ARG (it has no draft
- *     distributions or uniforms).
+ *     distributions or uniforms).  Inside rv_verify_step_sampled a bf16
+ *     handle's head writes no logits: per position and 32-row vocabulary
+ *     subtile it stores (max z, sum exp((z - max) / T)) in a second buffer
+ *     allocated here (max_batch * (max_gamma+1) * ceil(vocab / 32) pairs of
+ *     floats), and the draw recomputes the logits of one subtile;
+ *   RV_ACCEPT_TYPICAL_SAMPLED (eps > 0, delta > 0, the fused head mode):
+ *     typical acceptance as RV_ACCEPT_TYPICAL for the kept drafts and n, with
+ *     the next token drawn as Alg. 3 states, t ~ p_{n+1} at temperature T
+ *     (the draw of rv_accept_sampled at position n+1); it takes the same
+ *     buffers and applies to rv_verify_step_sampled only.
  * Errors: RV_ERR_INVALID_ARG for an unknown mode or bad eps / delta,
  * RV_ERR_CUDA if the buffer cannot be allocated. */
 RV_API int rv_set_acceptance(rv_handle* h, int32_t mode, float eps, float delta);
@@ -351,10 +361,12 @@ RV_API int rv_verify_step_speculative(
     void* attn_out, float* scores, int32_t* argmax, float* margin, uint8_t* accept_mask,
     int32_t* accepted_len, int32_t* next_token, int32_t* ctx_out, void* stream);
 
-/* rv_verify_step with exact-match verification against target tokens
- * sampled at temperature T (rv_accept_sampled) in place of the greedy rule;
- * needs the handle in RV_ACCEPT_SAMPLED mode.  temperature, u_uniform and
- * sampled as in rv_accept_sampled; two launches more than rv_verify_step. */
+/* rv_verify_step with target tokens sampled at temperature T in place of the
+ * greedy choice; needs the handle in RV_ACCEPT_SAMPLED mode (exact match
+ * against the draws, as rv_accept_sampled) or RV_ACCEPT_TYPICAL_SAMPLED
+ * (typical acceptance, t = the draw at position n+1).  temperature,
+ * u_uniform and sampled as in rv_accept_sampled.  On a bf16 handle one launch
+ * more than rv_verify_step (the draws and the acceptance); on fp32 two. */
 RV_API int rv_verify_step_sampled(
     rv_handle* h, const void* q, const void* k_blk, const void* v_blk, void* k_cache,
     void* v_cache, const void* hidden, const void* w_head, const int32_t* draft_ids,

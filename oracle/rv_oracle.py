@@ -515,6 +515,37 @@ def sampled_exact_accept(drafts, z, temperature: float, u):
     return acc, n, t, xhat, cdf_gap
 
 
+def typical_accept_sampled(drafts, logp_fused, ent_orig, z, eps: float, delta: float,
+                           temperature: float, u):
+    """Typical acceptance (Alg. 3) with the next token sampled at temperature T.
+
+    The kept drafts and n are those of ``typical_accept`` (the entropy
+    threshold on the fused distribution, Eq. 2); the next token is drawn as
+    Alg. 3 states, t ~ p_{n+1}, at sampling temperature T: the inverse CDF of
+    softmax(z_{n+1} / T) at the uniform u[b, n] (one uniform per position,
+    [B, gamma+1], as for ``sampled_exact_accept``).  T -> 0 gives the greedy t
+    of ``typical_accept``.
+
+    Returns (accept_mask [B, gamma] bool, n [B], t [B], gap [B, gamma],
+    cdf_gap [B]) with gap as in ``typical_accept`` and cdf_gap the distance of
+    u[b, n] from the nearest cumulative-weight boundary of the draw.
+    """
+    z = np.asarray(z, np.float64)
+    u = np.asarray(u, np.float64)
+    B = z.shape[0]
+    acc, n, _, gap = typical_accept(drafts, logp_fused, ent_orig,
+                                    np.zeros(z.shape[:2], np.int64), eps, delta)
+    t = np.zeros(B, np.int64)
+    cdf_gap = np.zeros(B)
+    for b in range(B):
+        zt = z[b, n[b]] / float(temperature)
+        w = np.exp(zt - zt.max())
+        t[b] = inverse_cdf_sample(w, float(u[b, n[b]]))
+        c = np.cumsum(w) / w.sum()
+        cdf_gap[b] = np.min(np.abs(c - u[b, n[b]]))
+    return acc, n, t, gap, cdf_gap
+
+
 def verify_step(inp_W, hidden, q, k_blk, v_blk, k_cache, v_cache, ctx_lens,
                 drafts, prompt_ids, prefix_ids, gamma: int, R: int, alpha: float):
     """One whole verify step: pack, attention, head + fusion, accept, prefix.

@@ -983,7 +983,7 @@ __global__ void __launch_bounds__(SUB_THREADS, 1)
                __shfl_sync(0xffffffffu, t, 0) == static_cast<unsigned>(npos - 1);
   }
   if (!last_pos) return;
-  // the sequence's last position: exact match against every draw (Alg. 2),
+  // the sequence's last position: the acceptance against every draw (Alg. 2 or 3),
   // 32 drafts per round (the ticket's acquire made the other draws visible to
   // lane 0; the warp barrier below passes that on to the warp)
   __syncwarp();
@@ -992,7 +992,17 @@ __global__ void __launch_bounds__(SUB_THREADS, 1)
   for (int i0 = 0; i0 <= d.gamma; i0 += 32) {  // the draws x^_1..x^_{gamma+1}
     const int i = i0 + lane;
     const int xh = i <= d.gamma ? __ldcg(d.xhat + b * npos + i) : 0;
-    const bool ok = i >= d.gamma || d.drafts[b * d.gamma + i] == xh;
+    bool ok = true;
+    if (i < d.gamma) {
+      const int x = d.drafts[b * d.gamma + i];
+      if (acc.mode == RV_ACCEPT_TYPICAL) {  // Alg. 3: the threshold, t still the draw at n+1
+        const float* sc = d.scores + static_cast<long long>(b * npos + i) * RV_NSCORES;
+        ok = position_kept(acc, x, xh, __ldcg(sc + RV_SCORE_LOGP_FUSED),
+                           __ldcg(sc + RV_SCORE_ENT_ORIG));
+      } else {
+        ok = x == xh;
+      }
+    }
     if (i < d.gamma) acc.accept_mask[b * d.gamma + i] = ok ? 1 : 0;
     const unsigned bad = __ballot_sync(0xffffffffu, !ok);
     if (bad != 0u && n == d.gamma) n = i0 + __ffs(bad) - 1;

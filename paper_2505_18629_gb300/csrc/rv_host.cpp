@@ -600,7 +600,8 @@ int check_head_args(rv_handle* h, const void* hidden, const void* w_head, const 
 
 // The head also writes the fused logits (speculative sampling, sampled exact match).
 bool writes_z(const rv_handle* h) {
-  return h->accept_mode == RV_ACCEPT_SPECULATIVE || h->accept_mode == RV_ACCEPT_SAMPLED;
+  return h->accept_mode == RV_ACCEPT_SPECULATIVE || h->accept_mode == RV_ACCEPT_SAMPLED ||
+         h->accept_mode == RV_ACCEPT_TYPICAL_SAMPLED;
 }
 
 // Sampled exact match inside the step (bf16): the head leaves subtile sums at
@@ -688,7 +689,7 @@ int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_
   const SubtileDraw d{h->zsub,    (c.vocab + 31) / 32, sub->u,      sub->inv_t,      w_head,
                       h->ws.hsel, c.vocab,            c.hidden,    pl.P,            gamma,
                       pl.pairs_per_chunk, pl.pad_pairs, pl.N,      pl.zonly ? 1 : 0, alpha,
-                      sub->xhat,  draft_ids,          h->ws.fin_tickets};
+                      sub->xhat,  draft_ids,          h->ws.fin_tickets, scores};
   e = launch_sample_subtiles(d, &sub->acc, s);
   h->launches += 1;
   return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "subtile draw launch");
@@ -765,7 +766,17 @@ extern "C" RV_API int rv_set_acceptance(rv_handle* h, int32_t mode, float eps, f
     h->accept_mode = mode;
     return RV_OK;
   }
-  if (mode == RV_ACCEPT_SPECULATIVE || mode == RV_ACCEPT_SAMPLED) {
+  const bool typical = mode == RV_ACCEPT_TYPICAL || mode == RV_ACCEPT_TYPICAL_SAMPLED;
+  if (typical) {
+    if (h->head_mode != RV_HEAD_FUSED_LOGITS)
+      return fail(h, RV_ERR_INVALID_ARG,
+                  "typical acceptance needs the original distribution's entropy, which the "
+                  "single-distribution heads do not form");
+    if (!(eps > 0.f) || !(delta > 0.f) || !std::isfinite(eps) || !std::isfinite(delta))
+      return fail(h, RV_ERR_INVALID_ARG, "typical acceptance needs finite eps > 0 and delta > 0");
+  }
+  if (mode == RV_ACCEPT_SPECULATIVE || mode == RV_ACCEPT_SAMPLED ||
+      mode == RV_ACCEPT_TYPICAL_SAMPLED) {
     const rv_config& c = h->cfg;
     if (!h->zbuf) {
       const size_t bytes = static_cast<size_t>(c.max_batch) * (c.max_gamma + 1) * c.vocab * 4;
@@ -776,7 +787,7 @@ extern "C" RV_API int rv_set_acceptance(rv_handle* h, int32_t mode, float eps, f
                     cudaGetErrorString(e));
       }
     }
-    if (mode == RV_ACCEPT_SAMPLED && c.dtype == RV_DTYPE_BF16 && !h->zsub) {
+    if (mode != RV_ACCEPT_SPECULATIVE && c.dtype == RV_DTYPE_BF16 && !h->zsub) {
       const size_t bytes =
           static_cast<size_t>(c.max_batch) * (c.max_gamma + 1) * ((c.vocab + 31) / 32) * 8;
       cudaError_t e = cudaMalloc(&h->zsub, bytes);
@@ -787,15 +798,13 @@ extern "C" RV_API int rv_set_acceptance(rv_handle* h, int32_t mode, float eps, f
       }
     }
     h->accept_mode = mode;
+    if (typical) {
+      h->accept_log_eps = logf(eps);
+      h->accept_log_delta = logf(delta);
+    }
     return RV_OK;
   }
   if (mode != RV_ACCEPT_TYPICAL) return fail(h, RV_ERR_INVALID_ARG, "unknown acceptance mode %d", mode);
-  if (h->head_mode != RV_HEAD_FUSED_LOGITS)
-    return fail(h, RV_ERR_INVALID_ARG,
-                "typical acceptance needs the original distribution's entropy, which the "
-                "single-distribution heads do not form");
-  if (!(eps > 0.f) || !(delta > 0.f) || !std::isfinite(eps) || !std::isfinite(delta))
-    return fail(h, RV_ERR_INVALID_ARG, "typical acceptance needs finite eps > 0 and delta > 0");
   h->accept_mode = mode;
   h->accept_log_eps = logf(eps);
   h->accept_log_delta = logf(delta);
@@ -813,7 +822,7 @@ extern "C" RV_API int rv_set_head_mode(rv_handle* h, int32_t mode) {
     return fail(h, RV_ERR_INVALID_ARG, "unknown head mode %d", mode);
   if (h->cfg.dtype != RV_DTYPE_BF16)
     return fail(h, RV_ERR_UNSUPPORTED, "the single-distribution heads are bf16 LM-head variants");
-  if (h->accept_mode == RV_ACCEPT_TYPICAL)
+  if (h->accept_mode == RV_ACCEPT_TYPICAL || h->accept_mode == RV_ACCEPT_TYPICAL_SAMPLED)
     return fail(h, RV_ERR_INVALID_ARG,
                 "typical acceptance needs the original distribution's entropy, which the "
                 "single-distribution heads do not form");
@@ -861,18 +870,26 @@ struct SpecInputs {
   int32_t* sampled = nullptr;
 };
 
+// The draws from the fused logits the head wrote, then the acceptance: exact
+// match against them, or (`typical_scores` given) the typical rule with t the
+// draw at n+1.
 int sampled_accept_launches(rv_handle* h, const int32_t* draft_ids, const float* u,
                             float temperature, int B, int gamma, int32_t* sampled,
                             uint8_t* accept_mask, int32_t* accepted_len, int32_t* next_token,
                             const int32_t* ctx_in, int32_t* ctx_out, cudaStream_t s,
-                            int ctx_extra = 0) {
+                            int ctx_extra = 0, const float* typical_scores = nullptr) {
   ProfScope prof(h, RV_PROF_ACCEPT, s);
   cudaError_t e = launch_sample_fused(h->zbuf, u, B * (gamma + 1), h->cfg.vocab, temperature,
                                       sampled, s);
   h->launches += 1;
   if (e != cudaSuccess) return cuda_fail(h, e, "sampling launch");
-  e = launch_accept(draft_ids, sampled, B, gamma, accept_mask, accepted_len, next_token, ctx_in,
-                    ctx_out, s, ctx_extra);
+  // (the typical kernel takes its t from the array in the argmax place)
+  e = typical_scores
+          ? launch_accept_typical(draft_ids, typical_scores, sampled, B, gamma, h->accept_log_eps,
+                                  h->accept_log_delta, accept_mask, accepted_len, next_token,
+                                  ctx_in, ctx_out, s, ctx_extra)
+          : launch_accept(draft_ids, sampled, B, gamma, accept_mask, accepted_len, next_token,
+                          ctx_in, ctx_out, s, ctx_extra);
   h->launches += 1;
   return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "accept launch");
 }
@@ -916,8 +933,11 @@ int step_impl(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
     AcceptArgs ac{accept_mask, accepted_len,       next_token,         ctx_in,
                   ctx_out,     h->accept_mode,     h->accept_log_eps,  h->accept_log_delta,
                   lead};
+    const bool typical_t = h->accept_mode == RV_ACCEPT_TYPICAL_SAMPLED;
     if (spec && spec->sampled_exact && h->zsub) {
-      const SubtileRequest sr{spec->u, 1.f / spec->temperature, spec->sampled, ac};
+      AcceptArgs sac = ac;  // the kept drafts: exact match with the draws, or typical
+      sac.mode = typical_t ? RV_ACCEPT_TYPICAL : RV_ACCEPT_EXACT;
+      const SubtileRequest sr{spec->u, 1.f / spec->temperature, spec->sampled, sac};
       return head_impl(h, hidden, w_head, draft_ids, B, gamma, R, alpha, scores, argmax, margin,
                        do_pack ? &pk : nullptr, nullptr, s, &sr);
     }
@@ -926,7 +946,7 @@ int step_impl(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
     if (r == RV_OK && spec && spec->sampled_exact) {
       r = sampled_accept_launches(h, draft_ids, spec->u, spec->temperature, B, gamma,
                                   spec->sampled, accept_mask, accepted_len, next_token, ctx_in,
-                                  ctx_out, s, lead);
+                                  ctx_out, s, lead, typical_t ? scores : nullptr);
     } else if (r == RV_OK && spec) {
       ProfScope prof(h, RV_PROF_ACCEPT, s);
       cudaError_t e2 = launch_accept_speculative(draft_ids, spec->q, spec->r, spec->u, scores,
@@ -969,9 +989,9 @@ extern "C" RV_API int rv_verify_step(
   if (h->accept_mode == RV_ACCEPT_SPECULATIVE)
     return fail(h, RV_ERR_INVALID_ARG,
                 "speculative sampling needs the draft distributions: use rv_verify_step_speculative");
-  if (h->accept_mode == RV_ACCEPT_SAMPLED)
+  if (h->accept_mode == RV_ACCEPT_SAMPLED || h->accept_mode == RV_ACCEPT_TYPICAL_SAMPLED)
     return fail(h, RV_ERR_INVALID_ARG,
-                "sampled exact match needs the uniforms: use rv_verify_step_sampled");
+                "a sampled next token needs the uniforms: use rv_verify_step_sampled");
   return step_impl(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, prompt_ids,
                    prefix_ids, ctx_in, B, gamma, n_prompt, n_prefix, alpha, block_ids, pos_ids,
                    attn_out, scores, argmax, margin, accept_mask, accepted_len, next_token, ctx_out,
@@ -988,7 +1008,8 @@ extern "C" RV_API int rv_verify_step_pending(
     void* stream) {
   if (!h) return RV_ERR_INVALID_ARG;
   h->err.clear();
-  if (h->accept_mode == RV_ACCEPT_SPECULATIVE || h->accept_mode == RV_ACCEPT_SAMPLED)
+  if (h->accept_mode == RV_ACCEPT_SPECULATIVE || h->accept_mode == RV_ACCEPT_SAMPLED ||
+      h->accept_mode == RV_ACCEPT_TYPICAL_SAMPLED)
     return fail(h, RV_ERR_INVALID_ARG,
                 "the pending-token step runs the exact-match or typical rule of the handle");
   if (B > 0 && !pending_ids)
@@ -1031,8 +1052,11 @@ extern "C" RV_API int rv_verify_step_sampled(
     int32_t* ctx_out, void* stream) {
   if (!h) return RV_ERR_INVALID_ARG;
   h->err.clear();
-  if (h->accept_mode != RV_ACCEPT_SAMPLED || !h->zbuf)
-    return fail(h, RV_ERR_INVALID_ARG, "call rv_set_acceptance(RV_ACCEPT_SAMPLED) on the handle first");
+  if ((h->accept_mode != RV_ACCEPT_SAMPLED && h->accept_mode != RV_ACCEPT_TYPICAL_SAMPLED) ||
+      !h->zbuf)
+    return fail(h, RV_ERR_INVALID_ARG,
+                "call rv_set_acceptance(RV_ACCEPT_SAMPLED or RV_ACCEPT_TYPICAL_SAMPLED) on the "
+                "handle first");
   if (!(temperature > 0.f) || !std::isfinite(temperature))
     return fail(h, RV_ERR_INVALID_ARG, "temperature must be finite and > 0");
   if (B > 0 && (!u_uniform || !sampled))

@@ -154,8 +154,9 @@ cudaError_t launch_sample_fused(const float* z, const float* u, int P, int V, fl
 // the 32-row subtile from the sums, then the row inside it from that
 // subtile's fused logits, recomputed from the head's operands (w rows, the
 // position's hsel rows as `launch_prep` laid them out for plan `pl`).  With
-// `acc`, the last of a sequence's positions to finish runs the exact-match
-// acceptance on the draws (a ticket per sequence in `tickets`, zero between
+// `acc`, the last of a sequence's positions to finish runs the acceptance: exact
+// match against the draws, or with acc->mode == RV_ACCEPT_TYPICAL the typical
+// rule on `scores`, with t the draw at n+1 (a ticket per sequence in `tickets`, zero between
 // launches).  One CTA per position.
 struct SubtileDraw {
   const float2* zsub;
@@ -171,6 +172,7 @@ struct SubtileDraw {
   int32_t* xhat;        // [P]
   const int32_t* drafts;
   unsigned* tickets;
+  const float* scores;  // [P][RV_NSCORES] (the typical rule's log-probability and entropy)
 };
 cudaError_t launch_sample_subtiles(const SubtileDraw& d, const AcceptArgs* acc, cudaStream_t s);
 // Typical acceptance (Alg. 3) from the head's scores and argmax.

@@ -38,6 +38,7 @@ RV_SCORE_LOGP_FUSED, RV_SCORE_LOGP_ORIG, RV_SCORE_LOGP_REFL = 3, 4, 5
 RV_SCORE_ENT_ORIG = 6
 
 RV_ACCEPT_EXACT, RV_ACCEPT_TYPICAL, RV_ACCEPT_SPECULATIVE, RV_ACCEPT_SAMPLED = 0, 1, 2, 3
+RV_ACCEPT_TYPICAL_SAMPLED = 4
 RV_HEAD_FUSED_LOGITS, RV_HEAD_PREBLENDED, RV_HEAD_STANDARD = 0, 1, 2
 
 RV_PROF_ATTENTION, RV_PROF_HEAD_GEMM, RV_PROF_HEAD, RV_PROF_ACCEPT = 0, 1, 2, 3

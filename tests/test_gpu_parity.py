@@ -646,13 +646,17 @@ def _sampled_inputs(inp, alpha, T, seed, keep=0.7, preblended=False):
     return z, u, drafts.astype(np.int64)
 
 
-def _run_sampled(gu, inp, drafts, alpha, T, u, separate=False, preblended=False):
+def _run_sampled(gu, inp, drafts, alpha, T, u, separate=False, preblended=False, typical=None):
+    """`typical`: (eps, delta) of typical acceptance with t sampled at T."""
     import torch
     from paper_2505_18629_gb300 import rv
     wl = inp.wl
     B, g = wl.B, wl.gamma
     h = gu.make_handle(wl)
-    rv.rv_set_acceptance(h, rv.RV_ACCEPT_SAMPLED)
+    if typical is not None:
+        rv.rv_set_acceptance(h, rv.RV_ACCEPT_TYPICAL_SAMPLED, *typical)
+    else:
+        rv.rv_set_acceptance(h, rv.RV_ACCEPT_SAMPLED)
     if preblended:
         rv.rv_set_head_mode(h, rv.RV_HEAD_PREBLENDED)
     du = gu.to_dev(u)
@@ -783,6 +787,46 @@ def test_sampled_exact_match_subtile_draw_layouts(gu, name):
         z, u, drafts = _sampled_inputs(inp, ALPHA, T, 97, preblended=pre)
         _check_sampled(inp, z, u, drafts, T, _run_sampled(gu, inp, drafts, ALPHA, T, u,
                                                            preblended=pre))
+
+
+@pytest.mark.parametrize("name,T", [("small", 0.8), ("pairs", 0.3), ("tiny", 1.0)])
+def test_typical_acceptance_sampled_t(gu, name, T):
+    # Alg. 3 with t ~ p_{n+1} at temperature T (rv_verify_step_sampled on a
+    # handle in RV_ACCEPT_TYPICAL_SAMPLED mode): the one-CTA head, the CTA-pair
+    # head and the fp32 head (which writes the fused logits)
+    import oracle.rv_oracle as orc
+    from paper_2505_18629_gb300 import synth
+    wl = {"small": _wl(B=6, gamma=5, seed=73),
+          "pairs": _wl(B=14, gamma=8, R=8, V=777, H=256, ctx=(10, 60), seed=74),
+          "tiny": synth.WORKLOADS["tiny"]}[name]
+    inp = synth.generate(wl)
+    drafts = gu.oracle_drafts(inp, ALPHA)
+    eps, delta = _typical_params(gu, inp, drafts, ALPHA, "delta")
+    head = orc.verify_head(inp.W, inp.hidden, drafts, wl.gamma, wl.R, ALPHA)
+    u = np.random.default_rng(75).uniform(0, 1, (wl.B, wl.gamma + 1)).astype(np.float32)
+    acc_o, n_o, t_o, gap, cdf_gap = orc.typical_accept_sampled(
+        drafts, head["logp_fused"], head["ent_orig"], head["z"], eps, delta, T,
+        u.astype(np.float64))
+    xs, acc, n, t, co, _, status = _run_sampled(gu, inp, drafts, ALPHA, T, u,
+                                                typical=(eps, delta))
+    assert status == 0
+    low = np.abs(gap) < gu.MARGIN_EPS
+    assert not ((acc != acc_o) & ~low).any()
+    # n follows the GPU's own mask; t is the GPU's own draw at n+1
+    for b in range(wl.B):
+        nb = wl.gamma
+        for i in range(wl.gamma):
+            if not acc[b, i]:
+                nb = i
+                break
+        assert n[b] == nb and t[b] == xs[b, n[b]] and co[b] == inp.ctx_lens[b] + n[b]
+    same = (n == n_o)
+    assert same.mean() >= 0.5
+    # where n agrees, t is the oracle's draw unless u[b, n] sits on a CDF boundary
+    for b in np.flatnonzero(same):
+        if t[b] != t_o[b]:
+            assert cdf_gap[b] < SPEC_TOL, f"sequence {b}: t {t[b]} vs {t_o[b]}"
+    assert 0 < acc_o.sum() < acc_o.size
 
 
 # ------------------------------------------------------------------ pending-token block

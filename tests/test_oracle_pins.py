@@ -444,6 +444,36 @@ def test_typical_threshold_worked_example():
     assert acc[0, 0] and abs(gap[0, 0] - (math.log(0.05) - (math.log(0.3) - 3.0))) < 1e-12
 
 
+def test_typical_accept_sampled_t_law_and_greedy_limit():
+    # Alg. 3 with t ~ p_{n+1} at temperature T: over a fine grid of uniforms
+    # the frequency of each t is softmax(z_{n+1} / T) (the inverse CDF's law);
+    # the kept drafts and n are typical_accept's; T -> 0 gives its greedy t
+    B, gamma, V = 2, 3, 5
+    z = np.array([[[0.0, 1.0, 2.0, 0.5, -1.0]] * (gamma + 1),
+                  [[3.0, 0.0, 0.0, 2.9, 1.0]] * (gamma + 1)])
+    logp = np.log(np.array([[0.5, 0.01, 0.4], [0.3, 0.3, 0.3]]))
+    H = np.full((B, gamma + 1), 1.0)
+    acc_g, n_g, t_g, _ = orc.typical_accept(np.zeros((B, gamma)), logp, H,
+                                            z.argmax(axis=-1), 0.2, 0.3)
+    for T in (1.0, 0.5):
+        K = 20000
+        counts = np.zeros((B, V))
+        for k in range(K):
+            u = np.full((B, gamma + 1), (k + 0.5) / K)
+            acc, n, t, _, _ = orc.typical_accept_sampled(np.zeros((B, gamma)), logp, H, z, 0.2, 0.3,
+                                                         T, u)
+            assert (acc == acc_g).all() and (n == n_g).all()
+            counts[np.arange(B), t] += 1
+        for b in range(B):
+            zt = z[b, n_g[b]] / T
+            p = np.exp(zt - zt.max())
+            p /= p.sum()
+            np.testing.assert_allclose(counts[b] / K, p, atol=2.0 / K)
+    u = np.full((B, gamma + 1), 0.37)
+    _, _, t0, _, _ = orc.typical_accept_sampled(np.zeros((B, gamma)), logp, H, z, 0.2, 0.3, 1e-6, u)
+    assert (t0 == t_g).all()
+
+
 def test_typical_accept_limits_and_monotonicity():
     rng = np.random.default_rng(13)
     B, gamma = 64, 6

@@ -563,130 +563,205 @@ cudaError_t launch_accept_speculative(const int32_t* drafts, const float* q, con
 }
 
 // ---------------------------------------------------------------- sampled target tokens (Alg. 2)
-// One CTA per position (b, i), i = 1..gamma+1: the target's token at
-// temperature T, x^_i ~ softmax(z_i / T), drawn by inverse CDF with the
-// position's uniform u: the smallest v whose cumulative weight
-// w_v = exp((z_i[v] - max z_i) / T) exceeds u * sum(w).  Pass 1 streams the
-// row once for (max, sum) (each thread an online pair over a strided, coalesced
-// range); pass 2 walks the row in order, 4 consecutive tokens per thread and
-// SAMP_THREADS * 4 tokens per tile: a block-wide exclusive scan of the
-// threads' weights gives each thread its cumulative range, and the one whose
-// range holds the target walks its 4 tokens.  The ranges of one tile are
-// gapless (each boundary is written once, to shared memory, and read by both
-// neighbours), so the target falls in exactly one range or past the last.
-constexpr int SAMP_THREADS = 512;
-constexpr int SAMP_PER = 4;
-constexpr int SAMP_TILE = SAMP_THREADS * SAMP_PER;
-
-__global__ void __launch_bounds__(SAMP_THREADS)
-    sample_fused_kernel(const float* __restrict__ z, const float* __restrict__ u, int V,
-                        float inv_t, int32_t* __restrict__ xhat) {
-  constexpr int NW = SAMP_THREADS / 32;
-  __shared__ float s_m[NW], s_s[NW];
-  __shared__ float s_wtot[NW];
-  __shared__ float s_lo[SAMP_THREADS + 1];
-  __shared__ float s_max, s_target;
-  __shared__ int s_t, s_last;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const long long prow = blockIdx.x;
-  const float* row = z + prow * V;
-  // pass 1: max and sum of exp((z - max) / T)
-  float m = NEG_INF, sm = 0.f;
-  for (int v = tid; v < V; v += SAMP_THREADS) {
-    const float x = row[v] * inv_t;
-    if (x > m) {
-      sm = sm * expf(m - x) + 1.f;
-      m = x;
-    } else {
-      sm += expf(x - m);
-    }
+// A cluster of CL CTAs per position (b, i), i = 1..gamma+1: the target's
+// token at temperature T, x^_i ~ softmax(z_i / T), drawn by inverse CDF with
+// the position's uniform u: the smallest v whose cumulative weight
+// w_v = exp((z_i[v] - max z_i) / T) exceeds u * sum(w).  CTA c owns the c-th
+// of CL slices of the row, as in accept_speculative_kernel: the slices'
+// maxima are exchanged first (every CTA then holds max z_i), then their
+// totals, and the CTA whose slice holds the target finds the token.
+__device__ __forceinline__ float samp_round(const float* zrow, float M, float inv_t, int base,
+                                            int v_hi, int lane, float (&w)[SPC_E],
+                                            float (&incl)[SPC_E], int& last) {
+  float zv[SPC_E];
+#pragma unroll
+  for (int j = 0; j < SPC_E; ++j) {
+    const int v = base + 32 * j;
+    zv[j] = v < v_hi ? __ldg(zrow + v) : NEG_INF;
   }
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1)
-    lse_merge(m, sm, __shfl_xor_sync(0xffffffffu, m, o), __shfl_xor_sync(0xffffffffu, sm, o));
-  if (lane == 0) {
-    s_m[warp] = m;
-    s_s[warp] = sm;
+  for (int j = 0; j < SPC_E; ++j) {
+    w[j] = zv[j] == NEG_INF ? 0.f : expf((zv[j] - M) * inv_t);
+    incl[j] = w[j];
+    if (w[j] > 0.f) last = base + 32 * j;
   }
-  __syncthreads();
-  if (warp == 0) {
-    m = lane < NW ? s_m[lane] : NEG_INF;
-    sm = lane < NW ? s_s[lane] : 0.f;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1)
-      lse_merge(m, sm, __shfl_xor_sync(0xffffffffu, m, o), __shfl_xor_sync(0xffffffffu, sm, o));
-    if (lane == 0) {
-      s_max = m;
-      s_target = u[prow] * sm;
-      s_t = -1;
-      s_last = -1;
+  for (int o = 1; o < 32; o <<= 1) {
+#pragma unroll
+    for (int j = 0; j < SPC_E; ++j) {
+      const float y = __shfl_up_sync(0xffffffffu, incl[j], o);
+      if (lane >= o) incl[j] += y;
     }
   }
-  __syncthreads();
-  const float M = s_max, target = s_target;
-  // pass 2: the inverse CDF, tile by tile in vocabulary order
-  float run = 0.f;  // cumulative weight before this tile (same value in every thread)
-  for (int t0 = 0; t0 < V; t0 += SAMP_TILE) {
-    const int v0 = t0 + tid * SAMP_PER;
-    float w[SAMP_PER];
-    float part = 0.f;
+  float carry = 0.f;
 #pragma unroll
-    for (int j = 0; j < SAMP_PER; ++j) {
-      w[j] = v0 + j < V ? expf(row[v0 + j] * inv_t - M) : 0.f;
-      part += w[j];
-    }
-    float incl = part;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const float y = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += y;
-    }
-    // exclusive prefix: exactly the previous lane's inclusive value, so the
-    // boundaries never decrease
-    float excl = __shfl_up_sync(0xffffffffu, incl, 1);
-    if (lane == 0) excl = 0.f;
-    if (lane == 31) s_wtot[warp] = incl;
-    __syncthreads();
-    float woff = 0.f;  // exclusive prefix of the warp totals
-    for (int k = 0; k < warp; ++k) woff += s_wtot[k];
-    s_lo[tid] = run + (woff + excl);
-    if (tid == SAMP_THREADS - 1) s_lo[SAMP_THREADS] = run + (woff + incl);
-    __syncthreads();
-    const float lo = s_lo[tid], hi = s_lo[tid + 1];
-    const unsigned live = __ballot_sync(0xffffffffu, part > 0.f);  // last weighted range
-    if (live != 0u && lane == 31 - __clz(live)) atomicMax(&s_last, v0);
-    if (target >= lo && target < hi) {
-      float c = lo;
-      int pick = -1;
-#pragma unroll
-      for (int j = 0; j < SAMP_PER; ++j) {
-        c += w[j];
-        if (w[j] > 0.f) pick = v0 + j;
-        if (w[j] > 0.f && c > target) break;
-      }
-      atomicMax(&s_t, pick);
-    }
-    run = s_lo[SAMP_THREADS];
-    __syncthreads();
-    if (s_t >= 0) break;
-  }
-  if (tid == 0) {
-    int t = s_t;
-    if (t < 0) {
-      // u * sum(w) at or past the rounded total: the last token with weight
-      t = s_last >= 0 ? s_last : 0;
-      const int vmax = min(V, t + SAMP_PER);
-      for (int v = t; v < vmax; ++v)
-        if (expf(row[v] * inv_t - M) > 0.f) t = v;
-    }
-    xhat[prow] = t;
-  }
+  for (int j = 0; j < SPC_E; ++j) carry = carry + __shfl_sync(0xffffffffu, incl[j], 31);
+  return carry;
 }
 
+template <int CL>
+__global__ void __launch_bounds__(SPC_THREADS)
+    sample_fused_kernel(const float* __restrict__ z, const float* __restrict__ u, int V,
+                        float inv_t, int32_t* __restrict__ xhat) {
+  constexpr int NW = SPC_THREADS / 32;
+  __shared__ float s_max[CL];   // every slice's max z (written by its CTA)
+  __shared__ float s_wc[CL];    // every slice's total weight
+  __shared__ int s_lastc[CL];   // every slice's last token of positive weight
+  __shared__ float s_wtot[NW];
+  __shared__ int s_last;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  uint32_t rank;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(rank));
+  const long long prow = blockIdx.x / CL;
+  const float* const row = z + prow * V;
+  // (other CTAs' shared memory is written only after every CTA has started)
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+  const int Vc = (V + CL - 1) / CL;
+  const int v_lo = min(V, static_cast<int>(rank) * Vc), v_hi = min(V, v_lo + Vc);
+  const int base0 = v_lo + SPC_WARP * warp + lane;
+  // this slice's max, to every CTA of the cluster
+  float m = NEG_INF;
+  for (int r0 = 0; r0 < v_hi - v_lo; r0 += SPC_ROUND)
+#pragma unroll
+    for (int j = 0; j < SPC_E; ++j) {
+      const int v = base0 + r0 + 32 * j;
+      if (v < v_hi) m = fmaxf(m, __ldg(row + v));
+    }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  if (lane == 0) s_wtot[warp] = m;
+  __syncthreads();
+  if (tid == 0) {
+    for (int k = 1; k < NW; ++k) m = fmaxf(m, s_wtot[k]);
+    s_wtot[0] = m;
+  }
+  __syncthreads();
+  m = s_wtot[0];
+  asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+  if (tid < CL) {
+    uint32_t d0;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;"
+                 : "=r"(d0) : "r"(smem_u32(&s_max[rank])), "r"(tid));
+    asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(d0), "f"(m) : "memory");
+  }
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                   : "memory");
+  float M = s_max[0];
+  for (int c = 1; c < CL; ++c) M = fmaxf(M, s_max[c]);
+  // this slice's weights and total, in the scan's own arithmetic
+  float w[SPC_E], incl[SPC_E];
+  float run = 0.f, wt_first = 0.f;
+  int last = -1;
+  const bool one_round = v_hi - v_lo <= SPC_ROUND;
+  for (int r0 = 0; r0 < v_hi - v_lo; r0 += SPC_ROUND) {
+    const float wt = samp_round(row, M, inv_t, base0 + r0, v_hi, lane, w, incl, last);
+    if (r0 == 0) wt_first = wt;
+    __syncthreads();
+    if (lane == 0) s_wtot[warp] = wt;
+    __syncthreads();
+    float total = 0.f;
+    for (int k = 0; k < NW; ++k) total = total + s_wtot[k];
+    run = run + total;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) last = max(last, __shfl_xor_sync(0xffffffffu, last, o));
+  if (tid == 0) s_last = -1;
+  __syncthreads();
+  if (lane == 0 && last >= 0) atomicMax(&s_last, last);
+  __syncthreads();
+  if (tid < CL) {
+    uint32_t d0, d1;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;"
+                 : "=r"(d0) : "r"(smem_u32(&s_wc[rank])), "r"(tid));
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;"
+                 : "=r"(d1) : "r"(smem_u32(&s_lastc[rank])), "r"(tid));
+    asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(d0), "f"(run) : "memory");
+    asm volatile("st.shared::cluster.s32 [%0], %1;" ::"r"(d1), "r"(s_last) : "memory");
+  }
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                   : "memory");
+  float W = 0.f;
+  for (int c = 0; c < CL; ++c) W = W + s_wc[c];
+  const float target = u[prow] * W;
+  float P = 0.f, P_owner = 0.f;
+  int owner = -1, last_c = -1;
+  for (int c = 0; c < CL; ++c) {
+    const float Pn = P + s_wc[c];
+    if (owner < 0 && target >= P && target < Pn) {
+      owner = c;
+      P_owner = P;
+    }
+    if (s_wc[c] > 0.f) last_c = c;
+    P = Pn;
+  }
+  if (owner < 0) {  // u * W at or past the rounded total: the last token with weight
+    if (static_cast<int>(rank) == max(last_c, 0) && tid == 0)
+      xhat[prow] = last_c >= 0 ? s_lastc[last_c] : 0;
+    return;
+  }
+  if (static_cast<int>(rank) != owner) return;
+  run = 0.f;
+  if (tid == 0) s_last = -1;  // reused: the token found
+  for (int r0 = 0; r0 < v_hi - v_lo; r0 += SPC_ROUND) {
+    int dummy = -1;
+    const float wt = one_round ? wt_first
+                               : samp_round(row, M, inv_t, base0 + r0, v_hi, lane, w, incl, dummy);
+    __syncthreads();
+    if (lane == 0) s_wtot[warp] = wt;
+    __syncthreads();
+    float woff = 0.f, total = 0.f;
+    for (int k = 0; k < NW; ++k) {
+      if (k == warp) woff = total;
+      total = total + s_wtot[k];
+    }
+    float carry = 0.f;
+#pragma unroll
+    for (int j = 0; j < SPC_E; ++j) {
+      const float ex = __shfl_up_sync(0xffffffffu, incl[j], 1);
+      const float tj = __shfl_sync(0xffffffffu, incl[j], 31);
+      const float lo = P_owner + (run + (woff + (carry + (lane == 0 ? 0.f : ex))));
+      const float hi = P_owner + (run + (woff + (carry + incl[j])));
+      if (target >= lo && target < hi) s_last = base0 + r0 + 32 * j;
+      carry = carry + tj;
+    }
+    run = run + total;
+    __syncthreads();
+    if (s_last >= 0) break;
+  }
+  if (tid == 0) xhat[prow] = s_last >= 0 ? s_last : s_lastc[owner];
+}
+
+template <int CL>
+static cudaError_t launch_sample_fused_cl(const float* z, const float* u, int P, int V,
+                                          float temperature, int32_t* xhat, cudaStream_t s) {
+  static bool configured = false;
+  if (!configured) {
+    const cudaError_t e = cudaFuncSetAttribute(sample_fused_kernel<CL>,
+                                               cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(P * CL, 1, 1);
+  cfg.blockDim = dim3(SPC_THREADS, 1, 1);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = CL;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, sample_fused_kernel<CL>, z, u, V, 1.f / temperature, xhat);
+}
+
+// A few positions: 16 CTAs each (the shortest chain per position); many: 4,
+// so that the clusters of all positions fit the GPU at once.
 cudaError_t launch_sample_fused(const float* z, const float* u, int P, int V, float temperature,
                                 int32_t* xhat, cudaStream_t s) {
-  sample_fused_kernel<<<P, SAMP_THREADS, 0, s>>>(z, u, V, 1.f / temperature, xhat);
-  return cudaGetLastError();
+  if (P <= 0) return cudaSuccess;
+  return P <= 16 ? launch_sample_fused_cl<16>(z, u, P, V, temperature, xhat, s)
+                 : launch_sample_fused_cl<4>(z, u, P, V, temperature, xhat, s);
 }
 
 // ---------------------------------------------------------------- draws from subtile sums (Alg. 2)

@@ -107,7 +107,10 @@ int head_tc_stages(int N, int pairs, size_t smem_limit) {
   return std::max(2, std::min(head_tc_max_stages(N, pairs, smem_limit), std::max(4, want)));
 }
 
-template <int EPI>
+// SUB: the epilogue also stores the subtile sums of sampled exact match (its
+// own instantiation, so that the other modes carry none of its registers: the
+// batch-1 attention CTA shares the SM with this one only within a register budget).
+template <int EPI, bool SUB>
 __global__ void __launch_bounds__(ht_threads(EPI), 1)
     head_tc_kernel(const __grid_constant__ CUtensorMap tm_w,
                    const __grid_constant__ CUtensorMap tm_w16,
@@ -320,7 +323,7 @@ __global__ void __launch_bounds__(ht_threads(EPI), 1)
       const uint32_t trow =
           tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(slot * p.N);
       float* const zout = p.zout ? p.zout + static_cast<long long>(pair0) * p.V : nullptr;
-      float2* const zsub = p.zsub ? p.zsub + static_cast<long long>(pair0) * p.n_sub : nullptr;
+      float2* const zsub = SUB ? p.zsub + static_cast<long long>(pair0) * p.n_sub : nullptr;
       for (int g8 = 8 * half; g8 < npairs; g8 += 8 * (EPI / 4)) {
         if (p.zonly) {
           float z[8];
@@ -375,19 +378,23 @@ __global__ void __launch_bounds__(ht_threads(EPI), 1)
 // The maximum shared-memory carveout lets the attention kernel's CTAs share an
 // SM with this kernel's (the SM is otherwise configured just large enough for
 // whichever kernel arrives first).
-template <int EPI>
+template <int EPI, bool SUB>
 static cudaError_t head_tc_configure_one(size_t smem_bytes) {
-  cudaError_t e = cudaFuncSetAttribute(head_tc_kernel<EPI>,
+  cudaError_t e = cudaFuncSetAttribute(head_tc_kernel<EPI, SUB>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem_bytes));
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(head_tc_kernel<EPI>, cudaFuncAttributePreferredSharedMemoryCarveout,
+  return cudaFuncSetAttribute(head_tc_kernel<EPI, SUB>,
+                              cudaFuncAttributePreferredSharedMemoryCarveout,
                               cudaSharedmemCarveoutMaxShared);
 }
 
 cudaError_t head_tc_configure(size_t smem_bytes) {
-  cudaError_t e = head_tc_configure_one<4>(smem_bytes);
-  return e != cudaSuccess ? e : head_tc_configure_one<8>(smem_bytes);
+  cudaError_t e = head_tc_configure_one<4, false>(smem_bytes);
+  if (e == cudaSuccess) e = head_tc_configure_one<8, false>(smem_bytes);
+  if (e == cudaSuccess) e = head_tc_configure_one<4, true>(smem_bytes);
+  if (e == cudaSuccess) e = head_tc_configure_one<8, true>(smem_bytes);
+  return e;
 }
 
 static uint32_t tmem_cols_for(int N) {
@@ -447,8 +454,13 @@ cudaError_t launch_head_tc(const HeadArgs& a, const HeadPlan& pl, const HeadTcLa
   }
   cfg.attrs = attr;
   cfg.numAttrs = na;
-  if (epi == 4) return cudaLaunchKernelEx(&cfg, head_tc_kernel<4>, l.tm_w, l.tm_w16, l.tm_h, p);
-  return cudaLaunchKernelEx(&cfg, head_tc_kernel<8>, l.tm_w, l.tm_w16, l.tm_h, p);
+  if (a.zsub != nullptr) {
+    if (epi == 4)
+      return cudaLaunchKernelEx(&cfg, head_tc_kernel<4, true>, l.tm_w, l.tm_w16, l.tm_h, p);
+    return cudaLaunchKernelEx(&cfg, head_tc_kernel<8, true>, l.tm_w, l.tm_w16, l.tm_h, p);
+  }
+  if (epi == 4) return cudaLaunchKernelEx(&cfg, head_tc_kernel<4, false>, l.tm_w, l.tm_w16, l.tm_h, p);
+  return cudaLaunchKernelEx(&cfg, head_tc_kernel<8, false>, l.tm_w, l.tm_w16, l.tm_h, p);
 }
 
 }  // namespace rv

@@ -51,9 +51,9 @@ FALLBACK_BF16_TFLOPS = 1900.0
 # dram__bytes_write.sum` on the workload named (see profiles/), valid only while
 # the kernel sources hash to `src_sha`.
 NCU_TRAFFIC = {
-    "llama3-8b-b1": {"bytes": 1051018496 + 2967296, "src_sha": "70d62aa259fa6653",
+    "llama3-8b-b1": {"bytes": 1050909696 + 2821120, "src_sha": "87af7aa7e3f64385",
                      "summary": "profiles/head_tc_llama3-8b-b1.md"},
-    "llama3-8b-b16": {"bytes": 1053353216 + 6040832, "src_sha": "70d62aa259fa6653",
+    "llama3-8b-b16": {"bytes": 1053354240 + 6161920, "src_sha": "87af7aa7e3f64385",
                       "summary": "profiles/head_tc2_llama3-8b-b16.md"},
 }
 
@@ -683,10 +683,11 @@ def measure_workload(wl, args, dev, world, rank, clocks):
         n_run_in += 1
         if n_run_in % 64 == 0:
             torch.cuda.synchronize(dev)
-    # An event pair around the row gather + LM head (+ its merge) leaves their
-    # programmatic overlap intact; the head time it gives includes the short
-    # gather.  It is recorded on every PROF_EVERY-th timed step (each event
-    # record costs the step a few microseconds of GPU time).
+    # Event pairs around the LM-head kernel's own launch (the roofline's
+    # duration) and around the row gather + LM head + merge (context: at
+    # batch 16 the merge may wait for SMs the concurrent attention holds).
+    # They are recorded on every PROF_EVERY-th timed step (each event record
+    # costs the step a few microseconds of GPU time).
     PROF_EVERY = 4
     launches0 = rv.rv_launch_count(h)
     if world > 1:
@@ -699,7 +700,7 @@ def measure_workload(wl, args, dev, world, rank, clocks):
         sampled = i % PROF_EVERY == PROF_EVERY - 1 or (args.steps < PROF_EVERY and
                                                        i == args.steps - 1)
         if sampled:
-            rv.rv_profile_enable(h, 1 << rv.RV_PROF_HEAD)
+            rv.rv_profile_enable(h, (1 << rv.RV_PROF_HEAD) | (1 << rv.RV_PROF_HEAD_GEMM))
         step()
         if sampled:
             rv.rv_profile_enable(h, 0)
@@ -710,7 +711,8 @@ def measure_workload(wl, args, dev, world, rank, clocks):
         dist.barrier()
     launches = rv.rv_launch_count(h) - launches0
     ms_total = e0.elapsed_time(e1)
-    head_ms, head_n = rv.rv_profile_read(h, rv.RV_PROF_HEAD)
+    region_ms, region_n = rv.rv_profile_read(h, rv.RV_PROF_HEAD)
+    head_ms, head_n = rv.rv_profile_read(h, rv.RV_PROF_HEAD_GEMM)
     rv.rv_profile_enable(h, 0)
     # Breakdown run (after the timed region, not part of `value`): the LM head
     # and the attention each alone (their own entry points, one after the
@@ -779,7 +781,8 @@ def measure_workload(wl, args, dev, world, rank, clocks):
     n_rows = (1 if args.head_mode == "preblended" else 2) * (g + 1) * B
     head_bytes = wl.V * wl.H * 2 + n_rows * wl.H * 2
     head_flops = 2.0 * n_rows * wl.H * wl.V
-    head_avg_s = head_ms * 1e-3 / max(head_n, 1)       # timed region: gather + LM head
+    head_avg_s = head_ms * 1e-3 / max(head_n, 1)       # timed region: the LM-head kernel
+    region_avg_s = region_ms * 1e-3 / max(region_n, 1)  # timed region: gather + head + merge
     gemm_avg_s = gemm_ms * 1e-3 / max(gemm_n, 1)       # breakdown run: LM head alone
     achieved_gbs = head_bytes / head_avg_s / 1e9
     achieved_tf = head_flops / head_avg_s / 1e12
@@ -802,9 +805,10 @@ def measure_workload(wl, args, dev, world, rank, clocks):
                 "peak_kind": "sustained bf16 (the kernel inside the step)",
                 "peak_kernel_alone": tf_burst}
     roof.update({"kernel": "LM head (head_tc_kernel; head_tc2_kernel on CTA pairs from N >= 96 "
-                           "hidden rows per chunk): GEMM + online log-softmax (+ merge), timed with the "
-                           f"row-gather launch before it by an event pair on every {PROF_EVERY}th "
-                           "timed step",
+                           "hidden rows per chunk): GEMM + online log-softmax (+ merge in its last "
+                           "CTA at small batches), timed by an event pair around its launch on "
+                           f"every {PROF_EVERY}th timed step",
+                 "head_region_us": region_avg_s * 1e6,
                  "peak_source": f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured"
                  else "fallback", "algorithmic_bytes": head_bytes,
                  "algorithmic_flops": head_flops, "avg_us": head_avg_s * 1e6, "launches": head_n,

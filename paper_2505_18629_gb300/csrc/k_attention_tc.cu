@@ -59,6 +59,10 @@ constexpr int TC_STAGES = 3;     // K/V ring depth
 constexpr int TC_THREADS = 192;  // producer, MMA, 4 softmax warps
 constexpr int TC_IRING = 4;      // item ring between the producer and the consumers
 constexpr float TC_RESCALE_LOG2 = 8.f;
+// Key chunks are sized for about this many items per SM at capacity; the
+// partial-result slots of the workspace (attn_tc_max_slots) are sized from the
+// same number, so the two cannot disagree.
+constexpr int TC_ITEMS_PER_SM = 4;
 
 constexpr uint32_t TC_KV_BYTES = TC_KT * TC_D * 2;  // 32 KB: two halves of [128 keys][128 B]
 constexpr uint32_t TC_Q_BYTES = TC_M * TC_D * 2;    // 32 KB: two halves of [128 rows][128 B]
@@ -719,8 +723,14 @@ AttnTcPlan attn_tc_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms) {
   p.rows = Lb * G;
   p.n_rg = (p.rows + TC_M - 1) / TC_M;
   const long long groups = static_cast<long long>(B) * Hkv * p.n_rg;
-  // chunks sized for about four items per SM when every sequence is full
-  long long ch = (groups * Cmax + 4LL * num_sms - 1) / (4LL * num_sms);
+  // chunks sized for about four items per SM when every sequence is full.
+  // Fewer, longer items run faster alone where there are many groups and
+  // short caches (70B B=32: 160.8 us at two items per SM against 167.8 us), but
+  // in the step, where the attention takes SMs as the LM head's CTAs finish,
+  // the finer items balance the late-starting CTAs (70B B=32 step 805-815 us
+  // at four against 870 us at two).
+  const long long per_sm = static_cast<long long>(TC_ITEMS_PER_SM) * num_sms;
+  long long ch = (groups * Cmax + per_sm - 1) / per_sm;
   ch = std::max<long long>(256, (ch + TC_KT - 1) / TC_KT * TC_KT);
   ch = std::min<long long>(ch, (Cmax + TC_KT - 1) / TC_KT * TC_KT + TC_KT);
   p.chunk = static_cast<int>(ch);
@@ -741,9 +751,10 @@ size_t attn_tc_smem_max(int max_batch) {
 }
 
 int attn_tc_max_slots(int max_batch, int Lb_max, int Hq, int Hkv, int num_sms) {
-  // chunk >= groups * Cmax / (4 * SMs), or one chunk per group: slots <= 4 * SMs + groups
+  // chunk >= groups * Cmax / (TC_ITEMS_PER_SM * SMs), or one chunk per group:
+  // slots <= TC_ITEMS_PER_SM * SMs + groups
   const int n_rg = (Lb_max * (Hq / Hkv) + TC_M - 1) / TC_M;
-  return 4 * num_sms + max_batch * Hkv * n_rg;
+  return TC_ITEMS_PER_SM * num_sms + max_batch * Hkv * n_rg;
 }
 
 cudaError_t attn_tc_configure(size_t smem_bytes) {
@@ -799,6 +810,7 @@ bool attn_tc_encode(PFN_cuTensorMapEncodeTiled_v12000 enc, const AttnArgs& x, At
 
 cudaError_t launch_attention_tc(const AttnArgs& x, const AttnTcPlan& p, const AttnTcMaps& m,
                                 const AttnTcScratch& sc, cudaStream_t s) {
+  if (p.slots > sc.max_slots) return cudaErrorInvalidValue;  // the partials would not fit
   TcArgs a;
   a.q = static_cast<const __nv_bfloat16*>(x.q);
   a.ctx = x.ctx;

@@ -338,6 +338,7 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
   h->ws.attn.part_o = reinterpret_cast<float*>(b + o_apo);
   h->ws.attn.part_ml = reinterpret_cast<float*>(b + o_aml);
   h->ws.attn.counters = reinterpret_cast<unsigned*>(b + o_act);
+  h->ws.attn.max_slots = a_slots;
   h->ws.fin_tickets = reinterpret_cast<unsigned*>(b + o_fin);
   h->ws.st_q = b + o_q;
   h->ws.st_kb = b + o_kb;

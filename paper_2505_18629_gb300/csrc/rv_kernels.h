@@ -282,6 +282,7 @@ struct AttnTcScratch {
   float* part_o;       // [slots][128][128]
   float* part_ml;      // [slots][128][2]
   unsigned* counters;  // [2], zero between launches
+  int max_slots = 0;   // slots allocated; a plan needing more is not launched
 };
 AttnTcPlan attn_tc_plan(int B, int Lb, int Hq, int Hkv, int Cmax, int num_sms);
 bool attn_tc_supported(int Hq, int Hkv, int D);

@@ -42,6 +42,7 @@ RV_ACCEPT_TYPICAL_SAMPLED = 4
 RV_HEAD_FUSED_LOGITS, RV_HEAD_PREBLENDED, RV_HEAD_STANDARD = 0, 1, 2
 
 RV_PROF_ATTENTION, RV_PROF_HEAD_GEMM, RV_PROF_HEAD, RV_PROF_ACCEPT = 0, 1, 2, 3
+RV_PROF_COUNT = 4
 
 
 class RVLibraryMissing(ImportError):

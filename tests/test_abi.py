@@ -108,3 +108,17 @@ def test_create_without_gpu_fails_cleanly(rv):
     rc = rv.lib().rv_create(ctypes.byref(cfg), ctypes.byref(out))
     assert rc in (rv.RV_ERR_CUDA, rv.RV_ERR_UNSUPPORTED)
     assert out.value is None
+
+
+def test_binding_constants_match_the_header():
+    # every integer constant of include/rv.h has the same value in the binding
+    from paper_2505_18629_gb300 import rv as rvmod
+    text = open(HEADER).read()
+    consts = {}
+    for name, val in re.findall(r"^#define\s+(RV_\w+)\s+(\(?-?\d+\)?u?)\b", text, flags=re.M):
+        consts[name] = int(val.strip("()u"))
+    assert "RV_ACCEPT_TYPICAL_SAMPLED" in consts and "RV_SCORE_ENT_ORIG" in consts
+    missing = [n for n in consts if not hasattr(rvmod, n)]
+    assert not missing, missing
+    wrong = {n: (getattr(rvmod, n), v) for n, v in consts.items() if getattr(rvmod, n) != v}
+    assert not wrong, wrong

@@ -517,14 +517,21 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             for (int i = 0; i < 32; ++i)
               if (kb + 32 * c + i > kmax) sv[c][i] = NEG_INF;
         }
-        float mx[4];
+        // row max: eight chains of three-input maxima (16 scores each)
+        float mx[8];
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
-          mx[c] = sv[c][0];
 #pragma unroll
-          for (int i = 1; i < 32; ++i) mx[c] = fmaxf(mx[c], sv[c][i]);
+          for (int e = 0; e < 2; ++e) {
+            float m = fmaxf(sv[c][e], sv[c][e + 2]);
+#pragma unroll
+            for (int i = e + 4; i < 32; i += 4) m = max3f(m, sv[c][i], sv[c][i + 2]);
+            mx[2 * c + e] = m;
+          }
         }
-        const float mt = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * a.scale_log2;
+        const float mt = max3f(max3f(mx[0], mx[1], mx[2]), max3f(mx[3], mx[4], mx[5]),
+                               fmaxf(mx[6], mx[7])) *
+                         a.scale_log2;
         float fac = 1.f;
         const bool rise = mt > m_used + TC_RESCALE_LOG2 || (m_used == NEG_INF && mt != NEG_INF);
         if (rise) {
@@ -550,21 +557,28 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           }
           tmem_st_wait();
         }
-        // P = 2^(s * scale - m), bf16, over the first half of S[sb]
+        // P = 2^(s * scale - m), bf16, over the first half of S[sb]; the
+        // exponent arguments and the row sum two scores per instruction
         const float neg_m = (m_used == NEG_INF) ? 0.f : -m_used;
-        float ls[4] = {0.f, 0.f, 0.f, 0.f};
+        const uint64_t sc2 = f32x2(a.scale_log2, a.scale_log2), nm2 = f32x2(neg_m, neg_m);
+        uint64_t ls2[2] = {f32x2(0.f, 0.f), f32x2(0.f, 0.f)};
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
           uint32_t pk[16];
 #pragma unroll
           for (int i = 0; i < 32; i += 2) {
-            const float p0 = ex2_approx(fmaf(sv[c][i], a.scale_log2, neg_m));
-            const float p1 = ex2_approx(fmaf(sv[c][i + 1], a.scale_log2, neg_m));
-            ls[c] += p0 + p1;
+            float x0, x1;
+            f32x2_split(fma_f32x2(f32x2(sv[c][i], sv[c][i + 1]), sc2, nm2), x0, x1);
+            const float p0 = ex2_approx(x0);
+            const float p1 = ex2_approx(x1);
+            ls2[c & 1] = add_f32x2(ls2[c & 1], f32x2(p0, p1));
             pk[i >> 1] = pack_bf16(p0, p1);
           }
           tmem_st16(s_col + 16 * c, pk);
         }
+        float ls[4];
+        f32x2_split(ls2[0], ls[0], ls[1]);
+        f32x2_split(ls2[1], ls[2], ls[3]);
         l = l * fac + ((ls[0] + ls[1]) + (ls[2] + ls[3]));
         tmem_st_wait();
         tc_fence_before();

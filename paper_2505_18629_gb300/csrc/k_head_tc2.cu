@@ -14,13 +14,20 @@
 // weight rows and only half of the hidden rows; every CTA gets its own 128-row
 // accumulator in its TMEM.
 //
-// Sub-groups.  The pairs of a chunk are split into H sub-groups of Ph pairs;
-// sub-group h has its own accumulator of Ns = 2 Ph columns (o of its pairs,
-// then o'), one MMA per 16-wide K step each.  Every sub-group reads the same
-// weight stage, so a chunk of up to 160 pairs (H = 2) streams each weight tile
-// into shared memory once.  The accumulators rotate through a ring of R slots
-// (R * Ns <= 512 TMEM columns, R >= H + 1): the next tile's first sub-group
-// starts in the free slot while the epilogue still reads this tile's.
+// Sub-groups.  The pairs of a chunk are split into H sub-groups of Ph[h]
+// pairs; sub-group h has its own accumulator of 2 Ph[h] columns (o of its
+// pairs, then o'), one MMA per 16-wide K step each.  Every sub-group reads the
+// same weight stage, so a chunk of up to 160 pairs (H = 2) streams each weight
+// tile into shared memory once.  Accumulator slots:
+//   ring  (H = 1, up to 128 pairs): R equal slots in turn, R >= 2, so a tile
+//         never waits for the epilogue of the tile before;
+//   split (H = 2, 129..160 pairs): two tiles' 2 x 2 Pc columns exceed TMEM's
+//         512, so sub-group 0 is small (Ph[0] = Pc - Ph[1], Ph[1] =
+//         256 - Pc pairs) and sits in one fixed slot, sub-group 1 alternates
+//         between two slots (2 Ph[0] + 4 Ph[1] = 512 columns).  The next
+//         tile's sub-group 1 starts at once; its sub-group 0 waits only until
+//         the epilogue has loaded this tile's sub-group 0 (at most three
+//         groups per warp, freed as soon as they are in registers).
 //
 // Per CTA, warp-specialised:
 //   warp 0      TMA producer: weight tile [128 x 128] + this CTA's hidden rows
@@ -75,7 +82,11 @@ constexpr int H2_MAX_R = 4;     // accumulator slots
 
 struct Head2Params {
   int V, n_kb;
-  int H, Ph, Ns, R;  // sub-groups per tile, pairs per sub-group, columns per slot, slots
+  int H, R, split;      // sub-groups per tile, slots, slot rule (0 ring, 1 split)
+  int Ph[H2_MAX_H];     // pairs of sub-group h (its columns: 2 Ph, or Ph pre-blended)
+  int pb[H2_MAX_H];     // its first pair (and first B row in each CTA) within the chunk
+  int scol[H2_MAX_R];   // first TMEM column of each slot
+  int b_rows;           // B rows per CTA per stage (the chunk's half)
   int Pcp, Pc, P, stages, gamma;
   int pair_slots;  // CTA pairs per chunk
   int n_ptiles;    // ceil(V / 256)
@@ -504,6 +515,23 @@ __device__ __forceinline__ TileOut group16_z(const uint32_t* la, const uint32_t*
 
 }  // namespace
 
+// Slot of sub-group h in the pair's t-th tile, and how many times that slot
+// was used before (the parity of its barriers).  Ring: the R slots in turn;
+// split: sub-group 0 in slot 0, sub-group 1 in slots 1 and 2 by turns.
+__device__ __forceinline__ int h2_slot(const Head2Params& p, int t, int h, int& uses) {
+  if (p.split) {
+    if (h == 0) {
+      uses = t;
+      return 0;
+    }
+    uses = t >> 1;
+    return 1 + (t & 1);
+  }
+  const int u = t * p.H + h;
+  uses = u / p.R;
+  return u - uses * p.R;
+}
+
 // Running statistics of the epilogue lane: one (m, s, t) per owned group, in
 // registers.  The group loop stays rolled (unrolled over the groups, its body
 // would not fit the instruction cache of the eight epilogue warps), so the
@@ -569,11 +597,11 @@ __global__ void __launch_bounds__(H2_THREADS, 1)
   const int pair = blockIdx.x >> 1;
   const int chunk = blockIdx.y;
   const int slot_id = blockIdx.x;  // partial slot within the chunk
-  const int S = p.stages, R = p.R, H = p.H;
-  // this CTA's rows of B per stage: Ns / 2 of every sub-group (the original
-  // or the reflective rows; for the pre-blended head the first or second half
-  // of the blended rows)
-  const uint32_t b_rows = static_cast<uint32_t>(H * p.Ns / 2);
+  const int S = p.stages, H = p.H;
+  // this CTA's rows of B per stage: half of every sub-group's columns (the
+  // original or the reflective rows; for the pre-blended head the first or
+  // second half of the blended rows)
+  const uint32_t b_rows = static_cast<uint32_t>(p.b_rows);
   const uint32_t b_half = b_rows * 128u;  // one 64-wide K half of this CTA's B
   const uint32_t b_bytes = 2u * b_half;
 
@@ -643,7 +671,7 @@ __global__ void __launch_bounds__(H2_THREADS, 1)
       int s = 0, issued = 0;
       uint32_t ph = 0;
       bool ok = true;
-      const int hrow = chunk * H * p.Ns + static_cast<int>(rank) * static_cast<int>(b_rows);
+      const int hrow = (2 * chunk + static_cast<int>(rank)) * static_cast<int>(b_rows);
       for (int pt = pt0; pt < pt1 && ok; ++pt) {
         const int v0 = pt * 2 * H2_BM + static_cast<int>(rank) * H2_BM;
         for (int kb = 0; kb < p.n_kb; ++kb) {
@@ -679,18 +707,20 @@ __global__ void __launch_bounds__(H2_THREADS, 1)
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer (even CTA)
     if (leader && lane == 0) {
-      const uint32_t idesc = idesc_bf16_f32(2 * H2_BM, p.Ns);
+      const int cols0 = p.zonly ? p.Ph[0] : 2 * p.Ph[0];
+      const int cols1 = p.zonly ? p.Ph[1] : 2 * p.Ph[1];
+      const uint32_t idesc0 = idesc_bf16_f32(2 * H2_BM, cols0);
+      const uint32_t idesc1 = H > 1 ? idesc_bf16_f32(2 * H2_BM, cols1) : idesc0;
       // descriptors of stage 0; stage s adds s * bytes / 16 to the start field
       const uint64_t ad0 = sw128_kmajor_desc(a_tiles), bd0 = sw128_kmajor_desc(b_tiles);
       const uint32_t a_step = H2_A_BYTES >> 4, b_step = b_bytes >> 4;
       const uint32_t a_hstep = H2_A_HALF >> 4, b_hstep = b_half >> 4;
-      const uint32_t b_sub = (static_cast<uint32_t>(p.Ns / 2) * 128u) >> 4;  // next sub-group's rows
+      const uint32_t b_sub1 = (static_cast<uint32_t>(p.pb[1]) * 128u) >> 4;  // sub-group 1's rows
       int s = 0;
       uint32_t ph = 0;
       bool ok = true;
-      int u = 0;  // accumulator uses so far (tile * H + sub-group)
-      for (int pt = pt0; pt < pt1 && ok; ++pt) {
-        uint32_t d_tmem[H2_MAX_H] = {0u, 0u};
+      for (int pt = pt0, t = 0; pt < pt1 && ok; ++pt, ++t) {
+        uint32_t d0 = 0u, d1 = 0u;
         for (int kb = 0; kb < p.n_kb && ok; ++kb) {
           if (!mbar_wait(full_bar(s), ph, abort_flag, p.status)) {
             ok = false;
@@ -699,20 +729,28 @@ __global__ void __launch_bounds__(H2_THREADS, 1)
           const uint64_t ad = ad0 + static_cast<uint32_t>(s) * a_step;
           const uint64_t bd = bd0 + static_cast<uint32_t>(s) * b_step;
 #pragma unroll
-          for (int h = 0; h < H2_MAX_H; ++h) {
-            if (h >= H) break;
+          for (int i = 0; i < H2_MAX_H; ++i) {
+            if (i >= H) break;
+            // split: sub-group 1 first, its slot is free; sub-group 0's may
+            // still be read by the epilogue of the tile before
+            const int h = p.split ? H - 1 - i : i;
             if (kb == 0) {
               // the slot of this sub-group must have been read by the epilogue
-              const int uu = u + h, sl = uu % R;
-              if (!mbar_wait(acce0 + 8u * sl, ((uu / R) & 1) ^ 1u, abort_flag, p.status)) {
+              int uses;
+              const int sl = h2_slot(p, t, h, uses);
+              if (!mbar_wait(acce0 + 8u * sl, (uses & 1) ^ 1, abort_flag, p.status)) {
                 ok = false;
                 break;
               }
               tc_fence_after();
-              d_tmem[h] = tmem_base + static_cast<uint32_t>(sl * p.Ns);
+              const uint32_t d = tmem_base + static_cast<uint32_t>(p.scol[sl]);
+              if (h == 0)
+                d0 = d;
+              else
+                d1 = d;
             }
-            tc2_mma_stage8(d_tmem[h], ad, bd + static_cast<uint32_t>(h) * b_sub, a_hstep, b_hstep,
-                           idesc, kb != 0 ? 1u : 0u);
+            tc2_mma_stage8(h == 0 ? d0 : d1, ad, h == 0 ? bd : bd + b_sub1, a_hstep, b_hstep,
+                           h == 0 ? idesc0 : idesc1, kb != 0 ? 1u : 0u);
           }
           tc2_commit(empty_bar(s), pair_mask);
           if (++s == S) {
@@ -721,9 +759,11 @@ __global__ void __launch_bounds__(H2_THREADS, 1)
           }
         }
         if (ok) {
-          for (int h = 0; h < H; ++h) tc2_commit(accf0 + 8u * ((u + h) % R), pair_mask);
+          for (int h = 0; h < H; ++h) {
+            int uses;
+            tc2_commit(accf0 + 8u * h2_slot(p, t, h, uses), pair_mask);
+          }
         }
-        u += H;
       }
       // every MMA issued must be complete before TMEM is released
       tc2_commit(drain_bar, static_cast<uint16_t>(1u << crank));
@@ -736,10 +776,12 @@ __global__ void __launch_bounds__(H2_THREADS, 1)
     const int kq = (warp - 2) >> 2;  // this warp's index within its quadrant
     const float beta = 1.f - p.alpha;
     constexpr int gsz = ZONLY ? 16 : 8;  // pairs per group
-    const int ng = p.Ph / gsz;           // groups per sub-group
     // this warp's groups: g = kq, kq + WPQ, ... of every sub-group, in order
-    const int n_h0 = kq < ng ? (ng - kq + H2_WPQ - 1) / H2_WPQ : 0;
-    const int n_mine = H * n_h0;
+    const int ng0 = p.Ph[0] / gsz, ng1 = H > 1 ? p.Ph[1] / gsz : 0;
+    const int cnt0 = kq < ng0 ? (ng0 - kq + H2_WPQ - 1) / H2_WPQ : 0;
+    const int cnt1 = kq < ng1 ? (ng1 - kq + H2_WPQ - 1) / H2_WPQ : 0;
+    const int n_mine = cnt0 + cnt1;
+    auto cnt_of = [&](int h) { return h == 0 ? cnt0 : cnt1; };
     LaneStats st;
     const int qn = ZONLY ? (lane >> 4) : (lane >> 3);
     const bool is_best = ZONLY ? qn == 1 : qn == 3;
@@ -754,8 +796,6 @@ __global__ void __launch_bounds__(H2_THREADS, 1)
     const ZSink zs{p.zout ? p.zout + static_cast<long long>(pair0) * p.V : nullptr,
                    p.zsub ? p.zsub + static_cast<long long>(pair0) * p.n_sub : nullptr, p.n_sub,
                    p.inv_t};
-    // slot and phase of the accumulator use the MMA issuer counts next
-    int use_slot = 0, use_phase = 0;
     bool ok = true;
     int slot0 = 0, slot1 = 0, phase0 = 0, phase1 = 0;  // of sub-groups 0 and 1 this tile
     auto slot_of = [&](int h) { return h == 0 ? slot0 : slot1; };
@@ -772,86 +812,91 @@ __global__ void __launch_bounds__(H2_THREADS, 1)
     };
     // first TMEM column of group g of sub-group h of the current tile
     auto tcol = [&](int h, int g) -> uint32_t {
-      return tmem_base + lane_q + static_cast<uint32_t>(slot_of(h) * p.Ns + g * gsz);
+      return tmem_base + lane_q + static_cast<uint32_t>(p.scol[slot_of(h)] + g * gsz);
     };
-    auto load_group = [&](uint32_t t0, uint32_t* b) {
+    // o' of sub-group h starts Ph[h] columns after its o
+    auto load_group = [&](uint32_t t0, int h, uint32_t* b) {
       if (ZONLY) {
         tmem_ld_16x256b_x2(t0, b);
         tmem_ld_16x256b_x2(t0 + (16u << 16), b + 8);
       } else {
+        const uint32_t po = static_cast<uint32_t>(h == 0 ? p.Ph[0] : p.Ph[1]);
         tmem_ld_16x256b(t0, b);
         tmem_ld_16x256b(t0 + (16u << 16), b + 4);
-        tmem_ld_16x256b(t0 + static_cast<uint32_t>(p.Ph), b + 8);
-        tmem_ld_16x256b(t0 + static_cast<uint32_t>(p.Ph) + (16u << 16), b + 12);
+        tmem_ld_16x256b(t0 + po, b + 8);
+        tmem_ld_16x256b(t0 + po + (16u << 16), b + 12);
       }
     };
     // drafts of this lane's columns of group (h, g)
     constexpr int NC = ZONLY ? 4 : 2;
     auto load_drafts = [&](int h, int g, int (&x)[NC]) {
       const int c4 = lane & 3;
-      const int gp = h * p.Ph + g * gsz;
+      const int gp = (h == 0 ? 0 : p.pb[1]) + g * gsz;
 #pragma unroll
       for (int j = 0; j < NC; ++j)
         x[j] = s_drafts[gp + 2 * c4 + (j & 1) + 8 * (j >> 1)];  // -1: no draft (or padding)
     };
-    for (int pt = pt0; pt < pt1 && ok; ++pt) {
-      slot0 = use_slot;
-      phase0 = use_phase;
-      if (++use_slot == R) {
-        use_slot = 0;
-        use_phase ^= 1;
-      }
-      if (H == 2) {
-        slot1 = use_slot;
-        phase1 = use_phase;
-        if (++use_slot == R) {
-          use_slot = 0;
-          use_phase ^= 1;
-        }
+    for (int pt = pt0, t = 0; pt < pt1 && ok; ++pt, ++t) {
+      // the slots and parities the MMA issuer uses for this tile
+      {
+        int u0, u1 = 0;
+        slot0 = h2_slot(p, t, 0, u0);
+        slot1 = H > 1 ? h2_slot(p, t, 1, u1) : 0;
+        phase0 = u0 & 1;
+        phase1 = u1 & 1;
       }
       const int v_row0 = pt * 2 * H2_BM + static_cast<int>(rank) * H2_BM + q * 32;
-      if (n_mine == 0) {
-        // a warp without groups still counts on every slot's barrier
-        for (int h = 0; h < H && ok; ++h) {
+      // a sub-group with none of this warp's groups: its slot's barrier still
+      // counts this warp, once the slot holds this tile's accumulator
+      for (int h = 0; h < H && ok; ++h) {
+        if (cnt_of(h) == 0) {
           ok = wait_slot(h);
           if (ok) release_slot(h);
         }
-        continue;
       }
+      if (!ok) break;
+      if (n_mine == 0) continue;
       uint32_t cb[16], nb[16];
       int cx[NC], nx[NC];
-      if (!wait_slot(0)) {
+      int h = cnt0 > 0 ? 0 : 1, gi = 0;  // sub-group and index within it of group idx
+      if (!wait_slot(h)) {
         ok = false;
         break;
       }
-      load_group(tcol(0, kq), cb);
-      load_drafts(0, kq, cx);
+      load_group(tcol(h, kq), h, cb);
+      load_drafts(h, kq, cx);
       tmem_ld_wait();
       after_ld(cb);
-      int h = 0, gi = 0;  // sub-group and index within it of group idx
+      bool freed = false;  // h's slot released already
 #pragma unroll 1
       for (int idx = 0; idx < n_mine; ++idx) {
         const int g = gi * H2_WPQ + kq;
         // the next group
         int nh = h, ngi = gi + 1;
-        if (ngi == n_h0) {
+        if (ngi == cnt_of(h)) {
           ++nh;
           ngi = 0;
         }
         const bool more = idx + 1 < n_mine;
-        // this group (the last of sub-group h unless the next one is h's too)
-        // is in registers already: h's slot is free before it is reduced, so
-        // the MMAs of the next tile need not wait for this reduction
-        if (!more || nh != h) release_slot(h);
+        // h's slot is released as soon as all of this warp's groups of h are
+        // in registers, before they are reduced, so that the MMAs of the next
+        // tile wait as little as possible: now, if this group is h's last ...
+        if ((!more || nh != h) && !freed) release_slot(h);
         if (more && nh != h && !wait_slot(nh)) {
           ok = false;
           break;
         }
         if (more) {  // lands while this group is reduced
-          load_group(tcol(nh, ngi * H2_WPQ + kq), nb);
+          load_group(tcol(nh, ngi * H2_WPQ + kq), nh, nb);
           load_drafts(nh, ngi * H2_WPQ + kq, nx);
         }
-        const int gpair = h * p.Ph + g * gsz;
+        // ... or once the next one, h's last, has landed
+        if (more && nh == h && ngi + 1 == cnt_of(h)) {
+          tmem_ld_wait();
+          release_slot(h);
+          freed = true;
+        }
+        const int gpair = (h == 0 ? 0 : p.pb[1]) + g * gsz;
         TileOut t;
         if constexpr (ZONLY)
           t = group16_z<SUB>(cb, cb + 8, v_row0, p.V, cx, gpair, npairs, gathered, zs, lane);
@@ -866,6 +911,7 @@ __global__ void __launch_bounds__(H2_THREADS, 1)
         for (int k = 0; k < 16; ++k) cb[k] = nb[k];
 #pragma unroll
         for (int j = 0; j < NC; ++j) cx[j] = nx[j];
+        if (nh != h) freed = false;
         h = nh;
         gi = ngi;
       }
@@ -882,13 +928,15 @@ __global__ void __launch_bounds__(H2_THREADS, 1)
 #pragma unroll
     for (int idx = 0; idx < H2_MAX_OWN; ++idx) {
       if (idx >= n_mine) break;
-      const int h = idx / n_h0, g = (idx % n_h0) * H2_WPQ + kq;
+      const int h = idx < cnt0 ? 0 : 1;
+      const int g = (idx < cnt0 ? idx : idx - cnt0) * H2_WPQ + kq;
+      const int p0 = h == 0 ? 0 : p.pb[1];
       int pj;
       if (ZONLY) {
         const int jj = rq & 3;
-        pj = h * p.Ph + g * 16 + 2 * c4 + (jj & 1) + 8 * (jj >> 1);
+        pj = p0 + g * 16 + 2 * c4 + (jj & 1) + 8 * (jj >> 1);
       } else {
-        pj = h * p.Ph + g * 8 + 2 * c4 + (rq & 1);
+        pj = p0 + g * 8 + 2 * c4 + (rq & 1);
       }
       if (pj < npairs) {
         float* d = stats + (q * tab + pj) * HEAD_STAT_STRIDE;
@@ -1035,31 +1083,72 @@ void head_pair_chunks(int P, int* n_chunks, int* pairs_per_chunk, int* sub, int*
   *sub_pairs = (per + 7) / 8 * 8;
 }
 
-int head_tc2_slots(const HeadPlan& pl) {
-  const int ns = pl.zonly ? pl.sub_pairs : 2 * pl.sub_pairs;
-  return std::min(H2_MAX_R, 512 / ns);
+namespace {
+// Sub-groups and accumulator slots of a chunk of pad_pairs (padded) pairs:
+// the ring for one sub-group, the split layout for two (the kernel's header
+// comment); false when the kernel cannot run the plan.
+struct H2Layout {
+  int H = 0, R = 0, split = 0;
+  int Ph[H2_MAX_H] = {}, pb[H2_MAX_H] = {}, scol[H2_MAX_R] = {};
+  int cols = 0;  // TMEM columns in use
+};
+
+bool h2_layout(const HeadPlan& pl, H2Layout* L) {
+  const int gsz = pl.zonly ? 16 : 8;
+  const int pad = pl.pad_pairs;
+  *L = H2Layout{};
+  if (pad < gsz || pad % gsz != 0) return false;
+  if (pl.sub == 1) {
+    const int ns = pl.zonly ? pad : 2 * pad;  // columns per slot
+    L->H = 1;
+    L->Ph[0] = pad;
+    L->R = std::min(H2_MAX_R, 512 / ns);
+    if (L->R < 2) return false;
+    for (int k = 0; k < L->R; ++k) L->scol[k] = k * ns;
+    L->cols = L->R * ns;
+  } else if (pl.sub == 2 && !pl.zonly) {
+    // 2 Ph[0] + 4 Ph[1] = 512 columns, Ph[0] + Ph[1] = pad
+    const int p1 = std::min(128, 256 - pad), p0 = pad - p1;
+    if (p0 < gsz || p1 < gsz || p0 > 128 || p1 % gsz != 0) return false;
+    L->H = 2;
+    L->split = 1;
+    L->R = 3;
+    L->Ph[0] = p0;
+    L->Ph[1] = p1;
+    L->pb[1] = p0;
+    L->scol[1] = 2 * p0;
+    L->scol[2] = 2 * p0 + 2 * p1;
+    L->cols = 2 * p0 + 4 * p1;
+  } else {
+    return false;
+  }
+  int own = 0;  // groups one epilogue warp owns at most
+  for (int h = 0; h < L->H; ++h) own += (L->Ph[h] / gsz + H2_WPQ - 1) / H2_WPQ;
+  return own <= H2_MAX_OWN && L->cols <= 512;
 }
+}  // namespace
 
 bool head_tc2_supports(const HeadPlan& pl) {
-  const int gsz = pl.zonly ? 16 : 8;
-  if (pl.sub < 1 || pl.sub > H2_MAX_H || pl.sub_pairs < gsz || pl.sub_pairs % gsz != 0)
-    return false;
-  if (pl.zonly && pl.sub != 1) return false;
-  if (pl.sub * pl.sub_pairs != pl.pad_pairs) return false;
-  const int ng = pl.sub_pairs / gsz;
-  const int per_warp = pl.sub * ((ng + H2_WPQ - 1) / H2_WPQ);
-  return per_warp <= H2_MAX_OWN && head_tc2_slots(pl) >= pl.sub + 1;
+  H2Layout L;
+  return h2_layout(pl, &L);
 }
 
 cudaError_t launch_head_tc2(const HeadArgs& a, const HeadPlan& pl, const HeadTcLaunch& l,
                             const HeadFinal* fin, cudaStream_t s) {
+  H2Layout L;
+  if (!h2_layout(pl, &L)) return cudaErrorInvalidValue;
   Head2Params p;
   p.V = a.V;
   p.n_kb = (a.H + H2_BK - 1) / H2_BK;
-  p.H = pl.sub;
-  p.Ph = pl.sub_pairs;
-  p.Ns = pl.zonly ? pl.sub_pairs : 2 * pl.sub_pairs;
-  p.R = head_tc2_slots(pl);
+  p.H = L.H;
+  p.R = L.R;
+  p.split = L.split;
+  for (int h = 0; h < H2_MAX_H; ++h) {
+    p.Ph[h] = L.Ph[h];
+    p.pb[h] = L.pb[h];
+  }
+  for (int k = 0; k < H2_MAX_R; ++k) p.scol[k] = L.scol[k];
+  p.b_rows = pl.zonly ? pl.pad_pairs / 2 : pl.pad_pairs;
   p.Pcp = pl.pad_pairs;
   p.Pc = pl.pairs_per_chunk;
   p.P = pl.P;
@@ -1072,7 +1161,7 @@ cudaError_t launch_head_tc2(const HeadArgs& a, const HeadPlan& pl, const HeadTcL
   p.fused = fin != nullptr ? 1 : 0;
   if (fin) p.fin = *fin;
   p.slots = pl.slots;
-  p.tmem_cols = h2_tmem_cols(p.R * p.Ns);
+  p.tmem_cols = h2_tmem_cols(L.cols);
   p.alpha = a.alpha;
   p.drafts = a.drafts;
   p.partials = a.partials;

@@ -228,8 +228,7 @@ cudaError_t head_tc2_configure(size_t smem_bytes);
 // co-resident CTA pairs (occupancy query)
 int head_tc2_max_pairs(int N, int pairs, int stages);
 
-// accumulator slots of the plan, and whether the kernel takes its sub-groups
-int head_tc2_slots(const HeadPlan& p);
+// whether the kernel takes the plan (its sub-groups fit an accumulator slot layout)
 bool head_tc2_supports(const HeadPlan& p);
 cudaError_t launch_head_tc2(const HeadArgs& a, const HeadPlan& p, const HeadTcLaunch& l,
                             const HeadFinal* fin, cudaStream_t s);

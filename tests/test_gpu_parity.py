@@ -157,10 +157,12 @@ def test_bf16_multi_chunk(gu):
 
 @pytest.mark.parametrize("B,gamma,V", [(16, 8, 1000), (16, 8, 60000), (15, 9, 60000)])
 def test_bf16_pair_kernel_two_chunks_many_tiles(gu, B, gamma, V):
-    # 144 / 150 pairs -> two chunks of 72 / 75 pairs on CTA pairs (the second
-    # shape with 5 padding pairs per chunk); at V = 60000 every CTA pair runs
-    # several vocab tiles, so both accumulator slots are reused and their
-    # barrier phases flip; H = 320 leaves a half-filled last K stage
+    # 144 / 150 pairs in one chunk on CTA pairs, two sub-groups in the split
+    # accumulator layout: 32 + 112 pairs / 64 + 96 (160 with 10 padding
+    # pairs); at V = 60000 every CTA pair runs several vocab tiles, so the
+    # small sub-group's slot is reused every tile, the large one's two by
+    # turns, and their barrier phases flip; H = 320 leaves a half-filled last
+    # K stage
     _check(gu, _wl(B=B, gamma=gamma, R=3, V=V, H=320, ctx=(1, 30), seed=47 + V % 7),
            check_attn=False)
 

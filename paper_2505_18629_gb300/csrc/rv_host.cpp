@@ -98,6 +98,11 @@ struct rv_handle {
   cudaStream_t side = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   cudaEvent_t ev_copy_start = nullptr, ev_copy_done = nullptr;  // rv_verify_step_host
+  // recorded after the row gather when `record_prep` is set (rv_verify_step_host:
+  // the side stream's copies wait for it, so they do not share the host link
+  // with the gather's reads of the hidden states)
+  cudaEvent_t ev_prep = nullptr;
+  bool record_prep = false;
   // pinned staging of rv_verify_step_host's small inputs / outputs, which the
   // kernels read / write in place (first rv_verify_step_host call)
   char* pin_in = nullptr;
@@ -353,6 +358,7 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_copy_start, cudaEventDisableTiming);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_copy_done, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_prep, cudaEventDisableTiming);
   if (e == cudaSuccess && bf16) e = attn_configure(&h->attn_max_cluster);
   if (e == cudaSuccess && h->attn_tc_ok) e = attn_tc_configure(attn_tc_smem_max(c.max_batch));
   if (e == cudaSuccess && bf16) e = head_tc_configure(h->smem_optin);
@@ -365,6 +371,7 @@ extern "C" RV_API int rv_create(const rv_config* cfg, rv_handle** out) {
     h->encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
   }
   if (e != cudaSuccess) {
+    if (h->ev_prep) cudaEventDestroy(h->ev_prep);
     if (h->ev_copy_done) cudaEventDestroy(h->ev_copy_done);
     if (h->ev_copy_start) cudaEventDestroy(h->ev_copy_start);
     if (h->ev_join) cudaEventDestroy(h->ev_join);
@@ -387,6 +394,7 @@ extern "C" RV_API int rv_destroy(rv_handle* h) {
   cudaEventDestroy(h->ev_fork);
   cudaEventDestroy(h->ev_copy_start);
   cudaEventDestroy(h->ev_copy_done);
+  cudaEventDestroy(h->ev_prep);
   cudaStreamDestroy(h->side);
   if (h->zbuf) cudaFree(h->zbuf);
   if (h->zsub) cudaFree(h->zsub);
@@ -671,6 +679,10 @@ int head_impl(rv_handle* h, const void* hidden, const void* w_head, const int32_
     h->launches += 1;
     if (e != cudaSuccess) return cuda_fail(h, e, "prep launch");
   }
+  if (h->record_prep) {
+    e = cudaEventRecord(h->ev_prep, s);
+    if (e != cudaSuccess) return cuda_fail(h, e, "event record");
+  }
   // Small pair counts: the head kernel's last CTA finishes the merge itself.
   // (one chunk only: the merge reads each pair's draft from the CTA's chunk table)
   const bool fused = bf16 && pl.P <= HEAD_FUSED_FINAL_MAX_PAIRS && pl.n_chunks == 1;
@@ -899,6 +911,18 @@ int sampled_accept_launches(rv_handle* h, const int32_t* draft_ids, const float*
   return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "accept launch");
 }
 
+// Host-to-device copies of the attention's inputs that rv_verify_step_host
+// leaves to the step: issued on the side stream once the row gather has run.
+struct SideCopies {
+  void* q;
+  const void* q_src;
+  void* k;
+  const void* k_src;
+  void* v;
+  const void* v_src;
+  size_t nq, nkv;
+};
+
 int step_impl(rv_handle* h, const void* q, const void* k_blk, const void* v_blk, void* k_cache,
               void* v_cache, const void* hidden, const void* w_head, const int32_t* draft_ids,
               const int32_t* prompt_ids, const int32_t* prefix_ids, const int32_t* ctx_in,
@@ -906,7 +930,7 @@ int step_impl(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
               int32_t* block_ids, int32_t* pos_ids, void* attn_out, float* scores,
               int32_t* argmax, float* margin, uint8_t* accept_mask, int32_t* accepted_len,
               int32_t* next_token, int32_t* ctx_out, const SpecInputs* spec, void* stream,
-              const int32_t* pending = nullptr) {
+              const int32_t* pending = nullptr, const SideCopies* copies = nullptr) {
   if (n_prompt < 0 || n_prefix < 0) return fail(h, RV_ERR_SHAPE, "negative template part");
   const int R = n_prompt + n_prefix;
   const int lead = pending ? 1 : 0;  // the pending-token block has one more position
@@ -964,7 +988,21 @@ int step_impl(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
     return r;
   };
   if (fork) {
+    h->record_prep = copies != nullptr;
     rc = run_head();
+    h->record_prep = false;
+    if (rc == RV_OK && copies) {
+      e = cudaStreamWaitEvent(h->side, h->ev_prep, 0);
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(copies->q, copies->q_src, copies->nq, cudaMemcpyHostToDevice, h->side);
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(copies->k, copies->k_src, copies->nkv, cudaMemcpyHostToDevice,
+                            h->side);
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(copies->v, copies->v_src, copies->nkv, cudaMemcpyHostToDevice,
+                            h->side);
+      if (e != cudaSuccess) rc = cuda_fail(h, e, "host->device copy");
+    }
     if (rc == RV_OK)
       rc = rv_verify_attention(h, q, k_blk, v_blk, k_cache, v_cache, ctx_in, B, Lb, attn_out,
                                h->side);
@@ -982,6 +1020,20 @@ int step_impl(rv_handle* h, const void* q, const void* k_blk, const void* v_blk,
 
 }  // namespace
 
+namespace {
+// The acceptance modes rv_verify_step (and its host-buffer form) can run: the
+// others need inputs of their own.
+int plain_step_mode(rv_handle* h) {
+  if (h->accept_mode == RV_ACCEPT_SPECULATIVE)
+    return fail(h, RV_ERR_INVALID_ARG,
+                "speculative sampling needs the draft distributions: use rv_verify_step_speculative");
+  if (h->accept_mode == RV_ACCEPT_SAMPLED || h->accept_mode == RV_ACCEPT_TYPICAL_SAMPLED)
+    return fail(h, RV_ERR_INVALID_ARG,
+                "a sampled next token needs the uniforms: use rv_verify_step_sampled");
+  return RV_OK;
+}
+}  // namespace
+
 extern "C" RV_API int rv_verify_step(
     rv_handle* h, const void* q, const void* k_blk, const void* v_blk, void* k_cache, void* v_cache,
     const void* hidden, const void* w_head, const int32_t* draft_ids, const int32_t* prompt_ids,
@@ -991,12 +1043,8 @@ extern "C" RV_API int rv_verify_step(
     int32_t* next_token, int32_t* ctx_out, void* stream) {
   if (!h) return RV_ERR_INVALID_ARG;
   h->err.clear();
-  if (h->accept_mode == RV_ACCEPT_SPECULATIVE)
-    return fail(h, RV_ERR_INVALID_ARG,
-                "speculative sampling needs the draft distributions: use rv_verify_step_speculative");
-  if (h->accept_mode == RV_ACCEPT_SAMPLED || h->accept_mode == RV_ACCEPT_TYPICAL_SAMPLED)
-    return fail(h, RV_ERR_INVALID_ARG,
-                "a sampled next token needs the uniforms: use rv_verify_step_sampled");
+  const int mrc = plain_step_mode(h);
+  if (mrc != RV_OK) return mrc;
   return step_impl(h, q, k_blk, v_blk, k_cache, v_cache, hidden, w_head, draft_ids, prompt_ids,
                    prefix_ids, ctx_in, B, gamma, n_prompt, n_prefix, alpha, block_ids, pos_ids,
                    attn_out, scores, argmax, margin, accept_mask, accepted_len, next_token, ctx_out,
@@ -1216,31 +1264,40 @@ extern "C" RV_API int rv_verify_step_host(
   auto I32 = [](char* p) { return reinterpret_cast<int32_t*>(p); };
   // The device part: copies in, the step, copies out (all stream-ordered).
   auto issue = [&]() -> int {
-    // q, k_blk, v_blk on the side stream, concurrently with the ids and the
-    // hidden states on `stream` (the side stream's attention follows its
-    // copies in stream order; otherwise `stream` waits for them before the step)
-    cudaError_t e = cudaEventRecord(h->ev_copy_start, s);
-    if (e == cudaSuccess) e = cudaStreamWaitEvent(h->side, h->ev_copy_start, 0);
-    if (e == cudaSuccess && !zc_hidden)
-      e = cudaMemcpyAsync(w.st_hidden, hidden_host, nh, cudaMemcpyHostToDevice, s);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(w.st_q, q_host, nq, cudaMemcpyHostToDevice, h->side);
-    if (e == cudaSuccess)
-      e = cudaMemcpyAsync(w.st_kb, k_blk_host, nkv, cudaMemcpyHostToDevice, h->side);
-    if (e == cudaSuccess)
-      e = cudaMemcpyAsync(w.st_vb, v_blk_host, nkv, cudaMemcpyHostToDevice, h->side);
-    if (e == cudaSuccess) e = cudaEventRecord(h->ev_copy_done, h->side);
-    if (e == cudaSuccess && !attn_forks(h, B, Lb)) e = cudaStreamWaitEvent(s, h->ev_copy_done, 0);
+    // The hidden states first (when they are not read in place), on `stream`.
+    // With the attention beside the head, q / k_blk / v_blk go on the side
+    // stream once the row gather has run (the gather's reads of the hidden
+    // states then have the host link to themselves, and the attention follows
+    // its copies in stream order); otherwise on the side stream at once, and
+    // `stream` waits for them before the attention that opens the step.
+    const bool fork = attn_forks(h, B, Lb);
+    const SideCopies copies{w.st_q, q_host, w.st_kb, k_blk_host, w.st_vb, v_blk_host, nq, nkv};
+    cudaError_t e = cudaSuccess;
+    if (!zc_hidden) e = cudaMemcpyAsync(w.st_hidden, hidden_host, nh, cudaMemcpyHostToDevice, s);
+    if (!fork) {
+      if (e == cudaSuccess) e = cudaEventRecord(h->ev_copy_start, s);
+      if (e == cudaSuccess) e = cudaStreamWaitEvent(h->side, h->ev_copy_start, 0);
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(w.st_q, q_host, nq, cudaMemcpyHostToDevice, h->side);
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(w.st_kb, k_blk_host, nkv, cudaMemcpyHostToDevice, h->side);
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(w.st_vb, v_blk_host, nkv, cudaMemcpyHostToDevice, h->side);
+      if (e == cudaSuccess) e = cudaEventRecord(h->ev_copy_done, h->side);
+      if (e == cudaSuccess) e = cudaStreamWaitEvent(s, h->ev_copy_done, 0);
+    }
     if (e != cudaSuccess) return cuda_fail(h, e, "host->device copy");
-    int rc = rv_verify_step(h, w.st_q, w.st_kb, w.st_vb, k_cache, v_cache,
-                            zc_hidden ? hidden_host : w.st_hidden, w_head,
-                            I32(di + i_dr), do_pack ? I32(di + i_pr) : nullptr,
-                            do_pack ? I32(di + i_px) : nullptr, I32(di + i_ci), B, gamma,
-                            n_prompt, n_prefix, alpha, do_pack ? I32(dout + o_bl) : nullptr,
-                            do_pack ? I32(dout + o_ps) : nullptr, w.st_attn,
-                            reinterpret_cast<float*>(dout + o_sc), I32(dout + o_am),
-                            reinterpret_cast<float*>(dout + o_mg),
-                            reinterpret_cast<uint8_t*>(dout + o_ac), I32(dout + o_al),
-                            I32(dout + o_nt), I32(dout + o_co), stream);
+    int rc = plain_step_mode(h);
+    if (rc != RV_OK) return rc;
+    rc = step_impl(h, w.st_q, w.st_kb, w.st_vb, k_cache, v_cache,
+                   zc_hidden ? hidden_host : w.st_hidden, w_head, I32(di + i_dr),
+                   do_pack ? I32(di + i_pr) : nullptr, do_pack ? I32(di + i_px) : nullptr,
+                   I32(di + i_ci), B, gamma, n_prompt, n_prefix, alpha,
+                   do_pack ? I32(dout + o_bl) : nullptr, do_pack ? I32(dout + o_ps) : nullptr,
+                   w.st_attn, reinterpret_cast<float*>(dout + o_sc), I32(dout + o_am),
+                   reinterpret_cast<float*>(dout + o_mg), reinterpret_cast<uint8_t*>(dout + o_ac),
+                   I32(dout + o_al), I32(dout + o_nt), I32(dout + o_co), nullptr, stream, nullptr,
+                   fork ? &copies : nullptr);
     if (rc != RV_OK) return rc;
     if (attn_out_host) e = cudaMemcpyAsync(attn_out_host, w.st_attn, nq, cudaMemcpyDeviceToHost, s);
     return e == cudaSuccess ? RV_OK : cuda_fail(h, e, "device->host copy");
